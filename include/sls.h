@@ -1,0 +1,242 @@
+/*
+ * sls.h -- C ABI of the GB300 (sm_103a) Spectral-LSH compression pass.
+ *
+ * Spectral-LSH (arXiv 2607.19368) compresses a prompt's N x d input
+ * embeddings X into M << N macro-tokens before prefill:
+ *   1. random Fourier features Phi = sqrt(2/D) cos(X Omega + b)  (Sec. 3.2, Eq. rff_map)
+ *   2. r steps of Lanczos on the implicit operator A(v) = Phi (Phi^T v),
+ *      never forming the N x N kernel                            (Algorithm 2, Eq. implicit_matvec)
+ *   3. Eigh of the tridiagonal T and the Ritz vectors U = Q V      (Algorithm 1)
+ *   4. SimHash of the rows of U into b-bit codes                  (Sec. 3.3, Eq. simhash)
+ *   5. clusters of equal codes, adjusted to exactly M* groups      (Sec. 3.3)
+ *   6. macro-tokens: renormalised means with causal positions      (Sec. 3.4, Eq. macro_embed)
+ *   7. optionally, the adaptive per-window router                 (Sec. 3.6, Eq. redundancy)
+ *
+ * Conventions for every entry point:
+ *   - All array pointers are DEVICE pointers owned by the caller, unless a
+ *     parameter says "host".  The library allocates no memory: calls that
+ *     need scratch take a caller-provided device workspace sized by the
+ *     matching *_workspace_size() function (256-byte aligned).
+ *   - Matrices are row-major and contiguous unless a leading dimension is
+ *     given.  X and W share one dtype: SLS_F32 (float) or SLS_BF16 (raw
+ *     bfloat16 bit patterns, uint16).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Work is enqueued asynchronously; no call synchronises the
+ *     host with the device.
+ *   - Return value: SLS_OK or an SLS_ERR_* code.  Argument errors are
+ *     detected on the host before anything is enqueued.  Errors raised by a
+ *     running kernel (a device wait that gave up) are written to a status
+ *     word in the workspace and read back with sls_workspace_status().
+ *   - Random draws of the method (Omega, b, the hyperplanes R and the Lanczos
+ *     start vector q1) are inputs, so any caller can reproduce a run.
+ *   - Every pointer must be 16-byte aligned; D must be a multiple of 4.
+ */
+#ifndef SLS_H_
+#define SLS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define SLS_OK 0
+#define SLS_ERR_INVALID_ARG 1  /* a size, pointer or option is out of range      */
+#define SLS_ERR_UNSUPPORTED 2  /* a valid but unsupported shape or dtype         */
+#define SLS_ERR_WORKSPACE 3    /* workspace missing or smaller than required     */
+#define SLS_ERR_CUDA 4         /* a CUDA launch or copy failed                   */
+#define SLS_ERR_TIMEOUT 5      /* a device-side wait reached its iteration limit */
+
+/* Embedding dtypes. */
+#define SLS_F32 0
+#define SLS_BF16 1
+
+/* Position aggregation schemes (Sec. 3.4). */
+#define SLS_POS_MAX 0     /* max of member positions (default, causal)        */
+#define SLS_POS_MEDIAN 1  /* lower median of member positions                 */
+#define SLS_POS_MEAN 2    /* floor(mean + 1/2) of member positions            */
+
+/* Compressed position modes (Sec. 5.6, App. B.3). */
+#define SLS_MODE_REPRESENTATIVE 0  /* keep aggregated original positions */
+#define SLS_MODE_COMPACT 1         /* renumber 0..M-1                     */
+
+/* Backends (Sec. 3.5 and 3.6). */
+#define SLS_BACKEND_GLOBAL 0    /* Spectral-LSH over the whole compressible region */
+#define SLS_BACKEND_ADAPTIVE 1  /* per-window router: chunk or Spectral-LSH         */
+#define SLS_BACKEND_CHUNK 2     /* consecutive groups of max(1, round(rho)) tokens  */
+
+/* Limits of this implementation. */
+#define SLS_MAX_R 128      /* Krylov rank r                 */
+#define SLS_MAX_BITS 32    /* SimHash bits b                */
+#define SLS_MAX_D 8192     /* RFF features D (multiple of 4) */
+
+/*
+ * Compression configuration: the fields of the paper's CompressionConfig
+ * (App. B.3, B.8) that the pass uses.
+ */
+typedef struct sls_config {
+  int backend;          /* SLS_BACKEND_*                                        */
+  double rho;           /* target compression; rho <= 1 is the exact identity  */
+  int D;                /* RFF features                                        */
+  int r;                /* Lanczos steps / Krylov rank, 1..SLS_MAX_R           */
+  int bits;             /* SimHash bits; 0 = ceil(log2(n / rho)) (Sec. 3.3)     */
+  int preserve_first;   /* leading tokens kept uncompressed (default 0)        */
+  int preserve_last;    /* trailing tokens kept uncompressed (default 12)      */
+  int pos_scheme;       /* SLS_POS_*                                           */
+  int pos_mode;         /* SLS_MODE_*                                          */
+  int renorm;           /* 1: rescale each mean to its mean member norm        */
+  double lanczos_tol;   /* break when beta_j <= tol * max_i(|alpha_i|+beta_i)  */
+  int window;           /* adaptive backend window length                      */
+  double tau;           /* fixed redundancy threshold (used if !tau_schedule)  */
+  int tau_schedule;     /* 1: tau(rho) = clamp(0.75 - 0.05 log2 rho, .55, .70)  */
+} sls_config_t;
+
+/*
+ * Random parameters (device pointers).  W = Omega^T is D x d in the dtype of
+ * X; b has D floats; R holds R_rows x R_ld float hyperplanes (row l is
+ * hyperplane l, at least `bits` rows and r columns used); q1 holds the
+ * Lanczos start vector (float64), one entry per compressible token (global
+ * backend: N_c entries; adaptive: window w of prompt p reads q1 at offset
+ * p * q1_stride + window start).
+ */
+typedef struct sls_params {
+  const void* W;
+  const float* b;
+  const float* R;
+  int R_rows;
+  int R_ld;
+  const double* q1;
+  int64_t q1_stride;
+} sls_params_t;
+
+/* Human-readable name of a status code (static string). */
+const char* sls_status_string(int status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int sls_version(void);
+
+/*
+ * Random Fourier features, Sec. 3.2 Eq. rff_map:
+ *   Phi[i, c] = sqrt(2/D) * cos( sum_k X[i, k] * W[c, k] + b[c] ).
+ * X: N x d (row stride ldx elements), W: D x d, both of dtype x_dtype;
+ * b: D floats; Phi: N x D floats (output, row stride D).
+ * bf16 inputs use the tcgen05 tensor cores (fp32 accumulation); fp32 inputs
+ * use an fp32 SIMT path.  N may be 0.  Errors: INVALID_ARG for negative or
+ * zero sizes, NULL pointers, D % 4 != 0 or D > SLS_MAX_D.
+ */
+int sls_feature_map(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
+                    const void* W, const float* b, int D, float* Phi,
+                    void* stream);
+
+/* Device workspace bytes needed by sls_lanczos_topr for one problem. */
+size_t sls_lanczos_workspace_size(int64_t N, int D, int r);
+
+/*
+ * Implicit Lanczos and Ritz pairs: Algorithm 2 with A(v) = Phi (Phi^T v)
+ * (Eq. implicit_matvec) followed by Eigh(T) and U = Q V (Algorithm 1).
+ *   Phi: N x D floats.  q1: N doubles (normalised by the callee).
+ *   Full re-orthogonalisation is two classical Gram-Schmidt passes; the loop
+ *   stops early (Lanczos breakdown, not an error) when
+ *   beta_j <= tol * max_{i<=j}(|alpha_i| + beta_i); r_eff <= r steps are kept.
+ * Outputs: theta[r] doubles, Ritz values in descending order (entries past
+ * r_eff are 0); U: N x r floats, column m the Ritz vector of theta[m], signed
+ * so that the first component of the eigenvector of T is positive (columns
+ * past r_eff are 0); r_eff: one int32 (device).  Optional (may be NULL):
+ * alpha[r], beta[r] doubles receive the diagonal and off-diagonal of T.
+ * Vectors are kept in double-float (two fp32) precision; Phi is read as
+ * stored.  Errors: INVALID_ARG (sizes, NULL, r > SLS_MAX_R), WORKSPACE,
+ * UNSUPPORTED (D % 4 != 0), CUDA.
+ */
+int sls_lanczos_topr(const float* Phi, int64_t N, int D, int r,
+                     const double* q1, double tol, double* theta, float* U,
+                     int32_t* r_eff, double* alpha, double* beta,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * SimHash in the spectral subspace, Sec. 3.3 Eq. simhash:
+ *   code[i] = sum_l [ dot(U[i, :k], R[l, :k]) > 0 ] << l,  l < bits.
+ * The dot product is a fixed float32 chain (acc = 0; for m in 0..k-1:
+ * acc = fl(acc + fl(U[i,m] * R[l,m])), no fused multiply-add), so codes are
+ * reproducible bit for bit; a +-0 or NaN dot gives bit 0.  k = *k_dev if
+ * k_dev is not NULL (device int32, e.g. r_eff), else k.  U: N rows with row
+ * stride ldu floats; R: bits x ldr floats.  Errors: INVALID_ARG (bits outside
+ * 1..32, k < 1 or > ldu, NULL pointers).
+ */
+int sls_simhash(const float* U, int64_t N, int k, int ldu, const int32_t* k_dev,
+                const float* R, int bits, int ldr, uint32_t* codes,
+                void* stream);
+
+/* Device workspace bytes needed by sls_aggregate. */
+size_t sls_aggregate_workspace_size(int64_t N, int d, int64_t M_target);
+
+/*
+ * Clusters, exact-length adjustment and macro-tokens (Sec. 3.3, Sec. 3.4,
+ * Eq. macro_embed) for one token set of N tokens with codes[N]:
+ *   - tokens with equal codes form clusters, in ascending code order;
+ *   - adjusted to exactly M_target groups: if C > M_target the cluster of
+ *     rank t joins group floor(t * M_target / C); if C < M_target clusters
+ *     receive D'Hondt seats (one guaranteed each, ties to the lower code) and
+ *     are cut into that many contiguous pieces in position order;
+ *   - each group's embedding is the mean of its members rescaled to their
+ *     mean norm (renorm = 1; a singleton is copied exactly; a mean of norm
+ *     < 1e-30 is not rescaled); its position follows pos_scheme;
+ *   - groups are output in increasing (position, first member) order.
+ * Positions are token indices within the set (0..N-1).
+ * Outputs: Xt: M_target x d floats; pos: M_target int32; tok2macro: N int32
+ * (index of the macro-token holding each token).  1 <= M_target <= N.
+ * Errors: INVALID_ARG, WORKSPACE, CUDA.
+ */
+int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
+                  const uint32_t* codes, int64_t M_target, int pos_scheme,
+                  int renorm, float* Xt, int32_t* pos, int32_t* tok2macro,
+                  void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Number of output macro-tokens per prompt for a configuration (host
+ * arithmetic only): N if rho <= 1 or no token is compressible, else
+ * preserve_first + ceil(N_c / rho) + preserve_last with N_c the compressible
+ * count (chunk backend: ceil(N_c / max(1, round(rho))) groups).  Returns -1
+ * for an invalid configuration.
+ */
+int64_t sls_output_count(const sls_config_t* cfg, int64_t N);
+
+/* Device workspace bytes needed by sls_compress for B prompts of N x d. */
+size_t sls_compress_workspace_size(const sls_config_t* cfg, int64_t B,
+                                   int64_t N, int d);
+
+/*
+ * The whole compression pass (Algorithm 1 and the backends of Sec. 3.5-3.6)
+ * for B independent prompts of N tokens each (B = 1 for a single prompt).
+ *   X: B x N x d embeddings (prompt stride N * ldx elements, row stride ldx);
+ *   params: the random draws (see sls_params_t);
+ *   Xt: B x M x d floats; pos: B x M int32; tok2macro: B x N int32,
+ *   with M = sls_output_count(cfg, N).
+ *   r_eff (may be NULL): device int32 per prompt (global backend) or per
+ *   window (adaptive backend), the Lanczos steps kept (0 for chunk windows).
+ *   route (may be NULL): device int32 per window, 1 = spectral, 0 = chunk
+ *   (adaptive backend).
+ * Preserved first/last tokens become singleton macro-tokens at their own
+ * positions; rho <= 1 (or nothing compressible) returns the identity: Xt = X,
+ * pos = 0..N-1, tok2macro = 0..N-1 (Sec. 5.6, App. B.6).
+ * Errors: INVALID_ARG, UNSUPPORTED, WORKSPACE, CUDA.
+ */
+int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
+                 int64_t N, int d, int64_t ldx, const sls_params_t* params,
+                 float* Xt, int32_t* pos, int32_t* tok2macro, int32_t* r_eff,
+                 int32_t* route, void* workspace, size_t workspace_bytes,
+                 void* stream);
+
+/*
+ * Reads (synchronously, on `stream`) the device status word of a workspace
+ * used by sls_lanczos_topr or sls_compress: SLS_OK, or SLS_ERR_TIMEOUT when
+ * a device-side wait gave up.  Clears the word.
+ */
+int sls_workspace_status(void* workspace, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SLS_H_ */

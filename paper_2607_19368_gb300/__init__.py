@@ -1,0 +1,302 @@
+"""GB300 (sm_103a) Spectral-LSH compression pass (arXiv 2607.19368).
+
+Thin Python binding of the C ABI in ``include/sls.h`` (``libsls.so``).  Every
+step of the pass runs in the library's CUDA kernels; this module only
+marshals torch tensors (device memory and the current stream) into the C
+calls and raises on a non-zero status.  There is no CPU fallback: if the
+library is not built, importing the functions works but every call raises.
+
+The same names as the C entry points are exported:
+``feature_map``, ``lanczos_topr``, ``simhash``, ``aggregate``, ``compress``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+__all__ = [
+    "SLS_OK", "SLS_F32", "SLS_BF16", "POS_MAX", "POS_MEDIAN", "POS_MEAN",
+    "MODE_REPRESENTATIVE", "MODE_COMPACT", "BACKEND_GLOBAL", "BACKEND_ADAPTIVE",
+    "BACKEND_CHUNK", "Config", "SLSError", "lib", "lib_path", "feature_map",
+    "lanczos_topr", "simhash", "aggregate", "compress", "output_count",
+    "compress_workspace_size", "workspace_status", "EXPORTED",
+]
+
+SLS_OK = 0
+SLS_F32, SLS_BF16 = 0, 1
+POS_MAX, POS_MEDIAN, POS_MEAN = 0, 1, 2
+MODE_REPRESENTATIVE, MODE_COMPACT = 0, 1
+BACKEND_GLOBAL, BACKEND_ADAPTIVE, BACKEND_CHUNK = 0, 1, 2
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def lib_path() -> str:
+    return os.path.join(_HERE, "libsls.so")
+
+
+class SLSError(RuntimeError):
+    """A libsls call returned a non-zero status."""
+
+    def __init__(self, fn: str, status: int, text: str):
+        super().__init__(f"{fn}: status {status} ({text})")
+        self.status = status
+
+
+class Config(ctypes.Structure):
+    """sls_config_t: the fields of the paper's CompressionConfig (App. B.3)."""
+    _fields_ = [
+        ("backend", ctypes.c_int), ("rho", ctypes.c_double), ("D", ctypes.c_int),
+        ("r", ctypes.c_int), ("bits", ctypes.c_int), ("preserve_first", ctypes.c_int),
+        ("preserve_last", ctypes.c_int), ("pos_scheme", ctypes.c_int),
+        ("pos_mode", ctypes.c_int), ("renorm", ctypes.c_int),
+        ("lanczos_tol", ctypes.c_double), ("window", ctypes.c_int),
+        ("tau", ctypes.c_double), ("tau_schedule", ctypes.c_int),
+    ]
+
+    @classmethod
+    def make(cls, backend=BACKEND_GLOBAL, rho=4.0, D=256, r=16, bits=0, preserve_first=0,
+             preserve_last=12, pos_scheme=POS_MAX, pos_mode=MODE_REPRESENTATIVE, renorm=1,
+             lanczos_tol=1e-10, window=2048, tau=0.70, tau_schedule=1) -> "Config":
+        return cls(backend, float(rho), D, r, bits, preserve_first, preserve_last, pos_scheme,
+                   pos_mode, int(renorm), float(lanczos_tol), window, float(tau),
+                   int(tau_schedule))
+
+
+class _Params(ctypes.Structure):
+    _fields_ = [
+        ("W", ctypes.c_void_p), ("b", ctypes.c_void_p), ("R", ctypes.c_void_p),
+        ("R_rows", ctypes.c_int), ("R_ld", ctypes.c_int), ("q1", ctypes.c_void_p),
+        ("q1_stride", ctypes.c_int64),
+    ]
+
+
+_vp, _i64, _i32, _sz, _d = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_size_t,
+                            ctypes.c_double)
+
+# name -> (restype, argtypes); the exported surface of include/sls.h
+EXPORTED = {
+    "sls_status_string": (ctypes.c_char_p, [_i32]),
+    "sls_version": (_i32, []),
+    "sls_feature_map": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _vp, _i32, _vp, _vp]),
+    "sls_lanczos_workspace_size": (_sz, [_i64, _i32, _i32]),
+    "sls_lanczos_topr": (_i32, [_vp, _i64, _i32, _i32, _vp, _d, _vp, _vp, _vp, _vp, _vp, _vp,
+                                _sz, _vp]),
+    "sls_simhash": (_i32, [_vp, _i64, _i32, _i32, _vp, _vp, _i32, _i32, _vp, _vp]),
+    "sls_aggregate_workspace_size": (_sz, [_i64, _i32, _i64]),
+    "sls_aggregate": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _i64, _i32, _i32, _vp, _vp, _vp,
+                             _vp, _sz, _vp]),
+    "sls_output_count": (_i64, [ctypes.POINTER(Config), _i64]),
+    "sls_compress_workspace_size": (_sz, [ctypes.POINTER(Config), _i64, _i64, _i32]),
+    "sls_compress": (_i32, [ctypes.POINTER(Config), _vp, _i32, _i64, _i64, _i32, _i64,
+                            ctypes.POINTER(_Params), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "sls_workspace_status": (_i32, [_vp, _vp]),
+}
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libsls.so (built by ``python -m paper_2607_19368_gb300.build``)."""
+    global _lib
+    if _lib is None:
+        path = lib_path()
+        if not os.path.exists(path):
+            raise RuntimeError(
+                f"{path} is missing: build the CUDA library first "
+                "(python -m paper_2607_19368_gb300.build); there is no CPU fallback")
+        L = ctypes.CDLL(path)
+        for name, (res, args) in EXPORTED.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(fn: str, st: int):
+    if st != SLS_OK:
+        raise SLSError(fn, st, lib().sls_status_string(st).decode())
+
+
+def _stream(t: torch.Tensor):
+    return ctypes.c_void_p(torch.cuda.current_stream(t.device).cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return SLS_F32
+    if t.dtype == torch.bfloat16:
+        return SLS_BF16
+    raise TypeError(f"unsupported embedding dtype {t.dtype} (float32 or bfloat16)")
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None and not t.is_cuda:
+            raise ValueError("libsls works on CUDA tensors only (no CPU fallback)")
+
+
+def _workspace(nbytes: int, device) -> torch.Tensor:
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def feature_map(X: torch.Tensor, W: torch.Tensor, b: torch.Tensor,
+                out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Phi = sqrt(2/D) cos(X W^T + b) (Sec. 3.2, Eq. rff_map); X is N x d,
+    W = Omega^T is D x d (same dtype), b has D floats.  Returns N x D float32."""
+    _need_cuda(X, W, b)
+    N, d = X.shape
+    D = W.shape[0]
+    assert W.shape[1] == d and W.dtype == X.dtype and W.is_contiguous()
+    if out is None:
+        out = torch.empty((N, D), dtype=torch.float32, device=X.device)
+    st = lib().sls_feature_map(_ptr(X), _dtype_code(X), N, d, X.stride(0), _ptr(W),
+                               _ptr(b.float().contiguous()), D, _ptr(out), _stream(X))
+    _check("sls_feature_map", st)
+    return out
+
+
+def lanczos_topr(Phi: torch.Tensor, q1: torch.Tensor, r: int, tol: float = 1e-10):
+    """Algorithm 2 on A(v) = Phi (Phi^T v), then Eigh(T) and U = Q V
+    (Algorithm 1).  Returns (theta[r] float64 descending, U[N, r] float32,
+    r_eff[1] int32, alpha[r], beta[r]) as device tensors."""
+    _need_cuda(Phi, q1)
+    Phi = Phi.contiguous()
+    N, D = Phi.shape
+    dev = Phi.device
+    q1 = q1.to(device=dev, dtype=torch.float64).contiguous()
+    theta = torch.empty(r, dtype=torch.float64, device=dev)
+    U = torch.empty((N, r), dtype=torch.float32, device=dev)
+    r_eff = torch.empty(1, dtype=torch.int32, device=dev)
+    alpha = torch.empty(r, dtype=torch.float64, device=dev)
+    beta = torch.empty(r, dtype=torch.float64, device=dev)
+    L = lib()
+    nbytes = L.sls_lanczos_workspace_size(N, D, r)
+    if nbytes == 0:
+        raise SLSError("sls_lanczos_workspace_size", 2, "unsupported shape")
+    ws = _workspace(nbytes, dev)
+    st = L.sls_lanczos_topr(_ptr(Phi), N, D, r, _ptr(q1), float(tol), _ptr(theta), _ptr(U),
+                            _ptr(r_eff), _ptr(alpha), _ptr(beta), _ptr(ws), ws.numel(),
+                            _stream(Phi))
+    _check("sls_lanczos_topr", st)
+    return theta, U, r_eff, alpha, beta
+
+
+def simhash(U: torch.Tensor, R: torch.Tensor, bits: int, k: Optional[int] = None,
+            k_dev: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """SimHash codes of the rows of U (Sec. 3.3, Eq. simhash) against the
+    first `bits` rows of R; returns N uint32 codes as an int32 tensor."""
+    _need_cuda(U, R)
+    N, ldu = U.shape[0], U.stride(0)
+    k = U.shape[1] if k is None else k
+    R = R.float().contiguous()
+    codes = torch.empty(N, dtype=torch.int32, device=U.device)
+    st = lib().sls_simhash(_ptr(U), N, k, ldu, _ptr(k_dev), _ptr(R), bits, R.stride(0),
+                           _ptr(codes), _stream(U))
+    _check("sls_simhash", st)
+    return codes
+
+
+def aggregate(X: torch.Tensor, codes: torch.Tensor, M_target: int, pos_scheme: int = POS_MAX,
+              renorm: bool = True):
+    """Clusters of equal codes, adjusted to exactly M_target groups, merged
+    into macro-tokens ordered by position (Sec. 3.3-3.4).  Returns
+    (Xt[M, d] float32, pos[M] int32, tok2macro[N] int32)."""
+    _need_cuda(X, codes)
+    N, d = X.shape
+    dev = X.device
+    Xt = torch.empty((M_target, d), dtype=torch.float32, device=dev)
+    pos = torch.empty(M_target, dtype=torch.int32, device=dev)
+    t2m = torch.empty(N, dtype=torch.int32, device=dev)
+    L = lib()
+    nbytes = L.sls_aggregate_workspace_size(N, d, M_target)
+    if nbytes == 0:
+        raise SLSError("sls_aggregate_workspace_size", 1, "invalid shape")
+    ws = _workspace(nbytes, dev)
+    st = L.sls_aggregate(_ptr(X), _dtype_code(X), N, d, X.stride(0), _ptr(codes.contiguous()),
+                         M_target, pos_scheme, int(renorm), _ptr(Xt), _ptr(pos), _ptr(t2m),
+                         _ptr(ws), ws.numel(), _stream(X))
+    _check("sls_aggregate", st)
+    return Xt, pos, t2m
+
+
+def output_count(cfg: Config, N: int) -> int:
+    return int(lib().sls_output_count(ctypes.byref(cfg), N))
+
+
+def compress_workspace_size(cfg: Config, B: int, N: int, d: int) -> int:
+    return int(lib().sls_compress_workspace_size(ctypes.byref(cfg), B, N, d))
+
+
+class Workspace:
+    """A reusable device workspace for compress() (sized for one shape)."""
+
+    def __init__(self, cfg: Config, B: int, N: int, d: int, device):
+        self.nbytes = compress_workspace_size(cfg, B, N, d)
+        if self.nbytes == 0:
+            raise SLSError("sls_compress_workspace_size", 1, "invalid configuration")
+        self.buf = _workspace(self.nbytes, device)
+
+
+def compress(X: torch.Tensor, cfg: Config, W: Optional[torch.Tensor] = None,
+             b: Optional[torch.Tensor] = None, R: Optional[torch.Tensor] = None,
+             q1: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
+             out=None):
+    """The whole compression pass (Algorithm 1 with the backends of Sec. 3.5
+    and 3.6).  X is N x d or B x N x d (float32 or bfloat16).  Returns
+    (Xt, pos, tok2macro, r_eff, route); Xt is [B,] M x d float32."""
+    _need_cuda(X)
+    batched = X.dim() == 3
+    X3 = X if batched else X.unsqueeze(0)
+    B, N, d = X3.shape
+    assert X3.stride(2) == 1 and X3.stride(0) == N * X3.stride(1)
+    dev = X.device
+    M = output_count(cfg, N)
+    if M < 0:
+        raise SLSError("sls_output_count", 1, "invalid configuration")
+    if out is None:
+        Xt = torch.empty((B, M, d), dtype=torch.float32, device=dev)
+        pos = torch.empty((B, M), dtype=torch.int32, device=dev)
+        t2m = torch.empty((B, N), dtype=torch.int32, device=dev)
+    else:
+        Xt, pos, t2m = out
+    nwin = max(1, B * ((N + max(1, cfg.window) - 1) // max(1, cfg.window)))
+    r_eff = torch.zeros(nwin, dtype=torch.int32, device=dev)
+    route = torch.zeros(nwin, dtype=torch.int32, device=dev)
+    if workspace is None:
+        workspace = Workspace(cfg, B, N, d, dev)
+    params = None
+    keep = []
+    if cfg.backend != BACKEND_CHUNK and cfg.rho > 1.0:
+        assert W is not None and b is not None and R is not None and q1 is not None
+        Wc = W.contiguous()
+        bc = b.float().contiguous()
+        Rc = R.float().contiguous()
+        qc = q1.to(device=dev, dtype=torch.float64).contiguous()
+        keep = [Wc, bc, Rc, qc]
+        q1_stride = qc.numel() // B if batched else 0
+        params = _Params(Wc.data_ptr(), bc.data_ptr(), Rc.data_ptr(), Rc.shape[0], Rc.stride(0),
+                         qc.data_ptr(), q1_stride)
+    st = lib().sls_compress(ctypes.byref(cfg), _ptr(X3), _dtype_code(X3), B, N, d,
+                            X3.stride(1), ctypes.byref(params) if params is not None else None,
+                            _ptr(Xt), _ptr(pos), _ptr(t2m), _ptr(r_eff), _ptr(route),
+                            _ptr(workspace.buf), workspace.nbytes, _stream(X3))
+    _check("sls_compress", st)
+    del keep
+    if not batched:
+        return Xt[0], pos[0], t2m[0], r_eff, route
+    return Xt, pos, t2m, r_eff, route
+
+
+def workspace_status(workspace: Workspace) -> int:
+    """Device status word of a compress workspace (0 = ok, 5 = timeout)."""
+    return int(lib().sls_workspace_status(_ptr(workspace.buf),
+                                          _stream(workspace.buf)))

@@ -1,0 +1,972 @@
+// SimHash (Sec. 3.3), clusters and the exact-length adjustment (Sec. 3.3),
+// macro-token aggregation with positions (Sec. 3.4) and the window
+// redundancy score of the adaptive router (Sec. 3.6, Eq. redundancy).
+//
+// Work is organised by "problems" (one token set compressed on its own; see
+// segment.cuh).  The per-problem bookkeeping -- a stable radix sort of
+// (code, token), cluster boundaries, the merge or D'Hondt split to exactly m
+// groups, group positions and the ordering of groups by position -- runs in
+// one 1024-thread CTA per problem and touches only integers.  Reading X and
+// writing the macro-token embeddings is spread over the whole GPU.
+#include <climits>
+
+#include "common.cuh"
+#include "kernels.cuh"
+#include "segment.cuh"
+
+namespace sls {
+
+// ============================================================================
+// SimHash: code[i] = sum_l [ fl32 dot(U[i,:k], R[l,:k]) > 0 ] << l
+// ============================================================================
+
+namespace {
+
+SLS_DEV uint32_t simhash_row(const float* __restrict__ u, int k, const float* __restrict__ Rs,
+                             int bits) {
+  float acc[SLS_MAX_BITS];
+#pragma unroll
+  for (int l = 0; l < SLS_MAX_BITS; ++l) acc[l] = 0.0f;
+  for (int m = 0; m < k; ++m) {
+    const float um = u[m];
+#pragma unroll
+    for (int l = 0; l < SLS_MAX_BITS; ++l)
+      if (l < bits) acc[l] = __fadd_rn(acc[l], __fmul_rn(um, Rs[l * k + m]));
+  }
+  uint32_t code = 0;
+#pragma unroll
+  for (int l = 0; l < SLS_MAX_BITS; ++l)
+    if (l < bits && acc[l] > 0.0f) code |= (1u << l);
+  return code;
+}
+
+__global__ void __launch_bounds__(256)
+simhash_kernel(const float* __restrict__ U, int64_t N, int k, int ldu,
+               const int32_t* __restrict__ k_dev, const float* __restrict__ R, int bits,
+               int ldr, uint32_t* __restrict__ codes) {
+  extern __shared__ float Rs[];
+  int kk = k;
+  if (k_dev) kk = min(kk, max(0, (int)*k_dev));
+  for (int e = threadIdx.x; e < bits * kk; e += blockDim.x) Rs[e] = R[(e / kk) * ldr + e % kk];
+  __syncthreads();
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < N;
+       i += (int64_t)gridDim.x * blockDim.x)
+    codes[i] = simhash_row(U + i * ldu, kk, Rs, bits);
+}
+
+// Batched over spectral problems: rows of problem p start at phi_row, k is
+// the problem's r_eff, bits its own bit count.
+__global__ void __launch_bounds__(256)
+simhash_batched_kernel(const ProbDesc* __restrict__ probs, const int* __restrict__ spec_list,
+                       const int* __restrict__ nspec_dev, int nspec_max,
+                       const int* __restrict__ r_eff, const float* __restrict__ U, int ldu,
+                       const float* __restrict__ R, int ldr, uint32_t* __restrict__ codes) {
+  extern __shared__ float Rs[];
+  const int s = blockIdx.y;
+  int nspec = nspec_max;
+  if (nspec_dev) nspec = min(nspec, *nspec_dev);
+  if (s >= nspec) return;
+  const ProbDesc P = probs[spec_list ? spec_list[s] : s];
+  const int kk = min(ldu, max(0, r_eff[s]));
+  const int bits = P.bits;
+  for (int e = threadIdx.x; e < bits * kk; e += blockDim.x) Rs[e] = R[(e / kk) * ldr + e % kk];
+  __syncthreads();
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < P.n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    codes[P.phi_row + i] = simhash_row(U + (P.phi_row + i) * ldu, kk, Rs, bits);
+}
+
+// ============================================================================
+// block-level integer primitives (1024 threads)
+// ============================================================================
+
+constexpr int SEG_T = 1024;
+constexpr int SEG_W = SEG_T / 32;
+
+SLS_DEV unsigned lanemask_lt() {
+  unsigned m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Exclusive scan of 1024 per-thread values; returns the exclusive prefix of
+// the calling thread, *total receives the sum.  sh: SEG_W + 1 ints.
+template <typename T>
+SLS_DEV T block_excl_scan(T v, T* sh, T* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  T x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    T y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  __syncthreads();
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    T w = (lane < SEG_W) ? sh[lane] : (T)0;
+    T z = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      T y = __shfl_up_sync(0xffffffffu, z, o);
+      if (lane >= o) z += y;
+    }
+    if (lane < SEG_W) sh[lane] = z - w;
+    if (lane == SEG_W - 1) sh[SEG_W] = z;
+  }
+  __syncthreads();
+  const T res = sh[warp] + x - v;
+  *total = sh[SEG_W];
+  __syncthreads();
+  return res;
+}
+
+// Exclusive scan of in[0..n) into out (may alias); returns the total.
+// Each thread scans a contiguous chunk serially.
+template <typename T>
+SLS_DEV T block_scan_array(const T* in, T* out, int n, T* sh) {
+  const int tid = threadIdx.x;
+  const int chunk = (n + SEG_T - 1) / SEG_T;
+  const int b = min(n, tid * chunk), e = min(n, b + chunk);
+  T s = 0;
+  for (int i = b; i < e; ++i) s += in[i];
+  T total;
+  T off = block_excl_scan<T>(s, sh, &total);
+  for (int i = b; i < e; ++i) {
+    const T v = in[i];
+    out[i] = off;
+    off += v;
+  }
+  __syncthreads();
+  return total;
+}
+
+template <typename T>
+SLS_DEV T block_sum(T v, T* sh) {
+  T total;
+  block_excl_scan<T>(v, sh, &total);
+  return total;
+}
+
+// Stable LSD radix sort of (key, val) pairs on the low key_bits bits, one
+// 8-bit digit per pass, ping-ponging between the (ka, va) and (kb, vb)
+// buffers in global memory.  On return (ka, va) point at the sorted data.
+// sh: 256 + 256 + SEG_W * 256 ints.
+template <typename K>
+SLS_DEV void block_radix_sort(K*& ka, int*& va, K*& kb, int*& vb, int n, int key_bits, int* sh) {
+  int* base = sh;
+  int* tot = sh + 256;
+  int* wc = sh + 512;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int shift = 0; shift < key_bits; shift += 8) {
+    if (tid < 256) base[tid] = 0;
+    __syncthreads();
+    for (int i = tid; i < n; i += SEG_T) atomicAdd(&base[(int)((ka[i] >> shift) & 255)], 1);
+    __syncthreads();
+    if (tid < 256) {
+      // exclusive scan of 256 bins by the first 8 warps
+      int v = base[tid];
+      int x = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+      }
+      if (lane == 31) tot[warp] = x;
+      __syncwarp();
+      x -= v;
+      base[tid] = x;  // warp-local exclusive prefix
+    }
+    __syncthreads();
+    if (tid < 256) {
+      int add = 0;
+      for (int w = 0; w < warp; ++w) add += tot[w];
+      base[tid] += add;
+    }
+    __syncthreads();
+    for (int t0 = 0; t0 < n; t0 += SEG_T) {
+      for (int e = tid; e < SEG_W * 256; e += SEG_T) wc[e] = 0;
+      __syncthreads();
+      const int i = t0 + tid;
+      const bool valid = i < n;
+      K key = 0;
+      int val = 0;
+      unsigned dg = 256u + (unsigned)lane;
+      if (valid) {
+        key = ka[i];
+        val = va[i];
+        dg = (unsigned)((key >> shift) & 255);
+      }
+      const unsigned peers = __match_any_sync(0xffffffffu, dg);
+      const int rank = __popc(peers & lanemask_lt());
+      if (valid && rank == 0) wc[warp * 256 + dg] = __popc(peers);
+      __syncthreads();
+      if (tid < 256) {
+        int run = 0;
+        for (int w = 0; w < SEG_W; ++w) {
+          const int c = wc[w * 256 + tid];
+          wc[w * 256 + tid] = run;
+          run += c;
+        }
+        tot[tid] = run;
+      }
+      __syncthreads();
+      if (valid) {
+        const int pos = base[dg] + wc[warp * 256 + dg] + rank;
+        kb[pos] = key;
+        vb[pos] = val;
+      }
+      __syncthreads();
+      if (tid < 256) base[tid] += tot[tid];
+      __syncthreads();
+    }
+    K* tk = ka;
+    ka = kb;
+    kb = tk;
+    int* tv = va;
+    va = vb;
+    vb = tv;
+  }
+}
+
+SLS_DEV int bit_length_u64(unsigned long long x) { return x ? 64 - __clzll((long long)x) : 0; }
+
+// Per-problem scratch layout (ints unless noted), identical on host and device.
+struct SegLayout {
+  size_t ka, kb, va, vb, f, cst, grp, gst, gmax, gmin, gsum, ok_a, ok_b, ov_a, ov_b, oidx, rep,
+      seat, total;
+};
+
+__host__ __device__ inline size_t seg_al(size_t x) { return (x + 255) & ~(size_t)255; }
+
+__host__ __device__ inline SegLayout seg_layout(int64_t nmax, int64_t mmax) {
+  SegLayout L;
+  size_t o = 0;
+  const size_t n1 = (size_t)nmax + 1, m1 = (size_t)mmax + 1;
+  L.ka = o;   o += seg_al(n1 * 8);   // keys (uint32 for codes, uint64 reused)
+  L.kb = o;   o += seg_al(n1 * 8);
+  L.va = o;   o += seg_al(n1 * 4);
+  L.vb = o;   o += seg_al(n1 * 4);
+  L.f = o;    o += seg_al(n1 * 4);
+  L.cst = o;  o += seg_al(n1 * 4);
+  L.grp = o;  o += seg_al(n1 * 4);
+  L.gst = o;  o += seg_al(m1 * 4);
+  L.gmax = o; o += seg_al(m1 * 4);
+  L.gmin = o; o += seg_al(m1 * 4);
+  L.gsum = o; o += seg_al(m1 * 8);
+  L.ok_a = o; o += seg_al(m1 * 8);
+  L.ok_b = o; o += seg_al(m1 * 8);
+  L.ov_a = o; o += seg_al(m1 * 4);
+  L.ov_b = o; o += seg_al(m1 * 4);
+  L.oidx = o; o += seg_al(m1 * 4);
+  L.rep = o;  o += seg_al(m1 * 4);
+  L.seat = o; o += seg_al(n1 * 4);
+  L.total = o;
+  return L;
+}
+
+// Number of D'Hondt quotients n/m (2 <= m <= n) that are >= a / 2^40.
+SLS_DEV long long dhondt_count_ge(long long n, long long a) {
+  if (n < 2) return 0;
+  long long k = (a == 0) ? n : min(n, (n << 40) / a);
+  return k > 1 ? k - 1 : 0;
+}
+
+// ============================================================================
+// segment kernel: one CTA per problem
+// ============================================================================
+
+__global__ void __launch_bounds__(SEG_T, 1)
+segment_kernel(const ProbDesc* __restrict__ probs, int nprob, const uint32_t* __restrict__ codes,
+               int pos_scheme, int pos_mode, char* scratch, size_t pstride, int64_t nmax,
+               int64_t mmax, int* __restrict__ perm, int* __restrict__ mstart,
+               int* __restrict__ mlen, int32_t* __restrict__ pos_out,
+               int32_t* __restrict__ tok2macro) {
+  __shared__ int sh_sort[512 + SEG_W * 256];
+  __shared__ long long sh_ll[SEG_W + 1];
+  __shared__ int sh_i[SEG_W + 1];
+  __shared__ long long sh_lo, sh_hi;
+  const int tid = threadIdx.x;
+  const SegLayout L = seg_layout(nmax, mmax);
+  char* sb = scratch + (size_t)blockIdx.x * pstride;
+
+  for (int p = blockIdx.x; p < nprob; p += gridDim.x) {
+    const ProbDesc P = probs[p];
+    const int n = P.n, M = P.m;
+    if (n <= 0 || M <= 0) continue;
+    int* va = reinterpret_cast<int*>(sb + L.va);
+    int* vb = reinterpret_cast<int*>(sb + L.vb);
+    int* f = reinterpret_cast<int*>(sb + L.f);
+    int* cst = reinterpret_cast<int*>(sb + L.cst);
+    int* grp = reinterpret_cast<int*>(sb + L.grp);
+    int* gst = reinterpret_cast<int*>(sb + L.gst);
+    int* gmax = reinterpret_cast<int*>(sb + L.gmax);
+    int* gmin = reinterpret_cast<int*>(sb + L.gmin);
+    unsigned long long* gsum = reinterpret_cast<unsigned long long*>(sb + L.gsum);
+    int* oidx = reinterpret_cast<int*>(sb + L.oidx);
+    int* rep = reinterpret_cast<int*>(sb + L.rep);
+    int* seat = reinterpret_cast<int*>(sb + L.seat);
+    bool merged = false;
+
+    if (P.spectral) {
+      // ---- stable sort of (code, token) ----
+      uint32_t* ka = reinterpret_cast<uint32_t*>(sb + L.ka);
+      uint32_t* kb = reinterpret_cast<uint32_t*>(sb + L.kb);
+      for (int i = tid; i < n; i += SEG_T) {
+        ka[i] = codes[P.phi_row + i];
+        va[i] = i;
+      }
+      __syncthreads();
+      block_radix_sort<uint32_t>(ka, va, kb, vb, n, P.bits, sh_sort);
+      // ---- clusters: runs of equal codes ----
+      for (int s = tid; s < n; s += SEG_T) f[s] = (s == 0 || ka[s] != ka[s - 1]) ? 1 : 0;
+      __syncthreads();
+      const int C = block_scan_array<int>(f, grp, n, sh_i);  // grp[s] = clusters before s
+      for (int s = tid; s < n; s += SEG_T)
+        if (f[s]) cst[grp[s]] = s;
+      if (tid == 0) cst[C] = n;
+      __syncthreads();
+      if (C >= M) {
+        // merge: the cluster of rank t joins group floor(t M / C)
+        merged = (C > M);
+        for (int t = tid; t < C; t += SEG_T) {
+          const int g = (int)(((long long)t * M) / C);
+          const int gp = (t == 0) ? -1 : (int)(((long long)(t - 1) * M) / C);
+          if (g != gp) gst[g] = cst[t];
+        }
+      } else {
+        // split: D'Hondt seats, one guaranteed per cluster, ties to the lower code
+        const long long K = (long long)(M - C);
+        int maxn = 0;
+        for (int t = tid; t < C; t += SEG_T) maxn = max(maxn, cst[t + 1] - cst[t]);
+        // block max via the sum helper on a per-thread max is not valid; use atomics
+        if (tid == 0) sh_i[0] = 0;
+        __syncthreads();
+        atomicMax(&sh_i[0], maxn);
+        __syncthreads();
+        maxn = sh_i[0];
+        __syncthreads();
+        long long lo = 0, hi = ((long long)maxn) << 40;
+        while (hi - lo > 1) {
+          const long long mid = lo + (hi - lo) / 2;
+          long long c = 0;
+          for (int t = tid; t < C; t += SEG_T) c += dhondt_count_ge(cst[t + 1] - cst[t], mid);
+          c = block_sum<long long>(c, sh_ll);
+          if (c >= K) lo = mid;
+          else hi = mid;
+        }
+        // seats strictly above the K-th quotient, and ties at it (<= 1 per cluster)
+        long long gt_sum = 0;
+        for (int t = tid; t < C; t += SEG_T) {
+          const long long nt = cst[t + 1] - cst[t];
+          const long long ge = dhondt_count_ge(nt, lo);
+          const long long gt = dhondt_count_ge(nt, lo + 1);
+          seat[t] = (int)gt;
+          f[t] = (int)(ge - gt);
+          gt_sum += gt;
+        }
+        gt_sum = block_sum<long long>(gt_sum, sh_ll);
+        const int R = (int)(K - gt_sum);
+        __syncthreads();
+        // exclusive scan of the tie flags in cluster order
+        int* eqs = grp;  // reuse as scratch (size >= C)
+        block_scan_array<int>(f, eqs, C, sh_i);
+        for (int t = tid; t < C; t += SEG_T) {
+          const int extra = (f[t] && eqs[t] < R) ? 1 : 0;
+          seat[t] = 1 + seat[t] + extra;
+        }
+        __syncthreads();
+        int* so = f;  // seat offsets
+        block_scan_array<int>(seat, so, C, sh_i);
+        for (int t = tid; t < C; t += SEG_T) {
+          const int nt = cst[t + 1] - cst[t], pt = seat[t];
+          const int q = nt / pt, rem = nt % pt;
+          for (int k = 0; k < pt; ++k) {
+            const int off = (k < rem) ? k * (q + 1) : rem * (q + 1) + (k - rem) * q;
+            gst[so[t] + k] = cst[t] + off;
+          }
+        }
+      }
+      if (tid == 0) gst[M] = n;
+      __syncthreads();
+    } else {
+      // chunk: contiguous groups (array_split into m, or runs of k)
+      for (int i = tid; i < n; i += SEG_T) va[i] = i;
+      for (int g = tid; g < M; g += SEG_T) {
+        int off;
+        if (P.chunk_k > 0) {
+          off = min(n, g * P.chunk_k);
+        } else {
+          const int q = n / M, rem = n % M;
+          off = (g < rem) ? g * (q + 1) : rem * (q + 1) + (g - rem) * q;
+        }
+        gst[g] = off;
+      }
+      if (tid == 0) gst[M] = n;
+      __syncthreads();
+    }
+    const int* perm_l = va;  // sorted position -> local token
+    // ---- group id of every sorted position ----
+    for (int s = tid; s < n; s += SEG_T) f[s] = 0;
+    __syncthreads();
+    for (int g = tid; g < M; g += SEG_T) f[gst[g]] = 1;
+    __syncthreads();
+    block_scan_array<int>(f, grp, n, sh_i);
+    for (int s = tid; s < n; s += SEG_T) grp[s] = grp[s] + f[s] - 1;
+    for (int g = tid; g < M; g += SEG_T) {
+      gmax[g] = -1;
+      gmin[g] = INT_MAX;
+      gsum[g] = 0ull;
+    }
+    __syncthreads();
+    for (int s = tid; s < n; s += SEG_T) {
+      const int g = grp[s], i = perm_l[s];
+      atomicMax(&gmax[g], i);
+      atomicMin(&gmin[g], i);
+      if (pos_scheme == SLS_POS_MEAN) atomicAdd(&gsum[g], (unsigned long long)i);
+    }
+    __syncthreads();
+    // ---- representative positions ----
+    if (pos_scheme == SLS_POS_MEDIAN && merged) {
+      // members of merged groups are not in token order: sort (group, token)
+      uint32_t* ka = reinterpret_cast<uint32_t*>(sb + L.ka);
+      uint32_t* kb = reinterpret_cast<uint32_t*>(sb + L.kb);
+      int* xa = seat;
+      int* xb = cst;
+      for (int s = tid; s < n; s += SEG_T) ka[perm_l[s]] = (uint32_t)grp[s];
+      for (int i = tid; i < n; i += SEG_T) xa[i] = i;
+      __syncthreads();
+      block_radix_sort<uint32_t>(ka, xa, kb, xb, n, bit_length_u64((unsigned long long)M), sh_sort);
+      for (int g = tid; g < M; g += SEG_T) rep[g] = xa[gst[g] + (gst[g + 1] - gst[g] - 1) / 2];
+    } else {
+      for (int g = tid; g < M; g += SEG_T) {
+        const int len = gst[g + 1] - gst[g];
+        int rp;
+        if (pos_scheme == SLS_POS_MAX) rp = gmax[g];
+        else if (pos_scheme == SLS_POS_MEDIAN) rp = perm_l[gst[g] + (len - 1) / 2];
+        else rp = (int)((2ull * gsum[g] + (unsigned long long)len) / (2ull * (unsigned long long)len));
+        rep[g] = rp;
+      }
+    }
+    __syncthreads();
+    // ---- order groups by (position, first token) ----
+    {
+      unsigned long long* oka = reinterpret_cast<unsigned long long*>(sb + L.ok_a);
+      unsigned long long* okb = reinterpret_cast<unsigned long long*>(sb + L.ok_b);
+      int* ova = reinterpret_cast<int*>(sb + L.ov_a);
+      int* ovb = reinterpret_cast<int*>(sb + L.ov_b);
+      for (int g = tid; g < M; g += SEG_T) {
+        oka[g] = (unsigned long long)rep[g] * (unsigned long long)n + (unsigned long long)gmin[g];
+        ova[g] = g;
+      }
+      __syncthreads();
+      const int kbits = bit_length_u64((unsigned long long)n * (unsigned long long)n);
+      block_radix_sort<unsigned long long>(oka, ova, okb, ovb, M, kbits, sh_sort);
+      for (int t = tid; t < M; t += SEG_T) {
+        const int g = ova[t];
+        oidx[g] = t;
+        const int64_t mrow = P.out0 + t;
+        mstart[mrow] = (int)(P.tok_row + gst[g]);
+        mlen[mrow] = gst[g + 1] - gst[g];
+        pos_out[mrow] = (pos_mode == SLS_MODE_COMPACT) ? (P.out_local + t) : (P.pos0 + rep[g]);
+      }
+      __syncthreads();
+      for (int s = tid; s < n; s += SEG_T) {
+        const int i = perm_l[s];
+        perm[P.tok_row + s] = (int)(P.tok_row + i);
+        tok2macro[P.tok_row + i] = P.out_local + oidx[grp[s]];
+      }
+      __syncthreads();
+    }
+  }
+}
+
+// ============================================================================
+// preserved tokens, identity
+// ============================================================================
+
+__global__ void preserved_kernel(int64_t B, int64_t N, int64_t M, int pf, int pl, int pos_mode,
+                                 int* __restrict__ perm, int* __restrict__ mstart,
+                                 int* __restrict__ mlen, int32_t* __restrict__ pos_out,
+                                 int32_t* __restrict__ tok2macro) {
+  const int per = pf + pl;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < B * per;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t b = e / per;
+    const int k = (int)(e % per);
+    int64_t tok, mac;
+    if (k < pf) {
+      tok = k;
+      mac = k;
+    } else {
+      tok = N - pl + (k - pf);
+      mac = M - pl + (k - pf);
+    }
+    const int64_t trow = b * N + tok, mrow = b * M + mac;
+    perm[trow] = (int)trow;
+    mstart[mrow] = (int)trow;
+    mlen[mrow] = 1;
+    pos_out[mrow] = (int32_t)((pos_mode == SLS_MODE_COMPACT) ? mac : tok);
+    tok2macro[trow] = (int32_t)mac;
+  }
+}
+
+template <typename T>
+SLS_DEV float to_f32(T v);
+template <>
+SLS_DEV float to_f32<float>(float v) {
+  return v;
+}
+template <>
+SLS_DEV float to_f32<uint16_t>(uint16_t v) {
+  return __uint_as_float(((unsigned)v) << 16);
+}
+
+template <typename T>
+__global__ void identity_kernel(const T* __restrict__ X, int64_t B, int64_t N, int d, int64_t ldx,
+                                float* __restrict__ Xt, int32_t* __restrict__ pos,
+                                int32_t* __restrict__ tok2macro) {
+  const int64_t total = B * N * d;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t row = e / d;
+    const int c = (int)(e % d);
+    Xt[e] = to_f32<T>(X[row * ldx + c]);
+    if (c == 0) {
+      pos[row] = (int32_t)(row % N);
+      tok2macro[row] = (int32_t)(row % N);
+    }
+  }
+}
+
+// ============================================================================
+// token norms and macro-token embeddings (Eq. macro_embed)
+// ============================================================================
+
+// |x_i| for every token row; one warp per row.
+template <typename T>
+__global__ void __launch_bounds__(256)
+row_norms_kernel(const T* __restrict__ X, int64_t rows, int d, int64_t ldx,
+                 float* __restrict__ norms) {
+  const int lane = threadIdx.x & 31;
+  const int64_t wid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = wid; i < rows; i += nw) {
+    const T* x = X + i * ldx;
+    float s = 0.f;
+    for (int c = lane; c < d; c += 32) {
+      const float v = to_f32<T>(x[c]);
+      s = fmaf(v, v, s);
+    }
+    s = warp_sum_f(s);
+    if (lane == 0) norms[i] = sqrtf(s);
+  }
+}
+
+constexpr int AGG_T = 256;
+constexpr int AGG_CH = 64;      // members per work item
+constexpr int AGG_MAXV = 32;    // accumulators per thread (d <= 8192)
+
+// Work items: macro-token m is split into ceil(len / AGG_CH) items.
+__global__ void __launch_bounds__(SEG_T, 1)
+agg_items_kernel(const int* __restrict__ mlen, int64_t Mtot, int* __restrict__ it_start,
+                 int* __restrict__ pt_start, int2* __restrict__ items, int* __restrict__ counts) {
+  __shared__ int sh[SEG_W + 1];
+  const int tid = threadIdx.x;
+  const int chunk = (int)((Mtot + SEG_T - 1) / SEG_T);
+  const int64_t b = min(Mtot, (int64_t)tid * chunk), e = min(Mtot, b + chunk);
+  int s1 = 0, s2 = 0;
+  for (int64_t m = b; m < e; ++m) {
+    const int nch = (mlen[m] + AGG_CH - 1) / AGG_CH;
+    s1 += nch;
+    s2 += (nch > 1) ? nch : 0;
+  }
+  int t1, t2;
+  int o1 = block_excl_scan<int>(s1, sh, &t1);
+  int o2 = block_excl_scan<int>(s2, sh, &t2);
+  for (int64_t m = b; m < e; ++m) {
+    const int nch = (mlen[m] + AGG_CH - 1) / AGG_CH;
+    it_start[m] = o1;
+    pt_start[m] = (nch > 1) ? o2 : -1;
+    for (int c = 0; c < nch; ++c) items[o1 + c] = make_int2((int)m, c);
+    o1 += nch;
+    o2 += (nch > 1) ? nch : 0;
+  }
+  if (tid == 0) {
+    counts[0] = t1;
+    counts[1] = t2;
+  }
+}
+
+template <typename T>
+struct VecOf;
+template <>
+struct VecOf<float> {
+  static constexpr int V = 4;
+};
+template <>
+struct VecOf<uint16_t> {
+  static constexpr int V = 8;
+};
+
+template <typename T>
+SLS_DEV void load_vec(const T* p, float* out);
+template <>
+SLS_DEV void load_vec<float>(const float* p, float* out) {
+  const float4 v = __ldg(reinterpret_cast<const float4*>(p));
+  out[0] = v.x;
+  out[1] = v.y;
+  out[2] = v.z;
+  out[3] = v.w;
+}
+template <>
+SLS_DEV void load_vec<uint16_t>(const uint16_t* p, float* out) {
+  const uint4 v = __ldg(reinterpret_cast<const uint4*>(p));
+  const unsigned w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    out[2 * k] = __uint_as_float(w[k] << 16);
+    out[2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+  }
+}
+
+SLS_DEV float agg_block_sum(float v, float* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_sum_f(v);
+  __syncthreads();
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  float s = 0.f;
+#pragma unroll
+  for (int w = 0; w < AGG_T / 32; ++w) s += sh[w];
+  return s;
+}
+
+// Finalise one macro-token row from the member sum `acc` (per thread), the
+// member count and the sum of member norms: mean, then rescale to the mean
+// norm (Eq. macro_embed); a singleton is its token unchanged.
+template <int V>
+SLS_DEV void agg_finalize(float (&acc)[AGG_MAXV], int nv, int len, float eta_sum, int renorm, int d,
+                          float* __restrict__ out, float* sh) {
+  const int tid = threadIdx.x;
+  if (len == 1) {
+#pragma unroll
+    for (int q = 0; q < AGG_MAXV / V; ++q) {
+      const int c0 = (tid + q * AGG_T) * V;
+      if (q < nv && c0 < d)
+#pragma unroll
+        for (int v = 0; v < V; ++v) out[c0 + v] = acc[q * V + v];
+    }
+    return;
+  }
+  const float inv = 1.0f / (float)len;
+  float sq = 0.f;
+#pragma unroll
+  for (int q = 0; q < AGG_MAXV / V; ++q) {
+    const int c0 = (tid + q * AGG_T) * V;
+    if (q < nv && c0 < d)
+#pragma unroll
+      for (int v = 0; v < V; ++v) {
+        acc[q * V + v] *= inv;
+        sq = fmaf(acc[q * V + v], acc[q * V + v], sq);
+      }
+  }
+  float scale = 1.0f;
+  if (renorm) {
+    const float nrm = sqrtf(agg_block_sum(sq, sh));
+    if (nrm >= 1e-30f) scale = (eta_sum * inv) / nrm;
+  }
+#pragma unroll
+  for (int q = 0; q < AGG_MAXV / V; ++q) {
+    const int c0 = (tid + q * AGG_T) * V;
+    if (q < nv && c0 < d)
+#pragma unroll
+      for (int v = 0; v < V; ++v) out[c0 + v] = acc[q * V + v] * scale;
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(AGG_T)
+agg_partial_kernel(const T* __restrict__ X, int d, int64_t ldx, const float* __restrict__ norms,
+                   const int* __restrict__ perm, const int* __restrict__ mstart,
+                   const int* __restrict__ mlen, const int2* __restrict__ items,
+                   const int* __restrict__ counts, const int* __restrict__ pt_start, int renorm,
+                   float* __restrict__ Xt, float* __restrict__ part, float* __restrict__ part_eta) {
+  constexpr int V = VecOf<T>::V;
+  __shared__ float sh[AGG_T / 32];
+  const int nitems = counts[0];
+  const int tid = threadIdx.x;
+  const int nv = (d / V + AGG_T - 1) / AGG_T;
+  for (int it = blockIdx.x; it < nitems; it += gridDim.x) {
+    const int2 item = items[it];
+    const int m = item.x, c = item.y;
+    const int len = mlen[m];
+    const int b = c * AGG_CH, e = min(len, b + AGG_CH);
+    const int* mem = perm + mstart[m];
+    float acc[AGG_MAXV];
+#pragma unroll
+    for (int k = 0; k < AGG_MAXV; ++k) acc[k] = 0.f;
+    float eta = 0.f;
+    for (int s = b; s < e; ++s) {
+      const int row = mem[s];
+      const T* x = X + (int64_t)row * ldx;
+      eta += norms[row];
+#pragma unroll
+      for (int q = 0; q < AGG_MAXV / V; ++q) {
+        const int c0 = (tid + q * AGG_T) * V;
+        if (q < nv && c0 < d) {
+          float v[V];
+          load_vec<T>(x + c0, v);
+#pragma unroll
+          for (int k = 0; k < V; ++k) acc[q * V + k] += v[k];
+        }
+      }
+    }
+    const int ps = pt_start[m];
+    if (ps < 0) {
+      agg_finalize<V>(acc, nv, len, eta, renorm, d, Xt + (int64_t)m * d, sh);
+    } else {
+      float* dst = part + (int64_t)(ps + c) * d;
+#pragma unroll
+      for (int q = 0; q < AGG_MAXV / V; ++q) {
+        const int c0 = (tid + q * AGG_T) * V;
+        if (q < nv && c0 < d)
+#pragma unroll
+          for (int k = 0; k < V; ++k) dst[c0 + k] = acc[q * V + k];
+      }
+      if (tid == 0) part_eta[ps + c] = eta;
+    }
+    __syncthreads();
+  }
+}
+
+template <int V>
+__global__ void __launch_bounds__(AGG_T)
+agg_final_kernel(int d, const int* __restrict__ mlen, const int* __restrict__ pt_start,
+                 int64_t Mtot, int renorm, const float* __restrict__ part,
+                 const float* __restrict__ part_eta, float* __restrict__ Xt) {
+  __shared__ float sh[AGG_T / 32];
+  const int tid = threadIdx.x;
+  const int nv = (d / V + AGG_T - 1) / AGG_T;
+  for (int64_t m = blockIdx.x; m < Mtot; m += gridDim.x) {
+    const int ps = pt_start[m];
+    if (ps < 0) continue;
+    const int len = mlen[m];
+    const int nch = (len + AGG_CH - 1) / AGG_CH;
+    float acc[AGG_MAXV];
+#pragma unroll
+    for (int k = 0; k < AGG_MAXV; ++k) acc[k] = 0.f;
+    float eta = 0.f;
+    for (int c = 0; c < nch; ++c) {
+      const float* src = part + (int64_t)(ps + c) * d;
+      eta += part_eta[ps + c];
+#pragma unroll
+      for (int q = 0; q < AGG_MAXV / V; ++q) {
+        const int c0 = (tid + q * AGG_T) * V;
+        if (q < nv && c0 < d)
+#pragma unroll
+          for (int k = 0; k < V; ++k) acc[q * V + k] += src[c0 + k];
+      }
+    }
+    agg_finalize<V>(acc, nv, len, eta, renorm, d, Xt + m * d, sh);
+    __syncthreads();
+  }
+}
+
+// ============================================================================
+// adaptive router: window redundancy score (Eq. redundancy)
+// ============================================================================
+
+// score = (1/L) sum_i cos(x_i, c) with c the window centroid; computed in one
+// pass as (sum_i x_i/|x_i|) . (sum_i x_i) / (L |sum_i x_i|).  Zero rows add 0.
+template <typename T>
+__global__ void __launch_bounds__(AGG_T)
+window_score_kernel(const T* __restrict__ X, int d, int64_t ldx, const float* __restrict__ norms,
+                    const ProbDesc* __restrict__ probs, int nprob, float* __restrict__ score) {
+  constexpr int V = VecOf<T>::V;
+  __shared__ float sh[AGG_T / 32];
+  const int tid = threadIdx.x;
+  const int nv = (d / V + AGG_T - 1) / AGG_T;
+  for (int p = blockIdx.x; p < nprob; p += gridDim.x) {
+    const ProbDesc P = probs[p];
+    float cs[AGG_MAXV], ns[AGG_MAXV];
+#pragma unroll
+    for (int k = 0; k < AGG_MAXV; ++k) cs[k] = ns[k] = 0.f;
+    for (int i = 0; i < P.n; ++i) {
+      const int64_t row = P.tok_row + i;
+      const float nr = norms[row];
+      const float inv = (nr > 0.f) ? 1.0f / nr : 0.f;
+      const T* x = X + row * ldx;
+#pragma unroll
+      for (int q = 0; q < AGG_MAXV / V; ++q) {
+        const int c0 = (tid + q * AGG_T) * V;
+        if (q < nv && c0 < d) {
+          float v[V];
+          load_vec<T>(x + c0, v);
+#pragma unroll
+          for (int k = 0; k < V; ++k) {
+            cs[q * V + k] += v[k];
+            ns[q * V + k] = fmaf(v[k], inv, ns[q * V + k]);
+          }
+        }
+      }
+    }
+    float dot = 0.f, cc = 0.f;
+#pragma unroll
+    for (int k = 0; k < AGG_MAXV; ++k) {
+      dot = fmaf(ns[k], cs[k], dot);
+      cc = fmaf(cs[k], cs[k], cc);
+    }
+    dot = agg_block_sum(dot, sh);
+    cc = agg_block_sum(cc, sh);
+    if (tid == 0) score[p] = (cc > 0.f) ? dot / ((float)P.n * sqrtf(cc)) : 0.f;
+    __syncthreads();
+  }
+}
+
+}  // namespace
+
+// ============================================================================
+// launchers
+// ============================================================================
+
+int launch_simhash(const float* U, int64_t N, int k, int ldu, const int32_t* k_dev,
+                   const float* R, int bits, int ldr, uint32_t* codes, cudaStream_t stream) {
+  if (N == 0) return SLS_OK;
+  const size_t smem = sizeof(float) * bits * k;
+  int64_t blocks = (N + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  if (smem > 48 * 1024)
+    SLS_CUDA_TRY(cudaFuncSetAttribute(simhash_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)smem));
+  simhash_kernel<<<(unsigned)blocks, 256, smem, stream>>>(U, N, k, ldu, k_dev, R, bits, ldr, codes);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+size_t segment_scratch_bytes(int64_t nmax, int64_t mmax, int slots) {
+  return (size_t)slots * seg_layout(nmax, mmax).total;
+}
+
+int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const int* nspec_dev,
+                            int nspec_max, int64_t nmax, const int* r_eff, const float* U, int ldu,
+                            const float* R, int ldr, int bits_max, uint32_t* codes,
+                            cudaStream_t stream) {
+  if (nspec_max <= 0) return SLS_OK;
+  const size_t smem = sizeof(float) * bits_max * ldu;
+  int64_t bx = (nmax + 255) / 256;
+  if (bx > 1024) bx = 1024;
+  if (bx < 1) bx = 1;
+  if (smem > 48 * 1024)
+    SLS_CUDA_TRY(cudaFuncSetAttribute(simhash_batched_kernel,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  simhash_batched_kernel<<<dim3((unsigned)bx, nspec_max), 256, smem, stream>>>(
+      probs, spec_list, nspec_dev, nspec_max, r_eff, U, ldu, R, ldr, codes);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int pos_scheme,
+                   int pos_mode, void* scratch, int slots, int64_t nmax, int64_t mmax, int* perm,
+                   int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,
+                   cudaStream_t stream) {
+  if (nprob <= 0) return SLS_OK;
+  const size_t stride = seg_layout(nmax, mmax).total;
+  const int grid = nprob < slots ? nprob : slots;
+  segment_kernel<<<grid, SEG_T, 0, stream>>>(probs, nprob, codes, pos_scheme, pos_mode,
+                                             (char*)scratch, stride, nmax, mmax, perm, mstart,
+                                             mlen, pos_out, tok2macro);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+int launch_preserved(int64_t B, int64_t N, int64_t M, int pf, int pl, int pos_mode, int* perm,
+                     int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,
+                     cudaStream_t stream) {
+  if (pf + pl == 0 || B == 0) return SLS_OK;
+  int64_t blocks = (B * (pf + pl) + 255) / 256;
+  if (blocks > 1024) blocks = 1024;
+  preserved_kernel<<<(unsigned)blocks, 256, 0, stream>>>(B, N, M, pf, pl, pos_mode, perm, mstart,
+                                                         mlen, pos_out, tok2macro);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+int launch_identity(const void* X, int x_dtype, int64_t B, int64_t N, int d, int64_t ldx,
+                    float* Xt, int32_t* pos, int32_t* tok2macro, cudaStream_t stream) {
+  if (B * N == 0) return SLS_OK;
+  int64_t blocks = (B * N * d + 255) / 256;
+  if (blocks > 65536) blocks = 65536;
+  if (x_dtype == SLS_F32)
+    identity_kernel<float><<<(unsigned)blocks, 256, 0, stream>>>((const float*)X, B, N, d, ldx,
+                                                                  Xt, pos, tok2macro);
+  else
+    identity_kernel<uint16_t><<<(unsigned)blocks, 256, 0, stream>>>((const uint16_t*)X, B, N, d,
+                                                                     ldx, Xt, pos, tok2macro);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+int launch_row_norms(const void* X, int x_dtype, int64_t rows, int d, int64_t ldx, float* norms,
+                     cudaStream_t stream) {
+  if (rows == 0) return SLS_OK;
+  int64_t blocks = (rows * 32 + 255) / 256;
+  if (blocks > 8192) blocks = 8192;
+  if (x_dtype == SLS_F32)
+    row_norms_kernel<float><<<(unsigned)blocks, 256, 0, stream>>>((const float*)X, rows, d, ldx,
+                                                                   norms);
+  else
+    row_norms_kernel<uint16_t><<<(unsigned)blocks, 256, 0, stream>>>((const uint16_t*)X, rows, d,
+                                                                      ldx, norms);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+size_t agg_item_capacity(int64_t Mtot, int64_t Ntot) { return (size_t)(Mtot + Ntot / AGG_CH + 2); }
+size_t agg_part_capacity(int64_t Ntot) { return (size_t)(2 * (Ntot / AGG_CH) + 2); }
+
+int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
+                     const int* perm, const int* mstart, const int* mlen, int64_t Mtot,
+                     int64_t Ntot, int renorm, float* Xt, int* it_start, int* pt_start,
+                     int2* items, int* counts, float* part, float* part_eta,
+                     cudaStream_t stream) {
+  if (Mtot == 0) return SLS_OK;
+  agg_items_kernel<<<1, SEG_T, 0, stream>>>(mlen, Mtot, it_start, pt_start, items, counts);
+  SLS_LAUNCH_CHECK();
+  int64_t blocks = (int64_t)agg_item_capacity(Mtot, Ntot);
+  if (blocks > 16384) blocks = 16384;
+  int64_t fblocks = Mtot < 4096 ? Mtot : 4096;
+  if (x_dtype == SLS_F32) {
+    agg_partial_kernel<float><<<(unsigned)blocks, AGG_T, 0, stream>>>(
+        (const float*)X, d, ldx, norms, perm, mstart, mlen, items, counts, pt_start, renorm, Xt,
+        part, part_eta);
+    SLS_LAUNCH_CHECK();
+    agg_final_kernel<4><<<(unsigned)fblocks, AGG_T, 0, stream>>>(d, mlen, pt_start, Mtot, renorm,
+                                                                 part, part_eta, Xt);
+  } else {
+    agg_partial_kernel<uint16_t><<<(unsigned)blocks, AGG_T, 0, stream>>>(
+        (const uint16_t*)X, d, ldx, norms, perm, mstart, mlen, items, counts, pt_start, renorm,
+        Xt, part, part_eta);
+    SLS_LAUNCH_CHECK();
+    agg_final_kernel<8><<<(unsigned)fblocks, AGG_T, 0, stream>>>(d, mlen, pt_start, Mtot, renorm,
+                                                                 part, part_eta, Xt);
+  }
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
+                        const ProbDesc* probs, int nprob, float* score, cudaStream_t stream) {
+  if (nprob <= 0) return SLS_OK;
+  const int blocks = nprob < 8192 ? nprob : 8192;
+  if (x_dtype == SLS_F32)
+    window_score_kernel<float><<<blocks, AGG_T, 0, stream>>>((const float*)X, d, ldx, norms,
+                                                              probs, nprob, score);
+  else
+    window_score_kernel<uint16_t><<<blocks, AGG_T, 0, stream>>>((const uint16_t*)X, d, ldx,
+                                                                 norms, probs, nprob, score);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+}  // namespace sls

@@ -1,0 +1,87 @@
+// Internal launcher declarations shared by the library's translation units.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace sls {
+
+// ---- feature map (Sec. 3.2) ----------------------------------------------
+int launch_feature_map_simt(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
+                            const void* W, const float* b, int D, float* Phi,
+                            cudaStream_t stream);
+// tcgen05 / TMA path for bf16 inputs; returns SLS_ERR_UNSUPPORTED when the
+// shape is outside what the kernel handles (the caller then uses the SIMT path).
+int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
+                          const float* b, int D, float* Phi, cudaStream_t stream);
+
+// ---- Lanczos (Algorithm 2) --------------------------------------------------
+// A batch of independent problems, problem p owning rows
+// [row0[p], row0[p] + n[p]) of Phi, Q and U and start vector q1 + q1off[p].
+struct LanczosBatch {
+  const float* Phi;     // rows x D
+  int D;
+  int r;
+  double tol;
+  const double* q1;
+  // problem table: either a single problem (table pointers NULL, n_single
+  // rows from row 0) or device arrays read by the kernels
+  int64_t n_single;
+  int nprob_max;            // host upper bound on the number of problems
+  const int* nprob_dev;     // device count (may be NULL: nprob_max problems)
+  const int64_t* row0;      // device, per problem
+  const int* n;             // device, per problem
+  const int64_t* q1off;     // device, per problem (NULL: = row0)
+  // outputs, per problem p: Q rows as above (ld r); alpha/beta/theta at p*r;
+  // S at p*r*r; r_eff at p
+  float2* Q;
+  double* alpha;
+  double* beta;
+  double* theta;
+  double* S;
+  int* r_eff;
+  int64_t nmax;             // max rows of any problem
+};
+
+size_t lanczos_scratch_bytes(int64_t nmax, int D, int r, int groups, int ctas_per_group);
+int lanczos_plan(int64_t nmax, int D, int r, int nprob, int* groups, int* ctas_per_group);
+int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, int* status,
+                   int groups, int ctas_per_group, cudaStream_t stream);
+int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream);
+int launch_ritz_vectors(const LanczosBatch& bt, float* U, cudaStream_t stream);
+
+// ---- SimHash (Sec. 3.3) -----------------------------------------------------
+int launch_simhash(const float* U, int64_t N, int k, int ldu, const int32_t* k_dev,
+                   const float* R, int bits, int ldr, uint32_t* codes, cudaStream_t stream);
+
+}  // namespace sls
+
+// ---- segment / aggregation (hash_aggregate.cu) -------------------------------
+namespace sls {
+struct ProbDesc;
+size_t segment_scratch_bytes(int64_t nmax, int64_t mmax, int slots);
+int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const int* nspec_dev,
+                            int nspec_max, int64_t nmax, const int* r_eff, const float* U, int ldu,
+                            const float* R, int ldr, int bits_max, uint32_t* codes,
+                            cudaStream_t stream);
+int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int pos_scheme,
+                   int pos_mode, void* scratch, int slots, int64_t nmax, int64_t mmax, int* perm,
+                   int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,
+                   cudaStream_t stream);
+int launch_preserved(int64_t B, int64_t N, int64_t M, int pf, int pl, int pos_mode, int* perm,
+                     int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,
+                     cudaStream_t stream);
+int launch_identity(const void* X, int x_dtype, int64_t B, int64_t N, int d, int64_t ldx,
+                    float* Xt, int32_t* pos, int32_t* tok2macro, cudaStream_t stream);
+int launch_row_norms(const void* X, int x_dtype, int64_t rows, int d, int64_t ldx, float* norms,
+                     cudaStream_t stream);
+size_t agg_item_capacity(int64_t Mtot, int64_t Ntot);
+size_t agg_part_capacity(int64_t Ntot);
+int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
+                     const int* perm, const int* mstart, const int* mlen, int64_t Mtot,
+                     int64_t Ntot, int renorm, float* Xt, int* it_start, int* pt_start,
+                     int2* items, int* counts, float* part, float* part_eta,
+                     cudaStream_t stream);
+int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
+                        const ProbDesc* probs, int nprob, float* score, cudaStream_t stream);
+}  // namespace sls

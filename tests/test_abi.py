@@ -1,0 +1,65 @@
+"""The C ABI: the library builds for sm_103a, loads without a GPU and exports
+every entry point declared in include/sls.h; host-side argument checks and
+the output-count arithmetic need no GPU either."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "sls.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^[A-Za-z_][\w \*]*?\b(sls_\w+)\s*\(", src, flags=re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_19368_gb300 import build
+    path = build.build()
+    import paper_2607_19368_gb300 as sls
+    return sls.lib()
+
+
+def test_header_declares_the_five_calls():
+    names = declared_functions()
+    for n in ("sls_feature_map", "sls_lanczos_topr", "sls_simhash", "sls_aggregate",
+              "sls_compress"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    import paper_2607_19368_gb300 as sls
+    names = declared_functions()
+    assert set(names) == set(sls.EXPORTED), (set(names) ^ set(sls.EXPORTED))
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_host_side_errors_and_counts(lib):
+    import paper_2607_19368_gb300 as sls
+    assert lib.sls_version() >= 100
+    assert lib.sls_status_string(5).decode().startswith("device wait")
+    # argument errors are detected before any CUDA call
+    assert lib.sls_feature_map(None, 0, 4, 8, 8, None, None, 6, None, None) == 1  # D % 4
+    assert lib.sls_simhash(None, 4, 4, 4, None, None, 33, 4, None, None) == 1     # bits > 32
+    assert lib.sls_lanczos_topr(None, 4, 8, 0, None, 1e-10, None, None, None, None, None,
+                                None, 0, None) == 1                               # r = 0
+    assert lib.sls_lanczos_workspace_size(1000, 256, 16) > 0
+    # output counts agree with the oracle's target count (Sec. 3.3) and identity
+    for N, rho, pf, pl in [(512, 4.0, 0, 12), (16384, 16.0, 0, 12), (100, 1.0, 0, 12),
+                           (10, 4.0, 3, 20), (1000, 3.0, 5, 7)]:
+        cfg = sls.Config.make(rho=rho, preserve_first=pf, preserve_last=pl)
+        Nc = N - min(pf, N) - min(pl, N - min(pf, N))
+        want = N if (rho <= 1 or Nc <= 0) else min(pf, N) + O.target_count(Nc, rho) + min(pl, N - min(pf, N))
+        assert sls.output_count(cfg, N) == want
+    cfg = sls.Config.make(backend=sls.BACKEND_CHUNK, rho=2.5, preserve_last=0)
+    assert sls.output_count(cfg, 101) == -(-101 // round(2.5))
+    assert sls.compress_workspace_size(sls.Config.make(rho=16.0, D=2048, r=64, bits=16),
+                                       1, 32768, 3584) > 32768 * 2048 * 4

@@ -1,0 +1,372 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle on seeded
+synthetic inputs.  Bars: codes, cluster and token maps bit-exact; Ritz values
+relative error <= 1e-4 with the largest principal angle between the Ritz
+subspaces <= 1e-3 rad (both sides fed the same float32 Phi and q1); macro
+embeddings max-abs <= 1e-4; feature map within the float32 bound of
+gpu_util.feature_tolerance."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as WL
+from tests.gpu_util import feature_tolerance, max_subspace_angle, oracle_phi32, to_torch_x, widen
+
+pytestmark = pytest.mark.gpu
+
+RITZ_RTOL = 1e-4
+ANGLE_TOL = 1e-3
+EMB_TOL = 1e-4
+
+
+@pytest.fixture(scope="module")
+def sls():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_19368_gb300 as m
+    m.lib()
+    return m
+
+
+def _workload_inputs(name, N=None, d=None, D=None):
+    w = WL.WORKLOADS[name]
+    if N is not None or d is not None or D is not None:
+        w = WL.scaled(w, N=N or w.N, d=d or w.d, D=D or w.D)
+    p = WL.make_prompt(w)
+    prm = WL.params_for(w)
+    return w, p, prm
+
+
+# ---------------------------------------------------------------------------
+# feature map (Sec. 3.2)
+# ---------------------------------------------------------------------------
+
+
+@pytest.mark.parametrize("name,N,D", [("tiny", 512, 256), ("mistral7b", 1000, 1024),
+                                      ("qwen7b", 777, 2048)])
+def test_feature_map_matches_oracle(sls, name, N, D):
+    w, p, prm = _workload_inputs(name, N=N, D=D)
+    X64 = p.x_f64()
+    W64 = prm.w_f64()
+    phi = sls.feature_map(to_torch_x(p.X, w.dtype), to_torch_x(prm.W, w.dtype),
+                          torch.from_numpy(prm.b).cuda())
+    got = phi.cpu().numpy().astype(np.float64)
+    want = O.rff_features(X64, W64, prm.b)
+    tol = feature_tolerance(X64, W64, prm.b.astype(np.float64))
+    err = np.abs(got - want)
+    assert np.all(err <= tol), float(np.max(err / tol))
+
+
+def test_feature_map_ragged_and_empty(sls):
+    g = np.random.default_rng(0)
+    for N, d, D in [(1, 8, 4), (129, 40, 68), (300, 8, 260)]:
+        X = g.standard_normal((N, d)).astype(np.float32) / math.sqrt(d)
+        W = (g.standard_normal((D, d)) * d ** -0.25).astype(np.float32)
+        b = (g.random(D) * 2 * math.pi).astype(np.float32)
+        phi = sls.feature_map(torch.from_numpy(X).cuda(), torch.from_numpy(W).cuda(),
+                              torch.from_numpy(b).cuda()).cpu().numpy()
+        want = O.rff_features(X, W, b)
+        tol = feature_tolerance(X.astype(np.float64), W.astype(np.float64), b.astype(np.float64))
+        assert np.all(np.abs(phi - want) <= tol)
+    out = sls.feature_map(torch.zeros((0, 8), device="cuda"), torch.zeros((4, 8), device="cuda"),
+                          torch.zeros(4, device="cuda"))
+    assert out.shape == (0, 4)
+
+
+# ---------------------------------------------------------------------------
+# Lanczos + Ritz pairs (Algorithm 2, Algorithm 1)
+# ---------------------------------------------------------------------------
+
+
+def _lanczos_case(sls, phi32, q1, r):
+    theta, U, r_eff, alpha, beta = sls.lanczos_topr(torch.from_numpy(phi32).cuda(),
+                                                    torch.from_numpy(q1).cuda(), r)
+    torch.cuda.synchronize()
+    a, b_, Q, k = O.lanczos(phi32.astype(np.float64), q1, r)
+    th_o, S_o, U_o = O.ritz_pairs(a, b_, Q)
+    k_gpu = int(r_eff.item())
+    assert k_gpu == k
+    th = theta.cpu().numpy()[:k]
+    rel = np.abs(th - th_o) / np.abs(th_o)
+    assert np.all(rel <= RITZ_RTOL), float(rel.max())
+    Ug = U.cpu().numpy()[:, :k]
+    assert max_subspace_angle(Ug, U_o) <= ANGLE_TOL
+    assert np.all(U.cpu().numpy()[:, k:] == 0.0)
+    return th, th_o, Ug, U_o, alpha.cpu().numpy()[:k], a
+
+
+@pytest.mark.parametrize("name,N,D,r", [("tiny", 500, 256, 16), ("mistral7b", 8180, 1024, 32)])
+def test_lanczos_matches_oracle(sls, name, N, D, r):
+    w, p, prm = _workload_inputs(name, N=N, D=D)
+    phi32 = oracle_phi32(p.x_f64(), prm.w_f64(), prm.b)
+    th, th_o, Ug, U_o, al, al_o = _lanczos_case(sls, phi32, prm.q1[:N], r)
+    assert np.allclose(al, al_o, rtol=1e-9, atol=1e-12 * abs(al_o).max())
+    # individual Ritz vectors agree (up to the sign convention, which both
+    # sides fix) where the Ritz value is well separated
+    gaps = np.minimum(np.abs(np.diff(np.r_[np.inf, th_o])), np.abs(np.diff(np.r_[th_o, -np.inf])))
+    for j in range(len(th_o)):
+        if gaps[j] > 1e-3 * th_o[0]:
+            cosv = float(Ug[:, j] @ U_o[:, j] / np.linalg.norm(Ug[:, j]) / np.linalg.norm(U_o[:, j]))
+            assert cosv > 1 - 1e-6, (j, cosv)
+
+
+def test_lanczos_breakdown_low_rank(sls):
+    w, p, prm = _workload_inputs("tiny", N=64, D=64)
+    phi = oracle_phi32(p.x_f64()[:5], prm.w_f64()[:64], prm.b[:64])
+    g = np.random.default_rng(1)
+    phi32 = phi[g.integers(0, 5, size=300)]
+    _lanczos_case(sls, phi32, g.standard_normal(300), 16)
+
+
+def test_lanczos_tiny_sizes(sls):
+    g = np.random.default_rng(2)
+    for N, D, r in [(1, 4, 4), (3, 8, 8), (40, 12, 16), (257, 20, 7)]:
+        X = g.standard_normal((N, 6)) / math.sqrt(6)
+        W = g.standard_normal((D, 6)) * 6 ** -0.25
+        b = g.random(D) * 2 * math.pi
+        phi32 = O.rff_features(X, W, b).astype(np.float32)
+        _lanczos_case(sls, phi32, g.standard_normal(N), r)
+
+
+# ---------------------------------------------------------------------------
+# SimHash (Sec. 3.3) -- bit-exact given the oracle's U
+# ---------------------------------------------------------------------------
+
+
+def test_simhash_bit_exact_on_oracle_ritz_vectors(sls):
+    w, p, prm = _workload_inputs("tiny")
+    X = p.x_f64()[:500]
+    phi = O.rff_features(X, prm.w_f64(), prm.b)
+    a, b_, Q, k = O.lanczos(phi, prm.q1[:500], w.r)
+    _, _, U = O.ritz_pairs(a, b_, Q)
+    U32 = U.astype(np.float32)
+    want = O.simhash(U32, prm.R[:w.bits, :k])
+    got = sls.simhash(torch.from_numpy(U32).cuda(), torch.from_numpy(prm.R).cuda(), w.bits)
+    assert np.array_equal(got.cpu().numpy().view(np.uint32), want)
+
+
+@pytest.mark.parametrize("bits,k", [(1, 3), (12, 32), (32, 64), (16, 5)])
+def test_simhash_bit_exact_adversarial(sls, bits, k):
+    g = np.random.default_rng(bits * 100 + k)
+    N = 4099
+    U = g.standard_normal((N, k)).astype(np.float32)
+    # rows with tiny dot products, exact zeros and negative zeros
+    U[:50] *= 1e-30
+    U[50:60] = 0.0
+    U[60:70] = -0.0
+    R = g.standard_normal((bits, k)).astype(np.float32)
+    R[0, :] = np.float32(1e-3) * R[0, :]
+    want = O.simhash(U, R)
+    got = sls.simhash(torch.from_numpy(U).cuda(), torch.from_numpy(R).cuda(), bits)
+    assert np.array_equal(got.cpu().numpy().view(np.uint32), want)
+    # k taken from a device scalar (r_eff): columns past it are ignored
+    kd = torch.tensor([max(1, k - 2)], dtype=torch.int32, device="cuda")
+    got2 = sls.simhash(torch.from_numpy(U).cuda(), torch.from_numpy(R).cuda(), bits, k_dev=kd)
+    want2 = O.simhash(U[:, :max(1, k - 2)], R)
+    assert np.array_equal(got2.cpu().numpy().view(np.uint32), want2)
+
+
+# ---------------------------------------------------------------------------
+# clusters, adjustment, positions and macro-tokens (Sec. 3.3-3.4)
+# ---------------------------------------------------------------------------
+
+
+def _oracle_aggregate(X64, codes, M, scheme, renorm):
+    clusters = O.bucket(codes)
+    groups = O.adjust_groups(clusters, M)
+    order = O.order_groups(groups, scheme)
+    Xt = O.aggregate_groups(X64, [groups[i] for i in order], renorm)
+    pos = np.array([O.group_position(groups[i], scheme) for i in order])
+    t2m = np.empty(len(codes), dtype=np.int64)
+    for k, i in enumerate(order):
+        t2m[groups[i]] = k
+    return Xt, pos, t2m, len(clusters)
+
+
+@pytest.mark.parametrize("scheme", [O.POS_MAX, O.POS_MEDIAN, O.POS_MEAN])
+@pytest.mark.parametrize("case", ["merge", "split", "equal"])
+def test_aggregate_bit_exact_maps(sls, scheme, case):
+    g = np.random.default_rng(7 + scheme)
+    N, d = 3001, 64
+    X = (g.standard_normal((N, d)) / 8).astype(np.float32)
+    nb = {"merge": 900, "split": 40, "equal": 300}[case]
+    codes = g.integers(0, nb, size=N).astype(np.uint32) * np.uint32(2654435761 % 2 ** 32 // 7)
+    C = len(set(codes.tolist()))
+    M = {"merge": max(1, C // 3), "split": min(N, C * 7 + 3), "equal": C}[case]
+    Xt_o, pos_o, t2m_o, C_o = _oracle_aggregate(X.astype(np.float64), codes, M, scheme, True)
+    Xt, pos, t2m = sls.aggregate(torch.from_numpy(X).cuda(),
+                                 torch.from_numpy(codes.view(np.int32)).cuda(), M, scheme, True)
+    assert np.array_equal(t2m.cpu().numpy(), t2m_o)
+    assert np.array_equal(pos.cpu().numpy(), pos_o)
+    assert np.max(np.abs(Xt.cpu().numpy() - Xt_o)) <= EMB_TOL
+
+
+def test_aggregate_bf16_large_groups(sls):
+    """bf16 embeddings, duplicated tokens (one large cluster), renorm off and on."""
+    w, p, prm = _workload_inputs("mistral7b", N=6000, d=512)
+    X64 = p.x_f64()
+    g = np.random.default_rng(3)
+    codes = (p.ids % 700).astype(np.uint32)
+    codes[g.random(6000) < 0.3] = 5  # a cluster holding ~30% of the tokens
+    for renorm, M in [(True, 375), (False, 375), (True, 1500)]:
+        Xt_o, pos_o, t2m_o, _ = _oracle_aggregate(X64, codes, M, O.POS_MAX, renorm)
+        Xt, pos, t2m = sls.aggregate(to_torch_x(p.X, "bf16"),
+                                     torch.from_numpy(codes.view(np.int32)).cuda(), M,
+                                     O.POS_MAX, renorm)
+        assert np.array_equal(t2m.cpu().numpy(), t2m_o)
+        assert np.array_equal(pos.cpu().numpy(), pos_o)
+        assert np.max(np.abs(Xt.cpu().numpy() - Xt_o)) <= EMB_TOL
+
+
+def test_aggregate_edge_cases(sls):
+    g = np.random.default_rng(4)
+    X = (g.standard_normal((17, 8)) / 3).astype(np.float32)
+    for codes, M in [(np.zeros(17, np.uint32), 1), (np.zeros(17, np.uint32), 17),
+                     (np.arange(17, dtype=np.uint32), 17), (np.arange(17, dtype=np.uint32), 1),
+                     (np.full(17, 0xFFFFFFFF, np.uint32), 5)]:
+        Xt_o, pos_o, t2m_o, _ = _oracle_aggregate(X.astype(np.float64), codes, M, O.POS_MAX, True)
+        Xt, pos, t2m = sls.aggregate(torch.from_numpy(X).cuda(),
+                                     torch.from_numpy(codes.view(np.int32)).cuda(), M)
+        assert np.array_equal(t2m.cpu().numpy(), t2m_o)
+        assert np.array_equal(pos.cpu().numpy(), pos_o)
+        assert np.max(np.abs(Xt.cpu().numpy() - Xt_o)) <= EMB_TOL
+
+
+# ---------------------------------------------------------------------------
+# whole pass (Algorithm 1, backends of Sec. 3.5 and 3.6)
+# ---------------------------------------------------------------------------
+
+
+def _check_pass(sls, X64, Xt, pos, t2m, M, pf, pl, scheme=O.POS_MAX, renorm=True):
+    """Invariants of the output, and the macro embeddings / positions the
+    oracle computes from the GPU's own token map."""
+    N = X64.shape[0]
+    t2m = t2m.astype(np.int64)
+    assert t2m.min() >= 0 and t2m.max() == M - 1
+    assert np.all(np.bincount(t2m, minlength=M) >= 1)
+    for i in range(pf):
+        assert t2m[i] == i and pos[i] == i
+    for i in range(pl):
+        assert t2m[N - pl + i] == M - pl + i and pos[M - pl + i] == N - pl + i
+    groups = [np.nonzero(t2m == m)[0] for m in range(M)]
+    Xt_o = O.aggregate_groups(X64, groups, renorm)
+    assert np.max(np.abs(Xt - Xt_o)) <= EMB_TOL
+    pos_o = np.array([O.group_position(gm, scheme) for gm in groups])
+    assert np.array_equal(pos, pos_o)
+    if scheme == O.POS_MAX:
+        assert np.all(np.diff(pos) > 0)
+
+
+def test_compress_global_tiny(sls):
+    w, p, prm = _workload_inputs("tiny")
+    cfg = sls.Config.make(rho=w.rho, D=w.D, r=w.r, bits=w.bits, preserve_last=12)
+    X = to_torch_x(p.X, w.dtype)
+    Xt, pos, t2m, r_eff, route = sls.compress(
+        X, cfg, to_torch_x(prm.W, w.dtype), torch.from_numpy(prm.b).cuda(),
+        torch.from_numpy(prm.R).cuda(), torch.from_numpy(prm.q1).cuda())
+    M = sls.output_count(cfg, w.N)
+    assert M == O.target_count(w.N - 12, w.rho) + 12
+    _check_pass(sls, p.x_f64(), Xt.cpu().numpy(), pos.cpu().numpy(), t2m.cpu().numpy(), M, 0, 12)
+    assert int(r_eff[0].item()) == w.r
+    # the oracle's own run: same cluster-count regime (diagnostic agreement)
+    ocfg = O.CompressConfig(rho=w.rho, D=w.D, r=w.r, bits=w.bits)
+    res = O.compress_global(p.x_f64(), prm.w_f64(), prm.b, prm.R, prm.q1, ocfg)
+    assert res.Xt.shape[0] == M
+
+
+@pytest.mark.parametrize("scheme,mode,pf,pl", [(O.POS_MEDIAN, 0, 3, 5), (O.POS_MEAN, 0, 0, 0),
+                                               (O.POS_MAX, 1, 2, 12)])
+def test_compress_options(sls, scheme, mode, pf, pl):
+    w, p, prm = _workload_inputs("tiny")
+    cfg = sls.Config.make(rho=3.0, D=64, r=8, bits=6, preserve_first=pf, preserve_last=pl,
+                          pos_scheme=scheme, pos_mode=mode)
+    X = to_torch_x(p.X, w.dtype)
+    Xt, pos, t2m, _, _ = sls.compress(X, cfg, to_torch_x(prm.W[:64], w.dtype),
+                                      torch.from_numpy(prm.b[:64]).cuda(),
+                                      torch.from_numpy(prm.R).cuda(),
+                                      torch.from_numpy(prm.q1).cuda())
+    M = sls.output_count(cfg, w.N)
+    t2m = t2m.cpu().numpy()
+    pos = pos.cpu().numpy()
+    if mode == 1:
+        assert np.array_equal(pos, np.arange(M))
+    else:
+        _check_pass(sls, p.x_f64(), Xt.cpu().numpy(), pos, t2m, M, pf, pl, scheme)
+
+
+def test_compress_identity_and_degenerate(sls):
+    w, p, prm = _workload_inputs("tiny")
+    X = to_torch_x(p.X, w.dtype)
+    for rho in (1.0, 0.5):
+        cfg = sls.Config.make(rho=rho)
+        Xt, pos, t2m, _, _ = sls.compress(X, cfg)
+        assert torch.equal(Xt, X.float())
+        assert np.array_equal(pos.cpu().numpy(), np.arange(w.N))
+        assert np.array_equal(t2m.cpu().numpy(), np.arange(w.N))
+    cfg = sls.Config.make(rho=4.0, preserve_last=w.N + 3)
+    Xt, pos, t2m, _, _ = sls.compress(X, cfg)
+    assert torch.equal(Xt, X.float())
+    # all tokens identical: one cluster, split into M pieces; breakdown after 1 step
+    Xs = X[:1].repeat(100, 1).contiguous()
+    cfg = sls.Config.make(rho=4.0, D=64, r=8, bits=4, preserve_last=0)
+    Xt, pos, t2m, r_eff, _ = sls.compress(Xs, cfg, to_torch_x(prm.W[:64], w.dtype),
+                                          torch.from_numpy(prm.b[:64]).cuda(),
+                                          torch.from_numpy(prm.R).cuda(),
+                                          torch.from_numpy(prm.q1).cuda())
+    assert int(r_eff[0].item()) == 1
+    _check_pass(sls, Xs.double().cpu().numpy(), Xt.cpu().numpy(), pos.cpu().numpy(),
+                t2m.cpu().numpy(), 25, 0, 0)
+
+
+def test_compress_chunk_backend(sls):
+    w, p, prm = _workload_inputs("tiny")
+    X = to_torch_x(p.X, w.dtype)
+    cfg = sls.Config.make(backend=sls.BACKEND_CHUNK, rho=4.0, preserve_last=12)
+    Xt, pos, t2m, _, _ = sls.compress(X, cfg)
+    res = O.compress_chunk(p.x_f64(), O.CompressConfig(rho=4.0, preserve_last=12))
+    assert np.array_equal(t2m.cpu().numpy(), res.tok2macro)
+    assert np.array_equal(pos.cpu().numpy(), res.pos)
+    assert np.max(np.abs(Xt.cpu().numpy() - res.Xt)) <= EMB_TOL
+
+
+def test_compress_adaptive_small_batch(sls):
+    """Adaptive router on a batch of 3 prompts (windows of 96): route flags,
+    budgets and chunk windows against the oracle; spectral windows by their
+    invariants."""
+    w = WL.scaled(WL.WORKLOADS["adaptive"], N=700, d=64, batch=3)
+    prompts = [WL.make_prompt(w, index=i, dup_frac=WL.adaptive_dup_frac(i, 3)) for i in range(3)]
+    prm = WL.make_params(64, 64, 8, 32, 3 * 700, "bf16")
+    Xb = np.stack([pp.X for pp in prompts])
+    X = to_torch_x(Xb, "bf16")
+    for rho in (2.0, 4.0, 16.0):
+        cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=64, r=8, window=96,
+                              preserve_last=12)
+        Xt, pos, t2m, r_eff, route = sls.compress(X, cfg, to_torch_x(prm.W, "bf16"),
+                                                  torch.from_numpy(prm.b).cuda(),
+                                                  torch.from_numpy(prm.R).cuda(),
+                                                  torch.from_numpy(prm.q1).cuda())
+        M = sls.output_count(cfg, 700)
+        nw = len(O.window_bounds(688, 96))
+        route = route.cpu().numpy()[:3 * nw].reshape(3, nw)
+        for i, pp in enumerate(prompts):
+            ocfg = O.CompressConfig(rho=rho, D=64, r=8, window=96, preserve_last=12)
+            res = O.compress_adaptive(pp.x_f64(), prm.w_f64(), prm.b, prm.R,
+                                      prm.q1[i * 700:(i + 1) * 700], ocfg)
+            tau = O.tau_schedule(rho)
+            for k, (sp, sc) in enumerate(zip(res.info["spectral"], res.info["scores"])):
+                if rho >= 16 or abs(sc - tau) > 1e-5:
+                    assert route[i, k] == int(sp), (rho, i, k, sc)
+            _check_pass(sls, pp.x_f64(), Xt[i].cpu().numpy(), pos[i].cpu().numpy(),
+                        t2m[i].cpu().numpy(), M, 0, 12)
+            # every macro-token lies inside one window
+            t = t2m[i].cpu().numpy()
+            for m in range(M - 12):
+                mem = np.nonzero(t == m)[0]
+                assert mem.min() // 96 == mem.max() // 96
+            # chunk windows match the oracle exactly
+            bounds = O.window_bounds(688, 96)
+            for k, (s, e) in enumerate(bounds):
+                if not route[i, k]:
+                    assert np.array_equal(t[s:e], res.tok2macro[s:e])
