@@ -229,6 +229,23 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
                  void* stream);
 
 /*
+ * Optional per-phase timing of sls_compress.  `events` is a host array of
+ * 2 * SLS_NUM_PHASES cudaEvent_t handles (passed as void*) owned by the
+ * caller; while set, every sls_compress call records events[2p] on its
+ * stream before phase p and events[2p+1] after it.  Phases, in launch order:
+ * 0 setup (problem table, token norms, router), 1 feature map, 2 Lanczos,
+ * 3 Eigh(T) and Ritz vectors, 4 SimHash, 5 clusters/adjust/order,
+ * 6 macro-token aggregation.  count = 0 (or events = NULL) switches timing
+ * off.  Process-wide setting, not thread-safe.  Errors: INVALID_ARG if
+ * count is neither 0 nor 2 * SLS_NUM_PHASES.
+ */
+#define SLS_NUM_PHASES 7
+int sls_set_phase_events(void* const* events, int count);
+
+/* Total number of kernels this library has launched in the process. */
+int64_t sls_launch_count(void);
+
+/*
  * Reads (synchronously, on `stream`) the device status word of a workspace
  * used by sls_lanczos_topr or sls_compress: SLS_OK, or SLS_ERR_TIMEOUT when
  * a device-side wait gave up.  Clears the word.

@@ -22,7 +22,8 @@ __all__ = [
     "MODE_REPRESENTATIVE", "MODE_COMPACT", "BACKEND_GLOBAL", "BACKEND_ADAPTIVE",
     "BACKEND_CHUNK", "Config", "SLSError", "lib", "lib_path", "feature_map",
     "lanczos_topr", "simhash", "aggregate", "compress", "output_count",
-    "compress_workspace_size", "workspace_status", "EXPORTED",
+    "compress_workspace_size", "workspace_status", "EXPORTED", "PHASES",
+    "set_phase_events", "launch_count", "Workspace",
 ]
 
 SLS_OK = 0
@@ -94,7 +95,11 @@ EXPORTED = {
     "sls_compress": (_i32, [ctypes.POINTER(Config), _vp, _i32, _i64, _i64, _i32, _i64,
                             ctypes.POINTER(_Params), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "sls_workspace_status": (_i32, [_vp, _vp]),
+    "sls_set_phase_events": (_i32, [ctypes.POINTER(ctypes.c_void_p), _i32]),
+    "sls_launch_count": (_i64, []),
 }
+
+PHASES = ("setup", "features", "lanczos", "ritz", "simhash", "segment", "aggregate")
 
 _lib = None
 
@@ -275,8 +280,9 @@ def compress(X: torch.Tensor, cfg: Config, W: Optional[torch.Tensor] = None,
         workspace = Workspace(cfg, B, N, d, dev)
     params = None
     keep = []
-    if cfg.backend != BACKEND_CHUNK and cfg.rho > 1.0:
-        assert W is not None and b is not None and R is not None and q1 is not None
+    if cfg.backend != BACKEND_CHUNK and M != N:
+        if W is None or b is None or R is None or q1 is None:
+            raise ValueError("the spectral backends need W, b, R and q1")
         Wc = W.contiguous()
         bc = b.float().contiguous()
         Rc = R.float().contiguous()
@@ -294,6 +300,21 @@ def compress(X: torch.Tensor, cfg: Config, W: Optional[torch.Tensor] = None,
     if not batched:
         return Xt[0], pos[0], t2m[0], r_eff, route
     return Xt, pos, t2m, r_eff, route
+
+
+def set_phase_events(events) -> None:
+    """Record torch.cuda.Event pairs around the phases of compress() (see
+    sls_set_phase_events); None switches timing off."""
+    if events is None:
+        _check("sls_set_phase_events", lib().sls_set_phase_events(None, 0))
+        return
+    arr = (ctypes.c_void_p * len(events))(*[e.cuda_event for e in events])
+    _check("sls_set_phase_events", lib().sls_set_phase_events(arr, len(events)))
+
+
+def launch_count() -> int:
+    """Kernels launched by libsls in this process so far."""
+    return int(lib().sls_launch_count())
 
 
 def workspace_status(workspace: Workspace) -> int:

@@ -10,9 +10,23 @@
 #include "kernels.cuh"
 #include "segment.cuh"
 
+#include <atomic>
+
 using namespace sls;
 
+namespace sls {
+static std::atomic<long long> g_launches{0};
+void count_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+}  // namespace sls
+
 namespace {
+
+void* g_phase_events[2 * SLS_NUM_PHASES];
+bool g_phase_on = false;
+
+inline void phase_mark(int phase, int end, cudaStream_t s) {
+  if (g_phase_on) cudaEventRecord((cudaEvent_t)g_phase_events[2 * phase + end], s);
+}
 
 // ---------------------------------------------------------------------------
 // workspace carving
@@ -609,6 +623,7 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   }
   SLS_CUDA_TRY(cudaMemsetAsync(W.status, 0, 256, s));
   const int nprob = (int)P.nprob;
+  phase_mark(0, 0, s);
   // problem table
   {
     int64_t blocks = (P.nprob + 255) / 256;
@@ -638,6 +653,8 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
                                           W.spec_list, W.lz_row0, W.lz_n, W.lz_q1off, W.nspec,
                                           route);
   SLS_LAUNCH_CHECK();
+  phase_mark(0, 1, s);
+  phase_mark(1, 0, s);
   if (spectral) {
     // features for every compressible row of every prompt
     for (int64_t b = 0; b < B; ++b) {
@@ -647,6 +664,8 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
                            W.Phi + (size_t)b * P.Nc * cfg->D, stream);
       if (st != SLS_OK) return st;
     }
+    phase_mark(1, 1, s);
+    phase_mark(2, 0, s);
     LanczosBatch bt{};
     bt.Phi = W.Phi;
     bt.D = cfg->D;
@@ -669,8 +688,12 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
     if ((st = launch_lanczos(bt, W.lz_scratch, W.lz_bytes, W.status, P.lz_groups, P.lz_g, s)) !=
         SLS_OK)
       return st;
+    phase_mark(2, 1, s);
+    phase_mark(3, 0, s);
     if ((st = launch_tridiag_eigen(bt, s)) != SLS_OK) return st;
     if ((st = launch_ritz_vectors(bt, W.U, s)) != SLS_OK) return st;
+    phase_mark(3, 1, s);
+    phase_mark(4, 0, s);
     if ((st = launch_simhash_problems(W.probs, W.spec_list, W.nspec, nprob, P.nmax, W.r_eff, W.U,
                                       cfg->r, params->R, params->R_ld, P.bits_max, W.codes, s)) !=
         SLS_OK)
@@ -679,7 +702,14 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
       finish_reff_kernel<<<(nprob + 255) / 256, 256, 0, s>>>(W.probs, nprob, W.r_eff, r_eff);
       SLS_LAUNCH_CHECK();
     }
+    phase_mark(4, 1, s);
+  } else {
+    for (int ph = 1; ph <= 4; ++ph) {
+      if (ph > 1) phase_mark(ph, 0, s);
+      phase_mark(ph, 1, s);
+    }
   }
+  phase_mark(5, 0, s);
   if ((st = launch_segment(W.probs, nprob, W.codes, cfg->pos_scheme, cfg->pos_mode, W.seg_scratch,
                            P.seg_slots, P.nmax, P.mmax, W.perm, W.mstart, W.mlen, pos, tok2macro,
                            s)) != SLS_OK)
@@ -687,10 +717,30 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   if ((st = launch_preserved(B, N, P.M, (int)P.pf, (int)P.pl, cfg->pos_mode, W.perm, W.mstart,
                              W.mlen, pos, tok2macro, s)) != SLS_OK)
     return st;
-  return launch_aggregate(X, x_dtype, d, ldx, W.norms, W.perm, W.mstart, W.mlen, B * P.M, B * N,
-                          cfg->renorm, Xt, W.it_start, W.pt_start, W.items, W.counts, W.part,
-                          W.part_eta, s);
+  phase_mark(5, 1, s);
+  phase_mark(6, 0, s);
+  st = launch_aggregate(X, x_dtype, d, ldx, W.norms, W.perm, W.mstart, W.mlen, B * P.M, B * N,
+                        cfg->renorm, Xt, W.it_start, W.pt_start, W.items, W.counts, W.part,
+                        W.part_eta, s);
+  phase_mark(6, 1, s);
+  return st;
 }
+
+int sls_set_phase_events(void* const* events, int count) {
+  if (count == 0 || events == nullptr) {
+    g_phase_on = false;
+    return SLS_OK;
+  }
+  if (count != 2 * SLS_NUM_PHASES) return SLS_ERR_INVALID_ARG;
+  for (int i = 0; i < count; ++i) {
+    if (!events[i]) return SLS_ERR_INVALID_ARG;
+    g_phase_events[i] = events[i];
+  }
+  g_phase_on = true;
+  return SLS_OK;
+}
+
+int64_t sls_launch_count(void) { return (int64_t)g_launches.load(); }
 
 int sls_workspace_status(void* workspace, void* stream) {
   if (!workspace) return SLS_ERR_INVALID_ARG;

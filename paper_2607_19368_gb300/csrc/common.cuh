@@ -230,8 +230,13 @@ static inline size_t sls_align256(size_t x) { return (x + 255) & ~(size_t)255; }
     if (e_ != cudaSuccess) return SLS_ERR_CUDA;     \
   } while (0)
 
+namespace sls {
+void count_launch(int n);  // library-wide kernel launch counter (api.cu)
+}
+
 #define SLS_LAUNCH_CHECK()                                   \
   do {                                                       \
     cudaError_t e_ = cudaGetLastError();                     \
     if (e_ != cudaSuccess) return SLS_ERR_CUDA;              \
+    sls::count_launch(1);                                    \
   } while (0)

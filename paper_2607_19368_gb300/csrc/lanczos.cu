@@ -704,6 +704,7 @@ int launch_lanczos_t(const LanczosBatch& bt, void* scratch, size_t gstride, int 
                   (void*)&rows_cap, (void*)&status};
   SLS_CUDA_TRY(cudaLaunchCooperativeKernel((const void*)fn, dim3(groups * g), dim3(LZ_THREADS),
                                            args, smem, stream));
+  count_launch(1);
   return SLS_OK;
 }
 

@@ -19,6 +19,7 @@ pytestmark = pytest.mark.gpu
 RITZ_RTOL = 1e-4
 ANGLE_TOL = 1e-3
 EMB_TOL = 1e-4
+ZERO_FLOOR = 1e-12
 
 
 @pytest.fixture(scope="module")
@@ -89,8 +90,12 @@ def _lanczos_case(sls, phi32, q1, r):
     k_gpu = int(r_eff.item())
     assert k_gpu == k
     th = theta.cpu().numpy()[:k]
-    rel = np.abs(th - th_o) / np.abs(th_o)
-    assert np.all(rel <= RITZ_RTOL), float(rel.max())
+    # Ritz values at the operator's noise floor (|theta| <= 1e-12 theta_1, the
+    # null space reached at a breakdown) are zero in exact arithmetic; they are
+    # compared against that absolute floor instead of relatively.
+    floor = ZERO_FLOOR * abs(th_o[0])
+    err = np.abs(th - th_o)
+    assert np.all(err <= RITZ_RTOL * np.abs(th_o) + floor), float(np.max(err / (np.abs(th_o) + floor)))
     Ug = U.cpu().numpy()[:, :k]
     assert max_subspace_angle(Ug, U_o) <= ANGLE_TOL
     assert np.all(U.cpu().numpy()[:, k:] == 0.0)
@@ -308,14 +313,15 @@ def test_compress_identity_and_degenerate(sls):
     cfg = sls.Config.make(rho=4.0, preserve_last=w.N + 3)
     Xt, pos, t2m, _, _ = sls.compress(X, cfg)
     assert torch.equal(Xt, X.float())
-    # all tokens identical: one cluster, split into M pieces; breakdown after 1 step
+    # all tokens identical: one cluster, split into M pieces.  Phi has rank 1,
+    # so the Krylov space is span{q1, A q1} and Lanczos stops after 2 steps.
     Xs = X[:1].repeat(100, 1).contiguous()
     cfg = sls.Config.make(rho=4.0, D=64, r=8, bits=4, preserve_last=0)
     Xt, pos, t2m, r_eff, _ = sls.compress(Xs, cfg, to_torch_x(prm.W[:64], w.dtype),
                                           torch.from_numpy(prm.b[:64]).cuda(),
                                           torch.from_numpy(prm.R).cuda(),
                                           torch.from_numpy(prm.q1).cuda())
-    assert int(r_eff[0].item()) == 1
+    assert int(r_eff[0].item()) == 2
     _check_pass(sls, Xs.double().cpu().numpy(), Xt.cpu().numpy(), pos.cpu().numpy(),
                 t2m.cpu().numpy(), 25, 0, 0)
 
