@@ -229,6 +229,34 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
                  void* stream);
 
 /*
+ * sls_lanczos_topr without a caller workspace.  The paper has no counterpart
+ * to this entry point: it exists for callers that may not allocate device
+ * memory themselves -- for example a plugin inside a host application whose
+ * memory manager owns every device allocation, or a serving path that forbids
+ * allocation after start-up -- and therefore cannot provide the workspace
+ * that sls_lanczos_topr takes.  Arguments and results are those of
+ * sls_lanczos_topr (the caller still passes Phi, q1 and the output arrays).
+ *
+ * Scratch lives in one statically sized device array of
+ * SLS_NOALLOC_MAX_BYTES inside the library; every GPU that loads the library
+ * holds it until the process exits.  No cudaMalloc, cudaFree or allocating
+ * library routine is called.  The first call on a device (with that device
+ * current) looks up the array's device address once; make that first call
+ * before any stream capture.  All calls share the array and it keeps the
+ * previous call's contents (what must start at zero is cleared by each
+ * call), so calls that overlap on the GPU -- on different streams, or from
+ * different host threads -- race and must be serialised by the caller.
+ * *r_eff is set to -1 when the call is enqueued and stays -1 if a device-side
+ * wait gave up.  Errors: those of sls_lanczos_topr, and SLS_ERR_WORKSPACE
+ * when sls_lanczos_workspace_size(N, D, r) exceeds SLS_NOALLOC_MAX_BYTES.
+ */
+#define SLS_NOALLOC_MAX_BYTES (32u << 20)
+int sls_lanczos_topr_noalloc(const float* Phi, int64_t N, int D, int r,
+                             const double* q1, double tol, double* theta,
+                             float* U, int32_t* r_eff, double* alpha,
+                             double* beta, void* stream);
+
+/*
  * Optional per-phase timing of sls_compress.  `events` is a host array of
  * 2 * SLS_NUM_PHASES cudaEvent_t handles (passed as void*) owned by the
  * caller; while set, every sls_compress call records events[2p] on its

@@ -95,6 +95,8 @@ EXPORTED = {
     "sls_compress": (_i32, [ctypes.POINTER(Config), _vp, _i32, _i64, _i64, _i32, _i64,
                             ctypes.POINTER(_Params), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "sls_workspace_status": (_i32, [_vp, _vp]),
+    "sls_lanczos_topr_noalloc": (_i32, [_vp, _i64, _i32, _i32, _vp, _d, _vp, _vp, _vp, _vp,
+                                        _vp, _vp]),
     "sls_set_phase_events": (_i32, [ctypes.POINTER(ctypes.c_void_p), _i32]),
     "sls_launch_count": (_i64, []),
 }
