@@ -145,6 +145,152 @@ SLS_DEV float warp_sum_f(float v) {
 }
 
 // ---------------------------------------------------------------------------
+// packed float32 pairs (sm_100-family f32x2 instructions): one instruction
+// performs the same IEEE round-to-nearest operation on both halves.
+// ---------------------------------------------------------------------------
+
+typedef unsigned long long f32x2_t;
+
+SLS_DEV f32x2_t pk2(float a, float b) {
+  f32x2_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+SLS_DEV void upk2(f32x2_t v, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+SLS_DEV f32x2_t add2(f32x2_t a, f32x2_t b) {
+  f32x2_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+SLS_DEV f32x2_t sub2(f32x2_t a, f32x2_t b) {
+  f32x2_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+SLS_DEV f32x2_t mul2(f32x2_t a, f32x2_t b) {
+  f32x2_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+SLS_DEV f32x2_t fma2(f32x2_t a, f32x2_t b, f32x2_t c) {
+  f32x2_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+SLS_DEV f32x2_t neg2(f32x2_t a) { return a ^ 0x8000000080000000ull; }
+
+// Dot2 step on two lanes at once: (sh, sl) += x * (yh + yl), with the
+// negated high part nyh = -yh supplied so that TwoProduct needs no sign flip.
+SLS_DEV void dot2_acc2n(f32x2_t& sh, f32x2_t& sl, f32x2_t x, f32x2_t yh, f32x2_t nyh,
+                        f32x2_t yl) {
+  const f32x2_t np = mul2(x, nyh);      // -p, p = fl(x * yh)
+  f32x2_t pe = fma2(x, yh, np);          // x * yh - p, exact
+  pe = fma2(x, yl, pe);
+  const f32x2_t s = sub2(sh, np);        // sh + p
+  const f32x2_t bb = sub2(s, sh);
+  const f32x2_t e = sub2(sub2(sh, sub2(s, bb)), add2(np, bb));  // TwoSum error
+  sh = s;
+  sl = add2(sl, add2(e, pe));
+}
+
+// Same step when only yh is at hand (the sign flip is an integer xor).
+SLS_DEV void dot2_acc2(f32x2_t& sh, f32x2_t& sl, f32x2_t x, f32x2_t yh, f32x2_t yl) {
+  const f32x2_t p = mul2(x, yh);
+  const f32x2_t np = neg2(p);
+  f32x2_t pe = fma2(x, yh, np);
+  pe = fma2(x, yl, pe);
+  const f32x2_t s = add2(sh, p);
+  const f32x2_t bb = sub2(s, sh);
+  const f32x2_t e = add2(sub2(sh, sub2(s, bb)), sub2(p, bb));
+  sh = s;
+  sl = add2(sl, add2(e, pe));
+}
+
+// ---------------------------------------------------------------------------
+// shared-memory barriers, bulk copies and named barriers
+// ---------------------------------------------------------------------------
+
+SLS_DEV uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+SLS_DEV void mbar_init(uint64_t* bar, unsigned count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+
+SLS_DEV void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+SLS_DEV void mbar_arrive(uint64_t* bar, unsigned count = 1) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(count)
+               : "memory");
+}
+
+SLS_DEV void mbar_expect_tx(uint64_t* bar, unsigned bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+SLS_DEV bool mbar_try_wait(uint64_t* bar, unsigned parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the phase with the given parity; false after the limit.
+SLS_DEV bool mbar_wait(uint64_t* bar, unsigned parity) {
+  for (unsigned it = 0; it < (1u << 26); ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (it > 64) __nanosleep(32);
+  }
+  return false;
+}
+
+// One-dimensional bulk copy global -> shared, completion counted on `bar`.
+SLS_DEV void bulk_g2s(void* dst, const void* src, unsigned bytes, uint64_t* bar,
+                      uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint "
+      "[%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+SLS_DEV uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+SLS_DEV uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+SLS_DEV uint64_t l2_policy_normal() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+SLS_DEV void named_sync(unsigned id, unsigned nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// ---------------------------------------------------------------------------
 // memory-model helpers
 // ---------------------------------------------------------------------------
 
@@ -215,6 +361,40 @@ SLS_DEV bool group_sync(const GroupBarrier& bar, unsigned& local_gen, int* statu
     *smem_flag = ok;
   }
   __syncthreads();
+  return *((volatile int*)smem_flag) != 0;
+}
+
+// Same barrier for kernels where only `nthreads` threads (ids 0..nthreads-1,
+// named barrier `bar_id`) take part, e.g. compute warps next to a copy warp.
+SLS_DEV bool group_sync_named(const GroupBarrier& bar, unsigned& local_gen, int* status,
+                              int* smem_flag, unsigned bar_id, unsigned nthreads) {
+  named_sync(bar_id, nthreads);
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    unsigned g = local_gen;
+    __threadfence();
+    unsigned arrived = atom_add_acq_rel_gpu(bar.count, 1u);
+    if (arrived == bar.nblocks - 1) {
+      *bar.count = 0;
+      __threadfence();
+      st_release_gpu(bar.gen, g + 1);
+    } else {
+      unsigned it = 0;
+      while (ld_acquire_gpu(bar.gen) == g) {
+        if (++it > SLS_SPIN_LIMIT) {
+          ok = 0;
+          atomicExch(status, SLS_ERR_TIMEOUT);
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    __threadfence();
+    local_gen = g + 1;
+    if (ok && *((volatile int*)status) == SLS_ERR_TIMEOUT) ok = 0;
+    *smem_flag = ok;
+  }
+  named_sync(bar_id, nthreads);
   return *((volatile int*)smem_flag) != 0;
 }
 

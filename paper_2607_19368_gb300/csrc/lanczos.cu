@@ -38,8 +38,10 @@ namespace sls {
 
 namespace {
 
-constexpr int LZ_THREADS = 256;
-constexpr int LZ_WARPS = LZ_THREADS / 32;
+constexpr int LZ_CW = 8;                  // compute warps
+constexpr int LZ_CT = LZ_CW * 32;         // compute threads
+constexpr int LZ_THREADS = LZ_CT + 32;    // plus one copy warp
+constexpr int LZ_WARPS = LZ_CW;
 
 // Per-group scratch layout (byte offsets), identical on host and device.
 struct LzLayout {
@@ -72,154 +74,235 @@ SLS_DEV dfloat shfl_df(dfloat v, int src) {
   return v;
 }
 
-// Block-wide double-float sum; result valid in every thread.
-SLS_DEV dfloat block_sum_df(dfloat v, float2* tmp /* LZ_WARPS */) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  v = warp_sum_df(v);
-  __syncthreads();
-  if (lane == 0) tmp[warp] = f2(v);
-  __syncthreads();
-  dfloat s = df_make(0.f, 0.f);
-#pragma unroll
-  for (int w = 0; w < LZ_WARPS; ++w) s = df_add(s, dfv(tmp[w]));
-  return s;
+// ---------------------------------------------------------------------------
+// The feature matrix is streamed through a shared-memory ring.  One copy warp
+// issues one-dimensional bulk copies (cp.async.bulk) of consecutive row chunks
+// of the CTA's strip, each completing on the stage's "full" mbarrier; the
+// eight compute warps release a stage on its "empty" mbarrier.  Sweep A walks
+// the strip forward and sweep B backward, so the chunks sweep A touched last
+// are still in L2 when sweep B starts (and vice versa at the next step).  The
+// copy warp runs ahead across the group barriers, so the loads of the next
+// sweep overlap the reductions between sweeps.
+// ---------------------------------------------------------------------------
+
+constexpr unsigned BAR_COMPUTE = 1;  // named barrier: the compute warps
+constexpr int RING_TARGET = 64 * 1024;  // bytes per ring stage (a few rows)
+
+struct RingShape {
+  int cr;            // rows per chunk
+  int S;             // stages
+  unsigned chunk;    // bytes per full chunk
+};
+
+__host__ __device__ inline RingShape ring_shape(int D, size_t budget) {
+  RingShape R;
+  R.cr = RING_TARGET / (4 * D);
+  if (R.cr < 1) R.cr = 1;
+  R.chunk = (unsigned)R.cr * (unsigned)D * 4u;
+  R.S = (int)(budget / R.chunk);
+  if (R.S > 6) R.S = 6;
+  return R;
 }
 
-// Sweep A: w_part[c] = sum over the strip of Phi[i, c] * u_i (Dot2).
-// GPT float4 column groups per thread; P row phases when D/4 < LZ_THREADS.
+struct RingState {
+  uint64_t* full;
+  uint64_t* empty;
+  float* ring;
+  RingShape shp;
+};
+
+// Sweep A over one chunk: acc[c] += Phi[i, c] * u_i for the chunk's rows,
+// column-parallel (GPT float4 groups per thread, P row phases).
 template <int GPT>
-SLS_DEV void sweep_phi_t_u(const float* __restrict__ Phi, int D, int64_t rs, int64_t re,
-                           const float2* __restrict__ us, float2* __restrict__ red,
-                           float2* __restrict__ wpart_row) {
+SLS_DEV void sweepA_chunk(const float* __restrict__ chunk, int nr, int D, int lb,
+                          const float2* __restrict__ us, f32x2_t (&ah)[GPT][2],
+                          f32x2_t (&al)[GPT][2]) {
   const int tid = threadIdx.x;
   const int C4 = D >> 2;
-  const int P = (C4 >= LZ_THREADS) ? 1 : (LZ_THREADS / C4);
-  const int act = (P == 1) ? LZ_THREADS : P * C4;
-  constexpr int UNR = (16 / GPT) < 2 ? 2 : (16 / GPT);
-  if (tid < act) {
-    const int ph = (P == 1) ? 0 : tid / C4;
-    const int cb = (P == 1) ? tid : tid % C4;
-    float ah[GPT][4], al[GPT][4];
-#pragma unroll
-    for (int q = 0; q < GPT; ++q)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) ah[q][c] = al[q][c] = 0.f;
-    const float4* base = reinterpret_cast<const float4*>(Phi);
-    int64_t i = rs + ph;
-    for (; i + (int64_t)(UNR - 1) * P < re; i += (int64_t)UNR * P) {
-      float4 f[UNR][GPT];
-      float2 uu[UNR];
-#pragma unroll
-      for (int t = 0; t < UNR; ++t) {
-        const int64_t row = i + (int64_t)t * P;
-        uu[t] = us[row - rs];
-#pragma unroll
-        for (int q = 0; q < GPT; ++q) {
-          const int cg = cb + q * LZ_THREADS;
-          f[t][q] = (cg < C4) ? __ldg(base + row * C4 + cg) : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-      }
-#pragma unroll
-      for (int t = 0; t < UNR; ++t)
-#pragma unroll
-        for (int q = 0; q < GPT; ++q) {
-          dot2_acc(ah[q][0], al[q][0], f[t][q].x, uu[t].x, uu[t].y);
-          dot2_acc(ah[q][1], al[q][1], f[t][q].y, uu[t].x, uu[t].y);
-          dot2_acc(ah[q][2], al[q][2], f[t][q].z, uu[t].x, uu[t].y);
-          dot2_acc(ah[q][3], al[q][3], f[t][q].w, uu[t].x, uu[t].y);
-        }
-    }
-    for (; i < re; i += P) {
-      const float2 u = us[i - rs];
-#pragma unroll
-      for (int q = 0; q < GPT; ++q) {
-        const int cg = cb + q * LZ_THREADS;
-        if (cg < C4) {
-          const float4 f = __ldg(base + i * C4 + cg);
-          dot2_acc(ah[q][0], al[q][0], f.x, u.x, u.y);
-          dot2_acc(ah[q][1], al[q][1], f.y, u.x, u.y);
-          dot2_acc(ah[q][2], al[q][2], f.z, u.x, u.y);
-          dot2_acc(ah[q][3], al[q][3], f.w, u.x, u.y);
-        }
-      }
-    }
-    float2* dst = (P == 1) ? wpart_row : red + (size_t)ph * D;
+  const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
+  if (P > 1 && tid >= P * C4) return;
+  const int ph = (P == 1) ? 0 : tid / C4;
+  const int cb = (P == 1) ? tid : tid % C4;
+  const float4* c4 = reinterpret_cast<const float4*>(chunk);
+  for (int i = ph; i < nr; i += P) {
+    const float2 u = us[lb + i];
+    const f32x2_t uh = pk2(u.x, u.x), nuh = pk2(-u.x, -u.x), ul = pk2(u.y, u.y);
 #pragma unroll
     for (int q = 0; q < GPT; ++q) {
-      const int cg = cb + q * LZ_THREADS;
+      const int cg = cb + q * LZ_CT;
       if (cg < C4) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          dfloat v = df_norm(ah[q][c], al[q][c]);
-          dst[4 * cg + c] = f2(v);
-        }
+        const float4 f = c4[i * C4 + cg];
+        dot2_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
+        dot2_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
       }
-    }
-  }
-  if (P > 1) {
-    __syncthreads();
-    for (int col = tid; col < D; col += LZ_THREADS) {
-      dfloat s = df_make(0.f, 0.f);
-      for (int ph = 0; ph < P; ++ph) s = df_add(s, dfv(red[(size_t)ph * D + col]));
-      wpart_row[col] = f2(s);
     }
   }
 }
 
-// Row dot product s = Phi[i, :] . w with w in shared memory (double-float);
-// one warp per row, every lane returns the sum.
-SLS_DEV dfloat row_dot_w(const float* __restrict__ Phi, int D, int64_t i,
-                         const float2* __restrict__ wsm) {
+// Row dot product with w from shared memory (layout: per column pair
+// {wh_even, wh_odd, wl_even, wl_odd}); one warp per row, all lanes get it.
+SLS_DEV dfloat row_dot_smem(const float* __restrict__ row, int D,
+                            const float4* __restrict__ wq) {
   const int lane = threadIdx.x & 31;
   const int C4 = D >> 2;
-  const float4* rowp = reinterpret_cast<const float4*>(Phi) + i * C4;
-  const float4* w4 = reinterpret_cast<const float4*>(wsm);  // (h0,l0,h1,l1),(h2,l2,h3,l3)
-  float h[4] = {0.f, 0.f, 0.f, 0.f}, l[4] = {0.f, 0.f, 0.f, 0.f};
-  constexpr int CH = 16;
-  for (int q0 = 0; q0 < C4; q0 += CH * 32) {
-    float4 f[CH];
+  const float4* r4 = reinterpret_cast<const float4*>(row);
+  f32x2_t h01 = 0, l01 = 0, h23 = 0, l23 = 0;
+  for (int cg = lane; cg < C4; cg += 32) {
+    const float4 f = r4[cg];
+    const float4 wa = wq[2 * cg], wb = wq[2 * cg + 1];
+    dot2_acc2(h01, l01, pk2(f.x, f.y), pk2(wa.x, wa.y), pk2(wa.z, wa.w));
+    dot2_acc2(h23, l23, pk2(f.z, f.w), pk2(wb.x, wb.y), pk2(wb.z, wb.w));
+  }
+  float a0, a1, b0, b1, c0, c1, d0, d1;
+  upk2(h01, a0, a1);
+  upk2(l01, b0, b1);
+  upk2(h23, c0, c1);
+  upk2(l23, d0, d1);
+  dfloat s = df_add(df_add(df_make(a0, b0), df_make(a1, b1)),
+                    df_add(df_make(c0, d0), df_make(c1, d1)));
+  return warp_sum_df(s);
+}
+
+SLS_DEV int nprob_of(const LanczosBatch& bt) {
+  int nprob = bt.nprob_max;
+  if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
+  return nprob;
+}
+
+constexpr int KT_MAX = (SLS_MAX_R + 1 + 31) / 32;  // basis columns per lane
+constexpr int RPW = 4;                               // rows per warp in the row passes
+
+// Sum of the per-CTA partial coefficients part[b * (r+1) + k] over the g CTAs
+// of a group, for k <= j, into cs[k].  Every CTA does it redundantly; the
+// loads are spread over all compute threads so they are in flight together.
+SLS_DEV void reduce_coeffs(const float2* __restrict__ part, int g, int r, int j,
+                           float2* __restrict__ cs, float2* __restrict__ tmp) {
+  const int tid = threadIdx.x;
+  const int K = j + 1;
+  int PH = LZ_CT / K;
+  if (PH < 1) PH = 1;
+  if (PH > 8) PH = 8;
+  for (int idx = tid; idx < K * PH; idx += LZ_CT) {
+    const int k = idx % K, ph = idx / K;
+    dfloat s = df_make(0.f, 0.f);
+    int b = ph;
+    for (; b + 7 * PH < g; b += 8 * PH) {
+      float2 v[8];
 #pragma unroll
-    for (int t = 0; t < CH; ++t) {
-      const int cg = q0 + lane + 32 * t;
-      f[t] = (cg < C4) ? __ldg(rowp + cg) : make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int u = 0; u < 8; ++u) v[u] = part[(size_t)(b + u * PH) * (r + 1) + k];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) s = df_add(s, dfv(v[u]));
     }
+    for (; b < g; b += PH) s = df_add(s, dfv(part[(size_t)b * (r + 1) + k]));
+    tmp[ph * K + k] = f2(s);
+  }
+  named_sync(BAR_COMPUTE, LZ_CT);
+  for (int k = tid; k < K; k += LZ_CT) {
+    dfloat s = df_make(0.f, 0.f);
+    for (int ph = 0; ph < PH; ++ph) s = df_add(s, dfv(tmp[ph * K + k]));
+    cs[k] = f2(s);
+  }
+  named_sync(BAR_COMPUTE, LZ_CT);
+}
+
+// Per-warp partial coefficients (lanes over k) -> the CTA's partial row.
+SLS_DEV void store_coeff_partials(dfloat (&cacc)[KT_MAX], int j, int r, float2* __restrict__ cw,
+                                  float2* __restrict__ dst) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 #pragma unroll
-    for (int t = 0; t < CH; ++t) {
-      const int cg = q0 + lane + 32 * t;
-      if (cg < C4) {
-        const float4 wa = w4[2 * cg], wb = w4[2 * cg + 1];
-        dot2_acc(h[0], l[0], f[t].x, wa.x, wa.y);
-        dot2_acc(h[1], l[1], f[t].y, wa.z, wa.w);
-        dot2_acc(h[2], l[2], f[t].z, wb.x, wb.y);
-        dot2_acc(h[3], l[3], f[t].w, wb.z, wb.w);
-      }
+  for (int t = 0; t < KT_MAX; ++t) {
+    const int k = lane + 32 * t;
+    if (k <= j) cw[(size_t)warp * (r + 1) + k] = f2(df_norm(cacc[t].hi, cacc[t].lo));
+  }
+  named_sync(BAR_COMPUTE, LZ_CT);
+  for (int k = tid; k <= j; k += LZ_CT) {
+    dfloat s = df_make(0.f, 0.f);
+    for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(cw[(size_t)w * (r + 1) + k]));
+    dst[k] = f2(s);
+  }
+}
+
+// Loads RPW basis rows (lanes over k < kend) and one double-float vector entry
+// per row; rows past `nb` read as zero.
+SLS_DEV void load_rows(const float2* __restrict__ Q, int r, int64_t i0, int nb, int kend,
+                       const float2* __restrict__ vec, float2 (&q)[RPW][KT_MAX],
+                       float2 (&v)[RPW]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int b = 0; b < RPW; ++b) {
+    const bool ok = b < nb;
+    v[b] = ok ? vec[i0 + b] : make_float2(0.f, 0.f);
+#pragma unroll
+    for (int t = 0; t < KT_MAX; ++t) {
+      const int k = lane + 32 * t;
+      q[b][t] = (ok && k < kend) ? Q[(i0 + b) * r + k] : make_float2(0.f, 0.f);
     }
   }
-  dfloat s = df_add(df_add(df_make(h[0], l[0]), df_make(h[1], l[1])),
-                    df_add(df_make(h[2], l[2]), df_make(h[3], l[3])));
-  return warp_sum_df(s);
+}
+
+// corr[b] = sum_{k < kend} Q[row b, k] * c[k] (float32: the coefficients are
+// tiny corrections), summed over the warp.
+SLS_DEV void row_corrections(const float2 (&q)[RPW][KT_MAX], int kend,
+                             const float2* __restrict__ cs, float (&corr)[RPW]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int b = 0; b < RPW; ++b) corr[b] = 0.f;
+#pragma unroll
+  for (int t = 0; t < KT_MAX; ++t) {
+    const int k = lane + 32 * t;
+    if (k < kend) {
+      const float2 ck = cs[k];
+#pragma unroll
+      for (int b = 0; b < RPW; ++b)
+        corr[b] = fmaf(q[b][t].x, ck.x, fmaf(q[b][t].x, ck.y, fmaf(q[b][t].y, ck.x, corr[b])));
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+    for (int b = 0; b < RPW; ++b) corr[b] += __shfl_xor_sync(0xffffffffu, corr[b], o);
 }
 
 template <int GPT>
 __global__ void __launch_bounds__(LZ_THREADS, 1)
 lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroups,
-               int rows_cap, int* status) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  __shared__ float2 tmpw[LZ_WARPS];
+               int rows_cap, int ring_stages, int* status) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ float2 tmpw[LZ_CW];
   __shared__ double shd[4];
   __shared__ int sflag, sbreak;
+  // copy warp <-> compute warps handshake (no named barrier involves the copy
+  // warp, so an early exit of either side can never leave the other one
+  // blocked in bar.sync; every wait on these flags is bounded)
+  __shared__ volatile int s_halt;       // compute -> copy: stop issuing this problem
+  __shared__ volatile int s_go;         // compute -> copy: may start problem s_go - 1
+  __shared__ volatile int s_pdone;      // copy -> compute: finished problem s_pdone - 1
+  __shared__ volatile unsigned s_issued;  // copy -> compute: chunks issued so far
 
-  const int D = bt.D, r = bt.r, C4 = D >> 2;
+  const int D = bt.D, r = bt.r;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int gi = blockIdx.x / g, rank = blockIdx.x % g;
-  const int P = (C4 >= LZ_THREADS) ? 1 : (LZ_THREADS / C4);
+  const int C4 = D >> 2;
+  const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
   const int redn = (P > 1) ? P * D : 0;
 
-  float2* wsm = reinterpret_cast<float2*>(smem_raw);
-  float2* red = wsm + D;
+  RingState rg;
+  rg.shp = ring_shape(D, 0);
+  rg.shp.S = ring_stages;
+  const int S = ring_stages;
+  const int cr = rg.shp.cr;
+  rg.ring = reinterpret_cast<float*>(smem_raw);
+  unsigned char* after_ring = smem_raw + (size_t)S * rg.shp.chunk;
+  float4* wq = reinterpret_cast<float4*>(after_ring);             // D/2 float4
+  float2* red = reinterpret_cast<float2*>(after_ring + (size_t)D * 8);
   float2* us = red + redn;
-  float2* cw = us + rows_cap;                    // LZ_WARPS x (r+1)
-  float2* cs = cw + (size_t)LZ_WARPS * (r + 1);  // r+1
+  float2* cw = us + rows_cap;                                      // LZ_CW x (r+1)
+  float2* cs = cw + (size_t)LZ_CW * (r + 1);                       // r+1
+  float2* red2 = cs + (r + 1);                                     // 2 * LZ_CT
+  uint64_t* bars = reinterpret_cast<uint64_t*>(
+      (reinterpret_cast<uintptr_t>(red2 + 2 * LZ_CT) + 15) & ~(uintptr_t)15);
+  rg.full = bars;
+  rg.empty = bars + S;
 
   const LzLayout L = lz_layout(bt.nmax, D, r, g);
   char* gb = scratch + (size_t)gi * gstride;
@@ -232,73 +315,203 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   float2* cpartD = reinterpret_cast<float2*>(gb + L.cpartD);
   float2* npart = reinterpret_cast<float2*>(gb + L.npart);
   const GroupBarrier bar{barw, barw + 32, (unsigned)g};
+
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&rg.full[s], 1);
+      mbar_init(&rg.empty[s], LZ_CW);
+    }
+    mbar_fence_init();
+    s_halt = 0;
+    s_go = 0;
+    s_pdone = 0;
+    s_issued = 0;
+  }
+  __syncthreads();
+
+  const int nprob = nprob_of(bt);
+
+  // ========================= copy warp ======================================
+  if (warp == LZ_CW) {
+    if (lane != 0) return;
+    const uint64_t pol = l2_policy_normal();
+    unsigned cnt = 0;
+    int pp = 0;
+    for (int p = gi; p < nprob; p += ngroups, ++pp) {
+      bool go = false;
+      for (unsigned it = 0; it < (1u << 26); ++it) {
+        if (s_go == pp + 1) {
+          go = true;
+          break;
+        }
+        __nanosleep(64);
+      }
+      if (!go) {
+        atomicExch(status, SLS_ERR_TIMEOUT);
+        break;
+      }
+      const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
+      const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
+      const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
+      const int nch = (int)((re - rs + cr - 1) / cr);
+      const float* Phi = bt.Phi + (row0 + rs) * D;
+      bool stop = false;
+      for (int j = 0; j < r && !stop; ++j) {
+        for (int sweep = 0; sweep < 2 && !stop; ++sweep) {
+          for (int t = 0; t < nch; ++t) {
+            if (s_halt) {
+              stop = true;
+              break;
+            }
+            const int k = (sweep == 0) ? t : nch - 1 - t;
+            const int slot = (int)(cnt % (unsigned)S);
+            const unsigned par = (cnt / (unsigned)S) & 1u;
+            if (!mbar_wait(&rg.empty[slot], par ^ 1u)) {
+              atomicExch(status, SLS_ERR_TIMEOUT);
+              stop = true;
+              break;
+            }
+            const int64_t nr = min((int64_t)cr, (re - rs) - (int64_t)k * cr);
+            const unsigned bytes = (unsigned)(nr * D * 4);
+            mbar_expect_tx(&rg.full[slot], bytes);
+            bulk_g2s(rg.ring + (size_t)slot * (rg.shp.chunk / 4), Phi + (int64_t)k * cr * D,
+                     bytes, &rg.full[slot], pol);
+            ++cnt;
+            __threadfence_block();
+            s_issued = cnt;
+          }
+        }
+      }
+      __threadfence_block();
+      s_pdone = pp + 1;
+      if (*((volatile int*)status) == SLS_ERR_TIMEOUT) break;
+    }
+    // every copy issued has landed before the CTA may exit
+    for (unsigned c = (cnt > (unsigned)S ? cnt - S : 0); c < cnt; ++c)
+      mbar_wait(&rg.full[c % S], (c / S) & 1u);
+    return;
+  }
+
+  // ========================= compute warps ===================================
   unsigned lgen = 0;
-
-  int nprob = bt.nprob_max;
-  if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
-
-  for (int p = gi; p < nprob; p += ngroups) {
+  unsigned ccnt = 0;  // chunks consumed
+  int pp = 0;
+  for (int p = gi; p < nprob; p += ngroups, ++pp) {
+    if (tid == 0) {
+      s_halt = 0;
+      __threadfence_block();
+      s_go = pp + 1;
+    }
     const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
     const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
     const int64_t q1o = bt.q1off ? bt.q1off[p] : row0;
-    const float* Phi = bt.Phi + row0 * D;
     float2* Q = bt.Q + row0 * r;
     const double* q1 = bt.q1 + q1o;
     const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
+    const int nrows = (int)(re - rs);
+    const int nch = (nrows + cr - 1) / cr;
     double* alpha_out = bt.alpha + (size_t)p * r;
     double* beta_out = bt.beta + (size_t)p * r;
     const int cbeg = (int)((int64_t)rank * D / g), cend = (int)((int64_t)(rank + 1) * D / g);
 
-    double scale = 0.0;
-    double alpha_prev = 0.0;
+    double scale = 0.0, alpha_prev = 0.0;
     dfloat alpha_df = df_make(0.f, 0.f), beta_df = df_make(0.f, 0.f), invb_df;
     int reff = 0;
 
     for (int j = 0; j < r; ++j) {
       // ---------------- phase A: u_j, stored as column j of Q ----------------
       dfloat nacc = df_make(0.f, 0.f);
-      for (int64_t i = rs + warp; i < re; i += LZ_WARPS) {
-        dfloat u;
+      for (int64_t i0 = rs + (int64_t)warp * RPW; i0 < re; i0 += (int64_t)LZ_CW * RPW) {
+        const int nb = (int)min((int64_t)RPW, re - i0);
+        dfloat u[RPW];
         if (j == 0) {
-          u = df_make(0.f, 0.f);
-          if (lane == 0) u = df_from_double(q1[i]);
-          u = shfl_df(u, 0);
+          dfloat mine = df_make(0.f, 0.f);
+          if (lane < nb) mine = df_from_double(q1[i0 + lane]);
+#pragma unroll
+          for (int b = 0; b < RPW; ++b) u[b] = shfl_df(mine, b);
         } else {
-          const float2* Qi = Q + i * r;
-          float corr = 0.f;
-          for (int k = lane; k < j; k += 32) {
-            const float2 qk = Qi[k], ck = cs[k];
-            corr = fmaf(qk.x, ck.x, fmaf(qk.x, ck.y, fmaf(qk.y, ck.x, corr)));
-          }
-          corr = warp_sum_f(corr);
-          u = df_add(dfv(z1[i]), df_make(-corr, 0.f));
+          float2 q[RPW][KT_MAX], zv[RPW];
+          load_rows(Q, r, i0, nb, j, z1, q, zv);
+          float corr[RPW];
+          row_corrections(q, j, cs, corr);
+#pragma unroll
+          for (int b = 0; b < RPW; ++b) u[b] = df_add(dfv(zv[b]), df_make(-corr[b], 0.f));
         }
         if (lane == 0) {
-          Q[i * r + j] = f2(u);
-          us[i - rs] = f2(u);
-          dot2_acc_df(nacc.hi, nacc.lo, u, u);
+#pragma unroll
+          for (int b = 0; b < RPW; ++b) {
+            if (b < nb) {
+              Q[(i0 + b) * r + j] = f2(u[b]);
+              us[i0 + b - rs] = f2(u[b]);
+              dot2_acc_df(nacc.hi, nacc.lo, u[b], u[b]);
+            }
+          }
         }
       }
       if (lane == 0) tmpw[warp] = f2(df_norm(nacc.hi, nacc.lo));
-      __syncthreads();
+      named_sync(BAR_COMPUTE, LZ_CT);
       if (tid == 0) {
         dfloat s = df_make(0.f, 0.f);
-        for (int w = 0; w < LZ_WARPS; ++w) s = df_add(s, dfv(tmpw[w]));
+        for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(tmpw[w]));
         npart[rank] = f2(s);
       }
-      sweep_phi_t_u<GPT>(Phi, D, rs, re, us, red, wpart + (size_t)rank * D);
-      if (!group_sync(bar, lgen, status, &sflag)) return;
+      // ---------------- sweep A: Phi^T u over the strip (forward) --------------
+      {
+        f32x2_t ah[GPT][2], al[GPT][2];
+#pragma unroll
+        for (int q = 0; q < GPT; ++q) ah[q][0] = ah[q][1] = al[q][0] = al[q][1] = 0ull;
+        for (int t = 0; t < nch; ++t) {
+          const int slot = (int)(ccnt % (unsigned)S);
+          if (!mbar_wait(&rg.full[slot], (ccnt / (unsigned)S) & 1u))
+            atomicExch(status, SLS_ERR_TIMEOUT);  // leave at the next group barrier
+          const int nr = min(cr, nrows - t * cr);
+          sweepA_chunk<GPT>(rg.ring + (size_t)slot * (rg.shp.chunk / 4), nr, D, t * cr, us, ah,
+                            al);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&rg.empty[slot]);
+          ++ccnt;
+        }
+        const int ph = (P == 1) ? 0 : tid / C4;
+        const int cb = (P == 1) ? tid : tid % C4;
+        float2* dst = (P == 1) ? wpart + (size_t)rank * D : red + (size_t)ph * D;
+        if (P == 1 || tid < P * C4) {
+#pragma unroll
+          for (int q = 0; q < GPT; ++q) {
+            const int cg = cb + q * LZ_CT;
+            if (cg < C4) {
+              float h0, h1, l0, l1, h2, h3, l2, l3;
+              upk2(ah[q][0], h0, h1);
+              upk2(al[q][0], l0, l1);
+              upk2(ah[q][1], h2, h3);
+              upk2(al[q][1], l2, l3);
+              dst[4 * cg + 0] = f2(df_norm(h0, l0));
+              dst[4 * cg + 1] = f2(df_norm(h1, l1));
+              dst[4 * cg + 2] = f2(df_norm(h2, l2));
+              dst[4 * cg + 3] = f2(df_norm(h3, l3));
+            }
+          }
+        }
+        if (P > 1) {
+          named_sync(BAR_COMPUTE, LZ_CT);
+          for (int col = tid; col < D; col += LZ_CT) {
+            dfloat s = df_make(0.f, 0.f);
+            for (int q = 0; q < P; ++q) s = df_add(s, dfv(red[(size_t)q * D + col]));
+            wpart[(size_t)rank * D + col] = f2(s);
+          }
+        }
+      }
+      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
 
       // slice reduction of w over the group's CTAs
-      for (int c = cbeg + warp; c < cend; c += LZ_WARPS) {
+      for (int c = cbeg + warp; c < cend; c += LZ_CW) {
         dfloat s = df_make(0.f, 0.f);
         for (int b = lane; b < g; b += 32) s = df_add(s, dfv(wpart[(size_t)b * D + c]));
         s = warp_sum_df(s);
         if (lane == 0) wred[c] = f2(s);
       }
-      if (!group_sync(bar, lgen, status, &sflag)) return;
+      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
 
-      // |u_j|^2, |w_red|^2, w into shared memory
+      // |u_j|^2, |w_red|^2 and the break test
       if (warp == 0) {
         dfloat s = df_make(0.f, 0.f);
         for (int b = lane; b < g; b += 32) s = df_add(s, dfv(npart[b]));
@@ -306,12 +519,18 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         if (lane == 0) shd[0] = df_to_double(s);
       }
       dfloat sq = df_make(0.f, 0.f);
-      for (int c = tid; c < D; c += LZ_THREADS) {
+      for (int c = tid; c < D; c += LZ_CT) {
         const float2 v = wred[c];
-        wsm[c] = v;
         dot2_acc_df(sq.hi, sq.lo, dfv(v), dfv(v));
       }
-      sq = block_sum_df(df_norm(sq.hi, sq.lo), tmpw);
+      {
+        sq = warp_sum_df(df_norm(sq.hi, sq.lo));
+        named_sync(BAR_COMPUTE, LZ_CT);
+        if (lane == 0) tmpw[warp] = f2(sq);
+        named_sync(BAR_COMPUTE, LZ_CT);
+        sq = df_make(0.f, 0.f);
+        for (int w = 0; w < LZ_CW; ++w) sq = df_add(sq, dfv(tmpw[w]));
+      }
       if (tid == 0) {
         const double nrm2 = shd[0];
         const double bnew = sqrt(nrm2);
@@ -321,7 +540,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           if (!(bnew > bt.tol * scale)) brk = 1;
           else if (rank == 0) beta_out[j - 1] = bnew;
         } else if (!(bnew > 0.0)) {
-          brk = 1;  // zero start vector: nothing to iterate
+          brk = 1;
         }
         const double a = brk ? 0.0 : df_to_double(sq) / nrm2;
         if (!brk && rank == 0) alpha_out[j] = a;
@@ -329,8 +548,9 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         shd[2] = a;
         shd[3] = (j > 0) ? bnew : 0.0;
         sbreak = brk;
+        if (brk) s_halt = 1;
       }
-      __syncthreads();
+      named_sync(BAR_COMPUTE, LZ_CT);
       if (sbreak) {
         reff = j;
         break;
@@ -339,98 +559,119 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       alpha_prev = shd[2];
       alpha_df = df_from_double(shd[2]);
       beta_df = df_from_double(shd[3]);
-      for (int c = tid; c < D; c += LZ_THREADS) wsm[c] = f2(df_mul(dfv(wsm[c]), invb_df));
-      __syncthreads();
+      // w = w_red / beta into shared memory as {wh_e, wh_o, wl_e, wl_o} pairs
+      for (int c2 = tid; c2 < D / 2; c2 += LZ_CT) {
+        const dfloat a = df_mul(dfv(wred[2 * c2]), invb_df);
+        const dfloat b = df_mul(dfv(wred[2 * c2 + 1]), invb_df);
+        wq[c2] = make_float4(a.hi, b.hi, a.lo, b.lo);
+      }
+      named_sync(BAR_COMPUTE, LZ_CT);
 
-      // ---------------- phase B: z' = A q_j - alpha q_j - beta q_{j-1} --------
+      // ---------------- sweep B (backward): z' = A q_j - alpha q_j - beta q_{j-1}
       const bool last = (j == r - 1);
       dfloat cacc[(SLS_MAX_R + 1 + 31) / 32];
 #pragma unroll
       for (int t = 0; t < (SLS_MAX_R + 1 + 31) / 32; ++t) cacc[t] = df_make(0.f, 0.f);
-      for (int64_t i = rs + warp; i < re; i += LZ_WARPS) {
-        const dfloat s = row_dot_w(Phi, D, i, wsm);
-        const float2* Qi = Q + i * r;
-        const dfloat qj = df_mul(dfv(Qi[j]), invb_df);
-        dfloat zp = df_sub(s, df_mul(alpha_df, qj));
-        if (j > 0) zp = df_sub(zp, df_mul(beta_df, dfv(Qi[j - 1])));
-        __syncwarp();
-        if (lane == 0) {
-          Q[i * r + j] = f2(qj);
-          z0[i] = f2(zp);
-        }
-        if (!last) {
+      for (int t = 0; t < nch; ++t) {
+        const int k = nch - 1 - t;
+        const int slot = (int)(ccnt % (unsigned)S);
+        if (!mbar_wait(&rg.full[slot], (ccnt / (unsigned)S) & 1u))
+          atomicExch(status, SLS_ERR_TIMEOUT);  // leave at the next group barrier
+        const float* chunk = rg.ring + (size_t)slot * (rg.shp.chunk / 4);
+        const int nr = min(cr, nrows - k * cr);
+        for (int ii = warp; ii < nr; ii += LZ_CW) {
+          const int64_t i = rs + (int64_t)k * cr + ii;
+          const float2* Qi = Q + i * r;
+          float2 qv[KT_MAX];
 #pragma unroll
-          for (int t = 0; t < (SLS_MAX_R + 1 + 31) / 32; ++t) {
-            const int k = lane + 32 * t;
-            if (k <= j) {
-              const dfloat qk = (k == j) ? qj : dfv(Qi[k]);
-              dot2_acc_df(cacc[t].hi, cacc[t].lo, qk, zp);
+          for (int tt = 0; tt < KT_MAX; ++tt) {
+            const int kk = lane + 32 * tt;
+            qv[tt] = (kk <= j) ? Qi[kk] : make_float2(0.f, 0.f);
+          }
+          const dfloat s = row_dot_smem(chunk + (size_t)ii * D, D, wq);
+          float2 sel_j = make_float2(0.f, 0.f), sel_jm1 = make_float2(0.f, 0.f);
+#pragma unroll
+          for (int tt = 0; tt < KT_MAX; ++tt) {
+            if (tt == (j >> 5)) sel_j = qv[tt];
+            if (j > 0 && tt == ((j - 1) >> 5)) sel_jm1 = qv[tt];
+          }
+          const dfloat uj = shfl_df(dfv(sel_j), j & 31);
+          const dfloat qj = df_mul(uj, invb_df);
+          dfloat zp = df_sub(s, df_mul(alpha_df, qj));
+          if (j > 0) zp = df_sub(zp, df_mul(beta_df, shfl_df(dfv(sel_jm1), (j - 1) & 31)));
+          if (lane == 0) {
+            Q[i * r + j] = f2(qj);
+            z0[i] = f2(zp);
+          }
+          if (!last) {
+#pragma unroll
+            for (int tt = 0; tt < KT_MAX; ++tt) {
+              const int kk = lane + 32 * tt;
+              if (kk <= j) {
+                const dfloat qk = (kk == j) ? qj : dfv(qv[tt]);
+                dot2_acc_df(cacc[tt].hi, cacc[tt].lo, qk, zp);
+              }
             }
           }
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&rg.empty[slot]);
+        ++ccnt;
       }
       if (last) {
         reff = r;
         break;
       }
-#pragma unroll
-      for (int t = 0; t < (SLS_MAX_R + 1 + 31) / 32; ++t) {
-        const int k = lane + 32 * t;
-        if (k <= j) cw[(size_t)warp * (r + 1) + k] = f2(df_norm(cacc[t].hi, cacc[t].lo));
-      }
-      __syncthreads();
-      for (int k = tid; k <= j; k += LZ_THREADS) {
-        dfloat s = df_make(0.f, 0.f);
-        for (int w = 0; w < LZ_WARPS; ++w) s = df_add(s, dfv(cw[(size_t)w * (r + 1) + k]));
-        cpartB[(size_t)rank * (r + 1) + k] = f2(s);
-      }
-      if (!group_sync(bar, lgen, status, &sflag)) return;
-      for (int k = warp; k <= j; k += LZ_WARPS) {
-        dfloat s = df_make(0.f, 0.f);
-        for (int b = lane; b < g; b += 32) s = df_add(s, dfv(cpartB[(size_t)b * (r + 1) + k]));
-        s = warp_sum_df(s);
-        if (lane == 0) cs[k] = f2(s);
-      }
-      __syncthreads();
+      store_coeff_partials(cacc, j, r, cw, cpartB + (size_t)rank * (r + 1));
+      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
+      reduce_coeffs(cpartB, g, r, j, cs, red2);
 
       // ---------------- phase D: z1 = z' - Q c, c2 = Q^T z1 ----------------------
 #pragma unroll
-      for (int t = 0; t < (SLS_MAX_R + 1 + 31) / 32; ++t) cacc[t] = df_make(0.f, 0.f);
-      for (int64_t i = rs + warp; i < re; i += LZ_WARPS) {
-        const float2* Qi = Q + i * r;
-        float corr = 0.f;
-        for (int k = lane; k <= j; k += 32) {
-          const float2 qk = Qi[k], ck = cs[k];
-          corr = fmaf(qk.x, ck.x, fmaf(qk.x, ck.y, fmaf(qk.y, ck.x, corr)));
-        }
-        corr = warp_sum_f(corr);
-        const dfloat zz = df_add(dfv(z0[i]), df_make(-corr, 0.f));
-        if (lane == 0) z1[i] = f2(zz);
+      for (int t = 0; t < KT_MAX; ++t) cacc[t] = df_make(0.f, 0.f);
+      for (int64_t i0 = rs + (int64_t)warp * RPW; i0 < re; i0 += (int64_t)LZ_CW * RPW) {
+        const int nb = (int)min((int64_t)RPW, re - i0);
+        float2 q[RPW][KT_MAX], zv[RPW];
+        load_rows(Q, r, i0, nb, j + 1, z0, q, zv);
+        float corr[RPW];
+        row_corrections(q, j + 1, cs, corr);
 #pragma unroll
-        for (int t = 0; t < (SLS_MAX_R + 1 + 31) / 32; ++t) {
-          const int k = lane + 32 * t;
-          if (k <= j) dot2_acc_df(cacc[t].hi, cacc[t].lo, dfv(Qi[k]), zz);
+        for (int b = 0; b < RPW; ++b) {
+          if (b < nb) {
+            const dfloat zz = df_add(dfv(zv[b]), df_make(-corr[b], 0.f));
+            if (lane == 0) z1[i0 + b] = f2(zz);
+#pragma unroll
+            for (int t = 0; t < KT_MAX; ++t) {
+              const int k = lane + 32 * t;
+              if (k <= j) dot2_acc_df(cacc[t].hi, cacc[t].lo, dfv(q[b][t]), zz);
+            }
+          }
         }
       }
-#pragma unroll
-      for (int t = 0; t < (SLS_MAX_R + 1 + 31) / 32; ++t) {
-        const int k = lane + 32 * t;
-        if (k <= j) cw[(size_t)warp * (r + 1) + k] = f2(df_norm(cacc[t].hi, cacc[t].lo));
+      store_coeff_partials(cacc, j, r, cw, cpartD + (size_t)rank * (r + 1));
+      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
+      reduce_coeffs(cpartD, g, r, j, cs, red2);
+    }
+    // a break leaves chunks issued ahead of it: consume them until the copy
+    // warp reports that it stopped
+    if (sbreak) {
+      for (unsigned it = 0; it < (1u << 26); ++it) {
+        const unsigned iss = s_issued;
+        if (ccnt < iss) {
+          const int slot = (int)(ccnt % (unsigned)S);
+          if (!mbar_wait(&rg.full[slot], (ccnt / (unsigned)S) & 1u)) {
+            atomicExch(status, SLS_ERR_TIMEOUT);
+            break;
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&rg.empty[slot]);
+          ++ccnt;
+        } else if (s_pdone == pp + 1) {
+          if (s_issued == ccnt) break;
+        } else {
+          __nanosleep(64);
+        }
       }
-      __syncthreads();
-      for (int k = tid; k <= j; k += LZ_THREADS) {
-        dfloat s = df_make(0.f, 0.f);
-        for (int w = 0; w < LZ_WARPS; ++w) s = df_add(s, dfv(cw[(size_t)w * (r + 1) + k]));
-        cpartD[(size_t)rank * (r + 1) + k] = f2(s);
-      }
-      if (!group_sync(bar, lgen, status, &sflag)) return;
-      for (int k = warp; k <= j; k += LZ_WARPS) {
-        dfloat s = df_make(0.f, 0.f);
-        for (int b = lane; b < g; b += 32) s = df_add(s, dfv(cpartD[(size_t)b * (r + 1) + k]));
-        s = warp_sum_df(s);
-        if (lane == 0) cs[k] = f2(s);
-      }
-      __syncthreads();
     }
     if (rank == 0 && tid == 0) {
       bt.r_eff[p] = reff;
@@ -438,7 +679,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       for (int k = (reff > 0 ? reff - 1 : 0); k < r; ++k) beta_out[k] = 0.0;
     }
     // problems on the same group run back to back; keep them apart
-    if (!group_sync(bar, lgen, status, &sflag)) return;
+    if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
   }
 }
 
@@ -696,12 +937,12 @@ ritz_vectors_kernel(LanczosBatch bt, float* __restrict__ U) {
 
 template <int GPT>
 int launch_lanczos_t(const LanczosBatch& bt, void* scratch, size_t gstride, int groups, int g,
-                     int rows_cap, int* status, size_t smem, cudaStream_t stream) {
+                     int rows_cap, int stages, int* status, size_t smem, cudaStream_t stream) {
   auto fn = lanczos_kernel<GPT>;
   SLS_CUDA_TRY(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   char* sc = (char*)scratch;
   void* args[] = {(void*)&bt, (void*)&sc, (void*)&gstride, (void*)&g, (void*)&groups,
-                  (void*)&rows_cap, (void*)&status};
+                  (void*)&rows_cap, (void*)&stages, (void*)&status};
   SLS_CUDA_TRY(cudaLaunchCooperativeKernel((const void*)fn, dim3(groups * g), dim3(LZ_THREADS),
                                            args, smem, stream));
   count_launch(1);
@@ -763,17 +1004,22 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
   for (int gi = 0; gi < groups; ++gi)
     SLS_CUDA_TRY(cudaMemsetAsync((char*)scratch + (size_t)gi * L.total + L.bar, 0, 256, stream));
   const int C4 = bt.D / 4;
-  const int P = (C4 >= LZ_THREADS) ? 1 : (LZ_THREADS / C4);
+  const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
   const int redn = (P > 1) ? P * bt.D : 0;
   const int rows_cap = (int)((bt.nmax + g - 1) / g) + 1;
-  const size_t smem = sizeof(float2) * ((size_t)bt.D + redn + rows_cap +
-                                        (size_t)(LZ_WARPS + 1) * (bt.r + 1));
-  if (smem > 200 * 1024) return SLS_ERR_UNSUPPORTED;
-  const int gpt = (C4 + LZ_THREADS - 1) / LZ_THREADS;
-  if (gpt <= 1) return launch_lanczos_t<1>(bt, scratch, L.total, groups, g, rows_cap, status, smem, stream);
-  if (gpt <= 2) return launch_lanczos_t<2>(bt, scratch, L.total, groups, g, rows_cap, status, smem, stream);
-  if (gpt <= 4) return launch_lanczos_t<4>(bt, scratch, L.total, groups, g, rows_cap, status, smem, stream);
-  if (gpt <= 8) return launch_lanczos_t<8>(bt, scratch, L.total, groups, g, rows_cap, status, smem, stream);
+  const size_t other = sizeof(float2) * ((size_t)bt.D + redn + rows_cap +
+                                         (size_t)(LZ_CW + 1) * (bt.r + 1) + 2 * LZ_CT) + 16;
+  const size_t limit = 227 * 1024 - 1024;  // leave room for static shared memory
+  if (other + 2 * 16 * 8 >= limit) return SLS_ERR_UNSUPPORTED;
+  RingShape R = ring_shape(bt.D, limit - other - 2 * 6 * 8);
+  if (R.S < 2) return SLS_ERR_UNSUPPORTED;
+  const size_t smem = (size_t)R.S * R.chunk + other + 2 * (size_t)R.S * 8;
+  const int stages = R.S;
+  const int gpt = (C4 + LZ_CT - 1) / LZ_CT;
+  if (gpt <= 1) return launch_lanczos_t<1>(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream);
+  if (gpt <= 2) return launch_lanczos_t<2>(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream);
+  if (gpt <= 4) return launch_lanczos_t<4>(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream);
+  if (gpt <= 8) return launch_lanczos_t<8>(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream);
   return SLS_ERR_UNSUPPORTED;
 }
 
