@@ -1,14 +1,350 @@
-// bf16 feature map on the tcgen05 tensor cores (placeholder until the
-// TMA/tcgen05 kernel lands): reports the shape as unsupported so the caller
-// takes the SIMT path.
+// Random Fourier feature map on the 5th-generation tensor cores (sm_103a):
+//   Phi = sqrt(2/D) * cos(X W^T + b)      (Sec. 3.2, Eq. rff_map)
+// X (N x d) and W = Omega^T (D x d) are bf16, K-major (row-major, K = d
+// contiguous); the contraction accumulates in fp32 in tensor memory; the
+// epilogue adds b, takes the cosine, scales and stores Phi (fp32) once.
+//
+// One persistent CTA per SM, 128 x 256 output tiles (tile index -> m-block
+// outer, n-block inner, so the D/256 tiles that share an X block run at the
+// same time and X is read from HBM once).  Warp roles:
+//   warp 0  TMA producer: 128B-swizzled 128x64 (X) and 256x64 (W) bf16 tiles
+//           into a 4-stage shared-memory ring (mbarrier complete_tx);
+//   warp 1  MMA issuer: one elected thread issues tcgen05.mma (M=128, N=256,
+//           K=16 per instruction, kind::f16 with bf16 inputs) into one of two
+//           256-column fp32 accumulators in tensor memory; tcgen05.commit
+//           releases ring stages and hands finished accumulators over;
+//   warps 2-5 epilogue: tcgen05.ld 32x32b (one TMEM lane = one output row
+//           per thread), cos epilogue, global stores; then release the
+//           accumulator, so the next tile's MMAs overlap this epilogue.
+// Every wait is bounded; a wait that gives up records SLS_ERR_TIMEOUT, the
+// other roles stop at their next wait, in-flight copies and MMAs are drained
+// and the tensor memory is freed before the CTA exits.
+#include <cuda.h>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
 namespace sls {
 
-int launch_feature_map_tc(const void*, int64_t, int, int64_t, const void*, const float*, int,
-                          float*, cudaStream_t) {
-  return SLS_ERR_UNSUPPORTED;
+namespace {
+
+constexpr int TC_BM = 128;
+constexpr int TC_BN = 256;
+constexpr int TC_BK = 64;  // one 128-byte swizzle atom of bf16
+constexpr int TC_STAGES = 4;
+constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;
+constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;
+constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
+constexpr int TC_THREADS = 192;
+constexpr int TC_TMEM_COLS = 2 * TC_BN;
+constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES + 1024 + 256;
+
+__device__ int g_fm_status;  // timeouts when the caller passes no status word
+
+// K-major, 128-byte swizzle shared-memory matrix descriptor (tcgen05 format):
+// start address >> 4, leading byte offset 16 B (unused for this layout),
+// stride byte offset 1024 B (eight 128-byte rows), descriptor version 1,
+// swizzle mode 2 (128B).
+SLS_DEV uint64_t sw128_desc(uint32_t smem_addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((smem_addr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)(16u >> 4) << 16;
+  d |= (uint64_t)(1024u >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, M = 128, N = 256.
+constexpr uint32_t TC_IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
+                              ((uint32_t)(TC_BN >> 3) << 17) | ((uint32_t)(TC_BM >> 4) << 24);
+
+SLS_DEV void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+SLS_DEV void tc_mma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(TC_IDESC), "r"(accumulate)
+      : "memory");
+}
+
+SLS_DEV void tc_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+SLS_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+SLS_DEV void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+SLS_DEV void tc_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+        "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+        "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Bounded wait that also gives up as soon as another role aborted.
+SLS_DEV bool tc_wait(uint64_t* bar, unsigned parity, volatile int* abort_flag) {
+  for (unsigned it = 0; it < (1u << 25); ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255) == 255 && *abort_flag) return false;
+    if (it > 64) __nanosleep(20);
+  }
+  return false;
+}
+
+__global__ void __launch_bounds__(TC_THREADS, 1)
+feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
+                      const __grid_constant__ CUtensorMap tmW, const float* __restrict__ bvec,
+                      float* __restrict__ Phi, int N, int D, int K, float scale, int* status) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  __shared__ uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES], tfull[2], tempty[2], done_bar;
+  __shared__ uint32_t tmem_holder;
+  __shared__ volatile int s_abort;
+
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const uint32_t smem_base = smem_u32(smem);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m_tiles = (N + TC_BM - 1) / TC_BM;
+  const int n_tiles = D / TC_BN;
+  const int num_tiles = m_tiles * n_tiles;
+  const int k_blocks = (K + TC_BK - 1) / TC_BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < TC_STAGES; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 4);
+    }
+    mbar_init(&done_bar, 1);
+    mbar_fence_init();
+    s_abort = 0;
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&tmem_holder)),
+                 "r"(TC_TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = tmem_holder;
+
+  auto fail = [&]() {
+    s_abort = 1;
+    atomicExch(status, SLS_ERR_TIMEOUT);
+  };
+
+  if (warp == 0) {
+    // ------------------------------ TMA producer ------------------------------
+    if (lane == 0) {
+      unsigned it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        const int mb = tile / n_tiles, nb = tile % n_tiles;
+        for (int kb = 0; kb < k_blocks; ++kb, ++it) {
+          const int s = it % TC_STAGES;
+          const unsigned par = (it / TC_STAGES) & 1u;
+          if (!tc_wait(&empty_bar[s], par ^ 1u, &s_abort)) {
+            fail();
+            ok = false;
+            break;
+          }
+          const uint32_t a_dst = smem_base + s * TC_STAGE_BYTES;
+          const uint32_t b_dst = a_dst + TC_A_BYTES;
+          mbar_expect_tx(&full_bar[s], TC_STAGE_BYTES);
+          tma_load_2d(a_dst, &tmX, kb * TC_BK, mb * TC_BM, smem_u32(&full_bar[s]));
+          tma_load_2d(b_dst, &tmW, kb * TC_BK, nb * TC_BN, smem_u32(&full_bar[s]));
+        }
+      }
+      // drain: every issued stage has landed before the CTA may exit
+      const unsigned first = it > TC_STAGES ? it - TC_STAGES : 0;
+      for (unsigned c = first; c < it; ++c) {
+        for (unsigned w = 0; w < (1u << 25); ++w) {
+          if (mbar_try_wait(&full_bar[c % TC_STAGES], (c / TC_STAGES) & 1u)) break;
+          __nanosleep(20);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------ MMA issuer --------------------------------
+    if (lane == 0) {
+      unsigned it = 0, acc_it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++acc_it) {
+        const int acc = acc_it & 1;
+        const unsigned apar = (acc_it >> 1) & 1u;
+        if (!tc_wait(&tempty[acc], apar ^ 1u, &s_abort)) {
+          fail();
+          break;
+        }
+        tc_fence_after();
+        const uint32_t tmem_d = tmem_base + (uint32_t)(acc * TC_BN);
+        for (int kb = 0; kb < k_blocks; ++kb, ++it) {
+          const int s = it % TC_STAGES;
+          const unsigned par = (it / TC_STAGES) & 1u;
+          if (!tc_wait(&full_bar[s], par, &s_abort)) {
+            fail();
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = smem_base + s * TC_STAGE_BYTES;
+          const uint32_t b_addr = a_addr + TC_A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < TC_BK / 16; ++kk) {
+            tc_mma(tmem_d, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32),
+                   (kb > 0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(smem_u32(&empty_bar[s]));
+        }
+        if (ok) tc_commit(smem_u32(&tfull[acc]));
+      }
+      // all MMAs issued by this thread have completed before TMEM is freed
+      tc_commit(smem_u32(&done_bar));
+      for (unsigned w = 0; w < (1u << 25); ++w) {
+        if (mbar_try_wait(&done_bar, 0)) break;
+        __nanosleep(20);
+      }
+    }
+  } else {
+    // ------------------------------ epilogue ----------------------------------
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    unsigned acc_it = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++acc_it) {
+      const int mb = tile / n_tiles, nb = tile % n_tiles;
+      const int acc = acc_it & 1;
+      const unsigned apar = (acc_it >> 1) & 1u;
+      if (!tc_wait(&tfull[acc], apar, &s_abort)) {
+        if (lane == 0) fail();
+        break;
+      }
+      tc_fence_after();
+      const int row = mb * TC_BM + q * 32 + lane;
+      float* out = Phi + (size_t)row * D + (size_t)nb * TC_BN;
+      const float* bb = bvec + (size_t)nb * TC_BN;
+      for (int c0 = 0; c0 < TC_BN; c0 += 32) {
+        uint32_t v[32];
+        tc_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + c0), v);
+        if (row < N) {
+#pragma unroll
+          for (int e = 0; e < 32; e += 4) {
+            const float4 bq = __ldg(reinterpret_cast<const float4*>(bb + c0 + e));
+            float4 o;
+            o.x = scale * cosf(__uint_as_float(v[e + 0]) + bq.x);
+            o.y = scale * cosf(__uint_as_float(v[e + 1]) + bq.y);
+            o.z = scale * cosf(__uint_as_float(v[e + 2]) + bq.z);
+            o.w = scale * cosf(__uint_as_float(v[e + 3]) + bq.w);
+            *reinterpret_cast<float4*>(out + c0 + e) = o;
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TC_TMEM_COLS)
+                 : "memory");
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+              uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {ld * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)TC_BK, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int sm_count() {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0)
+      sms = v;
+    else
+      return 1;
+  }
+  return sms;
+}
+
+}  // namespace
+
+int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
+                          const float* b, int D, float* Phi, cudaStream_t stream,
+                          int* status) {
+  // shapes the kernel covers; anything else takes the SIMT path
+  if (N <= 0 || N > (int64_t)INT32_MAX - TC_BM || D % TC_BN != 0 || d % 8 != 0 || ldx % 8 != 0)
+    return SLS_ERR_UNSUPPORTED;
+  if (((uintptr_t)X & 15) || ((uintptr_t)W & 15) || ((uintptr_t)b & 15) || ((uintptr_t)Phi & 15))
+    return SLS_ERR_UNSUPPORTED;
+  CUtensorMap mx, mw;
+  if (!make_map(&mx, X, (uint64_t)N, (uint64_t)d, (uint64_t)ldx, TC_BM)) return SLS_ERR_UNSUPPORTED;
+  if (!make_map(&mw, W, (uint64_t)D, (uint64_t)d, (uint64_t)d, TC_BN)) return SLS_ERR_UNSUPPORTED;
+  int* st = status;
+  if (!st) SLS_CUDA_TRY(cudaGetSymbolAddress((void**)&st, g_fm_status));
+  SLS_CUDA_TRY(cudaFuncSetAttribute(feature_map_tc_kernel,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TC_SMEM));
+  const int tiles = (int)((N + TC_BM - 1) / TC_BM) * (D / TC_BN);
+  const int grid = tiles < sm_count() ? tiles : sm_count();
+  const float scale = (float)sqrt(2.0 / (double)D);
+  feature_map_tc_kernel<<<grid, TC_THREADS, TC_SMEM, stream>>>(mx, mw, b, Phi, (int)N, D, d,
+                                                               scale, st);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
 }
 
 }  // namespace sls

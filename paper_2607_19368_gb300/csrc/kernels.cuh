@@ -13,7 +13,8 @@ int launch_feature_map_simt(const void* X, int x_dtype, int64_t N, int d, int64_
 // tcgen05 / TMA path for bf16 inputs; returns SLS_ERR_UNSUPPORTED when the
 // shape is outside what the kernel handles (the caller then uses the SIMT path).
 int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
-                          const float* b, int D, float* Phi, cudaStream_t stream);
+                          const float* b, int D, float* Phi, cudaStream_t stream,
+                          int* status = nullptr);
 
 // ---- Lanczos (Algorithm 2) --------------------------------------------------
 // A batch of independent problems, problem p owning rows
