@@ -364,7 +364,7 @@ void carve(const CompressPlan& P, void* ws, CompressWs* W) {
   W->nspec = cv.take<int>(1);
   W->score = cv.take<float>(np);
   W->Phi = cv.take<float>(spectral ? (size_t)rows * P.D : 0);
-  W->Q = cv.take<float2>(spectral ? (size_t)rows * P.r : 0);
+  W->Q = cv.take<float2>(spectral ? (size_t)rows * ((P.r + 1) & ~1) : 0);
   W->alpha = cv.take<double>(spectral ? (size_t)np * P.r : 0);
   W->beta = cv.take<double>(spectral ? (size_t)np * P.r : 0);
   W->theta = cv.take<double>(spectral ? (size_t)np * P.r : 0);
@@ -452,7 +452,7 @@ size_t sls_lanczos_workspace_size(int64_t N, int D, int r) {
   if (lanczos_plan(N, D, r, 1, &groups, &g) != SLS_OK) return 0;
   Carver cv(nullptr);
   cv.take<int>(64);
-  cv.take<float2>((size_t)N * r);
+  cv.take<float2>((size_t)N * ((r + 1) & ~1));
   cv.take<double>(r);
   cv.take<double>(r);
   cv.take<double>((size_t)r * r);
@@ -476,7 +476,7 @@ int sls_lanczos_topr(const float* Phi, int64_t N, int D, int r, const double* q1
   cudaStream_t s = (cudaStream_t)stream;
   Carver cv(workspace);
   int* status = cv.take<int>(64);
-  float2* Q = cv.take<float2>((size_t)N * r);
+  float2* Q = cv.take<float2>((size_t)N * ((r + 1) & ~1));
   double* al = cv.take<double>(r);
   double* be = cv.take<double>(r);
   double* S = cv.take<double>((size_t)r * r);

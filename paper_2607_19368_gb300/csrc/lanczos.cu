@@ -2,27 +2,39 @@
 //
 // Lanczos runs as one persistent cooperative kernel.  The grid is split into
 // groups of CTAs; a group owns one problem at a time (one prompt, or one
-// adaptive window) and its CTAs own contiguous row strips of that problem's
-// feature matrix Phi (N x D, float32).  One step j costs two streaming sweeps
-// over the strip and four group barriers:
+// adaptive window) and every CTA owns a contiguous strip of the problem's rows
+// of the feature matrix Phi (N x D, float32) and of the basis Q.  One copy warp
+// per CTA streams the strip through a shared-memory ring with one-dimensional
+// bulk copies (cp.async.bulk + mbarrier): each ring stage holds a few rows of
+// Phi and the same rows of Q.  Eight compute warps consume the ring.
 //
-//   A  u_j = z1 - Q c2 (second Gram-Schmidt correction of step j-1), stored
-//      as column j of Q; w_part = Phi^T u_j and |u_j|^2 per CTA.
-//      [barrier]  every CTA reduces a slice of the D columns
-//      [barrier]  beta_{j-1} = |u_j|, w = Phi^T q_j = w_red / beta_{j-1},
-//                 alpha_j = q_j^T A q_j = |w|^2, break test
-//   B  z' = Phi w - alpha_j q_j - beta_{j-1} q_{j-1}   (the implicit matvec of
-//      Eq. implicit_matvec and the three-term recurrence) and the first
-//      Gram-Schmidt coefficients c = Q^T z' per CTA
-//      [barrier]  c = sum of the CTA partials
-//   D  z1 = z' - Q c and the second coefficients c2 = Q^T z1 per CTA
-//      [barrier]  c2 = sum of the CTA partials
+// Step j (0-based) makes two passes over the strip and three group barriers:
 //
-// Normalisation is deferred (q_j = u_j / |u_j| is applied in B), so |u_j|
-// rides along with the first sweep.  All vectors are double-float (two
-// float32) and every sum over N or D is Dot2-compensated; reductions use a
-// fixed order, so results are bit-reproducible.  Barriers give up after a
-// bounded number of polls and report SLS_ERR_TIMEOUT through the status word.
+//   sweep A (forward)   per row: z1 = z' - Q c          (first Gram-Schmidt
+//                       pass of step j-1, c from the previous barrier 3),
+//                       c2 += Q^T z1, |z1|^2; then Phi^T z1 column-parallel.
+//                       [barrier 1]
+//   slice phase         c2 = sum of the CTA partials (second Gram-Schmidt
+//                       coefficients); each CTA finishes a slice of the D
+//                       columns of Phi^T u_j = Phi^T z1 - sum_k c2_k w_k with
+//                       w_k = Phi^T q_k kept from earlier steps.
+//                       [barrier 2]
+//                       beta_{j-1} = |u_j| = sqrt(|z1|^2 - |c2|^2), the break
+//                       test, w_j = Phi^T q_j, alpha_j = |w_j|^2.
+//   sweep B (backward)  per row: u = z1 - Q c2, q_j = u / beta_{j-1}, the
+//                       implicit matvec row Phi w_j (Eq. implicit_matvec), the
+//                       three-term recurrence z' = A q_j - alpha_j q_j -
+//                       beta_{j-1} q_{j-1}, and c += Q^T z'.
+//                       [barrier 3]  c = sum of the CTA partials
+//
+// For j = 0, z1 is the start vector q1.  This is Algorithm 2 with two-pass
+// classical Gram-Schmidt re-orthogonalisation, regrouped so that all per-row
+// work rides on the two streaming passes; in exact arithmetic it equals the
+// textbook order.  Sweep B runs backward so the rows sweep A touched last are
+// still in L2.  Vectors are double-float (two float32), every sum over N or D
+// is Dot2-compensated, reductions have a fixed order (bit-reproducible runs).
+// Barriers and waits give up after a bounded number of polls and report
+// SLS_ERR_TIMEOUT through the status word.
 //
 // The r x r (r <= 128) tridiagonal T is then solved on the device: Ritz values
 // by Sturm-count multisection (one warp per eigenvalue, 32 shifts per round,
@@ -41,26 +53,31 @@ namespace {
 constexpr int LZ_CW = 8;                  // compute warps
 constexpr int LZ_CT = LZ_CW * 32;         // compute threads
 constexpr int LZ_THREADS = LZ_CT + 32;    // plus one copy warp
-constexpr int LZ_WARPS = LZ_CW;
+constexpr unsigned BAR_COMPUTE = 1;       // named barrier: the compute warps
+constexpr int KT_MAX = (SLS_MAX_R + 1 + 31) / 32;  // basis columns per lane
+
+// leading dimension (float2) of the basis rows: even, so rows are 16-byte aligned
+__host__ __device__ inline int q_ld(int r) { return (r + 1) & ~1; }
 
 // Per-group scratch layout (byte offsets), identical on host and device.
 struct LzLayout {
-  size_t z0, z1, wpart, wred, cpartB, cpartD, npart, bar, total;
+  size_t bar, wpart, wred, Wm, cpartA, cpartB, npart, sqpart, total;
 };
 
 __host__ __device__ inline size_t lz_al(size_t x) { return (x + 255) & ~(size_t)255; }
 
 __host__ __device__ inline LzLayout lz_layout(int64_t nmax, int D, int r, int g) {
+  (void)nmax;
   LzLayout L;
   size_t o = 0;
   L.bar = o;    o += 256;
-  L.z0 = o;     o += lz_al((size_t)nmax * sizeof(float2));
-  L.z1 = o;     o += lz_al((size_t)nmax * sizeof(float2));
   L.wpart = o;  o += lz_al((size_t)g * D * sizeof(float2));
   L.wred = o;   o += lz_al((size_t)D * sizeof(float2));
+  L.Wm = o;     o += lz_al((size_t)D * r * sizeof(float2));
+  L.cpartA = o; o += lz_al((size_t)g * (r + 1) * sizeof(float2));
   L.cpartB = o; o += lz_al((size_t)g * (r + 1) * sizeof(float2));
-  L.cpartD = o; o += lz_al((size_t)g * (r + 1) * sizeof(float2));
   L.npart = o;  o += lz_al((size_t)g * sizeof(float2));
+  L.sqpart = o; o += lz_al((size_t)g * sizeof(float2));
   L.total = o;
   return L;
 }
@@ -74,44 +91,29 @@ SLS_DEV dfloat shfl_df(dfloat v, int src) {
   return v;
 }
 
-// ---------------------------------------------------------------------------
-// The feature matrix is streamed through a shared-memory ring.  One copy warp
-// issues one-dimensional bulk copies (cp.async.bulk) of consecutive row chunks
-// of the CTA's strip, each completing on the stage's "full" mbarrier; the
-// eight compute warps release a stage on its "empty" mbarrier.  Sweep A walks
-// the strip forward and sweep B backward, so the chunks sweep A touched last
-// are still in L2 when sweep B starts (and vice versa at the next step).  The
-// copy warp runs ahead across the group barriers, so the loads of the next
-// sweep overlap the reductions between sweeps.
-// ---------------------------------------------------------------------------
-
-constexpr unsigned BAR_COMPUTE = 1;  // named barrier: the compute warps
-constexpr int RING_TARGET = 64 * 1024;  // bytes per ring stage (a few rows)
-
+// Ring stage: cr rows of Phi (cr * D floats) followed by the same cr rows of Q
+// (cr * ldq float2).
 struct RingShape {
-  int cr;            // rows per chunk
-  int S;             // stages
-  unsigned chunk;    // bytes per full chunk
+  int cr;          // rows per chunk
+  int S;           // stages
+  unsigned phib;   // bytes of Phi per full chunk
+  unsigned stage;  // bytes per stage
 };
 
-__host__ __device__ inline RingShape ring_shape(int D, size_t budget) {
+constexpr int RING_TARGET = 56 * 1024;
+
+__host__ __device__ inline RingShape ring_shape(int D, int ldq, size_t budget) {
   RingShape R;
-  R.cr = RING_TARGET / (4 * D);
+  R.cr = RING_TARGET / (4 * D + 8 * ldq);
   if (R.cr < 1) R.cr = 1;
-  R.chunk = (unsigned)R.cr * (unsigned)D * 4u;
-  R.S = (int)(budget / R.chunk);
+  R.phib = (unsigned)R.cr * (unsigned)D * 4u;
+  R.stage = R.phib + (unsigned)R.cr * (unsigned)ldq * 8u;
+  R.S = (int)(budget / R.stage);
   if (R.S > 6) R.S = 6;
   return R;
 }
 
-struct RingState {
-  uint64_t* full;
-  uint64_t* empty;
-  float* ring;
-  RingShape shp;
-};
-
-// Sweep A over one chunk: acc[c] += Phi[i, c] * u_i for the chunk's rows,
+// Sweep A over one chunk: acc[c] += Phi[i, c] * z1_i for the chunk's rows,
 // column-parallel (GPT float4 groups per thread, P row phases).
 template <int GPT>
 SLS_DEV void sweepA_chunk(const float* __restrict__ chunk, int nr, int D, int lb,
@@ -139,19 +141,30 @@ SLS_DEV void sweepA_chunk(const float* __restrict__ chunk, int nr, int D, int lb
   }
 }
 
-// Row dot product with w from shared memory (layout: per column pair
-// {wh_even, wh_odd, wl_even, wl_odd}); one warp per row, all lanes get it.
-SLS_DEV dfloat row_dot_smem(const float* __restrict__ row, int D,
-                            const float4* __restrict__ wq) {
+// Row dot product with w from shared memory (separate hi / lo arrays); one
+// warp per row, all lanes get the sum.
+SLS_DEV dfloat row_dot_smem(const float* __restrict__ row, int D, const float* __restrict__ wsh,
+                            const float* __restrict__ wsl) {
   const int lane = threadIdx.x & 31;
   const int C4 = D >> 2;
   const float4* r4 = reinterpret_cast<const float4*>(row);
+  const float4* h4 = reinterpret_cast<const float4*>(wsh);
+  const float4* l4 = reinterpret_cast<const float4*>(wsl);
   f32x2_t h01 = 0, l01 = 0, h23 = 0, l23 = 0;
-  for (int cg = lane; cg < C4; cg += 32) {
+  int cg = lane;
+  for (; cg + 32 < C4; cg += 64) {
+    const float4 f0 = r4[cg], f1 = r4[cg + 32];
+    const float4 wh0 = h4[cg], wl0 = l4[cg], wh1 = h4[cg + 32], wl1 = l4[cg + 32];
+    dot2_acc2(h01, l01, pk2(f0.x, f0.y), pk2(wh0.x, wh0.y), pk2(wl0.x, wl0.y));
+    dot2_acc2(h23, l23, pk2(f0.z, f0.w), pk2(wh0.z, wh0.w), pk2(wl0.z, wl0.w));
+    dot2_acc2(h01, l01, pk2(f1.x, f1.y), pk2(wh1.x, wh1.y), pk2(wl1.x, wl1.y));
+    dot2_acc2(h23, l23, pk2(f1.z, f1.w), pk2(wh1.z, wh1.w), pk2(wl1.z, wl1.w));
+  }
+  for (; cg < C4; cg += 32) {
     const float4 f = r4[cg];
-    const float4 wa = wq[2 * cg], wb = wq[2 * cg + 1];
-    dot2_acc2(h01, l01, pk2(f.x, f.y), pk2(wa.x, wa.y), pk2(wa.z, wa.w));
-    dot2_acc2(h23, l23, pk2(f.z, f.w), pk2(wb.x, wb.y), pk2(wb.z, wb.w));
+    const float4 wh = h4[cg], wl = l4[cg];
+    dot2_acc2(h01, l01, pk2(f.x, f.y), pk2(wh.x, wh.y), pk2(wl.x, wl.y));
+    dot2_acc2(h23, l23, pk2(f.z, f.w), pk2(wh.z, wh.w), pk2(wl.z, wl.w));
   }
   float a0, a1, b0, b1, c0, c1, d0, d1;
   upk2(h01, a0, a1);
@@ -169,19 +182,17 @@ SLS_DEV int nprob_of(const LanczosBatch& bt) {
   return nprob;
 }
 
-constexpr int KT_MAX = (SLS_MAX_R + 1 + 31) / 32;  // basis columns per lane
-constexpr int RPW = 4;                               // rows per warp in the row passes
-
 // Sum of the per-CTA partial coefficients part[b * (r+1) + k] over the g CTAs
-// of a group, for k <= j, into cs[k].  Every CTA does it redundantly; the
-// loads are spread over all compute threads so they are in flight together.
-SLS_DEV void reduce_coeffs(const float2* __restrict__ part, int g, int r, int j,
+// of a group, for k < K, into cs[k].  Every CTA does it redundantly; the loads
+// are spread over all compute threads so they are in flight together.
+SLS_DEV void reduce_coeffs(const float2* __restrict__ part, int g, int r, int K,
                            float2* __restrict__ cs, float2* __restrict__ tmp) {
   const int tid = threadIdx.x;
-  const int K = j + 1;
+  if (K <= 0) return;
   int PH = LZ_CT / K;
   if (PH < 1) PH = 1;
   if (PH > 8) PH = 8;
+  while (PH > 1 && PH * K > 4 * LZ_CT) --PH;
   for (int idx = tid; idx < K * PH; idx += LZ_CT) {
     const int k = idx % K, ph = idx / K;
     dfloat s = df_make(0.f, 0.f);
@@ -205,62 +216,38 @@ SLS_DEV void reduce_coeffs(const float2* __restrict__ part, int g, int r, int j,
   named_sync(BAR_COMPUTE, LZ_CT);
 }
 
-// Per-warp partial coefficients (lanes over k) -> the CTA's partial row.
-SLS_DEV void store_coeff_partials(dfloat (&cacc)[KT_MAX], int j, int r, float2* __restrict__ cw,
+// Per-warp partial coefficients (lanes over k < K) -> the CTA's partial row.
+SLS_DEV void store_coeff_partials(dfloat (&cacc)[KT_MAX], int K, int r, float2* __restrict__ cw,
                                   float2* __restrict__ dst) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 #pragma unroll
   for (int t = 0; t < KT_MAX; ++t) {
     const int k = lane + 32 * t;
-    if (k <= j) cw[(size_t)warp * (r + 1) + k] = f2(df_norm(cacc[t].hi, cacc[t].lo));
+    if (k < K) cw[(size_t)warp * (r + 1) + k] = f2(df_norm(cacc[t].hi, cacc[t].lo));
   }
   named_sync(BAR_COMPUTE, LZ_CT);
-  for (int k = tid; k <= j; k += LZ_CT) {
+  for (int k = tid; k < K; k += LZ_CT) {
     dfloat s = df_make(0.f, 0.f);
     for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(cw[(size_t)w * (r + 1) + k]));
     dst[k] = f2(s);
   }
 }
 
-// Loads RPW basis rows (lanes over k < kend) and one double-float vector entry
-// per row; rows past `nb` read as zero.
-SLS_DEV void load_rows(const float2* __restrict__ Q, int r, int64_t i0, int nb, int kend,
-                       const float2* __restrict__ vec, float2 (&q)[RPW][KT_MAX],
-                       float2 (&v)[RPW]) {
+// sum_{k < K} q[k] * c[k] over the warp (lanes over k), float32: the
+// coefficients are small corrections; every lane gets the result.
+SLS_DEV float row_correction(const float2* __restrict__ qrow, const float2* __restrict__ c,
+                             int K) {
   const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int b = 0; b < RPW; ++b) {
-    const bool ok = b < nb;
-    v[b] = ok ? vec[i0 + b] : make_float2(0.f, 0.f);
-#pragma unroll
-    for (int t = 0; t < KT_MAX; ++t) {
-      const int k = lane + 32 * t;
-      q[b][t] = (ok && k < kend) ? Q[(i0 + b) * r + k] : make_float2(0.f, 0.f);
-    }
-  }
-}
-
-// corr[b] = sum_{k < kend} Q[row b, k] * c[k] (float32: the coefficients are
-// tiny corrections), summed over the warp.
-SLS_DEV void row_corrections(const float2 (&q)[RPW][KT_MAX], int kend,
-                             const float2* __restrict__ cs, float (&corr)[RPW]) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int b = 0; b < RPW; ++b) corr[b] = 0.f;
+  float s = 0.f;
 #pragma unroll
   for (int t = 0; t < KT_MAX; ++t) {
     const int k = lane + 32 * t;
-    if (k < kend) {
-      const float2 ck = cs[k];
-#pragma unroll
-      for (int b = 0; b < RPW; ++b)
-        corr[b] = fmaf(q[b][t].x, ck.x, fmaf(q[b][t].x, ck.y, fmaf(q[b][t].y, ck.x, corr[b])));
+    if (k < K) {
+      const float2 q = qrow[k], cc = c[k];
+      s = fmaf(q.x, cc.x, fmaf(q.x, cc.y, fmaf(q.y, cc.x, s)));
     }
   }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-    for (int b = 0; b < RPW; ++b) corr[b] += __shfl_xor_sync(0xffffffffu, corr[b], o);
+  return warp_sum_f(s);
 }
 
 template <int GPT>
@@ -272,59 +259,63 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   __shared__ double shd[4];
   __shared__ int sflag, sbreak;
   // copy warp <-> compute warps handshake (no named barrier involves the copy
-  // warp, so an early exit of either side can never leave the other one
-  // blocked in bar.sync; every wait on these flags is bounded)
-  __shared__ volatile int s_halt;       // compute -> copy: stop issuing this problem
-  __shared__ volatile int s_go;         // compute -> copy: may start problem s_go - 1
-  __shared__ volatile int s_pdone;      // copy -> compute: finished problem s_pdone - 1
+  // warp, so an early exit of either side can never leave the other blocked in
+  // bar.sync; every wait on these flags is bounded)
+  __shared__ volatile int s_halt;        // compute -> copy: stop issuing this problem
+  __shared__ volatile int s_go;          // compute -> copy: may start problem s_go - 1
+  __shared__ volatile int s_pdone;       // copy -> compute: finished problem s_pdone - 1
+  __shared__ volatile int s_bdone;       // compute -> copy: sweep B of (problem, step) done
   __shared__ volatile unsigned s_issued;  // copy -> compute: chunks issued so far
 
-  const int D = bt.D, r = bt.r;
+  const int D = bt.D, r = bt.r, ldq = q_ld(bt.r);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int gi = blockIdx.x / g, rank = blockIdx.x % g;
   const int C4 = D >> 2;
   const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
   const int redn = (P > 1) ? P * D : 0;
 
-  RingState rg;
-  rg.shp = ring_shape(D, 0);
-  rg.shp.S = ring_stages;
+  const RingShape shp0 = ring_shape(D, ldq, 0);
   const int S = ring_stages;
-  const int cr = rg.shp.cr;
-  rg.ring = reinterpret_cast<float*>(smem_raw);
-  unsigned char* after_ring = smem_raw + (size_t)S * rg.shp.chunk;
-  float4* wq = reinterpret_cast<float4*>(after_ring);             // D/2 float4
-  float2* red = reinterpret_cast<float2*>(after_ring + (size_t)D * 8);
-  float2* us = red + redn;
-  float2* cw = us + rows_cap;                                      // LZ_CW x (r+1)
-  float2* cs = cw + (size_t)LZ_CW * (r + 1);                       // r+1
-  float2* red2 = cs + (r + 1);                                     // 2 * LZ_CT
+  const int cr = shp0.cr;
+  const unsigned phib = shp0.phib, stage = shp0.stage;
+  unsigned char* ring = smem_raw;
+  unsigned char* after_ring = smem_raw + (size_t)S * stage;
+  float* wsh = reinterpret_cast<float*>(after_ring);   // D
+  float* wsl = wsh + D;                                // D
+  float2* red = reinterpret_cast<float2*>(wsl + D);    // redn
+  float2* us = red + redn;                             // rows_cap (z1 of the strip)
+  float2* zps = us + rows_cap;                         // rows_cap (z' of the strip)
+  float2* cw = zps + rows_cap;                         // LZ_CW x (r+1)
+  float2* cs = cw + (size_t)LZ_CW * (r + 1);           // r+1 (c, first pass)
+  float2* c2s = cs + (r + 1);                          // r+1 (c2, second pass)
+  float2* red2 = c2s + (r + 1);                        // 4 * LZ_CT
   uint64_t* bars = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(red2 + 2 * LZ_CT) + 15) & ~(uintptr_t)15);
-  rg.full = bars;
-  rg.empty = bars + S;
+      (reinterpret_cast<uintptr_t>(red2 + 4 * LZ_CT) + 15) & ~(uintptr_t)15);
+  uint64_t* fullb = bars;
+  uint64_t* emptyb = bars + S;
 
   const LzLayout L = lz_layout(bt.nmax, D, r, g);
   char* gb = scratch + (size_t)gi * gstride;
   unsigned* barw = reinterpret_cast<unsigned*>(gb + L.bar);
-  float2* z0 = reinterpret_cast<float2*>(gb + L.z0);
-  float2* z1 = reinterpret_cast<float2*>(gb + L.z1);
   float2* wpart = reinterpret_cast<float2*>(gb + L.wpart);
   float2* wred = reinterpret_cast<float2*>(gb + L.wred);
+  float2* Wm = reinterpret_cast<float2*>(gb + L.Wm);
+  float2* cpartA = reinterpret_cast<float2*>(gb + L.cpartA);
   float2* cpartB = reinterpret_cast<float2*>(gb + L.cpartB);
-  float2* cpartD = reinterpret_cast<float2*>(gb + L.cpartD);
   float2* npart = reinterpret_cast<float2*>(gb + L.npart);
+  float2* sqpart = reinterpret_cast<float2*>(gb + L.sqpart);
   const GroupBarrier bar{barw, barw + 32, (unsigned)g};
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(&rg.full[s], 1);
-      mbar_init(&rg.empty[s], LZ_CW);
+      mbar_init(&fullb[s], 1);
+      mbar_init(&emptyb[s], LZ_CW);
     }
     mbar_fence_init();
     s_halt = 0;
     s_go = 0;
     s_pdone = 0;
+    s_bdone = 0;
     s_issued = 0;
   }
   __syncthreads();
@@ -338,15 +329,15 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     unsigned cnt = 0;
     int pp = 0;
     for (int p = gi; p < nprob; p += ngroups, ++pp) {
-      bool go = false;
+      bool ok = false;
       for (unsigned it = 0; it < (1u << 26); ++it) {
         if (s_go == pp + 1) {
-          go = true;
+          ok = true;
           break;
         }
         __nanosleep(64);
       }
-      if (!go) {
+      if (!ok) {
         atomicExch(status, SLS_ERR_TIMEOUT);
         break;
       }
@@ -355,9 +346,27 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
       const int nch = (int)((re - rs + cr - 1) / cr);
       const float* Phi = bt.Phi + (row0 + rs) * D;
+      const float2* Qs = bt.Q + (row0 + rs) * ldq;
       bool stop = false;
       for (int j = 0; j < r && !stop; ++j) {
         for (int sweep = 0; sweep < 2 && !stop; ++sweep) {
+          if (sweep == 0 && j > 0) {
+            // sweep A of step j reads basis column j-1, written in sweep B of j-1
+            bool seen = false;
+            for (unsigned it = 0; it < (1u << 26); ++it) {
+              if (s_halt) break;
+              if (s_bdone == pp * 256 + j) {
+                seen = true;
+                break;
+              }
+              __nanosleep(32);
+            }
+            if (!seen) {
+              if (!s_halt) atomicExch(status, SLS_ERR_TIMEOUT);
+              stop = true;
+              break;
+            }
+          }
           for (int t = 0; t < nch; ++t) {
             if (s_halt) {
               stop = true;
@@ -366,16 +375,17 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
             const int k = (sweep == 0) ? t : nch - 1 - t;
             const int slot = (int)(cnt % (unsigned)S);
             const unsigned par = (cnt / (unsigned)S) & 1u;
-            if (!mbar_wait(&rg.empty[slot], par ^ 1u)) {
+            if (!mbar_wait(&emptyb[slot], par ^ 1u)) {
               atomicExch(status, SLS_ERR_TIMEOUT);
               stop = true;
               break;
             }
             const int64_t nr = min((int64_t)cr, (re - rs) - (int64_t)k * cr);
-            const unsigned bytes = (unsigned)(nr * D * 4);
-            mbar_expect_tx(&rg.full[slot], bytes);
-            bulk_g2s(rg.ring + (size_t)slot * (rg.shp.chunk / 4), Phi + (int64_t)k * cr * D,
-                     bytes, &rg.full[slot], pol);
+            const unsigned b1 = (unsigned)(nr * D * 4), b2 = (unsigned)(nr * ldq * 8);
+            unsigned char* dst = ring + (size_t)slot * stage;
+            mbar_expect_tx(&fullb[slot], b1 + b2);
+            bulk_g2s(dst, Phi + (int64_t)k * cr * D, b1, &fullb[slot], pol);
+            bulk_g2s(dst + phib, Qs + (int64_t)k * cr * ldq, b2, &fullb[slot], pol);
             ++cnt;
             __threadfence_block();
             s_issued = cnt;
@@ -388,7 +398,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     }
     // every copy issued has landed before the CTA may exit
     for (unsigned c = (cnt > (unsigned)S ? cnt - S : 0); c < cnt; ++c)
-      mbar_wait(&rg.full[c % S], (c / S) & 1u);
+      mbar_wait(&fullb[c % S], (c / S) & 1u);
     return;
   }
 
@@ -405,7 +415,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
     const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
     const int64_t q1o = bt.q1off ? bt.q1off[p] : row0;
-    float2* Q = bt.Q + row0 * r;
+    float2* Q = bt.Q + row0 * ldq;
     const double* q1 = bt.q1 + q1o;
     const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
     const int nrows = (int)(re - rs);
@@ -417,60 +427,55 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     double scale = 0.0, alpha_prev = 0.0;
     dfloat alpha_df = df_make(0.f, 0.f), beta_df = df_make(0.f, 0.f), invb_df;
     int reff = 0;
+    sbreak = 0;
 
     for (int j = 0; j < r; ++j) {
-      // ---------------- phase A: u_j, stored as column j of Q ----------------
-      dfloat nacc = df_make(0.f, 0.f);
-      for (int64_t i0 = rs + (int64_t)warp * RPW; i0 < re; i0 += (int64_t)LZ_CW * RPW) {
-        const int nb = (int)min((int64_t)RPW, re - i0);
-        dfloat u[RPW];
-        if (j == 0) {
-          dfloat mine = df_make(0.f, 0.f);
-          if (lane < nb) mine = df_from_double(q1[i0 + lane]);
-#pragma unroll
-          for (int b = 0; b < RPW; ++b) u[b] = shfl_df(mine, b);
-        } else {
-          float2 q[RPW][KT_MAX], zv[RPW];
-          load_rows(Q, r, i0, nb, j, z1, q, zv);
-          float corr[RPW];
-          row_corrections(q, j, cs, corr);
-#pragma unroll
-          for (int b = 0; b < RPW; ++b) u[b] = df_add(dfv(zv[b]), df_make(-corr[b], 0.f));
-        }
-        if (lane == 0) {
-#pragma unroll
-          for (int b = 0; b < RPW; ++b) {
-            if (b < nb) {
-              Q[(i0 + b) * r + j] = f2(u[b]);
-              us[i0 + b - rs] = f2(u[b]);
-              dot2_acc_df(nacc.hi, nacc.lo, u[b], u[b]);
-            }
-          }
-        }
-      }
-      if (lane == 0) tmpw[warp] = f2(df_norm(nacc.hi, nacc.lo));
-      named_sync(BAR_COMPUTE, LZ_CT);
-      if (tid == 0) {
-        dfloat s = df_make(0.f, 0.f);
-        for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(tmpw[w]));
-        npart[rank] = f2(s);
-      }
-      // ---------------- sweep A: Phi^T u over the strip (forward) --------------
+      // ---------------- sweep A (forward): z1 = z' - Q c, then Phi^T z1 --------
       {
         f32x2_t ah[GPT][2], al[GPT][2];
 #pragma unroll
         for (int q = 0; q < GPT; ++q) ah[q][0] = ah[q][1] = al[q][0] = al[q][1] = 0ull;
+        dfloat c2acc[KT_MAX];
+#pragma unroll
+        for (int t = 0; t < KT_MAX; ++t) c2acc[t] = df_make(0.f, 0.f);
+        dfloat nacc = df_make(0.f, 0.f);
         for (int t = 0; t < nch; ++t) {
           const int slot = (int)(ccnt % (unsigned)S);
-          if (!mbar_wait(&rg.full[slot], (ccnt / (unsigned)S) & 1u))
+          if (!mbar_wait(&fullb[slot], (ccnt / (unsigned)S) & 1u))
             atomicExch(status, SLS_ERR_TIMEOUT);  // leave at the next group barrier
+          const unsigned char* stg = ring + (size_t)slot * stage;
+          const float* chunk = reinterpret_cast<const float*>(stg);
+          const float2* qblk = reinterpret_cast<const float2*>(stg + phib);
           const int nr = min(cr, nrows - t * cr);
-          sweepA_chunk<GPT>(rg.ring + (size_t)slot * (rg.shp.chunk / 4), nr, D, t * cr, us, ah,
-                            al);
+          for (int ii = warp; ii < nr; ii += LZ_CW) {
+            const int il = t * cr + ii;
+            dfloat z;
+            if (j == 0) {
+              z = df_make(0.f, 0.f);
+              if (lane == 0) z = df_from_double(q1[rs + il]);
+              z = shfl_df(z, 0);
+            } else {
+              const float2* qrow = qblk + (size_t)ii * ldq;
+              const float corr = row_correction(qrow, cs, j);
+              z = df_add(dfv(zps[il]), df_make(-corr, 0.f));
+#pragma unroll
+              for (int tt = 0; tt < KT_MAX; ++tt) {
+                const int k = lane + 32 * tt;
+                if (k < j) dot2_acc_df(c2acc[tt].hi, c2acc[tt].lo, dfv(qrow[k]), z);
+              }
+            }
+            if (lane == 0) {
+              us[il] = f2(z);
+              dot2_acc_df(nacc.hi, nacc.lo, z, z);
+            }
+          }
+          named_sync(BAR_COMPUTE, LZ_CT);
+          sweepA_chunk<GPT>(chunk, nr, D, t * cr, us, ah, al);
           __syncwarp();
-          if (lane == 0) mbar_arrive(&rg.empty[slot]);
+          if (lane == 0) mbar_arrive(&emptyb[slot]);
           ++ccnt;
         }
+        // CTA partials: Phi^T z1, c2, |z1|^2
         const int ph = (P == 1) ? 0 : tid / C4;
         const int cb = (P == 1) ? tid : tid % C4;
         float2* dst = (P == 1) ? wpart + (size_t)rank * D : red + (size_t)ph * D;
@@ -499,56 +504,83 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
             wpart[(size_t)rank * D + col] = f2(s);
           }
         }
-      }
-      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
-
-      // slice reduction of w over the group's CTAs
-      for (int c = cbeg + warp; c < cend; c += LZ_CW) {
-        dfloat s = df_make(0.f, 0.f);
-        for (int b = lane; b < g; b += 32) s = df_add(s, dfv(wpart[(size_t)b * D + c]));
-        s = warp_sum_df(s);
-        if (lane == 0) wred[c] = f2(s);
-      }
-      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
-
-      // |u_j|^2, |w_red|^2 and the break test
-      if (warp == 0) {
-        dfloat s = df_make(0.f, 0.f);
-        for (int b = lane; b < g; b += 32) s = df_add(s, dfv(npart[b]));
-        s = warp_sum_df(s);
-        if (lane == 0) shd[0] = df_to_double(s);
-      }
-      dfloat sq = df_make(0.f, 0.f);
-      for (int c = tid; c < D; c += LZ_CT) {
-        const float2 v = wred[c];
-        dot2_acc_df(sq.hi, sq.lo, dfv(v), dfv(v));
-      }
-      {
-        sq = warp_sum_df(df_norm(sq.hi, sq.lo));
-        named_sync(BAR_COMPUTE, LZ_CT);
-        if (lane == 0) tmpw[warp] = f2(sq);
-        named_sync(BAR_COMPUTE, LZ_CT);
-        sq = df_make(0.f, 0.f);
-        for (int w = 0; w < LZ_CW; ++w) sq = df_add(sq, dfv(tmpw[w]));
-      }
-      if (tid == 0) {
-        const double nrm2 = shd[0];
-        const double bnew = sqrt(nrm2);
-        int brk = 0;
-        if (j > 0) {
-          scale = fmax(scale, fabs(alpha_prev) + bnew);
-          if (!(bnew > bt.tol * scale)) brk = 1;
-          else if (rank == 0) beta_out[j - 1] = bnew;
-        } else if (!(bnew > 0.0)) {
-          brk = 1;
+        if (lane == 0) tmpw[warp] = f2(df_norm(nacc.hi, nacc.lo));
+        store_coeff_partials(c2acc, j, r, cw, cpartA + (size_t)rank * (r + 1));
+        if (tid == 0) {
+          dfloat s = df_make(0.f, 0.f);
+          for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(tmpw[w]));
+          npart[rank] = f2(s);
         }
-        const double a = brk ? 0.0 : df_to_double(sq) / nrm2;
-        if (!brk && rank == 0) alpha_out[j] = a;
-        shd[1] = brk ? 0.0 : 1.0 / bnew;
-        shd[2] = a;
-        shd[3] = (j > 0) ? bnew : 0.0;
-        sbreak = brk;
-        if (brk) s_halt = 1;
+      }
+      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
+
+      // ---------------- slice phase: c2, Phi^T u_j for this CTA's columns --------
+      reduce_coeffs(cpartA, g, r, j, c2s, red2);
+      {
+        dfloat sq = df_make(0.f, 0.f);
+        for (int c = cbeg + warp; c < cend; c += LZ_CW) {
+          dfloat s = df_make(0.f, 0.f);
+          for (int b = lane; b < g; b += 32) s = df_add(s, dfv(wpart[(size_t)b * D + c]));
+          s = warp_sum_df(s);
+          // - sum_k c2_k w_k[c]
+          dfloat cor = df_make(0.f, 0.f);
+#pragma unroll
+          for (int tt = 0; tt < KT_MAX; ++tt) {
+            const int k = lane + 32 * tt;
+            if (k < j) dot2_acc_df(cor.hi, cor.lo, dfv(Wm[(size_t)c * r + k]), dfv(c2s[k]));
+          }
+          cor = warp_sum_df(df_norm(cor.hi, cor.lo));
+          s = df_sub(s, cor);
+          if (lane == 0) {
+            wred[c] = f2(s);
+            dot2_acc_df(sq.hi, sq.lo, s, s);
+          }
+        }
+        if (lane == 0) tmpw[warp] = f2(df_norm(sq.hi, sq.lo));
+        named_sync(BAR_COMPUTE, LZ_CT);
+        if (tid == 0) {
+          dfloat s = df_make(0.f, 0.f);
+          for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(tmpw[w]));
+          sqpart[rank] = f2(s);
+        }
+      }
+      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
+
+      // ---------------- beta_{j-1}, alpha_j, break test -------------------------
+      if (warp == 0) {
+        dfloat s = df_make(0.f, 0.f), q = df_make(0.f, 0.f);
+        for (int b = lane; b < g; b += 32) {
+          s = df_add(s, dfv(npart[b]));
+          q = df_add(q, dfv(sqpart[b]));
+        }
+        s = warp_sum_df(s);
+        q = warp_sum_df(q);
+        dfloat c2n = df_make(0.f, 0.f);
+#pragma unroll
+        for (int tt = 0; tt < KT_MAX; ++tt) {
+          const int k = lane + 32 * tt;
+          if (k < j) dot2_acc_df(c2n.hi, c2n.lo, dfv(c2s[k]), dfv(c2s[k]));
+        }
+        c2n = warp_sum_df(df_norm(c2n.hi, c2n.lo));
+        if (lane == 0) {
+          const double nrm2 = df_to_double(s) - df_to_double(c2n);  // |u_j|^2
+          const double bnew = sqrt(fmax(nrm2, 0.0));
+          int brk = 0;
+          if (j > 0) {
+            scale = fmax(scale, fabs(alpha_prev) + bnew);
+            if (!(bnew > bt.tol * scale)) brk = 1;
+            else if (rank == 0) beta_out[j - 1] = bnew;
+          } else if (!(bnew > 0.0)) {
+            brk = 1;
+          }
+          const double a = brk ? 0.0 : df_to_double(q) / (bnew * bnew);
+          if (!brk && rank == 0) alpha_out[j] = a;
+          shd[1] = brk ? 0.0 : 1.0 / bnew;
+          shd[2] = a;
+          shd[3] = (j > 0) ? bnew : 0.0;
+          sbreak = brk;
+          if (brk) s_halt = 1;
+        }
       }
       named_sync(BAR_COMPUTE, LZ_CT);
       if (sbreak) {
@@ -559,98 +591,73 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       alpha_prev = shd[2];
       alpha_df = df_from_double(shd[2]);
       beta_df = df_from_double(shd[3]);
-      // w = w_red / beta into shared memory as {wh_e, wh_o, wl_e, wl_o} pairs
-      for (int c2 = tid; c2 < D / 2; c2 += LZ_CT) {
-        const dfloat a = df_mul(dfv(wred[2 * c2]), invb_df);
-        const dfloat b = df_mul(dfv(wred[2 * c2 + 1]), invb_df);
-        wq[c2] = make_float4(a.hi, b.hi, a.lo, b.lo);
+      // w_j = (Phi^T u_j) / beta into shared memory; keep w_j (slice) for the
+      // second Gram-Schmidt correction of later steps
+      for (int c = tid; c < D; c += LZ_CT) {
+        const dfloat a = df_mul(dfv(wred[c]), invb_df);
+        wsh[c] = a.hi;
+        wsl[c] = a.lo;
+        if (c >= cbeg && c < cend) Wm[(size_t)c * r + j] = f2(a);
       }
       named_sync(BAR_COMPUTE, LZ_CT);
 
-      // ---------------- sweep B (backward): z' = A q_j - alpha q_j - beta q_{j-1}
+      // ---------------- sweep B (backward): q_j, z' and c ------------------------
       const bool last = (j == r - 1);
-      dfloat cacc[(SLS_MAX_R + 1 + 31) / 32];
+      dfloat cacc[KT_MAX];
 #pragma unroll
-      for (int t = 0; t < (SLS_MAX_R + 1 + 31) / 32; ++t) cacc[t] = df_make(0.f, 0.f);
+      for (int t = 0; t < KT_MAX; ++t) cacc[t] = df_make(0.f, 0.f);
       for (int t = 0; t < nch; ++t) {
-        const int k = nch - 1 - t;
+        const int kc = nch - 1 - t;
         const int slot = (int)(ccnt % (unsigned)S);
-        if (!mbar_wait(&rg.full[slot], (ccnt / (unsigned)S) & 1u))
+        if (!mbar_wait(&fullb[slot], (ccnt / (unsigned)S) & 1u))
           atomicExch(status, SLS_ERR_TIMEOUT);  // leave at the next group barrier
-        const float* chunk = rg.ring + (size_t)slot * (rg.shp.chunk / 4);
-        const int nr = min(cr, nrows - k * cr);
+        const unsigned char* stg = ring + (size_t)slot * stage;
+        const float* chunk = reinterpret_cast<const float*>(stg);
+        const float2* qblk = reinterpret_cast<const float2*>(stg + phib);
+        const int nr = min(cr, nrows - kc * cr);
         for (int ii = warp; ii < nr; ii += LZ_CW) {
-          const int64_t i = rs + (int64_t)k * cr + ii;
-          const float2* Qi = Q + i * r;
-          float2 qv[KT_MAX];
-#pragma unroll
-          for (int tt = 0; tt < KT_MAX; ++tt) {
-            const int kk = lane + 32 * tt;
-            qv[tt] = (kk <= j) ? Qi[kk] : make_float2(0.f, 0.f);
-          }
-          const dfloat s = row_dot_smem(chunk + (size_t)ii * D, D, wq);
-          float2 sel_j = make_float2(0.f, 0.f), sel_jm1 = make_float2(0.f, 0.f);
-#pragma unroll
-          for (int tt = 0; tt < KT_MAX; ++tt) {
-            if (tt == (j >> 5)) sel_j = qv[tt];
-            if (j > 0 && tt == ((j - 1) >> 5)) sel_jm1 = qv[tt];
-          }
-          const dfloat uj = shfl_df(dfv(sel_j), j & 31);
-          const dfloat qj = df_mul(uj, invb_df);
+          const int il = kc * cr + ii;
+          const int64_t i = rs + il;
+          const float2* qrow = qblk + (size_t)ii * ldq;
+          dfloat u = dfv(us[il]);
+          if (j > 0) u = df_add(u, df_make(-row_correction(qrow, c2s, j), 0.f));
+          const dfloat qj = df_mul(u, invb_df);
+          const dfloat s = row_dot_smem(chunk + (size_t)ii * D, D, wsh, wsl);
           dfloat zp = df_sub(s, df_mul(alpha_df, qj));
-          if (j > 0) zp = df_sub(zp, df_mul(beta_df, shfl_df(dfv(sel_jm1), (j - 1) & 31)));
+          if (j > 0) zp = df_sub(zp, df_mul(beta_df, dfv(qrow[j - 1])));
           if (lane == 0) {
-            Q[i * r + j] = f2(qj);
-            z0[i] = f2(zp);
+            Q[i * ldq + j] = f2(qj);
+            zps[il] = f2(zp);
           }
           if (!last) {
 #pragma unroll
             for (int tt = 0; tt < KT_MAX; ++tt) {
-              const int kk = lane + 32 * tt;
-              if (kk <= j) {
-                const dfloat qk = (kk == j) ? qj : dfv(qv[tt]);
+              const int k = lane + 32 * tt;
+              if (k <= j) {
+                const dfloat qk = (k == j) ? qj : dfv(qrow[k]);
                 dot2_acc_df(cacc[tt].hi, cacc[tt].lo, qk, zp);
               }
             }
           }
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&rg.empty[slot]);
+        if (lane == 0) mbar_arrive(&emptyb[slot]);
         ++ccnt;
       }
       if (last) {
         reff = r;
         break;
       }
-      store_coeff_partials(cacc, j, r, cw, cpartB + (size_t)rank * (r + 1));
-      if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
-      reduce_coeffs(cpartB, g, r, j, cs, red2);
-
-      // ---------------- phase D: z1 = z' - Q c, c2 = Q^T z1 ----------------------
-#pragma unroll
-      for (int t = 0; t < KT_MAX; ++t) cacc[t] = df_make(0.f, 0.f);
-      for (int64_t i0 = rs + (int64_t)warp * RPW; i0 < re; i0 += (int64_t)LZ_CW * RPW) {
-        const int nb = (int)min((int64_t)RPW, re - i0);
-        float2 q[RPW][KT_MAX], zv[RPW];
-        load_rows(Q, r, i0, nb, j + 1, z0, q, zv);
-        float corr[RPW];
-        row_corrections(q, j + 1, cs, corr);
-#pragma unroll
-        for (int b = 0; b < RPW; ++b) {
-          if (b < nb) {
-            const dfloat zz = df_add(dfv(zv[b]), df_make(-corr[b], 0.f));
-            if (lane == 0) z1[i0 + b] = f2(zz);
-#pragma unroll
-            for (int t = 0; t < KT_MAX; ++t) {
-              const int k = lane + 32 * t;
-              if (k <= j) dot2_acc_df(cacc[t].hi, cacc[t].lo, dfv(q[b][t]), zz);
-            }
-          }
-        }
+      // basis column j reaches the copy warp's bulk reads (async proxy)
+      if (lane == 0) asm volatile("fence.proxy.async.global;" ::: "memory");
+      named_sync(BAR_COMPUTE, LZ_CT);
+      if (tid == 0) {
+        __threadfence_block();
+        s_bdone = pp * 256 + j + 1;
       }
-      store_coeff_partials(cacc, j, r, cw, cpartD + (size_t)rank * (r + 1));
+      store_coeff_partials(cacc, j + 1, r, cw, cpartB + (size_t)rank * (r + 1));
       if (!group_sync_named(bar, lgen, status, &sflag, BAR_COMPUTE, LZ_CT)) return;
-      reduce_coeffs(cpartD, g, r, j, cs, red2);
+      reduce_coeffs(cpartB, g, r, j + 1, cs, red2);
     }
     // a break leaves chunks issued ahead of it: consume them until the copy
     // warp reports that it stopped
@@ -659,12 +666,12 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         const unsigned iss = s_issued;
         if (ccnt < iss) {
           const int slot = (int)(ccnt % (unsigned)S);
-          if (!mbar_wait(&rg.full[slot], (ccnt / (unsigned)S) & 1u)) {
+          if (!mbar_wait(&fullb[slot], (ccnt / (unsigned)S) & 1u)) {
             atomicExch(status, SLS_ERR_TIMEOUT);
             break;
           }
           __syncwarp();
-          if (lane == 0) mbar_arrive(&rg.empty[slot]);
+          if (lane == 0) mbar_arrive(&emptyb[slot]);
           ++ccnt;
         } else if (s_pdone == pp + 1) {
           if (s_issued == ccnt) break;
@@ -923,7 +930,7 @@ ritz_vectors_kernel(LanczosBatch bt, float* __restrict__ U) {
   const int sub = threadIdx.x / r, m = threadIdx.x % r;
   if (sub >= rpb) return;
   for (int64_t i = (int64_t)blockIdx.x * rpb + sub; i < n; i += (int64_t)gridDim.x * rpb) {
-    const float2* Qi = bt.Q + (row0 + i) * r;
+    const float2* Qi = bt.Q + (row0 + i) * q_ld(r);
     float acc = 0.f;
     for (int k = 0; k < kn; ++k) {
       const float2 q = Qi[k];
@@ -1007,13 +1014,17 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
   const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
   const int redn = (P > 1) ? P * bt.D : 0;
   const int rows_cap = (int)((bt.nmax + g - 1) / g) + 1;
-  const size_t other = sizeof(float2) * ((size_t)bt.D + redn + rows_cap +
-                                         (size_t)(LZ_CW + 1) * (bt.r + 1) + 2 * LZ_CT) + 16;
+  // shared memory besides the ring: w (hi, lo), phase partials, z1 and z' of
+  // the strip, coefficient partials and vectors, reduction scratch, barriers
+  const size_t other = sizeof(float) * 2 * (size_t)bt.D +
+                       sizeof(float2) * ((size_t)redn + 2 * (size_t)rows_cap +
+                                         (size_t)(LZ_CW + 2) * (bt.r + 1) + 4 * LZ_CT) +
+                       16 + 2 * 6 * 8;
   const size_t limit = 227 * 1024 - 1024;  // leave room for static shared memory
-  if (other + 2 * 16 * 8 >= limit) return SLS_ERR_UNSUPPORTED;
-  RingShape R = ring_shape(bt.D, limit - other - 2 * 6 * 8);
+  if (other >= limit) return SLS_ERR_UNSUPPORTED;
+  RingShape R = ring_shape(bt.D, q_ld(bt.r), limit - other);
   if (R.S < 2) return SLS_ERR_UNSUPPORTED;
-  const size_t smem = (size_t)R.S * R.chunk + other + 2 * (size_t)R.S * 8;
+  const size_t smem = (size_t)R.S * R.stage + other;
   const int stages = R.S;
   const int gpt = (C4 + LZ_CT - 1) / LZ_CT;
   if (gpt <= 1) return launch_lanczos_t<1>(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream);
