@@ -208,6 +208,32 @@ SLS_DEV void dot2_acc2(f32x2_t& sh, f32x2_t& sl, f32x2_t x, f32x2_t yh, f32x2_t 
   sl = add2(sl, add2(e, pe));
 }
 
+// Offset accumulation step on two lanes: (s, lo) += x * (yh + yl), nyh = -yh.
+// s carries a power-of-two offset C and every partial sum it accumulates is
+// at most C/2 in magnitude, so s stays in [C/2, 3C/2] and s + p (|p| <= C/2)
+// is an exact FastTwoSum (Dekker's condition: exponent of s >= exponent of
+// p).  8 operations per element instead of Dot2's 10; the value is
+// (s - C) + lo, and s - C is exact (Sterbenz).
+SLS_DEV void ofs_acc2n(f32x2_t& s, f32x2_t& lo, f32x2_t x, f32x2_t yh, f32x2_t nyh,
+                       f32x2_t yl) {
+  const f32x2_t np = mul2(x, nyh);            // -p, p = fl(x * yh)
+  f32x2_t e = fma2(x, yh, np);                // x * yh - p, exact
+  e = fma2(x, yl, e);
+  const f32x2_t s1 = sub2(s, np);             // fl(s + p)
+  const f32x2_t fn = add2(np, sub2(s1, s));   // minus the rounding error of s + p
+  s = s1;
+  lo = add2(lo, sub2(e, fn));
+}
+
+// The offset for a bound B on all partial sums: a power of two C > 2 B (with
+// a little slack for the rounding of B itself), clamped to [2^-100, 2^126].
+SLS_DEV float ofs_pow2(float bound) {
+  const float x = 2.f * bound * 1.00390625f;
+  if (!(x >= 0x1p-100f)) return 0x1p-100f;
+  if (x >= 0x1p125f) return 0x1p126f;
+  return __int_as_float((__float_as_int(x) & 0x7f800000) + 0x00800000);
+}
+
 // ---------------------------------------------------------------------------
 // shared-memory barriers, bulk copies and named barriers
 // ---------------------------------------------------------------------------
