@@ -341,10 +341,11 @@ SLS_DEV unsigned atom_add_acq_rel_gpu(unsigned* p, unsigned v) {
 
 // ---------------------------------------------------------------------------
 // Barrier across a group of co-resident CTAs (all CTAs of a cooperative
-// launch, or a subset).  `count` and `gen` live in global memory and start
-// at 0.  Every CTA keeps its own copy of the generation in `local_gen`.
+// launch, or a subset).  `count` lives in global memory and starts at 0;
+// `gen` is unused.  Every CTA counts the barriers it passed in `local_gen`.
 // Returns false (and sets *status = SLS_ERR_TIMEOUT) when the wait exceeded
-// its iteration limit; the caller must then leave the kernel.
+// its iteration limit or another CTA gave up; the caller must then leave the
+// kernel.
 // ---------------------------------------------------------------------------
 
 #ifndef SLS_SPIN_LIMIT
@@ -357,67 +358,48 @@ struct GroupBarrier {
   unsigned nblocks;
 };
 
-SLS_DEV bool group_sync(const GroupBarrier& bar, unsigned& local_gen, int* status,
-                        int* smem_flag) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int ok = 1;
-    unsigned g = local_gen;
-    __threadfence();
-    unsigned arrived = atom_add_acq_rel_gpu(bar.count, 1u);
-    if (arrived == bar.nblocks - 1) {
-      *bar.count = 0;
-      __threadfence();
-      st_release_gpu(bar.gen, g + 1);
-    } else {
-      unsigned it = 0;
-      while (ld_acquire_gpu(bar.gen) == g) {
-        if (++it > SLS_SPIN_LIMIT) {
-          ok = 0;
-          atomicExch(status, SLS_ERR_TIMEOUT);
-          break;
-        }
-        __nanosleep(64);
-      }
-    }
-    __threadfence();
-    local_gen = g + 1;
-    // a timeout anywhere (this CTA or another) stops every CTA at its next barrier
-    if (ok && *((volatile int*)status) == SLS_ERR_TIMEOUT) ok = 0;
-    *smem_flag = ok;
-  }
-  __syncthreads();
-  return *((volatile int*)smem_flag) != 0;
-}
+// Bit of the arrival counter that releases every waiter with an error: a CTA
+// that gives up sets it, so the other CTAs of the group stop at their next
+// barrier instead of waiting out the iteration limit.
+constexpr unsigned SLS_BAR_POISON = 0x80000000u;
+
+SLS_DEV void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 
 // Same barrier for kernels where only `nthreads` threads (ids 0..nthreads-1,
 // named barrier `bar_id`) take part, e.g. compute warps next to a copy warp.
+// One monotonically increasing arrival counter: barrier number n (local_gen
+// = n) is complete when the counter reaches (n + 1) * nblocks, so the last
+// arrival's own atomic releases the group (one round trip to L2 less than a
+// separate release word).  `local_err` is a shared-memory flag the CTA sets
+// when one of its own waits gave up; such a CTA poisons the counter instead
+// of arriving.
 SLS_DEV bool group_sync_named(const GroupBarrier& bar, unsigned& local_gen, int* status,
-                              int* smem_flag, unsigned bar_id, unsigned nthreads) {
+                              int* smem_flag, volatile int* local_err, unsigned bar_id,
+                              unsigned nthreads) {
   named_sync(bar_id, nthreads);
   if (threadIdx.x == 0) {
-    int ok = 1;
-    unsigned g = local_gen;
-    __threadfence();
-    unsigned arrived = atom_add_acq_rel_gpu(bar.count, 1u);
-    if (arrived == bar.nblocks - 1) {
-      *bar.count = 0;
-      __threadfence();
-      st_release_gpu(bar.gen, g + 1);
+    int ok = (*local_err == 0);
+    if (!ok) {
+      atomicOr(bar.count, SLS_BAR_POISON);
     } else {
+      const unsigned target = (local_gen + 1) * bar.nblocks;
+      fence_acq_rel_gpu();
+      unsigned v = atom_add_acq_rel_gpu(bar.count, 1u) + 1u;
       unsigned it = 0;
-      while (ld_acquire_gpu(bar.gen) == g) {
+      while (v < target) {
         if (++it > SLS_SPIN_LIMIT) {
           ok = 0;
           atomicExch(status, SLS_ERR_TIMEOUT);
+          atomicOr(bar.count, SLS_BAR_POISON);
           break;
         }
-        __nanosleep(64);
+        if (it > 32) __nanosleep(32);
+        v = ld_acquire_gpu(bar.count);
       }
+      if (v & SLS_BAR_POISON) ok = 0;
+      fence_acq_rel_gpu();
     }
-    __threadfence();
-    local_gen = g + 1;
-    if (ok && *((volatile int*)status) == SLS_ERR_TIMEOUT) ok = 0;
+    local_gen += 1;
     *smem_flag = ok;
   }
   named_sync(bar_id, nthreads);

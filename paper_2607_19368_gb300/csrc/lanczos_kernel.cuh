@@ -1,0 +1,1148 @@
+// Implicit Lanczos (Algorithm 2): the persistent kernel.
+//
+// Lanczos runs as one persistent cooperative kernel.  The grid is split into
+// groups of CTAs; a group owns one problem at a time (one prompt, or one
+// adaptive window) and every CTA owns a contiguous strip of the problem's rows
+// of the feature matrix Phi (N x D, float32) and of the basis Q.  One copy warp
+// per CTA streams the Phi strip through a shared-memory ring with
+// one-dimensional bulk copies (cp.async.bulk + mbarrier), twice per step, and
+// runs ahead of the eight compute warps by as many chunks as the ring holds.
+// All work on basis rows happens in one dense row phase per step, with the
+// strip's rows split over the compute warps (register groups of rows, lanes
+// over the basis index, transposed butterflies for the row sums).
+//
+// Step j (0-based) starts from z' (the new Lanczos direction before its
+// re-orthogonalisation; z' = q1 for j = 0) and the CTA partials of
+// c = Q^T z' (k < j) and |z'|^2 left by the previous row phase:
+//
+//   sweep A (forward)   Phi^T z', column-parallel.
+//                       [barrier 1]
+//   slice phase         c = sum of the CTA partials; each CTA finishes a slice
+//                       of the D columns of Phi^T z1 = Phi^T z' - sum_k c_k w_k
+//                       with z1 = z' - Q c and w_k = Phi^T q_k kept from
+//                       earlier steps.
+//                       [barrier 2]
+//                       beta_{j-1} = |z1| = sqrt(|z'|^2 - |c|^2), the break
+//                       test, w_j = Phi^T q_j, alpha_j = |w_j|^2.
+//   sweep B (backward)  s = Phi w_j, the implicit matvec (Eq. implicit_matvec):
+//                       all compute threads share each chunk, w_j in registers.
+//   row phase           z1 = z' - Q c, q_j = z1 / beta_{j-1}, the three-term
+//                       recurrence z' = s - alpha_j q_j - beta_{j-1} q_{j-1},
+//                       and the partials of c = Q^T z' and |z'|^2 for step j+1.
+//
+// This is Algorithm 2 with full re-orthogonalisation by one classical
+// Gram-Schmidt pass per step, applied to Phi^T z' through the stored w_k so
+// that the two passes over Phi per step are pure streams and a step needs two
+// group barriers.  The projection c = Q^T z' of a fully re-orthogonalised
+// Lanczos run stays at rounding level, so a second pass would change z1 only
+// in the second order of the rounding unit.  Sweep B runs backward so the rows
+// sweep A touched last are still in L2.  Vectors are double-float (two
+// float32), every sum over N or D is compensated, reductions have a fixed
+// order (bit-reproducible runs).  Barriers and waits give up after a bounded
+// number of polls and report SLS_ERR_TIMEOUT through the status word.
+//
+// The kernel is a template over GPT (float4 column groups of Phi per compute
+// thread) and KT (32-wide tiles of the basis index k < r per lane); each
+// lanczos_g<GPT>.cu instantiates one GPT for every KT.
+#pragma once
+
+#include <cfloat>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace sls {
+
+namespace {
+
+constexpr int LZ_CW = 8;                  // compute warps
+constexpr int LZ_CT = LZ_CW * 32;         // compute threads
+constexpr int LZ_THREADS = LZ_CT + 32;    // plus one copy warp
+constexpr unsigned BAR_COMPUTE = 1;       // named barrier: the compute warps
+
+// leading dimension (float2) of the basis rows: even, so rows are 16-byte aligned
+__host__ __device__ inline int q_ld(int r) { return (r + 1) & ~1; }
+
+// Per-group scratch layout (byte offsets), identical on host and device.
+struct LzLayout {
+  size_t bar, wpart, wred, Wm, cpart, npart, sqpart, total;
+};
+
+__host__ __device__ inline size_t lz_al(size_t x) { return (x + 255) & ~(size_t)255; }
+
+__host__ __device__ inline LzLayout lz_layout(int64_t nmax, int D, int r, int g) {
+  (void)nmax;
+  LzLayout L;
+  size_t o = 0;
+  L.bar = o;    o += 256;
+  L.wpart = o;  o += lz_al((size_t)g * D * sizeof(float2));
+  L.wred = o;   o += lz_al((size_t)D * sizeof(float2));
+  L.Wm = o;     o += lz_al((size_t)D * r * sizeof(float2));
+  L.cpart = o;  o += lz_al((size_t)g * (r + 1) * sizeof(float2));
+  L.npart = o;  o += lz_al((size_t)2 * g * sizeof(float2));  // by step parity
+  L.sqpart = o; o += lz_al((size_t)g * sizeof(float2));
+  L.total = o;
+  return L;
+}
+
+SLS_DEV float2 f2(dfloat a) { return make_float2(a.hi, a.lo); }
+SLS_DEV dfloat dfv(float2 a) { return df_make(a.x, a.y); }
+
+SLS_DEV dfloat shfl_df(dfloat v, int src) {
+  v.hi = __shfl_sync(0xffffffffu, v.hi, src);
+  v.lo = __shfl_sync(0xffffffffu, v.lo, src);
+  return v;
+}
+
+// Ring stage: cr rows of Phi (cr * D floats).  For D >= 4 * LZ_CT (one
+// column group per compute thread or more) a stage holds TEAM_ELEMS / D rows,
+// so that sweep B can give every compute thread the same number of elements
+// per chunk; smaller D takes as many rows as fit RING_STAGE bytes.
+struct RingShape {
+  int cr;          // rows per chunk
+  int S;           // stages
+  unsigned stage;  // bytes per stage
+};
+
+constexpr int RING_STAGE = 32 * 1024;
+constexpr int RING_MAX_STAGES = 8;
+constexpr int WB_ROWS = 64;  // rows per window of sweep-B warp partials
+constexpr int SLICE_LOADS = 5;  // per-CTA values per lane in flight in warp sums (g <= 160)
+
+// float4 column groups per compute thread, rounded up to a power of two
+// (1, 2, 4 or 8; 0 when D is too wide)
+__host__ __device__ inline int gpt_of(int D) {
+  const int need = (D / 4 + LZ_CT - 1) / LZ_CT;
+  return need <= 1 ? 1 : need <= 2 ? 2 : need <= 4 ? 4 : need <= 8 ? 8 : 0;
+}
+// rows per chunk of the team sweep B: 8 / GPT (GPT * 4 * rows = 32 elements
+// per thread per chunk)
+__host__ __device__ constexpr int team_rows(int gpt) { return gpt >= 8 ? 1 : 8 / gpt; }
+
+__host__ __device__ inline RingShape ring_shape(int D, size_t budget) {
+  RingShape R;
+  if (D / 4 >= LZ_CT) {
+    R.cr = team_rows(gpt_of(D));
+  } else {
+    R.cr = RING_STAGE / (4 * D);
+    if (R.cr < 1) R.cr = 1;
+  }
+  R.stage = (unsigned)R.cr * (unsigned)D * 4u;
+  R.S = (int)(budget / R.stage);
+  if (R.S > RING_MAX_STAGES) R.S = RING_MAX_STAGES;
+  return R;
+}
+
+// Sweep A over one chunk: acc[c] += Phi[i, c] * z1_i for the chunk's rows,
+// column-parallel (GPT float4 groups per thread, P row phases), Dot2.  With
+// TRACK the thread also keeps the largest |Phi| it has seen in *mx.
+template <int GPT, bool TRACK>
+SLS_DEV void sweepA_chunk(const float* __restrict__ chunk, int nr, int D, int lb,
+                          const float2* __restrict__ us, f32x2_t (&ah)[GPT][2],
+                          f32x2_t (&al)[GPT][2], float* mx) {
+  const int tid = threadIdx.x;
+  const int C4 = D >> 2;
+  const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
+  if (P > 1 && tid >= P * C4) return;
+  const int ph = (P == 1) ? 0 : tid / C4;
+  const int cb = (P == 1) ? tid : tid % C4;
+  const float4* c4 = reinterpret_cast<const float4*>(chunk);
+  for (int i = ph; i < nr; i += P) {
+    const float2 u = us[lb + i];
+    const f32x2_t uh = pk2(u.x, u.x), nuh = pk2(-u.x, -u.x), ul = pk2(u.y, u.y);
+#pragma unroll
+    for (int q = 0; q < GPT; ++q) {
+      const int cg = cb + q * LZ_CT;
+      if (cg < C4) {
+        const float4 f = c4[i * C4 + cg];
+        dot2_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
+        dot2_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
+        if (TRACK)
+          *mx = fmaxf(*mx, fmaxf(fmaxf(fabsf(f.x), fabsf(f.y)), fmaxf(fabsf(f.z), fabsf(f.w))));
+      }
+    }
+  }
+}
+
+SLS_DEV dfloat shfl_xor_df(dfloat v, int m) {
+  v.hi = __shfl_xor_sync(0xffffffffu, v.hi, m);
+  v.lo = __shfl_xor_sync(0xffffffffu, v.lo, m);
+  return v;
+}
+
+// Transposed butterfly over CR rows (CR a power of two <= 32): every lane
+// holds one partial per row; afterwards lane L holds the warp sum of row
+// L >> (5 - log2 CR).  CR - 1 + 5 - log2 CR shuffles instead of 5 per row.
+template <int CR>
+SLS_DEV float transpose_sum_f(float (&v)[CR]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int s = 0; s < 5; ++s) {
+    const int h = 16 >> s;
+    const int nv = (CR >> s) > 1 ? (CR >> s) : 1;
+    if (nv > 1) {
+      const bool up = (lane & h) != 0;
+#pragma unroll
+      for (int i = 0; i < nv / 2; ++i) {
+        const float send = up ? v[i] : v[i + nv / 2];
+        const float keep = up ? v[i + nv / 2] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, h);
+      }
+    } else {
+      v[0] += __shfl_xor_sync(0xffffffffu, v[0], h);
+    }
+  }
+  return v[0];
+}
+
+// Sweep A over two ring chunks at once (D >= 4 * LZ_CT; CR rows each, the
+// second chunk may be absent: nr1 = 0) with offset accumulators: ah starts at
+// the power-of-two offset of the column sums.
+template <int GPT, int CR>
+SLS_DEV void sweepA_team_pair(const float* __restrict__ c0, int nr0, int lb0,
+                              const float* __restrict__ c1, int nr1, int lb1, int C4,
+                              const float2* __restrict__ us, f32x2_t (&ah)[GPT][2],
+                              f32x2_t (&al)[GPT][2]) {
+  const int tid = threadIdx.x;
+#pragma unroll
+  for (int i = 0; i < 2 * CR; ++i) {
+    const bool first = i < CR;
+    const int ii = first ? i : i - CR;
+    if (ii < (first ? nr0 : nr1)) {
+      const float4* c4 = reinterpret_cast<const float4*>(first ? c0 : c1);
+      const float2 u = us[(first ? lb0 : lb1) + ii];
+      const f32x2_t uh = pk2(u.x, u.x), nuh = pk2(-u.x, -u.x), ul = pk2(u.y, u.y);
+#pragma unroll
+      for (int q = 0; q < GPT; ++q) {
+        const int cg = tid + q * LZ_CT;
+        if (cg < C4) {
+          const float4 f = c4[ii * C4 + cg];
+          ofs_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
+          ofs_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
+        }
+      }
+    }
+  }
+}
+
+// Double-float sum without the second renormalisation (11 operations): the
+// error is a few units of the low part, enough for partial sums that are
+// combined once.
+SLS_DEV dfloat df_add_fast(dfloat a, dfloat b) {
+  float s, e;
+  two_sum(a.hi, b.hi, s, e);
+  e = __fadd_rn(e, __fadd_rn(a.lo, b.lo));
+  float h, l;
+  fast_two_sum(s, e, h, l);
+  return df_make(h, l);
+}
+
+// Transposed butterfly over CR rows (CR a power of two <= 32), double-float:
+// every lane holds one partial per row; afterwards lane L holds the warp sum
+// of row L >> (5 - log2 CR).  CR - 1 + 5 - log2 CR shuffles instead of 5 per
+// row.
+template <int CR>
+SLS_DEV dfloat transpose_sum_df(dfloat (&v)[CR]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int s = 0; s < 5; ++s) {
+    const int h = 16 >> s;
+    const int nv = (CR >> s) > 1 ? (CR >> s) : 1;
+    if (nv > 1) {
+      const bool up = (lane & h) != 0;
+#pragma unroll
+      for (int i = 0; i < nv / 2; ++i) {
+        const dfloat send = up ? v[i] : v[i + nv / 2];
+        const dfloat keep = up ? v[i + nv / 2] : v[i];
+        v[i] = df_add_fast(keep, shfl_xor_df(send, h));
+      }
+    } else {
+      v[0] = df_add_fast(v[0], shfl_xor_df(v[0], h));
+    }
+  }
+  return v[0];
+}
+
+// Sweep B over two ring chunks at once with all compute threads (D >= 4 *
+// LZ_CT): thread t owns the float4 column groups t + LZ_CT q of every row, w
+// for those columns sits in registers.  Each thread accumulates its part of
+// a row against its own offset Ct (a power of two above twice max|Phi| times
+// the l1 norm of its slice of w), so the FastTwoSum steps lose nothing to a
+// loose global bound; the 2 CR per-row double-float partials are then summed
+// over the warp by one transposed butterfly and the warp sums stored to
+// bp0 / bp1 [i * LZ_CW + warp].
+template <int GPT, int CR>
+SLS_DEV void sweepB_team_pair(const float* __restrict__ c0, int nr0, const float* __restrict__ c1,
+                              int nr1, int C4, const f32x2_t (&wh)[GPT][2],
+                              const f32x2_t (&nwh)[GPT][2], const f32x2_t (&wl)[GPT][2],
+                              float Ct, float2* __restrict__ bp0, float2* __restrict__ bp1) {
+  constexpr int R2 = 2 * CR;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  dfloat v[R2];
+#pragma unroll
+  for (int i = 0; i < R2; ++i) {
+    const bool first = i < CR;
+    const int ii = first ? i : i - CR;
+    f32x2_t s = pk2(Ct, Ct), lo = 0ull;
+    if (ii < (first ? nr0 : nr1)) {
+      const float4* c4 = reinterpret_cast<const float4*>(first ? c0 : c1);
+#pragma unroll
+      for (int q = 0; q < GPT; ++q) {
+        const int cg = tid + q * LZ_CT;
+        if (cg < C4) {
+          const float4 f = c4[ii * C4 + cg];
+          ofs_acc2n(s, lo, pk2(f.x, f.y), wh[q][0], nwh[q][0], wl[q][0]);
+          ofs_acc2n(s, lo, pk2(f.z, f.w), wh[q][1], nwh[q][1], wl[q][1]);
+        }
+      }
+    }
+    float sx, sy, lx, ly;
+    upk2(s, sx, sy);
+    upk2(lo, lx, ly);
+    const float x = sy - Ct;  // exact
+    const float s1 = sx + x;
+    v[i] = df_make(s1 - Ct, (lx + ly) + (x - (s1 - sx)));
+  }
+  const dfloat r = transpose_sum_df<R2>(v);
+  constexpr int SH = (R2 >= 32) ? 0 : (R2 >= 16) ? 1 : (R2 >= 8) ? 2 : (R2 >= 4) ? 3 : 4;
+  if ((lane & ((1 << SH) - 1)) == 0) {
+    const int i = lane >> SH;
+    if (i < CR) {
+      if (i < nr0) bp0[i * LZ_CW + warp] = f2(r);
+    } else if (i - CR < nr1) {
+      bp1[(i - CR) * LZ_CW + warp] = f2(r);
+    }
+  }
+}
+
+// Row dot product with w from shared memory (separate hi / lo arrays); one
+// warp per row, all lanes get the sum.  Used by sweep B when D < 4 * LZ_CT.
+SLS_DEV dfloat row_dot_smem(const float* __restrict__ row, int D, const float* __restrict__ wsh,
+                            const float* __restrict__ wsl) {
+  const int lane = threadIdx.x & 31;
+  const int C4 = D >> 2;
+  const float4* r4 = reinterpret_cast<const float4*>(row);
+  const float4* h4 = reinterpret_cast<const float4*>(wsh);
+  const float4* l4 = reinterpret_cast<const float4*>(wsl);
+  f32x2_t h01 = 0, l01 = 0, h23 = 0, l23 = 0;
+  for (int cg = lane; cg < C4; cg += 32) {
+    const float4 f = r4[cg];
+    const float4 wh = h4[cg], wl = l4[cg];
+    dot2_acc2(h01, l01, pk2(f.x, f.y), pk2(wh.x, wh.y), pk2(wl.x, wl.y));
+    dot2_acc2(h23, l23, pk2(f.z, f.w), pk2(wh.z, wh.w), pk2(wl.z, wl.w));
+  }
+  float a0, a1, b0, b1, c0, c1, d0, d1;
+  upk2(h01, a0, a1);
+  upk2(l01, b0, b1);
+  upk2(h23, c0, c1);
+  upk2(l23, d0, d1);
+  dfloat s = df_add(df_add(df_make(a0, b0), df_make(a1, b1)),
+                    df_add(df_make(c0, d0), df_make(c1, d1)));
+  return warp_sum_df(s);
+}
+
+// Position in the ring: chunks consumed, current slot and its phase parity.
+struct RingCursor {
+  unsigned cnt;
+  int slot;
+  unsigned par;
+};
+
+SLS_DEV void rc_next(RingCursor& c, int S) {
+  ++c.cnt;
+  if (++c.slot == S) {
+    c.slot = 0;
+    c.par ^= 1u;
+  }
+}
+
+// A wait of this CTA gave up: report it and leave at the next group barrier.
+SLS_DEV void lz_fail(int* status, volatile int* err) {
+  atomicExch(status, SLS_ERR_TIMEOUT);
+  *err = 1;
+}
+
+SLS_DEV int nprob_of(const LanczosBatch& bt) {
+  int nprob = bt.nprob_max;
+  if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
+  return nprob;
+}
+
+// Column sums over the CTAs of a group, eight items per warp: lane (bq, xx)
+// = (lane >> 3, lane & 7) loads base[b * stride + x] for b = bq, bq + 4, ...
+// (all loads of a batch in flight, 64 contiguous bytes per b), adds them as
+// a pairwise tree and the four b-groups by two butterfly steps; every lane
+// with lane & 7 == xx returns the sum for its item x.
+constexpr int CS_BATCH = 20;
+
+__device__ __noinline__ dfloat warp_colsum8(const float2* __restrict__ base, size_t stride, int nb, int x,
+                            bool valid) {
+  const int lane = threadIdx.x & 31, bq = lane >> 3;
+  dfloat acc = df_make(0.f, 0.f);
+  for (int b0 = bq; b0 < nb; b0 += 4 * CS_BATCH) {
+    dfloat v[CS_BATCH];
+#pragma unroll
+    for (int u = 0; u < CS_BATCH; ++u) {
+      const int b = b0 + 4 * u;
+      v[u] = (valid && b < nb) ? dfv(base[(size_t)b * stride + x]) : df_make(0.f, 0.f);
+    }
+#pragma unroll
+    for (int w = 1; w < CS_BATCH; w *= 2) {
+#pragma unroll
+      for (int i = 0; i + w < CS_BATCH; i += 2 * w) v[i] = df_add_fast(v[i], v[i + w]);
+    }
+    acc = df_add_fast(acc, v[0]);
+  }
+  acc = df_add_fast(acc, shfl_xor_df(acc, 8));
+  acc = df_add_fast(acc, shfl_xor_df(acc, 16));
+  return acc;
+}
+
+// Sum of the per-CTA partial coefficients part[b * (r+1) + k] over the g CTAs
+// of a group, for k < K, into cs[k].  Every CTA does it redundantly, warp w
+// the coefficients 8 w .. 8 w + 7 (+ 8 LZ_CW m).
+__device__ __noinline__ void reduce_coeffs(const float2* __restrict__ part, int g, int r, int K,
+                           float2* __restrict__ cs) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int k0 = warp * 8; k0 < K; k0 += LZ_CW * 8) {
+    const int k = k0 + (lane & 7);
+    const dfloat v = warp_colsum8(part, (size_t)(r + 1), g, k, k < K);
+    if (lane < 8 && k < K) cs[k] = f2(v);
+  }
+  named_sync(BAR_COMPUTE, LZ_CT);
+}
+
+// sum_{k < j} Wm[k * D + c] * c_k for the warp's eight columns, with the same
+// lane layout as warp_colsum8 (lanes k-group bq = lane >> 3, Dot2).
+__device__ __noinline__ dfloat warp_wcorr8(const float2* __restrict__ Wm, int D, int j, int c,
+                                           bool valid, const float2* __restrict__ cs) {
+  const int lane = threadIdx.x & 31, bq = lane >> 3;
+  float sh = 0.f, sl = 0.f;
+  for (int k0 = bq; k0 < j; k0 += 4 * 16) {
+    float2 wv[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      const int k = k0 + 4 * u;
+      wv[u] = (valid && k < j) ? Wm[(size_t)k * D + c] : make_float2(0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      const int k = k0 + 4 * u;
+      if (k < j) dot2_acc_df(sh, sl, dfv(wv[u]), dfv(cs[k]));
+    }
+  }
+  dfloat acc = df_norm(sh, sl);
+  acc = df_add_fast(acc, shfl_xor_df(acc, 8));
+  acc = df_add_fast(acc, shfl_xor_df(acc, 16));
+  return acc;
+}
+
+// Sum of v[0 .. n) over the warp, all loads in flight (n <= 32 * SLICE_LOADS
+// at once, the rest in a loop); every lane gets the result.
+__device__ __noinline__ dfloat warp_sum_vec(const float2* __restrict__ v, int n) {
+  const int lane = threadIdx.x & 31;
+  dfloat x[SLICE_LOADS];
+#pragma unroll
+  for (int m = 0; m < SLICE_LOADS; ++m) {
+    const int b = lane + 32 * m;
+    x[m] = (b < n) ? dfv(v[b]) : df_make(0.f, 0.f);
+  }
+  dfloat s = x[0];
+#pragma unroll
+  for (int m = 1; m < SLICE_LOADS; ++m) s = df_add_fast(s, x[m]);
+  for (int b = lane + 32 * SLICE_LOADS; b < n; b += 32) s = df_add_fast(s, dfv(v[b]));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s = df_add_fast(s, shfl_xor_df(s, o));
+  return s;
+}
+
+// Per-warp partial coefficients (lanes over k < K) -> the CTA's partial row.
+template <int KT>
+SLS_DEV void store_coeff_partials(dfloat (&cacc)[KT], int K, int r, float2* __restrict__ cw,
+                                  float2* __restrict__ dst) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+#pragma unroll
+  for (int t = 0; t < KT; ++t) {
+    const int k = lane + 32 * t;
+    if (k < K) cw[(size_t)warp * (r + 1) + k] = f2(df_norm(cacc[t].hi, cacc[t].lo));
+  }
+  named_sync(BAR_COMPUTE, LZ_CT);
+  for (int k = tid; k < K; k += LZ_CT) {
+    dfloat s = df_make(0.f, 0.f);
+    for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(cw[(size_t)w * (r + 1) + k]));
+    dst[k] = f2(s);
+  }
+}
+
+// Basis rows per register group in the row phases: RG * KT = 32 basis
+// elements per lane in registers.
+template <int KT>
+struct RowGroup {
+  static constexpr int RG = 32 / KT;                       // rows per group
+  static constexpr int SH = (KT == 1) ? 0 : (KT == 2) ? 1 : 2;  // lane >> SH owns a row
+};
+
+// Basis rows 0 .. RG-1 of Qb (those < ng) at the columns k = lane + 32 kt < K,
+// zero elsewhere; all loads of a group are in flight together.
+template <int KT, int RG>
+SLS_DEV void load_qgroup(const float2* __restrict__ Qb, int ldq, int ng, int K,
+                         float2 (&q)[RG][KT]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < RG; ++i) {
+#pragma unroll
+    for (int kt = 0; kt < KT; ++kt) {
+      const int k = lane + 32 * kt;
+      q[i][kt] = make_float2(0.f, 0.f);
+      if (i < ng && k < K) q[i][kt] = Qb[(size_t)i * ldq + k];
+    }
+  }
+}
+
+// sum_k q[i][k] c_k for the RG rows of a group (float32: the coefficients are
+// at rounding level); lane L gets row L >> (5 - log2 RG).
+template <int KT, int RG>
+SLS_DEV float group_correction(const float2 (&q)[RG][KT], const float2 (&cv)[KT]) {
+  float v[RG];
+#pragma unroll
+  for (int i = 0; i < RG; ++i) {
+    float s = 0.f;
+#pragma unroll
+    for (int kt = 0; kt < KT; ++kt)
+      s = fmaf(q[i][kt].x, cv[kt].x, fmaf(q[i][kt].x, cv[kt].y, fmaf(q[i][kt].y, cv[kt].x, s)));
+    v[i] = s;
+  }
+  return transpose_sum_f<RG>(v);
+}
+
+// Row phase of step j for the warp's rows [wr0, wr1) of the strip, in groups
+// of RG rows held in registers (lanes over the basis index k):
+//   z1 = z' - Q c                    (the re-orthogonalisation, c = Q^T z'
+//                                     from the previous step, float32: the
+//                                     coefficients are at rounding level)
+//   q_j = z1 / beta_{j-1},  Q[:, j] = q_j
+//   z' <- s - alpha_j q_j - beta_{j-1} q_{j-1}   (s = Phi w_j from sweep B)
+// and, unless this is the last step, the partials of the next step:
+// c += Q^T z' over k <= j, |z'|^2, sum |z'|.
+template <int KT>
+SLS_DEV void row_phase(float2* __restrict__ Qs, int ldq, int wr0, int wr1, int j, bool last,
+                       const float2* __restrict__ cs, const float2* __restrict__ sv,
+                       float2* __restrict__ zps, dfloat invb, dfloat alpha, dfloat beta,
+                       dfloat (&cacc)[KT], dfloat& nacc, float& zl1) {
+  constexpr int RG = RowGroup<KT>::RG, SH = RowGroup<KT>::SH;
+  const int lane = threadIdx.x & 31;
+  float2 cv[KT];
+#pragma unroll
+  for (int kt = 0; kt < KT; ++kt) {
+    const int k = lane + 32 * kt;
+    cv[kt] = (k < j) ? cs[k] : make_float2(0.f, 0.f);
+  }
+  for (int b = wr0; b < wr1; b += RG) {
+    const int ng = min(RG, wr1 - b);
+    float2* Qb = Qs + (size_t)b * ldq;
+    float2 q[RG][KT];
+    load_qgroup<KT, RG>(Qb, ldq, ng, j, q);
+    const int i = lane >> SH;
+    float2 sin = make_float2(0.f, 0.f), zin = sin, qprev = sin;
+    if (i < ng) {
+      sin = sv[b + i];
+      zin = zps[b + i];
+      if (j > 0) qprev = Qb[(size_t)i * ldq + j - 1];
+    }
+    const float corr = group_correction<KT, RG>(q, cv);
+    dfloat qj = df_make(0.f, 0.f), zp = df_make(0.f, 0.f);
+    if (i < ng) {
+      dfloat z1 = dfv(zin);
+      if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
+      qj = df_mul(z1, invb);
+      zp = df_sub(dfv(sin), df_mul(alpha, qj));
+      if (j > 0) zp = df_sub(zp, df_mul(beta, dfv(qprev)));
+      if ((lane & ((1 << SH) - 1)) == 0) {
+        Qb[(size_t)i * ldq + j] = f2(qj);
+        zps[b + i] = f2(zp);
+        if (!last) {
+          dot2_acc_df(nacc.hi, nacc.lo, zp, zp);
+          zl1 += fabsf(zp.hi);
+        }
+      }
+    }
+    if (!last) {
+#pragma unroll
+      for (int ii = 0; ii < RG; ++ii) {
+        const dfloat zb = shfl_df(zp, ii << SH);
+        const dfloat qb = shfl_df(qj, ii << SH);
+#pragma unroll
+        for (int kt = 0; kt < KT; ++kt) {
+          const int k = lane + 32 * kt;
+          if (k <= j) {
+            const dfloat qk = (k == j) ? qb : dfv(q[ii][kt]);
+            dot2_acc_df(cacc[kt].hi, cacc[kt].lo, qk, zb);
+          }
+        }
+      }
+    }
+  }
+}
+
+// Block sums of a CTA: |z'|^2 (double-float, to *dst) and sum |z'| (per-warp
+// values in s_red1, added by their readers).
+SLS_DEV void store_cta_sums(dfloat nacc, float zl1, float2* tmpw, float* s_red1,
+                            float2* __restrict__ dst) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  nacc = df_norm(nacc.hi, nacc.lo);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) nacc = df_add_fast(nacc, shfl_xor_df(nacc, o));
+  zl1 = warp_sum_f(zl1);
+  if (lane == 0) {
+    tmpw[warp] = f2(nacc);
+    s_red1[warp] = zl1;
+  }
+  named_sync(BAR_COMPUTE, LZ_CT);
+  if (tid == 0) {
+    dfloat t = df_make(0.f, 0.f);
+    for (int w = 0; w < LZ_CW; ++w) t = df_add(t, dfv(tmpw[w]));
+    *dst = f2(t);
+  }
+}
+
+template <int GPT, int KT>
+__global__ void __launch_bounds__(LZ_THREADS, 1)
+lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroups,
+               int rows_cap, int ring_stages, int* status) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ float2 tmpw[LZ_CW];
+  __shared__ float s_red1[LZ_CW];  // per-warp max |Phi| and sum |z'| (offset bounds)
+  __shared__ double shd[4];
+  __shared__ int sflag, sbreak;
+  // copy warp <-> compute warps handshake (no named barrier involves the copy
+  // warp, so an early exit of either side can never leave the other blocked in
+  // bar.sync; every wait on these flags is bounded)
+  __shared__ volatile int s_halt;        // compute -> copy: stop issuing this problem
+  __shared__ volatile int s_go;          // compute -> copy: may start problem s_go - 1
+  __shared__ volatile int s_pdone;       // copy -> compute: finished problem s_pdone - 1
+  __shared__ volatile unsigned s_issued;  // copy -> compute: chunks issued so far
+  __shared__ volatile int s_err;          // a wait of this CTA gave up
+
+  constexpr int TCR = team_rows(GPT);
+  const int D = bt.D, r = bt.r, ldq = q_ld(bt.r);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int gi = blockIdx.x / g, rank = blockIdx.x % g;
+  const int C4 = D >> 2;
+  const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
+  const int redn = (P > 1) ? P * D : 0;
+
+  const RingShape shp0 = ring_shape(D, 0);
+  const int S = ring_stages;
+  const int cr = shp0.cr;
+  const unsigned stage = shp0.stage;
+  unsigned char* ring = smem_raw;
+  unsigned char* after_ring = smem_raw + (size_t)S * stage;
+  float* wsh = reinterpret_cast<float*>(after_ring);   // D
+  float* wsl = wsh + D;                                // D
+  float2* red = reinterpret_cast<float2*>(wsl + D);    // redn
+  float2* sv = red + redn;                             // rows_cap (s = Phi w_j of the strip)
+  float2* zps = sv + rows_cap;                         // rows_cap (z' of the strip)
+  float2* bpart = zps + rows_cap;                      // 2 x WB_ROWS x LZ_CW
+  float2* cw = bpart + 2 * WB_ROWS * LZ_CW;            // LZ_CW x (r+1)
+  float2* cs = cw + (size_t)LZ_CW * (r + 1);           // r+1 (c = Q^T z')
+  float2* red2 = cs + (r + 1);                         // 4 * LZ_CT
+  uint64_t* bars = reinterpret_cast<uint64_t*>(
+      (reinterpret_cast<uintptr_t>(red2 + 4 * LZ_CT) + 15) & ~(uintptr_t)15);
+  uint64_t* fullb = bars;
+  uint64_t* emptyb = bars + S;
+
+  const LzLayout L = lz_layout(bt.nmax, D, r, g);
+  char* gb = scratch + (size_t)gi * gstride;
+  unsigned* barw = reinterpret_cast<unsigned*>(gb + L.bar);
+  float2* wpart = reinterpret_cast<float2*>(gb + L.wpart);
+  float2* wred = reinterpret_cast<float2*>(gb + L.wred);
+  float2* Wm = reinterpret_cast<float2*>(gb + L.Wm);
+  float2* cpart = reinterpret_cast<float2*>(gb + L.cpart);
+  float2* npart = reinterpret_cast<float2*>(gb + L.npart);
+  float2* sqpart = reinterpret_cast<float2*>(gb + L.sqpart);
+  const GroupBarrier bar{barw, barw + 32, (unsigned)g};
+
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&fullb[s], 1);
+      mbar_init(&emptyb[s], LZ_CW);
+    }
+    mbar_fence_init();
+    s_halt = 0;
+    s_go = 0;
+    s_pdone = 0;
+    s_issued = 0;
+    s_err = 0;
+  }
+  __syncthreads();
+
+  const int nprob = nprob_of(bt);
+
+  // ========================= copy warp ======================================
+  // Phi is read-only, so the copy warp runs ahead of the compute warps by as
+  // many chunks as the ring holds: sweep A forward, sweep B backward, per step.
+  if (warp == LZ_CW) {
+    if (lane != 0) return;
+    const uint64_t pol = l2_policy_normal();
+    unsigned cnt = 0;
+    int pp = 0;
+    for (int p = gi; p < nprob; p += ngroups, ++pp) {
+      bool ok = false;
+      for (unsigned it = 0; it < (1u << 26); ++it) {
+        if (s_go == pp + 1) {
+          ok = true;
+          break;
+        }
+        __nanosleep(64);
+      }
+      if (!ok) {
+        lz_fail(status, &s_err);
+        break;
+      }
+      const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
+      const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
+      const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
+      const int nch = (int)((re - rs + cr - 1) / cr);
+      const float* Phi = bt.Phi + (row0 + rs) * D;
+      bool stop = false;
+      for (int j = 0; j < r && !stop; ++j) {
+        for (int sweep = 0; sweep < 2 && !stop; ++sweep) {
+          for (int t = 0; t < nch; ++t) {
+            if (s_halt) {
+              stop = true;
+              break;
+            }
+            const int k = (sweep == 0) ? t : nch - 1 - t;
+            const int slot = (int)(cnt % (unsigned)S);
+            const unsigned par = (cnt / (unsigned)S) & 1u;
+            if (!mbar_wait(&emptyb[slot], par ^ 1u)) {
+              lz_fail(status, &s_err);
+              stop = true;
+              break;
+            }
+            const int64_t nr = min((int64_t)cr, (re - rs) - (int64_t)k * cr);
+            const unsigned b1 = (unsigned)(nr * D * 4);
+            unsigned char* dst = ring + (size_t)slot * stage;
+            mbar_expect_tx(&fullb[slot], b1);
+            bulk_g2s(dst, Phi + (int64_t)k * cr * D, b1, &fullb[slot], pol);
+            ++cnt;
+            __threadfence_block();
+            s_issued = cnt;
+          }
+        }
+      }
+      __threadfence_block();
+      s_pdone = pp + 1;
+      if (*((volatile int*)status) == SLS_ERR_TIMEOUT) break;
+    }
+    // every copy issued has landed before the CTA may exit
+    for (unsigned c = (cnt > (unsigned)S ? cnt - S : 0); c < cnt; ++c)
+      mbar_wait(&fullb[c % S], (c / S) & 1u);
+    return;
+  }
+
+  // ========================= compute warps ===================================
+  unsigned lgen = 0;
+  RingCursor rc{0u, 0, 0u};  // chunks consumed
+  int pp = 0;
+  for (int p = gi; p < nprob; p += ngroups, ++pp) {
+    if (tid == 0) {
+      s_halt = 0;
+      __threadfence_block();
+      s_go = pp + 1;
+    }
+    const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
+    const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
+    const int64_t q1o = bt.q1off ? bt.q1off[p] : row0;
+    const double* q1 = bt.q1 + q1o;
+    const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
+    float2* Qs = bt.Q + (row0 + rs) * ldq;  // this CTA's rows of the basis
+    const int nrows = (int)(re - rs);
+    const int nch = (nrows + cr - 1) / cr;
+    const int wr0 = warp * nrows / LZ_CW, wr1 = (warp + 1) * nrows / LZ_CW;
+    double* alpha_out = bt.alpha + (size_t)p * r;
+    double* beta_out = bt.beta + (size_t)p * r;
+    const int cbeg = (int)((int64_t)rank * D / g), cend = (int)((int64_t)(rank + 1) * D / g);
+
+    double scale = 0.0, alpha_prev = 0.0;
+    dfloat alpha_df = df_make(0.f, 0.f), beta_df = df_make(0.f, 0.f), invb_df;
+    float phimax = 0.f;  // max |Phi| over this CTA's strip (step 0, sweep A)
+    int reff = 0;
+    sbreak = 0;
+
+    // step 0 starts from z' = q1: its partials |z'|^2 and sum |z'|
+    {
+      dfloat nacc = df_make(0.f, 0.f);
+      float zl1 = 0.f;
+      for (int il = tid; il < nrows; il += LZ_CT) {
+        const dfloat z = df_from_double(q1[rs + il]);
+        zps[il] = f2(z);
+        dot2_acc_df(nacc.hi, nacc.lo, z, z);
+        zl1 += fabsf(z.hi);
+      }
+      store_cta_sums(nacc, zl1, tmpw, s_red1, npart + (size_t)rank);
+    }
+
+    for (int j = 0; j < r; ++j) {
+      // ---------------- sweep A (forward): Phi^T z' ------------------------------
+      {
+        // offset for the column sums: all partial sums of Phi^T z' over the
+        // strip are bounded by max|Phi| * sum_i |z'_i|
+        const bool ofsA = (P == 1) && (j > 0);
+        float Ca = 0.f;
+        if (ofsA) {
+          float z1sum = 0.f;
+#pragma unroll
+          for (int w = 0; w < LZ_CW; ++w) z1sum += s_red1[w];
+          Ca = ofs_pow2(phimax * z1sum);
+        }
+        f32x2_t ah[GPT][2], al[GPT][2];
+        const f32x2_t a0 = pk2(Ca, Ca);
+#pragma unroll
+        for (int q = 0; q < GPT; ++q) {
+          ah[q][0] = ah[q][1] = a0;
+          al[q][0] = al[q][1] = 0ull;
+        }
+        float mx = 0.f;
+        if (ofsA) {
+          // two chunks per pass: more independent rows in flight per thread
+          for (int t = 0; t < nch; t += 2) {
+            const bool two = t + 1 < nch;
+            const int s0 = rc.slot;
+            if (!mbar_wait(&fullb[s0], rc.par)) lz_fail(status, &s_err);
+            rc_next(rc, S);
+            int s1 = s0;
+            if (two) {
+              s1 = rc.slot;
+              if (!mbar_wait(&fullb[s1], rc.par)) lz_fail(status, &s_err);
+              rc_next(rc, S);
+            }
+            const float* ch0 = reinterpret_cast<const float*>(ring + (size_t)s0 * stage);
+            const float* ch1 = reinterpret_cast<const float*>(ring + (size_t)s1 * stage);
+            const int nr0 = min(cr, nrows - t * cr);
+            const int nr1 = two ? min(cr, nrows - (t + 1) * cr) : 0;
+            sweepA_team_pair<GPT, TCR>(ch0, nr0, t * cr, ch1, nr1, (t + 1) * cr, C4, zps, ah, al);
+            __syncwarp();
+            if (lane == 0) {
+              mbar_arrive(&emptyb[s0]);
+              if (two) mbar_arrive(&emptyb[s1]);
+            }
+          }
+        } else {
+          for (int t = 0; t < nch; ++t) {
+            const int slot = rc.slot;
+            if (!mbar_wait(&fullb[slot], rc.par))
+              lz_fail(status, &s_err);  // leave at the next group barrier
+            const float* chunk = reinterpret_cast<const float*>(ring + (size_t)slot * stage);
+            const int nr = min(cr, nrows - t * cr);
+            if (j == 0)
+              sweepA_chunk<GPT, true>(chunk, nr, D, t * cr, zps, ah, al, &mx);
+            else
+              sweepA_chunk<GPT, false>(chunk, nr, D, t * cr, zps, ah, al, &mx);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&emptyb[slot]);
+            rc_next(rc, S);
+          }
+        }
+        if (j == 0) {
+          for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+          named_sync(BAR_COMPUTE, LZ_CT);  // s_red1 (sum |z'|) has been read
+          if (lane == 0) s_red1[warp] = mx;
+        }
+        // CTA partial of Phi^T z'
+        const int ph = (P == 1) ? 0 : tid / C4;
+        const int cb = (P == 1) ? tid : tid % C4;
+        float2* dst = (P == 1) ? wpart + (size_t)rank * D : red + (size_t)ph * D;
+        if (P == 1 || tid < P * C4) {
+#pragma unroll
+          for (int q = 0; q < GPT; ++q) {
+            const int cg = cb + q * LZ_CT;
+            if (cg < C4) {
+              float h0, h1, l0, l1, h2, h3, l2, l3;
+              upk2(ah[q][0], h0, h1);
+              upk2(al[q][0], l0, l1);
+              upk2(ah[q][1], h2, h3);
+              upk2(al[q][1], l2, l3);
+              dst[4 * cg + 0] = f2(df_norm(h0 - Ca, l0));
+              dst[4 * cg + 1] = f2(df_norm(h1 - Ca, l1));
+              dst[4 * cg + 2] = f2(df_norm(h2 - Ca, l2));
+              dst[4 * cg + 3] = f2(df_norm(h3 - Ca, l3));
+            }
+          }
+        }
+        if (P > 1) {
+          named_sync(BAR_COMPUTE, LZ_CT);
+          for (int col = tid; col < D; col += LZ_CT) {
+            dfloat s = df_make(0.f, 0.f);
+            for (int q = 0; q < P; ++q) s = df_add(s, dfv(red[(size_t)q * D + col]));
+            wpart[(size_t)rank * D + col] = f2(s);
+          }
+        }
+      }
+      if (!group_sync_named(bar, lgen, status, &sflag, &s_err, BAR_COMPUTE, LZ_CT)) return;
+
+      // ---------------- slice phase: c, Phi^T z1 for this CTA's columns ----------
+      // c = Q^T z' (k < j) from the partials of the previous row phase;
+      // Phi^T z1 = Phi^T z' - sum_k c_k w_k with w_k = Phi^T q_k kept in Wm.
+      reduce_coeffs(cpart, g, r, j, cs);
+      {
+        dfloat sq = df_make(0.f, 0.f);
+        for (int c0 = cbeg + warp * 8; c0 < cend; c0 += LZ_CW * 8) {
+          const int c = c0 + (lane & 7);
+          const bool valid = c < cend;
+          dfloat s = warp_colsum8(wpart, (size_t)D, g, c, valid);
+          if (j > 0) s = df_sub(s, warp_wcorr8(Wm, D, j, c, valid, cs));
+          if (lane < 8 && valid) {
+            wred[c] = f2(s);
+            dot2_acc_df(sq.hi, sq.lo, s, s);
+          }
+        }
+        sq = df_norm(sq.hi, sq.lo);
+#pragma unroll
+        for (int o = 4; o > 0; o >>= 1) sq = df_add_fast(sq, shfl_xor_df(sq, o));
+        if (lane == 0) tmpw[warp] = f2(sq);
+        named_sync(BAR_COMPUTE, LZ_CT);
+        if (tid == 0) {
+          dfloat s = df_make(0.f, 0.f);
+          for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(tmpw[w]));
+          sqpart[rank] = f2(s);
+        }
+      }
+      if (!group_sync_named(bar, lgen, status, &sflag, &s_err, BAR_COMPUTE, LZ_CT)) return;
+
+      // ---------------- beta_{j-1}, alpha_j, break test -------------------------
+      if (warp == 0) {
+        // |z1|^2 = |z'|^2 - |c|^2 (Q orthonormal), |Phi^T z1|^2
+        const dfloat s = warp_sum_vec(npart + (size_t)(j & 1) * g, g);
+        const dfloat q = warp_sum_vec(sqpart, g);
+        dfloat cn = df_make(0.f, 0.f);
+#pragma unroll
+        for (int tt = 0; tt < KT; ++tt) {
+          const int k = lane + 32 * tt;
+          if (k < j) dot2_acc_df(cn.hi, cn.lo, dfv(cs[k]), dfv(cs[k]));
+        }
+        cn = df_norm(cn.hi, cn.lo);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) cn = df_add_fast(cn, shfl_xor_df(cn, o));
+        if (lane == 0) {
+          const double nrm2 = df_to_double(s) - df_to_double(cn);  // |z1|^2
+          const double bnew = sqrt(fmax(nrm2, 0.0));
+          int brk = 0;
+          if (j > 0) {
+            scale = fmax(scale, fabs(alpha_prev) + bnew);
+            if (!(bnew > bt.tol * scale)) brk = 1;
+            else if (rank == 0) beta_out[j - 1] = bnew;
+          } else if (!(bnew > 0.0)) {
+            brk = 1;
+          }
+          const double a = brk ? 0.0 : df_to_double(q) / (bnew * bnew);
+          if (!brk && rank == 0) alpha_out[j] = a;
+          shd[1] = brk ? 0.0 : 1.0 / bnew;
+          shd[2] = a;
+          shd[3] = (j > 0) ? bnew : 0.0;
+          sbreak = brk;
+          if (brk) s_halt = 1;
+        }
+      }
+      named_sync(BAR_COMPUTE, LZ_CT);
+      if (sbreak) {
+        reff = j;
+        break;
+      }
+      invb_df = df_from_double(shd[1]);
+      alpha_prev = shd[2];
+      alpha_df = df_from_double(shd[2]);
+      beta_df = df_from_double(shd[3]);
+      if (j == 0) {
+#pragma unroll
+        for (int w = 0; w < LZ_CW; ++w) phimax = fmaxf(phimax, s_red1[w]);
+      }
+      // w_j = (Phi^T z1) / beta into shared memory; keep w_j (slice) for the
+      // correction of later steps
+      for (int c0 = tid; c0 < D; c0 += 8 * LZ_CT) {
+        float2 wv[8];
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+          const int c = c0 + m * LZ_CT;
+          wv[m] = (c < D) ? wred[c] : make_float2(0.f, 0.f);
+        }
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+          const int c = c0 + m * LZ_CT;
+          if (c < D) {
+            const dfloat a = df_mul(dfv(wv[m]), invb_df);
+            wsh[c] = a.hi;
+            wsl[c] = a.lo;
+            if (c >= cbeg && c < cend) Wm[(size_t)j * D + c] = f2(a);
+          }
+        }
+      }
+      named_sync(BAR_COMPUTE, LZ_CT);
+
+      // ---------------- sweep B (backward): s = Phi w_j per row -----------------
+      if (P == 1) {
+        f32x2_t wh[GPT][2], nwh[GPT][2], wl[GPT][2];
+        float wt1 = 0.f;  // l1 norm of this thread's slice of w_j
+        const float4* h4 = reinterpret_cast<const float4*>(wsh);
+        const float4* l4 = reinterpret_cast<const float4*>(wsl);
+#pragma unroll
+        for (int q = 0; q < GPT; ++q) {
+          const int cg = tid + q * LZ_CT;
+          float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
+          if (cg < C4) {
+            a = h4[cg];
+            b = l4[cg];
+          }
+          wh[q][0] = pk2(a.x, a.y);
+          wh[q][1] = pk2(a.z, a.w);
+          nwh[q][0] = pk2(-a.x, -a.y);
+          nwh[q][1] = pk2(-a.z, -a.w);
+          wl[q][0] = pk2(b.x, b.y);
+          wl[q][1] = pk2(b.z, b.w);
+          wt1 += (fabsf(a.x) + fabsf(a.y)) + (fabsf(a.z) + fabsf(a.w));
+        }
+        // offset of this thread's row partials: each is bounded by
+        // max|Phi| * |w slice|_1
+        const float Ct = ofs_pow2(phimax * wt1);
+        constexpr int WCH = WB_ROWS / TCR;  // chunks per window (even)
+        for (int t0p = 0; t0p < nch; t0p += 2) {
+          const bool two = t0p + 1 < nch;
+          const int kc0 = nch - 1 - t0p;
+          const int s0 = rc.slot;
+          if (!mbar_wait(&fullb[s0], rc.par)) lz_fail(status, &s_err);
+          rc_next(rc, S);
+          int s1 = s0;
+          if (two) {
+            s1 = rc.slot;
+            if (!mbar_wait(&fullb[s1], rc.par)) lz_fail(status, &s_err);
+            rc_next(rc, S);
+          }
+          const float* ch0 = reinterpret_cast<const float*>(ring + (size_t)s0 * stage);
+          const float* ch1 = reinterpret_cast<const float*>(ring + (size_t)s1 * stage);
+          const int nr0 = min(cr, nrows - kc0 * cr);
+          const int nr1 = two ? cr : 0;
+          const int win = t0p / WCH, tw0 = t0p % WCH;
+          float2* bp0 = bpart + (size_t)((win & 1) * WB_ROWS + tw0 * TCR) * LZ_CW;
+          float2* bp1 = bp0 + (size_t)TCR * LZ_CW;
+          sweepB_team_pair<GPT, TCR>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bp0, bp1);
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(&emptyb[s0]);
+            if (two) mbar_arrive(&emptyb[s1]);
+          }
+          const int t = two ? t0p + 1 : t0p;  // last chunk of the pass
+          const int tw = t % WCH;
+          if (tw == WCH - 1 || t == nch - 1) {
+            // the window's warp partials are complete: one row per thread sums
+            // them (the summing threads rotate from window to window)
+            named_sync(BAR_COMPUTE, LZ_CT);
+            const int t0 = t - tw;
+            const int pidx = (tid - 64 * (win & 3) + LZ_CT) % LZ_CT;
+            if (pidx < (tw + 1) * TCR) {
+              const int il = (nch - 1 - (t0 + pidx / TCR)) * cr + pidx % TCR;
+              if (il < nrows) {
+                const float2* src = bpart + (size_t)((win & 1) * WB_ROWS + pidx) * LZ_CW;
+                dfloat s = df_make(0.f, 0.f);
+#pragma unroll
+                for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(src[w]));
+                sv[il] = f2(s);
+              }
+            }
+          }
+        }
+      } else {
+        for (int t = 0; t < nch; ++t) {
+          const int kc = nch - 1 - t;
+          const int slot = rc.slot;
+          if (!mbar_wait(&fullb[slot], rc.par))
+            lz_fail(status, &s_err);  // leave at the next group barrier
+          const float* chunk = reinterpret_cast<const float*>(ring + (size_t)slot * stage);
+          const int nr = min(cr, nrows - kc * cr);
+          for (int ii = warp; ii < nr; ii += LZ_CW) {
+            const dfloat s = row_dot_smem(chunk + (size_t)ii * D, D, wsh, wsl);
+            if (lane == 0) sv[kc * cr + ii] = f2(s);
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&emptyb[slot]);
+          rc_next(rc, S);
+        }
+      }
+      named_sync(BAR_COMPUTE, LZ_CT);
+
+      // ---------------- row phase: q_j, next z', partials of step j+1 --------------
+      const bool last = (j == r - 1);
+      {
+        dfloat cacc[KT];
+#pragma unroll
+        for (int t = 0; t < KT; ++t) cacc[t] = df_make(0.f, 0.f);
+        dfloat nacc = df_make(0.f, 0.f);
+        float zl1 = 0.f;
+        row_phase<KT>(Qs, ldq, wr0, wr1, j, last, cs, sv, zps, invb_df, alpha_df, beta_df, cacc,
+                      nacc, zl1);
+        if (last) {
+          reff = r;
+          break;
+        }
+        // partials for step j+1 (read after its barrier 1): c, |z'|^2, sum |z'|
+        store_coeff_partials(cacc, j + 1, r, cw, cpart + (size_t)rank * (r + 1));
+        store_cta_sums(nacc, zl1, tmpw, s_red1, npart + (size_t)((j + 1) & 1) * g + rank);
+      }
+    }
+    // a break leaves chunks issued ahead of it: consume them until the copy
+    // warp reports that it stopped
+    if (sbreak) {
+      for (unsigned it = 0; it < (1u << 26); ++it) {
+        const unsigned iss = s_issued;
+        if (rc.cnt < iss) {
+          const int slot = rc.slot;
+          if (!mbar_wait(&fullb[slot], rc.par)) {
+            lz_fail(status, &s_err);
+            break;
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&emptyb[slot]);
+          rc_next(rc, S);
+        } else if (s_pdone == pp + 1) {
+          if (s_issued == rc.cnt) break;
+        } else {
+          __nanosleep(64);
+        }
+      }
+    }
+    if (rank == 0 && tid == 0) {
+      bt.r_eff[p] = reff;
+      for (int k = reff; k < r; ++k) alpha_out[k] = 0.0;
+      for (int k = (reff > 0 ? reff - 1 : 0); k < r; ++k) beta_out[k] = 0.0;
+    }
+    // problems on the same group run back to back; keep them apart
+    if (!group_sync_named(bar, lgen, status, &sflag, &s_err, BAR_COMPUTE, LZ_CT)) return;
+  }
+}
+
+template <int GPT, int KT>
+int launch_lanczos_t(const LanczosBatch& bt, void* scratch, size_t gstride, int groups, int g,
+                     int rows_cap, int stages, int* status, size_t smem, cudaStream_t stream) {
+  auto fn = lanczos_kernel<GPT, KT>;
+  SLS_CUDA_TRY(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  char* sc = (char*)scratch;
+  void* args[] = {(void*)&bt, (void*)&sc, (void*)&gstride, (void*)&g, (void*)&groups,
+                  (void*)&rows_cap, (void*)&stages, (void*)&status};
+  SLS_CUDA_TRY(cudaLaunchCooperativeKernel((const void*)fn, dim3(groups * g), dim3(LZ_THREADS),
+                                           args, smem, stream));
+  count_launch(1);
+  return SLS_OK;
+}
+
+}  // namespace
+
+// Launch the Lanczos kernel for GPT = 1, 2, 4 or 8 column groups per thread
+// and KT = 1, 2 or 4 basis tiles (lanczos_g<GPT>.cu).
+#define SLS_LZ_LAUNCH_ARGS                                                                \
+  const LanczosBatch &bt, void *scratch, size_t gstride, int groups, int g, int rows_cap, \
+      int stages, int *status, size_t smem, cudaStream_t stream, int kt
+int launch_lanczos_gpt1(SLS_LZ_LAUNCH_ARGS);
+int launch_lanczos_gpt2(SLS_LZ_LAUNCH_ARGS);
+int launch_lanczos_gpt4(SLS_LZ_LAUNCH_ARGS);
+int launch_lanczos_gpt8(SLS_LZ_LAUNCH_ARGS);
+
+}  // namespace sls
