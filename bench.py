@@ -66,6 +66,12 @@ def config_dict(w, extra=None):
     return d
 
 
+# Revision of the persistent Lanczos kernel whose DRAM counters are recorded in
+# profiles/lanczos_traffic.json; bumped with every change of the kernel, so a
+# stale capture reads as "traffic": null.
+LANCZOS_KERNEL_REV = "single-pass-cgs/2-barrier/offset-fts"
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -267,7 +273,7 @@ def run_native(args, rank, world):
         try:
             with open(tr) as f:
                 t = json.load(f)
-            if t.get("workload") == w.name and t.get("kernel_rev") == "v1":
+            if t.get("workload") == w.name and t.get("kernel_rev") == LANCZOS_KERNEL_REV:
                 roof["traffic"] = t["dram_bytes_per_launch"]
         except Exception:
             pass
