@@ -322,13 +322,12 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
   const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
   const int redn = (P > 1) ? P * bt.D : 0;
   const int rows_cap = (int)((bt.nmax + g - 1) / g) + 1;
-  // shared memory besides the ring: w (hi, lo), phase partials, s and z' of
-  // the strip, sweep-B warp partials, coefficient partials and c, reduction
-  // scratch, barriers
-  const size_t other = sizeof(float) * 2 * (size_t)bt.D +
+  // shared memory besides the ring: w (hi, lo; only for D < 4 LZ_CT), phase
+  // partials, s and z' of the strip, sweep-B warp partials, coefficient
+  // partials and c, barriers
+  const size_t other = sizeof(float) * 2 * (size_t)(P > 1 ? bt.D : 0) +
                        sizeof(float2) * ((size_t)redn + 2 * (size_t)rows_cap +
-                                         2 * WB_ROWS * LZ_CW +
-                                         (size_t)(LZ_CW + 1) * (bt.r + 1) + 4 * LZ_CT) +
+                                         2 * WB_ROWS * LZ_CW + (size_t)(LZ_CW + 1) * (bt.r + 1)) +
                        16 + 2 * RING_MAX_STAGES * 8;
   const size_t limit = 227 * 1024 - 1024;  // leave room for static shared memory
   if (other >= limit) return SLS_ERR_UNSUPPORTED;

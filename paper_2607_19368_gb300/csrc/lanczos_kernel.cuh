@@ -197,8 +197,9 @@ SLS_DEV float transpose_sum_f(float (&v)[CR]) {
 
 // Sweep A over two ring chunks at once (D >= 4 * LZ_CT; CR rows each, the
 // second chunk may be absent: nr1 = 0) with offset accumulators: ah starts at
-// the power-of-two offset of the column sums.
-template <int GPT, int CR>
+// the power-of-two offset of the column sums.  FULL: both chunks full and
+// D = 4 LZ_CT GPT (the steady state), so the row and column guards vanish.
+template <int GPT, int CR, bool FULL>
 SLS_DEV void sweepA_team_pair(const float* __restrict__ c0, int nr0, int lb0,
                               const float* __restrict__ c1, int nr1, int lb1, int C4,
                               const float2* __restrict__ us, f32x2_t (&ah)[GPT][2],
@@ -208,14 +209,14 @@ SLS_DEV void sweepA_team_pair(const float* __restrict__ c0, int nr0, int lb0,
   for (int i = 0; i < 2 * CR; ++i) {
     const bool first = i < CR;
     const int ii = first ? i : i - CR;
-    if (ii < (first ? nr0 : nr1)) {
+    if (FULL || ii < (first ? nr0 : nr1)) {
       const float4* c4 = reinterpret_cast<const float4*>(first ? c0 : c1);
       const float2 u = us[(first ? lb0 : lb1) + ii];
       const f32x2_t uh = pk2(u.x, u.x), nuh = pk2(-u.x, -u.x), ul = pk2(u.y, u.y);
 #pragma unroll
       for (int q = 0; q < GPT; ++q) {
         const int cg = tid + q * LZ_CT;
-        if (cg < C4) {
+        if (FULL || cg < C4) {
           const float4 f = c4[ii * C4 + cg];
           ofs_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
           ofs_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
@@ -271,7 +272,7 @@ SLS_DEV dfloat transpose_sum_df(dfloat (&v)[CR]) {
 // loose global bound; the 2 CR per-row double-float partials are then summed
 // over the warp by one transposed butterfly and the warp sums stored to
 // bp0 / bp1 [i * LZ_CW + warp].
-template <int GPT, int CR>
+template <int GPT, int CR, bool FULL>
 SLS_DEV void sweepB_team_pair(const float* __restrict__ c0, int nr0, const float* __restrict__ c1,
                               int nr1, int C4, const f32x2_t (&wh)[GPT][2],
                               const f32x2_t (&nwh)[GPT][2], const f32x2_t (&wl)[GPT][2],
@@ -284,12 +285,12 @@ SLS_DEV void sweepB_team_pair(const float* __restrict__ c0, int nr0, const float
     const bool first = i < CR;
     const int ii = first ? i : i - CR;
     f32x2_t s = pk2(Ct, Ct), lo = 0ull;
-    if (ii < (first ? nr0 : nr1)) {
+    if (FULL || ii < (first ? nr0 : nr1)) {
       const float4* c4 = reinterpret_cast<const float4*>(first ? c0 : c1);
 #pragma unroll
       for (int q = 0; q < GPT; ++q) {
         const int cg = tid + q * LZ_CT;
-        if (cg < C4) {
+        if (FULL || cg < C4) {
           const float4 f = c4[ii * C4 + cg];
           ofs_acc2n(s, lo, pk2(f.x, f.y), wh[q][0], nwh[q][0], wl[q][0]);
           ofs_acc2n(s, lo, pk2(f.z, f.w), wh[q][1], nwh[q][1], wl[q][1]);
@@ -630,6 +631,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   const int C4 = D >> 2;
   const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
   const int redn = (P > 1) ? P * D : 0;
+  const bool fullD = (C4 == GPT * LZ_CT);  // no ragged column groups
 
   const RingShape shp0 = ring_shape(D, 0);
   const int S = ring_stages;
@@ -637,17 +639,17 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   const unsigned stage = shp0.stage;
   unsigned char* ring = smem_raw;
   unsigned char* after_ring = smem_raw + (size_t)S * stage;
-  float* wsh = reinterpret_cast<float*>(after_ring);   // D
-  float* wsl = wsh + D;                                // D
-  float2* red = reinterpret_cast<float2*>(wsl + D);    // redn
+  const int wn = (P > 1) ? D : 0;                      // w_j staged for row_dot_smem
+  float* wsh = reinterpret_cast<float*>(after_ring);   // wn
+  float* wsl = wsh + wn;                               // wn
+  float2* red = reinterpret_cast<float2*>(wsl + wn);   // redn
   float2* sv = red + redn;                             // rows_cap (s = Phi w_j of the strip)
   float2* zps = sv + rows_cap;                         // rows_cap (z' of the strip)
   float2* bpart = zps + rows_cap;                      // 2 x WB_ROWS x LZ_CW
   float2* cw = bpart + 2 * WB_ROWS * LZ_CW;            // LZ_CW x (r+1)
   float2* cs = cw + (size_t)LZ_CW * (r + 1);           // r+1 (c = Q^T z')
-  float2* red2 = cs + (r + 1);                         // 4 * LZ_CT
   uint64_t* bars = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(red2 + 4 * LZ_CT) + 15) & ~(uintptr_t)15);
+      (reinterpret_cast<uintptr_t>(cs + (r + 1)) + 15) & ~(uintptr_t)15);
   uint64_t* fullb = bars;
   uint64_t* emptyb = bars + S;
 
@@ -821,7 +823,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
             const float* ch1 = reinterpret_cast<const float*>(ring + (size_t)s1 * stage);
             const int nr0 = min(cr, nrows - t * cr);
             const int nr1 = two ? min(cr, nrows - (t + 1) * cr) : 0;
-            sweepA_team_pair<GPT, TCR>(ch0, nr0, t * cr, ch1, nr1, (t + 1) * cr, C4, zps, ah, al);
+            if (fullD && nr0 == TCR && nr1 == TCR)
+              sweepA_team_pair<GPT, TCR, true>(ch0, nr0, t * cr, ch1, nr1, (t + 1) * cr, C4, zps, ah, al);
+            else
+              sweepA_team_pair<GPT, TCR, false>(ch0, nr0, t * cr, ch1, nr1, (t + 1) * cr, C4, zps, ah, al);
             __syncwarp();
             if (lane == 0) {
               mbar_arrive(&emptyb[s0]);
@@ -957,9 +962,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
 #pragma unroll
         for (int w = 0; w < LZ_CW; ++w) phimax = fmaxf(phimax, s_red1[w]);
       }
-      // w_j = (Phi^T z1) / beta into shared memory; keep w_j (slice) for the
-      // correction of later steps
-      for (int c0 = tid; c0 < D; c0 += 8 * LZ_CT) {
+      // w_j = (Phi^T z1) / beta: into shared memory for the row-per-warp
+      // sweep B (D < 4 LZ_CT; the team sweep takes its columns straight into
+      // registers below); keep w_j (slice) for the correction of later steps
+      if (P > 1) for (int c0 = tid; c0 < D; c0 += 8 * LZ_CT) {
         float2 wv[8];
 #pragma unroll
         for (int m = 0; m < 8; ++m) {
@@ -977,21 +983,40 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           }
         }
       }
-      named_sync(BAR_COMPUTE, LZ_CT);
+      if (P > 1) named_sync(BAR_COMPUTE, LZ_CT);
 
       // ---------------- sweep B (backward): s = Phi w_j per row -----------------
       if (P == 1) {
+        // this thread's columns of w_j, from the slices into registers
         f32x2_t wh[GPT][2], nwh[GPT][2], wl[GPT][2];
         float wt1 = 0.f;  // l1 norm of this thread's slice of w_j
-        const float4* h4 = reinterpret_cast<const float4*>(wsh);
-        const float4* l4 = reinterpret_cast<const float4*>(wsl);
+        const float4* wr4 = reinterpret_cast<const float4*>(wred);
+        float4 wv[GPT][2];
+#pragma unroll
+        for (int q = 0; q < GPT; ++q) {
+          const int cg = tid + q * LZ_CT;
+          wv[q][0] = wv[q][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (cg < C4) {
+            wv[q][0] = wr4[2 * cg];
+            wv[q][1] = wr4[2 * cg + 1];
+          }
+        }
 #pragma unroll
         for (int q = 0; q < GPT; ++q) {
           const int cg = tid + q * LZ_CT;
           float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
           if (cg < C4) {
-            a = h4[cg];
-            b = l4[cg];
+            const dfloat w0 = df_mul(df_make(wv[q][0].x, wv[q][0].y), invb_df);
+            const dfloat w1 = df_mul(df_make(wv[q][0].z, wv[q][0].w), invb_df);
+            const dfloat w2 = df_mul(df_make(wv[q][1].x, wv[q][1].y), invb_df);
+            const dfloat w3 = df_mul(df_make(wv[q][1].z, wv[q][1].w), invb_df);
+            a = make_float4(w0.hi, w1.hi, w2.hi, w3.hi);
+            b = make_float4(w0.lo, w1.lo, w2.lo, w3.lo);
+            const int c = 4 * cg;
+            if (c >= cbeg && c < cend) Wm[(size_t)j * D + c] = f2(w0);
+            if (c + 1 >= cbeg && c + 1 < cend) Wm[(size_t)j * D + c + 1] = f2(w1);
+            if (c + 2 >= cbeg && c + 2 < cend) Wm[(size_t)j * D + c + 2] = f2(w2);
+            if (c + 3 >= cbeg && c + 3 < cend) Wm[(size_t)j * D + c + 3] = f2(w3);
           }
           wh[q][0] = pk2(a.x, a.y);
           wh[q][1] = pk2(a.z, a.w);
@@ -1024,7 +1049,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           const int win = t0p / WCH, tw0 = t0p % WCH;
           float2* bp0 = bpart + (size_t)((win & 1) * WB_ROWS + tw0 * TCR) * LZ_CW;
           float2* bp1 = bp0 + (size_t)TCR * LZ_CW;
-          sweepB_team_pair<GPT, TCR>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bp0, bp1);
+          if (fullD && nr0 == TCR && nr1 == TCR)
+            sweepB_team_pair<GPT, TCR, true>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bp0, bp1);
+          else
+            sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bp0, bp1);
           __syncwarp();
           if (lane == 0) {
             mbar_arrive(&emptyb[s0]);
