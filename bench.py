@@ -69,7 +69,7 @@ def config_dict(w, extra=None):
 # Revision of the persistent Lanczos kernel whose DRAM counters are recorded in
 # profiles/lanczos_traffic.json; bumped with every change of the kernel, so a
 # stale capture reads as "traffic": null.
-LANCZOS_KERNEL_REV = "single-pass-cgs/2-barrier/offset-fts/full-pairs/6-stage"
+LANCZOS_KERNEL_REV = "fused-pass/1"
 
 
 def peaks():

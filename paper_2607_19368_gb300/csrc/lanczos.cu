@@ -323,15 +323,15 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
   const int redn = (P > 1) ? P * bt.D : 0;
   const int rows_cap = (int)((bt.nmax + g - 1) / g) + 1;
   // shared memory besides the ring: w (hi, lo; only for D < 4 LZ_CT), phase
-  // partials, s and z' of the strip, sweep-B warp partials, coefficient
-  // partials and c, barriers
+  // partials, z' of the strip, row-dot warp sums, coefficient partials and c,
+  // barriers
   const size_t other = sizeof(float) * 2 * (size_t)(P > 1 ? bt.D : 0) +
-                       sizeof(float2) * ((size_t)redn + 2 * (size_t)rows_cap +
-                                         2 * WB_ROWS * LZ_CW + (size_t)(LZ_CW + 1) * (bt.r + 1)) +
+                       sizeof(float2) * ((size_t)redn + (size_t)rows_cap + 16 * LZ_CW +
+                                         (size_t)(LZ_CW + 1) * (bt.r + 1)) +
                        16 + 2 * RING_MAX_STAGES * 8;
   const size_t limit = 227 * 1024 - 1024;  // leave room for static shared memory
   if (other >= limit) return SLS_ERR_UNSUPPORTED;
-  const RingShape R = ring_shape(bt.D, limit - other);
+  const RingShape R = ring_shape(bt.D, q_ld(bt.r), limit - other);
   if (R.S < 2) return SLS_ERR_UNSUPPORTED;
   const size_t smem = (size_t)R.S * R.stage + other;
   const int stages = R.S;

@@ -4,42 +4,41 @@
 // groups of CTAs; a group owns one problem at a time (one prompt, or one
 // adaptive window) and every CTA owns a contiguous strip of the problem's rows
 // of the feature matrix Phi (N x D, float32) and of the basis Q.  One copy warp
-// per CTA streams the Phi strip through a shared-memory ring with
-// one-dimensional bulk copies (cp.async.bulk + mbarrier), twice per step, and
-// runs ahead of the eight compute warps by as many chunks as the ring holds.
-// All work on basis rows happens in one dense row phase per step, with the
-// strip's rows split over the compute warps (register groups of rows, lanes
-// over the basis index, transposed butterflies for the row sums).
+// per CTA streams the strip through a shared-memory ring with one-dimensional
+// bulk copies (cp.async.bulk + mbarrier): each stage holds a few rows of Phi
+// and the same rows of Q.  Eight compute warps consume the ring.
 //
-// Step j (0-based) starts from z' (the new Lanczos direction before its
-// re-orthogonalisation; z' = q1 for j = 0) and the CTA partials of
-// c = Q^T z' (k < j) and |z'|^2 left by the previous row phase:
+// The whole run makes r passes over Phi: a prologue pass Phi^T q1, then one
+// fused pass per step but the last.  Step j starts from z' (the new Lanczos
+// direction before its re-orthogonalisation; z' = q1 for j = 0) and the CTA
+// partials of Phi^T z', of c = Q^T z' (k < j) and of |z'|^2:
 //
-//   sweep A (forward)   Phi^T z', column-parallel.
-//                       [barrier 1]
-//   slice phase         c = sum of the CTA partials; each CTA finishes a slice
-//                       of the D columns of Phi^T z1 = Phi^T z' - sum_k c_k w_k
-//                       with z1 = z' - Q c and w_k = Phi^T q_k kept from
-//                       earlier steps.
-//                       [barrier 2]
-//                       beta_{j-1} = |z1| = sqrt(|z'|^2 - |c|^2), the break
-//                       test, w_j = Phi^T q_j, alpha_j = |w_j|^2.
-//   sweep B (backward)  s = Phi w_j, the implicit matvec (Eq. implicit_matvec):
-//                       all compute threads share each chunk, w_j in registers.
-//   row phase           z1 = z' - Q c, q_j = z1 / beta_{j-1}, the three-term
-//                       recurrence z' = s - alpha_j q_j - beta_{j-1} q_{j-1},
-//                       and the partials of c = Q^T z' and |z'|^2 for step j+1.
+//   [barrier 1]
+//   slice phase   c = sum of the CTA partials; each CTA finishes a slice of the
+//                 D columns of Phi^T z1 = Phi^T z' - sum_k c_k w_k with
+//                 z1 = z' - Q c and w_k = Phi^T q_k kept from earlier steps.
+//   [barrier 2]
+//                 beta_{j-1} = |z1| = sqrt(|z'|^2 - |c|^2), the break test,
+//                 w_j = Phi^T q_j, alpha_j = |w_j|^2.
+//   fused pass    per pair of ring chunks: z1 = z' - Q c and q_j = z1 / beta
+//                 for its rows; the implicit matvec rows s = Phi w_j (Eq.
+//                 implicit_matvec, all compute threads on each row, w_j in
+//                 registers); the three-term recurrence z' = s - alpha_j q_j -
+//                 beta_{j-1} q_{j-1} with its partials of c and |z'|^2; and
+//                 the columns Phi^T z' of the next step, from the same rows
+//                 while they are in shared memory.
 //
-// This is Algorithm 2 with full re-orthogonalisation by one classical
-// Gram-Schmidt pass per step, applied to Phi^T z' through the stored w_k so
-// that the two passes over Phi per step are pure streams and a step needs two
-// group barriers.  The projection c = Q^T z' of a fully re-orthogonalised
-// Lanczos run stays at rounding level, so a second pass would change z1 only
-// in the second order of the rounding unit.  Sweep B runs backward so the rows
-// sweep A touched last are still in L2.  Vectors are double-float (two
-// float32), every sum over N or D is compensated, reductions have a fixed
-// order (bit-reproducible runs).  Barriers and waits give up after a bounded
-// number of polls and report SLS_ERR_TIMEOUT through the status word.
+// The last step only forms q_{r-1}.  This is Algorithm 2 with full
+// re-orthogonalisation by one classical Gram-Schmidt pass per step, applied to
+// Phi^T z' through the stored w_k so that one pass over Phi per step carries
+// both halves of the matvec.  The projection c = Q^T z' of a fully
+// re-orthogonalised Lanczos run stays at rounding level, so a second pass
+// would change z1 only in the second order of the rounding unit.  Passes
+// alternate direction so each starts on the rows the previous one left in
+// L2.  Vectors are double-float (two float32), every sum over N or D is
+// compensated, reductions have a fixed order (bit-reproducible runs).
+// Barriers and waits give up after a bounded number of polls and report
+// SLS_ERR_TIMEOUT through the status word.
 //
 // The kernel is a template over GPT (float4 column groups of Phi per compute
 // thread) and KT (32-wide tiles of the basis index k < r per lane); each
@@ -94,19 +93,20 @@ SLS_DEV dfloat shfl_df(dfloat v, int src) {
   return v;
 }
 
-// Ring stage: cr rows of Phi (cr * D floats).  For D >= 4 * LZ_CT (one
-// column group per compute thread or more) a stage holds TEAM_ELEMS / D rows,
-// so that sweep B can give every compute thread the same number of elements
-// per chunk; smaller D takes as many rows as fit RING_STAGE bytes.
+// Ring stage: cr rows of Phi (cr * D floats) followed by the same cr rows of
+// the basis Q (cr * ldq float2).  For D >= 4 * LZ_CT (one column group per
+// compute thread or more) a stage holds team_rows(GPT) rows, so that the team
+// row dots give every compute thread the same number of elements per chunk;
+// smaller D takes as many rows as fit RING_STAGE bytes.
 struct RingShape {
   int cr;          // rows per chunk
   int S;           // stages
+  unsigned phib;   // bytes of Phi per full chunk
   unsigned stage;  // bytes per stage
 };
 
 constexpr int RING_STAGE = 32 * 1024;
 constexpr int RING_MAX_STAGES = 8;
-constexpr int WB_ROWS = 64;  // rows per window of sweep-B warp partials
 constexpr int SLICE_LOADS = 5;  // per-CTA values per lane in flight in warp sums (g <= 160)
 
 // float4 column groups per compute thread, rounded up to a power of two
@@ -115,19 +115,20 @@ __host__ __device__ inline int gpt_of(int D) {
   const int need = (D / 4 + LZ_CT - 1) / LZ_CT;
   return need <= 1 ? 1 : need <= 2 ? 2 : need <= 4 ? 4 : need <= 8 ? 8 : 0;
 }
-// rows per chunk of the team sweep B: 8 / GPT (GPT * 4 * rows = 32 elements
+// rows per chunk of the team row dots: 8 / GPT (GPT * 4 * rows = 32 elements
 // per thread per chunk)
 __host__ __device__ constexpr int team_rows(int gpt) { return gpt >= 8 ? 1 : 8 / gpt; }
 
-__host__ __device__ inline RingShape ring_shape(int D, size_t budget) {
+__host__ __device__ inline RingShape ring_shape(int D, int ldq, size_t budget) {
   RingShape R;
   if (D / 4 >= LZ_CT) {
     R.cr = team_rows(gpt_of(D));
   } else {
-    R.cr = RING_STAGE / (4 * D);
+    R.cr = RING_STAGE / (4 * D + 8 * ldq);
     if (R.cr < 1) R.cr = 1;
   }
-  R.stage = (unsigned)R.cr * (unsigned)D * 4u;
+  R.phib = (unsigned)R.cr * (unsigned)D * 4u;
+  R.stage = R.phib + (unsigned)R.cr * (unsigned)ldq * 8u;
   R.S = (int)(budget / R.stage);
   if (R.S > RING_MAX_STAGES) R.S = RING_MAX_STAGES;
   return R;
@@ -195,10 +196,10 @@ SLS_DEV float transpose_sum_f(float (&v)[CR]) {
   return v[0];
 }
 
-// Sweep A over two ring chunks at once (D >= 4 * LZ_CT; CR rows each, the
-// second chunk may be absent: nr1 = 0) with offset accumulators: ah starts at
-// the power-of-two offset of the column sums.  FULL: both chunks full and
-// D = 4 LZ_CT GPT (the steady state), so the row and column guards vanish.
+// Column pass over two ring chunks at once (D >= 4 * LZ_CT; CR rows each, the
+// second chunk may be absent: nr1 = 0): acc[c] += Phi[i, c] * z'_i, Dot2.
+// FULL: both chunks full and D = 4 LZ_CT GPT (the steady state), so the row
+// and column guards vanish.
 template <int GPT, int CR, bool FULL>
 SLS_DEV void sweepA_team_pair(const float* __restrict__ c0, int nr0, int lb0,
                               const float* __restrict__ c1, int nr1, int lb1, int C4,
@@ -218,8 +219,8 @@ SLS_DEV void sweepA_team_pair(const float* __restrict__ c0, int nr0, int lb0,
         const int cg = tid + q * LZ_CT;
         if (FULL || cg < C4) {
           const float4 f = c4[ii * C4 + cg];
-          ofs_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
-          ofs_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
+          dot2_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
+          dot2_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
         }
       }
     }
@@ -516,6 +517,78 @@ SLS_DEV float group_correction(const float2 (&q)[RG][KT], const float2 (&cv)[KT]
   return transpose_sum_f<RG>(v);
 }
 
+// sum_{k < K} qrow[k] * c[k] over the warp (lanes over k), float32: the
+// coefficients are at rounding level; every lane gets the result.
+template <int KT>
+SLS_DEV float row_corr(const float2* __restrict__ qrow, const float2* __restrict__ c, int K) {
+  const int lane = threadIdx.x & 31;
+  float s = 0.f;
+#pragma unroll
+  for (int kt = 0; kt < KT; ++kt) {
+    const int k = lane + 32 * kt;
+    if (k < K) {
+      const float2 q = qrow[k], cc = c[k];
+      s = fmaf(q.x, cc.x, fmaf(q.x, cc.y, fmaf(q.y, cc.x, s)));
+    }
+  }
+  return warp_sum_f(s);
+}
+
+// Block sum of a double-float per-thread partial into *dst (tmpw: LZ_CW
+// shared scratch).
+SLS_DEV void store_cta_sum(dfloat acc, float2* tmpw, float2* __restrict__ dst) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  acc = df_norm(acc.hi, acc.lo);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc = df_add_fast(acc, shfl_xor_df(acc, o));
+  if (lane == 0) tmpw[warp] = f2(acc);
+  named_sync(BAR_COMPUTE, LZ_CT);
+  if (tid == 0) {
+    dfloat t = df_make(0.f, 0.f);
+    for (int w = 0; w < LZ_CW; ++w) t = df_add(t, dfv(tmpw[w]));
+    *dst = f2(t);
+  }
+  named_sync(BAR_COMPUTE, LZ_CT);
+}
+
+// The CTA's column partials of Phi^T z' (accumulators of the column pass, with
+// offset C, zero for Dot2) to dst[0 .. D): directly for P = 1, through the P
+// row-phase sums in red otherwise.
+template <int GPT>
+SLS_DEV void store_col_partials(const f32x2_t (&ah)[GPT][2], const f32x2_t (&al)[GPT][2],
+                                float C, int P, int C4, int D, float2* __restrict__ dst,
+                                float2* __restrict__ red) {
+  const int tid = threadIdx.x;
+  const int ph = (P == 1) ? 0 : tid / C4;
+  const int cb = (P == 1) ? tid : tid % C4;
+  float2* d = (P == 1) ? dst : red + (size_t)ph * D;
+  if (P == 1 || tid < P * C4) {
+#pragma unroll
+    for (int q = 0; q < GPT; ++q) {
+      const int cg = cb + q * LZ_CT;
+      if (cg < C4) {
+        float h0, h1, l0, l1, h2, h3, l2, l3;
+        upk2(ah[q][0], h0, h1);
+        upk2(al[q][0], l0, l1);
+        upk2(ah[q][1], h2, h3);
+        upk2(al[q][1], l2, l3);
+        d[4 * cg + 0] = f2(df_norm(h0 - C, l0));
+        d[4 * cg + 1] = f2(df_norm(h1 - C, l1));
+        d[4 * cg + 2] = f2(df_norm(h2 - C, l2));
+        d[4 * cg + 3] = f2(df_norm(h3 - C, l3));
+      }
+    }
+  }
+  if (P > 1) {
+    named_sync(BAR_COMPUTE, LZ_CT);
+    for (int col = tid; col < D; col += LZ_CT) {
+      dfloat s = df_make(0.f, 0.f);
+      for (int q = 0; q < P; ++q) s = df_add(s, dfv(red[(size_t)q * D + col]));
+      dst[col] = f2(s);
+    }
+  }
+}
+
 // Row phase of step j for the warp's rows [wr0, wr1) of the strip, in groups
 // of RG rows held in registers (lanes over the basis index k):
 //   z1 = z' - Q c                    (the re-orthogonalisation, c = Q^T z'
@@ -585,34 +658,13 @@ SLS_DEV void row_phase(float2* __restrict__ Qs, int ldq, int wr0, int wr1, int j
   }
 }
 
-// Block sums of a CTA: |z'|^2 (double-float, to *dst) and sum |z'| (per-warp
-// values in s_red1, added by their readers).
-SLS_DEV void store_cta_sums(dfloat nacc, float zl1, float2* tmpw, float* s_red1,
-                            float2* __restrict__ dst) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  nacc = df_norm(nacc.hi, nacc.lo);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) nacc = df_add_fast(nacc, shfl_xor_df(nacc, o));
-  zl1 = warp_sum_f(zl1);
-  if (lane == 0) {
-    tmpw[warp] = f2(nacc);
-    s_red1[warp] = zl1;
-  }
-  named_sync(BAR_COMPUTE, LZ_CT);
-  if (tid == 0) {
-    dfloat t = df_make(0.f, 0.f);
-    for (int w = 0; w < LZ_CW; ++w) t = df_add(t, dfv(tmpw[w]));
-    *dst = f2(t);
-  }
-}
-
 template <int GPT, int KT>
 __global__ void __launch_bounds__(LZ_THREADS, 1)
 lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroups,
                int rows_cap, int ring_stages, int* status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ float2 tmpw[LZ_CW];
-  __shared__ float s_red1[LZ_CW];  // per-warp max |Phi| and sum |z'| (offset bounds)
+  __shared__ float s_red1[LZ_CW];  // per-warp max |Phi| (offset bounds)
   __shared__ double shd[4];
   __shared__ int sflag, sbreak;
   // copy warp <-> compute warps handshake (no named barrier involves the copy
@@ -620,11 +672,13 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   // bar.sync; every wait on these flags is bounded)
   __shared__ volatile int s_halt;        // compute -> copy: stop issuing this problem
   __shared__ volatile int s_go;          // compute -> copy: may start problem s_go - 1
+  __shared__ volatile int s_pass;        // compute -> copy: passes completed (+ 256 per problem)
   __shared__ volatile int s_pdone;       // copy -> compute: finished problem s_pdone - 1
   __shared__ volatile unsigned s_issued;  // copy -> compute: chunks issued so far
   __shared__ volatile int s_err;          // a wait of this CTA gave up
 
   constexpr int TCR = team_rows(GPT);
+  constexpr int RPW = (2 * TCR + LZ_CW - 1) / LZ_CW;  // rows of a chunk pair per warp
   const int D = bt.D, r = bt.r, ldq = q_ld(bt.r);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int gi = blockIdx.x / g, rank = blockIdx.x % g;
@@ -633,20 +687,19 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   const int redn = (P > 1) ? P * D : 0;
   const bool fullD = (C4 == GPT * LZ_CT);  // no ragged column groups
 
-  const RingShape shp0 = ring_shape(D, 0);
+  const RingShape shp0 = ring_shape(D, ldq, 0);
   const int S = ring_stages;
   const int cr = shp0.cr;
-  const unsigned stage = shp0.stage;
+  const unsigned stage = shp0.stage, phib = shp0.phib;
   unsigned char* ring = smem_raw;
   unsigned char* after_ring = smem_raw + (size_t)S * stage;
   const int wn = (P > 1) ? D : 0;                      // w_j staged for row_dot_smem
   float* wsh = reinterpret_cast<float*>(after_ring);   // wn
   float* wsl = wsh + wn;                               // wn
   float2* red = reinterpret_cast<float2*>(wsl + wn);   // redn
-  float2* sv = red + redn;                             // rows_cap (s = Phi w_j of the strip)
-  float2* zps = sv + rows_cap;                         // rows_cap (z' of the strip)
-  float2* bpart = zps + rows_cap;                      // 2 x WB_ROWS x LZ_CW
-  float2* cw = bpart + 2 * WB_ROWS * LZ_CW;            // LZ_CW x (r+1)
+  float2* zps = red + redn;                            // rows_cap (z' of the strip)
+  float2* bpart = zps + rows_cap;                      // 16 x LZ_CW (row-dot warp sums)
+  float2* cw = bpart + 16 * LZ_CW;                     // LZ_CW x (r+1)
   float2* cs = cw + (size_t)LZ_CW * (r + 1);           // r+1 (c = Q^T z')
   uint64_t* bars = reinterpret_cast<uint64_t*>(
       (reinterpret_cast<uintptr_t>(cs + (r + 1)) + 15) & ~(uintptr_t)15);
@@ -672,6 +725,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     mbar_fence_init();
     s_halt = 0;
     s_go = 0;
+    s_pass = 0;
     s_pdone = 0;
     s_issued = 0;
     s_err = 0;
@@ -681,8 +735,11 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   const int nprob = nprob_of(bt);
 
   // ========================= copy warp ======================================
-  // Phi is read-only, so the copy warp runs ahead of the compute warps by as
-  // many chunks as the ring holds: sweep A forward, sweep B backward, per step.
+  // Streams r passes over the strip per problem (the prologue pass and one
+  // fused pass per step but the last), alternating direction so that each
+  // pass starts on the rows the previous one left in L2.  Each ring stage
+  // holds rows of Phi and the same rows of the basis Q; a pass is fetched only
+  // once the previous pass has written its column of Q.
   if (warp == LZ_CW) {
     if (lane != 0) return;
     const uint64_t pol = l2_policy_normal();
@@ -706,31 +763,47 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
       const int nch = (int)((re - rs + cr - 1) / cr);
       const float* Phi = bt.Phi + (row0 + rs) * D;
+      const float2* Qs = bt.Q + (row0 + rs) * ldq;
       bool stop = false;
-      for (int j = 0; j < r && !stop; ++j) {
-        for (int sweep = 0; sweep < 2 && !stop; ++sweep) {
-          for (int t = 0; t < nch; ++t) {
-            if (s_halt) {
-              stop = true;
+      for (int pass = 0; pass < r && !stop; ++pass) {
+        if (pass > 0) {
+          const int need = pp * 256 + pass;
+          bool open = false;
+          for (unsigned it = 0; it < (1u << 26); ++it) {
+            if (s_halt) break;
+            if (s_pass >= need) {
+              open = true;
               break;
             }
-            const int k = (sweep == 0) ? t : nch - 1 - t;
-            const int slot = (int)(cnt % (unsigned)S);
-            const unsigned par = (cnt / (unsigned)S) & 1u;
-            if (!mbar_wait(&emptyb[slot], par ^ 1u)) {
-              lz_fail(status, &s_err);
-              stop = true;
-              break;
-            }
-            const int64_t nr = min((int64_t)cr, (re - rs) - (int64_t)k * cr);
-            const unsigned b1 = (unsigned)(nr * D * 4);
-            unsigned char* dst = ring + (size_t)slot * stage;
-            mbar_expect_tx(&fullb[slot], b1);
-            bulk_g2s(dst, Phi + (int64_t)k * cr * D, b1, &fullb[slot], pol);
-            ++cnt;
-            __threadfence_block();
-            s_issued = cnt;
+            __nanosleep(32);
           }
+          if (!open) {
+            if (!s_halt) lz_fail(status, &s_err);
+            break;
+          }
+        }
+        for (int t = 0; t < nch; ++t) {
+          if (s_halt) {
+            stop = true;
+            break;
+          }
+          const int k = (pass & 1) ? nch - 1 - t : t;
+          const int slot = (int)(cnt % (unsigned)S);
+          const unsigned par = (cnt / (unsigned)S) & 1u;
+          if (!mbar_wait(&emptyb[slot], par ^ 1u)) {
+            lz_fail(status, &s_err);
+            stop = true;
+            break;
+          }
+          const int64_t nr = min((int64_t)cr, (re - rs) - (int64_t)k * cr);
+          const unsigned b1 = (unsigned)(nr * D * 4), b2 = (unsigned)(nr * ldq * 8);
+          unsigned char* dst = ring + (size_t)slot * stage;
+          mbar_expect_tx(&fullb[slot], b1 + b2);
+          bulk_g2s(dst, Phi + (int64_t)k * cr * D, b1, &fullb[slot], pol);
+          bulk_g2s(dst + phib, Qs + (int64_t)k * cr * ldq, b2, &fullb[slot], pol);
+          ++cnt;
+          __threadfence_block();
+          s_issued = cnt;
         }
       }
       __threadfence_block();
@@ -768,126 +841,48 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
 
     double scale = 0.0, alpha_prev = 0.0;
     dfloat alpha_df = df_make(0.f, 0.f), beta_df = df_make(0.f, 0.f), invb_df;
-    float phimax = 0.f;  // max |Phi| over this CTA's strip (step 0, sweep A)
+    float phimax = 0.f;  // max |Phi| over this CTA's strip (prologue pass)
     int reff = 0;
     sbreak = 0;
 
-    // step 0 starts from z' = q1: its partials |z'|^2 and sum |z'|
+    // ---------------- prologue: z' = q1, |z'|^2 and Phi^T z' (pass 0) ------------
     {
       dfloat nacc = df_make(0.f, 0.f);
-      float zl1 = 0.f;
       for (int il = tid; il < nrows; il += LZ_CT) {
         const dfloat z = df_from_double(q1[rs + il]);
         zps[il] = f2(z);
         dot2_acc_df(nacc.hi, nacc.lo, z, z);
-        zl1 += fabsf(z.hi);
       }
-      store_cta_sums(nacc, zl1, tmpw, s_red1, npart + (size_t)rank);
+      store_cta_sum(nacc, tmpw, npart + (size_t)rank);
+      f32x2_t ah[GPT][2], al[GPT][2];
+#pragma unroll
+      for (int q = 0; q < GPT; ++q) ah[q][0] = ah[q][1] = al[q][0] = al[q][1] = 0ull;
+      float mx = 0.f;
+      for (int t = 0; t < nch; ++t) {
+        const int slot = rc.slot;
+        if (!mbar_wait(&fullb[slot], rc.par)) lz_fail(status, &s_err);
+        const float* chunk = reinterpret_cast<const float*>(ring + (size_t)slot * stage);
+        const int nr = min(cr, nrows - t * cr);
+        sweepA_chunk<GPT, true>(chunk, nr, D, t * cr, zps, ah, al, &mx);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&emptyb[slot]);
+        rc_next(rc, S);
+      }
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      if (lane == 0) s_red1[warp] = mx;
+      store_col_partials<GPT>(ah, al, 0.f, P, C4, D, wpart + (size_t)rank * D, red);
+      named_sync(BAR_COMPUTE, LZ_CT);
+      if (tid == 0) {
+        __threadfence_block();
+        s_pass = pp * 256 + 1;
+      }
     }
 
     for (int j = 0; j < r; ++j) {
-      // ---------------- sweep A (forward): Phi^T z' ------------------------------
-      {
-        // offset for the column sums: all partial sums of Phi^T z' over the
-        // strip are bounded by max|Phi| * sum_i |z'_i|
-        const bool ofsA = (P == 1) && (j > 0);
-        float Ca = 0.f;
-        if (ofsA) {
-          float z1sum = 0.f;
-#pragma unroll
-          for (int w = 0; w < LZ_CW; ++w) z1sum += s_red1[w];
-          Ca = ofs_pow2(phimax * z1sum);
-        }
-        f32x2_t ah[GPT][2], al[GPT][2];
-        const f32x2_t a0 = pk2(Ca, Ca);
-#pragma unroll
-        for (int q = 0; q < GPT; ++q) {
-          ah[q][0] = ah[q][1] = a0;
-          al[q][0] = al[q][1] = 0ull;
-        }
-        float mx = 0.f;
-        if (ofsA) {
-          // two chunks per pass: more independent rows in flight per thread
-          for (int t = 0; t < nch; t += 2) {
-            const bool two = t + 1 < nch;
-            const int s0 = rc.slot;
-            if (!mbar_wait(&fullb[s0], rc.par)) lz_fail(status, &s_err);
-            rc_next(rc, S);
-            int s1 = s0;
-            if (two) {
-              s1 = rc.slot;
-              if (!mbar_wait(&fullb[s1], rc.par)) lz_fail(status, &s_err);
-              rc_next(rc, S);
-            }
-            const float* ch0 = reinterpret_cast<const float*>(ring + (size_t)s0 * stage);
-            const float* ch1 = reinterpret_cast<const float*>(ring + (size_t)s1 * stage);
-            const int nr0 = min(cr, nrows - t * cr);
-            const int nr1 = two ? min(cr, nrows - (t + 1) * cr) : 0;
-            if (fullD && nr0 == TCR && nr1 == TCR)
-              sweepA_team_pair<GPT, TCR, true>(ch0, nr0, t * cr, ch1, nr1, (t + 1) * cr, C4, zps, ah, al);
-            else
-              sweepA_team_pair<GPT, TCR, false>(ch0, nr0, t * cr, ch1, nr1, (t + 1) * cr, C4, zps, ah, al);
-            __syncwarp();
-            if (lane == 0) {
-              mbar_arrive(&emptyb[s0]);
-              if (two) mbar_arrive(&emptyb[s1]);
-            }
-          }
-        } else {
-          for (int t = 0; t < nch; ++t) {
-            const int slot = rc.slot;
-            if (!mbar_wait(&fullb[slot], rc.par))
-              lz_fail(status, &s_err);  // leave at the next group barrier
-            const float* chunk = reinterpret_cast<const float*>(ring + (size_t)slot * stage);
-            const int nr = min(cr, nrows - t * cr);
-            if (j == 0)
-              sweepA_chunk<GPT, true>(chunk, nr, D, t * cr, zps, ah, al, &mx);
-            else
-              sweepA_chunk<GPT, false>(chunk, nr, D, t * cr, zps, ah, al, &mx);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&emptyb[slot]);
-            rc_next(rc, S);
-          }
-        }
-        if (j == 0) {
-          for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-          named_sync(BAR_COMPUTE, LZ_CT);  // s_red1 (sum |z'|) has been read
-          if (lane == 0) s_red1[warp] = mx;
-        }
-        // CTA partial of Phi^T z'
-        const int ph = (P == 1) ? 0 : tid / C4;
-        const int cb = (P == 1) ? tid : tid % C4;
-        float2* dst = (P == 1) ? wpart + (size_t)rank * D : red + (size_t)ph * D;
-        if (P == 1 || tid < P * C4) {
-#pragma unroll
-          for (int q = 0; q < GPT; ++q) {
-            const int cg = cb + q * LZ_CT;
-            if (cg < C4) {
-              float h0, h1, l0, l1, h2, h3, l2, l3;
-              upk2(ah[q][0], h0, h1);
-              upk2(al[q][0], l0, l1);
-              upk2(ah[q][1], h2, h3);
-              upk2(al[q][1], l2, l3);
-              dst[4 * cg + 0] = f2(df_norm(h0 - Ca, l0));
-              dst[4 * cg + 1] = f2(df_norm(h1 - Ca, l1));
-              dst[4 * cg + 2] = f2(df_norm(h2 - Ca, l2));
-              dst[4 * cg + 3] = f2(df_norm(h3 - Ca, l3));
-            }
-          }
-        }
-        if (P > 1) {
-          named_sync(BAR_COMPUTE, LZ_CT);
-          for (int col = tid; col < D; col += LZ_CT) {
-            dfloat s = df_make(0.f, 0.f);
-            for (int q = 0; q < P; ++q) s = df_add(s, dfv(red[(size_t)q * D + col]));
-            wpart[(size_t)rank * D + col] = f2(s);
-          }
-        }
-      }
       if (!group_sync_named(bar, lgen, status, &sflag, &s_err, BAR_COMPUTE, LZ_CT)) return;
 
       // ---------------- slice phase: c, Phi^T z1 for this CTA's columns ----------
-      // c = Q^T z' (k < j) from the partials of the previous row phase;
+      // c = Q^T z' (k < j) from the partials of the previous pass;
       // Phi^T z1 = Phi^T z' - sum_k c_k w_k with w_k = Phi^T q_k kept in Wm.
       reduce_coeffs(cpart, g, r, j, cs);
       {
@@ -962,30 +957,57 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
 #pragma unroll
         for (int w = 0; w < LZ_CW; ++w) phimax = fmaxf(phimax, s_red1[w]);
       }
-      // w_j = (Phi^T z1) / beta: into shared memory for the row-per-warp
-      // sweep B (D < 4 LZ_CT; the team sweep takes its columns straight into
+
+      if (j == r - 1) {
+        // the last step needs no pass over Phi: q_{r-1} = z1 / beta_{r-2}
+        dfloat cacc[KT];
+#pragma unroll
+        for (int t = 0; t < KT; ++t) cacc[t] = df_make(0.f, 0.f);
+        dfloat nacc = df_make(0.f, 0.f);
+        float zl1 = 0.f;
+        row_phase<KT>(Qs, ldq, wr0, wr1, j, true, cs, zps, zps, invb_df, alpha_df, beta_df, cacc,
+                      nacc, zl1);
+        reff = r;
+        break;
+      }
+
+      // w_j = (Phi^T z1) / beta: into shared memory for the row-per-warp row
+      // dots (D < 4 LZ_CT; the team row dots take their columns straight into
       // registers below); keep w_j (slice) for the correction of later steps
-      if (P > 1) for (int c0 = tid; c0 < D; c0 += 8 * LZ_CT) {
-        float2 wv[8];
+      if (P > 1) {
+        for (int c0 = tid; c0 < D; c0 += 8 * LZ_CT) {
+          float2 wv[8];
 #pragma unroll
-        for (int m = 0; m < 8; ++m) {
-          const int c = c0 + m * LZ_CT;
-          wv[m] = (c < D) ? wred[c] : make_float2(0.f, 0.f);
-        }
+          for (int m = 0; m < 8; ++m) {
+            const int c = c0 + m * LZ_CT;
+            wv[m] = (c < D) ? wred[c] : make_float2(0.f, 0.f);
+          }
 #pragma unroll
-        for (int m = 0; m < 8; ++m) {
-          const int c = c0 + m * LZ_CT;
-          if (c < D) {
-            const dfloat a = df_mul(dfv(wv[m]), invb_df);
-            wsh[c] = a.hi;
-            wsl[c] = a.lo;
-            if (c >= cbeg && c < cend) Wm[(size_t)j * D + c] = f2(a);
+          for (int m = 0; m < 8; ++m) {
+            const int c = c0 + m * LZ_CT;
+            if (c < D) {
+              const dfloat a = df_mul(dfv(wv[m]), invb_df);
+              wsh[c] = a.hi;
+              wsl[c] = a.lo;
+              if (c >= cbeg && c < cend) Wm[(size_t)j * D + c] = f2(a);
+            }
           }
         }
+        named_sync(BAR_COMPUTE, LZ_CT);
       }
-      if (P > 1) named_sync(BAR_COMPUTE, LZ_CT);
 
-      // ---------------- sweep B (backward): s = Phi w_j per row -----------------
+      // ---------------- fused pass j+1 over Phi ----------------------------------
+      // per chunk (pair): z1 = z' - Q c, q_j = z1 / beta_{j-1} (row work);
+      // s = Phi w_j (row dots); z' <- s - alpha_j q_j - beta_{j-1} q_{j-1} and
+      // its partials of c = Q^T z' and |z'|^2 (row work); Phi^T z' (columns).
+      const bool fwd = ((j + 1) & 1) == 0;
+      f32x2_t ah[GPT][2], al[GPT][2];
+#pragma unroll
+      for (int q = 0; q < GPT; ++q) ah[q][0] = ah[q][1] = al[q][0] = al[q][1] = 0ull;
+      dfloat cacc[KT];
+#pragma unroll
+      for (int t = 0; t < KT; ++t) cacc[t] = df_make(0.f, 0.f);
+      dfloat nacc = df_make(0.f, 0.f);
       if (P == 1) {
         // this thread's columns of w_j, from the slices into registers
         f32x2_t wh[GPT][2], nwh[GPT][2], wl[GPT][2];
@@ -1029,10 +1051,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         // offset of this thread's row partials: each is bounded by
         // max|Phi| * |w slice|_1
         const float Ct = ofs_pow2(phimax * wt1);
-        constexpr int WCH = WB_ROWS / TCR;  // chunks per window (even)
         for (int t0p = 0; t0p < nch; t0p += 2) {
           const bool two = t0p + 1 < nch;
-          const int kc0 = nch - 1 - t0p;
+          const int kc0 = fwd ? t0p : nch - 1 - t0p;
+          const int kc1 = fwd ? t0p + 1 : nch - 2 - t0p;
           const int s0 = rc.slot;
           if (!mbar_wait(&fullb[s0], rc.par)) lz_fail(status, &s_err);
           rc_next(rc, S);
@@ -1044,76 +1066,132 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           }
           const float* ch0 = reinterpret_cast<const float*>(ring + (size_t)s0 * stage);
           const float* ch1 = reinterpret_cast<const float*>(ring + (size_t)s1 * stage);
+          const float2* qb0 = reinterpret_cast<const float2*>(ring + (size_t)s0 * stage + phib);
+          const float2* qb1 = reinterpret_cast<const float2*>(ring + (size_t)s1 * stage + phib);
           const int nr0 = min(cr, nrows - kc0 * cr);
-          const int nr1 = two ? cr : 0;
-          const int win = t0p / WCH, tw0 = t0p % WCH;
-          float2* bp0 = bpart + (size_t)((win & 1) * WB_ROWS + tw0 * TCR) * LZ_CW;
-          float2* bp1 = bp0 + (size_t)TCR * LZ_CW;
+          const int nr1 = two ? min(cr, nrows - kc1 * cr) : 0;
+          // row work before the row dots: q_j of the warp's rows of the pair
+          dfloat qjv[RPW];
+          float2 qpv[RPW];
+#pragma unroll
+          for (int m = 0; m < RPW; ++m) {
+            const int ri = warp + m * LZ_CW;
+            const bool first = ri < TCR;
+            const int ii = first ? ri : ri - TCR;
+            qjv[m] = df_make(0.f, 0.f);
+            qpv[m] = make_float2(0.f, 0.f);
+            if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
+              const int il = (first ? kc0 : kc1) * cr + ii;
+              const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
+              const float corr = row_corr<KT>(qrow, cs, j);
+              dfloat z1 = dfv(zps[il]);
+              if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
+              qjv[m] = df_mul(z1, invb_df);
+              if (j > 0) qpv[m] = qrow[j - 1];
+              if (lane == 0) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
+            }
+          }
+          // row dots s = Phi w_j, warp sums into bpart[row * LZ_CW + warp]
           if (fullD && nr0 == TCR && nr1 == TCR)
-            sweepB_team_pair<GPT, TCR, true>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bp0, bp1);
+            sweepB_team_pair<GPT, TCR, true>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bpart,
+                                             bpart + TCR * LZ_CW);
           else
-            sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bp0, bp1);
+            sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bpart,
+                                              bpart + TCR * LZ_CW);
+          named_sync(BAR_COMPUTE, LZ_CT);
+          // row work after the row dots: z', its partials of c and |z'|^2
+#pragma unroll
+          for (int m = 0; m < RPW; ++m) {
+            const int ri = warp + m * LZ_CW;
+            const bool first = ri < TCR;
+            const int ii = first ? ri : ri - TCR;
+            if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
+              const int il = (first ? kc0 : kc1) * cr + ii;
+              const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
+              dfloat s = (lane < LZ_CW) ? dfv(bpart[ri * LZ_CW + lane]) : df_make(0.f, 0.f);
+#pragma unroll
+              for (int o = 16; o > 0; o >>= 1) s = df_add_fast(s, shfl_xor_df(s, o));
+              dfloat zp = df_sub(s, df_mul(alpha_df, qjv[m]));
+              if (j > 0) zp = df_sub(zp, df_mul(beta_df, dfv(qpv[m])));
+              if (lane == 0) {
+                zps[il] = f2(zp);
+                dot2_acc_df(nacc.hi, nacc.lo, zp, zp);
+              }
+#pragma unroll
+              for (int kt = 0; kt < KT; ++kt) {
+                const int k = lane + 32 * kt;
+                if (k <= j) {
+                  const dfloat qk = (k == j) ? qjv[m] : dfv(qrow[k]);
+                  dot2_acc_df(cacc[kt].hi, cacc[kt].lo, qk, zp);
+                }
+              }
+            }
+          }
+          named_sync(BAR_COMPUTE, LZ_CT);
+          // columns: Phi^T z' for the next step
+          if (fullD && nr0 == TCR && nr1 == TCR)
+            sweepA_team_pair<GPT, TCR, true>(ch0, nr0, kc0 * cr, ch1, nr1, kc1 * cr, C4, zps, ah, al);
+          else
+            sweepA_team_pair<GPT, TCR, false>(ch0, nr0, kc0 * cr, ch1, nr1, kc1 * cr, C4, zps, ah,
+                                              al);
           __syncwarp();
           if (lane == 0) {
             mbar_arrive(&emptyb[s0]);
             if (two) mbar_arrive(&emptyb[s1]);
           }
-          const int t = two ? t0p + 1 : t0p;  // last chunk of the pass
-          const int tw = t % WCH;
-          if (tw == WCH - 1 || t == nch - 1) {
-            // the window's warp partials are complete: one row per thread sums
-            // them (the summing threads rotate from window to window)
-            named_sync(BAR_COMPUTE, LZ_CT);
-            const int t0 = t - tw;
-            const int pidx = (tid - 64 * (win & 3) + LZ_CT) % LZ_CT;
-            if (pidx < (tw + 1) * TCR) {
-              const int il = (nch - 1 - (t0 + pidx / TCR)) * cr + pidx % TCR;
-              if (il < nrows) {
-                const float2* src = bpart + (size_t)((win & 1) * WB_ROWS + pidx) * LZ_CW;
-                dfloat s = df_make(0.f, 0.f);
-#pragma unroll
-                for (int w = 0; w < LZ_CW; ++w) s = df_add(s, dfv(src[w]));
-                sv[il] = f2(s);
-              }
-            }
-          }
         }
       } else {
+        float mx = 0.f;
         for (int t = 0; t < nch; ++t) {
-          const int kc = nch - 1 - t;
+          const int kc = fwd ? t : nch - 1 - t;
           const int slot = rc.slot;
           if (!mbar_wait(&fullb[slot], rc.par))
             lz_fail(status, &s_err);  // leave at the next group barrier
           const float* chunk = reinterpret_cast<const float*>(ring + (size_t)slot * stage);
+          const float2* qblk = reinterpret_cast<const float2*>(ring + (size_t)slot * stage + phib);
           const int nr = min(cr, nrows - kc * cr);
           for (int ii = warp; ii < nr; ii += LZ_CW) {
+            const int il = kc * cr + ii;
+            const float2* qrow = qblk + (size_t)ii * ldq;
+            const float corr = row_corr<KT>(qrow, cs, j);
+            dfloat z1 = dfv(zps[il]);
+            if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
+            const dfloat qj = df_mul(z1, invb_df);
+            if (lane == 0) Qs[(size_t)il * ldq + j] = f2(qj);
             const dfloat s = row_dot_smem(chunk + (size_t)ii * D, D, wsh, wsl);
-            if (lane == 0) sv[kc * cr + ii] = f2(s);
+            dfloat zp = df_sub(s, df_mul(alpha_df, qj));
+            if (j > 0) zp = df_sub(zp, df_mul(beta_df, dfv(qrow[j - 1])));
+            if (lane == 0) {
+              zps[il] = f2(zp);
+              dot2_acc_df(nacc.hi, nacc.lo, zp, zp);
+            }
+#pragma unroll
+            for (int kt = 0; kt < KT; ++kt) {
+              const int k = lane + 32 * kt;
+              if (k <= j) {
+                const dfloat qk = (k == j) ? qj : dfv(qrow[k]);
+                dot2_acc_df(cacc[kt].hi, cacc[kt].lo, qk, zp);
+              }
+            }
           }
+          named_sync(BAR_COMPUTE, LZ_CT);
+          sweepA_chunk<GPT, false>(chunk, nr, D, kc * cr, zps, ah, al, &mx);
           __syncwarp();
           if (lane == 0) mbar_arrive(&emptyb[slot]);
           rc_next(rc, S);
         }
       }
+      // partials for step j+1 (read after its barrier 1): Phi^T z', c, |z'|^2
+      store_col_partials<GPT>(ah, al, 0.f, P, C4, D, wpart + (size_t)rank * D, red);
+      store_coeff_partials(cacc, j + 1, r, cw, cpart + (size_t)rank * (r + 1));
+      store_cta_sum(nacc, tmpw, npart + (size_t)((j + 1) & 1) * g + rank);
+      // the column j of Q written in this pass reaches the copy warp's bulk
+      // reads of the next pass (async proxy)
+      if (lane == 0) asm volatile("fence.proxy.async.global;" ::: "memory");
       named_sync(BAR_COMPUTE, LZ_CT);
-
-      // ---------------- row phase: q_j, next z', partials of step j+1 --------------
-      const bool last = (j == r - 1);
-      {
-        dfloat cacc[KT];
-#pragma unroll
-        for (int t = 0; t < KT; ++t) cacc[t] = df_make(0.f, 0.f);
-        dfloat nacc = df_make(0.f, 0.f);
-        float zl1 = 0.f;
-        row_phase<KT>(Qs, ldq, wr0, wr1, j, last, cs, sv, zps, invb_df, alpha_df, beta_df, cacc,
-                      nacc, zl1);
-        if (last) {
-          reff = r;
-          break;
-        }
-        // partials for step j+1 (read after its barrier 1): c, |z'|^2, sum |z'|
-        store_coeff_partials(cacc, j + 1, r, cw, cpart + (size_t)rank * (r + 1));
-        store_cta_sums(nacc, zl1, tmpw, s_red1, npart + (size_t)((j + 1) & 1) * g + rank);
+      if (tid == 0) {
+        __threadfence_block();
+        s_pass = pp * 256 + j + 2;
       }
     }
     // a break leaves chunks issued ahead of it: consume them until the copy
