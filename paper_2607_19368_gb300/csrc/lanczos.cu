@@ -13,44 +13,63 @@ namespace sls {
 namespace {
 
 // ----------------------------------------------------------------------------
-// Eigenvalues of T: multisection on Sturm counts (float64)
+// Eigenvalues of T: multisection on Sturm counts.  The arithmetic of the
+// recurrences is double-float on the FP32 pipes: float64 on this part has a
+// 64-cycle dependent latency (and a divide of several hundred cycles), which
+// a serial recurrence pays at every step.
 // ----------------------------------------------------------------------------
+
+SLS_DEV dfloat df_div(dfloat a, dfloat b) {
+  const float q1 = __fdividef(a.hi, b.hi);
+  float p, e;
+  two_prod(q1, b.hi, p, e);
+  const float rr = (((a.hi - p) - e) + a.lo) - q1 * b.lo;
+  const float q2 = __fdividef(rr, b.hi);
+  return df_norm(q1, q2);
+}
+
+SLS_DEV dfloat df_scale(dfloat a, float s) { return df_make(a.hi * s, a.lo * s); }
 
 // Number of eigenvalues of the (scaled) tridiagonal below x, from the signs of
 // the leading principal minors p_i(x) (three-term recurrence, Sturm sequence).
 // Powers of two rescale the pair (p_{i-1}, p_i) to keep it in range; a zero
 // minor takes the sign opposite to its predecessor.
-SLS_DEV int sturm_count(const double* a, const double* b2, int n, double x) {
-  double pm = 1.0, pc = a[0] - x;
+SLS_DEV int sturm_count(const float2* __restrict__ a, const float2* __restrict__ b2, int n,
+                        dfloat x) {
+  dfloat pm = df_make(1.f, 0.f), pc = df_sub(dfv(a[0]), x);
   int sprev = 0;
-  int s = (pc < 0.0) ? 1 : ((pc > 0.0) ? 0 : 1);
+  int s = (pc.hi < 0.f) ? 1 : ((pc.hi > 0.f) ? 0 : 1);
   int cnt = (s != sprev);
   sprev = s;
   for (int i = 1; i < n; ++i) {
-    const double pn = fma(a[i] - x, pc, -b2[i - 1] * pm);
+    const dfloat d = df_sub(dfv(a[i]), x);
+    const dfloat t = df_mul(dfv(b2[i - 1]), pm);
+    const dfloat pn = df_sub(df_mul(d, pc), t);
     pm = pc;
     pc = pn;
-    const int ec = (__double2hiint(pc) >> 20) & 0x7ff;
-    const int em = (__double2hiint(pm) >> 20) & 0x7ff;
-    const int e = max(ec, em);
-    if (e > 1023 + 400) {
-      pc = pc * 0x1p-400;
-      pm = pm * 0x1p-400;
-    } else if (e < 1023 - 400) {
-      pc = pc * 0x1p400;
-      pm = pm * 0x1p400;
+    const float mg = fmaxf(fabsf(pc.hi), fabsf(pm.hi));
+    if (mg > 0x1p60f) {
+      pc = df_scale(pc, 0x1p-60f);
+      pm = df_scale(pm, 0x1p-60f);
+    } else if (mg < 0x1p-60f && mg > 0.f) {
+      pc = df_scale(pc, 0x1p60f);
+      pm = df_scale(pm, 0x1p60f);
     }
-    s = (pc < 0.0) ? 1 : ((pc > 0.0) ? 0 : 1 - sprev);
+    s = (pc.hi < 0.f) ? 1 : ((pc.hi > 0.f) ? 0 : 1 - sprev);
     cnt += (s != sprev);
     sprev = s;
   }
   return cnt;
 }
 
-__global__ void __launch_bounds__(32)
+constexpr int EIG_THREADS = 256;  // shifts per multisection round
+
+__global__ void __launch_bounds__(EIG_THREADS)
 tridiag_eigvals_kernel(LanczosBatch bt) {
-  __shared__ double sa[SLS_MAX_R], sb2[SLS_MAX_R];
-  const int m = blockIdx.x, p = blockIdx.y, lane = threadIdx.x;
+  __shared__ float2 sa[SLS_MAX_R], sb2[SLS_MAX_R];
+  __shared__ int s_first[EIG_THREADS / 32];
+  __shared__ double s_lo, s_hi, s_sc;
+  const int m = blockIdx.x, p = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int nprob = bt.nprob_max;
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
   if (p >= nprob) return;
@@ -58,67 +77,81 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
   const int n = bt.r_eff[p];
   double* theta = bt.theta + (size_t)p * r;
   if (m >= n) {
-    if (lane == 0) theta[m] = 0.0;
+    if (tid == 0) theta[m] = 0.0;
     return;
   }
   const double* a = bt.alpha + (size_t)p * r;
   const double* b = bt.beta + (size_t)p * r;
-  double glo = DBL_MAX, ghi = -DBL_MAX;
-  for (int i = lane; i < n; i += 32) {
-    const double bl = (i > 0) ? fabs(b[i - 1]) : 0.0;
-    const double br = (i < n - 1) ? fabs(b[i]) : 0.0;
-    glo = fmin(glo, a[i] - bl - br);
-    ghi = fmax(ghi, a[i] + bl + br);
-  }
+  if (warp == 0) {
+    // Gershgorin interval, and a power-of-two scale that maps it into [-1, 1]
+    double glo = DBL_MAX, ghi = -DBL_MAX;
+    for (int i = lane; i < n; i += 32) {
+      const double bl = (i > 0) ? fabs(b[i - 1]) : 0.0;
+      const double br = (i < n - 1) ? fabs(b[i]) : 0.0;
+      glo = fmin(glo, a[i] - bl - br);
+      ghi = fmax(ghi, a[i] + bl + br);
+    }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    glo = fmin(glo, __shfl_xor_sync(0xffffffffu, glo, o));
-    ghi = fmax(ghi, __shfl_xor_sync(0xffffffffu, ghi, o));
+    for (int o = 16; o > 0; o >>= 1) {
+      glo = fmin(glo, __shfl_xor_sync(0xffffffffu, glo, o));
+      ghi = fmax(ghi, __shfl_xor_sync(0xffffffffu, ghi, o));
+    }
+    if (lane == 0) {
+      const double big = fmax(fabs(glo), fabs(ghi));
+      int ex = 0;
+      frexp(big > 0.0 ? big : 1.0, &ex);
+      const double sc = ldexp(1.0, -ex);  // exact scaling
+      double lo = glo * sc, hi = ghi * sc;
+      const double pad = 0x1p-40 * fmax(fabs(lo), fabs(hi)) + 0x1p-100;
+      s_lo = lo - pad;
+      s_hi = hi + pad;
+      s_sc = sc;
+    }
   }
-  const double big = fmax(fabs(glo), fabs(ghi));
-  int ex = 0;
-  frexp(big > 0.0 ? big : 1.0, &ex);
-  const double sc = ldexp(1.0, -ex);  // power of two: exact scaling
-  for (int i = lane; i < n; i += 32) {
-    sa[i] = a[i] * sc;
+  __syncthreads();
+  const double sc = s_sc;
+  for (int i = tid; i < n; i += EIG_THREADS) {
+    sa[i] = f2(df_from_double(a[i] * sc));
     if (i < n - 1) {
       const double bs = b[i] * sc;
-      sb2[i] = bs * bs;
+      sb2[i] = f2(df_from_double(bs * bs));
     }
   }
-  __syncwarp();
-  double lo = glo * sc, hi = ghi * sc;
-  const double pad = 4.0 * DBL_EPSILON * fmax(fabs(lo), fabs(hi)) + DBL_MIN;
-  lo -= pad;
-  hi += pad;
+  __syncthreads();
   const int k = n - 1 - m;  // ascending index of the wanted eigenvalue
-  for (int round = 0; round < 64; ++round) {
-    const double x = lo + (hi - lo) * ((double)(lane + 1) / 33.0);
-    const int c = sturm_count(sa, sb2, n, x);
+  for (int round = 0; round < 40; ++round) {
+    const double lo = s_lo, hi = s_hi;
+    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-120) break;
+    const double x = lo + (hi - lo) * ((double)(tid + 1) / (double)(EIG_THREADS + 1));
+    const int c = sturm_count(sa, sb2, n, df_from_double(x));
     const unsigned ball = __ballot_sync(0xffffffffu, c > k);
-    if (ball == 0u) {
-      lo = __shfl_sync(0xffffffffu, x, 31);
-    } else {
-      const int f = __ffs(ball) - 1;
-      const double xf = __shfl_sync(0xffffffffu, x, f);
-      const double xl = __shfl_sync(0xffffffffu, x, f > 0 ? f - 1 : 0);
-      hi = xf;
-      if (f > 0) lo = xl;
+    if (lane == 0) s_first[warp] = ball ? warp * 32 + __ffs(ball) - 1 : EIG_THREADS;
+    __syncthreads();
+    if (tid == 0) {
+      int f = EIG_THREADS;
+      for (int w = 0; w < EIG_THREADS / 32; ++w) f = min(f, s_first[w]);
+      // count(x_t) is non-decreasing in t: the eigenvalue lies in (x_{f-1}, x_f]
+      const double step = (hi - lo) / (double)(EIG_THREADS + 1);
+      (void)step;
+      const double xf = lo + (hi - lo) * ((double)(f + 1) / (double)(EIG_THREADS + 1));
+      const double xp = lo + (hi - lo) * ((double)f / (double)(EIG_THREADS + 1));
+      if (f < EIG_THREADS) s_hi = xf;
+      if (f > 0) s_lo = xp;
     }
-    if (hi - lo <= 2.0 * DBL_EPSILON * fmax(fabs(lo), fabs(hi)) || hi - lo <= 2.0 * DBL_MIN)
-      break;
+    __syncthreads();
   }
-  if (lane == 0) theta[m] = (0.5 * (lo + hi)) / sc;
+  if (tid == 0) theta[m] = (0.5 * (s_lo + s_hi)) / sc;
 }
 
 // ----------------------------------------------------------------------------
-// Eigenvectors of T: inverse iteration (float64), MGS within clusters
+// Eigenvectors of T: inverse iteration with partial-pivoting LU (double-float),
+// modified Gram-Schmidt within clusters of close eigenvalues
 // ----------------------------------------------------------------------------
 
 __global__ void __launch_bounds__(32)
 tridiag_eigvecs_kernel(LanczosBatch bt) {
-  __shared__ double d[SLS_MAX_R], du[SLS_MAX_R], du2[SLS_MAX_R], dl[SLS_MAX_R];
-  __shared__ double y[SLS_MAX_R];
+  __shared__ float2 d[SLS_MAX_R], du[SLS_MAX_R], du2[SLS_MAX_R], dl[SLS_MAX_R];
+  __shared__ float2 y[SLS_MAX_R];
   __shared__ unsigned char piv[SLS_MAX_R];
   const int m = blockIdx.x, p = blockIdx.y, lane = threadIdx.x;
   int nprob = bt.nprob_max;
@@ -147,120 +180,182 @@ tridiag_eigvecs_kernel(LanczosBatch bt) {
   for (int k = lane + n; k < r; k += 32)
     for (int mm = first; mm <= last; ++mm) S[(size_t)k * r + mm] = 0.0;
   if (lane != 0) return;
-  const double pert = DBL_EPSILON * tnorm;
+  // a power-of-two scale of T (the eigenvectors do not change)
+  int ex = 0;
+  frexp(tnorm, &ex);
+  const double sc = ldexp(1.0, -ex);
+  const double pert = 0x1p-44 * tnorm * sc;
+  const dfloat pert_df = df_from_double(pert);
   for (int mm = first; mm <= last; ++mm) {
     // distinct shifts inside a cluster
-    const double shift = th[mm] - (double)(mm - first) * 4.0 * pert;
+    const dfloat shift = df_from_double((th[mm] - (double)(mm - first) * 4.0 * (pert / sc)) * sc);
     for (int i = 0; i < n; ++i) {
-      d[i] = a[i] - shift;
+      d[i] = f2(df_sub(df_from_double(a[i] * sc), shift));
       if (i < n - 1) {
-        du[i] = b[i];
-        dl[i] = b[i];
+        du[i] = f2(df_from_double(b[i] * sc));
+        dl[i] = du[i];
       }
-      du2[i] = 0.0;
+      du2[i] = make_float2(0.f, 0.f);
     }
     if (n == 1) {
-      y[0] = 1.0;
+      y[0] = make_float2(1.f, 0.f);
     } else {
       // LU with partial pivoting of T - shift I
       for (int i = 0; i < n - 1; ++i) {
-        if (fabs(d[i]) >= fabs(dl[i])) {
-          if (d[i] == 0.0) d[i] = pert;
-          const double f = dl[i] / d[i];
-          dl[i] = f;
-          d[i + 1] -= f * du[i];
+        dfloat di = dfv(d[i]);
+        const dfloat li = dfv(dl[i]);
+        if (fabsf(di.hi) >= fabsf(li.hi)) {
+          if (di.hi == 0.f) di = pert_df;
+          const dfloat f = df_div(li, di);
+          d[i] = f2(di);
+          dl[i] = f2(f);
+          d[i + 1] = f2(df_sub(dfv(d[i + 1]), df_mul(f, dfv(du[i]))));
           piv[i] = 0;
         } else {
-          const double f = d[i] / dl[i];
-          d[i] = dl[i];
-          dl[i] = f;
-          const double tmp = du[i];
-          du[i] = d[i + 1];
-          d[i + 1] = tmp - f * d[i + 1];
+          const dfloat f = df_div(di, li);
+          const dfloat dn = dfv(d[i + 1]);
+          d[i] = f2(li);
+          dl[i] = f2(f);
+          const dfloat tmp = dfv(du[i]);
+          du[i] = f2(dn);
+          d[i + 1] = f2(df_sub(tmp, df_mul(f, dn)));
           if (i < n - 2) {
             du2[i] = du[i + 1];
-            du[i + 1] = -f * du[i + 1];
+            du[i + 1] = f2(df_neg(df_mul(f, dfv(du[i + 1]))));
           }
           piv[i] = 1;
         }
       }
-      if (d[n - 1] == 0.0) d[n - 1] = pert;
+      if (d[n - 1].x == 0.f) d[n - 1] = f2(pert_df);
       // deterministic start vector
       for (int i = 0; i < n; ++i) {
         unsigned h = (unsigned)(i + 1) * 2654435761u ^ (unsigned)(mm + 7) * 40503u;
         h ^= h >> 13;
         h *= 0x5bd1e995u;
         h ^= h >> 15;
-        y[i] = 0.5 + (double)(h & 0xffffu) / 65536.0;
+        y[i] = make_float2(0.5f + (float)(h & 0xffffu) / 65536.f, 0.f);
       }
       for (int it = 0; it < 3; ++it) {
         for (int i = 0; i < n - 1; ++i) {
           if (!piv[i]) {
-            y[i + 1] -= dl[i] * y[i];
+            y[i + 1] = f2(df_sub(dfv(y[i + 1]), df_mul(dfv(dl[i]), dfv(y[i]))));
           } else {
-            const double t = y[i];
+            const dfloat t = dfv(y[i]);
             y[i] = y[i + 1];
-            y[i + 1] = t - dl[i] * y[i];
+            y[i + 1] = f2(df_sub(t, df_mul(dfv(dl[i]), dfv(y[i]))));
           }
         }
-        y[n - 1] /= d[n - 1];
-        y[n - 2] = (y[n - 2] - du[n - 2] * y[n - 1]) / d[n - 2];
-        for (int i = n - 3; i >= 0; --i)
-          y[i] = (y[i] - du[i] * y[i + 1] - du2[i] * y[i + 2]) / d[i];
+        y[n - 1] = f2(df_div(dfv(y[n - 1]), dfv(d[n - 1])));
+        y[n - 2] = f2(df_div(df_sub(dfv(y[n - 2]), df_mul(dfv(du[n - 2]), dfv(y[n - 1]))),
+                             dfv(d[n - 2])));
+        for (int i = n - 3; i >= 0; --i) {
+          const dfloat t = df_sub(df_sub(dfv(y[i]), df_mul(dfv(du[i]), dfv(y[i + 1]))),
+                                  df_mul(dfv(du2[i]), dfv(y[i + 2])));
+          y[i] = f2(df_div(t, dfv(d[i])));
+        }
+        // keep the iterate in range: divide by its largest entry (a power of two)
+        float ymax = 0.f;
+        for (int i = 0; i < n; ++i) ymax = fmaxf(ymax, fabsf(y[i].x));
+        if (ymax > 0.f && isfinite(ymax)) {
+          int e2 = 0;
+          frexpf(ymax, &e2);
+          const float s2 = ldexpf(1.f, -e2);
+          for (int i = 0; i < n; ++i) y[i] = f2(df_scale(dfv(y[i]), s2));
+        }
         // orthogonalise against the cluster members found so far
         for (int pm = first; pm < mm; ++pm) {
-          double dot = 0.0;
-          for (int i = 0; i < n; ++i) dot += S[(size_t)i * r + pm] * y[i];
-          for (int i = 0; i < n; ++i) y[i] -= dot * S[(size_t)i * r + pm];
+          dfloat dot = df_make(0.f, 0.f);
+          for (int i = 0; i < n; ++i)
+            dot = df_add(dot, df_mul(df_from_double(S[(size_t)i * r + pm]), dfv(y[i])));
+          for (int i = 0; i < n; ++i)
+            y[i] = f2(df_sub(dfv(y[i]), df_mul(dot, df_from_double(S[(size_t)i * r + pm]))));
         }
-        double nr = 0.0;
-        for (int i = 0; i < n; ++i) nr += y[i] * y[i];
-        nr = sqrt(nr);
+        dfloat nr2 = df_make(0.f, 0.f);
+        for (int i = 0; i < n; ++i) nr2 = df_add(nr2, df_mul(dfv(y[i]), dfv(y[i])));
+        const double nr = sqrt(df_to_double(nr2));
         if (!(nr > 0.0) || !isfinite(nr)) {
-          for (int i = 0; i < n; ++i) y[i] = (i == mm) ? 1.0 : 0.0;
-          nr = 1.0;
+          for (int i = 0; i < n; ++i) y[i] = make_float2((i == mm) ? 1.f : 0.f, 0.f);
+        } else {
+          const dfloat inv = df_from_double(1.0 / nr);
+          for (int i = 0; i < n; ++i) y[i] = f2(df_mul(dfv(y[i]), inv));
         }
-        const double inv = 1.0 / nr;
-        for (int i = 0; i < n; ++i) y[i] *= inv;
       }
     }
-    const double sg = (y[0] < 0.0) ? -1.0 : 1.0;
-    for (int i = 0; i < n; ++i) S[(size_t)i * r + mm] = sg * y[i];
+    const double sg = (y[0].x < 0.f) ? -1.0 : 1.0;
+    for (int i = 0; i < n; ++i) S[(size_t)i * r + mm] = sg * df_to_double(dfv(y[i]));
     __threadfence_block();
   }
 }
 
 // ----------------------------------------------------------------------------
-// Ritz vectors U = Q S (float32 output)
+// Ritz vectors U = Q S (float32 output): tiles of basis rows in shared memory,
+// 4 x 4 outputs per thread
 // ----------------------------------------------------------------------------
 
-__global__ void __launch_bounds__(256)
+constexpr int RITZ_THREADS = 256;
+
+__host__ __device__ inline int ritz_tile_rows(int r) {
+  const int cg = (r + 3) / 4;
+  return (RITZ_THREADS / cg) * 4;
+}
+
+__global__ void __launch_bounds__(RITZ_THREADS)
 ritz_vectors_kernel(LanczosBatch bt, float* __restrict__ U) {
-  extern __shared__ float Ss[];  // r x r
+  extern __shared__ float rsm[];
   const int p = blockIdx.y;
   int nprob = bt.nprob_max;
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
   if (p >= nprob) return;
-  const int r = bt.r;
+  const int r = bt.r, ldq = q_ld(r);
   const int kn = bt.r_eff[p];
   const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
   const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
+  const int cg = (r + 3) / 4, rg = RITZ_THREADS / cg, TR = rg * 4, qs = r + 1;
+  float* Ss = rsm;                    // r x r
+  float* Qh = Ss + (size_t)r * r;     // TR x (r+1)
+  float* Ql = Qh + (size_t)TR * qs;   // TR x (r+1)
   const double* S = bt.S + (size_t)p * r * r;
-  for (int e = threadIdx.x; e < r * r; e += blockDim.x) Ss[e] = (float)S[e];
-  __syncthreads();
-  const int rpb = blockDim.x / r;
-  const int sub = threadIdx.x / r, m = threadIdx.x % r;
-  if (sub >= rpb) return;
-  for (int64_t i = (int64_t)blockIdx.x * rpb + sub; i < n; i += (int64_t)gridDim.x * rpb) {
-    const float2* Qi = bt.Q + (row0 + i) * q_ld(r);
-    float acc = 0.f;
-    for (int k = 0; k < kn; ++k) {
-      const float2 q = Qi[k];
-      const float s = Ss[k * r + m];
-      acc = fmaf(q.x, s, acc);
-      acc = fmaf(q.y, s, acc);
+  for (int e = threadIdx.x; e < r * r; e += RITZ_THREADS) Ss[e] = (float)S[e];
+  const int t = threadIdx.x;
+  const int rgi = t / cg, cgi = t % cg;
+  const bool active = rgi < rg;
+  for (int64_t i0 = (int64_t)blockIdx.x * TR; i0 < n; i0 += (int64_t)gridDim.x * TR) {
+    const int nt = (int)min((int64_t)TR, n - i0);
+    __syncthreads();
+    const float2* Qt = bt.Q + (row0 + i0) * ldq;
+    for (int e = t; e < nt * kn; e += RITZ_THREADS) {
+      const int rr = e / kn, k = e % kn;
+      const float2 q = Qt[(size_t)rr * ldq + k];
+      Qh[rr * qs + k] = q.x;
+      Ql[rr * qs + k] = q.y;
     }
-    U[(row0 + i) * r + m] = (m < kn) ? acc : 0.f;
+    __syncthreads();
+    if (!active) continue;
+    float acc[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[a][c] = 0.f;
+    const int rb = rgi * 4, cb = cgi * 4;
+    for (int k = 0; k < kn; ++k) {
+      float s[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) s[c] = (cb + c < r) ? Ss[k * r + cb + c] : 0.f;
+#pragma unroll
+      for (int a = 0; a < 4; ++a) {
+        const float qh = Qh[(rb + a) * qs + k], ql = Ql[(rb + a) * qs + k];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[a][c] = fmaf(qh, s[c], fmaf(ql, s[c], acc[a][c]));
+      }
+    }
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+      if (rb + a < nt) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          if (cb + c < r) U[(row0 + i0 + rb + a) * r + cb + c] = (cb + c < kn) ? acc[a][c] : 0.f;
+      }
+    }
   }
 }
 
@@ -348,7 +443,7 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
 
 int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream) {
   dim3 grid(bt.r, bt.nprob_max);
-  tridiag_eigvals_kernel<<<grid, 32, 0, stream>>>(bt);
+  tridiag_eigvals_kernel<<<grid, EIG_THREADS, 0, stream>>>(bt);
   SLS_LAUNCH_CHECK();
   tridiag_eigvecs_kernel<<<grid, 32, 0, stream>>>(bt);
   SLS_LAUNCH_CHECK();
@@ -357,14 +452,14 @@ int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream) {
 
 int launch_ritz_vectors(const LanczosBatch& bt, float* U, cudaStream_t stream) {
   const int r = bt.r;
-  const int rpb = 256 / r;
-  int64_t blocks = (bt.nmax + rpb - 1) / rpb;
-  if (blocks > 1024) blocks = 1024;
+  const int TR = ritz_tile_rows(r);
+  int64_t blocks = (bt.nmax + TR - 1) / TR;
+  if (blocks > 4 * (int64_t)num_sms()) blocks = 4 * (int64_t)num_sms();
   if (blocks < 1) blocks = 1;
-  const size_t smem = sizeof(float) * r * r;
+  const size_t smem = sizeof(float) * ((size_t)r * r + 2 * (size_t)TR * (r + 1));
   SLS_CUDA_TRY(cudaFuncSetAttribute(ritz_vectors_kernel,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  ritz_vectors_kernel<<<dim3((unsigned)blocks, bt.nprob_max), 256, smem, stream>>>(bt, U);
+  ritz_vectors_kernel<<<dim3((unsigned)blocks, bt.nprob_max), RITZ_THREADS, smem, stream>>>(bt, U);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
