@@ -547,7 +547,7 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
   if (!workspace || workspace_bytes < need) return SLS_ERR_WORKSPACE;
   cudaStream_t s = (cudaStream_t)stream;
   Carver cv(workspace);
-  cv.take<int>(64);
+  int* status = cv.take<int>(64);
   ProbDesc* prob = cv.take<ProbDesc>(1);
   void* seg = cv.take<char>(segment_scratch_bytes(N, M_target, 1));
   float* norms = cv.take<float>(N);
@@ -560,11 +560,12 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
   int* counts = cv.take<int>(4);
   float* part = cv.take<float>(agg_part_capacity(N) * (size_t)d);
   float* part_eta = cv.take<float>(agg_part_capacity(N));
+  SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
   single_prob_kernel<<<1, 1, 0, s>>>(prob, N, M_target, 32);
   SLS_LAUNCH_CHECK();
   int st;
   if ((st = launch_segment(prob, 1, codes, pos_scheme, SLS_MODE_REPRESENTATIVE, seg, 1, N,
-                           M_target, perm, mstart, mlen, pos, tok2macro, s)) != SLS_OK)
+                           M_target, perm, mstart, mlen, pos, tok2macro, status, s)) != SLS_OK)
     return st;
   if ((st = launch_row_norms(X, x_dtype, N, d, ldx, norms, s)) != SLS_OK) return st;
   return launch_aggregate(X, x_dtype, d, ldx, norms, perm, mstart, mlen, M_target, N, renorm, Xt,
@@ -712,7 +713,7 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   phase_mark(5, 0, s);
   if ((st = launch_segment(W.probs, nprob, W.codes, cfg->pos_scheme, cfg->pos_mode, W.seg_scratch,
                            P.seg_slots, P.nmax, P.mmax, W.perm, W.mstart, W.mlen, pos, tok2macro,
-                           s)) != SLS_OK)
+                           W.status, s)) != SLS_OK)
     return st;
   if ((st = launch_preserved(B, N, P.M, (int)P.pf, (int)P.pl, cfg->pos_mode, W.perm, W.mstart,
                              W.mlen, pos, tok2macro, s)) != SLS_OK)

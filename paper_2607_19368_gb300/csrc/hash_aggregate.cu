@@ -234,7 +234,7 @@ SLS_DEV int bit_length_u64(unsigned long long x) { return x ? 64 - __clzll((long
 // Per-problem scratch layout (ints unless noted), identical on host and device.
 struct SegLayout {
   size_t ka, kb, va, vb, f, cst, grp, gst, gmax, gmin, gsum, ok_a, ok_b, ov_a, ov_b, oidx, rep,
-      seat, total;
+      seat, gbar, ghist, gcsum, total;
 };
 
 __host__ __device__ inline size_t seg_al(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -261,6 +261,11 @@ __host__ __device__ inline SegLayout seg_layout(int64_t nmax, int64_t mmax) {
   L.oidx = o; o += seg_al(m1 * 4);
   L.rep = o;  o += seg_al(m1 * 4);
   L.seat = o; o += seg_al(n1 * 4);
+  // grid version (one large problem): barrier words, digit counts per CTA,
+  // CTA sums of the scans
+  L.gbar = o;  o += 256;
+  L.ghist = o; o += seg_al((size_t)256 * 256 * 4);
+  L.gcsum = o; o += seg_al((size_t)256 * 4);
   L.total = o;
   return L;
 }
@@ -478,6 +483,373 @@ segment_kernel(const ProbDesc* __restrict__ probs, int nprob, const uint32_t* __
       }
       __syncthreads();
     }
+  }
+}
+
+// ============================================================================
+// segment kernel for one large problem: the same computation spread over a
+// cooperative grid (G CTAs of SEG_T threads), for the single-prompt pass
+// ============================================================================
+
+constexpr int SEGG_MAX = 256;           // CTAs of the grid segment kernel, at most
+constexpr int64_t SEG_GRID_MIN_N = 8192;  // tokens from which one problem uses the grid kernel
+
+struct GridSync {
+  GroupBarrier bar;
+  unsigned lgen;
+  int* status;
+  int* sflag;
+  volatile int* serr;
+};
+
+SLS_DEV bool gsync(GridSync& gs) {
+  return group_sync_named(gs.bar, gs.lgen, gs.status, gs.sflag, gs.serr, 1, SEG_T);
+}
+
+// Exclusive scan of in[0..n) into out over the grid; CTA b owns the slice
+// [b n / G, (b+1) n / G).  On return this CTA's slice of out is final and the
+// total is returned; other slices are final after the next gsync.  csum: G
+// ints in global memory.
+SLS_DEV bool grid_scan(const int* in, int* out, int n, int* csum, GridSync& gs, int* sh,
+                       int* total) {
+  const int G = gridDim.x, b = blockIdx.x, tid = threadIdx.x;
+  const int c0 = (int)((int64_t)b * n / G), c1 = (int)((int64_t)(b + 1) * n / G);
+  const int loc = block_scan_array<int>(in + c0, out + c0, c1 - c0, sh);
+  if (tid == 0) csum[b] = loc;
+  if (!gsync(gs)) return false;
+  int pre = 0, tot = 0;
+  for (int c = tid; c < G; c += SEG_T) {
+    const int v = csum[c];
+    tot += v;
+    if (c < b) pre += v;
+  }
+  pre = block_sum<int>(pre, sh);
+  tot = block_sum<int>(tot, sh);
+  for (int i = c0 + tid; i < c1; i += SEG_T) out[i] += pre;
+  *total = tot;
+  __syncthreads();
+  return true;
+}
+
+// One stable LSD pass (8 bits at `shift`) of (key, val) pairs over the grid:
+// per-CTA digit counts, the prefix over (digit, CTA), then the CTA's slice is
+// scattered in order (stable within the CTA as in block_radix_sort).
+// hist: 256 x G ints in global memory.  sh: 256 + 256 + SEG_W * 256 ints.
+template <typename K>
+SLS_DEV bool grid_radix_pass(const K* ka, const int* va, K* kb, int* vb, int n, int shift,
+                             int* hist, GridSync& gs, int* sh) {
+  const int G = gridDim.x, b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int* base = sh;
+  int* tot = sh + 256;
+  int* wc = sh + 512;
+  const int c0 = (int)((int64_t)b * n / G), c1 = (int)((int64_t)(b + 1) * n / G);
+  if (tid < 256) base[tid] = 0;
+  __syncthreads();
+  for (int i = c0 + tid; i < c1; i += SEG_T) atomicAdd(&base[(int)((ka[i] >> shift) & 255)], 1);
+  __syncthreads();
+  if (tid < 256) hist[tid * G + b] = base[tid];
+  if (!gsync(gs)) return false;
+  if (tid < 256) {
+    int all = 0, part = 0;
+    for (int c = 0; c < G; ++c) {
+      const int h = hist[tid * G + c];
+      all += h;
+      if (c < b) part += h;
+    }
+    // exclusive scan of the digit totals by the first 8 warps
+    int x = all;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) tot[warp] = x;
+    base[tid] = x - all + part;
+  }
+  __syncthreads();
+  if (tid < 256) {
+    int add = 0;
+    for (int w = 0; w < warp; ++w) add += tot[w];
+    base[tid] += add;
+  }
+  __syncthreads();
+  for (int t0 = c0; t0 < c1; t0 += SEG_T) {
+    for (int e = tid; e < SEG_W * 256; e += SEG_T) wc[e] = 0;
+    __syncthreads();
+    const int i = t0 + tid;
+    const bool valid = i < c1;
+    K key = 0;
+    int val = 0;
+    unsigned dg = 256u + (unsigned)lane;
+    if (valid) {
+      key = ka[i];
+      val = va[i];
+      dg = (unsigned)((key >> shift) & 255);
+    }
+    const unsigned peers = __match_any_sync(0xffffffffu, dg);
+    const int rank = __popc(peers & lanemask_lt());
+    if (valid && rank == 0) wc[warp * 256 + dg] = __popc(peers);
+    __syncthreads();
+    if (tid < 256) {
+      int run = 0;
+      for (int w = 0; w < SEG_W; ++w) {
+        const int c = wc[w * 256 + tid];
+        wc[w * 256 + tid] = run;
+        run += c;
+      }
+      tot[tid] = run;
+    }
+    __syncthreads();
+    if (valid) {
+      const int pos = base[dg] + wc[warp * 256 + dg] + rank;
+      kb[pos] = key;
+      vb[pos] = val;
+    }
+    __syncthreads();
+    if (tid < 256) base[tid] += tot[tid];
+    __syncthreads();
+  }
+  return gsync(gs);
+}
+
+template <typename K>
+SLS_DEV bool grid_radix_sort(K*& ka, int*& va, K*& kb, int*& vb, int n, int key_bits, int* hist,
+                             GridSync& gs, int* sh) {
+  for (int shift = 0; shift < key_bits; shift += 8) {
+    if (!grid_radix_pass<K>(ka, va, kb, vb, n, shift, hist, gs, sh)) return false;
+    K* tk = ka;
+    ka = kb;
+    kb = tk;
+    int* tv = va;
+    va = vb;
+    vb = tv;
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(SEG_T, 1)
+segment_grid_kernel(const ProbDesc* __restrict__ probs, const uint32_t* __restrict__ codes,
+                    int pos_scheme, int pos_mode, char* sb, int64_t nmax, int64_t mmax,
+                    int* __restrict__ perm, int* __restrict__ mstart, int* __restrict__ mlen,
+                    int32_t* __restrict__ pos_out, int32_t* __restrict__ tok2macro,
+                    int* status) {
+  __shared__ int sh_sort[512 + SEG_W * 256];
+  __shared__ long long sh_ll[SEG_W + 1];
+  __shared__ int sh_i[SEG_W + 1];
+  __shared__ int sflag;
+  __shared__ volatile int serr;
+  const int tid = threadIdx.x, G = gridDim.x, b = blockIdx.x;
+  const SegLayout L = seg_layout(nmax, mmax);
+  if (tid == 0) serr = 0;
+  __syncthreads();
+  GridSync gs{GroupBarrier{reinterpret_cast<unsigned*>(sb + L.gbar),
+                           reinterpret_cast<unsigned*>(sb + L.gbar) + 32, (unsigned)G},
+              0u, status, &sflag, &serr};
+  const ProbDesc P = probs[0];
+  const int n = P.n, M = P.m;
+  if (n <= 0 || M <= 0) return;
+  uint32_t* ka = reinterpret_cast<uint32_t*>(sb + L.ka);
+  uint32_t* kb = reinterpret_cast<uint32_t*>(sb + L.kb);
+  int* va = reinterpret_cast<int*>(sb + L.va);
+  int* vb = reinterpret_cast<int*>(sb + L.vb);
+  int* f = reinterpret_cast<int*>(sb + L.f);
+  int* cst = reinterpret_cast<int*>(sb + L.cst);
+  int* grp = reinterpret_cast<int*>(sb + L.grp);
+  int* gst = reinterpret_cast<int*>(sb + L.gst);
+  int* gmax = reinterpret_cast<int*>(sb + L.gmax);
+  int* gmin = reinterpret_cast<int*>(sb + L.gmin);
+  unsigned long long* gsum = reinterpret_cast<unsigned long long*>(sb + L.gsum);
+  int* oidx = reinterpret_cast<int*>(sb + L.oidx);
+  int* rep = reinterpret_cast<int*>(sb + L.rep);
+  int* seat = reinterpret_cast<int*>(sb + L.seat);
+  int* hist = reinterpret_cast<int*>(sb + L.ghist);
+  int* csum = reinterpret_cast<int*>(sb + L.gcsum);
+  const int s0 = (int)((int64_t)b * n / G), s1 = (int)((int64_t)(b + 1) * n / G);
+  const int m0 = (int)((int64_t)b * M / G), m1 = (int)((int64_t)(b + 1) * M / G);
+  bool merged = false;
+
+  if (P.spectral) {
+    // ---- stable sort of (code, token) ----
+    for (int i = s0 + tid; i < s1; i += SEG_T) {
+      ka[i] = codes[P.phi_row + i];
+      va[i] = i;
+    }
+    if (!gsync(gs)) return;
+    if (!grid_radix_sort<uint32_t>(ka, va, kb, vb, n, P.bits, hist, gs, sh_sort)) return;
+    // ---- clusters: runs of equal codes ----
+    for (int s = s0 + tid; s < s1; s += SEG_T) f[s] = (s == 0 || ka[s] != ka[s - 1]) ? 1 : 0;
+    __syncthreads();
+    int C = 0;
+    if (!grid_scan(f, grp, n, csum, gs, sh_i, &C)) return;  // grp[s] = clusters before s
+    for (int s = s0 + tid; s < s1; s += SEG_T)
+      if (f[s]) cst[grp[s]] = s;
+    if (b == 0 && tid == 0) cst[C] = n;
+    if (!gsync(gs)) return;
+    if (C >= M) {
+      // merge: the cluster of rank t joins group floor(t M / C)
+      merged = (C > M);
+      const int t0 = (int)((int64_t)b * C / G), t1 = (int)((int64_t)(b + 1) * C / G);
+      for (int t = t0 + tid; t < t1; t += SEG_T) {
+        const int g = (int)(((long long)t * M) / C);
+        const int gp = (t == 0) ? -1 : (int)(((long long)(t - 1) * M) / C);
+        if (g != gp) gst[g] = cst[t];
+      }
+    } else if (b == 0) {
+      // split: D'Hondt seats, one guaranteed per cluster, ties to the lower
+      // code (few clusters: one CTA)
+      const long long K = (long long)(M - C);
+      int maxn = 0;
+      for (int t = tid; t < C; t += SEG_T) maxn = max(maxn, cst[t + 1] - cst[t]);
+      if (tid == 0) sh_i[0] = 0;
+      __syncthreads();
+      atomicMax(&sh_i[0], maxn);
+      __syncthreads();
+      maxn = sh_i[0];
+      __syncthreads();
+      long long lo = 0, hi = ((long long)maxn) << 40;
+      while (hi - lo > 1) {
+        const long long mid = lo + (hi - lo) / 2;
+        long long c = 0;
+        for (int t = tid; t < C; t += SEG_T) c += dhondt_count_ge(cst[t + 1] - cst[t], mid);
+        c = block_sum<long long>(c, sh_ll);
+        if (c >= K) lo = mid;
+        else hi = mid;
+      }
+      long long gt_sum = 0;
+      for (int t = tid; t < C; t += SEG_T) {
+        const long long nt = cst[t + 1] - cst[t];
+        const long long ge = dhondt_count_ge(nt, lo);
+        const long long gt = dhondt_count_ge(nt, lo + 1);
+        seat[t] = (int)gt;
+        f[t] = (int)(ge - gt);
+        gt_sum += gt;
+      }
+      gt_sum = block_sum<long long>(gt_sum, sh_ll);
+      const int R = (int)(K - gt_sum);
+      __syncthreads();
+      int* eqs = grp;  // scratch (size >= C)
+      block_scan_array<int>(f, eqs, C, sh_i);
+      for (int t = tid; t < C; t += SEG_T) {
+        const int extra = (f[t] && eqs[t] < R) ? 1 : 0;
+        seat[t] = 1 + seat[t] + extra;
+      }
+      __syncthreads();
+      int* so = f;
+      block_scan_array<int>(seat, so, C, sh_i);
+      for (int t = tid; t < C; t += SEG_T) {
+        const int nt = cst[t + 1] - cst[t], pt = seat[t];
+        const int q = nt / pt, rem = nt % pt;
+        for (int k = 0; k < pt; ++k) {
+          const int off = (k < rem) ? k * (q + 1) : rem * (q + 1) + (k - rem) * q;
+          gst[so[t] + k] = cst[t] + off;
+        }
+      }
+    }
+  } else {
+    // chunk: contiguous groups (array_split into m, or runs of k)
+    for (int i = s0 + tid; i < s1; i += SEG_T) va[i] = i;
+    for (int g = m0 + tid; g < m1; g += SEG_T) {
+      int off;
+      if (P.chunk_k > 0) {
+        off = min(n, g * P.chunk_k);
+      } else {
+        const int q = n / M, rem = n % M;
+        off = (g < rem) ? g * (q + 1) : rem * (q + 1) + (g - rem) * q;
+      }
+      gst[g] = off;
+    }
+  }
+  if (b == 0 && tid == 0) gst[M] = n;
+  if (!gsync(gs)) return;
+  const int* perm_l = va;  // sorted position -> local token
+  // ---- group id of every sorted position ----
+  for (int s = s0 + tid; s < s1; s += SEG_T) f[s] = 0;
+  if (!gsync(gs)) return;
+  for (int g = m0 + tid; g < m1; g += SEG_T) f[gst[g]] = 1;
+  if (!gsync(gs)) return;
+  int Mchk = 0;
+  if (!grid_scan(f, grp, n, csum, gs, sh_i, &Mchk)) return;
+  for (int s = s0 + tid; s < s1; s += SEG_T) grp[s] = grp[s] + f[s] - 1;
+  for (int g = m0 + tid; g < m1; g += SEG_T) {
+    gmax[g] = -1;
+    gmin[g] = INT_MAX;
+    gsum[g] = 0ull;
+  }
+  if (!gsync(gs)) return;
+  for (int s = s0 + tid; s < s1; s += SEG_T) {
+    const int g = grp[s], i = perm_l[s];
+    atomicMax(&gmax[g], i);
+    atomicMin(&gmin[g], i);
+    if (pos_scheme == SLS_POS_MEAN) atomicAdd(&gsum[g], (unsigned long long)i);
+  }
+  if (!gsync(gs)) return;
+  // ---- representative positions ----
+  if (pos_scheme == SLS_POS_MEDIAN && merged) {
+    // members of merged groups are not in token order: sort (group, token)
+    int* xa = seat;
+    int* xb = cst;
+    uint32_t* ga = ka;
+    uint32_t* gb2 = kb;
+    for (int s = s0 + tid; s < s1; s += SEG_T) ga[perm_l[s]] = (uint32_t)grp[s];
+    for (int i = s0 + tid; i < s1; i += SEG_T) xa[i] = i;
+    if (!gsync(gs)) return;
+    if (!grid_radix_sort<uint32_t>(ga, xa, gb2, xb, n, bit_length_u64((unsigned long long)M),
+                                   hist, gs, sh_sort))
+      return;
+    for (int g = m0 + tid; g < m1; g += SEG_T) rep[g] = xa[gst[g] + (gst[g + 1] - gst[g] - 1) / 2];
+  } else {
+    for (int g = m0 + tid; g < m1; g += SEG_T) {
+      const int len = gst[g + 1] - gst[g];
+      int rp;
+      if (pos_scheme == SLS_POS_MAX) rp = gmax[g];
+      else if (pos_scheme == SLS_POS_MEDIAN) rp = perm_l[gst[g] + (len - 1) / 2];
+      else rp = (int)((2ull * gsum[g] + (unsigned long long)len) / (2ull * (unsigned long long)len));
+      rep[g] = rp;
+    }
+  }
+  if (!gsync(gs)) return;
+  // ---- order groups by (position, first token) ----
+  if (pos_scheme != SLS_POS_MEAN) {
+    // max and median positions are member tokens of disjoint groups, hence
+    // distinct: the rank of a group is the number of marked positions below
+    // its own (one scan over the token positions)
+    for (int s = s0 + tid; s < s1; s += SEG_T) f[s] = 0;
+    if (!gsync(gs)) return;
+    for (int g = m0 + tid; g < m1; g += SEG_T) f[rep[g]] = 1;
+    if (!gsync(gs)) return;
+    int* rk = cst;  // rank of a marked position
+    int tmk = 0;
+    if (!grid_scan(f, rk, n, csum, gs, sh_i, &tmk)) return;
+    if (!gsync(gs)) return;
+    for (int g = m0 + tid; g < m1; g += SEG_T) oidx[g] = rk[rep[g]];
+  } else {
+    unsigned long long* oka = reinterpret_cast<unsigned long long*>(sb + L.ok_a);
+    unsigned long long* okb = reinterpret_cast<unsigned long long*>(sb + L.ok_b);
+    int* ova = reinterpret_cast<int*>(sb + L.ov_a);
+    int* ovb = reinterpret_cast<int*>(sb + L.ov_b);
+    for (int g = m0 + tid; g < m1; g += SEG_T) {
+      oka[g] = (unsigned long long)rep[g] * (unsigned long long)n + (unsigned long long)gmin[g];
+      ova[g] = g;
+    }
+    if (!gsync(gs)) return;
+    const int kbits = bit_length_u64((unsigned long long)n * (unsigned long long)n);
+    if (!grid_radix_sort<unsigned long long>(oka, ova, okb, ovb, M, kbits, hist, gs, sh_sort))
+      return;
+    for (int t = m0 + tid; t < m1; t += SEG_T) oidx[ova[t]] = t;
+  }
+  if (!gsync(gs)) return;
+  // ---- outputs ----
+  for (int g = m0 + tid; g < m1; g += SEG_T) {
+    const int t = oidx[g];
+    const int64_t mrow = P.out0 + t;
+    mstart[mrow] = (int)(P.tok_row + gst[g]);
+    mlen[mrow] = gst[g + 1] - gst[g];
+    pos_out[mrow] = (pos_mode == SLS_MODE_COMPACT) ? (P.out_local + t) : (P.pos0 + rep[g]);
+  }
+  for (int s = s0 + tid; s < s1; s += SEG_T) {
+    const int i = perm_l[s];
+    perm[P.tok_row + s] = (int)(P.tok_row + i);
+    tok2macro[P.tok_row + i] = P.out_local + oidx[grp[s]];
   }
 }
 
@@ -868,10 +1240,31 @@ int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const i
 
 int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int pos_scheme,
                    int pos_mode, void* scratch, int slots, int64_t nmax, int64_t mmax, int* perm,
-                   int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,
+                   int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro, int* status,
                    cudaStream_t stream) {
   if (nprob <= 0) return SLS_OK;
-  const size_t stride = seg_layout(nmax, mmax).total;
+  const SegLayout L = seg_layout(nmax, mmax);
+  const size_t stride = L.total;
+  if (nprob == 1 && nmax >= SEG_GRID_MIN_N && status) {
+    // one large problem: spread it over a cooperative grid
+    int dev = 0, sms = 0;
+    SLS_CUDA_TRY(cudaGetDevice(&dev));
+    SLS_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    int G = sms < SEGG_MAX ? sms : SEGG_MAX;
+    const int64_t want = (nmax + 255) / 256;
+    if (want < G) G = (int)want;
+    if (G < 1) G = 1;
+    char* sb = (char*)scratch;
+    SLS_CUDA_TRY(cudaMemsetAsync(sb + L.gbar, 0, 256, stream));
+    int64_t nm = nmax, mm = mmax;
+    void* args[] = {(void*)&probs, (void*)&codes, (void*)&pos_scheme, (void*)&pos_mode,
+                    (void*)&sb, (void*)&nm, (void*)&mm, (void*)&perm, (void*)&mstart,
+                    (void*)&mlen, (void*)&pos_out, (void*)&tok2macro, (void*)&status};
+    SLS_CUDA_TRY(cudaLaunchCooperativeKernel((const void*)segment_grid_kernel, dim3(G), dim3(SEG_T),
+                                             args, 0, stream));
+    count_launch(1);
+    return SLS_OK;
+  }
   const int grid = nprob < slots ? nprob : slots;
   segment_kernel<<<grid, SEG_T, 0, stream>>>(probs, nprob, codes, pos_scheme, pos_mode,
                                              (char*)scratch, stride, nmax, mmax, perm, mstart,

@@ -67,7 +67,7 @@ int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const i
                             cudaStream_t stream);
 int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int pos_scheme,
                    int pos_mode, void* scratch, int slots, int64_t nmax, int64_t mmax, int* perm,
-                   int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,
+                   int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro, int* status,
                    cudaStream_t stream);
 int launch_preserved(int64_t B, int64_t N, int64_t M, int pf, int pl, int pos_mode, int* perm,
                      int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,

@@ -208,6 +208,25 @@ def test_aggregate_bit_exact_maps(sls, scheme, case):
     assert np.max(np.abs(Xt.cpu().numpy() - Xt_o)) <= EMB_TOL
 
 
+@pytest.mark.parametrize("scheme", [O.POS_MAX, O.POS_MEDIAN, O.POS_MEAN])
+@pytest.mark.parametrize("case", ["merge", "split", "equal"])
+def test_aggregate_bit_exact_maps_one_large_problem(sls, scheme, case):
+    """A single problem large enough for the grid-wide segment kernel."""
+    g = np.random.default_rng(11 + scheme)
+    N, d = 20000, 16
+    X = (g.standard_normal((N, d)) / 4).astype(np.float32)
+    nb = {"merge": 6000, "split": 130, "equal": 2000}[case]
+    codes = g.integers(0, nb, size=N).astype(np.uint32) * np.uint32(2654435761 % 2 ** 32 // 7)
+    C = len(set(codes.tolist()))
+    M = {"merge": max(1, C // 3), "split": min(N, C * 7 + 3), "equal": C}[case]
+    Xt_o, pos_o, t2m_o, C_o = _oracle_aggregate(X.astype(np.float64), codes, M, scheme, True)
+    Xt, pos, t2m = sls.aggregate(torch.from_numpy(X).cuda(),
+                                 torch.from_numpy(codes.view(np.int32)).cuda(), M, scheme, True)
+    assert np.array_equal(t2m.cpu().numpy(), t2m_o)
+    assert np.array_equal(pos.cpu().numpy(), pos_o)
+    assert np.max(np.abs(Xt.cpu().numpy() - Xt_o)) <= EMB_TOL
+
+
 def test_aggregate_bf16_large_groups(sls):
     """bf16 embeddings, duplicated tokens (one large cluster), renorm off and on."""
     w, p, prm = _workload_inputs("mistral7b", N=6000, d=512)
