@@ -261,9 +261,9 @@ int sls_lanczos_topr_noalloc(const float* Phi, int64_t N, int D, int r,
  * 2 * SLS_NUM_PHASES cudaEvent_t handles (passed as void*) owned by the
  * caller; while set, every sls_compress call records events[2p] on its
  * stream before phase p and events[2p+1] after it.  Phases, in launch order:
- * 0 setup (problem table, token norms, router), 1 feature map, 2 Lanczos,
- * 3 Eigh(T) and Ritz vectors, 4 SimHash, 5 clusters/adjust/order,
- * 6 macro-token aggregation.  count = 0 (or events = NULL) switches timing
+ * 0 setup (problem table; token norms and router when adaptive), 1 feature
+ * map, 2 Lanczos, 3 Eigh(T) and Ritz vectors, 4 SimHash, 5 clusters/adjust/
+ * order, 6 macro-token aggregation.  count = 0 (or events = NULL) switches timing
  * off.  Process-wide setting, not thread-safe.  Errors: INVALID_ARG if
  * count is neither 0 nor 2 * SLS_NUM_PHASES.
  */

@@ -521,7 +521,6 @@ size_t sls_aggregate_workspace_size(int64_t N, int d, int64_t M_target) {
   cv.take<int>(64);
   cv.take<ProbDesc>(1);
   cv.take<char>(segment_scratch_bytes(N, M_target, 1));
-  cv.take<float>(N);
   cv.take<int>(N);
   cv.take<int>(M_target);
   cv.take<int>(M_target);
@@ -550,7 +549,6 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
   int* status = cv.take<int>(64);
   ProbDesc* prob = cv.take<ProbDesc>(1);
   void* seg = cv.take<char>(segment_scratch_bytes(N, M_target, 1));
-  float* norms = cv.take<float>(N);
   int* perm = cv.take<int>(N);
   int* mstart = cv.take<int>(M_target);
   int* mlen = cv.take<int>(M_target);
@@ -567,8 +565,7 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
   if ((st = launch_segment(prob, 1, codes, pos_scheme, SLS_MODE_REPRESENTATIVE, seg, 1, N,
                            M_target, perm, mstart, mlen, pos, tok2macro, status, s)) != SLS_OK)
     return st;
-  if ((st = launch_row_norms(X, x_dtype, N, d, ldx, norms, s)) != SLS_OK) return st;
-  return launch_aggregate(X, x_dtype, d, ldx, norms, perm, mstart, mlen, M_target, N, renorm, Xt,
+  return launch_aggregate(X, x_dtype, d, ldx, perm, mstart, mlen, M_target, N, renorm, Xt,
                           it_start, pt_start, items, counts, part, part_eta, s);
 }
 
@@ -634,12 +631,11 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
         cfg->backend == SLS_BACKEND_CHUNK ? P.k_chunk : 0, spectral ? params->q1_stride : 0);
     SLS_LAUNCH_CHECK();
   }
-  // token norms (aggregation and the router)
-  if ((st = launch_row_norms(X, x_dtype, B * N, d, ldx, W.norms, s)) != SLS_OK) return st;
-  // routing
+  // routing (the window score needs every token's norm first)
   int mode = spectral ? 0 : 1;
   if (cfg->backend == SLS_BACKEND_ADAPTIVE) {
     mode = 2;
+    if ((st = launch_row_norms(X, x_dtype, B * N, d, ldx, W.norms, s)) != SLS_OK) return st;
     if ((st = launch_window_score(X, x_dtype, d, ldx, W.norms, W.probs, nprob, W.score, s)) !=
         SLS_OK)
       return st;
@@ -720,7 +716,7 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
     return st;
   phase_mark(5, 1, s);
   phase_mark(6, 0, s);
-  st = launch_aggregate(X, x_dtype, d, ldx, W.norms, W.perm, W.mstart, W.mlen, B * P.M, B * N,
+  st = launch_aggregate(X, x_dtype, d, ldx, W.perm, W.mstart, W.mlen, B * P.M, B * N,
                         cfg->renorm, Xt, W.it_start, W.pt_start, W.items, W.counts, W.part,
                         W.part_eta, s);
   phase_mark(6, 1, s);

@@ -1014,29 +1014,42 @@ SLS_DEV float agg_block_sum(float v, float* sh) {
   return s;
 }
 
+SLS_DEV void store_vec4(float* p, float a, float b, float c, float e) {
+  *reinterpret_cast<float4*>(p) = make_float4(a, b, c, e);
+}
+
+// Thread `tid` owns the V-wide column groups c0 = (tid + q * AGG_T) * V, q < NV.
+template <int V, int NV>
+SLS_DEV void store_row(const float (&acc)[NV * V], float scale, int d, float* __restrict__ out) {
+  const int tid = threadIdx.x;
+#pragma unroll
+  for (int q = 0; q < NV; ++q) {
+    const int c0 = (tid + q * AGG_T) * V;
+    if (c0 < d)
+#pragma unroll
+      for (int v = 0; v < V; v += 4)
+        store_vec4(out + c0 + v, acc[q * V + v] * scale, acc[q * V + v + 1] * scale,
+                   acc[q * V + v + 2] * scale, acc[q * V + v + 3] * scale);
+  }
+}
+
 // Finalise one macro-token row from the member sum `acc` (per thread), the
 // member count and the sum of member norms: mean, then rescale to the mean
 // norm (Eq. macro_embed); a singleton is its token unchanged.
-template <int V>
-SLS_DEV void agg_finalize(float (&acc)[AGG_MAXV], int nv, int len, float eta_sum, int renorm, int d,
+template <int V, int NV>
+SLS_DEV void agg_finalize(float (&acc)[NV * V], int len, float eta_sum, int renorm, int d,
                           float* __restrict__ out, float* sh) {
-  const int tid = threadIdx.x;
   if (len == 1) {
-#pragma unroll
-    for (int q = 0; q < AGG_MAXV / V; ++q) {
-      const int c0 = (tid + q * AGG_T) * V;
-      if (q < nv && c0 < d)
-#pragma unroll
-        for (int v = 0; v < V; ++v) out[c0 + v] = acc[q * V + v];
-    }
+    store_row<V, NV>(acc, 1.0f, d, out);
     return;
   }
+  const int tid = threadIdx.x;
   const float inv = 1.0f / (float)len;
   float sq = 0.f;
 #pragma unroll
-  for (int q = 0; q < AGG_MAXV / V; ++q) {
+  for (int q = 0; q < NV; ++q) {
     const int c0 = (tid + q * AGG_T) * V;
-    if (q < nv && c0 < d)
+    if (c0 < d)
 #pragma unroll
       for (int v = 0; v < V; ++v) {
         acc[q * V + v] *= inv;
@@ -1048,99 +1061,136 @@ SLS_DEV void agg_finalize(float (&acc)[AGG_MAXV], int nv, int len, float eta_sum
     const float nrm = sqrtf(agg_block_sum(sq, sh));
     if (nrm >= 1e-30f) scale = (eta_sum * inv) / nrm;
   }
-#pragma unroll
-  for (int q = 0; q < AGG_MAXV / V; ++q) {
-    const int c0 = (tid + q * AGG_T) * V;
-    if (q < nv && c0 < d)
-#pragma unroll
-      for (int v = 0; v < V; ++v) out[c0 + v] = acc[q * V + v] * scale;
-  }
+  store_row<V, NV>(acc, scale, d, out);
 }
 
-template <typename T>
-__global__ void __launch_bounds__(AGG_T)
-agg_partial_kernel(const T* __restrict__ X, int d, int64_t ldx, const float* __restrict__ norms,
-                   const int* __restrict__ perm, const int* __restrict__ mstart,
-                   const int* __restrict__ mlen, const int2* __restrict__ items,
-                   const int* __restrict__ counts, const int* __restrict__ pt_start, int renorm,
-                   float* __restrict__ Xt, float* __restrict__ part, float* __restrict__ part_eta) {
+// Member rows loaded per batch, so that about eight 16-byte loads per thread
+// are in flight.
+template <int NV>
+constexpr int agg_batch() {
+  return NV >= 8 ? 1 : 8 / NV;
+}
+
+// One work item = up to AGG_CH members of one macro-token.  The member rows
+// are gathered in batches of agg_batch<NV>() rows (all loads of a batch issued
+// before any is used); every member's |x|^2 is reduced from the same values,
+// per warp into shared memory, so X is read once.  A macro-token of one item
+// is finalised here; longer ones leave a partial sum for agg_final_kernel.
+template <typename T, int NV>
+__global__ void __launch_bounds__(AGG_T, 2)
+agg_partial_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restrict__ perm,
+                   const int* __restrict__ mstart, const int* __restrict__ mlen,
+                   const int2* __restrict__ items, const int* __restrict__ counts,
+                   const int* __restrict__ pt_start, int renorm, float* __restrict__ Xt,
+                   float* __restrict__ part, float* __restrict__ part_eta) {
   constexpr int V = VecOf<T>::V;
-  __shared__ float sh[AGG_T / 32];
+  constexpr int MB = agg_batch<NV>();
+  constexpr int NW = AGG_T / 32;
+  __shared__ float sh[NW];
+  __shared__ float shq[NW][AGG_CH];
   const int nitems = counts[0];
-  const int tid = threadIdx.x;
-  const int nv = (d / V + AGG_T - 1) / AGG_T;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int it = blockIdx.x; it < nitems; it += gridDim.x) {
     const int2 item = items[it];
     const int m = item.x, c = item.y;
     const int len = mlen[m];
-    const int b = c * AGG_CH, e = min(len, b + AGG_CH);
-    const int* mem = perm + mstart[m];
-    float acc[AGG_MAXV];
+    const int b = c * AGG_CH;
+    const int n = min(len - b, AGG_CH);
+    const int* mem = perm + mstart[m] + b;
+    const int id0 = lane < n ? mem[lane] : 0;
+    const int id1 = lane + 32 < n ? mem[lane + 32] : 0;
+    float acc[NV * V];
 #pragma unroll
-    for (int k = 0; k < AGG_MAXV; ++k) acc[k] = 0.f;
-    float eta = 0.f;
-    for (int s = b; s < e; ++s) {
-      const int row = mem[s];
-      const T* x = X + (int64_t)row * ldx;
-      eta += norms[row];
+    for (int k = 0; k < NV * V; ++k) acc[k] = 0.f;
+    for (int s0 = 0; s0 < n; s0 += MB) {
+      float v[MB][NV * V];
 #pragma unroll
-      for (int q = 0; q < AGG_MAXV / V; ++q) {
-        const int c0 = (tid + q * AGG_T) * V;
-        if (q < nv && c0 < d) {
-          float v[V];
-          load_vec<T>(x + c0, v);
+      for (int j = 0; j < MB; ++j) {
+        const int s = s0 + j;
+        const int row = __shfl_sync(0xffffffffu, s < 32 ? id0 : id1, s & 31);
+        const T* x = X + (int64_t)row * ldx;
 #pragma unroll
-          for (int k = 0; k < V; ++k) acc[q * V + k] += v[k];
+        for (int q = 0; q < NV; ++q) {
+          const int c0 = (tid + q * AGG_T) * V;
+          if (s < n && c0 < d) {
+            load_vec<T>(x + c0, &v[j][q * V]);
+          } else {
+#pragma unroll
+            for (int k = 0; k < V; ++k) v[j][q * V + k] = 0.f;
+          }
         }
       }
+#pragma unroll
+      for (int j = 0; j < MB; ++j) {
+        float sq = 0.f;
+#pragma unroll
+        for (int k = 0; k < NV * V; ++k) {
+          acc[k] += v[j][k];
+          sq = fmaf(v[j][k], v[j][k], sq);
+        }
+        sq = warp_sum_f(sq);
+        if (lane == 0 && s0 + j < n) shq[warp][s0 + j] = sq;
+      }
     }
+    __syncthreads();
+    // sum of member norms (every warp forms the same total)
+    float eta = 0.f;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int s = lane + 32 * h;
+      if (s < n) {
+        float t = 0.f;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) t += shq[w][s];
+        eta += sqrtf(t);
+      }
+    }
+    eta = warp_sum_f(eta);
     const int ps = pt_start[m];
     if (ps < 0) {
-      agg_finalize<V>(acc, nv, len, eta, renorm, d, Xt + (int64_t)m * d, sh);
+      agg_finalize<V, NV>(acc, len, eta, renorm, d, Xt + (int64_t)m * d, sh);
     } else {
-      float* dst = part + (int64_t)(ps + c) * d;
-#pragma unroll
-      for (int q = 0; q < AGG_MAXV / V; ++q) {
-        const int c0 = (tid + q * AGG_T) * V;
-        if (q < nv && c0 < d)
-#pragma unroll
-          for (int k = 0; k < V; ++k) dst[c0 + k] = acc[q * V + k];
-      }
+      store_row<V, NV>(acc, 1.0f, d, part + (int64_t)(ps + c) * d);
       if (tid == 0) part_eta[ps + c] = eta;
     }
     __syncthreads();
   }
 }
 
-template <int V>
+template <int V, int NV>
 __global__ void __launch_bounds__(AGG_T)
 agg_final_kernel(int d, const int* __restrict__ mlen, const int* __restrict__ pt_start,
                  int64_t Mtot, int renorm, const float* __restrict__ part,
                  const float* __restrict__ part_eta, float* __restrict__ Xt) {
   __shared__ float sh[AGG_T / 32];
   const int tid = threadIdx.x;
-  const int nv = (d / V + AGG_T - 1) / AGG_T;
   for (int64_t m = blockIdx.x; m < Mtot; m += gridDim.x) {
     const int ps = pt_start[m];
     if (ps < 0) continue;
     const int len = mlen[m];
     const int nch = (len + AGG_CH - 1) / AGG_CH;
-    float acc[AGG_MAXV];
+    float acc[NV * V];
 #pragma unroll
-    for (int k = 0; k < AGG_MAXV; ++k) acc[k] = 0.f;
+    for (int k = 0; k < NV * V; ++k) acc[k] = 0.f;
     float eta = 0.f;
     for (int c = 0; c < nch; ++c) {
       const float* src = part + (int64_t)(ps + c) * d;
       eta += part_eta[ps + c];
 #pragma unroll
-      for (int q = 0; q < AGG_MAXV / V; ++q) {
+      for (int q = 0; q < NV; ++q) {
         const int c0 = (tid + q * AGG_T) * V;
-        if (q < nv && c0 < d)
+        if (c0 < d)
 #pragma unroll
-          for (int k = 0; k < V; ++k) acc[q * V + k] += src[c0 + k];
+          for (int k = 0; k < V; k += 4) {
+            const float4 f = *reinterpret_cast<const float4*>(src + c0 + k);
+            acc[q * V + k] += f.x;
+            acc[q * V + k + 1] += f.y;
+            acc[q * V + k + 2] += f.z;
+            acc[q * V + k + 3] += f.w;
+          }
       }
     }
-    agg_finalize<V>(acc, nv, len, eta, renorm, d, Xt + m * d, sh);
+    agg_finalize<V, NV>(acc, len, eta, renorm, d, Xt + m * d, sh);
     __syncthreads();
   }
 }
@@ -1318,34 +1368,63 @@ int launch_row_norms(const void* X, int x_dtype, int64_t rows, int d, int64_t ld
 size_t agg_item_capacity(int64_t Mtot, int64_t Ntot) { return (size_t)(Mtot + Ntot / AGG_CH + 2); }
 size_t agg_part_capacity(int64_t Ntot) { return (size_t)(2 * (Ntot / AGG_CH) + 2); }
 
-int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
-                     const int* perm, const int* mstart, const int* mlen, int64_t Mtot,
-                     int64_t Ntot, int renorm, float* Xt, int* it_start, int* pt_start,
-                     int2* items, int* counts, float* part, float* part_eta,
-                     cudaStream_t stream) {
+namespace {
+template <typename T, int NV>
+void launch_agg_t(const void* X, int d, int64_t ldx, const int* perm, const int* mstart,
+                  const int* mlen, int64_t Mtot, int64_t blocks, int64_t fblocks, int renorm,
+                  float* Xt, const int* pt_start, const int2* items, const int* counts,
+                  float* part, float* part_eta, cudaStream_t stream) {
+  constexpr int V = VecOf<T>::V;
+  agg_partial_kernel<T, NV><<<(unsigned)blocks, AGG_T, 0, stream>>>(
+      (const T*)X, d, ldx, perm, mstart, mlen, items, counts, pt_start, renorm, Xt, part,
+      part_eta);
+  count_launch(1);
+  agg_final_kernel<V, NV><<<(unsigned)fblocks, AGG_T, 0, stream>>>(d, mlen, pt_start, Mtot,
+                                                                   renorm, part, part_eta, Xt);
+  count_launch(1);
+}
+
+template <typename T>
+int launch_agg_dtype(const void* X, int d, int64_t ldx, const int* perm, const int* mstart,
+                     const int* mlen, int64_t Mtot, int64_t blocks, int64_t fblocks, int renorm,
+                     float* Xt, const int* pt_start, const int2* items, const int* counts,
+                     float* part, float* part_eta, cudaStream_t stream) {
+  constexpr int V = VecOf<T>::V;
+  const int nv = (d / V + AGG_T - 1) / AGG_T;
+#define SLS_AGG_NV(N)                                                                      \
+  launch_agg_t<T, N>(X, d, ldx, perm, mstart, mlen, Mtot, blocks, fblocks, renorm, Xt,    \
+                     pt_start, items, counts, part, part_eta, stream)
+  if (nv <= 1)
+    SLS_AGG_NV(1);
+  else if (nv <= 2)
+    SLS_AGG_NV(2);
+  else if (nv <= 4)
+    SLS_AGG_NV(4);
+  else if (nv <= 8)
+    SLS_AGG_NV(8);
+  else
+    return SLS_ERR_UNSUPPORTED;
+#undef SLS_AGG_NV
+  SLS_CUDA_TRY(cudaGetLastError());
+  return SLS_OK;
+}
+}  // namespace
+
+int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* perm,
+                     const int* mstart, const int* mlen, int64_t Mtot, int64_t Ntot, int renorm,
+                     float* Xt, int* it_start, int* pt_start, int2* items, int* counts,
+                     float* part, float* part_eta, cudaStream_t stream) {
   if (Mtot == 0) return SLS_OK;
   agg_items_kernel<<<1, SEG_T, 0, stream>>>(mlen, Mtot, it_start, pt_start, items, counts);
   SLS_LAUNCH_CHECK();
   int64_t blocks = (int64_t)agg_item_capacity(Mtot, Ntot);
   if (blocks > 16384) blocks = 16384;
-  int64_t fblocks = Mtot < 4096 ? Mtot : 4096;
-  if (x_dtype == SLS_F32) {
-    agg_partial_kernel<float><<<(unsigned)blocks, AGG_T, 0, stream>>>(
-        (const float*)X, d, ldx, norms, perm, mstart, mlen, items, counts, pt_start, renorm, Xt,
-        part, part_eta);
-    SLS_LAUNCH_CHECK();
-    agg_final_kernel<4><<<(unsigned)fblocks, AGG_T, 0, stream>>>(d, mlen, pt_start, Mtot, renorm,
-                                                                 part, part_eta, Xt);
-  } else {
-    agg_partial_kernel<uint16_t><<<(unsigned)blocks, AGG_T, 0, stream>>>(
-        (const uint16_t*)X, d, ldx, norms, perm, mstart, mlen, items, counts, pt_start, renorm,
-        Xt, part, part_eta);
-    SLS_LAUNCH_CHECK();
-    agg_final_kernel<8><<<(unsigned)fblocks, AGG_T, 0, stream>>>(d, mlen, pt_start, Mtot, renorm,
-                                                                 part, part_eta, Xt);
-  }
-  SLS_LAUNCH_CHECK();
-  return SLS_OK;
+  const int64_t fblocks = Mtot < 4096 ? Mtot : 4096;
+  if (x_dtype == SLS_F32)
+    return launch_agg_dtype<float>(X, d, ldx, perm, mstart, mlen, Mtot, blocks, fblocks, renorm,
+                                   Xt, pt_start, items, counts, part, part_eta, stream);
+  return launch_agg_dtype<uint16_t>(X, d, ldx, perm, mstart, mlen, Mtot, blocks, fblocks, renorm,
+                                    Xt, pt_start, items, counts, part, part_eta, stream);
 }
 
 int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
