@@ -7,6 +7,13 @@ D = 2048 RFF features, r = 64 Lanczos steps, b = 16 SimHash bits, rho = 16,
 last 12 tokens preserved, global backend.  Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
+                  [--workload qwen7b|qwen14b|mistral7b|adaptive] [--rho R]
+
+--workload qwen14b (N = 131072, d = 5120) and mistral7b (N = 8192, d = 4096)
+time the other single-prompt shapes; --workload adaptive times the windowed
+batch: 64 prompts of N = 16384, d = 4096 bf16 (duplication 0.6 p / 63 for
+prompt p), windows of 2048 routed to the chunk or the spectral chain, D = 1024,
+r = 32, bits from the window budget, rho from --rho (default 8).
 
 The prompt (235 MB of embeddings) and the feature matrix (268 MB) are both
 larger than the 129 MB L2, so no extra flush runs between steps.  With
@@ -39,7 +46,10 @@ def parse():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
-    ap.add_argument("--workload", default="qwen7b")
+    ap.add_argument("--workload", default="qwen7b",
+                    choices=["qwen7b", "qwen14b", "mistral7b", "adaptive"])
+    ap.add_argument("--rho", type=float, default=None,
+                    help="compression ratio (default: the workload's)")
     ap.add_argument("--cpu-sample", type=int, default=4096,
                     help="tokens of the prompt the CPU oracle compresses per baseline step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -55,12 +65,21 @@ def workload(name):
     return WL.WORKLOADS[name]
 
 
-def config_dict(w, extra=None):
-    d = {"workload": f"{w.name}-shaped prompt: N={w.N} d={w.d} bf16, D={w.D} r={w.r} "
-                     f"b={w.bits} rho={int(w.rho)} preserve_last={w.preserve_last}, "
-                     f"global backend",
-         "N": w.N, "d": w.d, "D": w.D, "r": w.r, "bits": w.bits, "rho": w.rho,
-         "l2": "inputs larger than L2 (X 235 MB and Phi 268 MB per step), no flush"}
+def config_dict(w, rho, extra=None):
+    if w.batch > 1:
+        d = {"workload": f"{w.name}: {w.batch} prompts of N={w.N} d={w.d} bf16, windows of "
+                         f"{w.window}, D={w.D} r={w.r} b=auto rho={rho:g} "
+                         f"preserve_last={w.preserve_last}, adaptive backend",
+             "B": w.batch, "window": w.window,
+             "l2": (f"inputs larger than L2 (X {w.batch * w.N * w.d * 2 / 1e9:.1f} GB per "
+                    f"step), no flush")}
+    else:
+        d = {"workload": f"{w.name}-shaped prompt: N={w.N} d={w.d} bf16, D={w.D} r={w.r} "
+                         f"b={w.bits} rho={rho:g} preserve_last={w.preserve_last}, "
+                         f"global backend",
+             "l2": (f"inputs larger than L2 (X {w.N * w.d * 2 / 1e6:.0f} MB and Phi "
+                    f"{w.N * w.D * 4 / 1e6:.0f} MB per step), no flush")}
+    d.update({"N": w.N, "d": w.d, "D": w.D, "r": w.r, "bits": w.bits, "rho": rho})
     if extra:
         d.update(extra)
     return d
@@ -130,53 +149,105 @@ def lanczos_algorithmic_bytes(n_tokens, D, r):
     return n_tokens * (8 * r * D + 16 * r * (r + 1))
 
 
-def cpu_oracle_step(w, X64, prm, n):
+def window_lengths(w):
+    """Lengths of the adaptive windows over one prompt's compressible region
+    (consecutive windows, the last one shorter)."""
+    nc = w.N - w.preserve_first - w.preserve_last
+    return [min(w.window, nc - s) for s in range(0, nc, w.window)]
+
+
+def oracle_config(w, rho):
     import oracle as O
-    cfg = O.CompressConfig(rho=w.rho, D=w.D, r=w.r, bits=w.bits, preserve_last=w.preserve_last)
+    return O.CompressConfig(rho=rho, D=w.D, r=w.r, bits=w.bits,
+                            preserve_first=w.preserve_first, preserve_last=w.preserve_last,
+                            window=w.window if w.batch > 1 else 2048)
+
+
+def cpu_oracle_step(w, rho, X64, prm, n):
+    """One oracle compression of the first n tokens of a prompt (global
+    backend, or the adaptive backend for the windowed batch)."""
+    import oracle as O
+    cfg = oracle_config(w, rho)
     t = time.perf_counter()
-    O.compress_global(X64[:n], prm.w_f64(), prm.b, prm.R, prm.q1, cfg)
+    if w.batch > 1:
+        O.compress_adaptive(X64[:n], prm.w_f64(), prm.b, prm.R, prm.q1[:n], cfg)
+    else:
+        O.compress_global(X64[:n], prm.w_f64(), prm.b, prm.R, prm.q1, cfg)
     return time.perf_counter() - t
 
 
-def cpu_baseline(w, p, prm, n, budget_s=10.0):
-    """The oracle as it stands, on the first n tokens of the prompt, repeated
+def sample_prompt(w):
+    """The prompt the CPU oracle samples: the only prompt of a single-prompt
+    workload, the middle prompt of the adaptive batch."""
+    import workloads as WL
+    if w.batch > 1:
+        i = w.batch // 2
+        return WL.make_prompt(w, index=i, dup_frac=WL.adaptive_dup_frac(i, w.batch)), i
+    return WL.make_prompt(w), 0
+
+
+def cpu_baseline(w, rho, X64, prm, n, pidx, budget_s=10.0):
+    """The oracle as it stands, on the first n tokens of one prompt, repeated
     until about budget_s seconds of CPU work have been timed."""
-    X64 = p.x_f64()
     tot, reps = 0.0, 0
     while reps == 0 or tot < budget_s:
-        tot += cpu_oracle_step(w, X64, prm, n)
+        tot += cpu_oracle_step(w, rho, X64, prm, n)
         reps += 1
+    kind = "compress_adaptive" if w.batch > 1 else "compress_global"
     return {"value": n * reps / tot, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"oracle compress_global (numpy float64, BLAS threads = all cores) on the "
-                      f"first {n} tokens of the {w.name}-shaped prompt, D={w.D} r={w.r} "
-                      f"b={w.bits} rho={int(w.rho)}; {reps} run(s), {tot:.1f} s"}
+            "sample": f"oracle {kind} (numpy float64, BLAS threads = all cores) on the first "
+                      f"{n} tokens of prompt {pidx} of the {w.name} workload, D={w.D} r={w.r} "
+                      f"b={w.bits or 'auto'} rho={rho:g}; {reps} run(s), {tot:.1f} s"}
 
 
 def run_reference(args, rank, world):
     import workloads as WL
     w = workload(args.workload)
+    rho = args.rho or w.rho
     if rank != 0:
         return
-    p = WL.make_prompt(w)
+    p, pidx = sample_prompt(w)
     prm = WL.params_for(w)
     X64 = p.x_f64()
     n = args.ref_sample
     for _ in range(args.warmup):
-        cpu_oracle_step(w, X64, prm, min(n, 512))
-    ts = [cpu_oracle_step(w, X64, prm, n) for _ in range(args.steps)]
+        cpu_oracle_step(w, rho, X64, prm, min(n, 512))
+    ts = [cpu_oracle_step(w, rho, X64, prm, n) for _ in range(args.steps)]
     tot = sum(ts)
     value = n * args.steps / tot
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
-            "config": config_dict(w, {"sample_tokens": n}),
+            "config": config_dict(w, rho, {"sample_tokens": n}),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
                              "kind": "oracle",
-                             "sample": f"oracle compress_global on the first {n} tokens per step"},
+                             "sample": f"oracle on the first {n} tokens of prompt {pidx} "
+                                       f"per step"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def device_inputs(w, rank, dev):
+    """Embeddings on the device: one prompt, or the adaptive batch of
+    w.batch prompts gathered on the device from one bf16 vocabulary table
+    (the same rows and ids as workloads.make_prompt)."""
+    import numpy as np
+    import torch
+    import workloads as WL
+    if w.batch == 1:
+        p = WL.make_prompt(w, index=rank)
+        return torch.from_numpy(p.X.view(np.int16)).view(torch.bfloat16).to(dev)
+    ids = [WL.prompt_ids(w, index=i, dup_frac=WL.adaptive_dup_frac(i, w.batch))
+           for i in range(w.batch)]
+    uniq, inv = np.unique(np.concatenate(ids), return_inverse=True)
+    table = WL.f32_to_bf16_bits(WL.vocab_rows(WL.DATA_SEED, uniq, w.d).astype(np.float32))
+    tab = torch.from_numpy(table.view(np.int16)).to(dev)
+    idx = torch.from_numpy(inv.astype(np.int64)).to(dev)
+    X = tab.index_select(0, idx).view(torch.bfloat16).view(w.batch, w.N, w.d)
+    del tab
+    return X
 
 
 def run_native(args, rank, world):
@@ -190,31 +261,48 @@ def run_native(args, rank, world):
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
     w = workload(args.workload)
-    p = WL.make_prompt(w, index=rank)
+    rho = args.rho or w.rho
+    adaptive = w.batch > 1
+    X = device_inputs(w, rank, dev)
     prm = WL.params_for(w)
-    X = torch.from_numpy(p.X.view(np.int16)).view(torch.bfloat16).to(dev)
     Wt = torch.from_numpy(prm.W.view(np.int16)).view(torch.bfloat16).to(dev)
     bt = torch.from_numpy(prm.b).to(dev)
     Rt = torch.from_numpy(prm.R).to(dev)
     qt = torch.from_numpy(prm.q1).to(dev)
-    cfg = sls.Config.make(backend=sls.BACKEND_GLOBAL, rho=w.rho, D=w.D, r=w.r, bits=w.bits,
-                          preserve_last=w.preserve_last)
-    N, d = w.N, w.d
+    if adaptive:
+        cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=w.D, r=w.r, bits=w.bits,
+                              window=w.window, preserve_first=w.preserve_first,
+                              preserve_last=w.preserve_last)
+    else:
+        cfg = sls.Config.make(backend=sls.BACKEND_GLOBAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
+                              preserve_first=w.preserve_first, preserve_last=w.preserve_last)
+    B, N, d = w.batch, w.N, w.d
     M = sls.output_count(cfg, N)
-    ws = sls.Workspace(cfg, 1, N, d, dev)
-    Xt = torch.empty((1, M, d), dtype=torch.float32, device=dev)
-    pos = torch.empty((1, M), dtype=torch.int32, device=dev)
-    t2m = torch.empty((1, N), dtype=torch.int32, device=dev)
+    ws = sls.Workspace(cfg, B, N, d, dev)
+    Xt = torch.empty((B, M, d), dtype=torch.float32, device=dev)
+    pos = torch.empty((B, M), dtype=torch.int32, device=dev)
+    t2m = torch.empty((B, N), dtype=torch.int32, device=dev)
     out = (Xt, pos, t2m)
+    Xin = X if adaptive else X.view(1, N, d)
 
     def step():
-        sls.compress(X, cfg, Wt, bt, Rt, qt, workspace=ws, out=out)
+        return sls.compress(Xin, cfg, Wt, bt, Rt, qt, workspace=ws, out=out)
 
     for _ in range(args.warmup):
-        step()
+        res = step()
     torch.cuda.synchronize()
     if sls.workspace_status(ws) != 0:
         raise RuntimeError("device wait timed out during warm-up")
+    # tokens that run through the spectral chain (Lanczos)
+    if adaptive:
+        lens = window_lengths(w)
+        route = res[4].cpu().numpy()[:B * len(lens)].reshape(B, len(lens))
+        lz_tokens = int(sum(int(route[i, k]) * lens[k]
+                            for i in range(B) for k in range(len(lens))))
+        n_spec = int(route.sum())
+    else:
+        lz_tokens = N - w.preserve_first - w.preserve_last
+        n_spec = 1
 
     nph = len(sls.PHASES)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * nph)]
@@ -257,14 +345,13 @@ def run_native(args, rank, world):
     if world > 1:
         dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
     ms_max = float(ms_t.item())
-    value = world * N / (ms_max / 1e3)
+    value = world * B * N / (ms_max / 1e3)
 
     # roofline of the dominant kernel (the persistent Lanczos kernel)
-    Nc = N - w.preserve_last
-    alg = lanczos_algorithmic_bytes(Nc, w.D, w.r)
+    alg = lanczos_algorithmic_bytes(lz_tokens, w.D, w.r)
     lz_s = phases["lanczos"] / 1e3
     peak, src = peaks()
-    achieved = alg / lz_s / 1e9
+    achieved = alg / lz_s / 1e9 if lz_s > 0 else 0.0
     roof = {"bound": "hbm", "kernel": "lanczos_kernel", "achieved": achieved, "peak": peak,
             "unit": "GB/s", "frac": achieved / peak, "peak_source": src,
             "algorithmic_bytes": alg, "traffic": None}
@@ -273,7 +360,8 @@ def run_native(args, rank, world):
         try:
             with open(tr) as f:
                 t = json.load(f)
-            if t.get("workload") == w.name and t.get("kernel_rev") == LANCZOS_KERNEL_REV:
+            if (t.get("workload") == w.name and t.get("kernel_rev") == LANCZOS_KERNEL_REV
+                    and not adaptive):
                 roof["traffic"] = t["dram_bytes_per_launch"]
         except Exception:
             pass
@@ -281,8 +369,8 @@ def run_native(args, rank, world):
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        Xh = X.cpu().pin_memory()
-        Xd = torch.empty_like(X)
+        Xh = Xin.cpu().pin_memory()
+        Xd = torch.empty_like(Xin)
         Xth = torch.empty(Xt.shape, dtype=Xt.dtype).pin_memory()
         posh = torch.empty(pos.shape, dtype=pos.dtype).pin_memory()
         t2mh = torch.empty(t2m.shape, dtype=t2m.dtype).pin_memory()
@@ -307,22 +395,25 @@ def run_native(args, rank, world):
         m2 = torch.tensor([ms2], device=dev)
         if world > 1:
             dist.all_reduce(m2, op=dist.ReduceOp.MAX)
-        e2e = {"value": world * N / (float(m2.item()) / 1e3), "unit": UNIT,
-               "h2d_bytes_per_step": X.numel() * 2,
+        e2e = {"value": world * B * N / (float(m2.item()) / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": Xin.numel() * 2,
                "d2h_bytes_per_step": Xt.numel() * 4 + pos.numel() * 4 + t2m.numel() * 4}
 
     if rank != 0:
         return
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        cpu = cpu_baseline(w, p, prm, args.cpu_sample)
+        p, pidx = sample_prompt(w)
+        cpu = cpu_baseline(w, rho, p.x_f64(), prm, args.cpu_sample, pidx)
+    extra = {"parallelism": f"replicas x{world}",
+             "inputs": "bf16 embeddings and Omega; float32 Phi; double-float Lanczos vectors"}
+    if adaptive:
+        extra.update({"spectral_windows": n_spec, "spectral_tokens": lz_tokens})
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f32", "data": "synthetic",
-            "config": config_dict(w, {"parallelism": f"replicas x{world}",
-                                      "inputs": "bf16 embeddings and Omega; float32 Phi; "
-                                                "double-float Lanczos vectors"}),
+            "config": config_dict(w, rho, extra),
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
             "clocks": clk, "phases_ms": phases,
             "lanczos_gbs_algorithmic": achieved}
