@@ -130,6 +130,26 @@ int sls_feature_map(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
                     const void* W, const float* b, int D, float* Phi,
                     void* stream);
 
+/*
+ * The same features for a batch of nb equal-length prompts in one launch
+ * (Sec. 3.2 Eq. rff_map, per token), optionally only for the windows the
+ * adaptive router sent to the spectral chain (Sec. 3.6):
+ *   prompt k, row i < rows:  X row k * x_stride + i  ->  Phi row k * rows + i.
+ * X rows have stride ldx elements; W: D x d; b: D floats; Phi: nb * rows x D.
+ * live (may be NULL = every row): device int32, nwin flags per prompt
+ * (prompt-major); flag w covers rows [w * win, (w + 1) * win) of its prompt.
+ * Phi rows are written for every 128-row tile that touches a window with a
+ * nonzero flag and may be left unwritten elsewhere.  bf16 only, on the
+ * tensor cores; requires D % 256 == 0, d % 8 == 0, ldx % 8 == 0 and 16-byte
+ * aligned pointers.  Errors: INVALID_ARG for bad sizes or NULL pointers,
+ * UNSUPPORTED outside the shapes above.
+ */
+int sls_feature_map_batched(const void* X, int64_t nb, int64_t rows,
+                            int64_t x_stride, int d, int64_t ldx,
+                            const void* W, const float* b, int D, float* Phi,
+                            const int32_t* live, int nwin, int win,
+                            void* stream);
+
 /* Device workspace bytes needed by sls_lanczos_topr for one problem. */
 size_t sls_lanczos_workspace_size(int64_t N, int D, int r);
 

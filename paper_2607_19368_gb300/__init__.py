@@ -21,6 +21,7 @@ __all__ = [
     "SLS_OK", "SLS_F32", "SLS_BF16", "POS_MAX", "POS_MEDIAN", "POS_MEAN",
     "MODE_REPRESENTATIVE", "MODE_COMPACT", "BACKEND_GLOBAL", "BACKEND_ADAPTIVE",
     "BACKEND_CHUNK", "Config", "SLSError", "lib", "lib_path", "feature_map",
+    "feature_map_batched",
     "lanczos_topr", "simhash", "aggregate", "compress", "output_count",
     "compress_workspace_size", "workspace_status", "EXPORTED", "PHASES",
     "set_phase_events", "launch_count", "Workspace",
@@ -83,6 +84,8 @@ EXPORTED = {
     "sls_status_string": (ctypes.c_char_p, [_i32]),
     "sls_version": (_i32, []),
     "sls_feature_map": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _vp, _i32, _vp, _vp]),
+    "sls_feature_map_batched": (_i32, [_vp, _i64, _i64, _i64, _i32, _i64, _vp, _vp, _i32, _vp,
+                                       _vp, _i32, _i32, _vp]),
     "sls_lanczos_workspace_size": (_sz, [_i64, _i32, _i32]),
     "sls_lanczos_topr": (_i32, [_vp, _i64, _i32, _i32, _vp, _d, _vp, _vp, _vp, _vp, _vp, _vp,
                                 _sz, _vp]),
@@ -168,6 +171,33 @@ def feature_map(X: torch.Tensor, W: torch.Tensor, b: torch.Tensor,
     st = lib().sls_feature_map(_ptr(X), _dtype_code(X), N, d, X.stride(0), _ptr(W),
                                _ptr(b.float().contiguous()), D, _ptr(out), _stream(X))
     _check("sls_feature_map", st)
+    return out
+
+
+def feature_map_batched(X: torch.Tensor, W: torch.Tensor, b: torch.Tensor, rows: int,
+                        live: Optional[torch.Tensor] = None, win: int = 0,
+                        out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Features of the first `rows` rows of every prompt of a B x N x d bf16
+    batch in one launch (Sec. 3.2, Eq. rff_map); with `live` (int32, B x nwin
+    window flags, Sec. 3.6) only the row tiles of live windows are written.
+    Returns B * rows x D float32."""
+    _need_cuda(X, W, b)
+    B, N, d = X.shape
+    D = W.shape[0]
+    assert X.stride(2) == 1 and X.stride(0) == N * X.stride(1)
+    assert W.shape[1] == d and W.dtype == X.dtype and W.is_contiguous()
+    if out is None:
+        out = torch.empty((B * rows, D), dtype=torch.float32, device=X.device)
+    nwin = 0
+    lp = None
+    if live is not None:
+        live = live.to(device=X.device, dtype=torch.int32).contiguous()
+        nwin = live.numel() // max(1, B)
+        lp = _ptr(live)
+    st = lib().sls_feature_map_batched(_ptr(X), B, rows, N, d, X.stride(1), _ptr(W),
+                                       _ptr(b.float().contiguous()), D, _ptr(out), lp, nwin,
+                                       win, _stream(X))
+    _check("sls_feature_map_batched", st)
     return out
 
 

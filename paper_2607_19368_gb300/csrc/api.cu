@@ -274,6 +274,7 @@ struct CompressWs {
   int64_t* lz_q1off;
   int* nspec;
   float* score;
+  int32_t* route;  // spectral flag per problem
   float* Phi;
   float2* Q;
   double *alpha, *beta, *theta, *S;
@@ -283,7 +284,6 @@ struct CompressWs {
   void* lz_scratch;
   size_t lz_bytes;
   void* seg_scratch;
-  float* norms;
   int *perm, *mstart, *mlen;
   int *it_start, *pt_start;
   int2* items;
@@ -363,6 +363,7 @@ void carve(const CompressPlan& P, void* ws, CompressWs* W) {
   W->lz_q1off = cv.take<int64_t>(np);
   W->nspec = cv.take<int>(1);
   W->score = cv.take<float>(np);
+  W->route = cv.take<int>(np);
   W->Phi = cv.take<float>(spectral ? (size_t)rows * P.D : 0);
   W->Q = cv.take<float2>(spectral ? (size_t)rows * ((P.r + 1) & ~1) : 0);
   W->alpha = cv.take<double>(spectral ? (size_t)np * P.r : 0);
@@ -375,7 +376,6 @@ void carve(const CompressPlan& P, void* ws, CompressWs* W) {
   W->lz_bytes = spectral ? lanczos_scratch_bytes(P.nmax, P.D, P.r, P.lz_groups, P.lz_g) : 0;
   W->lz_scratch = cv.take<char>(W->lz_bytes);
   W->seg_scratch = cv.take<char>(segment_scratch_bytes(P.nmax, P.mmax, P.seg_slots));
-  W->norms = cv.take<float>(toks);
   W->perm = cv.take<int>(toks);
   W->mstart = cv.take<int>(macs);
   W->mlen = cv.take<int>(macs);
@@ -444,6 +444,18 @@ int sls_feature_map(const void* X, int x_dtype, int64_t N, int d, int64_t ldx, c
     if (st != SLS_ERR_UNSUPPORTED) return st;
   }
   return launch_feature_map_simt(X, x_dtype, N, d, ldx, W, b, D, Phi, s);
+}
+
+int sls_feature_map_batched(const void* X, int64_t nb, int64_t rows, int64_t x_stride, int d,
+                            int64_t ldx, const void* W, const float* b, int D, float* Phi,
+                            const int32_t* live, int nwin, int win, void* stream) {
+  if (nb < 0 || rows < 0 || x_stride < rows || d < 1 || ldx < d || D < 4 || D > SLS_MAX_D)
+    return SLS_ERR_INVALID_ARG;
+  if (live && (nwin < 1 || win < 1 || (int64_t)nwin * win < rows)) return SLS_ERR_INVALID_ARG;
+  if (nb == 0 || rows == 0) return SLS_OK;
+  if (!X || !W || !b || !Phi) return SLS_ERR_INVALID_ARG;
+  return launch_feature_map_tc_batched(X, nb, rows, x_stride, d, ldx, W, b, D, Phi, live, nwin,
+                                       win, (cudaStream_t)stream, nullptr);
 }
 
 size_t sls_lanczos_workspace_size(int64_t N, int D, int r) {
@@ -631,13 +643,12 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
         cfg->backend == SLS_BACKEND_CHUNK ? P.k_chunk : 0, spectral ? params->q1_stride : 0);
     SLS_LAUNCH_CHECK();
   }
-  // routing (the window score needs every token's norm first)
+  // routing; at rho >= 16 every window is spectral and no score is needed
   int mode = spectral ? 0 : 1;
   if (cfg->backend == SLS_BACKEND_ADAPTIVE) {
     mode = 2;
-    if ((st = launch_row_norms(X, x_dtype, B * N, d, ldx, W.norms, s)) != SLS_OK) return st;
-    if ((st = launch_window_score(X, x_dtype, d, ldx, W.norms, W.probs, nprob, W.score, s)) !=
-        SLS_OK)
+    if (cfg->rho < 16.0 &&
+        (st = launch_window_score(X, x_dtype, d, ldx, W.probs, nprob, W.score, s)) != SLS_OK)
       return st;
   }
   double tau = cfg->tau;
@@ -646,21 +657,32 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
     if (tau > 0.70) tau = 0.70;
     if (tau < 0.55) tau = 0.55;
   }
+  int32_t* rflags = route ? route : W.route;
   route_compact_kernel<<<1, 1024, 0, s>>>(W.probs, nprob, mode, W.score, cfg->rho, tau,
                                           W.spec_list, W.lz_row0, W.lz_n, W.lz_q1off, W.nspec,
-                                          route);
+                                          rflags);
   SLS_LAUNCH_CHECK();
   phase_mark(0, 1, s);
   phase_mark(1, 0, s);
   if (spectral) {
-    // features for every compressible row of every prompt
-    for (int64_t b = 0; b < B; ++b) {
-      const char* xb = (const char*)X +
-                       (size_t)(b * N + P.pf) * ldx * (x_dtype == SLS_BF16 ? 2 : 4);
-      st = sls_feature_map(xb, x_dtype, P.Nc, d, ldx, params->W, params->b, cfg->D,
-                           W.Phi + (size_t)b * P.Nc * cfg->D, stream);
-      if (st != SLS_OK) return st;
+    // features of the compressible rows of every prompt, in one launch on the
+    // tensor cores (bf16); windows routed to the chunk path are skipped
+    st = SLS_ERR_UNSUPPORTED;
+    if (x_dtype == SLS_BF16)
+      st = launch_feature_map_tc_batched(
+          (const char*)X + (size_t)P.pf * ldx * 2, B, P.Nc, N, d, ldx, params->W, params->b,
+          cfg->D, W.Phi, mode == 2 ? rflags : nullptr, (int)P.bud.W, (int)P.bud.L_full, s,
+          W.status);
+    if (st == SLS_ERR_UNSUPPORTED) {
+      for (int64_t b = 0; b < B; ++b) {
+        const char* xb = (const char*)X +
+                         (size_t)(b * N + P.pf) * ldx * (x_dtype == SLS_BF16 ? 2 : 4);
+        st = sls_feature_map(xb, x_dtype, P.Nc, d, ldx, params->W, params->b, cfg->D,
+                             W.Phi + (size_t)b * P.Nc * cfg->D, stream);
+        if (st != SLS_OK) return st;
+      }
     }
+    if (st != SLS_OK) return st;
     phase_mark(1, 1, s);
     phase_mark(2, 0, s);
     LanczosBatch bt{};

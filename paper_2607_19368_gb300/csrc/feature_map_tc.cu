@@ -4,9 +4,12 @@
 // contiguous); the contraction accumulates in fp32 in tensor memory; the
 // epilogue adds b, takes the cosine, scales and stores Phi (fp32) once.
 //
-// One persistent CTA per SM, 128 x 256 output tiles (tile index -> m-block
-// outer, n-block inner, so the D/256 tiles that share an X block run at the
-// same time and X is read from HBM once).  Warp roles:
+// One persistent CTA per SM, 128 x 256 output tiles (tile index -> prompt,
+// then m-block, then n-block innermost, so the D/256 tiles that share an X
+// block run at the same time and X is read from HBM once).  One launch covers
+// a batch of prompts (equal row counts, a fixed row stride in X); with a
+// per-window route table, the row tiles whose windows all went to the chunk
+// path (Sec. 3.6) are skipped by every role alike.  Warp roles:
 //   warp 0  TMA producer: 128B-swizzled 128x64 (X) and 256x64 (W) bf16 tiles
 //           into a 4-stage shared-memory ring (mbarrier complete_tx);
 //   warp 1  MMA issuer: one elected thread issues tcgen05.mma (M=128, N=256,
@@ -109,10 +112,32 @@ SLS_DEV bool tc_wait(uint64_t* bar, unsigned parity, volatile int* abort_flag) {
   return false;
 }
 
+// Rows of one launch: nb prompts of `rows` rows each, prompt b starting at
+// X row b * x_stride (of the tensor map) and Phi row b * rows.  live, when
+// set, holds one flag per window of `win` rows (nwin per prompt,
+// prompt-major); a row tile is computed only if a window it touches is live.
+struct FmJob {
+  int nb;
+  int rows;
+  int x_stride;
+  const int* live;
+  int nwin;
+  int win;
+};
+
+SLS_DEV bool fm_tile_live(const FmJob& J, int b, int mb) {
+  if (!J.live) return true;
+  const int r0 = mb * 128;
+  const int r1 = min(J.rows, r0 + 128) - 1;
+  for (int k = r0 / J.win; k <= r1 / J.win && k < J.nwin; ++k)
+    if (J.live[(int64_t)b * J.nwin + k]) return true;
+  return false;
+}
+
 __global__ void __launch_bounds__(TC_THREADS, 1)
 feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
                       const __grid_constant__ CUtensorMap tmW, const float* __restrict__ bvec,
-                      float* __restrict__ Phi, int N, int D, int K, float scale, int* status) {
+                      float* __restrict__ Phi, FmJob J, int D, int K, float scale, int* status) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES], tfull[2], tempty[2], done_bar;
   __shared__ uint32_t tmem_holder;
@@ -122,9 +147,10 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const uint32_t smem_base = smem_u32(smem);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m_tiles = (N + TC_BM - 1) / TC_BM;
+  const int m_tiles = (J.rows + TC_BM - 1) / TC_BM;
   const int n_tiles = D / TC_BN;
-  const int num_tiles = m_tiles * n_tiles;
+  const int per_prompt = m_tiles * n_tiles;
+  const int num_tiles = J.nb * per_prompt;
   const int k_blocks = (K + TC_BK - 1) / TC_BK;
 
   if (threadIdx.x == 0) {
@@ -163,7 +189,10 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       unsigned it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        const int mb = tile / n_tiles, nb = tile % n_tiles;
+        const int pb = tile / per_prompt, rem = tile % per_prompt;
+        const int mb = rem / n_tiles, nb = rem % n_tiles;
+        if (!fm_tile_live(J, pb, mb)) continue;
+        const int y = pb * J.x_stride + mb * TC_BM;
         for (int kb = 0; kb < k_blocks; ++kb, ++it) {
           const int s = it % TC_STAGES;
           const unsigned par = (it / TC_STAGES) & 1u;
@@ -175,7 +204,7 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
           const uint32_t a_dst = smem_base + s * TC_STAGE_BYTES;
           const uint32_t b_dst = a_dst + TC_A_BYTES;
           mbar_expect_tx(&full_bar[s], TC_STAGE_BYTES);
-          tma_load_2d(a_dst, &tmX, kb * TC_BK, mb * TC_BM, smem_u32(&full_bar[s]));
+          tma_load_2d(a_dst, &tmX, kb * TC_BK, y, smem_u32(&full_bar[s]));
           tma_load_2d(b_dst, &tmW, kb * TC_BK, nb * TC_BN, smem_u32(&full_bar[s]));
         }
       }
@@ -193,7 +222,8 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
     if (lane == 0) {
       unsigned it = 0, acc_it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++acc_it) {
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        if (!fm_tile_live(J, tile / per_prompt, (tile % per_prompt) / n_tiles)) continue;
         const int acc = acc_it & 1;
         const unsigned apar = (acc_it >> 1) & 1u;
         if (!tc_wait(&tempty[acc], apar ^ 1u, &s_abort)) {
@@ -221,6 +251,7 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
           tc_commit(smem_u32(&empty_bar[s]));
         }
         if (ok) tc_commit(smem_u32(&tfull[acc]));
+        ++acc_it;
       }
       // all MMAs issued by this thread have completed before TMEM is freed
       tc_commit(smem_u32(&done_bar));
@@ -233,8 +264,10 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
     // ------------------------------ epilogue ----------------------------------
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     unsigned acc_it = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++acc_it) {
-      const int mb = tile / n_tiles, nb = tile % n_tiles;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      const int pb = tile / per_prompt, rem = tile % per_prompt;
+      const int mb = rem / n_tiles, nb = rem % n_tiles;
+      if (!fm_tile_live(J, pb, mb)) continue;
       const int acc = acc_it & 1;
       const unsigned apar = (acc_it >> 1) & 1u;
       if (!tc_wait(&tfull[acc], apar, &s_abort)) {
@@ -243,12 +276,12 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       }
       tc_fence_after();
       const int row = mb * TC_BM + q * 32 + lane;
-      float* out = Phi + (size_t)row * D + (size_t)nb * TC_BN;
+      float* out = Phi + ((int64_t)pb * J.rows + row) * D + (int64_t)nb * TC_BN;
       const float* bb = bvec + (size_t)nb * TC_BN;
       for (int c0 = 0; c0 < TC_BN; c0 += 32) {
         uint32_t v[32];
         tc_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + c0), v);
-        if (row < N) {
+        if (row < J.rows) {
 #pragma unroll
           for (int e = 0; e < 32; e += 4) {
             const float4 bq = __ldg(reinterpret_cast<const float4*>(bb + c0 + e));
@@ -264,6 +297,7 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
+      ++acc_it;
     }
   }
   __syncthreads();
@@ -323,28 +357,43 @@ int sm_count() {
 
 }  // namespace
 
-int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
-                          const float* b, int D, float* Phi, cudaStream_t stream,
-                          int* status) {
+int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64_t x_stride,
+                                  int d, int64_t ldx, const void* W, const float* b, int D,
+                                  float* Phi, const int* live, int nwin, int win,
+                                  cudaStream_t stream, int* status) {
   // shapes the kernel covers; anything else takes the SIMT path
-  if (N <= 0 || N > (int64_t)INT32_MAX - TC_BM || D % TC_BN != 0 || d % 8 != 0 || ldx % 8 != 0)
+  if (nb <= 0 || rows <= 0 || x_stride < rows || D % TC_BN != 0 || d % 8 != 0 || ldx % 8 != 0)
     return SLS_ERR_UNSUPPORTED;
+  const int64_t map_rows = (nb - 1) * x_stride + rows;
+  const int64_t m_tiles = (rows + TC_BM - 1) / TC_BM;
+  if (map_rows > (int64_t)INT32_MAX - TC_BM || nb * m_tiles * (D / TC_BN) > (int64_t)INT32_MAX)
+    return SLS_ERR_UNSUPPORTED;
+  if (live && (nwin < 1 || win < 1)) return SLS_ERR_INVALID_ARG;
   if (((uintptr_t)X & 15) || ((uintptr_t)W & 15) || ((uintptr_t)b & 15) || ((uintptr_t)Phi & 15))
     return SLS_ERR_UNSUPPORTED;
   CUtensorMap mx, mw;
-  if (!make_map(&mx, X, (uint64_t)N, (uint64_t)d, (uint64_t)ldx, TC_BM)) return SLS_ERR_UNSUPPORTED;
+  if (!make_map(&mx, X, (uint64_t)map_rows, (uint64_t)d, (uint64_t)ldx, TC_BM))
+    return SLS_ERR_UNSUPPORTED;
   if (!make_map(&mw, W, (uint64_t)D, (uint64_t)d, (uint64_t)d, TC_BN)) return SLS_ERR_UNSUPPORTED;
   int* st = status;
   if (!st) SLS_CUDA_TRY(cudaGetSymbolAddress((void**)&st, g_fm_status));
   SLS_CUDA_TRY(cudaFuncSetAttribute(feature_map_tc_kernel,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TC_SMEM));
-  const int tiles = (int)((N + TC_BM - 1) / TC_BM) * (D / TC_BN);
-  const int grid = tiles < sm_count() ? tiles : sm_count();
+  const int64_t tiles = nb * m_tiles * (D / TC_BN);
+  const int grid = tiles < sm_count() ? (int)tiles : sm_count();
   const float scale = (float)sqrt(2.0 / (double)D);
-  feature_map_tc_kernel<<<grid, TC_THREADS, TC_SMEM, stream>>>(mx, mw, b, Phi, (int)N, D, d,
-                                                               scale, st);
+  FmJob J{(int)nb, (int)rows, (int)x_stride, live, nwin, win};
+  feature_map_tc_kernel<<<grid, TC_THREADS, TC_SMEM, stream>>>(mx, mw, b, Phi, J, D, d, scale,
+                                                               st);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
+}
+
+int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
+                          const float* b, int D, float* Phi, cudaStream_t stream,
+                          int* status) {
+  return launch_feature_map_tc_batched(X, 1, N, N, d, ldx, W, b, D, Phi, nullptr, 0, 0, stream,
+                                       status);
 }
 
 }  // namespace sls

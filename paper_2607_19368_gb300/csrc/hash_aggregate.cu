@@ -915,26 +915,6 @@ __global__ void identity_kernel(const T* __restrict__ X, int64_t B, int64_t N, i
 // token norms and macro-token embeddings (Eq. macro_embed)
 // ============================================================================
 
-// |x_i| for every token row; one warp per row.
-template <typename T>
-__global__ void __launch_bounds__(256)
-row_norms_kernel(const T* __restrict__ X, int64_t rows, int d, int64_t ldx,
-                 float* __restrict__ norms) {
-  const int lane = threadIdx.x & 31;
-  const int64_t wid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t i = wid; i < rows; i += nw) {
-    const T* x = X + i * ldx;
-    float s = 0.f;
-    for (int c = lane; c < d; c += 32) {
-      const float v = to_f32<T>(x[c]);
-      s = fmaf(v, v, s);
-    }
-    s = warp_sum_f(s);
-    if (lane == 0) norms[i] = sqrtf(s);
-  }
-}
-
 constexpr int AGG_T = 256;
 constexpr int AGG_CH = 64;      // members per work item
 constexpr int AGG_MAXV = 32;    // accumulators per thread (d <= 8192)
@@ -1201,41 +1181,67 @@ agg_final_kernel(int d, const int* __restrict__ mlen, const int* __restrict__ pt
 
 // score = (1/L) sum_i cos(x_i, c) with c the window centroid; computed in one
 // pass as (sum_i x_i/|x_i|) . (sum_i x_i) / (L |sum_i x_i|).  Zero rows add 0.
-template <typename T>
-__global__ void __launch_bounds__(AGG_T)
-window_score_kernel(const T* __restrict__ X, int d, int64_t ldx, const float* __restrict__ norms,
+// Rows are gathered in batches of agg_batch<NV>(); each row's |x|^2 is reduced
+// from the same registers (per warp, then across warps through a
+// double-buffered shared array, one barrier per batch), so X is read once.
+template <typename T, int NV>
+__global__ void __launch_bounds__(AGG_T, 2)
+window_score_kernel(const T* __restrict__ X, int d, int64_t ldx,
                     const ProbDesc* __restrict__ probs, int nprob, float* __restrict__ score) {
   constexpr int V = VecOf<T>::V;
-  __shared__ float sh[AGG_T / 32];
-  const int tid = threadIdx.x;
-  const int nv = (d / V + AGG_T - 1) / AGG_T;
+  constexpr int MB = agg_batch<NV>();
+  constexpr int NW = AGG_T / 32;
+  __shared__ float sh[NW];
+  __shared__ float shq[2][MB][NW];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int p = blockIdx.x; p < nprob; p += gridDim.x) {
     const ProbDesc P = probs[p];
-    float cs[AGG_MAXV], ns[AGG_MAXV];
+    float cs[NV * V], ns[NV * V];
 #pragma unroll
-    for (int k = 0; k < AGG_MAXV; ++k) cs[k] = ns[k] = 0.f;
-    for (int i = 0; i < P.n; ++i) {
-      const int64_t row = P.tok_row + i;
-      const float nr = norms[row];
-      const float inv = (nr > 0.f) ? 1.0f / nr : 0.f;
-      const T* x = X + row * ldx;
+    for (int k = 0; k < NV * V; ++k) cs[k] = ns[k] = 0.f;
+    int buf = 0;
+    for (int s0 = 0; s0 < P.n; s0 += MB, buf ^= 1) {
+      float v[MB][NV * V];
 #pragma unroll
-      for (int q = 0; q < AGG_MAXV / V; ++q) {
-        const int c0 = (tid + q * AGG_T) * V;
-        if (q < nv && c0 < d) {
-          float v[V];
-          load_vec<T>(x + c0, v);
+      for (int j = 0; j < MB; ++j) {
+        const bool live = s0 + j < P.n;
+        const T* x = X + (P.tok_row + s0 + j) * ldx;
 #pragma unroll
-          for (int k = 0; k < V; ++k) {
-            cs[q * V + k] += v[k];
-            ns[q * V + k] = fmaf(v[k], inv, ns[q * V + k]);
+        for (int q = 0; q < NV; ++q) {
+          const int c0 = (tid + q * AGG_T) * V;
+          if (live && c0 < d) {
+            load_vec<T>(x + c0, &v[j][q * V]);
+          } else {
+#pragma unroll
+            for (int k = 0; k < V; ++k) v[j][q * V + k] = 0.f;
           }
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < MB; ++j) {
+        float sq = 0.f;
+#pragma unroll
+        for (int k = 0; k < NV * V; ++k) sq = fmaf(v[j][k], v[j][k], sq);
+        sq = warp_sum_f(sq);
+        if (lane == 0) shq[buf][j][warp] = sq;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int j = 0; j < MB; ++j) {
+        float t = 0.f;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) t += shq[buf][j][w];
+        const float inv = (t > 0.f) ? 1.0f / sqrtf(t) : 0.f;
+#pragma unroll
+        for (int k = 0; k < NV * V; ++k) {
+          cs[k] += v[j][k];
+          ns[k] = fmaf(v[j][k], inv, ns[k]);
         }
       }
     }
     float dot = 0.f, cc = 0.f;
 #pragma unroll
-    for (int k = 0; k < AGG_MAXV; ++k) {
+    for (int k = 0; k < NV * V; ++k) {
       dot = fmaf(ns[k], cs[k], dot);
       cc = fmaf(cs[k], cs[k], cc);
     }
@@ -1350,21 +1356,6 @@ int launch_identity(const void* X, int x_dtype, int64_t B, int64_t N, int d, int
   return SLS_OK;
 }
 
-int launch_row_norms(const void* X, int x_dtype, int64_t rows, int d, int64_t ldx, float* norms,
-                     cudaStream_t stream) {
-  if (rows == 0) return SLS_OK;
-  int64_t blocks = (rows * 32 + 255) / 256;
-  if (blocks > 8192) blocks = 8192;
-  if (x_dtype == SLS_F32)
-    row_norms_kernel<float><<<(unsigned)blocks, 256, 0, stream>>>((const float*)X, rows, d, ldx,
-                                                                   norms);
-  else
-    row_norms_kernel<uint16_t><<<(unsigned)blocks, 256, 0, stream>>>((const uint16_t*)X, rows, d,
-                                                                      ldx, norms);
-  SLS_LAUNCH_CHECK();
-  return SLS_OK;
-}
-
 size_t agg_item_capacity(int64_t Mtot, int64_t Ntot) { return (size_t)(Mtot + Ntot / AGG_CH + 2); }
 size_t agg_part_capacity(int64_t Ntot) { return (size_t)(2 * (Ntot / AGG_CH) + 2); }
 
@@ -1427,18 +1418,38 @@ int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* 
                                     Xt, pt_start, items, counts, part, part_eta, stream);
 }
 
-int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
-                        const ProbDesc* probs, int nprob, float* score, cudaStream_t stream) {
-  if (nprob <= 0) return SLS_OK;
+namespace {
+template <typename T>
+int launch_score_dtype(const void* X, int d, int64_t ldx, const ProbDesc* probs, int nprob,
+                       float* score, cudaStream_t stream) {
+  constexpr int V = VecOf<T>::V;
+  const int nv = (d / V + AGG_T - 1) / AGG_T;
   const int blocks = nprob < 8192 ? nprob : 8192;
-  if (x_dtype == SLS_F32)
-    window_score_kernel<float><<<blocks, AGG_T, 0, stream>>>((const float*)X, d, ldx, norms,
-                                                              probs, nprob, score);
+#define SLS_SCORE_NV(N)                                                          \
+  window_score_kernel<T, N><<<blocks, AGG_T, 0, stream>>>((const T*)X, d, ldx, probs, \
+                                                          nprob, score)
+  if (nv <= 1)
+    SLS_SCORE_NV(1);
+  else if (nv <= 2)
+    SLS_SCORE_NV(2);
+  else if (nv <= 4)
+    SLS_SCORE_NV(4);
+  else if (nv <= 8)
+    SLS_SCORE_NV(8);
   else
-    window_score_kernel<uint16_t><<<blocks, AGG_T, 0, stream>>>((const uint16_t*)X, d, ldx,
-                                                                 norms, probs, nprob, score);
+    return SLS_ERR_UNSUPPORTED;
+#undef SLS_SCORE_NV
   SLS_LAUNCH_CHECK();
   return SLS_OK;
+}
+}  // namespace
+
+int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,
+                        int nprob, float* score, cudaStream_t stream) {
+  if (nprob <= 0) return SLS_OK;
+  if (x_dtype == SLS_F32)
+    return launch_score_dtype<float>(X, d, ldx, probs, nprob, score, stream);
+  return launch_score_dtype<uint16_t>(X, d, ldx, probs, nprob, score, stream);
 }
 
 }  // namespace sls

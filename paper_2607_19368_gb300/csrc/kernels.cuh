@@ -15,6 +15,14 @@ int launch_feature_map_simt(const void* X, int x_dtype, int64_t N, int d, int64_
 int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
                           const float* b, int D, float* Phi, cudaStream_t stream,
                           int* status = nullptr);
+// The same over nb prompts in one launch: prompt k has `rows` rows starting at
+// X row k * x_stride and writes Phi rows [k * rows, (k + 1) * rows).  With
+// `live` set (one flag per window of `win` rows, nwin per prompt,
+// prompt-major), row tiles whose windows are all 0 are not computed.
+int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64_t x_stride,
+                                  int d, int64_t ldx, const void* W, const float* b, int D,
+                                  float* Phi, const int* live, int nwin, int win,
+                                  cudaStream_t stream, int* status);
 
 // ---- Lanczos (Algorithm 2) --------------------------------------------------
 // A batch of independent problems, problem p owning rows
@@ -74,14 +82,12 @@ int launch_preserved(int64_t B, int64_t N, int64_t M, int pf, int pl, int pos_mo
                      cudaStream_t stream);
 int launch_identity(const void* X, int x_dtype, int64_t B, int64_t N, int d, int64_t ldx,
                     float* Xt, int32_t* pos, int32_t* tok2macro, cudaStream_t stream);
-int launch_row_norms(const void* X, int x_dtype, int64_t rows, int d, int64_t ldx, float* norms,
-                     cudaStream_t stream);
 size_t agg_item_capacity(int64_t Mtot, int64_t Ntot);
 size_t agg_part_capacity(int64_t Ntot);
 int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* perm,
                      const int* mstart, const int* mlen, int64_t Mtot, int64_t Ntot, int renorm,
                      float* Xt, int* it_start, int* pt_start, int2* items, int* counts,
                      float* part, float* part_eta, cudaStream_t stream);
-int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const float* norms,
-                        const ProbDesc* probs, int nprob, float* score, cudaStream_t stream);
+int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,
+                        int nprob, float* score, cudaStream_t stream);
 }  // namespace sls

@@ -49,6 +49,11 @@ def test_host_side_errors_and_counts(lib):
     # argument errors are detected before any CUDA call
     assert lib.sls_feature_map(None, 0, 4, 8, 8, None, None, 6, None, None) == 1  # D % 4
     assert lib.sls_simhash(None, 4, 4, 4, None, None, 33, 4, None, None) == 1     # bits > 32
+    # batched features: prompt stride below the row count; windows not covering the rows
+    assert lib.sls_feature_map_batched(None, 2, 10, 5, 8, 8, None, None, 256, None, None, 0, 0,
+                                       None) == 1
+    assert lib.sls_feature_map_batched(None, 2, 10, 10, 8, 8, None, None, 256, None,
+                                       ctypes.c_void_p(16), 2, 4, None) == 1
     assert lib.sls_lanczos_topr(None, 4, 8, 0, None, 1e-10, None, None, None, None, None,
                                 None, 0, None) == 1                               # r = 0
     assert lib.sls_lanczos_workspace_size(1000, 256, 16) > 0

@@ -76,6 +76,43 @@ def test_feature_map_ragged_and_empty(sls):
     assert out.shape == (0, 4)
 
 
+def test_feature_map_batched_live_windows(sls):
+    """One launch over a batch of prompts (Sec. 3.2) that computes only the
+    row tiles touching a live window (Sec. 3.6): computed rows match the
+    oracle; tiles with no live window stay unwritten; without flags every row
+    of every prompt matches."""
+    B, N, rows, d, D, win = 3, 700, 650, 128, 512, 200
+    w = WL.scaled(WL.WORKLOADS["mistral7b"], N=N, d=d, D=D)
+    prompts = [WL.make_prompt(w, index=k) for k in range(B)]
+    prm = WL.make_params(D, d, 8, 8, 1, "bf16")
+    Xb = np.stack([pp.X for pp in prompts])
+    X = to_torch_x(Xb, "bf16")
+    W64 = prm.w_f64()
+    tol = [feature_tolerance(pp.x_f64()[:rows], W64, prm.b.astype(np.float64))
+           for pp in prompts]
+    want = [O.rff_features(pp.x_f64()[:rows], W64, prm.b) for pp in prompts]
+    nwin = -(-rows // win)
+    live = np.array([[1, 0, 0, 1], [0, 0, 0, 0], [0, 1, 0, 0]], dtype=np.int32)
+    assert live.shape == (B, nwin)
+    out = torch.full((B * rows, D), float("nan"), device="cuda")
+    sls.feature_map_batched(X, to_torch_x(prm.W, "bf16"), torch.from_numpy(prm.b).cuda(), rows,
+                            live=torch.from_numpy(live).cuda(), win=win, out=out)
+    got = out.cpu().numpy().astype(np.float64).reshape(B, rows, D)
+    for k in range(B):
+        for t0 in range(0, rows, 128):
+            t1 = min(rows, t0 + 128)
+            touched = range(t0 // win, (t1 - 1) // win + 1)
+            tile = got[k, t0:t1]
+            if any(live[k, j] for j in touched):
+                assert np.all(np.abs(tile - want[k][t0:t1]) <= tol[k][t0:t1]), (k, t0)
+            else:
+                assert np.all(np.isnan(tile)), (k, t0)
+    full = sls.feature_map_batched(X, to_torch_x(prm.W, "bf16"), torch.from_numpy(prm.b).cuda(),
+                                   rows).cpu().numpy().astype(np.float64).reshape(B, rows, D)
+    for k in range(B):
+        assert np.all(np.abs(full[k] - want[k]) <= tol[k]), k
+
+
 # ---------------------------------------------------------------------------
 # Lanczos + Ritz pairs (Algorithm 2, Algorithm 1)
 # ---------------------------------------------------------------------------
@@ -356,17 +393,19 @@ def test_compress_chunk_backend(sls):
     assert np.max(np.abs(Xt.cpu().numpy() - res.Xt)) <= EMB_TOL
 
 
-def test_compress_adaptive_small_batch(sls):
+@pytest.mark.parametrize("D", [64, 256])
+def test_compress_adaptive_small_batch(sls, D):
     """Adaptive router on a batch of 3 prompts (windows of 96): route flags,
     budgets and chunk windows against the oracle; spectral windows by their
-    invariants."""
+    invariants.  D = 256 takes the batched tensor-core feature map, whose
+    128-row tiles straddle the windows."""
     w = WL.scaled(WL.WORKLOADS["adaptive"], N=700, d=64, batch=3)
     prompts = [WL.make_prompt(w, index=i, dup_frac=WL.adaptive_dup_frac(i, 3)) for i in range(3)]
-    prm = WL.make_params(64, 64, 8, 32, 3 * 700, "bf16")
+    prm = WL.make_params(D, 64, 8, 32, 3 * 700, "bf16")
     Xb = np.stack([pp.X for pp in prompts])
     X = to_torch_x(Xb, "bf16")
     for rho in (2.0, 4.0, 16.0):
-        cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=64, r=8, window=96,
+        cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=D, r=8, window=96,
                               preserve_last=12)
         Xt, pos, t2m, r_eff, route = sls.compress(X, cfg, to_torch_x(prm.W, "bf16"),
                                                   torch.from_numpy(prm.b).cuda(),
@@ -376,7 +415,7 @@ def test_compress_adaptive_small_batch(sls):
         nw = len(O.window_bounds(688, 96))
         route = route.cpu().numpy()[:3 * nw].reshape(3, nw)
         for i, pp in enumerate(prompts):
-            ocfg = O.CompressConfig(rho=rho, D=64, r=8, window=96, preserve_last=12)
+            ocfg = O.CompressConfig(rho=rho, D=D, r=8, window=96, preserve_last=12)
             res = O.compress_adaptive(pp.x_f64(), prm.w_f64(), prm.b, prm.R,
                                       prm.q1[i * 700:(i + 1) * 700], ocfg)
             tau = O.tau_schedule(rho)
