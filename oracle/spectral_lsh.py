@@ -24,7 +24,8 @@ __all__ = [
     "array_split_sizes", "group_position", "aggregate_groups", "order_groups",
     "compress_global", "tau_schedule", "redundancy_score", "window_bounds",
     "window_budgets", "route_windows", "chunk_groups", "spectral_groups",
-    "compress_adaptive", "compress_chunk", "complexity_ops", "CompressResult",
+    "compress_adaptive", "compress_local", "compress_chunk", "complexity_ops",
+    "CompressResult",
     "POS_MAX", "POS_MEDIAN", "POS_MEAN", "MODE_REPRESENTATIVE", "MODE_COMPACT",
 ]
 
@@ -48,7 +49,7 @@ class CompressConfig:
     pos_mode: int = MODE_REPRESENTATIVE  # Sec. 5.6 / App. B.3
     renorm: bool = True           # Eq. macro_embed
     lanczos_tol: float = 1e-10    # break threshold of Algorithm 2 (reading)
-    window: int = 2048            # adaptive backend window
+    window: int = 2048            # adaptive / local backend window
     tau: float = 0.70             # fixed threshold (App. B.3)
     tau_schedule: bool = True     # compression-aware schedule (Sec. 3.6)
 
@@ -512,12 +513,12 @@ def chunk_groups(L: int, m: int) -> List[np.ndarray]:
     return out
 
 
-def compress_adaptive(X: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray,
-                      q1: np.ndarray, cfg: CompressConfig) -> CompressResult:
-    """Adaptive backend (Sec. 3.6): windows, exact budgets, redundancy score,
-    chunk or per-window Spectral-LSH, concatenation in window order.  Each
-    spectral window uses the slice of q1 at its offset and
-    b_w = cfg.bits or ceil(log2(L_w / rho))."""
+def _windowed(X: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray,
+              q1: np.ndarray, cfg: CompressConfig, route: bool) -> CompressResult:
+    """Consecutive windows of cfg.window tokens over the compressible region,
+    exact per-window budgets (App. B.8), each window either chunk-averaged or
+    compressed by Spectral-LSH on its own tokens, macro-tokens concatenated in
+    window order.  route=False sends every window down the spectral path."""
     X = np.asarray(X, dtype=np.float64)
     N = X.shape[0]
     pf, pl, Nc = _region(N, cfg)
@@ -527,21 +528,45 @@ def compress_adaptive(X: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray
     Xc = X[pf:N - pl]
     bounds = window_bounds(Nc, cfg.window)
     budgets = window_budgets([e - s for s, e in bounds], M)
-    spectral, scores = route_windows(Xc, bounds, cfg.rho, cfg)
+    if route:
+        spectral, scores = route_windows(Xc, bounds, cfg.rho, cfg)
+    else:
+        spectral, scores = [True] * len(bounds), []
     groups_abs: List[np.ndarray] = []
+    r_effs = []
     for (s, e), m, sp in zip(bounds, budgets, spectral):
         L = e - s
         if sp:
             bits = cfg.bits if cfg.bits > 0 else auto_bits(L, cfg.rho)
-            gs, _ = spectral_groups(Xc[s:e], W, b, R, q1[s:e], cfg.r, bits, m,
-                                    cfg.lanczos_tol)
+            gs, inf = spectral_groups(Xc[s:e], W, b, R, q1[s:e], cfg.r, bits, m,
+                                      cfg.lanczos_tol)
+            r_effs.append(inf["r_eff"])
         else:
             gs = chunk_groups(L, m)
+            r_effs.append(0)
         groups_abs.extend(g + s + pf for g in gs)
     res = _assemble(X, pf, pl, groups_abs, cfg)
     res.info.update({"M_star": M, "budgets": budgets, "spectral": spectral,
-                     "scores": scores})
+                     "scores": scores, "r_eff": r_effs})
     return res
+
+
+def compress_adaptive(X: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray,
+                      q1: np.ndarray, cfg: CompressConfig) -> CompressResult:
+    """Adaptive backend (Sec. 3.6): windows, exact budgets, redundancy score,
+    chunk or per-window Spectral-LSH, concatenation in window order.  Each
+    spectral window uses the slice of q1 at its offset and
+    b_w = cfg.bits or ceil(log2(L_w / rho))."""
+    return _windowed(X, W, b, R, q1, cfg, route=True)
+
+
+def compress_local(X: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray,
+                   q1: np.ndarray, cfg: CompressConfig) -> CompressResult:
+    """Local-LSH backend (Sec. 3.5): Spectral-LSH run independently inside
+    each window of cfg.window tokens (the paper's default window is 16), with
+    the exact per-window budgets of the adaptive backend and no routing; the
+    adaptive backend at rho >= 16 delegates to exactly this (Sec. 3.6)."""
+    return _windowed(X, W, b, R, q1, cfg, route=False)
 
 
 # ---------------------------------------------------------------------------

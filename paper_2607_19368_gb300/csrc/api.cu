@@ -578,7 +578,7 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
                            M_target, perm, mstart, mlen, pos, tok2macro, status, s)) != SLS_OK)
     return st;
   return launch_aggregate(X, x_dtype, d, ldx, perm, mstart, mlen, M_target, N, renorm, Xt,
-                          it_start, pt_start, items, counts, part, part_eta, s);
+                          it_start, pt_start, items, counts, part, part_eta, status, s);
 }
 
 int64_t sls_output_count(const sls_config_t* cfg, int64_t N) {
@@ -740,7 +740,7 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   phase_mark(6, 0, s);
   st = launch_aggregate(X, x_dtype, d, ldx, W.perm, W.mstart, W.mlen, B * P.M, B * N,
                         cfg->renorm, Xt, W.it_start, W.pt_start, W.items, W.counts, W.part,
-                        W.part_eta, s);
+                        W.part_eta, W.status, s);
   phase_mark(6, 1, s);
   return st;
 }

@@ -1051,92 +1051,6 @@ constexpr int agg_batch() {
   return NV >= 8 ? 1 : 8 / NV;
 }
 
-// One work item = up to AGG_CH members of one macro-token.  The member rows
-// are gathered in batches of agg_batch<NV>() rows (all loads of a batch issued
-// before any is used); every member's |x|^2 is reduced from the same values,
-// per warp into shared memory, so X is read once.  A macro-token of one item
-// is finalised here; longer ones leave a partial sum for agg_final_kernel.
-template <typename T, int NV>
-__global__ void __launch_bounds__(AGG_T, 2)
-agg_partial_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restrict__ perm,
-                   const int* __restrict__ mstart, const int* __restrict__ mlen,
-                   const int2* __restrict__ items, const int* __restrict__ counts,
-                   const int* __restrict__ pt_start, int renorm, float* __restrict__ Xt,
-                   float* __restrict__ part, float* __restrict__ part_eta) {
-  constexpr int V = VecOf<T>::V;
-  constexpr int MB = agg_batch<NV>();
-  constexpr int NW = AGG_T / 32;
-  __shared__ float sh[NW];
-  __shared__ float shq[NW][AGG_CH];
-  const int nitems = counts[0];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int it = blockIdx.x; it < nitems; it += gridDim.x) {
-    const int2 item = items[it];
-    const int m = item.x, c = item.y;
-    const int len = mlen[m];
-    const int b = c * AGG_CH;
-    const int n = min(len - b, AGG_CH);
-    const int* mem = perm + mstart[m] + b;
-    const int id0 = lane < n ? mem[lane] : 0;
-    const int id1 = lane + 32 < n ? mem[lane + 32] : 0;
-    float acc[NV * V];
-#pragma unroll
-    for (int k = 0; k < NV * V; ++k) acc[k] = 0.f;
-    for (int s0 = 0; s0 < n; s0 += MB) {
-      float v[MB][NV * V];
-#pragma unroll
-      for (int j = 0; j < MB; ++j) {
-        const int s = s0 + j;
-        const int row = __shfl_sync(0xffffffffu, s < 32 ? id0 : id1, s & 31);
-        const T* x = X + (int64_t)row * ldx;
-#pragma unroll
-        for (int q = 0; q < NV; ++q) {
-          const int c0 = (tid + q * AGG_T) * V;
-          if (s < n && c0 < d) {
-            load_vec<T>(x + c0, &v[j][q * V]);
-          } else {
-#pragma unroll
-            for (int k = 0; k < V; ++k) v[j][q * V + k] = 0.f;
-          }
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < MB; ++j) {
-        float sq = 0.f;
-#pragma unroll
-        for (int k = 0; k < NV * V; ++k) {
-          acc[k] += v[j][k];
-          sq = fmaf(v[j][k], v[j][k], sq);
-        }
-        sq = warp_sum_f(sq);
-        if (lane == 0 && s0 + j < n) shq[warp][s0 + j] = sq;
-      }
-    }
-    __syncthreads();
-    // sum of member norms (every warp forms the same total)
-    float eta = 0.f;
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int s = lane + 32 * h;
-      if (s < n) {
-        float t = 0.f;
-#pragma unroll
-        for (int w = 0; w < NW; ++w) t += shq[w][s];
-        eta += sqrtf(t);
-      }
-    }
-    eta = warp_sum_f(eta);
-    const int ps = pt_start[m];
-    if (ps < 0) {
-      agg_finalize<V, NV>(acc, len, eta, renorm, d, Xt + (int64_t)m * d, sh);
-    } else {
-      store_row<V, NV>(acc, 1.0f, d, part + (int64_t)(ps + c) * d);
-      if (tid == 0) part_eta[ps + c] = eta;
-    }
-    __syncthreads();
-  }
-}
-
 template <int V, int NV>
 __global__ void __launch_bounds__(AGG_T)
 agg_final_kernel(int d, const int* __restrict__ mlen, const int* __restrict__ pt_start,
@@ -1153,25 +1067,356 @@ agg_final_kernel(int d, const int* __restrict__ mlen, const int* __restrict__ pt
 #pragma unroll
     for (int k = 0; k < NV * V; ++k) acc[k] = 0.f;
     float eta = 0.f;
-    for (int c = 0; c < nch; ++c) {
-      const float* src = part + (int64_t)(ps + c) * d;
-      eta += part_eta[ps + c];
+    // AF_B partial rows in flight per thread (the chunks are independent)
+    constexpr int AF_B = (NV * V <= 16) ? 4 : 2;
+    for (int cb = 0; cb < nch; cb += AF_B) {
+      float4 buf[AF_B][NV * V / 4];
 #pragma unroll
-      for (int q = 0; q < NV; ++q) {
-        const int c0 = (tid + q * AGG_T) * V;
-        if (c0 < d)
+      for (int j = 0; j < AF_B; ++j) {
+        const float* src = part + (int64_t)(ps + cb + j) * d;
+#pragma unroll
+        for (int q = 0; q < NV; ++q) {
+          const int c0 = (tid + q * AGG_T) * V;
 #pragma unroll
           for (int k = 0; k < V; k += 4) {
-            const float4 f = *reinterpret_cast<const float4*>(src + c0 + k);
-            acc[q * V + k] += f.x;
-            acc[q * V + k + 1] += f.y;
-            acc[q * V + k + 2] += f.z;
-            acc[q * V + k + 3] += f.w;
+            float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (cb + j < nch && c0 < d) f = *reinterpret_cast<const float4*>(src + c0 + k);
+            buf[j][(q * V + k) / 4] = f;
           }
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < AF_B; ++j) {
+        if (cb + j < nch) eta += part_eta[ps + cb + j];
+#pragma unroll
+        for (int e = 0; e < NV * V / 4; ++e) {
+          acc[4 * e] += buf[j][e].x;
+          acc[4 * e + 1] += buf[j][e].y;
+          acc[4 * e + 2] += buf[j][e].z;
+          acc[4 * e + 3] += buf[j][e].w;
+        }
       }
     }
     agg_finalize<V, NV>(acc, len, eta, renorm, d, Xt + m * d, sh);
     __syncthreads();
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Member pass with a shared-memory row ring.  Warp 0 is the producer: it walks
+// this CTA's work items (items blockIdx.x, blockIdx.x + G, ...), loads each
+// item's descriptor and member ids one item ahead, and streams every member
+// row into an S-stage ring with one bulk async copy per row (mbarrier
+// complete_tx); the item descriptor travels with the item's first row.  Warps
+// 1..8 consume the rows in the same order: each consumer thread owns the
+// column groups c0 = (ct + q * 256) * V, sums them and the row's |x|^2, and
+// releases the stage.  At the end of an item the consumers meet at a named
+// barrier (which also ORs their failure flags), form the sum of member norms
+// and finalise the macro-token (Eq. macro_embed) or store a partial sum.
+// Every wait is bounded; a wait that gives up records SLS_ERR_TIMEOUT, the
+// other roles stop at their next check, and in-flight copies are drained.
+// ---------------------------------------------------------------------------
+
+constexpr int AGR_CW = 8;                    // consumer warps
+constexpr int AGR_CT = AGR_CW * 32;          // consumer threads
+constexpr int AGR_THREADS = AGR_CT + 32;     // + producer warp
+constexpr int AGR_MAX_STAGES = 16;
+constexpr int AGR_BAR = 1;                   // named barrier of the consumers
+
+struct AggDesc {
+  int m, c, n, len, ps, pad0, pad1, pad2;
+};
+
+SLS_DEV bool named_sync_or(unsigned id, unsigned nthreads, bool pred) {
+  unsigned r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
+      " bar.red.or.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((unsigned)pred), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
+template <typename T>
+SLS_DEV void load_vec_smem(const T* p, float* out);
+template <>
+SLS_DEV void load_vec_smem<float>(const float* p, float* out) {
+  const float4 v = *reinterpret_cast<const float4*>(p);
+  out[0] = v.x;
+  out[1] = v.y;
+  out[2] = v.z;
+  out[3] = v.w;
+}
+template <>
+SLS_DEV void load_vec_smem<uint16_t>(const uint16_t* p, float* out) {
+  const uint4 v = *reinterpret_cast<const uint4*>(p);
+  const unsigned w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    out[2 * k] = __uint_as_float(w[k] << 16);
+    out[2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+  }
+}
+
+// Bounded wait that also returns early once another role has aborted.
+SLS_DEV bool agr_wait(uint64_t* bar, unsigned parity, volatile int* abort_flag) {
+  for (unsigned it = 0; it < (1u << 25); ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255) == 255 && *abort_flag) return false;
+    if (it > 64) __nanosleep(32);
+  }
+  return false;
+}
+
+// Descriptor of the local item kidx of this CTA (global item blockIdx.x +
+// kidx * gridDim.x), or an empty one past the end.
+struct LaneDesc {
+  int m, c, n, len, ps, off;
+};
+
+SLS_DEV LaneDesc agr_lane_desc(const int2* __restrict__ items, const int* __restrict__ mlen,
+                               const int* __restrict__ mstart, const int* __restrict__ pt_start,
+                               int nitems, int kidx) {
+  LaneDesc L{0, 0, 0, 0, -1, 0};
+  const int64_t it = (int64_t)blockIdx.x + (int64_t)kidx * gridDim.x;
+  if (it < nitems) {
+    const int2 item = items[it];
+    L.m = item.x;
+    L.c = item.y;
+    L.len = mlen[L.m];
+    L.n = min(L.len - L.c * AGG_CH, AGG_CH);
+    L.ps = pt_start[L.m];
+    L.off = mstart[L.m] + L.c * AGG_CH;
+  }
+  return L;
+}
+
+// Member row f (flattened over the 32 items of a batch whose inclusive row
+// prefix is `pre`): its item j, index s inside the item and token row id.
+SLS_DEV void agr_fetch_row(const int* __restrict__ perm, int pre, int nrows, int off, int f0,
+                           int lane, int& rid, int& rj, int& rs) {
+  const int f = f0 + lane;
+  int j = 0;
+#pragma unroll
+  for (int step = 16; step >= 1; step >>= 1) {
+    const int pv = __shfl_sync(0xffffffffu, pre, j + step - 1);
+    if (pv <= f) j += step;
+  }
+  j = min(j, 31);
+  const int base = __shfl_sync(0xffffffffu, pre, j > 0 ? j - 1 : 0);
+  const int off_j = __shfl_sync(0xffffffffu, off, j);
+  rs = f - (j > 0 ? base : 0);
+  rj = j;
+  rid = (f < nrows) ? perm[off_j + rs] : 0;
+}
+
+template <typename T, int NV>
+__global__ void __launch_bounds__(AGR_THREADS, 2)
+agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restrict__ perm,
+                const int* __restrict__ mstart, const int* __restrict__ mlen,
+                const int2* __restrict__ items, const int* __restrict__ counts,
+                const int* __restrict__ pt_start, int renorm, float* __restrict__ Xt,
+                float* __restrict__ part, float* __restrict__ part_eta, int S, int stage_bytes,
+                int* status) {
+  constexpr int V = VecOf<T>::V;
+  extern __shared__ __align__(128) unsigned char agr_smem[];
+  __shared__ uint64_t fullb[AGR_MAX_STAGES], emptyb[AGR_MAX_STAGES];
+  __shared__ AggDesc dring[AGR_MAX_STAGES + 2];
+  __shared__ float shq[2][AGR_CW][AGG_CH];
+  __shared__ float sh[AGR_CW];
+  __shared__ volatile int s_abort;
+  const int DQ = S + 2;
+  const int nitems = counts[0];
+  const int G = gridDim.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const unsigned row_bytes = (unsigned)d * sizeof(T);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&fullb[s], 1);
+      mbar_init(&emptyb[s], AGR_CW);
+    }
+    mbar_fence_init();
+    s_abort = 0;
+  }
+  __syncthreads();
+
+  if (warp == 0) {
+    // ------------------------------ producer ------------------------------
+    // Lane j holds the descriptor of local item kb + j; the member ids of the
+    // batch are fetched 32 rows at a time, one chunk ahead of the copies.
+    const uint64_t pol = l2_policy_evict_first();
+    unsigned issued = 0;
+    bool ok = true;
+    int kb = 0;
+    LaneDesc cd = agr_lane_desc(items, mlen, mstart, pt_start, nitems, kb + lane);
+    while (ok) {
+      int pre = cd.n;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, pre, o);
+        if (lane >= o) pre += t;
+      }
+      const int nrows = __shfl_sync(0xffffffffu, pre, 31);
+      if (nrows == 0) break;
+      const LaneDesc nd = agr_lane_desc(items, mlen, mstart, pt_start, nitems, kb + 32 + lane);
+      int rid, rj, rs;
+      agr_fetch_row(perm, pre, nrows, cd.off, 0, lane, rid, rj, rs);
+      for (int f0 = 0; f0 < nrows && ok; f0 += 32) {
+        int nrid = 0, nrj = 0, nrs = 0;
+        if (f0 + 32 < nrows) agr_fetch_row(perm, pre, nrows, cd.off, f0 + 32, lane, nrid, nrj, nrs);
+        const int cnt = min(32, nrows - f0);
+        for (int l = 0; l < cnt; ++l) {
+          const int row = __shfl_sync(0xffffffffu, rid, l);
+          const int j = __shfl_sync(0xffffffffu, rj, l);
+          const int s = __shfl_sync(0xffffffffu, rs, l);
+          AggDesc D;
+          D.m = __shfl_sync(0xffffffffu, cd.m, j);
+          D.c = __shfl_sync(0xffffffffu, cd.c, j);
+          D.n = __shfl_sync(0xffffffffu, cd.n, j);
+          D.len = __shfl_sync(0xffffffffu, cd.len, j);
+          D.ps = __shfl_sync(0xffffffffu, cd.ps, j);
+          D.pad0 = D.pad1 = D.pad2 = 0;
+          if (lane == 0) {
+            const int st = (int)(issued % (unsigned)S);
+            const unsigned par = (issued / (unsigned)S) & 1u;
+            if (!agr_wait(&emptyb[st], par ^ 1u, &s_abort)) {
+              ok = false;
+              s_abort = 1;
+              atomicExch(status, SLS_ERR_TIMEOUT);
+            } else {
+              if (s == 0) dring[(kb + j) % DQ] = D;
+              unsigned char* dst = agr_smem + (size_t)st * stage_bytes;
+              mbar_expect_tx(&fullb[st], row_bytes);
+              bulk_g2s(dst, X + (int64_t)row * ldx, row_bytes, &fullb[st], pol);
+            }
+          }
+          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+          if (!ok) break;
+          ++issued;
+        }
+        rid = nrid;
+        rj = nrj;
+        rs = nrs;
+      }
+      kb += 32;
+      cd = nd;
+    }
+    // every issued copy has landed before the CTA may exit
+    if (lane == 0) {
+      const unsigned first = issued > (unsigned)S ? issued - (unsigned)S : 0u;
+      for (unsigned c = first; c < issued; ++c) {
+        for (unsigned w = 0; w < (1u << 25); ++w) {
+          if (mbar_try_wait(&fullb[c % (unsigned)S], (c / (unsigned)S) & 1u)) break;
+          __nanosleep(32);
+        }
+      }
+    }
+  } else {
+    // ------------------------------ consumers -----------------------------
+    const int cw = warp - 1, ct = threadIdx.x - 32;
+    unsigned consumed = 0;
+    bool ok = true;
+    int k = 0;
+    for (int it = blockIdx.x; it < nitems; it += G, ++k) {
+      float acc[NV * V];
+#pragma unroll
+      for (int e = 0; e < NV * V; ++e) acc[e] = 0.f;
+      AggDesc D{};
+      D.n = 1;
+      float* q = &shq[k & 1][cw][0];
+      for (int s = 0; s < D.n && ok; ++s) {
+        const int st = (int)(consumed % (unsigned)S);
+        const unsigned par = (consumed / (unsigned)S) & 1u;
+        if (!agr_wait(&fullb[st], par, &s_abort)) {
+          ok = false;
+          if (lane == 0) {
+            s_abort = 1;
+            atomicExch(status, SLS_ERR_TIMEOUT);
+          }
+          break;
+        }
+        if (s == 0) D = dring[k % DQ];
+        const T* rowp = reinterpret_cast<const T*>(agr_smem + (size_t)st * stage_bytes);
+        float sq = 0.f;
+#pragma unroll
+        for (int qv = 0; qv < NV; ++qv) {
+          const int c0 = (ct + qv * AGR_CT) * V;
+          if (c0 < d) {
+            float v[V];
+            load_vec_smem<T>(rowp + c0, v);
+#pragma unroll
+            for (int e = 0; e < V; ++e) {
+              acc[qv * V + e] += v[e];
+              sq = fmaf(v[e], v[e], sq);
+            }
+          }
+        }
+        sq = warp_sum_f(sq);
+        __syncwarp();
+        if (lane == 0) {
+          q[s] = sq;
+          mbar_arrive(&emptyb[st]);
+        }
+        ++consumed;
+      }
+      if (named_sync_or(AGR_BAR, AGR_CT, !ok)) break;
+      // sum of member norms (every warp forms the same total)
+      float eta = 0.f;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int s = lane + 32 * h;
+        if (s < D.n) {
+          float t = 0.f;
+#pragma unroll
+          for (int w = 0; w < AGR_CW; ++w) t += shq[k & 1][w][s];
+          eta += sqrtf(t);
+        }
+      }
+      eta = warp_sum_f(eta);
+      float scale = 1.0f;
+      float* dst;
+      if (D.ps < 0) {
+        dst = Xt + (int64_t)D.m * d;
+        if (D.len > 1) {
+          const float inv = 1.0f / (float)D.len;
+          float sq = 0.f;
+#pragma unroll
+          for (int qv = 0; qv < NV; ++qv) {
+            const int c0 = (ct + qv * AGR_CT) * V;
+            if (c0 < d)
+#pragma unroll
+              for (int e = 0; e < V; ++e) {
+                acc[qv * V + e] *= inv;
+                sq = fmaf(acc[qv * V + e], acc[qv * V + e], sq);
+              }
+          }
+          if (renorm) {
+            sq = warp_sum_f(sq);
+            if (lane == 0) sh[cw] = sq;
+            named_sync(AGR_BAR, AGR_CT);
+            float tot = 0.f;
+#pragma unroll
+            for (int w = 0; w < AGR_CW; ++w) tot += sh[w];
+            named_sync(AGR_BAR, AGR_CT);
+            const float nrm = sqrtf(tot);
+            if (nrm >= 1e-30f) scale = (eta * inv) / nrm;
+          }
+        }
+      } else {
+        dst = part + (int64_t)(D.ps + D.c) * d;
+        if (ct == 0) part_eta[D.ps + D.c] = eta;
+      }
+#pragma unroll
+      for (int qv = 0; qv < NV; ++qv) {
+        const int c0 = (ct + qv * AGR_CT) * V;
+        if (c0 < d)
+#pragma unroll
+          for (int e = 0; e < V; e += 4)
+            store_vec4(dst + c0 + e, acc[qv * V + e] * scale, acc[qv * V + e + 1] * scale,
+                       acc[qv * V + e + 2] * scale, acc[qv * V + e + 3] * scale);
+      }
+    }
   }
 }
 
@@ -1361,61 +1606,76 @@ size_t agg_part_capacity(int64_t Ntot) { return (size_t)(2 * (Ntot / AGG_CH) + 2
 
 namespace {
 template <typename T, int NV>
-void launch_agg_t(const void* X, int d, int64_t ldx, const int* perm, const int* mstart,
-                  const int* mlen, int64_t Mtot, int64_t blocks, int64_t fblocks, int renorm,
-                  float* Xt, const int* pt_start, const int2* items, const int* counts,
-                  float* part, float* part_eta, cudaStream_t stream) {
+int launch_agg_t(const void* X, int d, int64_t ldx, const int* perm, const int* mstart,
+                 const int* mlen, int64_t Mtot, int64_t fblocks, int renorm, float* Xt,
+                 const int* pt_start, const int2* items, const int* counts, float* part,
+                 float* part_eta, int* status, cudaStream_t stream) {
   constexpr int V = VecOf<T>::V;
-  agg_partial_kernel<T, NV><<<(unsigned)blocks, AGG_T, 0, stream>>>(
+  const int stage = (int)(((size_t)d * sizeof(T) + 127) & ~(size_t)127);
+  // two CTAs per SM when each still gets at least 6 ring stages in ~100 KB
+  int per_sm = 2;
+  int S = (100 * 1024) / stage;
+  if (S < 6) {
+    per_sm = 1;
+    S = (200 * 1024) / stage;
+  }
+  if (S > AGR_MAX_STAGES) S = AGR_MAX_STAGES;
+  if (S < 2) return SLS_ERR_UNSUPPORTED;
+  const size_t smem = (size_t)S * stage;
+  SLS_CUDA_TRY(cudaFuncSetAttribute(agg_ring_kernel<T, NV>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  int occ = 0;
+  SLS_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, agg_ring_kernel<T, NV>,
+                                                             AGR_THREADS, smem));
+  if (occ < 1) return SLS_ERR_UNSUPPORTED;
+  if (occ < per_sm) per_sm = occ;
+  int dev = 0, sms = 0;
+  SLS_CUDA_TRY(cudaGetDevice(&dev));
+  SLS_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  const int grid = sms * per_sm;
+  agg_ring_kernel<T, NV><<<grid, AGR_THREADS, smem, stream>>>(
       (const T*)X, d, ldx, perm, mstart, mlen, items, counts, pt_start, renorm, Xt, part,
-      part_eta);
-  count_launch(1);
+      part_eta, S, stage, status);
+  SLS_LAUNCH_CHECK();
   agg_final_kernel<V, NV><<<(unsigned)fblocks, AGG_T, 0, stream>>>(d, mlen, pt_start, Mtot,
                                                                    renorm, part, part_eta, Xt);
-  count_launch(1);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
 }
 
 template <typename T>
 int launch_agg_dtype(const void* X, int d, int64_t ldx, const int* perm, const int* mstart,
-                     const int* mlen, int64_t Mtot, int64_t blocks, int64_t fblocks, int renorm,
-                     float* Xt, const int* pt_start, const int2* items, const int* counts,
-                     float* part, float* part_eta, cudaStream_t stream) {
+                     const int* mlen, int64_t Mtot, int64_t fblocks, int renorm, float* Xt,
+                     const int* pt_start, const int2* items, const int* counts, float* part,
+                     float* part_eta, int* status, cudaStream_t stream) {
   constexpr int V = VecOf<T>::V;
-  const int nv = (d / V + AGG_T - 1) / AGG_T;
-#define SLS_AGG_NV(N)                                                                      \
-  launch_agg_t<T, N>(X, d, ldx, perm, mstart, mlen, Mtot, blocks, fblocks, renorm, Xt,    \
-                     pt_start, items, counts, part, part_eta, stream)
-  if (nv <= 1)
-    SLS_AGG_NV(1);
-  else if (nv <= 2)
-    SLS_AGG_NV(2);
-  else if (nv <= 4)
-    SLS_AGG_NV(4);
-  else if (nv <= 8)
-    SLS_AGG_NV(8);
-  else
-    return SLS_ERR_UNSUPPORTED;
+  const int nv = (d / V + AGR_CT - 1) / AGR_CT;
+#define SLS_AGG_NV(N)                                                                       \
+  return launch_agg_t<T, N>(X, d, ldx, perm, mstart, mlen, Mtot, fblocks, renorm, Xt,      \
+                            pt_start, items, counts, part, part_eta, status, stream)
+  if (nv <= 1) SLS_AGG_NV(1);
+  if (nv <= 2) SLS_AGG_NV(2);
+  if (nv <= 4) SLS_AGG_NV(4);
+  if (nv <= 8) SLS_AGG_NV(8);
 #undef SLS_AGG_NV
-  SLS_CUDA_TRY(cudaGetLastError());
-  return SLS_OK;
+  return SLS_ERR_UNSUPPORTED;
 }
 }  // namespace
 
 int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* perm,
                      const int* mstart, const int* mlen, int64_t Mtot, int64_t Ntot, int renorm,
                      float* Xt, int* it_start, int* pt_start, int2* items, int* counts,
-                     float* part, float* part_eta, cudaStream_t stream) {
+                     float* part, float* part_eta, int* status, cudaStream_t stream) {
   if (Mtot == 0) return SLS_OK;
+  (void)Ntot;
   agg_items_kernel<<<1, SEG_T, 0, stream>>>(mlen, Mtot, it_start, pt_start, items, counts);
   SLS_LAUNCH_CHECK();
-  int64_t blocks = (int64_t)agg_item_capacity(Mtot, Ntot);
-  if (blocks > 16384) blocks = 16384;
   const int64_t fblocks = Mtot < 4096 ? Mtot : 4096;
   if (x_dtype == SLS_F32)
-    return launch_agg_dtype<float>(X, d, ldx, perm, mstart, mlen, Mtot, blocks, fblocks, renorm,
-                                   Xt, pt_start, items, counts, part, part_eta, stream);
-  return launch_agg_dtype<uint16_t>(X, d, ldx, perm, mstart, mlen, Mtot, blocks, fblocks, renorm,
-                                    Xt, pt_start, items, counts, part, part_eta, stream);
+    return launch_agg_dtype<float>(X, d, ldx, perm, mstart, mlen, Mtot, fblocks, renorm, Xt,
+                                   pt_start, items, counts, part, part_eta, status, stream);
+  return launch_agg_dtype<uint16_t>(X, d, ldx, perm, mstart, mlen, Mtot, fblocks, renorm, Xt,
+                                    pt_start, items, counts, part, part_eta, status, stream);
 }
 
 namespace {

@@ -87,7 +87,7 @@ size_t agg_part_capacity(int64_t Ntot);
 int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* perm,
                      const int* mstart, const int* mlen, int64_t Mtot, int64_t Ntot, int renorm,
                      float* Xt, int* it_start, int* pt_start, int2* items, int* counts,
-                     float* part, float* part_eta, cudaStream_t stream);
+                     float* part, float* part_eta, int* status, cudaStream_t stream);
 int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,
                         int nprob, float* score, cudaStream_t stream);
 }  // namespace sls

@@ -522,3 +522,54 @@ def test_route_rules_and_adaptive_invariants():
     # tiny last window is routed to chunk
     spf, _ = O.route_windows(X[:100], [(0, 96), (96, 100)], 4.0, O.CompressConfig())
     assert spf[1] is False
+
+
+def test_local_backend_reductions():
+    """Local LSH (Sec. 3.5) against what fixes it: at rho >= 16 the adaptive
+    backend is local LSH (Sec. 3.6); one window over the whole region is the
+    global backend; a budget of one macro-token per window makes every window
+    one group, i.e. the chunk backend with k = window."""
+    w = WL.scaled(WL.WORKLOADS["tiny"], N=300)
+    p = WL.make_prompt(w)
+    prm = WL.params_for(w)
+    X = p.x_f64()
+    W64, b, R, q1 = prm.w_f64()[:64], prm.b[:64], prm.R, prm.q1
+
+    def same(a, c):
+        return (np.array_equal(a.tok2macro, c.tok2macro) and np.array_equal(a.pos, c.pos)
+                and np.array_equal(a.Xt, c.Xt))
+
+    cfg = O.CompressConfig(rho=16.0, D=64, r=8, window=40, preserve_last=12)
+    assert same(O.compress_local(X, W64, b, R, q1, cfg),
+                O.compress_adaptive(X, W64, b, R, q1, cfg))
+    cfg = O.CompressConfig(rho=4.0, D=64, r=8, window=1000, preserve_last=12)
+    assert same(O.compress_local(X, W64, b, R, q1, cfg),
+                O.compress_global(X, W64, b, R, q1, cfg))
+    cfg = O.CompressConfig(rho=16.0, D=64, r=8, window=16, preserve_last=12)
+    res = O.compress_local(X, W64, b, R, q1, cfg)
+    assert same(res, O.compress_chunk(X, cfg))
+    assert all(res.info["spectral"])
+
+
+def test_local_backend_w16_invariants():
+    """w = 16 (the paper's default): every window yields exactly its budget
+    of macro-tokens, none crosses a window, positions are causal."""
+    w = WL.scaled(WL.WORKLOADS["tiny"], N=500)
+    p = WL.make_prompt(w)
+    prm = WL.params_for(w)
+    X = p.x_f64()
+    for rho in (2.0, 4.0, 8.0):
+        cfg = O.CompressConfig(rho=rho, D=64, r=16, window=16, preserve_last=12)
+        res = O.compress_local(X, prm.w_f64()[:64], prm.b[:64], prm.R, prm.q1, cfg)
+        Nc = 488
+        _check_result(res, 500, O.target_count(Nc, rho) + 12, 0, 12)
+        bounds = O.window_bounds(Nc, 16)
+        budgets = res.info["budgets"]
+        assert sum(budgets) == O.target_count(Nc, rho)
+        t = res.tok2macro[:Nc]
+        for (s_, e_), m in zip(bounds, budgets):
+            assert len(np.unique(t[s_:e_])) == m
+        for m in range(res.Xt.shape[0] - 12):
+            mem = np.nonzero(res.tok2macro == m)[0]
+            assert mem.min() // 16 == mem.max() // 16
+        assert all(1 <= k <= 16 for k in res.info["r_eff"])
