@@ -7,13 +7,15 @@ D = 2048 RFF features, r = 64 Lanczos steps, b = 16 SimHash bits, rho = 16,
 last 12 tokens preserved, global backend.  Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
-                  [--workload qwen7b|qwen14b|mistral7b|adaptive] [--rho R]
+                  [--workload qwen7b|qwen14b|mistral7b|adaptive|local] [--rho R]
 
 --workload qwen14b (N = 131072, d = 5120) and mistral7b (N = 8192, d = 4096)
 time the other single-prompt shapes; --workload adaptive times the windowed
 batch: 64 prompts of N = 16384, d = 4096 bf16 (duplication 0.6 p / 63 for
 prompt p), windows of 2048 routed to the chunk or the spectral chain, D = 1024,
-r = 32, bits from the window budget, rho from --rho (default 8).
+r = 32, bits from the window budget, rho from --rho (default 8); --workload
+local times local LSH (Spectral-LSH inside every window of 16 tokens) on the
+Qwen2.5-7B-shaped prompt at the paper's defaults D = 256, r = 16, rho = 8.
 
 The prompt (235 MB of embeddings) and the feature matrix (268 MB) are both
 larger than the 129 MB L2, so no extra flush runs between steps.  With
@@ -47,7 +49,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--workload", default="qwen7b",
-                    choices=["qwen7b", "qwen14b", "mistral7b", "adaptive"])
+                    choices=["qwen7b", "qwen14b", "mistral7b", "adaptive", "local"])
     ap.add_argument("--rho", type=float, default=None,
                     help="compression ratio (default: the workload's)")
     ap.add_argument("--cpu-sample", type=int, default=4096,
@@ -66,7 +68,14 @@ def workload(name):
 
 
 def config_dict(w, rho, extra=None):
-    if w.batch > 1:
+    if w.backend == "local":
+        d = {"workload": f"{w.name}: qwen7b-shaped prompt N={w.N} d={w.d} bf16, local LSH "
+                         f"with windows of {w.window}, D={w.D} r={w.r} b=auto rho={rho:g} "
+                         f"preserve_last={w.preserve_last}",
+             "window": w.window,
+             "l2": (f"inputs larger than L2 (X {w.N * w.d * 2 / 1e6:.0f} MB per step), "
+                    f"no flush")}
+    elif w.batch > 1:
         d = {"workload": f"{w.name}: {w.batch} prompts of N={w.N} d={w.d} bf16, windows of "
                          f"{w.window}, D={w.D} r={w.r} b=auto rho={rho:g} "
                          f"preserve_last={w.preserve_last}, adaptive backend",
@@ -149,8 +158,12 @@ def lanczos_algorithmic_bytes(n_tokens, D, r):
     return n_tokens * (8 * r * D + 16 * r * (r + 1))
 
 
+def windowed(w):
+    return w.backend in ("adaptive", "local")
+
+
 def window_lengths(w):
-    """Lengths of the adaptive windows over one prompt's compressible region
+    """Lengths of the windows over one prompt's compressible region
     (consecutive windows, the last one shorter)."""
     nc = w.N - w.preserve_first - w.preserve_last
     return [min(w.window, nc - s) for s in range(0, nc, w.window)]
@@ -160,17 +173,19 @@ def oracle_config(w, rho):
     import oracle as O
     return O.CompressConfig(rho=rho, D=w.D, r=w.r, bits=w.bits,
                             preserve_first=w.preserve_first, preserve_last=w.preserve_last,
-                            window=w.window if w.batch > 1 else 2048)
+                            window=w.window if windowed(w) else 2048)
 
 
 def cpu_oracle_step(w, rho, X64, prm, n):
     """One oracle compression of the first n tokens of a prompt (global
-    backend, or the adaptive backend for the windowed batch)."""
+    backend, or the windowed backend of the workload)."""
     import oracle as O
     cfg = oracle_config(w, rho)
     t = time.perf_counter()
-    if w.batch > 1:
+    if w.backend == "adaptive":
         O.compress_adaptive(X64[:n], prm.w_f64(), prm.b, prm.R, prm.q1[:n], cfg)
+    elif w.backend == "local":
+        O.compress_local(X64[:n], prm.w_f64(), prm.b, prm.R, prm.q1[:n], cfg)
     else:
         O.compress_global(X64[:n], prm.w_f64(), prm.b, prm.R, prm.q1, cfg)
     return time.perf_counter() - t
@@ -193,7 +208,7 @@ def cpu_baseline(w, rho, X64, prm, n, pidx, budget_s=10.0):
     while reps == 0 or tot < budget_s:
         tot += cpu_oracle_step(w, rho, X64, prm, n)
         reps += 1
-    kind = "compress_adaptive" if w.batch > 1 else "compress_global"
+    kind = "compress_" + w.backend
     return {"value": n * reps / tot, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
             "sample": f"oracle {kind} (numpy float64, BLAS threads = all cores) on the first "
                       f"{n} tokens of prompt {pidx} of the {w.name} workload, D={w.D} r={w.r} "
@@ -262,7 +277,8 @@ def run_native(args, rank, world):
     torch.cuda.set_device(dev)
     w = workload(args.workload)
     rho = args.rho or w.rho
-    adaptive = w.batch > 1
+    adaptive = w.backend == "adaptive"
+    local = w.backend == "local"
     X = device_inputs(w, rank, dev)
     prm = WL.params_for(w)
     Wt = torch.from_numpy(prm.W.view(np.int16)).view(torch.bfloat16).to(dev)
@@ -271,6 +287,10 @@ def run_native(args, rank, world):
     qt = torch.from_numpy(prm.q1).to(dev)
     if adaptive:
         cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=w.D, r=w.r, bits=w.bits,
+                              window=w.window, preserve_first=w.preserve_first,
+                              preserve_last=w.preserve_last)
+    elif local:
+        cfg = sls.Config.make(backend=sls.BACKEND_LOCAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
                               window=w.window, preserve_first=w.preserve_first,
                               preserve_last=w.preserve_last)
     else:
@@ -294,7 +314,7 @@ def run_native(args, rank, world):
     if sls.workspace_status(ws) != 0:
         raise RuntimeError("device wait timed out during warm-up")
     # tokens that run through the spectral chain (Lanczos)
-    if adaptive:
+    if adaptive or local:
         lens = window_lengths(w)
         route = res[4].cpu().numpy()[:B * len(lens)].reshape(B, len(lens))
         lz_tokens = int(sum(int(route[i, k]) * lens[k]
@@ -361,7 +381,7 @@ def run_native(args, rank, world):
             with open(tr) as f:
                 t = json.load(f)
             if (t.get("workload") == w.name and t.get("kernel_rev") == LANCZOS_KERNEL_REV
-                    and not adaptive):
+                    and not windowed(w)):
                 roof["traffic"] = t["dram_bytes_per_launch"]
         except Exception:
             pass
@@ -407,7 +427,7 @@ def run_native(args, rank, world):
         cpu = cpu_baseline(w, rho, p.x_f64(), prm, args.cpu_sample, pidx)
     extra = {"parallelism": f"replicas x{world}",
              "inputs": "bf16 embeddings and Omega; float32 Phi; double-float Lanczos vectors"}
-    if adaptive:
+    if windowed(w):
         extra.update({"spectral_windows": n_spec, "spectral_tokens": lz_tokens})
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,

@@ -66,6 +66,7 @@ extern "C" {
 #define SLS_BACKEND_GLOBAL 0    /* Spectral-LSH over the whole compressible region */
 #define SLS_BACKEND_ADAPTIVE 1  /* per-window router: chunk or Spectral-LSH         */
 #define SLS_BACKEND_CHUNK 2     /* consecutive groups of max(1, round(rho)) tokens  */
+#define SLS_BACKEND_LOCAL 3     /* Spectral-LSH inside every window (no routing)    */
 
 /* Limits of this implementation. */
 #define SLS_MAX_R 128      /* Krylov rank r                 */
@@ -88,7 +89,7 @@ typedef struct sls_config {
   int pos_mode;         /* SLS_MODE_*                                          */
   int renorm;           /* 1: rescale each mean to its mean member norm        */
   double lanczos_tol;   /* break when beta_j <= tol * max_i(|alpha_i|+beta_i)  */
-  int window;           /* adaptive backend window length                      */
+  int window;           /* adaptive / local backend window length              */
   double tau;           /* fixed redundancy threshold (used if !tau_schedule)  */
   int tau_schedule;     /* 1: tau(rho) = clamp(0.75 - 0.05 log2 rho, .55, .70)  */
 } sls_config_t;
@@ -234,9 +235,14 @@ size_t sls_compress_workspace_size(const sls_config_t* cfg, int64_t B,
  *   Xt: B x M x d floats; pos: B x M int32; tok2macro: B x N int32,
  *   with M = sls_output_count(cfg, N).
  *   r_eff (may be NULL): device int32 per prompt (global backend) or per
- *   window (adaptive backend), the Lanczos steps kept (0 for chunk windows).
+ *   window (adaptive and local backends), the Lanczos steps kept (0 for chunk
+ *   windows).
  *   route (may be NULL): device int32 per window, 1 = spectral, 0 = chunk
- *   (adaptive backend).
+ *   (adaptive backend; all 1 for the local backend).
+ * The windowed backends (adaptive, local) cut the compressible region into
+ * windows of cfg->window tokens (the last one shorter) and give every window
+ * an exact budget summing to ceil(N_c / rho) (App. B.8); INVALID_ARG if that
+ * leaves a window without a macro-token (ceil(N_c / rho) < window count).
  * Preserved first/last tokens become singleton macro-tokens at their own
  * positions; rho <= 1 (or nothing compressible) returns the identity: Xt = X,
  * pos = 0..N-1, tok2macro = 0..N-1 (Sec. 5.6, App. B.6).

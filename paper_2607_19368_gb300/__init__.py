@@ -20,7 +20,7 @@ import torch
 __all__ = [
     "SLS_OK", "SLS_F32", "SLS_BF16", "POS_MAX", "POS_MEDIAN", "POS_MEAN",
     "MODE_REPRESENTATIVE", "MODE_COMPACT", "BACKEND_GLOBAL", "BACKEND_ADAPTIVE",
-    "BACKEND_CHUNK", "Config", "SLSError", "lib", "lib_path", "feature_map",
+    "BACKEND_CHUNK", "BACKEND_LOCAL", "Config", "SLSError", "lib", "lib_path", "feature_map",
     "feature_map_batched",
     "lanczos_topr", "simhash", "aggregate", "compress", "output_count",
     "compress_workspace_size", "workspace_status", "EXPORTED", "PHASES",
@@ -31,7 +31,7 @@ SLS_OK = 0
 SLS_F32, SLS_BF16 = 0, 1
 POS_MAX, POS_MEDIAN, POS_MEAN = 0, 1, 2
 MODE_REPRESENTATIVE, MODE_COMPACT = 0, 1
-BACKEND_GLOBAL, BACKEND_ADAPTIVE, BACKEND_CHUNK = 0, 1, 2
+BACKEND_GLOBAL, BACKEND_ADAPTIVE, BACKEND_CHUNK, BACKEND_LOCAL = 0, 1, 2, 3
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 

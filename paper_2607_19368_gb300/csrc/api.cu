@@ -392,7 +392,7 @@ bool ptr_ok(const void* p) { return p != nullptr && ((uintptr_t)p & 15u) == 0; }
 
 int validate_config(const sls_config_t* c) {
   if (!c) return SLS_ERR_INVALID_ARG;
-  if (c->backend < 0 || c->backend > 2) return SLS_ERR_INVALID_ARG;
+  if (c->backend < 0 || c->backend > 3) return SLS_ERR_INVALID_ARG;
   if (!(c->rho == c->rho)) return SLS_ERR_INVALID_ARG;
   if (c->rho > 1.0 && c->backend != SLS_BACKEND_CHUNK) {
     if (c->D < 4 || c->D > SLS_MAX_D || (c->D & 3)) return SLS_ERR_INVALID_ARG;
@@ -510,8 +510,13 @@ int sls_lanczos_topr(const float* Phi, int64_t N, int D, int r, const double* q1
   bt.S = S;
   bt.r_eff = r_eff;
   bt.nmax = N;
-  if ((st = launch_lanczos(bt, lz, lzb, status, groups, g, s)) != SLS_OK) return st;
-  if ((st = launch_tridiag_eigen(bt, s)) != SLS_OK) return st;
+  const bool small = lanczos_window_fits(N, D, r);
+  if (small) {
+    if ((st = launch_lanczos_window(bt, s)) != SLS_OK) return st;
+  } else if ((st = launch_lanczos(bt, lz, lzb, status, groups, g, s)) != SLS_OK) {
+    return st;
+  }
+  if ((st = launch_tridiag_eigen(bt, s, small)) != SLS_OK) return st;
   if ((st = launch_ritz_vectors(bt, U, s)) != SLS_OK) return st;
   if (alpha) SLS_CUDA_TRY(cudaMemcpyAsync(alpha, al, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
   if (beta) SLS_CUDA_TRY(cudaMemcpyAsync(beta, be, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
@@ -704,12 +709,17 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
     bt.S = W.S;
     bt.r_eff = W.r_eff;
     bt.nmax = P.nmax;
-    if ((st = launch_lanczos(bt, W.lz_scratch, W.lz_bytes, W.status, P.lz_groups, P.lz_g, s)) !=
-        SLS_OK)
+    // windows of at most 32 tokens: one warp per window (values of T included)
+    const bool small = lanczos_window_fits(P.nmax, cfg->D, cfg->r);
+    if (small) {
+      if ((st = launch_lanczos_window(bt, s)) != SLS_OK) return st;
+    } else if ((st = launch_lanczos(bt, W.lz_scratch, W.lz_bytes, W.status, P.lz_groups,
+                                    P.lz_g, s)) != SLS_OK) {
       return st;
+    }
     phase_mark(2, 1, s);
     phase_mark(3, 0, s);
-    if ((st = launch_tridiag_eigen(bt, s)) != SLS_OK) return st;
+    if ((st = launch_tridiag_eigen(bt, s, small)) != SLS_OK) return st;
     if ((st = launch_ritz_vectors(bt, W.U, s)) != SLS_OK) return st;
     phase_mark(3, 1, s);
     phase_mark(4, 0, s);

@@ -59,6 +59,9 @@ SLS_DEV dfloat df_from_double(double x) {
 
 SLS_DEV double df_to_double(dfloat a) { return (double)a.hi + (double)a.lo; }
 
+SLS_DEV float2 f2(dfloat a) { return make_float2(a.hi, a.lo); }
+SLS_DEV dfloat dfv(float2 a) { return df_make(a.x, a.y); }
+
 SLS_DEV dfloat df_norm(float s, float e) {
   float h, l;
   fast_two_sum(s, e, h, l);

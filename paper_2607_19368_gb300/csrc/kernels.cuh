@@ -25,6 +25,9 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
                                   cudaStream_t stream, int* status);
 
 // ---- Lanczos (Algorithm 2) --------------------------------------------------
+// Row stride (in float2) of the double-float basis Q: r rounded up to even.
+__host__ __device__ inline int q_ld(int r) { return (r + 1) & ~1; }
+
 // A batch of independent problems, problem p owning rows
 // [row0[p], row0[p] + n[p]) of Phi, Q and U and start vector q1 + q1off[p].
 struct LanczosBatch {
@@ -56,7 +59,12 @@ size_t lanczos_scratch_bytes(int64_t nmax, int D, int r, int groups, int ctas_pe
 int lanczos_plan(int64_t nmax, int D, int r, int nprob, int* groups, int* ctas_per_group);
 int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, int* status,
                    int groups, int ctas_per_group, cudaStream_t stream);
-int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream);
+int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream, bool values_done = false);
+// Small problems (every window at most 32 rows, r <= 32): one warp per
+// problem runs Algorithm 2 exactly (two Gram-Schmidt passes, beta = |z|) and
+// the Ritz values; launch_tridiag_eigen(values_done = true) then adds S.
+bool lanczos_window_fits(int64_t nmax, int D, int r);
+int launch_lanczos_window(const LanczosBatch& bt, cudaStream_t stream);
 int launch_ritz_vectors(const LanczosBatch& bt, float* U, cudaStream_t stream);
 
 // ---- SimHash (Sec. 3.3) -----------------------------------------------------

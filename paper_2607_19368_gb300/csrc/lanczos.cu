@@ -7,6 +7,7 @@
 // modified Gram-Schmidt inside clusters of nearly equal eigenvalues.  Finally
 // U = Q S.
 #include "lanczos_kernel.cuh"
+#include "tridiag.cuh"
 
 namespace sls {
 
@@ -18,49 +19,6 @@ namespace {
 // 64-cycle dependent latency (and a divide of several hundred cycles), which
 // a serial recurrence pays at every step.
 // ----------------------------------------------------------------------------
-
-SLS_DEV dfloat df_div(dfloat a, dfloat b) {
-  const float q1 = __fdividef(a.hi, b.hi);
-  float p, e;
-  two_prod(q1, b.hi, p, e);
-  const float rr = (((a.hi - p) - e) + a.lo) - q1 * b.lo;
-  const float q2 = __fdividef(rr, b.hi);
-  return df_norm(q1, q2);
-}
-
-SLS_DEV dfloat df_scale(dfloat a, float s) { return df_make(a.hi * s, a.lo * s); }
-
-// Number of eigenvalues of the (scaled) tridiagonal below x, from the signs of
-// the leading principal minors p_i(x) (three-term recurrence, Sturm sequence).
-// Powers of two rescale the pair (p_{i-1}, p_i) to keep it in range; a zero
-// minor takes the sign opposite to its predecessor.
-SLS_DEV int sturm_count(const float2* __restrict__ a, const float2* __restrict__ b2, int n,
-                        dfloat x) {
-  dfloat pm = df_make(1.f, 0.f), pc = df_sub(dfv(a[0]), x);
-  int sprev = 0;
-  int s = (pc.hi < 0.f) ? 1 : ((pc.hi > 0.f) ? 0 : 1);
-  int cnt = (s != sprev);
-  sprev = s;
-  for (int i = 1; i < n; ++i) {
-    const dfloat d = df_sub(dfv(a[i]), x);
-    const dfloat t = df_mul(dfv(b2[i - 1]), pm);
-    const dfloat pn = df_sub(df_mul(d, pc), t);
-    pm = pc;
-    pc = pn;
-    const float mg = fmaxf(fabsf(pc.hi), fabsf(pm.hi));
-    if (mg > 0x1p60f) {
-      pc = df_scale(pc, 0x1p-60f);
-      pm = df_scale(pm, 0x1p-60f);
-    } else if (mg < 0x1p-60f && mg > 0.f) {
-      pc = df_scale(pc, 0x1p60f);
-      pm = df_scale(pm, 0x1p60f);
-    }
-    s = (pc.hi < 0.f) ? 1 : ((pc.hi > 0.f) ? 0 : 1 - sprev);
-    cnt += (s != sprev);
-    sprev = s;
-  }
-  return cnt;
-}
 
 constexpr int EIG_THREADS = 256;  // shifts per multisection round
 
@@ -148,38 +106,21 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
 // modified Gram-Schmidt within clusters of close eigenvalues
 // ----------------------------------------------------------------------------
 
-__global__ void __launch_bounds__(32)
-tridiag_eigvecs_kernel(LanczosBatch bt) {
-  __shared__ float2 d[SLS_MAX_R], du[SLS_MAX_R], du2[SLS_MAX_R], dl[SLS_MAX_R];
-  __shared__ float2 y[SLS_MAX_R];
-  __shared__ unsigned char piv[SLS_MAX_R];
-  const int m = blockIdx.x, p = blockIdx.y, lane = threadIdx.x;
-  int nprob = bt.nprob_max;
-  if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
-  if (p >= nprob) return;
+// Eigenvectors of one cluster [first, last] of nearly equal Ritz values of
+// problem p (n = r_eff), written as columns of S: inverse iteration with
+// partial-pivoting LU of T - shift I in double-float, three iterations, each
+// followed by modified Gram-Schmidt against the cluster members already
+// found.  One thread; the work arrays (n entries each) belong to the caller.
+SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int last,
+                            float2* __restrict__ d, float2* __restrict__ du,
+                            float2* __restrict__ du2, float2* __restrict__ dl,
+                            float2* __restrict__ y, unsigned char* __restrict__ piv) {
   const int r = bt.r;
-  const int n = bt.r_eff[p];
   double* S = bt.S + (size_t)p * r * r;
-  if (m >= n) {
-    for (int k = lane; k < r; k += 32) S[(size_t)k * r + m] = 0.0;
-    return;
-  }
   const double* th = bt.theta + (size_t)p * r;
   const double* a = bt.alpha + (size_t)p * r;
   const double* b = bt.beta + (size_t)p * r;
   const double tnorm = fmax(fabs(th[0]), fabs(th[n - 1])) + DBL_MIN;
-  const double ctol = 1e-7 * tnorm;
-  int first = m;
-  while (first > 0 && th[first - 1] - th[first] <= ctol) --first;
-  if (first != m) {
-    // another CTA (the first member of this cluster) writes this column
-    return;
-  }
-  int last = m;
-  while (last + 1 < n && th[last] - th[last + 1] <= ctol) ++last;
-  for (int k = lane + n; k < r; k += 32)
-    for (int mm = first; mm <= last; ++mm) S[(size_t)k * r + mm] = 0.0;
-  if (lane != 0) return;
   // a power-of-two scale of T (the eigenvectors do not change)
   int ex = 0;
   frexp(tnorm, &ex);
@@ -283,8 +224,75 @@ tridiag_eigvecs_kernel(LanczosBatch bt) {
     }
     const double sg = (y[0].x < 0.f) ? -1.0 : 1.0;
     for (int i = 0; i < n; ++i) S[(size_t)i * r + mm] = sg * df_to_double(dfv(y[i]));
-    __threadfence_block();
   }
+}
+
+// Cluster bounds of eigenvalue m: [first, last] with neighbours closer than
+// 1e-7 * |T| merged (the eigenvectors of a cluster are computed together).
+SLS_DEV void eig_cluster(const double* th, int n, int m, int& first, int& last) {
+  const double tnorm = fmax(fabs(th[0]), fabs(th[n - 1])) + DBL_MIN;
+  const double ctol = 1e-7 * tnorm;
+  first = m;
+  while (first > 0 && th[first - 1] - th[first] <= ctol) --first;
+  last = m;
+  while (last + 1 < n && th[last] - th[last + 1] <= ctol) ++last;
+}
+
+// One CTA (lane 0 working) per Ritz value: the CTA of a cluster's first
+// member computes the whole cluster.
+__global__ void __launch_bounds__(32)
+tridiag_eigvecs_kernel(LanczosBatch bt) {
+  __shared__ float2 d[SLS_MAX_R], du[SLS_MAX_R], du2[SLS_MAX_R], dl[SLS_MAX_R];
+  __shared__ float2 y[SLS_MAX_R];
+  __shared__ unsigned char piv[SLS_MAX_R];
+  const int m = blockIdx.x, p = blockIdx.y, lane = threadIdx.x;
+  int nprob = bt.nprob_max;
+  if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
+  if (p >= nprob) return;
+  const int r = bt.r;
+  const int n = bt.r_eff[p];
+  double* S = bt.S + (size_t)p * r * r;
+  if (m >= n) {
+    for (int k = lane; k < r; k += 32) S[(size_t)k * r + m] = 0.0;
+    return;
+  }
+  int first, last;
+  eig_cluster(bt.theta + (size_t)p * r, n, m, first, last);
+  if (first != m) return;  // another CTA (the first member of this cluster) writes this column
+  for (int k = lane + n; k < r; k += 32)
+    for (int mm = first; mm <= last; ++mm) S[(size_t)k * r + mm] = 0.0;
+  if (lane != 0) return;
+  eigvec_cluster(bt, p, n, first, last, d, du, du2, dl, y, piv);
+}
+
+// Small problems (r <= 32): one warp per problem, one lane per Ritz value;
+// the lane of a cluster's first member computes the whole cluster, with its
+// work arrays in local memory.
+constexpr int EIGW_WARPS = 4;
+constexpr int EIGW_MAXR = 32;
+
+__global__ void __launch_bounds__(EIGW_WARPS * 32)
+tridiag_eigvecs_warp_kernel(LanczosBatch bt) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int p = blockIdx.x * EIGW_WARPS + warp;
+  int nprob = bt.nprob_max;
+  if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
+  if (p >= nprob) return;
+  const int r = bt.r;
+  const int n = bt.r_eff[p];
+  double* S = bt.S + (size_t)p * r * r;
+  // S rows and columns beyond r_eff are zero
+  for (int e = lane; e < r * r; e += 32) {
+    const int i = e / r, m = e % r;
+    if (i >= n || m >= n) S[e] = 0.0;
+  }
+  if (lane >= n) return;
+  int first, last;
+  eig_cluster(bt.theta + (size_t)p * r, n, lane, first, last);
+  if (first != lane) return;
+  float2 d[EIGW_MAXR], du[EIGW_MAXR], du2[EIGW_MAXR], dl[EIGW_MAXR], y[EIGW_MAXR];
+  unsigned char piv[EIGW_MAXR];
+  eigvec_cluster(bt, p, n, first, last, d, du, du2, dl, y, piv);
 }
 
 // ----------------------------------------------------------------------------
@@ -441,11 +449,18 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
   return SLS_ERR_UNSUPPORTED;
 }
 
-int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream) {
+int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream, bool values_done) {
   dim3 grid(bt.r, bt.nprob_max);
-  tridiag_eigvals_kernel<<<grid, EIG_THREADS, 0, stream>>>(bt);
-  SLS_LAUNCH_CHECK();
-  tridiag_eigvecs_kernel<<<grid, 32, 0, stream>>>(bt);
+  if (!values_done) {
+    tridiag_eigvals_kernel<<<grid, EIG_THREADS, 0, stream>>>(bt);
+    SLS_LAUNCH_CHECK();
+  }
+  if (bt.r <= EIGW_MAXR) {
+    const int blocks = (bt.nprob_max + EIGW_WARPS - 1) / EIGW_WARPS;
+    tridiag_eigvecs_warp_kernel<<<blocks, EIGW_WARPS * 32, 0, stream>>>(bt);
+  } else {
+    tridiag_eigvecs_kernel<<<grid, 32, 0, stream>>>(bt);
+  }
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }

@@ -60,7 +60,6 @@ constexpr int LZ_THREADS = LZ_CT + 32;    // plus one copy warp
 constexpr unsigned BAR_COMPUTE = 1;       // named barrier: the compute warps
 
 // leading dimension (float2) of the basis rows: even, so rows are 16-byte aligned
-__host__ __device__ inline int q_ld(int r) { return (r + 1) & ~1; }
 
 // Per-group scratch layout (byte offsets), identical on host and device.
 struct LzLayout {
@@ -84,8 +83,6 @@ __host__ __device__ inline LzLayout lz_layout(int64_t nmax, int D, int r, int g)
   return L;
 }
 
-SLS_DEV float2 f2(dfloat a) { return make_float2(a.hi, a.lo); }
-SLS_DEV dfloat dfv(float2 a) { return df_make(a.x, a.y); }
 
 SLS_DEV dfloat shfl_df(dfloat v, int src) {
   v.hi = __shfl_sync(0xffffffffu, v.hi, src);

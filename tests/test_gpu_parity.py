@@ -172,6 +172,23 @@ def test_lanczos_tiny_sizes(sls):
         _lanczos_case(sls, phi32, g.standard_normal(N), r)
 
 
+@pytest.mark.parametrize("N,D,r,distinct", [(2, 4, 4, 2), (5, 64, 16, 5), (16, 256, 16, 16),
+                                             (16, 256, 16, 9), (17, 100, 32, 17),
+                                             (32, 1024, 32, 20), (32, 256, 8, 32)])
+def test_lanczos_window_sizes(sls, N, D, r, distinct):
+    """Window-sized problems (N <= 32, the local backend's windows) take the
+    warp-per-problem kernel: r_eff (breakdown on repeated tokens), Ritz
+    values and subspace against the oracle."""
+    g = np.random.default_rng(N * 1000 + D + distinct)
+    d = 48
+    X = g.standard_normal((distinct, d)) / math.sqrt(d)
+    X = X[np.concatenate([np.arange(distinct), g.integers(0, distinct, N - distinct)])]
+    W = g.standard_normal((D, d)) * d ** -0.25
+    b = g.random(D) * 2 * math.pi
+    phi32 = O.rff_features(X, W, b).astype(np.float32)
+    _lanczos_case(sls, phi32, g.standard_normal(N), r)
+
+
 # ---------------------------------------------------------------------------
 # SimHash (Sec. 3.3) -- bit-exact given the oracle's U
 # ---------------------------------------------------------------------------
@@ -434,3 +451,66 @@ def test_compress_adaptive_small_batch(sls, D):
             for k, (s, e) in enumerate(bounds):
                 if not route[i, k]:
                     assert np.array_equal(t[s:e], res.tok2macro[s:e])
+
+
+BREAK_BAND = 30.0
+
+
+def _reff_agrees(phi, q1, r, tol, r_gpu):
+    """r_eff of Algorithm 2 on one window against the oracle.  Equal, or one
+    apart where the oracle's beta_j / max_i(|alpha_i| + beta_i) at the step in
+    question lies within a factor BREAK_BAND of tol: there beta is rounding
+    noise amplified near a breakdown (Phi of lower rank than r), the decision
+    belongs to the rounding, and both outcomes are Algorithm 2 executed
+    exactly up to rounding (the factor is the ratio of the double-float and
+    float64 unit roundoffs of the two matvecs)."""
+    a, be, _, _ = O.lanczos(phi, q1, r, tol=0.0)
+    rel = be / np.maximum.accumulate(np.abs(a[:len(be)]) + be)
+    hit = np.nonzero(rel <= tol)[0]
+    r_o = int(hit[0]) + 1 if hit.size else len(a)
+    if r_gpu == r_o:
+        return True
+    if abs(r_gpu - r_o) != 1:
+        return False
+    j = min(r_gpu, r_o) - 1
+    return tol / BREAK_BAND <= rel[j] <= tol * BREAK_BAND
+
+
+@pytest.mark.parametrize("dtype,D", [("bf16", 256), ("f32", 64)])
+def test_compress_local_w16(sls, dtype, D):
+    """Local LSH at the paper's default window of 16 (Sec. 3.5): every window
+    spectral with its exact budget; r_eff per window matches the oracle; at
+    rho = 16 every window is one macro-token, so the whole output matches the
+    oracle; otherwise the invariants and the per-window macro counts."""
+    w = WL.scaled(WL.WORKLOADS["mistral7b"], N=700, d=64, D=D, dtype=dtype)
+    p = WL.make_prompt(w)
+    prm = WL.make_params(D, 64, 16, 16, 700, dtype)
+    X = to_torch_x(p.X, dtype)
+    X64 = p.x_f64()
+    Nc = 688
+    bounds = O.window_bounds(Nc, 16)
+    for rho in (2.0, 4.0, 16.0):
+        cfg = sls.Config.make(backend=sls.BACKEND_LOCAL, rho=rho, D=D, r=16, window=16,
+                              preserve_last=12)
+        Xt, pos, t2m, r_eff, route = sls.compress(X, cfg, to_torch_x(prm.W, dtype),
+                                                  torch.from_numpy(prm.b).cuda(),
+                                                  torch.from_numpy(prm.R).cuda(),
+                                                  torch.from_numpy(prm.q1).cuda())
+        M = sls.output_count(cfg, 700)
+        ocfg = O.CompressConfig(rho=rho, D=D, r=16, window=16, preserve_last=12)
+        res = O.compress_local(X64, prm.w_f64(), prm.b, prm.R, prm.q1, ocfg)
+        assert np.all(route.cpu().numpy()[:len(bounds)] == 1)
+        rg = r_eff.cpu().numpy()[:len(bounds)]
+        for k, (s_, e_) in enumerate(bounds):
+            if rg[k] != res.info["r_eff"][k]:
+                phi = oracle_phi32(X64[s_:e_], prm.w_f64(), prm.b).astype(np.float64)
+                assert _reff_agrees(phi, prm.q1[s_:e_], 16, 1e-10, int(rg[k])), (rho, k)
+        assert np.mean(rg == np.array(res.info["r_eff"])) >= 0.9
+        t = t2m.cpu().numpy()
+        _check_pass(sls, X64, Xt.cpu().numpy(), pos.cpu().numpy(), t, M, 0, 12)
+        for (s_, e_), m in zip(bounds, res.info["budgets"]):
+            assert len(np.unique(t[s_:e_])) == m
+        if rho >= 16:
+            assert np.array_equal(t, res.tok2macro)
+            assert np.array_equal(pos.cpu().numpy(), res.pos)
+            assert np.max(np.abs(Xt.cpu().numpy() - res.Xt)) <= EMB_TOL

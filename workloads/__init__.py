@@ -21,6 +21,9 @@ available here):
                 table-like structure of the paper's stress test, Table 4)
 * ``adaptive``  64 prompts of N=16384, d=4096, bf16, generated like
                 ``mistral7b`` with duplication 0.6*p/63 for prompt p.
+* ``local``     the ``qwen7b`` prompt at the paper's local-LSH defaults
+                (Sec. 5.1 hyperparameters: D=256, r=16, window 16, bits from
+                the window budget), rho=8.
 
 Vocabulary rows are N(0, 1/d) and are produced by a counter-based generator
 (numpy Philox keyed by the seed, counter = token id), so the V x d table is
@@ -178,8 +181,9 @@ class Workload:
     span_hi: int = 64
     template_frac: float = 0.0
     batch: int = 1      # independent prompts (adaptive workload)
-    window: int = 0     # adaptive window length (0 = global backend)
+    window: int = 0     # window length of the windowed backends (0 = global backend)
     rhos: tuple = ()    # swept compression ratios (adaptive workload)
+    backend: str = "global"   # "global", "adaptive" or "local"
 
 
 WORKLOADS = {
@@ -197,7 +201,11 @@ WORKLOADS = {
     "adaptive": Workload("adaptive", N=16384, d=4096, V=32768, zipf=1.1,
                          dtype="bf16", D=1024, r=32, bits=0, rho=8.0,
                          dup_frac=0.0, span_lo=64, span_hi=64, batch=64,
-                         window=2048, rhos=(2.0, 4.0, 8.0, 16.0)),
+                         window=2048, rhos=(2.0, 4.0, 8.0, 16.0), backend="adaptive"),
+    "local": Workload("local", N=32768, d=3584, V=151936, zipf=1.05,
+                      dtype="bf16", D=256, r=16, bits=0, rho=8.0,
+                      dup_frac=0.3, span_lo=16, span_hi=256, window=16,
+                      backend="local"),
 }
 
 
