@@ -285,7 +285,7 @@ struct CompressWs {
   size_t lz_bytes;
   void* seg_scratch;
   int *perm, *mstart, *mlen;
-  int *it_start, *pt_start;
+  int* pt_start;
   int2* items;
   int* counts;
   float *part, *part_eta;
@@ -379,10 +379,9 @@ void carve(const CompressPlan& P, void* ws, CompressWs* W) {
   W->perm = cv.take<int>(toks);
   W->mstart = cv.take<int>(macs);
   W->mlen = cv.take<int>(macs);
-  W->it_start = cv.take<int>(macs);
   W->pt_start = cv.take<int>(macs);
   W->items = cv.take<int2>(agg_item_capacity(macs, toks));
-  W->counts = cv.take<int>(4);
+  W->counts = cv.take<int>(agg_aux_ints(macs, toks));
   W->part = cv.take<float>(0);  // sized below (depends on d)
   W->part_eta = nullptr;
   W->total = cv.off;
@@ -542,9 +541,8 @@ size_t sls_aggregate_workspace_size(int64_t N, int d, int64_t M_target) {
   cv.take<int>(M_target);
   cv.take<int>(M_target);
   cv.take<int>(M_target);
-  cv.take<int>(M_target);
   cv.take<int2>(agg_item_capacity(M_target, N));
-  cv.take<int>(4);
+  cv.take<int>(agg_aux_ints(M_target, N));
   return cv.off + part_bytes(N, d);
 }
 
@@ -569,10 +567,9 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
   int* perm = cv.take<int>(N);
   int* mstart = cv.take<int>(M_target);
   int* mlen = cv.take<int>(M_target);
-  int* it_start = cv.take<int>(M_target);
   int* pt_start = cv.take<int>(M_target);
   int2* items = cv.take<int2>(agg_item_capacity(M_target, N));
-  int* counts = cv.take<int>(4);
+  int* counts = cv.take<int>(agg_aux_ints(M_target, N));
   float* part = cv.take<float>(agg_part_capacity(N) * (size_t)d);
   float* part_eta = cv.take<float>(agg_part_capacity(N));
   SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
@@ -583,7 +580,7 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
                            M_target, perm, mstart, mlen, pos, tok2macro, status, s)) != SLS_OK)
     return st;
   return launch_aggregate(X, x_dtype, d, ldx, perm, mstart, mlen, M_target, N, renorm, Xt,
-                          it_start, pt_start, items, counts, part, part_eta, status, s);
+                          pt_start, items, counts, part, part_eta, status, s);
 }
 
 int64_t sls_output_count(const sls_config_t* cfg, int64_t N) {
@@ -749,8 +746,8 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   phase_mark(5, 1, s);
   phase_mark(6, 0, s);
   st = launch_aggregate(X, x_dtype, d, ldx, W.perm, W.mstart, W.mlen, B * P.M, B * N,
-                        cfg->renorm, Xt, W.it_start, W.pt_start, W.items, W.counts, W.part,
-                        W.part_eta, W.status, s);
+                        cfg->renorm, Xt, W.pt_start, W.items, W.counts, W.part, W.part_eta,
+                        W.status, s);
   phase_mark(6, 1, s);
   return st;
 }

@@ -278,13 +278,19 @@ SLS_DEV bool mbar_try_wait(uint64_t* bar, unsigned parity) {
   return ok != 0;
 }
 
-// Bounded wait for the phase with the given parity; false after the limit.
+// Clock cycles after which a wait on a barrier gives up (about a second).
+constexpr long long SLS_WAIT_CYCLES = 1ll << 31;
+
+// Bounded wait for the phase with the given parity; false after about a
+// second.  try_wait itself suspends the thread in hardware for a while, so
+// the loop polls without sleeping (a sleep delays the waiter's wake-up and
+// with it the stage hand-over of a copy ring).
 SLS_DEV bool mbar_wait(uint64_t* bar, unsigned parity) {
-  for (unsigned it = 0; it < (1u << 26); ++it) {
+  const long long t0 = clock64();
+  for (unsigned it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (it > 64) __nanosleep(32);
+    if ((it & 63) == 63 && clock64() - t0 > SLS_WAIT_CYCLES) return false;
   }
-  return false;
 }
 
 // One-dimensional bulk copy global -> shared, completion counted on `bar`.
@@ -347,13 +353,9 @@ SLS_DEV unsigned atom_add_acq_rel_gpu(unsigned* p, unsigned v) {
 // launch, or a subset).  `count` lives in global memory and starts at 0;
 // `gen` is unused.  Every CTA counts the barriers it passed in `local_gen`.
 // Returns false (and sets *status = SLS_ERR_TIMEOUT) when the wait exceeded
-// its iteration limit or another CTA gave up; the caller must then leave the
-// kernel.
+// about a second (SLS_WAIT_CYCLES) or another CTA gave up; the caller must
+// then leave the kernel.
 // ---------------------------------------------------------------------------
-
-#ifndef SLS_SPIN_LIMIT
-#define SLS_SPIN_LIMIT (1u << 21)  // ~2M polls of ~1 us each: a few seconds
-#endif
 
 struct GroupBarrier {
   unsigned* count;
@@ -363,7 +365,7 @@ struct GroupBarrier {
 
 // Bit of the arrival counter that releases every waiter with an error: a CTA
 // that gives up sets it, so the other CTAs of the group stop at their next
-// barrier instead of waiting out the iteration limit.
+// barrier instead of waiting out the time limit.
 constexpr unsigned SLS_BAR_POISON = 0x80000000u;
 
 SLS_DEV void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
@@ -388,15 +390,15 @@ SLS_DEV bool group_sync_named(const GroupBarrier& bar, unsigned& local_gen, int*
       const unsigned target = (local_gen + 1) * bar.nblocks;
       fence_acq_rel_gpu();
       unsigned v = atom_add_acq_rel_gpu(bar.count, 1u) + 1u;
+      const long long t0 = clock64();
       unsigned it = 0;
       while (v < target) {
-        if (++it > SLS_SPIN_LIMIT) {
+        if ((++it & 63) == 0 && clock64() - t0 > SLS_WAIT_CYCLES) {
           ok = 0;
           atomicExch(status, SLS_ERR_TIMEOUT);
           atomicOr(bar.count, SLS_BAR_POISON);
           break;
         }
-        if (it > 32) __nanosleep(32);
         v = ld_acquire_gpu(bar.count);
       }
       if (v & SLS_BAR_POISON) ok = 0;

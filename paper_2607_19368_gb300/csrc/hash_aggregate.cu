@@ -919,34 +919,133 @@ constexpr int AGG_T = 256;
 constexpr int AGG_CH = 64;      // members per work item
 constexpr int AGG_MAXV = 32;    // accumulators per thread (d <= 8192)
 
-// Work items: macro-token m is split into ceil(len / AGG_CH) items.
-__global__ void __launch_bounds__(SEG_T, 1)
-agg_items_kernel(const int* __restrict__ mlen, int64_t Mtot, int* __restrict__ it_start,
-                 int* __restrict__ pt_start, int2* __restrict__ items, int* __restrict__ counts) {
+// Work items: macro-token m is split into ceil(len / AGG_CH) items, listed in
+// macro order.  Three grid-wide passes: per-block totals over the macro
+// lengths; per macro its item offset, member-row offset, partial-sum slot and
+// (for macros spanning several items) its place in a compact list; then one
+// thread per item finds its macro by binary search over the increasing item
+// offsets, writes the item and, for each of the G member-pass CTAs whose
+// balanced row boundary falls inside the item, that CTA's first item.
+constexpr int AI_BLOCK = SEG_T;           // macros per block (one per thread)
+constexpr int AGG_MAX_GRID = 2048;        // member-pass CTAs at most
+
+// Auxiliary integers of the aggregation: counts (16), block totals (4 per
+// block), CTA range starts (AGG_MAX_GRID + 1), multi-item macro list, and per
+// macro its first item and first member row.
+struct AggAux {
+  int* counts;  // [0] items, [1] partial slots, [2] multi-item macros, [3] member rows
+  int4* btot;
+  int* cta_first;
+  int* multi;
+  int* it_start;
+  int* r_start;
+};
+
+__host__ __device__ inline int64_t agg_blocks(int64_t Mtot) { return (Mtot + AI_BLOCK - 1) / AI_BLOCK; }
+
+__host__ __device__ inline AggAux agg_aux(int* base, int64_t Mtot, int64_t Ntot) {
+  AggAux A;
+  A.counts = base;
+  A.btot = reinterpret_cast<int4*>(base + 16);
+  A.cta_first = base + 16 + 4 * agg_blocks(Mtot);
+  A.multi = A.cta_first + AGG_MAX_GRID + 1;
+  A.it_start = A.multi + Ntot / AGG_CH + 2;
+  A.r_start = A.it_start + Mtot;
+  return A;
+}
+
+SLS_DEV int nchunks(int len) { return (len + AGG_CH - 1) / AGG_CH; }
+
+__global__ void __launch_bounds__(SEG_T)
+agg_count_kernel(const int* __restrict__ mlen, int64_t Mtot, int64_t Ntot, int* __restrict__ aux) {
   __shared__ int sh[SEG_W + 1];
-  const int tid = threadIdx.x;
-  const int chunk = (int)((Mtot + SEG_T - 1) / SEG_T);
-  const int64_t b = min(Mtot, (int64_t)tid * chunk), e = min(Mtot, b + chunk);
-  int s1 = 0, s2 = 0;
-  for (int64_t m = b; m < e; ++m) {
-    const int nch = (mlen[m] + AGG_CH - 1) / AGG_CH;
-    s1 += nch;
-    s2 += (nch > 1) ? nch : 0;
+  const AggAux A = agg_aux(aux, Mtot, Ntot);
+  const int64_t m = (int64_t)blockIdx.x * AI_BLOCK + threadIdx.x;
+  const int len = (m < Mtot) ? mlen[m] : 0, nch = nchunks(len);
+  int t0, t1, t2, t3;
+  block_excl_scan<int>(nch, sh, &t0);
+  block_excl_scan<int>((nch > 1) ? nch : 0, sh, &t1);
+  block_excl_scan<int>((nch > 1) ? 1 : 0, sh, &t2);
+  block_excl_scan<int>(len, sh, &t3);
+  if (threadIdx.x == 0) A.btot[blockIdx.x] = make_int4(t0, t1, t2, t3);
+}
+
+__global__ void __launch_bounds__(SEG_T)
+agg_offsets_kernel(const int* __restrict__ mlen, int64_t Mtot, int64_t Ntot,
+                   int* __restrict__ aux, int* __restrict__ pt_start) {
+  __shared__ int sh[SEG_W + 1];
+  const AggAux A = agg_aux(aux, Mtot, Ntot);
+  const int nb = (int)agg_blocks(Mtot);
+  // offsets of this block (sum over the blocks before it) and the totals
+  int b0 = 0, b1 = 0, b2 = 0, b3 = 0, a0 = 0, a1 = 0, a2 = 0, a3 = 0;
+  for (int k = threadIdx.x; k < nb; k += SEG_T) {
+    const int4 v = A.btot[k];
+    if (k < (int)blockIdx.x) {
+      b0 += v.x;
+      b1 += v.y;
+      b2 += v.z;
+      b3 += v.w;
+    }
+    a0 += v.x;
+    a1 += v.y;
+    a2 += v.z;
+    a3 += v.w;
   }
-  int t1, t2;
-  int o1 = block_excl_scan<int>(s1, sh, &t1);
-  int o2 = block_excl_scan<int>(s2, sh, &t2);
-  for (int64_t m = b; m < e; ++m) {
-    const int nch = (mlen[m] + AGG_CH - 1) / AGG_CH;
-    it_start[m] = o1;
-    pt_start[m] = (nch > 1) ? o2 : -1;
-    for (int c = 0; c < nch; ++c) items[o1 + c] = make_int2((int)m, c);
-    o1 += nch;
-    o2 += (nch > 1) ? nch : 0;
+  int o0, o1, o2, o3, n0, n1, n2, n3;
+  block_excl_scan<int>(b0, sh, &o0);
+  block_excl_scan<int>(b1, sh, &o1);
+  block_excl_scan<int>(b2, sh, &o2);
+  block_excl_scan<int>(b3, sh, &o3);
+  block_excl_scan<int>(a0, sh, &n0);
+  block_excl_scan<int>(a1, sh, &n1);
+  block_excl_scan<int>(a2, sh, &n2);
+  block_excl_scan<int>(a3, sh, &n3);
+  const int64_t m = (int64_t)blockIdx.x * AI_BLOCK + threadIdx.x;
+  const int len = (m < Mtot) ? mlen[m] : 0, nch = nchunks(len);
+  int tt;
+  const int ito = o0 + block_excl_scan<int>(nch, sh, &tt);
+  const int pto = o1 + block_excl_scan<int>((nch > 1) ? nch : 0, sh, &tt);
+  const int muo = o2 + block_excl_scan<int>((nch > 1) ? 1 : 0, sh, &tt);
+  const int ro = o3 + block_excl_scan<int>(len, sh, &tt);
+  if (m < Mtot) {
+    A.it_start[m] = ito;
+    A.r_start[m] = ro;
+    pt_start[m] = (nch > 1) ? pto : -1;
+    if (nch > 1) A.multi[muo] = (int)m;
   }
-  if (tid == 0) {
-    counts[0] = t1;
-    counts[1] = t2;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    A.cta_first[0] = 0;
+    A.counts[0] = n0;
+    A.counts[1] = n1;
+    A.counts[2] = n2;
+    A.counts[3] = n3;
+  }
+}
+
+__global__ void __launch_bounds__(256)
+agg_fill_kernel(const int* __restrict__ mlen, int64_t Mtot, int64_t Ntot, int G,
+                int* __restrict__ aux, int2* __restrict__ items) {
+  const AggAux A = agg_aux(aux, Mtot, Ntot);
+  const int nitems = A.counts[0];
+  const int64_t rtot = A.counts[3];
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nitems; i += gridDim.x * blockDim.x) {
+    // the macro of item i: the last m with it_start[m] <= i
+    int lo = 0, hi = (int)Mtot - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (A.it_start[mid] <= i)
+        lo = mid;
+      else
+        hi = mid - 1;
+    }
+    const int m = lo, c = i - A.it_start[m], len = mlen[m];
+    items[i] = make_int2(m, c);
+    // CTA t starts at the first item whose first row is at or past
+    // t * rtot / G: the item after the last one starting before it
+    const int64_t rs = (int64_t)A.r_start[m] + (int64_t)c * AGG_CH;
+    const int64_t re = (int64_t)A.r_start[m] + min((int64_t)len, (int64_t)(c + 1) * AGG_CH);
+    const int64_t tlo = rs * G / rtot + 1, thi = re * G / rtot;
+    for (int64_t t = tlo; t <= thi && t <= G; ++t) A.cta_first[t] = i + 1;
   }
 }
 
@@ -1051,16 +1150,21 @@ constexpr int agg_batch() {
   return NV >= 8 ? 1 : 8 / NV;
 }
 
+// The macro-tokens whose members span several items: sum their partial rows
+// and finalise (one CTA per macro-token of the compact list).
 template <int V, int NV>
 __global__ void __launch_bounds__(AGG_T)
 agg_final_kernel(int d, const int* __restrict__ mlen, const int* __restrict__ pt_start,
-                 int64_t Mtot, int renorm, const float* __restrict__ part,
-                 const float* __restrict__ part_eta, float* __restrict__ Xt) {
+                 int64_t Mtot, int64_t Ntot, int renorm, const int* __restrict__ aux,
+                 const float* __restrict__ part, const float* __restrict__ part_eta,
+                 float* __restrict__ Xt) {
   __shared__ float sh[AGG_T / 32];
   const int tid = threadIdx.x;
-  for (int64_t m = blockIdx.x; m < Mtot; m += gridDim.x) {
+  const AggAux A = agg_aux(const_cast<int*>(aux), Mtot, Ntot);
+  const int nmulti = A.counts[2];
+  for (int t = blockIdx.x; t < nmulti; t += gridDim.x) {
+    const int64_t m = A.multi[t];
     const int ps = pt_start[m];
-    if (ps < 0) continue;
     const int len = mlen[m];
     const int nch = (len + AGG_CH - 1) / AGG_CH;
     float acc[NV * V];
@@ -1104,7 +1208,7 @@ agg_final_kernel(int d, const int* __restrict__ mlen, const int* __restrict__ pt
 
 // ---------------------------------------------------------------------------
 // Member pass with a shared-memory row ring.  Warp 0 is the producer: it walks
-// this CTA's work items (items blockIdx.x, blockIdx.x + G, ...), loads each
+// this CTA's contiguous range of work items (balanced by member rows), loads each
 // item's descriptor and member ids one item ahead, and streams every member
 // row into an S-stage ring with one bulk async copy per row (mbarrier
 // complete_tx); the item descriptor travels with the item's first row.  Warps
@@ -1159,28 +1263,33 @@ SLS_DEV void load_vec_smem<uint16_t>(const uint16_t* p, float* out) {
   }
 }
 
-// Bounded wait that also returns early once another role has aborted.
+// Bounded wait (about a second of clock cycles) that also returns early once
+// another role has aborted.  The producer polls without sleeping so that it
+// refills a stage as soon as it is released; the eight consumer warps back
+// off after a few polls so that their polling does not take the producer's
+// issue slots.
+template <bool BACKOFF>
 SLS_DEV bool agr_wait(uint64_t* bar, unsigned parity, volatile int* abort_flag) {
-  for (unsigned it = 0; it < (1u << 25); ++it) {
+  const long long t0 = clock64();
+  for (unsigned it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255) == 255 && *abort_flag) return false;
-    if (it > 64) __nanosleep(32);
+    if ((it & 63) == 63 && (*abort_flag || clock64() - t0 > SLS_WAIT_CYCLES)) return false;
+    if (BACKOFF && it > 64) __nanosleep(32);
   }
-  return false;
 }
 
-// Descriptor of the local item kidx of this CTA (global item blockIdx.x +
-// kidx * gridDim.x), or an empty one past the end.
+// Descriptor of the local item kidx of this CTA (item i0 + kidx of its
+// contiguous range [i0, i1)), or an empty one past the end.
 struct LaneDesc {
   int m, c, n, len, ps, off;
 };
 
 SLS_DEV LaneDesc agr_lane_desc(const int2* __restrict__ items, const int* __restrict__ mlen,
                                const int* __restrict__ mstart, const int* __restrict__ pt_start,
-                               int nitems, int kidx) {
+                               int i0, int i1, int kidx) {
   LaneDesc L{0, 0, 0, 0, -1, 0};
-  const int64_t it = (int64_t)blockIdx.x + (int64_t)kidx * gridDim.x;
-  if (it < nitems) {
+  const int it = i0 + kidx;
+  if (it < i1) {
     const int2 item = items[it];
     L.m = item.x;
     L.c = item.y;
@@ -1215,7 +1324,7 @@ template <typename T, int NV>
 __global__ void __launch_bounds__(AGR_THREADS, 2)
 agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restrict__ perm,
                 const int* __restrict__ mstart, const int* __restrict__ mlen,
-                const int2* __restrict__ items, const int* __restrict__ counts,
+                const int2* __restrict__ items, const int* __restrict__ cta_first,
                 const int* __restrict__ pt_start, int renorm, float* __restrict__ Xt,
                 float* __restrict__ part, float* __restrict__ part_eta, int S, int stage_bytes,
                 int* status) {
@@ -1227,8 +1336,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
   __shared__ float sh[AGR_CW];
   __shared__ volatile int s_abort;
   const int DQ = S + 2;
-  const int nitems = counts[0];
-  const int G = gridDim.x;
+  const int i0 = cta_first[blockIdx.x], i1 = cta_first[blockIdx.x + 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const unsigned row_bytes = (unsigned)d * sizeof(T);
   if (threadIdx.x == 0) {
@@ -1249,7 +1357,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
     unsigned issued = 0;
     bool ok = true;
     int kb = 0;
-    LaneDesc cd = agr_lane_desc(items, mlen, mstart, pt_start, nitems, kb + lane);
+    LaneDesc cd = agr_lane_desc(items, mlen, mstart, pt_start, i0, i1, kb + lane);
     while (ok) {
       int pre = cd.n;
 #pragma unroll
@@ -1259,7 +1367,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
       }
       const int nrows = __shfl_sync(0xffffffffu, pre, 31);
       if (nrows == 0) break;
-      const LaneDesc nd = agr_lane_desc(items, mlen, mstart, pt_start, nitems, kb + 32 + lane);
+      const LaneDesc nd = agr_lane_desc(items, mlen, mstart, pt_start, i0, i1, kb + 32 + lane);
       int rid, rj, rs;
       agr_fetch_row(perm, pre, nrows, cd.off, 0, lane, rid, rj, rs);
       for (int f0 = 0; f0 < nrows && ok; f0 += 32) {
@@ -1280,7 +1388,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
           if (lane == 0) {
             const int st = (int)(issued % (unsigned)S);
             const unsigned par = (issued / (unsigned)S) & 1u;
-            if (!agr_wait(&emptyb[st], par ^ 1u, &s_abort)) {
+            if (!agr_wait<false>(&emptyb[st], par ^ 1u, &s_abort)) {
               ok = false;
               s_abort = 1;
               atomicExch(status, SLS_ERR_TIMEOUT);
@@ -1318,7 +1426,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
     unsigned consumed = 0;
     bool ok = true;
     int k = 0;
-    for (int it = blockIdx.x; it < nitems; it += G, ++k) {
+    for (int it = i0; it < i1; ++it, ++k) {
       float acc[NV * V];
 #pragma unroll
       for (int e = 0; e < NV * V; ++e) acc[e] = 0.f;
@@ -1328,7 +1436,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
       for (int s = 0; s < D.n && ok; ++s) {
         const int st = (int)(consumed % (unsigned)S);
         const unsigned par = (consumed / (unsigned)S) & 1u;
-        if (!agr_wait(&fullb[st], par, &s_abort)) {
+        if (!agr_wait<true>(&fullb[st], par, &s_abort)) {
           ok = false;
           if (lane == 0) {
             s_abort = 1;
@@ -1602,14 +1710,18 @@ int launch_identity(const void* X, int x_dtype, int64_t B, int64_t N, int d, int
 }
 
 size_t agg_item_capacity(int64_t Mtot, int64_t Ntot) { return (size_t)(Mtot + Ntot / AGG_CH + 2); }
+size_t agg_aux_ints(int64_t Mtot, int64_t Ntot) {
+  return (size_t)(16 + 4 * agg_blocks(Mtot) + (AGG_MAX_GRID + 1) + Ntot / AGG_CH + 2 + 2 * Mtot);
+}
 size_t agg_part_capacity(int64_t Ntot) { return (size_t)(2 * (Ntot / AGG_CH) + 2); }
 
 namespace {
 template <typename T, int NV>
 int launch_agg_t(const void* X, int d, int64_t ldx, const int* perm, const int* mstart,
-                 const int* mlen, int64_t Mtot, int64_t fblocks, int renorm, float* Xt,
-                 const int* pt_start, const int2* items, const int* counts, float* part,
-                 float* part_eta, int* status, cudaStream_t stream) {
+                 const int* mlen, int64_t Mtot, int64_t Ntot, int64_t fblocks, int renorm,
+                 float* Xt,
+                 int* pt_start, int2* items, int* aux, float* part, float* part_eta,
+                 int* status, cudaStream_t stream) {
   constexpr int V = VecOf<T>::V;
   const int stage = (int)(((size_t)d * sizeof(T) + 127) & ~(size_t)127);
   // two CTAs per SM when each still gets at least 6 ring stages in ~100 KB
@@ -1632,27 +1744,40 @@ int launch_agg_t(const void* X, int d, int64_t ldx, const int* perm, const int* 
   int dev = 0, sms = 0;
   SLS_CUDA_TRY(cudaGetDevice(&dev));
   SLS_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  const int grid = sms * per_sm;
+  int grid = sms * per_sm;
+  if (grid > AGG_MAX_GRID) grid = AGG_MAX_GRID;
+  // work items, partial slots and the balanced CTA ranges
+  const unsigned nb = (unsigned)agg_blocks(Mtot);
+  agg_count_kernel<<<nb, SEG_T, 0, stream>>>(mlen, Mtot, Ntot, aux);
+  SLS_LAUNCH_CHECK();
+  agg_offsets_kernel<<<nb, SEG_T, 0, stream>>>(mlen, Mtot, Ntot, aux, pt_start);
+  SLS_LAUNCH_CHECK();
+  int64_t fill = (Mtot + Ntot / AGG_CH + 255) / 256;
+  if (fill > 8 * (int64_t)sms) fill = 8 * (int64_t)sms;
+  agg_fill_kernel<<<(unsigned)fill, 256, 0, stream>>>(mlen, Mtot, Ntot, grid, aux, items);
+  SLS_LAUNCH_CHECK();
+  const AggAux A = agg_aux(aux, Mtot, Ntot);
   agg_ring_kernel<T, NV><<<grid, AGR_THREADS, smem, stream>>>(
-      (const T*)X, d, ldx, perm, mstart, mlen, items, counts, pt_start, renorm, Xt, part,
+      (const T*)X, d, ldx, perm, mstart, mlen, items, A.cta_first, pt_start, renorm, Xt, part,
       part_eta, S, stage, status);
   SLS_LAUNCH_CHECK();
-  agg_final_kernel<V, NV><<<(unsigned)fblocks, AGG_T, 0, stream>>>(d, mlen, pt_start, Mtot,
-                                                                   renorm, part, part_eta, Xt);
+  agg_final_kernel<V, NV><<<(unsigned)fblocks, AGG_T, 0, stream>>>(
+      d, mlen, pt_start, Mtot, Ntot, renorm, aux, part, part_eta, Xt);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
 
 template <typename T>
 int launch_agg_dtype(const void* X, int d, int64_t ldx, const int* perm, const int* mstart,
-                     const int* mlen, int64_t Mtot, int64_t fblocks, int renorm, float* Xt,
-                     const int* pt_start, const int2* items, const int* counts, float* part,
-                     float* part_eta, int* status, cudaStream_t stream) {
+                     const int* mlen, int64_t Mtot, int64_t Ntot, int64_t fblocks, int renorm,
+                     float* Xt,
+                     int* pt_start, int2* items, int* aux, float* part, float* part_eta,
+                     int* status, cudaStream_t stream) {
   constexpr int V = VecOf<T>::V;
   const int nv = (d / V + AGR_CT - 1) / AGR_CT;
 #define SLS_AGG_NV(N)                                                                       \
-  return launch_agg_t<T, N>(X, d, ldx, perm, mstart, mlen, Mtot, fblocks, renorm, Xt,      \
-                            pt_start, items, counts, part, part_eta, status, stream)
+  return launch_agg_t<T, N>(X, d, ldx, perm, mstart, mlen, Mtot, Ntot, fblocks, renorm, Xt, \
+                            pt_start, items, aux, part, part_eta, status, stream)
   if (nv <= 1) SLS_AGG_NV(1);
   if (nv <= 2) SLS_AGG_NV(2);
   if (nv <= 4) SLS_AGG_NV(4);
@@ -1664,18 +1789,16 @@ int launch_agg_dtype(const void* X, int d, int64_t ldx, const int* perm, const i
 
 int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* perm,
                      const int* mstart, const int* mlen, int64_t Mtot, int64_t Ntot, int renorm,
-                     float* Xt, int* it_start, int* pt_start, int2* items, int* counts,
-                     float* part, float* part_eta, int* status, cudaStream_t stream) {
+                     float* Xt, int* pt_start, int2* items, int* aux, float* part,
+                     float* part_eta, int* status, cudaStream_t stream) {
   if (Mtot == 0) return SLS_OK;
-  (void)Ntot;
-  agg_items_kernel<<<1, SEG_T, 0, stream>>>(mlen, Mtot, it_start, pt_start, items, counts);
-  SLS_LAUNCH_CHECK();
-  const int64_t fblocks = Mtot < 4096 ? Mtot : 4096;
+  int64_t fblocks = Ntot / AGG_CH + 1;
+  if (fblocks > 1024) fblocks = 1024;
   if (x_dtype == SLS_F32)
-    return launch_agg_dtype<float>(X, d, ldx, perm, mstart, mlen, Mtot, fblocks, renorm, Xt,
-                                   pt_start, items, counts, part, part_eta, status, stream);
-  return launch_agg_dtype<uint16_t>(X, d, ldx, perm, mstart, mlen, Mtot, fblocks, renorm, Xt,
-                                    pt_start, items, counts, part, part_eta, status, stream);
+    return launch_agg_dtype<float>(X, d, ldx, perm, mstart, mlen, Mtot, Ntot, fblocks, renorm,
+                                   Xt, pt_start, items, aux, part, part_eta, status, stream);
+  return launch_agg_dtype<uint16_t>(X, d, ldx, perm, mstart, mlen, Mtot, Ntot, fblocks, renorm,
+                                    Xt, pt_start, items, aux, part, part_eta, status, stream);
 }
 
 namespace {

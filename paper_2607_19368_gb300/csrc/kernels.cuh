@@ -92,10 +92,13 @@ int launch_identity(const void* X, int x_dtype, int64_t B, int64_t N, int d, int
                     float* Xt, int32_t* pos, int32_t* tok2macro, cudaStream_t stream);
 size_t agg_item_capacity(int64_t Mtot, int64_t Ntot);
 size_t agg_part_capacity(int64_t Ntot);
+// Integers of the aggregation's auxiliary area (counts, block totals, CTA
+// ranges, list of macro-tokens spanning several work items).
+size_t agg_aux_ints(int64_t Mtot, int64_t Ntot);
 int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* perm,
                      const int* mstart, const int* mlen, int64_t Mtot, int64_t Ntot, int renorm,
-                     float* Xt, int* it_start, int* pt_start, int2* items, int* counts,
-                     float* part, float* part_eta, int* status, cudaStream_t stream);
+                     float* Xt, int* pt_start, int2* items, int* aux, float* part,
+                     float* part_eta, int* status, cudaStream_t stream);
 int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,
                         int nprob, float* score, cudaStream_t stream);
 }  // namespace sls

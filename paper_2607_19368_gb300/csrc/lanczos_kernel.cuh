@@ -744,12 +744,13 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     int pp = 0;
     for (int p = gi; p < nprob; p += ngroups, ++pp) {
       bool ok = false;
-      for (unsigned it = 0; it < (1u << 26); ++it) {
+      const long long t0 = clock64();
+      for (unsigned it = 0;; ++it) {
         if (s_go == pp + 1) {
           ok = true;
           break;
         }
-        __nanosleep(64);
+        if ((it & 63) == 63 && clock64() - t0 > SLS_WAIT_CYCLES) break;
       }
       if (!ok) {
         lz_fail(status, &s_err);
@@ -765,14 +766,17 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       for (int pass = 0; pass < r && !stop; ++pass) {
         if (pass > 0) {
           const int need = pp * 256 + pass;
+          // poll without sleeping: the ring refill of the next pass starts
+          // as soon as the compute warps open it
           bool open = false;
-          for (unsigned it = 0; it < (1u << 26); ++it) {
+          const long long t0 = clock64();
+          for (unsigned it = 0;; ++it) {
             if (s_halt) break;
             if (s_pass >= need) {
               open = true;
               break;
             }
-            __nanosleep(32);
+            if ((it & 63) == 63 && clock64() - t0 > SLS_WAIT_CYCLES) break;
           }
           if (!open) {
             if (!s_halt) lz_fail(status, &s_err);

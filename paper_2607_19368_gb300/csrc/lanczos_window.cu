@@ -66,10 +66,11 @@ SLS_DEV double warp_sum_d(double v) {
 }
 
 // Transposed butterfly on float64: lane l ends with the sum over all lanes of
-// v[l] (32 values per lane, 31 exchanges).
-SLS_DEV double transpose_reduce_d(double (&v)[32], int lane) {
+// v[l % RV] (RV in {16, 32}; RV - 1 exchanges, then one more for RV = 16).
+template <int RV>
+SLS_DEV double transpose_reduce_d(double (&v)[RV], int lane) {
 #pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
+  for (int o = RV / 2; o >= 1; o >>= 1) {
     const bool up = (lane & o) != 0;
 #pragma unroll
     for (int t = 0; t < o; ++t) {
@@ -78,7 +79,10 @@ SLS_DEV double transpose_reduce_d(double (&v)[32], int lane) {
       v[t] = keep + __shfl_xor_sync(FULL, send, o);
     }
   }
-  return v[0];
+  double r = v[0];
+#pragma unroll
+  for (int o = RV; o < 32; o <<= 1) r += __shfl_xor_sync(FULL, r, o);
+  return r;
 }
 
 // Transposed butterfly: lane l ends with the sum over all lanes of v[l % NV]
@@ -101,7 +105,7 @@ SLS_DEV dfloat transpose_reduce(dfloat (&v)[NV], int lane) {
   return r;
 }
 
-template <int NV>
+template <int NV, int RV>
 __global__ void __launch_bounds__(LW_MAX_WARPS * 32)
 lanczos_window_kernel(LanczosBatch bt) {
   constexpr int CU = (NV <= 16) ? 2 : 1;  // columns in flight per lane
@@ -178,10 +182,10 @@ lanczos_window_kernel(LanczosBatch bt) {
     z = z - a * q - bprev * qprev;
     // full re-orthogonalisation: two classical Gram-Schmidt passes
     for (int pass = 0; pass < 2; ++pass) {
-      double pr[LW_MAXR];
+      double pr[RV];
 #pragma unroll
-      for (int k = 0; k < LW_MAXR; ++k) pr[k] = (k <= j && mine) ? Qs[lane * R1 + k] * z : 0.0;
-      const double c = transpose_reduce_d(pr, lane);  // lane k: (Q^T z)_k
+      for (int k = 0; k < RV; ++k) pr[k] = (k <= j && mine) ? Qs[lane * R1 + k] * z : 0.0;
+      const double c = transpose_reduce_d<RV>(pr, lane);  // lane k (mod RV): (Q^T z)_k
       double corr = 0.0;
       for (int k = 0; k <= j; ++k) {
         const double ck = __shfl_sync(FULL, c, k);
@@ -276,15 +280,21 @@ int launch_lanczos_window(const LanczosBatch& bt, cudaStream_t stream) {
   if (warps < 1) warps = 1;
   const size_t smem = per_warp * warps;
   const int blocks = (bt.nprob_max + warps - 1) / warps;
-  if (bt.nmax <= 16) {
-    SLS_CUDA_TRY(cudaFuncSetAttribute(lanczos_window_kernel<16>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    lanczos_window_kernel<16><<<blocks, warps * 32, smem, stream>>>(bt);
-  } else {
-    SLS_CUDA_TRY(cudaFuncSetAttribute(lanczos_window_kernel<32>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    lanczos_window_kernel<32><<<blocks, warps * 32, smem, stream>>>(bt);
-  }
+#define SLS_LW_LAUNCH(NV, RV)                                                               \
+  do {                                                                                      \
+    SLS_CUDA_TRY(cudaFuncSetAttribute(lanczos_window_kernel<NV, RV>,                        \
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)); \
+    lanczos_window_kernel<NV, RV><<<blocks, warps * 32, smem, stream>>>(bt);                 \
+  } while (0)
+  if (bt.nmax <= 16 && bt.r <= 16)
+    SLS_LW_LAUNCH(16, 16);
+  else if (bt.nmax <= 16)
+    SLS_LW_LAUNCH(16, 32);
+  else if (bt.r <= 16)
+    SLS_LW_LAUNCH(32, 16);
+  else
+    SLS_LW_LAUNCH(32, 32);
+#undef SLS_LW_LAUNCH
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
