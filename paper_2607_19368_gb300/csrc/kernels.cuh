@@ -25,7 +25,8 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
                                   cudaStream_t stream, int* status);
 
 // ---- Lanczos (Algorithm 2) --------------------------------------------------
-// Row stride (in float2) of the double-float basis Q: r rounded up to even.
+// Row stride (in float2) of the double-float basis Q: r rounded up to even,
+// so every basis row starts on a 16-byte boundary.
 __host__ __device__ inline int q_ld(int r) { return (r + 1) & ~1; }
 
 // A batch of independent problems, problem p owning rows

@@ -37,8 +37,8 @@
 // alternate direction so each starts on the rows the previous one left in
 // L2.  Vectors are double-float (two float32), every sum over N or D is
 // compensated, reductions have a fixed order (bit-reproducible runs).
-// Barriers and waits give up after a bounded number of polls and report
-// SLS_ERR_TIMEOUT through the status word.
+// Barriers and waits poll without sleeping and give up after about a second
+// of clock cycles, reporting SLS_ERR_TIMEOUT through the status word.
 //
 // The kernel is a template over GPT (float4 column groups of Phi per compute
 // thread) and KT (32-wide tiles of the basis index k < r per lane); each
@@ -59,7 +59,6 @@ constexpr int LZ_CT = LZ_CW * 32;         // compute threads
 constexpr int LZ_THREADS = LZ_CT + 32;    // plus one copy warp
 constexpr unsigned BAR_COMPUTE = 1;       // named barrier: the compute warps
 
-// leading dimension (float2) of the basis rows: even, so rows are 16-byte aligned
 
 // Per-group scratch layout (byte offsets), identical on host and device.
 struct LzLayout {
