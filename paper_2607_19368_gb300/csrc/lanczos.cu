@@ -2,8 +2,10 @@
 // lanczos_kernel.cuh, plus the planning and launch of the Lanczos kernel.
 //
 // The r x r (r <= 128) tridiagonal T is solved on the device: Ritz values by
-// Sturm-count multisection (one warp per eigenvalue, 32 shifts per round,
-// float64), eigenvectors by inverse iteration with partial-pivoting LU, with
+// Sturm-count multisection (a CTA of 256 shifts per eigenvalue when the
+// launch has few, one warp of 32 shifts when it has many; double-float
+// recurrence), eigenvectors by inverse iteration with
+// partial-pivoting LU (double-float), with
 // modified Gram-Schmidt inside clusters of nearly equal eigenvalues.  Finally
 // U = Q S.
 #include "lanczos_kernel.cuh"
@@ -20,10 +22,12 @@ namespace {
 // a serial recurrence pays at every step.
 // ----------------------------------------------------------------------------
 
+// Ritz values of few problems: one CTA per eigenvalue, 256 shifts per round
+// (fewer, longer rounds: the faster form when the launch has few eigenvalues)
 constexpr int EIG_THREADS = 256;  // shifts per multisection round
 
 __global__ void __launch_bounds__(EIG_THREADS)
-tridiag_eigvals_kernel(LanczosBatch bt) {
+tridiag_eigvals_cta_kernel(LanczosBatch bt) {
   __shared__ float2 sa[SLS_MAX_R], sb2[SLS_MAX_R];
   __shared__ int s_first[EIG_THREADS / 32];
   __shared__ double s_lo, s_hi, s_sc;
@@ -99,6 +103,84 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
     __syncthreads();
   }
   if (tid == 0) theta[m] = (0.5 * (s_lo + s_hi)) / sc;
+}
+
+constexpr int EIG_WARPS = 8;  // eigenvalues per CTA (one warp each)
+
+// Ritz values of many problems: one warp per eigenvalue, multisection on
+// Sturm counts (32 shifts per round, one per lane; a ballot finds the
+// subinterval that holds the wanted eigenvalue), the warps of a CTA sharing
+// the problem's scaled T.
+__global__ void __launch_bounds__(EIG_WARPS * 32)
+tridiag_eigvals_kernel(LanczosBatch bt) {
+  __shared__ float2 sa[SLS_MAX_R], sb2[SLS_MAX_R];
+  __shared__ double s_glo, s_ghi;
+  const int p = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int nprob = bt.nprob_max;
+  if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
+  if (p >= nprob) return;
+  const int r = bt.r;
+  const int n = bt.r_eff[p];
+  const int m = blockIdx.x * EIG_WARPS + warp;  // descending index of this warp's value
+  double* theta = bt.theta + (size_t)p * r;
+  const double* a = bt.alpha + (size_t)p * r;
+  const double* b = bt.beta + (size_t)p * r;
+  if (warp == 0) {
+    // Gershgorin interval
+    double glo = DBL_MAX, ghi = -DBL_MAX;
+    for (int i = lane; i < n; i += 32) {
+      const double bl = (i > 0) ? fabs(b[i - 1]) : 0.0;
+      const double br = (i < n - 1) ? fabs(b[i]) : 0.0;
+      glo = fmin(glo, a[i] - bl - br);
+      ghi = fmax(ghi, a[i] + bl + br);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      glo = fmin(glo, __shfl_xor_sync(0xffffffffu, glo, o));
+      ghi = fmax(ghi, __shfl_xor_sync(0xffffffffu, ghi, o));
+    }
+    if (lane == 0) {
+      s_glo = glo;
+      s_ghi = ghi;
+    }
+  }
+  __syncthreads();
+  // a power-of-two scale that maps the interval into [-1, 1] (exact)
+  const double glo = s_glo, ghi = s_ghi;
+  const double big = fmax(fabs(glo), fabs(ghi));
+  int ex = 0;
+  frexp(big > 0.0 ? big : 1.0, &ex);
+  const double sc = ldexp(1.0, -ex);
+  for (int i = tid; i < n; i += EIG_WARPS * 32) {
+    sa[i] = f2(df_from_double(a[i] * sc));
+    if (i < n - 1) {
+      const double bs = b[i] * sc;
+      sb2[i] = f2(df_from_double(bs * bs));
+    }
+  }
+  __syncthreads();
+  if (m >= r) return;
+  if (m >= n) {
+    if (lane == 0) theta[m] = 0.0;
+    return;
+  }
+  const double pad = 0x1p-40 * fmax(fabs(glo * sc), fabs(ghi * sc)) + 0x1p-100;
+  double lo = glo * sc - pad, hi = ghi * sc + pad;
+  const int k = n - 1 - m;  // ascending index of the wanted eigenvalue
+  for (int round = 0; round < 40; ++round) {
+    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-120) break;
+    const double step = (hi - lo) / 33.0;
+    const double x = lo + step * (double)(lane + 1);
+    const int c = sturm_count(sa, sb2, n, df_from_double(x));
+    // count(x_t) is non-decreasing in t: the eigenvalue lies in (x_{f-1}, x_f]
+    const unsigned ball = __ballot_sync(0xffffffffu, c > k);
+    const int f = ball ? __ffs(ball) - 1 : 32;
+    const double nhi = (f < 32) ? lo + step * (double)(f + 1) : hi;
+    const double nlo = (f > 0) ? lo + step * (double)f : lo;
+    lo = nlo;
+    hi = nhi;
+  }
+  if (lane == 0) theta[m] = (0.5 * (lo + hi)) / sc;
 }
 
 // ----------------------------------------------------------------------------
@@ -455,7 +537,12 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
 int launch_tridiag_eigen(const LanczosBatch& bt, cudaStream_t stream, bool values_done) {
   dim3 grid(bt.r, bt.nprob_max);
   if (!values_done) {
-    tridiag_eigvals_kernel<<<grid, EIG_THREADS, 0, stream>>>(bt);
+    if ((int64_t)bt.r * bt.nprob_max <= 1024) {
+      tridiag_eigvals_cta_kernel<<<grid, EIG_THREADS, 0, stream>>>(bt);
+    } else {
+      dim3 vgrid((bt.r + EIG_WARPS - 1) / EIG_WARPS, bt.nprob_max);
+      tridiag_eigvals_kernel<<<vgrid, EIG_WARPS * 32, 0, stream>>>(bt);
+    }
     SLS_LAUNCH_CHECK();
   }
   if (bt.r <= EIGW_MAXR) {
