@@ -274,6 +274,7 @@ struct CompressWs {
   int64_t* lz_q1off;
   int* nspec;
   float* score;
+  float* score_part;  // window-score partial sums (adaptive backend)
   int32_t* route;  // spectral flag per problem
   float* Phi;
   float2* Q;
@@ -402,6 +403,11 @@ int validate_config(const sls_config_t* c) {
   if (c->pos_mode < 0 || c->pos_mode > 1) return SLS_ERR_INVALID_ARG;
   if (c->preserve_first < 0 || c->preserve_last < 0) return SLS_ERR_INVALID_ARG;
   return SLS_OK;
+}
+
+size_t score_bytes(const CompressPlan& P, int d, int backend) {
+  if (backend != SLS_BACKEND_ADAPTIVE) return 0;
+  return sls_align256(score_part_floats(P.nprob, P.nmax, d) * sizeof(float));
 }
 
 size_t part_bytes(int64_t toks, int d) {
@@ -598,7 +604,7 @@ size_t sls_compress_workspace_size(const sls_config_t* cfg, int64_t B, int64_t N
   if (make_plan(cfg, B, N, &P) != SLS_OK) return 0;
   CompressWs W;
   carve(P, nullptr, &W);
-  return W.total + part_bytes(B * N, d);
+  return W.total + part_bytes(B * N, d) + score_bytes(P, d, cfg->backend);
 }
 
 int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B, int64_t N, int d,
@@ -626,12 +632,15 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   }
   CompressWs W;
   carve(P, workspace, &W);
-  const size_t need = W.total + part_bytes(B * N, d);
+  const size_t need = W.total + part_bytes(B * N, d) + score_bytes(P, d, cfg->backend);
   if (!workspace || workspace_bytes < need) return SLS_ERR_WORKSPACE;
   {
     Carver tail((char*)workspace + W.total);
     W.part = tail.take<float>(agg_part_capacity(B * N) * (size_t)d);
     W.part_eta = tail.take<float>(agg_part_capacity(B * N));
+    W.score_part = (cfg->backend == SLS_BACKEND_ADAPTIVE)
+                       ? tail.take<float>(score_part_floats(P.nprob, P.nmax, d))
+                       : nullptr;
   }
   SLS_CUDA_TRY(cudaMemsetAsync(W.status, 0, 256, s));
   const int nprob = (int)P.nprob;
@@ -650,7 +659,8 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   if (cfg->backend == SLS_BACKEND_ADAPTIVE) {
     mode = 2;
     if (cfg->rho < 16.0 &&
-        (st = launch_window_score(X, x_dtype, d, ldx, W.probs, nprob, W.score, s)) != SLS_OK)
+        (st = launch_window_score(X, x_dtype, d, ldx, W.probs, nprob, P.nmax, W.score_part,
+                                  W.score, s)) != SLS_OK)
       return st;
   }
   double tau = cfg->tau;

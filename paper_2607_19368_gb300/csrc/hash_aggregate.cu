@@ -1333,7 +1333,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
   __shared__ uint64_t fullb[AGR_MAX_STAGES], emptyb[AGR_MAX_STAGES];
   __shared__ AggDesc dring[AGR_MAX_STAGES + 2];
   __shared__ float shq[2][AGR_CW][AGG_CH];
-  __shared__ float sh[AGR_CW];
+  __shared__ float shm[2][AGR_CW];  // per-warp |member sum|^2 of the item
   __shared__ volatile int s_abort;
   const int DQ = S + 2;
   const int i0 = cta_first[blockIdx.x], i1 = cta_first[blockIdx.x + 1];
@@ -1468,6 +1468,15 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
         }
         ++consumed;
       }
+      // this warp's share of |sum of the members|^2, published with the
+      // item-end barrier (the renorm needs no barrier of its own)
+      {
+        float msq = 0.f;
+#pragma unroll
+        for (int e = 0; e < NV * V; ++e) msq = fmaf(acc[e], acc[e], msq);
+        msq = warp_sum_f(msq);
+        if (lane == 0) shm[k & 1][cw] = msq;
+      }
       if (named_sync_or(AGR_BAR, AGR_CT, !ok)) break;
       // sum of member norms (every warp forms the same total)
       float eta = 0.f;
@@ -1487,28 +1496,15 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
       if (D.ps < 0) {
         dst = Xt + (int64_t)D.m * d;
         if (D.len > 1) {
+          // mean = sum / len, rescaled to the mean member norm
           const float inv = 1.0f / (float)D.len;
-          float sq = 0.f;
-#pragma unroll
-          for (int qv = 0; qv < NV; ++qv) {
-            const int c0 = (ct + qv * AGR_CT) * V;
-            if (c0 < d)
-#pragma unroll
-              for (int e = 0; e < V; ++e) {
-                acc[qv * V + e] *= inv;
-                sq = fmaf(acc[qv * V + e], acc[qv * V + e], sq);
-              }
-          }
+          scale = inv;
           if (renorm) {
-            sq = warp_sum_f(sq);
-            if (lane == 0) sh[cw] = sq;
-            named_sync(AGR_BAR, AGR_CT);
             float tot = 0.f;
 #pragma unroll
-            for (int w = 0; w < AGR_CW; ++w) tot += sh[w];
-            named_sync(AGR_BAR, AGR_CT);
-            const float nrm = sqrtf(tot);
-            if (nrm >= 1e-30f) scale = (eta * inv) / nrm;
+            for (int w = 0; w < AGR_CW; ++w) tot += shm[k & 1][w];
+            const float nrm = sqrtf(tot) * inv;
+            if (nrm >= 1e-30f) scale = inv * ((eta * inv) / nrm);
           }
         }
       } else {
@@ -1533,31 +1529,45 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
 // ============================================================================
 
 // score = (1/L) sum_i cos(x_i, c) with c the window centroid; computed in one
-// pass as (sum_i x_i/|x_i|) . (sum_i x_i) / (L |sum_i x_i|).  Zero rows add 0.
-// Rows are gathered in batches of agg_batch<NV>(); each row's |x|^2 is reduced
-// from the same registers (per warp, then across warps through a
-// double-buffered shared array, one barrier per batch), so X is read once.
+// pass over X as (sum_i x_i/|x_i|) . (sum_i x_i) / (L |sum_i x_i|).  Zero rows
+// add 0.  Every window is cut into parts of SCORE_PR rows (so that a batch of
+// windows spreads evenly over the SMs); a CTA takes a part at a time, gathers
+// its rows in batches of agg_batch<NV>(), reduces each row's |x|^2 from the
+// same registers (per warp, then across warps through a double-buffered
+// shared array, one barrier per batch) and writes the part's sums of x and of
+// x/|x|; window_score_combine_kernel adds a window's parts and forms the
+// score.
+constexpr int SCORE_PR = 512;  // rows per part
+
+__host__ __device__ inline int score_parts(int64_t nmax) {
+  return (int)((nmax + SCORE_PR - 1) / SCORE_PR);
+}
+
 template <typename T, int NV>
 __global__ void __launch_bounds__(AGG_T, 2)
 window_score_kernel(const T* __restrict__ X, int d, int64_t ldx,
-                    const ProbDesc* __restrict__ probs, int nprob, float* __restrict__ score) {
+                    const ProbDesc* __restrict__ probs, int nprob, int KP,
+                    float* __restrict__ part) {
   constexpr int V = VecOf<T>::V;
   constexpr int MB = agg_batch<NV>();
   constexpr int NW = AGG_T / 32;
-  __shared__ float sh[NW];
   __shared__ float shq[2][MB][NW];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int p = blockIdx.x; p < nprob; p += gridDim.x) {
+  const int units = nprob * KP;
+  for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    const int p = u / KP, k = u % KP;
     const ProbDesc P = probs[p];
+    const int r0 = min(P.n, k * SCORE_PR), r1 = min(P.n, r0 + SCORE_PR);
+    if (r0 >= r1) continue;
     float cs[NV * V], ns[NV * V];
 #pragma unroll
-    for (int k = 0; k < NV * V; ++k) cs[k] = ns[k] = 0.f;
+    for (int e = 0; e < NV * V; ++e) cs[e] = ns[e] = 0.f;
     int buf = 0;
-    for (int s0 = 0; s0 < P.n; s0 += MB, buf ^= 1) {
+    for (int s0 = r0; s0 < r1; s0 += MB, buf ^= 1) {
       float v[MB][NV * V];
 #pragma unroll
       for (int j = 0; j < MB; ++j) {
-        const bool live = s0 + j < P.n;
+        const bool live = s0 + j < r1;
         const T* x = X + (P.tok_row + s0 + j) * ldx;
 #pragma unroll
         for (int q = 0; q < NV; ++q) {
@@ -1566,7 +1576,7 @@ window_score_kernel(const T* __restrict__ X, int d, int64_t ldx,
             load_vec<T>(x + c0, &v[j][q * V]);
           } else {
 #pragma unroll
-            for (int k = 0; k < V; ++k) v[j][q * V + k] = 0.f;
+            for (int e = 0; e < V; ++e) v[j][q * V + e] = 0.f;
           }
         }
       }
@@ -1574,7 +1584,7 @@ window_score_kernel(const T* __restrict__ X, int d, int64_t ldx,
       for (int j = 0; j < MB; ++j) {
         float sq = 0.f;
 #pragma unroll
-        for (int k = 0; k < NV * V; ++k) sq = fmaf(v[j][k], v[j][k], sq);
+        for (int e = 0; e < NV * V; ++e) sq = fmaf(v[j][e], v[j][e], sq);
         sq = warp_sum_f(sq);
         if (lane == 0) shq[buf][j][warp] = sq;
       }
@@ -1586,21 +1596,51 @@ window_score_kernel(const T* __restrict__ X, int d, int64_t ldx,
         for (int w = 0; w < NW; ++w) t += shq[buf][j][w];
         const float inv = (t > 0.f) ? 1.0f / sqrtf(t) : 0.f;
 #pragma unroll
-        for (int k = 0; k < NV * V; ++k) {
-          cs[k] += v[j][k];
-          ns[k] = fmaf(v[j][k], inv, ns[k]);
+        for (int e = 0; e < NV * V; ++e) {
+          cs[e] += v[j][e];
+          ns[e] = fmaf(v[j][e], inv, ns[e]);
         }
       }
     }
-    float dot = 0.f, cc = 0.f;
+    float* dst = part + (size_t)u * 2 * d;
 #pragma unroll
-    for (int k = 0; k < NV * V; ++k) {
-      dot = fmaf(ns[k], cs[k], dot);
-      cc = fmaf(cs[k], cs[k], cc);
+    for (int q = 0; q < NV; ++q) {
+      const int c0 = (tid + q * AGG_T) * V;
+      if (c0 < d)
+#pragma unroll
+        for (int e = 0; e < V; e += 4) {
+          store_vec4(dst + c0 + e, cs[q * V + e], cs[q * V + e + 1], cs[q * V + e + 2],
+                     cs[q * V + e + 3]);
+          store_vec4(dst + d + c0 + e, ns[q * V + e], ns[q * V + e + 1], ns[q * V + e + 2],
+                     ns[q * V + e + 3]);
+        }
+    }
+    __syncthreads();
+  }
+}
+
+// score[p] = (sum of the parts' x / |x|) . (sum of the parts' x) / (n |sum x|)
+__global__ void __launch_bounds__(AGG_T)
+window_score_combine_kernel(int d, const ProbDesc* __restrict__ probs, int nprob, int KP,
+                            const float* __restrict__ part, float* __restrict__ score) {
+  __shared__ float sh[AGG_T / 32];
+  for (int p = blockIdx.x; p < nprob; p += gridDim.x) {
+    const int n = probs[p].n;
+    const int kp = score_parts(n);
+    float dot = 0.f, cc = 0.f;
+    for (int c = threadIdx.x; c < d; c += AGG_T) {
+      float cs = 0.f, ns = 0.f;
+      for (int k = 0; k < kp; ++k) {
+        const float* src = part + ((size_t)p * KP + k) * 2 * d;
+        cs += src[c];
+        ns += src[d + c];
+      }
+      dot = fmaf(ns, cs, dot);
+      cc = fmaf(cs, cs, cc);
     }
     dot = agg_block_sum(dot, sh);
     cc = agg_block_sum(cc, sh);
-    if (tid == 0) score[p] = (cc > 0.f) ? dot / ((float)P.n * sqrtf(cc)) : 0.f;
+    if (threadIdx.x == 0) score[p] = (cc > 0.f) ? dot / ((float)n * sqrtf(cc)) : 0.f;
     __syncthreads();
   }
 }
@@ -1804,13 +1844,15 @@ int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* 
 namespace {
 template <typename T>
 int launch_score_dtype(const void* X, int d, int64_t ldx, const ProbDesc* probs, int nprob,
-                       float* score, cudaStream_t stream) {
+                       int64_t nmax, float* part, float* score, cudaStream_t stream) {
   constexpr int V = VecOf<T>::V;
   const int nv = (d / V + AGG_T - 1) / AGG_T;
-  const int blocks = nprob < 8192 ? nprob : 8192;
-#define SLS_SCORE_NV(N)                                                          \
-  window_score_kernel<T, N><<<blocks, AGG_T, 0, stream>>>((const T*)X, d, ldx, probs, \
-                                                          nprob, score)
+  const int KP = score_parts(nmax);
+  const int64_t units = (int64_t)nprob * KP;
+  const int blocks = (int)(units < 65535 ? units : 65535);
+#define SLS_SCORE_NV(N)                                                                    \
+  window_score_kernel<T, N><<<blocks, AGG_T, 0, stream>>>((const T*)X, d, ldx, probs, nprob, \
+                                                          KP, part)
   if (nv <= 1)
     SLS_SCORE_NV(1);
   else if (nv <= 2)
@@ -1823,16 +1865,23 @@ int launch_score_dtype(const void* X, int d, int64_t ldx, const ProbDesc* probs,
     return SLS_ERR_UNSUPPORTED;
 #undef SLS_SCORE_NV
   SLS_LAUNCH_CHECK();
+  const int cb = nprob < 4096 ? nprob : 4096;
+  window_score_combine_kernel<<<cb, AGG_T, 0, stream>>>(d, probs, nprob, KP, part, score);
+  SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
 }  // namespace
 
+size_t score_part_floats(int64_t nprob, int64_t nmax, int d) {
+  return (size_t)nprob * score_parts(nmax) * 2 * (size_t)d;
+}
+
 int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,
-                        int nprob, float* score, cudaStream_t stream) {
+                        int nprob, int64_t nmax, float* part, float* score, cudaStream_t stream) {
   if (nprob <= 0) return SLS_OK;
   if (x_dtype == SLS_F32)
-    return launch_score_dtype<float>(X, d, ldx, probs, nprob, score, stream);
-  return launch_score_dtype<uint16_t>(X, d, ldx, probs, nprob, score, stream);
+    return launch_score_dtype<float>(X, d, ldx, probs, nprob, nmax, part, score, stream);
+  return launch_score_dtype<uint16_t>(X, d, ldx, probs, nprob, nmax, part, score, stream);
 }
 
 }  // namespace sls

@@ -100,6 +100,9 @@ int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* 
                      const int* mstart, const int* mlen, int64_t Mtot, int64_t Ntot, int renorm,
                      float* Xt, int* pt_start, int2* items, int* aux, float* part,
                      float* part_eta, int* status, cudaStream_t stream);
+// Redundancy score of every window (Sec. 3.6, Eq. redundancy); part holds
+// score_part_floats(nprob, nmax, d) floats of scratch.
+size_t score_part_floats(int64_t nprob, int64_t nmax, int d);
 int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,
-                        int nprob, float* score, cudaStream_t stream);
+                        int nprob, int64_t nmax, float* part, float* score, cudaStream_t stream);
 }  // namespace sls

@@ -503,9 +503,8 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
                    int groups, int g, cudaStream_t stream) {
   const LzLayout L = lz_layout(bt.nmax, bt.D, bt.r, g);
   if ((size_t)groups * L.total > scratch_bytes) return SLS_ERR_WORKSPACE;
-  // barrier words start at zero
-  for (int gi = 0; gi < groups; ++gi)
-    SLS_CUDA_TRY(cudaMemsetAsync((char*)scratch + (size_t)gi * L.total + L.bar, 0, 256, stream));
+  // barrier words of every group start at zero (one strided memset)
+  SLS_CUDA_TRY(cudaMemset2DAsync((char*)scratch + L.bar, L.total, 0, 256, groups, stream));
   const int C4 = bt.D / 4;
   const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
   const int redn = (P > 1) ? P * bt.D : 0;
