@@ -854,6 +854,183 @@ segment_grid_kernel(const ProbDesc* __restrict__ probs, const uint32_t* __restri
 }
 
 // ============================================================================
+// small problems (windows of at most 32 tokens): one warp per problem
+// ============================================================================
+
+// The same clusters, exact-length adjust, positions and causal order as
+// segment_kernel for a problem of n <= 32 tokens, held in one warp: lane s
+// holds the s-th token of the order the groups are cut from ((code, token)
+// order for spectral windows, token order for chunk windows), so every group
+// is a run of consecutive lanes.
+constexpr int SEGW_WARPS = 8;
+
+SLS_DEV unsigned long long shfl_u64(unsigned long long v, int src) {
+  return ((unsigned long long)__shfl_sync(0xffffffffu, (unsigned)(v >> 32), src) << 32) |
+         __shfl_sync(0xffffffffu, (unsigned)v, src);
+}
+
+__global__ void __launch_bounds__(SEGW_WARPS * 32)
+segment_warp_kernel(const ProbDesc* __restrict__ probs, int nprob,
+                    const uint32_t* __restrict__ codes, int pos_scheme, int pos_mode,
+                    int* __restrict__ perm, int* __restrict__ mstart, int* __restrict__ mlen,
+                    int32_t* __restrict__ pos_out, int32_t* __restrict__ tok2macro) {
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int w0 = blockIdx.x * SEGW_WARPS + (threadIdx.x >> 5);
+  const int nw = gridDim.x * SEGW_WARPS;
+  for (int p = w0; p < nprob; p += nw) {
+    const ProbDesc P = probs[p];
+    const int n = P.n, M = P.m;
+    if (n <= 0 || M <= 0) continue;
+    const bool valid = lane < n;
+    // ---- order: (code, token) for spectral windows, token order otherwise ----
+    unsigned long long key = ~0ull;
+    if (valid)
+      key = P.spectral ? (((unsigned long long)codes[P.phi_row + lane] << 5) | (unsigned)lane)
+                       : (unsigned long long)lane;
+    if (P.spectral) {
+      // bitonic sort over the 32 lanes, ascending
+#pragma unroll
+      for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+        for (int j = k >> 1; j > 0; j >>= 1) {
+          const unsigned long long o = shfl_u64(key, lane ^ j);
+          const bool up = ((lane & k) == 0);
+          const bool lower = (lane & j) == 0;
+          // the lower lane of the pair keeps the smaller key when ascending
+          const bool keep_min = (lower == up);
+          key = keep_min ? (o < key ? o : key) : (o > key ? o : key);
+        }
+      }
+    }
+    const int tok = (int)(key & 31u);
+    // ---- group of each position ----
+    int g = 0;
+    if (!P.spectral) {
+      const int q = n / M, rem = n % M;
+      g = (lane < (q + 1) * rem) ? lane / (q + 1) : rem + (lane - (q + 1) * rem) / max(q, 1);
+    } else {
+      const unsigned long long code = key >> 5;
+      const unsigned long long prevc = shfl_u64(code, max(lane - 1, 0));
+      const bool head = valid && (lane == 0 || code != prevc);
+      const unsigned hm = __ballot_sync(FULL, head);
+      const int C = __popc(hm);
+      const int cl = __popc(hm & (0xffffffffu >> (31 - lane))) - 1;  // cluster of this position
+      if (C >= M) {
+        // merge: the cluster of rank t joins group floor(t M / C)
+        g = (int)(((long long)cl * M) / C);
+      } else {
+        // split: D'Hondt seats, one guaranteed per cluster, ties to the lower
+        // code; lane c holds cluster c
+        const int cs = (lane < C) ? (int)__fns(hm, 0, lane + 1) : n;
+        const int cn = (lane + 1 < C) ? (int)__fns(hm, 0, lane + 2) : n;
+        const int size = (lane < C) ? cn - cs : 0;
+        int seats = (lane < C) ? 1 : 0;
+        for (int it = 0; it < M - C; ++it) {
+          bool el = lane < C && seats < size;
+          int num = size, den = seats + 1, idx = lane;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            const bool el2 = __shfl_xor_sync(FULL, el ? 1 : 0, o) != 0;
+            const int num2 = __shfl_xor_sync(FULL, num, o);
+            const int den2 = __shfl_xor_sync(FULL, den, o);
+            const int idx2 = __shfl_xor_sync(FULL, idx, o);
+            const long long a = (long long)num2 * den, b = (long long)num * den2;
+            const bool better = el2 && (!el || a > b || (a == b && idx2 < idx));
+            if (better) {
+              el = el2;
+              num = num2;
+              den = den2;
+              idx = idx2;
+            }
+          }
+          if (lane == idx) ++seats;
+        }
+        int gfirst = seats;  // exclusive prefix of seats: first group of each cluster
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(FULL, gfirst, o);
+          if (lane >= o) gfirst += y;
+        }
+        gfirst -= seats;
+        const int ccl = max(cl, 0);
+        const int c_start = __shfl_sync(FULL, cs, ccl);
+        const int c_size = __shfl_sync(FULL, size, ccl);
+        const int c_seats = __shfl_sync(FULL, seats, ccl);
+        const int c_g0 = __shfl_sync(FULL, gfirst, ccl);
+        const int j = lane - c_start;
+        const int q = c_size / max(c_seats, 1), rem = c_size % max(c_seats, 1);
+        g = c_g0 + ((j < (q + 1) * rem) ? j / (q + 1) : rem + (j - (q + 1) * rem) / max(q, 1));
+      }
+    }
+    if (!valid) g = M;  // past every group
+    // ---- group runs: start, end, positions ----
+    const int gp = __shfl_sync(FULL, g, max(lane - 1, 0));
+    const bool ghead = valid && (lane == 0 || g != gp);
+    const unsigned gm = __ballot_sync(FULL, ghead);
+    const int gs = valid ? (int)__fns(gm, 0, g + 1) : 32;
+    const int ge = (valid && g + 1 < M) ? (int)__fns(gm, 0, g + 2) : n;
+    int vmax = valid ? tok : -1, vmin = valid ? tok : 1 << 30, vsum = valid ? tok : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int ymax = __shfl_down_sync(FULL, vmax, o);
+      const int ymin = __shfl_down_sync(FULL, vmin, o);
+      const int ysum = __shfl_down_sync(FULL, vsum, o);
+      if (lane + o < ge) {
+        vmax = max(vmax, ymax);
+        vmin = min(vmin, ymin);
+      }
+      // a sum over [lane, ge) needs the partial of lane + o to cover
+      // [lane + o, ge) exactly: doubling steps keep that true
+      if (lane + o < ge) vsum += ysum;
+    }
+    // lower median: the member whose token has (len - 1) / 2 smaller members
+    int rank = 0;
+#pragma unroll
+    for (int o = 0; o < 32; ++o) {
+      const int t = __shfl_sync(FULL, tok, o);
+      if (o >= gs && o < ge && t < tok) ++rank;
+    }
+    const int len = ge - gs;
+    const bool ismed = valid && rank == (len - 1) / 2;
+    const unsigned medm = __ballot_sync(FULL, ismed);
+    // group g's summary moves to lane g
+    const int src = (lane < M) ? (int)__fns(gm, 0, lane + 1) : 0;
+    const int g_start = src;
+    const int g_end = __shfl_sync(FULL, ge, src);
+    const int g_len = g_end - g_start;
+    const int g_max = __shfl_sync(FULL, vmax, src);
+    const int g_min = __shfl_sync(FULL, vmin, src);
+    const int g_sum = __shfl_sync(FULL, vsum, src);
+    const unsigned g_end_mask = (g_end >= 32) ? 0xffffffffu : ((1u << g_end) - 1u);
+    const unsigned g_mask = g_end_mask & ~((1u << g_start) - 1u);
+    const int med_lane = (lane < M) ? (int)__fns(medm & g_mask, 0, 1) : 0;
+    const int g_med = __shfl_sync(FULL, tok, med_lane);
+    int rep = g_max;
+    if (pos_scheme == SLS_POS_MEDIAN) rep = g_med;
+    if (pos_scheme == SLS_POS_MEAN) rep = (2 * g_sum + g_len) / (2 * max(g_len, 1));
+    // ---- causal order of the groups: by (position, first token) ----
+    int orank = 0;
+#pragma unroll
+    for (int o = 0; o < 32; ++o) {
+      const int r2 = __shfl_sync(FULL, rep, o), m2 = __shfl_sync(FULL, g_min, o);
+      if (o < M && lane < M && (r2 < rep || (r2 == rep && m2 < g_min))) ++orank;
+    }
+    if (lane < M) {
+      const int64_t mrow = P.out0 + orank;
+      mstart[mrow] = (int)(P.tok_row + g_start);
+      mlen[mrow] = g_len;
+      pos_out[mrow] = (pos_mode == SLS_MODE_COMPACT) ? (P.out_local + orank) : (P.pos0 + rep);
+    }
+    const int my_rank = __shfl_sync(FULL, orank, min(g, 31));
+    if (valid) {
+      perm[P.tok_row + lane] = (int)(P.tok_row + tok);
+      tok2macro[P.tok_row + tok] = P.out_local + my_rank;
+    }
+  }
+}
+
+// ============================================================================
 // preserved tokens, identity
 // ============================================================================
 
@@ -1694,6 +1871,15 @@ int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int 
   if (nprob <= 0) return SLS_OK;
   const SegLayout L = seg_layout(nmax, mmax);
   const size_t stride = L.total;
+  if (nmax <= 32) {
+    // windows of at most 32 tokens: one warp per window
+    int64_t blocks = ((int64_t)nprob + SEGW_WARPS - 1) / SEGW_WARPS;
+    if (blocks > 65535) blocks = 65535;
+    segment_warp_kernel<<<(unsigned)blocks, SEGW_WARPS * 32, 0, stream>>>(
+        probs, nprob, codes, pos_scheme, pos_mode, perm, mstart, mlen, pos_out, tok2macro);
+    SLS_LAUNCH_CHECK();
+    return SLS_OK;
+  }
   if (nprob == 1 && nmax >= SEG_GRID_MIN_N && status) {
     // one large problem: spread it over a cooperative grid
     int dev = 0, sms = 0;

@@ -281,6 +281,29 @@ def test_aggregate_bit_exact_maps_one_large_problem(sls, scheme, case):
     assert np.max(np.abs(Xt.cpu().numpy() - Xt_o)) <= EMB_TOL
 
 
+@pytest.mark.parametrize("scheme", [O.POS_MAX, O.POS_MEDIAN, O.POS_MEAN])
+@pytest.mark.parametrize("N", [1, 2, 5, 16, 17, 31, 32])
+def test_aggregate_window_sized_bit_exact(sls, scheme, N):
+    """Problems of at most 32 tokens (the local backend's windows) take the
+    one-warp segment kernel: merge, split (D'Hondt, repeated sizes and ties)
+    and equal cases against the oracle, bit-exact maps and positions."""
+    g = np.random.default_rng(100 * N + scheme)
+    d = 24
+    X = (g.standard_normal((N, d)) / 5).astype(np.float32)
+    for nb in (1, 2, 3, max(1, N // 2), N):
+        codes = (g.integers(0, nb, size=N).astype(np.uint32) * np.uint32(40503)) ^ np.uint32(7)
+        C = len(set(codes.tolist()))
+        for M in sorted({1, max(1, C - 1), C, min(N, C + 1), min(N, 2 * C + 1), N}):
+            Xt_o, pos_o, t2m_o, _ = _oracle_aggregate(X.astype(np.float64), codes, M, scheme,
+                                                      True)
+            Xt, pos, t2m = sls.aggregate(torch.from_numpy(X).cuda(),
+                                         torch.from_numpy(codes.view(np.int32)).cuda(), M,
+                                         scheme, True)
+            assert np.array_equal(t2m.cpu().numpy(), t2m_o), (nb, M)
+            assert np.array_equal(pos.cpu().numpy(), pos_o), (nb, M)
+            assert np.max(np.abs(Xt.cpu().numpy() - Xt_o)) <= EMB_TOL
+
+
 def test_aggregate_bf16_large_groups(sls):
     """bf16 embeddings, duplicated tokens (one large cluster), renorm off and on."""
     w, p, prm = _workload_inputs("mistral7b", N=6000, d=512)
