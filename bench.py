@@ -151,6 +151,17 @@ class Clocks:
                 "reasons": sorted(reasons)}
 
 
+def max_over_ranks(values, world, device):
+    """The largest of each timing over all ranks (the slowest rank sets the
+    job's time); the identity on one rank."""
+    import torch
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t.tolist()]
+
+
 def lanczos_algorithmic_bytes(n_tokens, D, r):
     """Per launch: two float32 sweeps over Phi per step (8 r D bytes per token)
     plus the double-float basis traffic of the two Gram-Schmidt passes
@@ -361,10 +372,7 @@ def run_native(args, rank, world):
     phases = {name: statistics.mean(ev[k][2 * i].elapsed_time(ev[k][2 * i + 1])
                                     for k in range(args.steps))
               for i, name in enumerate(sls.PHASES)}
-    ms_t = torch.tensor([ms], device=dev)
-    if world > 1:
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms_max = float(ms_t.item())
+    ms_max = max_over_ranks([ms], world, dev)[0]
     value = world * B * N / (ms_max / 1e3)
 
     # roofline of the dominant kernel (the persistent Lanczos kernel)
@@ -460,15 +468,13 @@ def run_native(args, rank, world):
             comp.wait_stream(cps)
 
         ms_pipe = timed(pipelined, args.e2e_steps)
-        m2 = torch.tensor([ms_pipe, ms_serial], device=dev)
-        if world > 1:
-            dist.all_reduce(m2, op=dist.ReduceOp.MAX)
-        e2e = {"value": world * B * N / (float(m2[0].item()) / 1e3), "unit": UNIT,
+        m2 = max_over_ranks([ms_pipe, ms_serial], world, dev)
+        e2e = {"value": world * B * N / (m2[0] / 1e3), "unit": UNIT,
                "h2d_bytes_per_step": Xin.numel() * 2,
                "d2h_bytes_per_step": Xt.numel() * 4 + pos.numel() * 4 + t2m.numel() * 4,
                "mode": "pipelined: the copies of step k+1 in and step k out overlap the "
                        "compression of step k on a second stream (double-buffered)",
-               "serial_value": world * B * N / (float(m2[1].item()) / 1e3)}
+               "serial_value": world * B * N / (m2[1] / 1e3)}
 
     if rank != 0:
         return
