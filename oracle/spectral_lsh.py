@@ -27,6 +27,7 @@ __all__ = [
     "compress_adaptive", "compress_local", "compress_chunk", "complexity_ops",
     "CompressResult",
     "POS_MAX", "POS_MEDIAN", "POS_MEAN", "MODE_REPRESENTATIVE", "MODE_COMPACT",
+    "normalized_features",
 ]
 
 # ---------------------------------------------------------------------------
@@ -50,6 +51,7 @@ class CompressConfig:
     renorm: bool = True           # Eq. macro_embed
     lanczos_tol: float = 1e-10    # break threshold of Algorithm 2 (reading)
     window: int = 2048            # adaptive / local backend window
+    normalize: bool = False       # row-normalised operator (Sec. 3.2 variant)
     tau: float = 0.70             # fixed threshold (App. B.3)
     tau_schedule: bool = True     # compression-aware schedule (Sec. 3.6)
 
@@ -129,6 +131,22 @@ def lanczos(Phi: np.ndarray, q1: np.ndarray, r: int, tol: float = 1e-10):
         q_prev, q, b_prev = q, z / b, b
     return (np.array(alpha), np.array(beta[:max(r_eff - 1, 0)]),
             Q[:, :r_eff].copy(), r_eff)
+
+
+def normalized_features(Phi: np.ndarray):
+    """The cheap normalised operator of Sec. 3.2, diag(s)^-1 Phi (Phi^T v) with
+    row sums s = Phi (Phi^T 1), taken in its symmetric form
+    D^{-1/2} Phi Phi^T D^{-1/2} (D = diag(s)): the same eigenvalues (the two
+    are similar), eigenvectors D^{1/2}-scaled, which SimHash cannot see (a
+    positive row scale keeps every sign).  It is the unnormalised operator of
+    the rows Phi_i / sqrt(s_i); a row with s_i <= 0 has no positive mass and is
+    scaled by 0.  Returns (s, the scaled rows)."""
+    Phi = np.asarray(Phi, dtype=np.float64)
+    s = Phi @ Phi.sum(axis=0)
+    w = np.zeros_like(s)
+    pos = s > 0
+    w[pos] = 1.0 / np.sqrt(s[pos])
+    return s, Phi * w[:, None]
 
 
 # ---------------------------------------------------------------------------
@@ -370,14 +388,19 @@ def _region(N: int, cfg: CompressConfig) -> Tuple[int, int, int]:
 
 def spectral_groups(Xc: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray,
                     q1: np.ndarray, r: int, bits: int, M: int, tol: float = 1e-10,
-                    phi32: bool = True):
+                    phi32: bool = True, normalize: bool = False):
     """Algorithm 1 on one token set: features, Lanczos, Ritz vectors, SimHash,
     clusters and the exact-length adjustment.  Group members are indices into
     Xc.  Phi is rounded to float32 before Lanczos when phi32 (the precision
-    the feature matrix is stored in)."""
+    the feature matrix is stored in); with normalize, Lanczos runs on the
+    row-normalised operator (normalized_features), rounded likewise."""
     Phi = rff_features(Xc, W, b)
     if phi32:
         Phi = Phi.astype(np.float32).astype(np.float64)
+    if normalize:
+        Phi = normalized_features(Phi)[1]
+        if phi32:
+            Phi = Phi.astype(np.float32).astype(np.float64)
     alpha, beta, Q, r_eff = lanczos(Phi, q1[:Xc.shape[0]], r, tol)
     theta, S, U = ritz_pairs(alpha, beta, Q)
     codes = simhash(U.astype(np.float32), R[:bits, :r_eff])
@@ -401,7 +424,7 @@ def compress_global(X: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray,
     M = target_count(Nc, cfg.rho)
     bits = cfg.bits if cfg.bits > 0 else auto_bits(Nc, cfg.rho)
     groups, info = spectral_groups(X[pf:N - pl], W, b, R, q1, cfg.r, bits, M,
-                                   cfg.lanczos_tol)
+                                   cfg.lanczos_tol, normalize=cfg.normalize)
     res = _assemble(X, pf, pl, [g + pf for g in groups], cfg)
     res.info.update(info)
     res.info.update({"M_star": M, "bits": bits})
@@ -539,7 +562,7 @@ def _windowed(X: np.ndarray, W: np.ndarray, b: np.ndarray, R: np.ndarray,
         if sp:
             bits = cfg.bits if cfg.bits > 0 else auto_bits(L, cfg.rho)
             gs, inf = spectral_groups(Xc[s:e], W, b, R, q1[s:e], cfg.r, bits, m,
-                                      cfg.lanczos_tol)
+                                      cfg.lanczos_tol, normalize=cfg.normalize)
             r_effs.append(inf["r_eff"])
         else:
             gs = chunk_groups(L, m)

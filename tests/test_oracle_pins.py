@@ -573,3 +573,47 @@ def test_local_backend_w16_invariants():
             mem = np.nonzero(res.tok2macro == m)[0]
             assert mem.min() // 16 == mem.max() // 16
         assert all(1 <= k <= 16 for k in res.info["r_eff"])
+
+
+def test_normalized_operator_pins():
+    """The row-normalised operator (Sec. 3.2 variant) against what fixes it:
+    D^{-1/2} K D^{-1/2} with D = diag(K 1) has eigenvalue exactly 1 with
+    eigenvector D^{1/2} 1 (K (1) = D 1), its largest for a kernel with positive
+    entries; its spectrum is that of diag(s)^-1 K (similar matrices); Lanczos
+    on the scaled rows finds theta_1 = 1; positive row scales leave SimHash
+    codes unchanged."""
+    w = WL.scaled(WL.WORKLOADS["tiny"], N=200)
+    p = WL.make_prompt(w)
+    prm = WL.params_for(w)
+    Phi = O.rff_features(p.x_f64(), prm.w_f64(), prm.b)
+    K = Phi @ Phi.T
+    s, Phin = O.normalized_features(Phi)
+    assert np.allclose(s, K.sum(axis=1), rtol=1e-12)
+    assert np.all(K > 0) and np.all(s > 0)
+    S = Phin @ Phin.T
+    assert np.allclose(S, K / np.sqrt(np.outer(s, s)), rtol=1e-11, atol=0)
+    ev, V = np.linalg.eigh(S)
+    assert abs(ev[-1] - 1.0) < 1e-12
+    u = np.sqrt(s) / np.linalg.norm(np.sqrt(s))
+    assert abs(abs(V[:, -1] @ u) - 1.0) < 1e-10
+    evP = np.sort(np.linalg.eigvals(K / s[:, None]).real)
+    assert np.allclose(evP, np.sort(ev), atol=1e-11)
+    a, be, Q, k = O.lanczos(Phin, prm.q1[:200], 16)
+    th, S_, U = O.ritz_pairs(a, be, Q)
+    assert abs(th[0] - 1.0) < 1e-10
+    g = np.random.default_rng(3)
+    U32 = U.astype(np.float32)
+    scale = (g.random(U.shape[0]) + 0.5).astype(np.float32)
+    R = prm.R[:8, :k]
+    assert np.array_equal(O.simhash(U32, R), O.simhash(U32 * scale[:, None], R))
+
+
+def test_normalized_compress_invariants():
+    w = WL.WORKLOADS["tiny"]
+    p = WL.make_prompt(w)
+    prm = WL.params_for(w)
+    cfg = O.CompressConfig(rho=w.rho, D=w.D, r=w.r, bits=w.bits,
+                           preserve_last=w.preserve_last, normalize=True)
+    res = O.compress_global(p.x_f64(), prm.w_f64(), prm.b, prm.R, prm.q1, cfg)
+    _check_result(res, w.N, O.target_count(w.N - 12, w.rho) + 12, 0, 12)
+    assert abs(res.info["theta"][0] - 1.0) < 1e-6
