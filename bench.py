@@ -52,6 +52,8 @@ def parse():
                     choices=["qwen7b", "qwen14b", "mistral7b", "adaptive", "local"])
     ap.add_argument("--rho", type=float, default=None,
                     help="compression ratio (default: the workload's)")
+    ap.add_argument("--normalize", action="store_true",
+                    help="row-normalised operator (the paper's untested Sec. 3.2 variant)")
     ap.add_argument("--cpu-sample", type=int, default=4096,
                     help="tokens of the prompt the CPU oracle compresses per baseline step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -299,14 +301,15 @@ def run_native(args, rank, world):
     if adaptive:
         cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=w.D, r=w.r, bits=w.bits,
                               window=w.window, preserve_first=w.preserve_first,
-                              preserve_last=w.preserve_last)
+                              preserve_last=w.preserve_last, normalize=int(args.normalize))
     elif local:
         cfg = sls.Config.make(backend=sls.BACKEND_LOCAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
                               window=w.window, preserve_first=w.preserve_first,
-                              preserve_last=w.preserve_last)
+                              preserve_last=w.preserve_last, normalize=int(args.normalize))
     else:
         cfg = sls.Config.make(backend=sls.BACKEND_GLOBAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
-                              preserve_first=w.preserve_first, preserve_last=w.preserve_last)
+                              preserve_first=w.preserve_first, preserve_last=w.preserve_last,
+                              normalize=int(args.normalize))
     B, N, d = w.batch, w.N, w.d
     M = sls.output_count(cfg, N)
     ws = sls.Workspace(cfg, B, N, d, dev)
@@ -486,6 +489,8 @@ def run_native(args, rank, world):
              "inputs": "bf16 embeddings and Omega; float32 Phi; double-float Lanczos vectors"}
     if windowed(w):
         extra.update({"spectral_windows": n_spec, "spectral_tokens": lz_tokens})
+    if args.normalize:
+        extra["operator"] = "row-normalised (Sec. 3.2 variant, symmetric form)"
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,

@@ -92,6 +92,8 @@ typedef struct sls_config {
   int window;           /* adaptive / local backend window length              */
   double tau;           /* fixed redundancy threshold (used if !tau_schedule)  */
   int tau_schedule;     /* 1: tau(rho) = clamp(0.75 - 0.05 log2 rho, .55, .70)  */
+  int normalize;        /* 1: row-normalised operator (Sec. 3.2), see
+                           sls_feature_normalize                               */
 } sls_config_t;
 
 /*
@@ -150,6 +152,23 @@ int sls_feature_map_batched(const void* X, int64_t nb, int64_t rows,
                             const void* W, const float* b, int D, float* Phi,
                             const int32_t* live, int nwin, int win,
                             void* stream);
+
+/*
+ * The row-normalised operator of Sec. 3.2, diag(s)^-1 Phi (Phi^T v) with the
+ * estimated row sums s = Phi (Phi^T 1), in the symmetric form Lanczos needs:
+ * D^{-1/2} Phi Phi^T D^{-1/2} (D = diag(s); same eigenvalues, eigenvectors
+ * D^{1/2}-scaled, which leaves every SimHash code unchanged) -- i.e. the rows
+ * of Phi scaled in place by 1 / sqrt(s_i) (by 0 where s_i <= 0).
+ *   Phi: N x D floats (device, in place); s_hat (may be NULL): N doubles
+ *   (device, output); workspace: sls_feature_normalize_workspace_size(N, D)
+ *   device bytes.  Column sums and row dots are compensated (double-float);
+ *   each scaled element is rounded once from its float64 product.
+ * Errors: INVALID_ARG for bad sizes or NULL pointers, WORKSPACE if the
+ * workspace is too small.
+ */
+size_t sls_feature_normalize_workspace_size(int64_t N, int D);
+int sls_feature_normalize(float* Phi, int64_t N, int D, double* s_hat,
+                          void* workspace, size_t workspace_bytes, void* stream);
 
 /* Device workspace bytes needed by sls_lanczos_topr for one problem. */
 size_t sls_lanczos_workspace_size(int64_t N, int D, int r);

@@ -21,7 +21,7 @@ __all__ = [
     "SLS_OK", "SLS_F32", "SLS_BF16", "POS_MAX", "POS_MEDIAN", "POS_MEAN",
     "MODE_REPRESENTATIVE", "MODE_COMPACT", "BACKEND_GLOBAL", "BACKEND_ADAPTIVE",
     "BACKEND_CHUNK", "BACKEND_LOCAL", "Config", "SLSError", "lib", "lib_path", "feature_map",
-    "feature_map_batched",
+    "feature_map_batched", "feature_normalize",
     "lanczos_topr", "simhash", "aggregate", "compress", "output_count",
     "compress_workspace_size", "workspace_status", "EXPORTED", "PHASES",
     "set_phase_events", "launch_count", "Workspace",
@@ -57,15 +57,17 @@ class Config(ctypes.Structure):
         ("pos_mode", ctypes.c_int), ("renorm", ctypes.c_int),
         ("lanczos_tol", ctypes.c_double), ("window", ctypes.c_int),
         ("tau", ctypes.c_double), ("tau_schedule", ctypes.c_int),
+        ("normalize", ctypes.c_int),
     ]
 
     @classmethod
     def make(cls, backend=BACKEND_GLOBAL, rho=4.0, D=256, r=16, bits=0, preserve_first=0,
              preserve_last=12, pos_scheme=POS_MAX, pos_mode=MODE_REPRESENTATIVE, renorm=1,
-             lanczos_tol=1e-10, window=2048, tau=0.70, tau_schedule=1) -> "Config":
+             lanczos_tol=1e-10, window=2048, tau=0.70, tau_schedule=1,
+             normalize=0) -> "Config":
         return cls(backend, float(rho), D, r, bits, preserve_first, preserve_last, pos_scheme,
                    pos_mode, int(renorm), float(lanczos_tol), window, float(tau),
-                   int(tau_schedule))
+                   int(tau_schedule), int(normalize))
 
 
 class _Params(ctypes.Structure):
@@ -84,6 +86,8 @@ EXPORTED = {
     "sls_status_string": (ctypes.c_char_p, [_i32]),
     "sls_version": (_i32, []),
     "sls_feature_map": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _vp, _i32, _vp, _vp]),
+    "sls_feature_normalize_workspace_size": (ctypes.c_size_t, [_i64, _i32]),
+    "sls_feature_normalize": (_i32, [_vp, _i64, _i32, _vp, _vp, ctypes.c_size_t, _vp]),
     "sls_feature_map_batched": (_i32, [_vp, _i64, _i64, _i64, _i32, _i64, _vp, _vp, _i32, _vp,
                                        _vp, _i32, _i32, _vp]),
     "sls_lanczos_workspace_size": (_sz, [_i64, _i32, _i32]),
@@ -199,6 +203,22 @@ def feature_map_batched(X: torch.Tensor, W: torch.Tensor, b: torch.Tensor, rows:
                                        win, _stream(X))
     _check("sls_feature_map_batched", st)
     return out
+
+
+def feature_normalize(Phi: torch.Tensor):
+    """The row-normalised operator of Sec. 3.2 in its symmetric form: the rows
+    of Phi (N x D float32, in place) scaled by 1 / sqrt(s_i) with
+    s = Phi (Phi^T 1).  Returns s (N float64)."""
+    _need_cuda(Phi)
+    assert Phi.dtype == torch.float32 and Phi.is_contiguous()
+    N, D = Phi.shape
+    s = torch.empty(N, dtype=torch.float64, device=Phi.device)
+    L = lib()
+    nbytes = L.sls_feature_normalize_workspace_size(N, D)
+    ws = _workspace(max(nbytes, 256), Phi.device)
+    _check("sls_feature_normalize",
+           L.sls_feature_normalize(_ptr(Phi), N, D, _ptr(s), _ptr(ws), nbytes, _stream(Phi)))
+    return s
 
 
 def lanczos_topr(Phi: torch.Tensor, q1: torch.Tensor, r: int, tol: float = 1e-10):

@@ -263,6 +263,7 @@ struct CompressPlan {
   int lz_groups, lz_g;
   int seg_slots;
   int64_t k_chunk;
+  int normalize;
 };
 
 struct CompressWs {
@@ -275,6 +276,7 @@ struct CompressWs {
   int* nspec;
   float* score;
   float* score_part;  // window-score partial sums (adaptive backend)
+  float2* norm_scratch;  // row-normalised operator: column sums
   int32_t* route;  // spectral flag per problem
   float* Phi;
   float2* Q;
@@ -317,6 +319,7 @@ int make_plan(const sls_config_t* c, int64_t B, int64_t N, CompressPlan* P,
   P->D = c->D;
   P->r = c->r;
   P->k_chunk = chunk_k(c->rho);
+  P->normalize = c->normalize ? 1 : 0;
   if (c->backend == SLS_BACKEND_CHUNK) {
     P->Mstar = (R.Nc + P->k_chunk - 1) / P->k_chunk;
     P->bud = Budgets{1, R.Nc, R.Nc, P->Mstar, P->Mstar, 0};
@@ -366,6 +369,10 @@ void carve(const CompressPlan& P, void* ws, CompressWs* W) {
   W->score = cv.take<float>(np);
   W->route = cv.take<int>(np);
   W->Phi = cv.take<float>(spectral ? (size_t)rows * P.D : 0);
+  W->norm_scratch = cv.take<float2>(
+      (spectral && P.normalize)
+          ? feature_normalize_scratch_bytes(P.nmax, P.D, (int)P.nprob) / sizeof(float2)
+          : 0);
   W->Q = cv.take<float2>(spectral ? (size_t)rows * ((P.r + 1) & ~1) : 0);
   W->alpha = cv.take<double>(spectral ? (size_t)np * P.r : 0);
   W->beta = cv.take<double>(spectral ? (size_t)np * P.r : 0);
@@ -461,6 +468,22 @@ int sls_feature_map_batched(const void* X, int64_t nb, int64_t rows, int64_t x_s
   if (!X || !W || !b || !Phi) return SLS_ERR_INVALID_ARG;
   return launch_feature_map_tc_batched(X, nb, rows, x_stride, d, ldx, W, b, D, Phi, live, nwin,
                                        win, (cudaStream_t)stream, nullptr);
+}
+
+size_t sls_feature_normalize_workspace_size(int64_t N, int D) {
+  if (N < 1 || D < 1) return 0;
+  return feature_normalize_scratch_bytes(N, D, 1);
+}
+
+int sls_feature_normalize(float* Phi, int64_t N, int D, double* s_hat, void* workspace,
+                          size_t workspace_bytes, void* stream) {
+  if (N < 0 || D < 1) return SLS_ERR_INVALID_ARG;
+  if (N == 0) return SLS_OK;
+  if (!ptr_ok(Phi)) return SLS_ERR_INVALID_ARG;
+  const size_t need = sls_feature_normalize_workspace_size(N, D);
+  if (!workspace || workspace_bytes < need) return SLS_ERR_WORKSPACE;
+  return launch_feature_normalize(Phi, D, nullptr, nullptr, 1, nullptr, N, N,
+                                  (float2*)workspace, s_hat, (cudaStream_t)stream);
 }
 
 size_t sls_lanczos_workspace_size(int64_t N, int D, int r) {
@@ -695,6 +718,12 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
       }
     }
     if (st != SLS_OK) return st;
+    // the row-normalised operator: each spectral problem's rows scaled by
+    // 1 / sqrt of its estimated row sums (Sec. 3.2)
+    if (cfg->normalize &&
+        (st = launch_feature_normalize(W.Phi, cfg->D, W.lz_row0, W.lz_n, nprob, W.nspec, 0,
+                                       P.nmax, W.norm_scratch, nullptr, s)) != SLS_OK)
+      return st;
     phase_mark(1, 1, s);
     phase_mark(2, 0, s);
     LanczosBatch bt{};

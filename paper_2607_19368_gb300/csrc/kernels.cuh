@@ -24,6 +24,15 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
                                   float* Phi, const int* live, int nwin, int win,
                                   cudaStream_t stream, int* status);
 
+// ---- row-normalised operator (Sec. 3.2 variant) ------------------------------
+// Rows of every problem (rows [row0[p], row0[p] + n[p]) of Phi, or one problem
+// of n_single rows when row0 is NULL) scaled in place by 1 / sqrt(s_i) with
+// s = Phi (Phi^T 1) of the problem; s_out (may be NULL) receives s per row.
+size_t feature_normalize_scratch_bytes(int64_t nmax, int D, int nprob);
+int launch_feature_normalize(float* Phi, int D, const int64_t* row0, const int* n,
+                             int nprob_max, const int* nprob_dev, int64_t n_single, int64_t nmax,
+                             float2* scratch, double* s_out, cudaStream_t stream);
+
 // ---- Lanczos (Algorithm 2) --------------------------------------------------
 // Row stride (in float2) of the double-float basis Q: r rounded up to even,
 // so every basis row starts on a 16-byte boundary.

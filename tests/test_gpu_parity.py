@@ -537,3 +537,55 @@ def test_compress_local_w16(sls, dtype, D):
             assert np.array_equal(t, res.tok2macro)
             assert np.array_equal(pos.cpu().numpy(), res.pos)
             assert np.max(np.abs(Xt.cpu().numpy() - res.Xt)) <= EMB_TOL
+
+
+# ---------------------------------------------------------------------------
+# row-normalised operator (Sec. 3.2 variant)
+# ---------------------------------------------------------------------------
+
+
+@pytest.mark.parametrize("name,N,D", [("tiny", 500, 256), ("mistral7b", 3000, 1024)])
+def test_feature_normalize_matches_oracle(sls, name, N, D):
+    """Rows scaled by 1/sqrt(s_i), s = Phi (Phi^T 1): s to the float64
+    rounding level, every scaled element within one float32 ulp of the
+    oracle's float64 value rounded to float32."""
+    w, p, prm = _workload_inputs(name, N=N, D=D)
+    phi32 = oracle_phi32(p.x_f64(), prm.w_f64(), prm.b)
+    s_o, phin_o = O.normalized_features(phi32.astype(np.float64))
+    t = torch.from_numpy(phi32).cuda()
+    s = sls.feature_normalize(t).cpu().numpy()
+    assert np.allclose(s, s_o, rtol=1e-12, atol=0)
+    got = t.cpu().numpy()
+    want = phin_o.astype(np.float32)
+    ulp = np.spacing(np.abs(want).astype(np.float32))
+    assert np.all(np.abs(got - want) <= ulp)
+
+
+def test_lanczos_normalized_operator(sls):
+    """Lanczos on the GPU's normalised rows against the oracle on the same
+    float32 rows; the top Ritz value of the normalised operator is 1."""
+    w, p, prm = _workload_inputs("mistral7b", N=3000, D=1024)
+    phi32 = oracle_phi32(p.x_f64(), prm.w_f64(), prm.b)
+    t = torch.from_numpy(phi32).cuda()
+    sls.feature_normalize(t)
+    phin = t.cpu().numpy()
+    th, th_o, Ug, U_o, _, _ = _lanczos_case(sls, phin, prm.q1[:3000], 32)
+    assert abs(th[0] - 1.0) < 1e-5 and abs(th_o[0] - 1.0) < 1e-5
+
+
+@pytest.mark.parametrize("backend", ["global", "local"])
+def test_compress_normalized(sls, backend):
+    w, p, prm = _workload_inputs("tiny")
+    kw = dict(rho=w.rho, D=w.D, r=w.r, bits=w.bits, preserve_last=12, normalize=1)
+    if backend == "local":
+        cfg = sls.Config.make(backend=sls.BACKEND_LOCAL, window=16, **kw)
+    else:
+        cfg = sls.Config.make(**kw)
+    X = to_torch_x(p.X, w.dtype)
+    Xt, pos, t2m, r_eff, route = sls.compress(
+        X, cfg, to_torch_x(prm.W, w.dtype), torch.from_numpy(prm.b).cuda(),
+        torch.from_numpy(prm.R).cuda(), torch.from_numpy(prm.q1).cuda())
+    M = sls.output_count(cfg, w.N)
+    _check_pass(sls, p.x_f64(), Xt.cpu().numpy(), pos.cpu().numpy(), t2m.cpu().numpy(), M, 0, 12)
+    if backend == "global":
+        assert int(r_eff[0].item()) == w.r
