@@ -260,13 +260,15 @@ def run_reference(args, rank, world):
 def device_inputs(w, rank, dev):
     """Embeddings on the device: one prompt, or the adaptive batch of
     w.batch prompts gathered on the device from one bf16 vocabulary table
-    (the same rows and ids as workloads.make_prompt)."""
+    (the same rows and ids as workloads.make_prompt).  Returns (X, ids) with
+    ids the B x N token ids (numpy int32)."""
     import numpy as np
     import torch
     import workloads as WL
     if w.batch == 1:
         p = WL.make_prompt(w, index=rank)
-        return torch.from_numpy(p.X.view(np.int16)).view(torch.bfloat16).to(dev)
+        X = torch.from_numpy(p.X.view(np.int16)).view(torch.bfloat16).to(dev)
+        return X, p.ids.astype(np.int32).reshape(1, w.N)
     ids = [WL.prompt_ids(w, index=i, dup_frac=WL.adaptive_dup_frac(i, w.batch))
            for i in range(w.batch)]
     uniq, inv = np.unique(np.concatenate(ids), return_inverse=True)
@@ -275,7 +277,21 @@ def device_inputs(w, rank, dev):
     idx = torch.from_numpy(inv.astype(np.int64)).to(dev)
     X = tab.index_select(0, idx).view(torch.bfloat16).view(w.batch, w.N, w.d)
     del tab
-    return X
+    return X, np.stack(ids).astype(np.int32)
+
+
+def vocab_table(X, ids, V, dev):
+    """The model's input embedding table as it would sit in HBM: V x d bf16,
+    the rows of the prompt's ids taken from X (every other row zero, never
+    read), so that table[ids] is X."""
+    import numpy as np
+    import torch
+    d = X.shape[-1]
+    uniq, first = np.unique(ids.reshape(-1), return_index=True)
+    table = torch.zeros((V, d), dtype=X.dtype, device=dev)
+    src = X.reshape(-1, d).index_select(0, torch.from_numpy(first.astype(np.int64)).to(dev))
+    table.index_copy_(0, torch.from_numpy(uniq.astype(np.int64)).to(dev), src)
+    return table
 
 
 def run_native(args, rank, world):
@@ -292,7 +308,7 @@ def run_native(args, rank, world):
     rho = args.rho or w.rho
     adaptive = w.backend == "adaptive"
     local = w.backend == "local"
-    X = device_inputs(w, rank, dev)
+    X, ids = device_inputs(w, rank, dev)
     prm = WL.params_for(w)
     Wt = torch.from_numpy(prm.W.view(np.int16)).view(torch.bfloat16).to(dev)
     bt = torch.from_numpy(prm.b).to(dev)
@@ -433,51 +449,74 @@ def run_native(args, rank, world):
 
         ms_serial = timed(serial, args.e2e_steps)
         # pipelined (the serving pattern): two device buffers; a copy stream
-        # brings step k+1's embeddings in and takes step k's outputs out while
+        # brings step k+1's inputs in and takes step k's outputs out while
         # step k compresses on the compute stream
         comp = torch.cuda.current_stream(dev)
         cps = torch.cuda.Stream(device=dev)
-        Xds = [torch.empty_like(Xin) for _ in range(2)]
         outs = [out, (torch.empty_like(Xt), torch.empty_like(pos), torch.empty_like(t2m))]
         hos = [ho, host_outs()]
-        h2d = [torch.cuda.Event() for _ in range(2)]
-        done = [torch.cuda.Event() for _ in range(2)]
-        d2h = [torch.cuda.Event() for _ in range(2)]
 
-        def pipelined(n):
-            cps.wait_stream(comp)
-            with torch.cuda.stream(cps):
-                Xds[0].copy_(Xh, non_blocking=True)
-                h2d[0].record(cps)
-            for k in range(n):
-                b = k % 2
-                if k + 1 < n:
-                    nb = (k + 1) % 2
-                    with torch.cuda.stream(cps):
-                        if k >= 1:
-                            cps.wait_event(done[nb])
-                        Xds[nb].copy_(Xh, non_blocking=True)
-                        h2d[nb].record(cps)
-                comp.wait_event(h2d[b])
-                if k >= 2:
-                    comp.wait_event(d2h[b])
-                sls.compress(Xds[b], cfg, Wt, bt, Rt, qt, workspace=ws, out=outs[b])
-                done[b].record(comp)
+        def pipeline(Ih, run):
+            Ids = [torch.empty(Ih.shape, dtype=Ih.dtype, device=dev) for _ in range(2)]
+            h2d = [torch.cuda.Event() for _ in range(2)]
+            done = [torch.cuda.Event() for _ in range(2)]
+            d2h = [torch.cuda.Event() for _ in range(2)]
+
+            def go(n):
+                cps.wait_stream(comp)
                 with torch.cuda.stream(cps):
-                    cps.wait_event(done[b])
-                    for h, o in zip(hos[b], outs[b]):
-                        h.copy_(o, non_blocking=True)
-                    d2h[b].record(cps)
-            comp.wait_stream(cps)
+                    Ids[0].copy_(Ih, non_blocking=True)
+                    h2d[0].record(cps)
+                for k in range(n):
+                    b = k % 2
+                    if k + 1 < n:
+                        nb = (k + 1) % 2
+                        with torch.cuda.stream(cps):
+                            if k >= 1:
+                                cps.wait_event(done[nb])
+                            Ids[nb].copy_(Ih, non_blocking=True)
+                            h2d[nb].record(cps)
+                    comp.wait_event(h2d[b])
+                    if k >= 2:
+                        comp.wait_event(d2h[b])
+                    run(Ids[b], outs[b])
+                    done[b].record(comp)
+                    with torch.cuda.stream(cps):
+                        cps.wait_event(done[b])
+                        for h, o in zip(hos[b], outs[b]):
+                            h.copy_(o, non_blocking=True)
+                        d2h[b].record(cps)
+                comp.wait_stream(cps)
+            return go
 
-        ms_pipe = timed(pipelined, args.e2e_steps)
-        m2 = max_over_ranks([ms_pipe, ms_serial], world, dev)
+        ms_pipe = timed(pipeline(Xh, lambda x, o: sls.compress(x, cfg, Wt, bt, Rt, qt,
+                                                                 workspace=ws, out=o)),
+                        args.e2e_steps)
+        # from token ids: the model's embedding table stays in HBM and only
+        # the ids come in; the lookup X = E[ids] runs inside the call
+        table = vocab_table(X, ids, w.V, dev)
+        Ih = torch.from_numpy(ids if adaptive else ids.reshape(N)).pin_memory()
+        tws = sls.TokensWorkspace(cfg, table.dtype, B, N, d, dev)
+        ms_ids = timed(pipeline(Ih, lambda i, o: sls.compress_tokens(i, table, cfg, Wt, bt, Rt,
+                                                                       qt, workspace=tws,
+                                                                       out=o)),
+                       args.e2e_steps)
+        del table, tws
+        m2 = max_over_ranks([ms_pipe, ms_serial, ms_ids], world, dev)
+        d2h_bytes = Xt.numel() * 4 + pos.numel() * 4 + t2m.numel() * 4
         e2e = {"value": world * B * N / (m2[0] / 1e3), "unit": UNIT,
                "h2d_bytes_per_step": Xin.numel() * 2,
-               "d2h_bytes_per_step": Xt.numel() * 4 + pos.numel() * 4 + t2m.numel() * 4,
+               "d2h_bytes_per_step": d2h_bytes,
                "mode": "pipelined: the copies of step k+1 in and step k out overlap the "
                        "compression of step k on a second stream (double-buffered)",
-               "serial_value": world * B * N / (m2[1] / 1e3)}
+               "serial_value": world * B * N / (m2[1] / 1e3),
+               "from_token_ids": {
+                   "value": world * B * N / (m2[2] / 1e3), "unit": UNIT,
+                   "h2d_bytes_per_step": int(Ih.numel()) * 4,
+                   "d2h_bytes_per_step": d2h_bytes,
+                   "mode": "pipelined as above; token ids in, the V x d bf16 embedding "
+                           "table resident on the device, lookup inside "
+                           "sls_compress_tokens"}}
 
     if rank != 0:
         return

@@ -162,7 +162,7 @@ int sls_feature_map_batched(const void* X, int64_t nb, int64_t rows,
  *   Phi: N x D floats (device, in place); s_hat (may be NULL): N doubles
  *   (device, output); workspace: sls_feature_normalize_workspace_size(N, D)
  *   device bytes.  Column sums and row dots are compensated (double-float);
- *   each scaled element is rounded once from its float64 product.
+ *   each scaled element is x / sqrt(s_i) to within one float32 rounding.
  * Errors: INVALID_ARG for bad sizes or NULL pointers, WORKSPACE if the
  * workspace is too small.
  */
@@ -272,6 +272,45 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
                  float* Xt, int32_t* pos, int32_t* tok2macro, int32_t* r_eff,
                  int32_t* route, void* workspace, size_t workspace_bytes,
                  void* stream);
+
+/*
+ * The step before the pass: a prompt's input embeddings, one row of the
+ * model's input embedding table per token (Sec. 3.1: X is the output of the
+ * LLM's input embedding layer; Fig. 1: prompt tokens -> input embeddings):
+ *   X[i, :] = table[ids[i], :]   for i < N.
+ * table: V x d of x_dtype (row stride ld_table elements); ids: N int32;
+ * X: N x d of x_dtype (output, row stride ldx).  An id outside [0, V) gives a
+ * zero row of X; bad (may be NULL): one device int32, set to the number of
+ * such ids.  Rows move as 16-byte vectors when the table and X bases, their
+ * row strides and d * element size are all multiples of 16 bytes, else by
+ * element.  N may be 0.  Errors: INVALID_ARG for bad sizes, dtype or NULL
+ * pointers.
+ */
+int sls_embed_gather(const void* table, int x_dtype, int64_t V, int d,
+                     int64_t ld_table, const int32_t* ids, int64_t N, void* X,
+                     int64_t ldx, int32_t* bad, void* stream);
+
+/* Device workspace bytes needed by sls_compress_tokens. */
+size_t sls_compress_tokens_workspace_size(const sls_config_t* cfg, int x_dtype,
+                                          int64_t B, int64_t N, int d);
+
+/*
+ * sls_compress from token ids: B prompts of N ids each (ids: B x N int32,
+ * prompt-major) are looked up in the embedding table (see sls_embed_gather)
+ * into a B x N x d buffer at the start of the workspace, which sls_compress
+ * then compresses; every other argument and output is that of sls_compress.
+ * The macro-token embeddings Xt are what the frozen model's prefill takes
+ * through its inputs_embeds interface (Sec. 3.4).  bad_ids (may be NULL):
+ * one device int32, the number of ids outside [0, V) (their rows are zero).
+ * workspace: sls_compress_tokens_workspace_size(cfg, x_dtype, B, N, d)
+ * bytes, 16-byte aligned.  Errors: those of sls_compress.
+ */
+int sls_compress_tokens(const sls_config_t* cfg, const void* table, int x_dtype,
+                        int64_t V, int d, int64_t ld_table, const int32_t* ids,
+                        int64_t B, int64_t N, const sls_params_t* params,
+                        float* Xt, int32_t* pos, int32_t* tok2macro,
+                        int32_t* r_eff, int32_t* route, int32_t* bad_ids,
+                        void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * sls_lanczos_topr without a caller workspace.  The paper has no counterpart

@@ -27,7 +27,7 @@ __all__ = [
     "compress_adaptive", "compress_local", "compress_chunk", "complexity_ops",
     "CompressResult",
     "POS_MAX", "POS_MEDIAN", "POS_MEAN", "MODE_REPRESENTATIVE", "MODE_COMPACT",
-    "normalized_features",
+    "normalized_features", "embed_lookup",
 ]
 
 # ---------------------------------------------------------------------------
@@ -62,6 +62,29 @@ class CompressResult:
     pos: np.ndarray       # (M,) int64 positions
     tok2macro: np.ndarray  # (N,) int64 macro index of every token
     info: dict
+
+
+# ---------------------------------------------------------------------------
+# Step 0: input embeddings (Sec. 3.1, Fig. 1)
+# ---------------------------------------------------------------------------
+
+
+def embed_lookup(table: np.ndarray, ids: np.ndarray) -> np.ndarray:
+    """The prompt's input embeddings: row ids[i] of the model's input
+    embedding table for token i (Sec. 3.1 takes X from the LLM's input
+    embedding layer; Fig. 1 draws prompt tokens -> input embeddings).
+
+    Values are copied as stored (same dtype as the table).  An id outside
+    [0, V) has no row: this statement of the lookup gives it a zero row (the
+    paper never feeds one)."""
+    table = np.asarray(table)
+    ids = np.asarray(ids, dtype=np.int64)
+    V = table.shape[0]
+    X = np.zeros(ids.shape + table.shape[1:], dtype=table.dtype)
+    for i, v in enumerate(ids.reshape(-1)):
+        if 0 <= v < V:
+            X.reshape(-1, *table.shape[1:])[i] = table[v]
+    return X
 
 
 # ---------------------------------------------------------------------------

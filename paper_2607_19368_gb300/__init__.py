@@ -7,7 +7,8 @@ calls and raises on a non-zero status.  There is no CPU fallback: if the
 library is not built, importing the functions works but every call raises.
 
 The same names as the C entry points are exported:
-``feature_map``, ``lanczos_topr``, ``simhash``, ``aggregate``, ``compress``.
+``feature_map``, ``lanczos_topr``, ``simhash``, ``aggregate``, ``compress``,
+``embed_gather``, ``compress_tokens``.
 """
 from __future__ import annotations
 
@@ -24,7 +25,8 @@ __all__ = [
     "feature_map_batched", "feature_normalize",
     "lanczos_topr", "simhash", "aggregate", "compress", "output_count",
     "compress_workspace_size", "workspace_status", "EXPORTED", "PHASES",
-    "set_phase_events", "launch_count", "Workspace",
+    "set_phase_events", "launch_count", "Workspace", "embed_gather", "compress_tokens",
+    "compress_tokens_workspace_size", "TokensWorkspace",
 ]
 
 SLS_OK = 0
@@ -102,6 +104,12 @@ EXPORTED = {
     "sls_compress": (_i32, [ctypes.POINTER(Config), _vp, _i32, _i64, _i64, _i32, _i64,
                             ctypes.POINTER(_Params), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "sls_workspace_status": (_i32, [_vp, _vp]),
+    "sls_embed_gather": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _i64, _vp, _i64, _vp, _vp]),
+    "sls_compress_tokens_workspace_size": (_sz, [ctypes.POINTER(Config), _i32, _i64, _i64,
+                                                 _i32]),
+    "sls_compress_tokens": (_i32, [ctypes.POINTER(Config), _vp, _i32, _i64, _i32, _i64, _vp,
+                                   _i64, _i64, ctypes.POINTER(_Params), _vp, _vp, _vp, _vp, _vp,
+                                   _vp, _vp, _sz, _vp]),
     "sls_lanczos_topr_noalloc": (_i32, [_vp, _i64, _i32, _i32, _vp, _d, _vp, _vp, _vp, _vp,
                                         _vp, _vp]),
     "sls_set_phase_events": (_i32, [ctypes.POINTER(ctypes.c_void_p), _i32]),
@@ -303,6 +311,39 @@ class Workspace:
         self.buf = _workspace(self.nbytes, device)
 
 
+def _outputs(cfg: Config, B: int, N: int, d: int, dev, out):
+    M = output_count(cfg, N)
+    if M < 0:
+        raise SLSError("sls_output_count", 1, "invalid configuration")
+    if out is None:
+        Xt = torch.empty((B, M, d), dtype=torch.float32, device=dev)
+        pos = torch.empty((B, M), dtype=torch.int32, device=dev)
+        t2m = torch.empty((B, N), dtype=torch.int32, device=dev)
+    else:
+        Xt, pos, t2m = out
+    nwin = max(1, B * ((N + max(1, cfg.window) - 1) // max(1, cfg.window)))
+    r_eff = torch.zeros(nwin, dtype=torch.int32, device=dev)
+    route = torch.zeros(nwin, dtype=torch.int32, device=dev)
+    return M, Xt, pos, t2m, r_eff, route
+
+
+def _params(cfg: Config, M: int, N: int, B: int, batched: bool, dev, W, b, R, q1):
+    """sls_params_t for the spectral backends (None for chunk or identity),
+    and the contiguous tensors it points into (kept alive by the caller)."""
+    if cfg.backend == BACKEND_CHUNK or M == N:
+        return None, []
+    if W is None or b is None or R is None or q1 is None:
+        raise ValueError("the spectral backends need W, b, R and q1")
+    Wc = W.contiguous()
+    bc = b.float().contiguous()
+    Rc = R.float().contiguous()
+    qc = q1.to(device=dev, dtype=torch.float64).contiguous()
+    q1_stride = qc.numel() // B if batched else 0
+    params = _Params(Wc.data_ptr(), bc.data_ptr(), Rc.data_ptr(), Rc.shape[0], Rc.stride(0),
+                     qc.data_ptr(), q1_stride)
+    return params, [Wc, bc, Rc, qc]
+
+
 def compress(X: torch.Tensor, cfg: Config, W: Optional[torch.Tensor] = None,
              b: Optional[torch.Tensor] = None, R: Optional[torch.Tensor] = None,
              q1: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
@@ -316,38 +357,83 @@ def compress(X: torch.Tensor, cfg: Config, W: Optional[torch.Tensor] = None,
     B, N, d = X3.shape
     assert X3.stride(2) == 1 and X3.stride(0) == N * X3.stride(1)
     dev = X.device
-    M = output_count(cfg, N)
-    if M < 0:
-        raise SLSError("sls_output_count", 1, "invalid configuration")
-    if out is None:
-        Xt = torch.empty((B, M, d), dtype=torch.float32, device=dev)
-        pos = torch.empty((B, M), dtype=torch.int32, device=dev)
-        t2m = torch.empty((B, N), dtype=torch.int32, device=dev)
-    else:
-        Xt, pos, t2m = out
-    nwin = max(1, B * ((N + max(1, cfg.window) - 1) // max(1, cfg.window)))
-    r_eff = torch.zeros(nwin, dtype=torch.int32, device=dev)
-    route = torch.zeros(nwin, dtype=torch.int32, device=dev)
+    M, Xt, pos, t2m, r_eff, route = _outputs(cfg, B, N, d, dev, out)
     if workspace is None:
         workspace = Workspace(cfg, B, N, d, dev)
-    params = None
-    keep = []
-    if cfg.backend != BACKEND_CHUNK and M != N:
-        if W is None or b is None or R is None or q1 is None:
-            raise ValueError("the spectral backends need W, b, R and q1")
-        Wc = W.contiguous()
-        bc = b.float().contiguous()
-        Rc = R.float().contiguous()
-        qc = q1.to(device=dev, dtype=torch.float64).contiguous()
-        keep = [Wc, bc, Rc, qc]
-        q1_stride = qc.numel() // B if batched else 0
-        params = _Params(Wc.data_ptr(), bc.data_ptr(), Rc.data_ptr(), Rc.shape[0], Rc.stride(0),
-                         qc.data_ptr(), q1_stride)
+    params, keep = _params(cfg, M, N, B, batched, dev, W, b, R, q1)
     st = lib().sls_compress(ctypes.byref(cfg), _ptr(X3), _dtype_code(X3), B, N, d,
                             X3.stride(1), ctypes.byref(params) if params is not None else None,
                             _ptr(Xt), _ptr(pos), _ptr(t2m), _ptr(r_eff), _ptr(route),
                             _ptr(workspace.buf), workspace.nbytes, _stream(X3))
     _check("sls_compress", st)
+    del keep
+    if not batched:
+        return Xt[0], pos[0], t2m[0], r_eff, route
+    return Xt, pos, t2m, r_eff, route
+
+
+def embed_gather(table: torch.Tensor, ids: torch.Tensor, out: Optional[torch.Tensor] = None,
+                 bad: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Input embeddings X = table[ids] (Sec. 3.1): table is V x d (float32 or
+    bfloat16), ids any shape of int32 token ids; returns ids.shape + (d,) in
+    the table's dtype.  Rows of out-of-range ids are zero; `bad` (one int32,
+    optional) receives their count."""
+    _need_cuda(table, ids, out, bad)
+    V, d = table.shape
+    assert table.stride(1) == 1
+    ids_c = ids.to(dtype=torch.int32).contiguous()
+    N = ids_c.numel()
+    if out is None:
+        out = torch.empty(tuple(ids.shape) + (d,), dtype=table.dtype, device=table.device)
+    assert out.dtype == table.dtype and out.is_contiguous()
+    st = lib().sls_embed_gather(_ptr(table), _dtype_code(table), V, d, table.stride(0),
+                                _ptr(ids_c), N, _ptr(out), d, _ptr(bad), _stream(table))
+    _check("sls_embed_gather", st)
+    return out
+
+
+def compress_tokens_workspace_size(cfg: Config, dtype: torch.dtype, B: int, N: int,
+                                   d: int) -> int:
+    code = SLS_BF16 if dtype == torch.bfloat16 else SLS_F32
+    return int(lib().sls_compress_tokens_workspace_size(ctypes.byref(cfg), code, B, N, d))
+
+
+class TokensWorkspace:
+    """A reusable device workspace for compress_tokens() (one shape)."""
+
+    def __init__(self, cfg: Config, dtype: torch.dtype, B: int, N: int, d: int, device):
+        self.nbytes = compress_tokens_workspace_size(cfg, dtype, B, N, d)
+        if self.nbytes == 0:
+            raise SLSError("sls_compress_tokens_workspace_size", 1, "invalid configuration")
+        self.buf = _workspace(self.nbytes, device)
+
+
+def compress_tokens(ids: torch.Tensor, table: torch.Tensor, cfg: Config,
+                    W: Optional[torch.Tensor] = None, b: Optional[torch.Tensor] = None,
+                    R: Optional[torch.Tensor] = None, q1: Optional[torch.Tensor] = None,
+                    workspace: Optional[TokensWorkspace] = None, out=None,
+                    bad: Optional[torch.Tensor] = None):
+    """compress() from token ids (N or B x N int32) and the model's input
+    embedding table (V x d): the lookup X = table[ids] (Sec. 3.1) and the
+    compression pass in one call.  Returns what compress() returns."""
+    _need_cuda(ids, table, bad)
+    batched = ids.dim() == 2
+    ids2 = (ids if batched else ids.view(1, -1)).to(dtype=torch.int32).contiguous()
+    B, N = ids2.shape
+    V, d = table.shape
+    assert table.stride(1) == 1
+    dev = table.device
+    M, Xt, pos, t2m, r_eff, route = _outputs(cfg, B, N, d, dev, out)
+    if workspace is None:
+        workspace = TokensWorkspace(cfg, table.dtype, B, N, d, dev)
+    params, keep = _params(cfg, M, N, B, batched, dev, W, b, R, q1)
+    st = lib().sls_compress_tokens(ctypes.byref(cfg), _ptr(table), _dtype_code(table), V, d,
+                                   table.stride(0), _ptr(ids2), B, N,
+                                   ctypes.byref(params) if params is not None else None,
+                                   _ptr(Xt), _ptr(pos), _ptr(t2m), _ptr(r_eff), _ptr(route),
+                                   _ptr(bad), _ptr(workspace.buf), workspace.nbytes,
+                                   _stream(table))
+    _check("sls_compress_tokens", st)
     del keep
     if not batched:
         return Xt[0], pos[0], t2m[0], r_eff, route

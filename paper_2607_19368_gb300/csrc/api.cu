@@ -791,6 +791,47 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   return st;
 }
 
+int sls_embed_gather(const void* table, int x_dtype, int64_t V, int d, int64_t ld_table,
+                     const int32_t* ids, int64_t N, void* X, int64_t ldx, int32_t* bad,
+                     void* stream) {
+  if (N < 0 || V < 1 || d < 1 || ld_table < d || ldx < d) return SLS_ERR_INVALID_ARG;
+  if (x_dtype != SLS_F32 && x_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
+  if (N > 0 && (!table || !ids || !X)) return SLS_ERR_INVALID_ARG;
+  return launch_embed_gather(table, x_dtype, V, d, ld_table, ids, N, X, ldx, bad,
+                             (cudaStream_t)stream);
+}
+
+size_t sls_compress_tokens_workspace_size(const sls_config_t* cfg, int x_dtype, int64_t B,
+                                          int64_t N, int d) {
+  if (x_dtype != SLS_F32 && x_dtype != SLS_BF16) return 0;
+  const size_t inner = sls_compress_workspace_size(cfg, B, N, d);
+  if (inner == 0) return 0;
+  const size_t elt = (x_dtype == SLS_BF16) ? 2 : 4;
+  return sls_align256((size_t)B * (size_t)N * (size_t)d * elt) + inner;
+}
+
+int sls_compress_tokens(const sls_config_t* cfg, const void* table, int x_dtype, int64_t V, int d,
+                        int64_t ld_table, const int32_t* ids, int64_t B, int64_t N,
+                        const sls_params_t* params, float* Xt, int32_t* pos, int32_t* tok2macro,
+                        int32_t* r_eff, int32_t* route, int32_t* bad_ids, void* workspace,
+                        size_t workspace_bytes, void* stream) {
+  if (validate_config(cfg) != SLS_OK) return SLS_ERR_INVALID_ARG;
+  if (B < 1 || N < 1 || V < 1 || d < 1 || ld_table < d) return SLS_ERR_INVALID_ARG;
+  if (x_dtype != SLS_F32 && x_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
+  if (!table || !ids) return SLS_ERR_INVALID_ARG;
+  const size_t need = sls_compress_tokens_workspace_size(cfg, x_dtype, B, N, d);
+  if (need == 0) return SLS_ERR_INVALID_ARG;
+  if (!ptr_ok(workspace) || workspace_bytes < need) return SLS_ERR_WORKSPACE;
+  const size_t elt = (x_dtype == SLS_BF16) ? 2 : 4;
+  const size_t xb = sls_align256((size_t)B * (size_t)N * (size_t)d * elt);
+  void* X = workspace;
+  int st = launch_embed_gather(table, x_dtype, V, d, ld_table, ids, B * N, X, d, bad_ids,
+                               (cudaStream_t)stream);
+  if (st != SLS_OK) return st;
+  return sls_compress(cfg, X, x_dtype, B, N, d, d, params, Xt, pos, tok2macro, r_eff, route,
+                      (char*)workspace + xb, workspace_bytes - xb, stream);
+}
+
 int sls_set_phase_events(void* const* events, int count) {
   if (count == 0 || events == nullptr) {
     g_phase_on = false;

@@ -24,6 +24,14 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
                                   float* Phi, const int* live, int nwin, int win,
                                   cudaStream_t stream, int* status);
 
+// ---- input embeddings: X = E[ids] (Sec. 3.1) ---------------------------------
+// Rows of a V x d table (row stride ld_table elements) gathered into X (row
+// stride ldx); an id outside [0, V) gives a zero row and is counted in *bad
+// (zeroed first; may be NULL).
+int launch_embed_gather(const void* table, int x_dtype, int64_t V, int d, int64_t ld_table,
+                        const int32_t* ids, int64_t N, void* X, int64_t ldx, int* bad,
+                        cudaStream_t stream);
+
 // ---- row-normalised operator (Sec. 3.2 variant) ------------------------------
 // Rows of every problem (rows [row0[p], row0[p] + n[p]) of Phi, or one problem
 // of n_single rows when row0 is NULL) scaled in place by 1 / sqrt(s_i) with

@@ -6,6 +6,7 @@ import os
 import re
 
 import pytest
+import torch
 
 import oracle as O
 
@@ -57,6 +58,15 @@ def test_host_side_errors_and_counts(lib):
     assert lib.sls_lanczos_topr(None, 4, 8, 0, None, 1e-10, None, None, None, None, None,
                                 None, 0, None) == 1                               # r = 0
     assert lib.sls_lanczos_workspace_size(1000, 256, 16) > 0
+    # embedding lookup: table stride below d, unknown dtype, missing ids
+    assert lib.sls_embed_gather(None, 1, 10, 8, 4, None, 4, None, 8, None, None) == 1
+    assert lib.sls_embed_gather(None, 7, 10, 8, 8, None, 4, None, 8, None, None) == 1
+    assert lib.sls_embed_gather(ctypes.c_void_p(16), 1, 10, 8, 8, None, 4, ctypes.c_void_p(16),
+                                8, None, None) == 1
+    assert lib.sls_embed_gather(None, 1, 10, 8, 8, None, 0, None, 8, None, None) == 0  # N = 0
+    cfg = sls.Config.make(rho=16.0, D=2048, r=64, bits=16)
+    assert (sls.compress_tokens_workspace_size(cfg, torch.bfloat16, 1, 32768, 3584)
+            >= sls.compress_workspace_size(cfg, 1, 32768, 3584) + 32768 * 3584 * 2)
     # output counts agree with the oracle's target count (Sec. 3.3) and identity
     for N, rho, pf, pl in [(512, 4.0, 0, 12), (16384, 16.0, 0, 12), (100, 1.0, 0, 12),
                            (10, 4.0, 3, 20), (1000, 3.0, 5, 7)]:

@@ -544,7 +544,8 @@ def test_compress_local_w16(sls, dtype, D):
 # ---------------------------------------------------------------------------
 
 
-@pytest.mark.parametrize("name,N,D", [("tiny", 500, 256), ("mistral7b", 3000, 1024)])
+@pytest.mark.parametrize("name,N,D", [("tiny", 500, 256), ("mistral7b", 3000, 1024),
+                                      ("tiny", 777, 2048), ("tiny", 130, 8192), ("tiny", 97, 4)])
 def test_feature_normalize_matches_oracle(sls, name, N, D):
     """Rows scaled by 1/sqrt(s_i), s = Phi (Phi^T 1): s to the float64
     rounding level, every scaled element within one float32 ulp of the

@@ -617,3 +617,34 @@ def test_normalized_compress_invariants():
     res = O.compress_global(p.x_f64(), prm.w_f64(), prm.b, prm.R, prm.q1, cfg)
     _check_result(res, w.N, O.target_count(w.N - 12, w.rho) + 12, 0, 12)
     assert abs(res.info["theta"][0] - 1.0) < 1e-6
+
+
+# ---------------------------------------------------------------------------
+# input embeddings (Sec. 3.1, Fig. 1): X = E[ids]
+# ---------------------------------------------------------------------------
+
+
+def test_embed_lookup_is_the_one_hot_product():
+    """The lookup equals the product of the one-hot token matrix with the
+    table (a row of zeros for an id with no row), element for element."""
+    rng = np.random.default_rng(5)
+    V, d = 37, 9
+    table = rng.standard_normal((V, d))
+    ids = rng.integers(-3, V + 3, size=400)
+    onehot = (ids[:, None] == np.arange(V)[None, :]).astype(np.float64)
+    X = O.embed_lookup(table, ids)
+    assert X.shape == (400, d) and X.dtype == table.dtype
+    assert np.array_equal(X, onehot @ table)
+    assert np.all(X[(ids < 0) | (ids >= V)] == 0)
+
+
+def test_embed_lookup_reproduces_the_prompt_generator():
+    """The seeded prompts are table lookups: the bf16 table of every vocabulary
+    row, looked up at the prompt's ids, is the prompt's X bit for bit (so a
+    device-resident table and the ids stand in for X)."""
+    w = WL.scaled(WL.WORKLOADS["qwen7b"], N=300, d=32, V=400)
+    p = WL.make_prompt(w)
+    table = WL.f32_to_bf16_bits(
+        WL.vocab_rows(WL.DATA_SEED, np.arange(w.V), w.d).astype(np.float32))
+    X = O.embed_lookup(table, p.ids)
+    assert X.dtype == np.uint16 and np.array_equal(X, p.X)
