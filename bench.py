@@ -54,6 +54,8 @@ def parse():
                     help="compression ratio (default: the workload's)")
     ap.add_argument("--normalize", action="store_true",
                     help="row-normalised operator (the paper's untested Sec. 3.2 variant)")
+    ap.add_argument("--phi", default="f32", choices=["f32", "bf16"],
+                    help="storage of the feature matrix (bf16: opt-in half-size Phi)")
     ap.add_argument("--cpu-sample", type=int, default=4096,
                     help="tokens of the prompt the CPU oracle compresses per baseline step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -164,11 +166,11 @@ def max_over_ranks(values, world, device):
     return [float(x) for x in t.tolist()]
 
 
-def lanczos_algorithmic_bytes(n_tokens, D, r):
-    """Per launch: two float32 sweeps over Phi per step (8 r D bytes per token)
-    plus the double-float basis traffic of the two Gram-Schmidt passes
-    (16 r (r + 1) bytes per token)."""
-    return n_tokens * (8 * r * D + 16 * r * (r + 1))
+def lanczos_algorithmic_bytes(n_tokens, D, r, esz=4):
+    """Per launch: two sweeps over Phi per step (2 r D esz bytes per token:
+    8 r D for float32 Phi, 4 r D for bf16) plus the double-float basis
+    traffic of the two Gram-Schmidt passes (16 r (r + 1) bytes per token)."""
+    return n_tokens * (2 * esz * r * D + 16 * r * (r + 1))
 
 
 def windowed(w):
@@ -314,18 +316,21 @@ def run_native(args, rank, world):
     bt = torch.from_numpy(prm.b).to(dev)
     Rt = torch.from_numpy(prm.R).to(dev)
     qt = torch.from_numpy(prm.q1).to(dev)
+    phi_code = sls.SLS_BF16 if args.phi == "bf16" else sls.SLS_F32
     if adaptive:
         cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=w.D, r=w.r, bits=w.bits,
                               window=w.window, preserve_first=w.preserve_first,
-                              preserve_last=w.preserve_last, normalize=int(args.normalize))
+                              preserve_last=w.preserve_last, normalize=int(args.normalize),
+                              phi_dtype=phi_code)
     elif local:
         cfg = sls.Config.make(backend=sls.BACKEND_LOCAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
                               window=w.window, preserve_first=w.preserve_first,
-                              preserve_last=w.preserve_last, normalize=int(args.normalize))
+                              preserve_last=w.preserve_last, normalize=int(args.normalize),
+                              phi_dtype=phi_code)
     else:
         cfg = sls.Config.make(backend=sls.BACKEND_GLOBAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
                               preserve_first=w.preserve_first, preserve_last=w.preserve_last,
-                              normalize=int(args.normalize))
+                              normalize=int(args.normalize), phi_dtype=phi_code)
     B, N, d = w.batch, w.N, w.d
     M = sls.output_count(cfg, N)
     ws = sls.Workspace(cfg, B, N, d, dev)
@@ -395,7 +400,7 @@ def run_native(args, rank, world):
     value = world * B * N / (ms_max / 1e3)
 
     # roofline of the dominant kernel (the persistent Lanczos kernel)
-    alg = lanczos_algorithmic_bytes(lz_tokens, w.D, w.r)
+    alg = lanczos_algorithmic_bytes(lz_tokens, w.D, w.r, 2 if args.phi == "bf16" else 4)
     lz_s = phases["lanczos"] / 1e3
     peak, src = peaks()
     achieved = alg / lz_s / 1e9 if lz_s > 0 else 0.0
@@ -408,7 +413,7 @@ def run_native(args, rank, world):
             with open(tr) as f:
                 t = json.load(f)
             if (t.get("workload") == w.name and t.get("kernel_rev") == LANCZOS_KERNEL_REV
-                    and not windowed(w)):
+                    and not windowed(w) and args.phi == "f32"):
                 roof["traffic"] = t["dram_bytes_per_launch"]
         except Exception:
             pass
@@ -530,6 +535,9 @@ def run_native(args, rank, world):
         extra.update({"spectral_windows": n_spec, "spectral_tokens": lz_tokens})
     if args.normalize:
         extra["operator"] = "row-normalised (Sec. 3.2 variant, symmetric form)"
+    if args.phi == "bf16":
+        extra["inputs"] = ("bf16 embeddings and Omega; Phi stored as bf16 (opt-in); "
+                           "double-float Lanczos vectors")
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,

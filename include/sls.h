@@ -94,6 +94,10 @@ typedef struct sls_config {
   int tau_schedule;     /* 1: tau(rho) = clamp(0.75 - 0.05 log2 rho, .55, .70)  */
   int normalize;        /* 1: row-normalised operator (Sec. 3.2), see
                            sls_feature_normalize                               */
+  int phi_dtype;        /* storage of the feature matrix Phi: SLS_F32 (default)
+                           or SLS_BF16 (half the bytes; Lanczos then runs on
+                           the bf16-rounded features, see sls_lanczos_topr_ex;
+                           needs D % 8 == 0 and normalize = 0)                 */
 } sls_config_t;
 
 /*
@@ -132,6 +136,16 @@ int sls_version(void);
 int sls_feature_map(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
                     const void* W, const float* b, int D, float* Phi,
                     void* stream);
+
+/*
+ * sls_feature_map with a choice of storage for Phi: phi_dtype SLS_F32 (as
+ * sls_feature_map) or SLS_BF16 (Phi: N x D raw bfloat16 values, uint16, each
+ * the float32 feature rounded to nearest even).  Errors: those of
+ * sls_feature_map, INVALID_ARG for another phi_dtype.
+ */
+int sls_feature_map_ex(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
+                       const void* W, const float* b, int D, void* Phi,
+                       int phi_dtype, void* stream);
 
 /*
  * The same features for a batch of nb equal-length prompts in one launch
@@ -193,6 +207,20 @@ int sls_lanczos_topr(const float* Phi, int64_t N, int D, int r,
                      const double* q1, double tol, double* theta, float* U,
                      int32_t* r_eff, double* alpha, double* beta,
                      void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * sls_lanczos_topr on a feature matrix stored as phi_dtype: SLS_F32 (exactly
+ * sls_lanczos_topr) or SLS_BF16 (Phi: N x D raw bfloat16 values, uint16;
+ * requires D % 8 == 0).  bf16 elements are widened exactly to float32, so the
+ * run is Algorithm 2 on the operator of the stored (rounded) features, with
+ * the same arithmetic as the float32 case; only the bytes read differ.
+ * Errors: those of sls_lanczos_topr, INVALID_ARG for another phi_dtype,
+ * UNSUPPORTED for bf16 with D % 8 != 0.
+ */
+int sls_lanczos_topr_ex(const void* Phi, int phi_dtype, int64_t N, int D, int r,
+                        const double* q1, double tol, double* theta, float* U,
+                        int32_t* r_eff, double* alpha, double* beta,
+                        void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * SimHash in the spectral subspace, Sec. 3.3 Eq. simhash:

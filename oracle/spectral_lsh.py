@@ -27,7 +27,7 @@ __all__ = [
     "compress_adaptive", "compress_local", "compress_chunk", "complexity_ops",
     "CompressResult",
     "POS_MAX", "POS_MEDIAN", "POS_MEAN", "MODE_REPRESENTATIVE", "MODE_COMPACT",
-    "normalized_features", "embed_lookup",
+    "normalized_features", "embed_lookup", "bf16_round",
 ]
 
 # ---------------------------------------------------------------------------
@@ -105,6 +105,25 @@ def rff_features(X: np.ndarray, W: np.ndarray, b: np.ndarray) -> np.ndarray:
     b = np.asarray(b, dtype=np.float64)
     D = W.shape[0]
     return math.sqrt(2.0 / D) * np.cos(X @ W.T + b[None, :])
+
+
+def bf16_round(x: np.ndarray) -> np.ndarray:
+    """The feature matrix stored in bfloat16 (the opt-in half-size storage of
+    Phi): every value rounded to 8 significant bits, to nearest with ties to
+    even, returned as float64.
+
+    Reading: the paper computes Eq. rff_map without fixing a storage
+    precision (its runs use float16 throughout, App. B); bf16 keeps float32's
+    exponent range, and its relative rounding error (2^-8) is several times below
+    the Monte-Carlo error of the RFF estimate itself (O(D^-1/2), Sec. 3.2),
+    so the stored features define a slightly different operator on which
+    Algorithm 2 then runs exactly.  Domain: finite |x| below the bf16
+    maximum; values under 2^-126 keep bf16's subnormal spacing 2^-133."""
+    x = np.asarray(x, dtype=np.float64)
+    _, e = np.frexp(x)                       # x = f 2^e, 1/2 <= |f| < 1
+    e = np.maximum(e, -125)                  # subnormal range: spacing 2^-133
+    scale = np.ldexp(1.0, e - 8)             # spacing of 8-bit significands
+    return np.round(x / scale) * scale       # np.round: ties to even
 
 
 # ---------------------------------------------------------------------------

@@ -59,17 +59,18 @@ class Config(ctypes.Structure):
         ("pos_mode", ctypes.c_int), ("renorm", ctypes.c_int),
         ("lanczos_tol", ctypes.c_double), ("window", ctypes.c_int),
         ("tau", ctypes.c_double), ("tau_schedule", ctypes.c_int),
-        ("normalize", ctypes.c_int),
+        ("normalize", ctypes.c_int), ("phi_dtype", ctypes.c_int),
     ]
 
     @classmethod
     def make(cls, backend=BACKEND_GLOBAL, rho=4.0, D=256, r=16, bits=0, preserve_first=0,
              preserve_last=12, pos_scheme=POS_MAX, pos_mode=MODE_REPRESENTATIVE, renorm=1,
              lanczos_tol=1e-10, window=2048, tau=0.70, tau_schedule=1,
-             normalize=0) -> "Config":
+             normalize=0, phi_dtype=SLS_F32) -> "Config":
+        """phi_dtype: storage of the feature matrix, SLS_F32 or SLS_BF16."""
         return cls(backend, float(rho), D, r, bits, preserve_first, preserve_last, pos_scheme,
                    pos_mode, int(renorm), float(lanczos_tol), window, float(tau),
-                   int(tau_schedule), int(normalize))
+                   int(tau_schedule), int(normalize), int(phi_dtype))
 
 
 class _Params(ctypes.Structure):
@@ -88,6 +89,9 @@ EXPORTED = {
     "sls_status_string": (ctypes.c_char_p, [_i32]),
     "sls_version": (_i32, []),
     "sls_feature_map": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _vp, _i32, _vp, _vp]),
+    "sls_feature_map_ex": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _vp, _i32, _vp, _i32, _vp]),
+    "sls_lanczos_topr_ex": (_i32, [_vp, _i32, _i64, _i32, _i32, _vp, _d, _vp, _vp, _vp, _vp,
+                                   _vp, _vp, _sz, _vp]),
     "sls_feature_normalize_workspace_size": (ctypes.c_size_t, [_i64, _i32]),
     "sls_feature_normalize": (_i32, [_vp, _i64, _i32, _vp, _vp, ctypes.c_size_t, _vp]),
     "sls_feature_map_batched": (_i32, [_vp, _i64, _i64, _i64, _i32, _i64, _vp, _vp, _i32, _vp,
@@ -171,18 +175,21 @@ def _workspace(nbytes: int, device) -> torch.Tensor:
 
 
 def feature_map(X: torch.Tensor, W: torch.Tensor, b: torch.Tensor,
-                out: Optional[torch.Tensor] = None) -> torch.Tensor:
+                out: Optional[torch.Tensor] = None,
+                phi_dtype: torch.dtype = torch.float32) -> torch.Tensor:
     """Phi = sqrt(2/D) cos(X W^T + b) (Sec. 3.2, Eq. rff_map); X is N x d,
-    W = Omega^T is D x d (same dtype), b has D floats.  Returns N x D float32."""
+    W = Omega^T is D x d (same dtype), b has D floats.  Returns N x D in
+    phi_dtype: float32, or bfloat16 (each feature rounded to nearest even)."""
     _need_cuda(X, W, b)
     N, d = X.shape
     D = W.shape[0]
     assert W.shape[1] == d and W.dtype == X.dtype and W.is_contiguous()
     if out is None:
-        out = torch.empty((N, D), dtype=torch.float32, device=X.device)
-    st = lib().sls_feature_map(_ptr(X), _dtype_code(X), N, d, X.stride(0), _ptr(W),
-                               _ptr(b.float().contiguous()), D, _ptr(out), _stream(X))
-    _check("sls_feature_map", st)
+        out = torch.empty((N, D), dtype=phi_dtype, device=X.device)
+    st = lib().sls_feature_map_ex(_ptr(X), _dtype_code(X), N, d, X.stride(0), _ptr(W),
+                                  _ptr(b.float().contiguous()), D, _ptr(out), _dtype_code(out),
+                                  _stream(X))
+    _check("sls_feature_map_ex", st)
     return out
 
 
@@ -231,8 +238,9 @@ def feature_normalize(Phi: torch.Tensor):
 
 def lanczos_topr(Phi: torch.Tensor, q1: torch.Tensor, r: int, tol: float = 1e-10):
     """Algorithm 2 on A(v) = Phi (Phi^T v), then Eigh(T) and U = Q V
-    (Algorithm 1).  Returns (theta[r] float64 descending, U[N, r] float32,
-    r_eff[1] int32, alpha[r], beta[r]) as device tensors."""
+    (Algorithm 1); Phi is float32 or bfloat16 (N x D).  Returns (theta[r]
+    float64 descending, U[N, r] float32, r_eff[1] int32, alpha[r], beta[r])
+    as device tensors."""
     _need_cuda(Phi, q1)
     Phi = Phi.contiguous()
     N, D = Phi.shape
@@ -248,10 +256,10 @@ def lanczos_topr(Phi: torch.Tensor, q1: torch.Tensor, r: int, tol: float = 1e-10
     if nbytes == 0:
         raise SLSError("sls_lanczos_workspace_size", 2, "unsupported shape")
     ws = _workspace(nbytes, dev)
-    st = L.sls_lanczos_topr(_ptr(Phi), N, D, r, _ptr(q1), float(tol), _ptr(theta), _ptr(U),
-                            _ptr(r_eff), _ptr(alpha), _ptr(beta), _ptr(ws), ws.numel(),
-                            _stream(Phi))
-    _check("sls_lanczos_topr", st)
+    st = L.sls_lanczos_topr_ex(_ptr(Phi), _dtype_code(Phi), N, D, r, _ptr(q1), float(tol),
+                               _ptr(theta), _ptr(U), _ptr(r_eff), _ptr(alpha), _ptr(beta),
+                               _ptr(ws), ws.numel(), _stream(Phi))
+    _check("sls_lanczos_topr_ex", st)
     return theta, U, r_eff, alpha, beta
 
 

@@ -264,6 +264,7 @@ struct CompressPlan {
   int seg_slots;
   int64_t k_chunk;
   int normalize;
+  int phi_bf16;
 };
 
 struct CompressWs {
@@ -278,7 +279,7 @@ struct CompressWs {
   float* score_part;  // window-score partial sums (adaptive backend)
   float2* norm_scratch;  // row-normalised operator: column sums
   int32_t* route;  // spectral flag per problem
-  float* Phi;
+  void* Phi;  // float32, or bfloat16 bits when the plan stores Phi as bf16
   float2* Q;
   double *alpha, *beta, *theta, *S;
   int* r_eff;
@@ -320,6 +321,7 @@ int make_plan(const sls_config_t* c, int64_t B, int64_t N, CompressPlan* P,
   P->r = c->r;
   P->k_chunk = chunk_k(c->rho);
   P->normalize = c->normalize ? 1 : 0;
+  P->phi_bf16 = (c->phi_dtype == SLS_BF16) ? 1 : 0;
   if (c->backend == SLS_BACKEND_CHUNK) {
     P->Mstar = (R.Nc + P->k_chunk - 1) / P->k_chunk;
     P->bud = Budgets{1, R.Nc, R.Nc, P->Mstar, P->Mstar, 0};
@@ -368,7 +370,7 @@ void carve(const CompressPlan& P, void* ws, CompressWs* W) {
   W->nspec = cv.take<int>(1);
   W->score = cv.take<float>(np);
   W->route = cv.take<int>(np);
-  W->Phi = cv.take<float>(spectral ? (size_t)rows * P.D : 0);
+  W->Phi = cv.take<char>(spectral ? (size_t)rows * P.D * (P.phi_bf16 ? 2 : 4) : 0);
   W->norm_scratch = cv.take<float2>(
       (spectral && P.normalize)
           ? feature_normalize_scratch_bytes(P.nmax, P.D, (int)P.nprob) / sizeof(float2)
@@ -409,6 +411,12 @@ int validate_config(const sls_config_t* c) {
   if (c->pos_scheme < 0 || c->pos_scheme > 2) return SLS_ERR_INVALID_ARG;
   if (c->pos_mode < 0 || c->pos_mode > 1) return SLS_ERR_INVALID_ARG;
   if (c->preserve_first < 0 || c->preserve_last < 0) return SLS_ERR_INVALID_ARG;
+  if (c->phi_dtype != SLS_F32 && c->phi_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
+  // bf16 storage: 16-byte rows for the bulk copies; the normalised operator
+  // scales float32 rows in place
+  if (c->phi_dtype == SLS_BF16 && c->rho > 1.0 && c->backend != SLS_BACKEND_CHUNK &&
+      ((c->D & 7) || c->normalize))
+    return SLS_ERR_UNSUPPORTED;
   return SLS_OK;
 }
 
@@ -458,6 +466,23 @@ int sls_feature_map(const void* X, int x_dtype, int64_t N, int d, int64_t ldx, c
   return launch_feature_map_simt(X, x_dtype, N, d, ldx, W, b, D, Phi, s);
 }
 
+int sls_feature_map_ex(const void* X, int x_dtype, int64_t N, int d, int64_t ldx, const void* W,
+                       const float* b, int D, void* Phi, int phi_dtype, void* stream) {
+  if (phi_dtype == SLS_F32)
+    return sls_feature_map(X, x_dtype, N, d, ldx, W, b, D, (float*)Phi, stream);
+  if (phi_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
+  if (N < 0 || d < 1 || D < 4 || D > SLS_MAX_D || (D & 3) || ldx < d) return SLS_ERR_INVALID_ARG;
+  if (x_dtype != SLS_F32 && x_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
+  if (N == 0) return SLS_OK;
+  if (!X || !W || !b || !Phi) return SLS_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (x_dtype == SLS_BF16) {
+    const int st = launch_feature_map_tc(X, N, d, ldx, W, b, D, Phi, s, nullptr, 1);
+    if (st != SLS_ERR_UNSUPPORTED) return st;
+  }
+  return launch_feature_map_simt(X, x_dtype, N, d, ldx, W, b, D, Phi, s, 1);
+}
+
 int sls_feature_map_batched(const void* X, int64_t nb, int64_t rows, int64_t x_stride, int d,
                             int64_t ldx, const void* W, const float* b, int D, float* Phi,
                             const int32_t* live, int nwin, int win, void* stream) {
@@ -503,9 +528,17 @@ size_t sls_lanczos_workspace_size(int64_t N, int D, int r) {
 int sls_lanczos_topr(const float* Phi, int64_t N, int D, int r, const double* q1, double tol,
                      double* theta, float* U, int32_t* r_eff, double* alpha, double* beta,
                      void* workspace, size_t workspace_bytes, void* stream) {
+  return sls_lanczos_topr_ex(Phi, SLS_F32, N, D, r, q1, tol, theta, U, r_eff, alpha, beta,
+                             workspace, workspace_bytes, stream);
+}
+
+int sls_lanczos_topr_ex(const void* Phi, int phi_dtype, int64_t N, int D, int r, const double* q1,
+                        double tol, double* theta, float* U, int32_t* r_eff, double* alpha,
+                        double* beta, void* workspace, size_t workspace_bytes, void* stream) {
   if (N < 1 || D < 4 || D > SLS_MAX_D || r < 1 || r > SLS_MAX_R || !(tol >= 0.0))
     return SLS_ERR_INVALID_ARG;
-  if ((D & 3) != 0) return SLS_ERR_UNSUPPORTED;
+  if (phi_dtype != SLS_F32 && phi_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
+  if ((D & 3) != 0 || (phi_dtype == SLS_BF16 && (D & 7) != 0)) return SLS_ERR_UNSUPPORTED;
   if (!ptr_ok(Phi) || !q1 || !theta || !U || !r_eff) return SLS_ERR_INVALID_ARG;
   const size_t need = sls_lanczos_workspace_size(N, D, r);
   if (need == 0) return SLS_ERR_UNSUPPORTED;
@@ -525,6 +558,7 @@ int sls_lanczos_topr(const float* Phi, int64_t N, int D, int r, const double* q1
   SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
   LanczosBatch bt{};
   bt.Phi = Phi;
+  bt.phi_bf16 = (phi_dtype == SLS_BF16) ? 1 : 0;
   bt.D = D;
   bt.r = r;
   bt.tol = tol;
@@ -707,13 +741,15 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
       st = launch_feature_map_tc_batched(
           (const char*)X + (size_t)P.pf * ldx * 2, B, P.Nc, N, d, ldx, params->W, params->b,
           cfg->D, W.Phi, mode == 2 ? rflags : nullptr, (int)P.bud.W, (int)P.bud.L_full, s,
-          W.status);
+          W.status, P.phi_bf16);
     if (st == SLS_ERR_UNSUPPORTED) {
+      const size_t esz = P.phi_bf16 ? 2 : 4;
       for (int64_t b = 0; b < B; ++b) {
         const char* xb = (const char*)X +
                          (size_t)(b * N + P.pf) * ldx * (x_dtype == SLS_BF16 ? 2 : 4);
-        st = sls_feature_map(xb, x_dtype, P.Nc, d, ldx, params->W, params->b, cfg->D,
-                             W.Phi + (size_t)b * P.Nc * cfg->D, stream);
+        st = sls_feature_map_ex(xb, x_dtype, P.Nc, d, ldx, params->W, params->b, cfg->D,
+                                (char*)W.Phi + (size_t)b * P.Nc * cfg->D * esz,
+                                P.phi_bf16 ? SLS_BF16 : SLS_F32, stream);
         if (st != SLS_OK) return st;
       }
     }
@@ -721,13 +757,14 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
     // the row-normalised operator: each spectral problem's rows scaled by
     // 1 / sqrt of its estimated row sums (Sec. 3.2)
     if (cfg->normalize &&
-        (st = launch_feature_normalize(W.Phi, cfg->D, W.lz_row0, W.lz_n, nprob, W.nspec, 0,
+        (st = launch_feature_normalize((float*)W.Phi, cfg->D, W.lz_row0, W.lz_n, nprob, W.nspec, 0,
                                        P.nmax, W.norm_scratch, nullptr, s)) != SLS_OK)
       return st;
     phase_mark(1, 1, s);
     phase_mark(2, 0, s);
     LanczosBatch bt{};
     bt.Phi = W.Phi;
+    bt.phi_bf16 = P.phi_bf16;
     bt.D = cfg->D;
     bt.r = cfg->r;
     bt.tol = cfg->lanczos_tol;

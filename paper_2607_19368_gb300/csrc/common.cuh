@@ -13,6 +13,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "../../include/sls.h"
@@ -60,6 +61,27 @@ SLS_DEV dfloat df_from_double(double x) {
 SLS_DEV double df_to_double(dfloat a) { return (double)a.hi + (double)a.lo; }
 
 SLS_DEV float2 f2(dfloat a) { return make_float2(a.hi, a.lo); }
+
+// Elements of the feature matrix as stored: float32, or raw bfloat16 bits
+// (uint16), widened to float32 exactly.  phi_ld reads through the read-only
+// cache (global memory); phi_ld4 reads the four elements 4 g .. 4 g + 3 of a
+// row in shared or global memory (16-byte aligned for float32, 8 for bf16).
+SLS_DEV float bf16_bits_to_float(uint32_t u) { return __uint_as_float(u << 16); }
+SLS_DEV float phi_ld(const float* p, size_t i) { return __ldg(p + i); }
+SLS_DEV float phi_ld(const uint16_t* p, size_t i) {
+  return bf16_bits_to_float((uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p) + i));
+}
+// Stores of a feature value: float32 as is, bfloat16 rounded to nearest even.
+SLS_DEV void phi_st(float* p, float v) { *p = v; }
+SLS_DEV void phi_st(uint16_t* p, float v) {
+  *reinterpret_cast<unsigned short*>(p) = __bfloat16_as_ushort(__float2bfloat16_rn(v));
+}
+SLS_DEV float4 phi_ld4(const float* p, size_t g) { return reinterpret_cast<const float4*>(p)[g]; }
+SLS_DEV float4 phi_ld4(const uint16_t* p, size_t g) {
+  const uint2 u = reinterpret_cast<const uint2*>(p)[g];
+  return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                     __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+}
 SLS_DEV dfloat dfv(float2 a) { return df_make(a.x, a.y); }
 
 SLS_DEV dfloat df_norm(float s, float e) {

@@ -5,7 +5,8 @@
 // This file holds the fp32 SIMT kernel (used for float32 embeddings and as
 // the reference path for small shapes); the bf16 tcgen05 kernel lives in
 // feature_map_tc.cu.  Both fuse the bias, cosine and scale into the epilogue,
-// so Phi is written exactly once.
+// so Phi is written exactly once, as float32 or (opt-in) as bfloat16 rounded
+// to nearest even from the float32 value.
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -31,12 +32,13 @@ SLS_DEV float load_elem<uint16_t>(const uint16_t* p) {
   return __uint_as_float(((unsigned)*p) << 16);
 }
 
-// One CTA computes a 64 x 64 tile; each thread a 4 x 4 block.
-template <typename T>
+// One CTA computes a 64 x 64 tile; each thread a 4 x 4 block.  T: element
+// type of X and W; OT: of Phi (float, or uint16_t for bfloat16).
+template <typename T, typename OT>
 __global__ void __launch_bounds__(FM_THREADS)
 feature_map_simt_kernel(const T* __restrict__ X, int64_t N, int d, int64_t ldx,
                         const T* __restrict__ W, const float* __restrict__ bvec,
-                        int D, float scale, float* __restrict__ Phi) {
+                        int D, float scale, OT* __restrict__ Phi) {
   __shared__ float As[FM_BK][FM_BM + 4];
   __shared__ float Bs[FM_BK][FM_BN + 4];
   const int tid = threadIdx.x;
@@ -83,27 +85,35 @@ feature_map_simt_kernel(const T* __restrict__ X, int64_t N, int d, int64_t ldx,
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       int c = col0 + tx * 4 + j;
-      if (c < D) Phi[gr * D + c] = scale * cosf(acc[i][j] + bvec[c]);
+      if (c < D) phi_st(Phi + gr * D + c, scale * cosf(acc[i][j] + bvec[c]));
     }
   }
+}
+
+template <typename T>
+void launch_simt_t(const void* X, int64_t N, int d, int64_t ldx, const void* W, const float* b,
+                   int D, float scale, void* Phi, int phi_bf16, dim3 grid, cudaStream_t stream) {
+  if (phi_bf16)
+    feature_map_simt_kernel<T, uint16_t><<<grid, FM_THREADS, 0, stream>>>(
+        (const T*)X, N, d, ldx, (const T*)W, b, D, scale, (uint16_t*)Phi);
+  else
+    feature_map_simt_kernel<T, float><<<grid, FM_THREADS, 0, stream>>>(
+        (const T*)X, N, d, ldx, (const T*)W, b, D, scale, (float*)Phi);
 }
 
 }  // namespace
 
 int launch_feature_map_simt(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
-                            const void* W, const float* b, int D, float* Phi,
-                            cudaStream_t stream) {
+                            const void* W, const float* b, int D, void* Phi,
+                            cudaStream_t stream, int phi_bf16) {
   if (N == 0) return SLS_OK;
   const float scale = (float)sqrt(2.0 / (double)D);
   dim3 grid((D + FM_BN - 1) / FM_BN, (unsigned)((N + FM_BM - 1) / FM_BM));
   if (grid.y > 65535u) return SLS_ERR_UNSUPPORTED;
-  if (x_dtype == SLS_F32) {
-    feature_map_simt_kernel<float><<<grid, FM_THREADS, 0, stream>>>(
-        (const float*)X, N, d, ldx, (const float*)W, b, D, scale, Phi);
-  } else {
-    feature_map_simt_kernel<uint16_t><<<grid, FM_THREADS, 0, stream>>>(
-        (const uint16_t*)X, N, d, ldx, (const uint16_t*)W, b, D, scale, Phi);
-  }
+  if (x_dtype == SLS_F32)
+    launch_simt_t<float>(X, N, d, ldx, W, b, D, scale, Phi, phi_bf16, grid, stream);
+  else
+    launch_simt_t<uint16_t>(X, N, d, ldx, W, b, D, scale, Phi, phi_bf16, grid, stream);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }

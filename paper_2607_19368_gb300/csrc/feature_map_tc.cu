@@ -2,7 +2,8 @@
 //   Phi = sqrt(2/D) * cos(X W^T + b)      (Sec. 3.2, Eq. rff_map)
 // X (N x d) and W = Omega^T (D x d) are bf16, K-major (row-major, K = d
 // contiguous); the contraction accumulates in fp32 in tensor memory; the
-// epilogue adds b, takes the cosine, scales and stores Phi (fp32) once.
+// epilogue adds b, takes the cosine, scales and stores Phi once (float32, or
+// bfloat16 rounded to nearest even when the caller asks for bf16 storage).
 //
 // One persistent CTA per SM, 128 x 256 output tiles (tile index -> prompt,
 // then m-block, then n-block innermost, so the D/256 tiles that share an X
@@ -134,10 +135,23 @@ SLS_DEV bool fm_tile_live(const FmJob& J, int b, int mb) {
   return false;
 }
 
+// Four consecutive features: one 16-byte store (float32), or one 8-byte
+// store of four bfloat16 values rounded to nearest even.
+SLS_DEV void store4(float* p, float4 o) { *reinterpret_cast<float4*>(p) = o; }
+SLS_DEV void store4(uint16_t* p, float4 o) {
+  const __nv_bfloat162 a = __floats2bfloat162_rn(o.x, o.y), b = __floats2bfloat162_rn(o.z, o.w);
+  uint2 u;
+  u.x = *reinterpret_cast<const unsigned*>(&a);
+  u.y = *reinterpret_cast<const unsigned*>(&b);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+
+// OT: element type of Phi (float, or uint16_t for bfloat16 storage).
+template <typename OT>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
                       const __grid_constant__ CUtensorMap tmW, const float* __restrict__ bvec,
-                      float* __restrict__ Phi, FmJob J, int D, int K, float scale, int* status) {
+                      OT* __restrict__ Phi, FmJob J, int D, int K, float scale, int* status) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES], tfull[2], tempty[2], done_bar;
   __shared__ uint32_t tmem_holder;
@@ -276,7 +290,7 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       }
       tc_fence_after();
       const int row = mb * TC_BM + q * 32 + lane;
-      float* out = Phi + ((int64_t)pb * J.rows + row) * D + (int64_t)nb * TC_BN;
+      OT* out = Phi + ((int64_t)pb * J.rows + row) * D + (int64_t)nb * TC_BN;
       const float* bb = bvec + (size_t)nb * TC_BN;
       for (int c0 = 0; c0 < TC_BN; c0 += 32) {
         uint32_t v[32];
@@ -290,7 +304,7 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
             o.y = scale * cosf(__uint_as_float(v[e + 1]) + bq.y);
             o.z = scale * cosf(__uint_as_float(v[e + 2]) + bq.z);
             o.w = scale * cosf(__uint_as_float(v[e + 3]) + bq.w);
-            *reinterpret_cast<float4*>(out + c0 + e) = o;
+            store4(out + c0 + e, o);
           }
         }
       }
@@ -359,8 +373,8 @@ int sm_count() {
 
 int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64_t x_stride,
                                   int d, int64_t ldx, const void* W, const float* b, int D,
-                                  float* Phi, const int* live, int nwin, int win,
-                                  cudaStream_t stream, int* status) {
+                                  void* Phi, const int* live, int nwin, int win,
+                                  cudaStream_t stream, int* status, int phi_bf16) {
   // shapes the kernel covers; anything else takes the SIMT path
   if (nb <= 0 || rows <= 0 || x_stride < rows || D % TC_BN != 0 || d % 8 != 0 || ldx % 8 != 0)
     return SLS_ERR_UNSUPPORTED;
@@ -377,23 +391,29 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
   if (!make_map(&mw, W, (uint64_t)D, (uint64_t)d, (uint64_t)d, TC_BN)) return SLS_ERR_UNSUPPORTED;
   int* st = status;
   if (!st) SLS_CUDA_TRY(cudaGetSymbolAddress((void**)&st, g_fm_status));
-  SLS_CUDA_TRY(cudaFuncSetAttribute(feature_map_tc_kernel,
+  SLS_CUDA_TRY(cudaFuncSetAttribute(feature_map_tc_kernel<float>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TC_SMEM));
+  SLS_CUDA_TRY(cudaFuncSetAttribute(feature_map_tc_kernel<uint16_t>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TC_SMEM));
   const int64_t tiles = nb * m_tiles * (D / TC_BN);
   const int grid = tiles < sm_count() ? (int)tiles : sm_count();
   const float scale = (float)sqrt(2.0 / (double)D);
   FmJob J{(int)nb, (int)rows, (int)x_stride, live, nwin, win};
-  feature_map_tc_kernel<<<grid, TC_THREADS, TC_SMEM, stream>>>(mx, mw, b, Phi, J, D, d, scale,
-                                                               st);
+  if (phi_bf16)
+    feature_map_tc_kernel<uint16_t><<<grid, TC_THREADS, TC_SMEM, stream>>>(
+        mx, mw, b, (uint16_t*)Phi, J, D, d, scale, st);
+  else
+    feature_map_tc_kernel<float><<<grid, TC_THREADS, TC_SMEM, stream>>>(mx, mw, b, (float*)Phi, J,
+                                                                      D, d, scale, st);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
 
 int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
-                          const float* b, int D, float* Phi, cudaStream_t stream,
-                          int* status) {
+                          const float* b, int D, void* Phi, cudaStream_t stream,
+                          int* status, int phi_bf16) {
   return launch_feature_map_tc_batched(X, 1, N, N, d, ldx, W, b, D, Phi, nullptr, 0, 0, stream,
-                                       status);
+                                       status, phi_bf16);
 }
 
 }  // namespace sls

@@ -7,22 +7,24 @@
 namespace sls {
 
 // ---- feature map (Sec. 3.2) ----------------------------------------------
+// Phi is written as float32, or as bfloat16 (round to nearest even from the
+// float32 value) when phi_bf16 is set.
 int launch_feature_map_simt(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
-                            const void* W, const float* b, int D, float* Phi,
-                            cudaStream_t stream);
+                            const void* W, const float* b, int D, void* Phi,
+                            cudaStream_t stream, int phi_bf16 = 0);
 // tcgen05 / TMA path for bf16 inputs; returns SLS_ERR_UNSUPPORTED when the
 // shape is outside what the kernel handles (the caller then uses the SIMT path).
 int launch_feature_map_tc(const void* X, int64_t N, int d, int64_t ldx, const void* W,
-                          const float* b, int D, float* Phi, cudaStream_t stream,
-                          int* status = nullptr);
+                          const float* b, int D, void* Phi, cudaStream_t stream,
+                          int* status = nullptr, int phi_bf16 = 0);
 // The same over nb prompts in one launch: prompt k has `rows` rows starting at
 // X row k * x_stride and writes Phi rows [k * rows, (k + 1) * rows).  With
 // `live` set (one flag per window of `win` rows, nwin per prompt,
 // prompt-major), row tiles whose windows are all 0 are not computed.
 int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64_t x_stride,
                                   int d, int64_t ldx, const void* W, const float* b, int D,
-                                  float* Phi, const int* live, int nwin, int win,
-                                  cudaStream_t stream, int* status);
+                                  void* Phi, const int* live, int nwin, int win,
+                                  cudaStream_t stream, int* status, int phi_bf16 = 0);
 
 // ---- input embeddings: X = E[ids] (Sec. 3.1) ---------------------------------
 // Rows of a V x d table (row stride ld_table elements) gathered into X (row
@@ -49,7 +51,7 @@ __host__ __device__ inline int q_ld(int r) { return (r + 1) & ~1; }
 // A batch of independent problems, problem p owning rows
 // [row0[p], row0[p] + n[p]) of Phi, Q and U and start vector q1 + q1off[p].
 struct LanczosBatch {
-  const float* Phi;     // rows x D
+  const void* Phi;      // rows x D: float32, or raw bfloat16 bits when phi_bf16
   int D;
   int r;
   double tol;
@@ -71,6 +73,7 @@ struct LanczosBatch {
   double* S;
   int* r_eff;
   int64_t nmax;             // max rows of any problem
+  int phi_bf16;             // Phi stored as bfloat16 (D % 8 == 0)
 };
 
 size_t lanczos_scratch_bytes(int64_t nmax, int D, int r, int groups, int ctas_per_group);

@@ -518,18 +518,31 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
                        16 + 2 * RING_MAX_STAGES * 8;
   const size_t limit = 227 * 1024 - 1024;  // leave room for static shared memory
   if (other >= limit) return SLS_ERR_UNSUPPORTED;
-  const RingShape R = ring_shape(bt.D, q_ld(bt.r), limit - other);
+  if (bt.phi_bf16 && (bt.D % 8)) return SLS_ERR_UNSUPPORTED;  // 16-byte rows for the copies
+  const RingShape R = ring_shape(bt.D, q_ld(bt.r), limit - other, bt.phi_bf16 ? 2 : 4);
   if (R.S < 2) return SLS_ERR_UNSUPPORTED;
   const size_t smem = (size_t)R.S * R.stage + other;
   const int stages = R.S;
   const int kt = (bt.r <= 32) ? 1 : (bt.r <= 64) ? 2 : 4;  // 32-wide tiles of k < r
-  switch (gpt_of(bt.D)) {
-    case 1: return launch_lanczos_gpt1(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream, kt);
-    case 2: return launch_lanczos_gpt2(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream, kt);
-    case 4: return launch_lanczos_gpt4(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream, kt);
-    case 8: return launch_lanczos_gpt8(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream, kt);
-    default: break;
+#define SLS_LZ_CALL(fn) fn(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream, kt)
+  if (bt.phi_bf16) {
+    switch (gpt_of(bt.D)) {
+      case 1: return SLS_LZ_CALL(launch_lanczos_bf16_gpt1);
+      case 2: return SLS_LZ_CALL(launch_lanczos_bf16_gpt2);
+      case 4: return SLS_LZ_CALL(launch_lanczos_bf16_gpt4);
+      case 8: return SLS_LZ_CALL(launch_lanczos_bf16_gpt8);
+      default: break;
+    }
+  } else {
+    switch (gpt_of(bt.D)) {
+      case 1: return SLS_LZ_CALL(launch_lanczos_gpt1);
+      case 2: return SLS_LZ_CALL(launch_lanczos_gpt2);
+      case 4: return SLS_LZ_CALL(launch_lanczos_gpt4);
+      case 8: return SLS_LZ_CALL(launch_lanczos_gpt8);
+      default: break;
+    }
   }
+#undef SLS_LZ_CALL
   return SLS_ERR_UNSUPPORTED;
 }
 

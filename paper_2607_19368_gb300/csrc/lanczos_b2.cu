@@ -1,0 +1,13 @@
+// Lanczos kernel instantiations for 2 four-element column group(s) of Phi
+// per compute thread (D <= 2048), Phi stored as bfloat16, for every basis tile
+// count KT.
+#include "lanczos_kernel.cuh"
+
+namespace sls {
+
+int launch_lanczos_bf16_gpt2(SLS_LZ_LAUNCH_ARGS) {
+  return launch_lanczos_kt<2, uint16_t>(bt, scratch, gstride, groups, g, rows_cap, stages,
+                                         status, smem, stream, kt);
+}
+
+}  // namespace sls

@@ -1,16 +1,12 @@
-// Lanczos kernel instantiations for 1 float4 column group of Phi per compute
-// thread (D <= 1024), for every basis tile count KT.
+// Lanczos kernel instantiations for 1 float4 column group(s) of Phi per
+// compute thread (D <= 1024), float32 Phi, for every basis tile count KT.
 #include "lanczos_kernel.cuh"
 
 namespace sls {
 
 int launch_lanczos_gpt1(SLS_LZ_LAUNCH_ARGS) {
-  switch (kt) {
-    case 1: return launch_lanczos_t<1, 1>(bt, scratch, gstride, groups, g, rows_cap, stages, status, smem, stream);
-    case 2: return launch_lanczos_t<1, 2>(bt, scratch, gstride, groups, g, rows_cap, stages, status, smem, stream);
-    case 4: return launch_lanczos_t<1, 4>(bt, scratch, gstride, groups, g, rows_cap, stages, status, smem, stream);
-    default: return SLS_ERR_UNSUPPORTED;
-  }
+  return launch_lanczos_kt<1, float>(bt, scratch, gstride, groups, g, rows_cap, stages, status,
+                                      smem, stream, kt);
 }
 
 }  // namespace sls

@@ -1,16 +1,12 @@
-// Lanczos kernel instantiations for 8 float4 column groups of Phi per compute
-// thread (D <= 8192), for every basis tile count KT.
+// Lanczos kernel instantiations for 8 float4 column group(s) of Phi per
+// compute thread (D <= 8192), float32 Phi, for every basis tile count KT.
 #include "lanczos_kernel.cuh"
 
 namespace sls {
 
 int launch_lanczos_gpt8(SLS_LZ_LAUNCH_ARGS) {
-  switch (kt) {
-    case 1: return launch_lanczos_t<8, 1>(bt, scratch, gstride, groups, g, rows_cap, stages, status, smem, stream);
-    case 2: return launch_lanczos_t<8, 2>(bt, scratch, gstride, groups, g, rows_cap, stages, status, smem, stream);
-    case 4: return launch_lanczos_t<8, 4>(bt, scratch, gstride, groups, g, rows_cap, stages, status, smem, stream);
-    default: return SLS_ERR_UNSUPPORTED;
-  }
+  return launch_lanczos_kt<8, float>(bt, scratch, gstride, groups, g, rows_cap, stages, status,
+                                      smem, stream, kt);
 }
 
 }  // namespace sls

@@ -89,7 +89,8 @@ SLS_DEV dfloat shfl_df(dfloat v, int src) {
   return v;
 }
 
-// Ring stage: cr rows of Phi (cr * D floats) followed by the same cr rows of
+// Ring stage: cr rows of Phi (cr * D elements of esz bytes: 4 for float32, 2
+// for bfloat16) followed by the same cr rows of
 // the basis Q (cr * ldq float2).  For D >= 4 * LZ_CT (one column group per
 // compute thread or more) a stage holds team_rows(GPT) rows, so that the team
 // row dots give every compute thread the same number of elements per chunk;
@@ -115,15 +116,15 @@ __host__ __device__ inline int gpt_of(int D) {
 // per thread per chunk)
 __host__ __device__ constexpr int team_rows(int gpt) { return gpt >= 8 ? 1 : 8 / gpt; }
 
-__host__ __device__ inline RingShape ring_shape(int D, int ldq, size_t budget) {
+__host__ __device__ inline RingShape ring_shape(int D, int ldq, size_t budget, int esz) {
   RingShape R;
   if (D / 4 >= LZ_CT) {
     R.cr = team_rows(gpt_of(D));
   } else {
-    R.cr = RING_STAGE / (4 * D + 8 * ldq);
+    R.cr = RING_STAGE / (esz * D + 8 * ldq);
     if (R.cr < 1) R.cr = 1;
   }
-  R.phib = (unsigned)R.cr * (unsigned)D * 4u;
+  R.phib = (unsigned)R.cr * (unsigned)D * (unsigned)esz;
   R.stage = R.phib + (unsigned)R.cr * (unsigned)ldq * 8u;
   R.S = (int)(budget / R.stage);
   if (R.S > RING_MAX_STAGES) R.S = RING_MAX_STAGES;
@@ -133,8 +134,8 @@ __host__ __device__ inline RingShape ring_shape(int D, int ldq, size_t budget) {
 // Sweep A over one chunk: acc[c] += Phi[i, c] * z1_i for the chunk's rows,
 // column-parallel (GPT float4 groups per thread, P row phases), Dot2.  With
 // TRACK the thread also keeps the largest |Phi| it has seen in *mx.
-template <int GPT, bool TRACK>
-SLS_DEV void sweepA_chunk(const float* __restrict__ chunk, int nr, int D, int lb,
+template <int GPT, bool TRACK, typename PT>
+SLS_DEV void sweepA_chunk(const PT* __restrict__ chunk, int nr, int D, int lb,
                           const float2* __restrict__ us, f32x2_t (&ah)[GPT][2],
                           f32x2_t (&al)[GPT][2], float* mx) {
   const int tid = threadIdx.x;
@@ -143,7 +144,6 @@ SLS_DEV void sweepA_chunk(const float* __restrict__ chunk, int nr, int D, int lb
   if (P > 1 && tid >= P * C4) return;
   const int ph = (P == 1) ? 0 : tid / C4;
   const int cb = (P == 1) ? tid : tid % C4;
-  const float4* c4 = reinterpret_cast<const float4*>(chunk);
   for (int i = ph; i < nr; i += P) {
     const float2 u = us[lb + i];
     const f32x2_t uh = pk2(u.x, u.x), nuh = pk2(-u.x, -u.x), ul = pk2(u.y, u.y);
@@ -151,7 +151,7 @@ SLS_DEV void sweepA_chunk(const float* __restrict__ chunk, int nr, int D, int lb
     for (int q = 0; q < GPT; ++q) {
       const int cg = cb + q * LZ_CT;
       if (cg < C4) {
-        const float4 f = c4[i * C4 + cg];
+        const float4 f = phi_ld4(chunk, (size_t)i * C4 + cg);
         dot2_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
         dot2_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
         if (TRACK)
@@ -196,9 +196,9 @@ SLS_DEV float transpose_sum_f(float (&v)[CR]) {
 // second chunk may be absent: nr1 = 0): acc[c] += Phi[i, c] * z'_i, Dot2.
 // FULL: both chunks full and D = 4 LZ_CT GPT (the steady state), so the row
 // and column guards vanish.
-template <int GPT, int CR, bool FULL>
-SLS_DEV void sweepA_team_pair(const float* __restrict__ c0, int nr0, int lb0,
-                              const float* __restrict__ c1, int nr1, int lb1, int C4,
+template <int GPT, int CR, bool FULL, typename PT>
+SLS_DEV void sweepA_team_pair(const PT* __restrict__ c0, int nr0, int lb0,
+                              const PT* __restrict__ c1, int nr1, int lb1, int C4,
                               const float2* __restrict__ us, f32x2_t (&ah)[GPT][2],
                               f32x2_t (&al)[GPT][2]) {
   const int tid = threadIdx.x;
@@ -207,14 +207,14 @@ SLS_DEV void sweepA_team_pair(const float* __restrict__ c0, int nr0, int lb0,
     const bool first = i < CR;
     const int ii = first ? i : i - CR;
     if (FULL || ii < (first ? nr0 : nr1)) {
-      const float4* c4 = reinterpret_cast<const float4*>(first ? c0 : c1);
+      const PT* ch = first ? c0 : c1;
       const float2 u = us[(first ? lb0 : lb1) + ii];
       const f32x2_t uh = pk2(u.x, u.x), nuh = pk2(-u.x, -u.x), ul = pk2(u.y, u.y);
 #pragma unroll
       for (int q = 0; q < GPT; ++q) {
         const int cg = tid + q * LZ_CT;
         if (FULL || cg < C4) {
-          const float4 f = c4[ii * C4 + cg];
+          const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
           dot2_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
           dot2_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
         }
@@ -269,8 +269,8 @@ SLS_DEV dfloat transpose_sum_df(dfloat (&v)[CR]) {
 // loose global bound; the 2 CR per-row double-float partials are then summed
 // over the warp by one transposed butterfly and the warp sums stored to
 // bp0 / bp1 [i * LZ_CW + warp].
-template <int GPT, int CR, bool FULL>
-SLS_DEV void sweepB_team_pair(const float* __restrict__ c0, int nr0, const float* __restrict__ c1,
+template <int GPT, int CR, bool FULL, typename PT>
+SLS_DEV void sweepB_team_pair(const PT* __restrict__ c0, int nr0, const PT* __restrict__ c1,
                               int nr1, int C4, const f32x2_t (&wh)[GPT][2],
                               const f32x2_t (&nwh)[GPT][2], const f32x2_t (&wl)[GPT][2],
                               float Ct, float2* __restrict__ bp0, float2* __restrict__ bp1) {
@@ -283,12 +283,12 @@ SLS_DEV void sweepB_team_pair(const float* __restrict__ c0, int nr0, const float
     const int ii = first ? i : i - CR;
     f32x2_t s = pk2(Ct, Ct), lo = 0ull;
     if (FULL || ii < (first ? nr0 : nr1)) {
-      const float4* c4 = reinterpret_cast<const float4*>(first ? c0 : c1);
+      const PT* ch = first ? c0 : c1;
 #pragma unroll
       for (int q = 0; q < GPT; ++q) {
         const int cg = tid + q * LZ_CT;
         if (FULL || cg < C4) {
-          const float4 f = c4[ii * C4 + cg];
+          const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
           ofs_acc2n(s, lo, pk2(f.x, f.y), wh[q][0], nwh[q][0], wl[q][0]);
           ofs_acc2n(s, lo, pk2(f.z, f.w), wh[q][1], nwh[q][1], wl[q][1]);
         }
@@ -315,16 +315,16 @@ SLS_DEV void sweepB_team_pair(const float* __restrict__ c0, int nr0, const float
 
 // Row dot product with w from shared memory (separate hi / lo arrays); one
 // warp per row, all lanes get the sum.  Used by sweep B when D < 4 * LZ_CT.
-SLS_DEV dfloat row_dot_smem(const float* __restrict__ row, int D, const float* __restrict__ wsh,
+template <typename PT>
+SLS_DEV dfloat row_dot_smem(const PT* __restrict__ row, int D, const float* __restrict__ wsh,
                             const float* __restrict__ wsl) {
   const int lane = threadIdx.x & 31;
   const int C4 = D >> 2;
-  const float4* r4 = reinterpret_cast<const float4*>(row);
   const float4* h4 = reinterpret_cast<const float4*>(wsh);
   const float4* l4 = reinterpret_cast<const float4*>(wsl);
   f32x2_t h01 = 0, l01 = 0, h23 = 0, l23 = 0;
   for (int cg = lane; cg < C4; cg += 32) {
-    const float4 f = r4[cg];
+    const float4 f = phi_ld4(row, cg);
     const float4 wh = h4[cg], wl = l4[cg];
     dot2_acc2(h01, l01, pk2(f.x, f.y), pk2(wh.x, wh.y), pk2(wl.x, wl.y));
     dot2_acc2(h23, l23, pk2(f.z, f.w), pk2(wh.z, wh.w), pk2(wl.z, wl.w));
@@ -654,7 +654,7 @@ SLS_DEV void row_phase(float2* __restrict__ Qs, int ldq, int wr0, int wr1, int j
   }
 }
 
-template <int GPT, int KT>
+template <int GPT, int KT, typename PT>
 __global__ void __launch_bounds__(LZ_THREADS, 1)
 lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroups,
                int rows_cap, int ring_stages, int* status) {
@@ -683,7 +683,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   const int redn = (P > 1) ? P * D : 0;
   const bool fullD = (C4 == GPT * LZ_CT);  // no ragged column groups
 
-  const RingShape shp0 = ring_shape(D, ldq, 0);
+  const RingShape shp0 = ring_shape(D, ldq, 0, (int)sizeof(PT));
   const int S = ring_stages;
   const int cr = shp0.cr;
   const unsigned stage = shp0.stage, phib = shp0.phib;
@@ -759,7 +759,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
       const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
       const int nch = (int)((re - rs + cr - 1) / cr);
-      const float* Phi = bt.Phi + (row0 + rs) * D;
+      const PT* Phi = reinterpret_cast<const PT*>(bt.Phi) + (row0 + rs) * D;
       const float2* Qs = bt.Q + (row0 + rs) * ldq;
       bool stop = false;
       for (int pass = 0; pass < r && !stop; ++pass) {
@@ -796,7 +796,8 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
             break;
           }
           const int64_t nr = min((int64_t)cr, (re - rs) - (int64_t)k * cr);
-          const unsigned b1 = (unsigned)(nr * D * 4), b2 = (unsigned)(nr * ldq * 8);
+          const unsigned b1 = (unsigned)(nr * D * (int64_t)sizeof(PT));
+          const unsigned b2 = (unsigned)(nr * ldq * 8);
           unsigned char* dst = ring + (size_t)slot * stage;
           mbar_expect_tx(&fullb[slot], b1 + b2);
           bulk_g2s(dst, Phi + (int64_t)k * cr * D, b1, &fullb[slot], pol);
@@ -861,7 +862,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       for (int t = 0; t < nch; ++t) {
         const int slot = rc.slot;
         if (!mbar_wait(&fullb[slot], rc.par)) lz_fail(status, &s_err);
-        const float* chunk = reinterpret_cast<const float*>(ring + (size_t)slot * stage);
+        const PT* chunk = reinterpret_cast<const PT*>(ring + (size_t)slot * stage);
         const int nr = min(cr, nrows - t * cr);
         sweepA_chunk<GPT, true>(chunk, nr, D, t * cr, zps, ah, al, &mx);
         __syncwarp();
@@ -1064,8 +1065,8 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
             if (!mbar_wait(&fullb[s1], rc.par)) lz_fail(status, &s_err);
             rc_next(rc, S);
           }
-          const float* ch0 = reinterpret_cast<const float*>(ring + (size_t)s0 * stage);
-          const float* ch1 = reinterpret_cast<const float*>(ring + (size_t)s1 * stage);
+          const PT* ch0 = reinterpret_cast<const PT*>(ring + (size_t)s0 * stage);
+          const PT* ch1 = reinterpret_cast<const PT*>(ring + (size_t)s1 * stage);
           const float2* qb0 = reinterpret_cast<const float2*>(ring + (size_t)s0 * stage + phib);
           const float2* qb1 = reinterpret_cast<const float2*>(ring + (size_t)s1 * stage + phib);
           const int nr0 = min(cr, nrows - kc0 * cr);
@@ -1147,7 +1148,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           const int slot = rc.slot;
           if (!mbar_wait(&fullb[slot], rc.par))
             lz_fail(status, &s_err);  // leave at the next group barrier
-          const float* chunk = reinterpret_cast<const float*>(ring + (size_t)slot * stage);
+          const PT* chunk = reinterpret_cast<const PT*>(ring + (size_t)slot * stage);
           const float2* qblk = reinterpret_cast<const float2*>(ring + (size_t)slot * stage + phib);
           const int nr = min(cr, nrows - kc * cr);
           for (int ii = warp; ii < nr; ii += LZ_CW) {
@@ -1225,10 +1226,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   }
 }
 
-template <int GPT, int KT>
+template <int GPT, int KT, typename PT>
 int launch_lanczos_t(const LanczosBatch& bt, void* scratch, size_t gstride, int groups, int g,
                      int rows_cap, int stages, int* status, size_t smem, cudaStream_t stream) {
-  auto fn = lanczos_kernel<GPT, KT>;
+  auto fn = lanczos_kernel<GPT, KT, PT>;
   SLS_CUDA_TRY(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   char* sc = (char*)scratch;
   void* args[] = {(void*)&bt, (void*)&sc, (void*)&gstride, (void*)&g, (void*)&groups,
@@ -1239,10 +1240,31 @@ int launch_lanczos_t(const LanczosBatch& bt, void* scratch, size_t gstride, int 
   return SLS_OK;
 }
 
+// KT = 1, 2 or 4 basis tiles for one GPT and element type
+template <int GPT, typename PT>
+int launch_lanczos_kt(const LanczosBatch& bt, void* scratch, size_t gstride, int groups, int g,
+                      int rows_cap, int stages, int* status, size_t smem, cudaStream_t stream,
+                      int kt) {
+  switch (kt) {
+    case 1:
+      return launch_lanczos_t<GPT, 1, PT>(bt, scratch, gstride, groups, g, rows_cap, stages,
+                                          status, smem, stream);
+    case 2:
+      return launch_lanczos_t<GPT, 2, PT>(bt, scratch, gstride, groups, g, rows_cap, stages,
+                                          status, smem, stream);
+    case 4:
+      return launch_lanczos_t<GPT, 4, PT>(bt, scratch, gstride, groups, g, rows_cap, stages,
+                                          status, smem, stream);
+    default:
+      return SLS_ERR_UNSUPPORTED;
+  }
+}
+
 }  // namespace
 
 // Launch the Lanczos kernel for GPT = 1, 2, 4 or 8 column groups per thread
-// and KT = 1, 2 or 4 basis tiles (lanczos_g<GPT>.cu).
+// and KT = 1, 2 or 4 basis tiles, Phi in float32 (lanczos_g<GPT>.cu) or
+// bfloat16 (lanczos_b<GPT>.cu).
 #define SLS_LZ_LAUNCH_ARGS                                                                \
   const LanczosBatch &bt, void *scratch, size_t gstride, int groups, int g, int rows_cap, \
       int stages, int *status, size_t smem, cudaStream_t stream, int kt
@@ -1250,5 +1272,9 @@ int launch_lanczos_gpt1(SLS_LZ_LAUNCH_ARGS);
 int launch_lanczos_gpt2(SLS_LZ_LAUNCH_ARGS);
 int launch_lanczos_gpt4(SLS_LZ_LAUNCH_ARGS);
 int launch_lanczos_gpt8(SLS_LZ_LAUNCH_ARGS);
+int launch_lanczos_bf16_gpt1(SLS_LZ_LAUNCH_ARGS);
+int launch_lanczos_bf16_gpt2(SLS_LZ_LAUNCH_ARGS);
+int launch_lanczos_bf16_gpt4(SLS_LZ_LAUNCH_ARGS);
+int launch_lanczos_bf16_gpt8(SLS_LZ_LAUNCH_ARGS);
 
 }  // namespace sls

@@ -105,7 +105,7 @@ SLS_DEV dfloat transpose_reduce(dfloat (&v)[NV], int lane) {
   return r;
 }
 
-template <int NV, int RV>
+template <int NV, int RV, typename PT>
 __global__ void __launch_bounds__(LW_MAX_WARPS * 32)
 lanczos_window_kernel(LanczosBatch bt) {
   constexpr int CU = (NV <= 16) ? 2 : 1;  // columns in flight per lane
@@ -127,7 +127,7 @@ lanczos_window_kernel(LanczosBatch bt) {
   const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
   const int n = bt.n ? bt.n[p] : (int)bt.n_single;
   const int64_t qoff = bt.q1off ? bt.q1off[p] : row0;
-  const float* __restrict__ Phi = bt.Phi + row0 * D;
+  const PT* __restrict__ Phi = reinterpret_cast<const PT*>(bt.Phi) + row0 * D;
   const int rmax = min(r, n);
   const bool mine = lane < n;
 
@@ -146,7 +146,7 @@ lanczos_window_kernel(LanczosBatch bt) {
     for (int c = lane; c < D; c += 32) {
       float ph[NV];
 #pragma unroll
-      for (int i = 0; i < NV; ++i) ph[i] = (i < n) ? __ldg(Phi + (size_t)i * D + c) : 0.f;
+      for (int i = 0; i < NV; ++i) ph[i] = (i < n) ? phi_ld(Phi, (size_t)i * D + c) : 0.f;
       float sh = 0.f, sl = 0.f;
 #pragma unroll
       for (int i = 0; i < NV; ++i) {
@@ -168,7 +168,7 @@ lanczos_window_kernel(LanczosBatch bt) {
       const float2 yc = ys[c];
       float ph[NV];
 #pragma unroll
-      for (int i = 0; i < NV; ++i) ph[i] = (i < n) ? __ldg(Phi + (size_t)i * D + c) : 0.f;
+      for (int i = 0; i < NV; ++i) ph[i] = (i < n) ? phi_ld(Phi, (size_t)i * D + c) : 0.f;
 #pragma unroll
       for (int i = 0; i < NV; ++i)
         if (i < n) dot2_acc(part[i].hi, part[i].lo, ph[i], yc.x, yc.y);
@@ -280,11 +280,18 @@ int launch_lanczos_window(const LanczosBatch& bt, cudaStream_t stream) {
   if (warps < 1) warps = 1;
   const size_t smem = per_warp * warps;
   const int blocks = (bt.nprob_max + warps - 1) / warps;
+#define SLS_LW_LAUNCH_T(NV, RV, PT)                                                         \
+  do {                                                                                      \
+    SLS_CUDA_TRY(cudaFuncSetAttribute(lanczos_window_kernel<NV, RV, PT>,                    \
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)); \
+    lanczos_window_kernel<NV, RV, PT><<<blocks, warps * 32, smem, stream>>>(bt);             \
+  } while (0)
 #define SLS_LW_LAUNCH(NV, RV)                                                               \
   do {                                                                                      \
-    SLS_CUDA_TRY(cudaFuncSetAttribute(lanczos_window_kernel<NV, RV>,                        \
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)); \
-    lanczos_window_kernel<NV, RV><<<blocks, warps * 32, smem, stream>>>(bt);                 \
+    if (bt.phi_bf16)                                                                        \
+      SLS_LW_LAUNCH_T(NV, RV, uint16_t);                                                    \
+    else                                                                                    \
+      SLS_LW_LAUNCH_T(NV, RV, float);                                                       \
   } while (0)
   if (bt.nmax <= 16 && bt.r <= 16)
     SLS_LW_LAUNCH(16, 16);
@@ -295,6 +302,7 @@ int launch_lanczos_window(const LanczosBatch& bt, cudaStream_t stream) {
   else
     SLS_LW_LAUNCH(32, 32);
 #undef SLS_LW_LAUNCH
+#undef SLS_LW_LAUNCH_T
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }

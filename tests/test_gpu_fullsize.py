@@ -112,6 +112,24 @@ def test_qwen7b_lanczos_full_size(sls, q7, q7_oracle):
     assert max_subspace_angle(U.cpu().numpy()[:, :k], q7_oracle["U"]) <= ANGLE_TOL
 
 
+def test_qwen7b_lanczos_bf16_phi_full_size(sls, q7):
+    """bf16 storage of Phi at the qwen7b shape: the GPU's bf16 features (the
+    feature map's bf16 epilogue) run through the bf16 Lanczos kernel, against
+    the oracle's Lanczos on the same stored values."""
+    w, Nc = q7["w"], q7["Nc"]
+    phib = sls.feature_map(q7["X"][:Nc], q7["W"], q7["b"], phi_dtype=torch.bfloat16)
+    theta, U, r_eff, _, _ = sls.lanczos_topr(phib, q7["q1"][:Nc], w.r)
+    torch.cuda.synchronize()
+    a, be, Q, k = O.lanczos(phib.float().cpu().numpy().astype(np.float64),
+                            q7["prm"].q1[:Nc], w.r)
+    th_o, S, U_o = O.ritz_pairs(a, be, Q)
+    assert int(r_eff.item()) == k
+    th = theta.cpu().numpy()[:k]
+    err = np.abs(th - th_o)
+    assert np.all(err <= RITZ_RTOL * np.abs(th_o) + ZERO_FLOOR * abs(th_o[0]))
+    assert max_subspace_angle(U.cpu().numpy()[:, :k], U_o) <= ANGLE_TOL
+
+
 def test_qwen7b_simhash_full_size_bit_exact(sls, q7, q7_oracle):
     w = q7["w"]
     got = sls.simhash(torch.from_numpy(q7_oracle["U32"]).cuda(), q7["R"], w.bits)

@@ -648,3 +648,59 @@ def test_embed_lookup_reproduces_the_prompt_generator():
         WL.vocab_rows(WL.DATA_SEED, np.arange(w.V), w.d).astype(np.float32))
     X = O.embed_lookup(table, p.ids)
     assert X.dtype == np.uint16 and np.array_equal(X, p.X)
+
+
+# ---------------------------------------------------------------------------
+# bfloat16 storage of the feature matrix (opt-in half-size Phi)
+# ---------------------------------------------------------------------------
+
+
+def test_bf16_round_closed_forms():
+    """Representable values stay; halfway cases go to the even neighbour; the
+    spacing below 2^-126 is 2^-133; signs and zeros are kept."""
+    r = O.bf16_round
+    for v in [1.0, 1.5, -3.0, 2.0 ** -100, 2.0 ** 100, 1 + 2.0 ** -7, 0.0]:
+        assert r(np.array([v]))[0] == v
+    assert r(np.array([1 + 2.0 ** -8]))[0] == 1.0                  # tie -> even (1.0)
+    assert r(np.array([1 + 3 * 2.0 ** -8]))[0] == 1 + 2.0 ** -6    # tie -> even (k = 2)
+    assert r(np.array([1 + 2.0 ** -8 + 2.0 ** -30]))[0] == 1 + 2.0 ** -7  # above the tie
+    assert r(np.array([-(1 + 3 * 2.0 ** -8)]))[0] == -(1 + 2.0 ** -6)
+    assert r(np.array([2.0 ** -133 * 2.5]))[0] == 2.0 ** -132      # subnormal tie -> even
+    assert np.signbit(r(np.array([-0.0]))[0])
+
+
+def test_bf16_round_matches_bit_level_rounding():
+    """Against the input generator's independent bit-level rounding of
+    float32 values (round-to-nearest-even on the high 16 bits), over many
+    magnitudes, and within half a unit of the 8-bit significand."""
+    rng = np.random.default_rng(11)
+    x = (rng.standard_normal(200000) * np.exp2(rng.integers(-60, 60, 200000))).astype(np.float32)
+    want = WL.bf16_bits_to_f32(WL.f32_to_bf16_bits(x)).astype(np.float64)
+    got = O.bf16_round(x.astype(np.float64))
+    assert np.array_equal(got, want)
+    assert np.all(np.abs(got - x) <= 2.0 ** -8 * np.abs(x))
+
+
+def test_bf16_storage_tolerance_class():
+    """The opt-in bf16 Phi defines a nearby operator: its eigenvalues are
+    within ||Phi_b Phi_b^T - Phi Phi^T||_2 <= (2 u + u^2) ||Phi||_2^2
+    (u = 2^-8, bf16's unit roundoff) of the float32 ones (Weyl), and the Lanczos run on it keeps
+    the leading Ritz value within that bound -- far below the RFF estimate's
+    own error O(D^-1/2) -- while the Ritz subspace moves measurably (which
+    is why bf16 storage is opt-in with its own tolerance class)."""
+    w = WL.scaled(WL.WORKLOADS["tiny"], N=400)
+    p, prm = WL.make_prompt(w), WL.params_for(w)
+    phi = O.rff_features(p.x_f64(), prm.w_f64(), prm.b).astype(np.float32).astype(np.float64)
+    phib = O.bf16_round(phi)
+    u = 2.0 ** -8
+    assert np.all(np.abs(phib - phi) <= u * np.abs(phi))
+    lam = np.linalg.eigvalsh(phi @ phi.T)
+    lamb = np.linalg.eigvalsh(phib @ phib.T)
+    bound = (2 * u + u * u) * np.linalg.norm(phi, 2) ** 2
+    assert np.max(np.abs(lam - lamb)) <= bound
+    a, b_, Q, k = O.lanczos(phi, prm.q1[:w.N], w.r)
+    ab, bb, Qb, kb = O.lanczos(phib, prm.q1[:w.N], w.r)
+    th = O.ritz_pairs(a, b_, Q)[0]
+    thb = O.ritz_pairs(ab, bb, Qb)[0]
+    assert abs(th[0] - thb[0]) <= bound
+    assert bound < th[0] / math.sqrt(w.D)
