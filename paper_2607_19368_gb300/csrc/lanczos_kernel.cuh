@@ -370,8 +370,9 @@ SLS_DEV int nprob_of(const LanczosBatch& bt) {
 // = (lane >> 3, lane & 7) loads base[b * stride + x] for b = bq, bq + 4, ...
 // (all loads of a batch in flight, 64 contiguous bytes per b), adds them as
 // a pairwise tree and the four b-groups by two butterfly steps; every lane
-// with lane & 7 == xx returns the sum for its item x.
-constexpr int CS_BATCH = 20;
+// with lane & 7 == xx returns the sum for its item x.  One batch covers the
+// partials of up to 160 CTAs, so a group's sums take one round of loads.
+constexpr int CS_BATCH = 40;
 
 __device__ __noinline__ dfloat warp_colsum8(const float2* __restrict__ base, size_t stride, int nb, int x,
                             bool valid) {
@@ -435,23 +436,35 @@ __device__ __noinline__ dfloat warp_wcorr8(const float2* __restrict__ Wm, int D,
   return acc;
 }
 
-// Sum of v[0 .. n) over the warp, all loads in flight (n <= 32 * SLICE_LOADS
-// at once, the rest in a loop); every lane gets the result.
-__device__ __noinline__ dfloat warp_sum_vec(const float2* __restrict__ v, int n) {
+// Sums of a[0 .. n) and b[0 .. n) over the warp, both batches of loads in
+// flight together; every lane gets both.
+__device__ __noinline__ void warp_sum_vec2(const float2* __restrict__ a,
+                                           const float2* __restrict__ b, int n, float2* out) {
   const int lane = threadIdx.x & 31;
-  dfloat x[SLICE_LOADS];
+  dfloat x[SLICE_LOADS], y[SLICE_LOADS];
 #pragma unroll
   for (int m = 0; m < SLICE_LOADS; ++m) {
-    const int b = lane + 32 * m;
-    x[m] = (b < n) ? dfv(v[b]) : df_make(0.f, 0.f);
+    const int i = lane + 32 * m;
+    x[m] = (i < n) ? dfv(a[i]) : df_make(0.f, 0.f);
+    y[m] = (i < n) ? dfv(b[i]) : df_make(0.f, 0.f);
   }
-  dfloat s = x[0];
+  dfloat s = x[0], t = y[0];
 #pragma unroll
-  for (int m = 1; m < SLICE_LOADS; ++m) s = df_add_fast(s, x[m]);
-  for (int b = lane + 32 * SLICE_LOADS; b < n; b += 32) s = df_add_fast(s, dfv(v[b]));
+  for (int m = 1; m < SLICE_LOADS; ++m) {
+    s = df_add_fast(s, x[m]);
+    t = df_add_fast(t, y[m]);
+  }
+  for (int i = lane + 32 * SLICE_LOADS; i < n; i += 32) {
+    s = df_add_fast(s, dfv(a[i]));
+    t = df_add_fast(t, dfv(b[i]));
+  }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) s = df_add_fast(s, shfl_xor_df(s, o));
-  return s;
+  for (int o = 16; o > 0; o >>= 1) {
+    s = df_add_fast(s, shfl_xor_df(s, o));
+    t = df_add_fast(t, shfl_xor_df(t, o));
+  }
+  out[0] = f2(s);
+  out[1] = f2(t);
 }
 
 // Per-warp partial coefficients (lanes over k < K) -> the CTA's partial row.
@@ -914,8 +927,9 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       // ---------------- beta_{j-1}, alpha_j, break test -------------------------
       if (warp == 0) {
         // |z1|^2 = |z'|^2 - |c|^2 (Q orthonormal), |Phi^T z1|^2
-        const dfloat s = warp_sum_vec(npart + (size_t)(j & 1) * g, g);
-        const dfloat q = warp_sum_vec(sqpart, g);
+        float2 sq2[2];
+        warp_sum_vec2(npart + (size_t)(j & 1) * g, sqpart, g, sq2);
+        const dfloat s = dfv(sq2[0]), q = dfv(sq2[1]);
         dfloat cn = df_make(0.f, 0.f);
 #pragma unroll
         for (int tt = 0; tt < KT; ++tt) {
