@@ -751,7 +751,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   // once the previous pass has written its column of Q.
   if (warp == LZ_CW) {
     if (lane != 0) return;
-    const uint64_t pol = l2_policy_normal();
+    const uint64_t pol_first = l2_policy_evict_first(), pol_last = l2_policy_evict_last();
     unsigned cnt = 0;
     int pp = 0;
     for (int p = gi; p < nprob; p += ngroups, ++pp) {
@@ -772,6 +772,11 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
       const int64_t rs = (int64_t)rank * n / g, re = (int64_t)(rank + 1) * n / g;
       const int nch = (int)((re - rs + cr - 1) / cr);
+      // the chunks a pass fetches last are the next pass's first (passes
+      // alternate direction): keep about 64 MB of them in L2 over the whole
+      // grid, stream the rest
+      const size_t cbytes = (size_t)cr * D * sizeof(PT);
+      const int nkeep = (int)min((size_t)nch, ((size_t)64 << 20) / ((size_t)gridDim.x * cbytes));
       const PT* Phi = reinterpret_cast<const PT*>(bt.Phi) + (row0 + rs) * D;
       const float2* Qs = bt.Q + (row0 + rs) * ldq;
       bool stop = false;
@@ -813,6 +818,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           const unsigned b2 = (unsigned)(nr * ldq * 8);
           unsigned char* dst = ring + (size_t)slot * stage;
           mbar_expect_tx(&fullb[slot], b1 + b2);
+          const uint64_t pol = (t >= nch - nkeep) ? pol_last : pol_first;
           bulk_g2s(dst, Phi + (int64_t)k * cr * D, b1, &fullb[slot], pol);
           bulk_g2s(dst + phib, Qs + (int64_t)k * cr * ldq, b2, &fullb[slot], pol);
           ++cnt;
@@ -1123,9 +1129,11 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
             if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
               const int il = (first ? kc0 : kc1) * cr + ii;
               const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
+              // the LZ_CW warp sums sit in lanes 0 .. LZ_CW - 1
               dfloat s = (lane < LZ_CW) ? dfv(bpart[ri * LZ_CW + lane]) : df_make(0.f, 0.f);
 #pragma unroll
-              for (int o = 16; o > 0; o >>= 1) s = df_add_fast(s, shfl_xor_df(s, o));
+              for (int o = LZ_CW / 2; o > 0; o >>= 1) s = df_add_fast(s, shfl_xor_df(s, o));
+              s = shfl_df(s, 0);
               dfloat zp = df_sub(s, df_mul(alpha_df, qjv[m]));
               if (j > 0) zp = df_sub(zp, df_mul(beta_df, dfv(qpv[m])));
               if (lane == 0) {
