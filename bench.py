@@ -216,18 +216,89 @@ def sample_prompt(w):
     return WL.make_prompt(w), 0
 
 
+def cpu_phases(w, rho, X64, prm, n):
+    """Seconds per phase of one oracle run of the global backend on the first
+    n tokens, calling the oracle's steps one by one in the order its
+    compress_global takes them (features, Lanczos, Ritz pairs, SimHash,
+    clusters and adjustment, macro-token means)."""
+    import numpy as np
+    import oracle as O
+    cfg = oracle_config(w, rho)
+    Xc = X64[:n - w.preserve_last]
+    M = O.target_count(Xc.shape[0], rho)
+    bits = cfg.bits if cfg.bits > 0 else O.auto_bits(Xc.shape[0], rho)
+    t, out = time.perf_counter(), {}
+
+    def lap(name):
+        nonlocal t
+        now = time.perf_counter()
+        out[name] = now - t
+        t = now
+    phi = O.rff_features(Xc, prm.w_f64(), prm.b).astype(np.float32).astype(np.float64)
+    lap("features")
+    a, b_, Q, k = O.lanczos(phi, prm.q1[:Xc.shape[0]], w.r, cfg.lanczos_tol)
+    lap("lanczos")
+    _, _, U = O.ritz_pairs(a, b_, Q)
+    lap("ritz")
+    codes = O.simhash(U.astype(np.float32), prm.R[:bits, :k])
+    lap("simhash")
+    groups = O.adjust_groups(O.bucket(codes), M)
+    order = O.order_groups(groups, O.POS_MAX)
+    lap("segment")
+    O.aggregate_groups(Xc, [groups[i] for i in order], True)
+    lap("aggregate")
+    return out
+
+
 def cpu_baseline(w, rho, X64, prm, n, pidx, budget_s=10.0):
     """The oracle as it stands, on the first n tokens of one prompt, repeated
-    until about budget_s seconds of CPU work have been timed."""
+    until about budget_s seconds of CPU work have been timed; then the same
+    on one core (a child process with single-threaded BLAS) and, for the
+    global backend, the oracle's time per phase."""
     tot, reps = 0.0, 0
     while reps == 0 or tot < budget_s:
         tot += cpu_oracle_step(w, rho, X64, prm, n)
         reps += 1
     kind = "compress_" + w.backend
-    return {"value": n * reps / tot, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"oracle {kind} (numpy float64, BLAS threads = all cores) on the first "
-                      f"{n} tokens of prompt {pidx} of the {w.name} workload, D={w.D} r={w.r} "
-                      f"b={w.bits or 'auto'} rho={rho:g}; {reps} run(s), {tot:.1f} s"}
+    res = {"value": n * reps / tot, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+           "sample": f"oracle {kind} (numpy float64, BLAS threads = all cores) on the first "
+                     f"{n} tokens of prompt {pidx} of the {w.name} workload, D={w.D} r={w.r} "
+                     f"b={w.bits or 'auto'} rho={rho:g}; {reps} run(s), {tot:.1f} s"}
+    if not windowed(w):
+        res["phases_s"] = {k: round(v, 4) for k, v in cpu_phases(w, rho, X64, prm, n).items()}
+    one = single_core_baseline(w, rho, n)
+    if one is not None:
+        res["single_core"] = one
+    return res
+
+
+def single_core_baseline(w, rho, n, budget_s=8.0):
+    """The same oracle sample timed in a child process whose BLAS and OpenMP
+    pools have one thread (the variables must be set before numpy loads)."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1",
+               MKL_NUM_THREADS="1")
+    code = ("import json, bench\n"
+            f"print(json.dumps(bench.single_core_child({w.name!r}, {rho!r}, {n}, {budget_s})))")
+    try:
+        r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env,
+                           capture_output=True, text=True, timeout=600)
+        return json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception:
+        return None
+
+
+def single_core_child(name, rho, n, budget_s):
+    w = workload(name)
+    p, _ = sample_prompt(w)
+    import workloads as WL
+    prm = WL.params_for(w)
+    X64 = p.x_f64()
+    tot, reps = 0.0, 0
+    while reps == 0 or tot < budget_s:
+        tot += cpu_oracle_step(w, rho, X64, prm, n)
+        reps += 1
+    return {"value": n * reps / tot, "unit": UNIT, "cores": 1, "runs": reps,
+            "seconds": round(tot, 2)}
 
 
 def run_reference(args, rank, world):

@@ -154,6 +154,35 @@ def test_lanczos_matches_oracle(sls, name, N, D, r):
             assert cosv > 1 - 1e-6, (j, cosv)
 
 
+@pytest.mark.parametrize("name,N,D,r", [("mistral7b", 3000, 1024, 128),   # KT = 4 (r = SLS_MAX_R)
+                                        ("tiny", 2000, 4096, 32),        # GPT = 4
+                                        ("tiny", 1500, 8192, 16),        # GPT = 8 (D = SLS_MAX_D)
+                                        ("tiny", 333, 8192, 128)])       # both, ragged strips
+def test_lanczos_widest_shapes(sls, name, N, D, r):
+    """The kernel instantiations for the widest feature counts and the
+    largest Krylov rank the interface accepts."""
+    w, p, prm = _workload_inputs(name, N=N, D=D)
+    phi32 = oracle_phi32(p.x_f64(), prm.w_f64(), prm.b)
+    _lanczos_case(sls, phi32, prm.q1[:N], r)
+
+
+def test_compress_at_interface_limits(sls):
+    """The whole pass at D = 8192, r = 128 and b = 32 (the interface's
+    maxima): the output invariants and the oracle's macro embeddings and
+    positions of the GPU's own groups."""
+    w, p, prm = _workload_inputs("tiny", N=900, D=8192)
+    prm32 = WL.make_params(8192, w.d, 128, 32, w.N, w.dtype)
+    cfg = sls.Config.make(rho=4.0, D=8192, r=128, bits=32, preserve_last=12)
+    X = to_torch_x(p.X, w.dtype)
+    Xt, pos, t2m, r_eff, _ = sls.compress(
+        X, cfg, to_torch_x(prm32.W, w.dtype), torch.from_numpy(prm32.b).cuda(),
+        torch.from_numpy(prm32.R).cuda(), torch.from_numpy(prm32.q1).cuda())
+    torch.cuda.synchronize()
+    M = sls.output_count(cfg, w.N)
+    assert int(r_eff[0].item()) == 128
+    _check_pass(sls, p.x_f64(), Xt.cpu().numpy(), pos.cpu().numpy(), t2m.cpu().numpy(), M, 0, 12)
+
+
 def test_lanczos_breakdown_low_rank(sls):
     w, p, prm = _workload_inputs("tiny", N=64, D=64)
     phi = oracle_phi32(p.x_f64()[:5], prm.w_f64()[:64], prm.b[:64])
