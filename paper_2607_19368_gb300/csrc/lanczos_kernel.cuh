@@ -944,7 +944,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         for (int o = 16; o > 0; o >>= 1) cn = df_add_fast(cn, shfl_xor_df(cn, o));
         if (lane == 0) {
           const double nrm2 = df_to_double(s) - df_to_double(cn);  // |z1|^2
-          const double bnew = sqrt(fmax(nrm2, 0.0));
+          // one reciprocal square root instead of a square root and two
+          // divides (float64 runs at a fraction of the float32 rate here)
+          const double inv = (nrm2 > 0.0) ? rsqrt(nrm2) : 0.0;    // 1 / beta
+          const double bnew = (nrm2 > 0.0) ? nrm2 * inv : 0.0;
           int brk = 0;
           if (j > 0) {
             scale = fmax(scale, fabs(alpha_prev) + bnew);
@@ -953,9 +956,9 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           } else if (!(bnew > 0.0)) {
             brk = 1;
           }
-          const double a = brk ? 0.0 : df_to_double(q) / (bnew * bnew);
+          const double a = brk ? 0.0 : (df_to_double(q) * inv) * inv;
           if (!brk && rank == 0) alpha_out[j] = a;
-          shd[1] = brk ? 0.0 : 1.0 / bnew;
+          shd[1] = brk ? 0.0 : inv;
           shd[2] = a;
           shd[3] = (j > 0) ? bnew : 0.0;
           sbreak = brk;
@@ -1088,25 +1091,30 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           const float2* qb1 = reinterpret_cast<const float2*>(ring + (size_t)s1 * stage + phib);
           const int nr0 = min(cr, nrows - kc0 * cr);
           const int nr1 = two ? min(cr, nrows - kc1 * cr) : 0;
-          // row work before the row dots: q_j of the warp's rows of the pair
+          // row work before the row dots: q_j of the warp's rows of the pair (it
+          // feeds only the row work after them; with two or more column groups per
+          // thread it runs after the row dots, measured faster there, with one
+          // before them)
           dfloat qjv[RPW];
           float2 qpv[RPW];
+          if constexpr (GPT == 1) {
 #pragma unroll
-          for (int m = 0; m < RPW; ++m) {
-            const int ri = warp + m * LZ_CW;
-            const bool first = ri < TCR;
-            const int ii = first ? ri : ri - TCR;
-            qjv[m] = df_make(0.f, 0.f);
-            qpv[m] = make_float2(0.f, 0.f);
-            if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
-              const int il = (first ? kc0 : kc1) * cr + ii;
-              const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
-              const float corr = row_corr<KT>(qrow, cs, j);
-              dfloat z1 = dfv(zps[il]);
-              if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
-              qjv[m] = df_mul(z1, invb_df);
-              if (j > 0) qpv[m] = qrow[j - 1];
-              if (lane == 0) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
+            for (int m = 0; m < RPW; ++m) {
+              const int ri = warp + m * LZ_CW;
+              const bool first = ri < TCR;
+              const int ii = first ? ri : ri - TCR;
+              qjv[m] = df_make(0.f, 0.f);
+              qpv[m] = make_float2(0.f, 0.f);
+              if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
+                const int il = (first ? kc0 : kc1) * cr + ii;
+                const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
+                const float corr = row_corr<KT>(qrow, cs, j);
+                dfloat z1 = dfv(zps[il]);
+                if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
+                qjv[m] = df_mul(z1, invb_df);
+                if (j > 0) qpv[m] = qrow[j - 1];
+                if (lane == 0) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
+              }
             }
           }
           // row dots s = Phi w_j, warp sums into bpart[row * LZ_CW + warp]
@@ -1116,6 +1124,26 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           else
             sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bpart,
                                               bpart + TCR * LZ_CW);
+          if constexpr (GPT != 1) {
+#pragma unroll
+            for (int m = 0; m < RPW; ++m) {
+              const int ri = warp + m * LZ_CW;
+              const bool first = ri < TCR;
+              const int ii = first ? ri : ri - TCR;
+              qjv[m] = df_make(0.f, 0.f);
+              qpv[m] = make_float2(0.f, 0.f);
+              if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
+                const int il = (first ? kc0 : kc1) * cr + ii;
+                const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
+                const float corr = row_corr<KT>(qrow, cs, j);
+                dfloat z1 = dfv(zps[il]);
+                if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
+                qjv[m] = df_mul(z1, invb_df);
+                if (j > 0) qpv[m] = qrow[j - 1];
+                if (lane == 0) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
+              }
+            }
+          }
           named_sync(BAR_COMPUTE, LZ_CT);
           // row work after the row dots: z', its partials of c and |z'|^2
 #pragma unroll
