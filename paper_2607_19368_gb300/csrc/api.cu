@@ -715,9 +715,12 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   int mode = spectral ? 0 : 1;
   if (cfg->backend == SLS_BACKEND_ADAPTIVE) {
     mode = 2;
+    // below rho = 16 the score pass also writes every window's chunk-path
+    // output, so the segment and aggregation steps only see spectral windows
     if (cfg->rho < 16.0 &&
-        (st = launch_window_score(X, x_dtype, d, ldx, W.probs, nprob, P.nmax, W.score_part,
-                                  W.score, s)) != SLS_OK)
+        (st = launch_window_score_chunk(X, x_dtype, d, ldx, W.probs, nprob, P.nmax,
+                                        W.score_part, W.score, cfg->pos_scheme, cfg->pos_mode,
+                                        cfg->renorm, Xt, pos, tok2macro, s)) != SLS_OK)
       return st;
   }
   double tau = cfg->tau;
@@ -812,9 +815,10 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
     }
   }
   phase_mark(5, 0, s);
+  const int chunk_done = (cfg->backend == SLS_BACKEND_ADAPTIVE && cfg->rho < 16.0) ? 1 : 0;
   if ((st = launch_segment(W.probs, nprob, W.codes, cfg->pos_scheme, cfg->pos_mode, W.seg_scratch,
                            P.seg_slots, P.nmax, P.mmax, W.perm, W.mstart, W.mlen, pos, tok2macro,
-                           W.status, s)) != SLS_OK)
+                           W.status, s, chunk_done)) != SLS_OK)
     return st;
   if ((st = launch_preserved(B, N, P.M, (int)P.pf, (int)P.pl, cfg->pos_mode, W.perm, W.mstart,
                              W.mlen, pos, tok2macro, s)) != SLS_OK)

@@ -286,7 +286,7 @@ segment_kernel(const ProbDesc* __restrict__ probs, int nprob, const uint32_t* __
                int pos_scheme, int pos_mode, char* scratch, size_t pstride, int64_t nmax,
                int64_t mmax, int* __restrict__ perm, int* __restrict__ mstart,
                int* __restrict__ mlen, int32_t* __restrict__ pos_out,
-               int32_t* __restrict__ tok2macro) {
+               int32_t* __restrict__ tok2macro, int chunk_done) {
   __shared__ int sh_sort[512 + SEG_W * 256];
   __shared__ long long sh_ll[SEG_W + 1];
   __shared__ int sh_i[SEG_W + 1];
@@ -299,6 +299,11 @@ segment_kernel(const ProbDesc* __restrict__ probs, int nprob, const uint32_t* __
     const ProbDesc P = probs[p];
     const int n = P.n, M = P.m;
     if (n <= 0 || M <= 0) continue;
+    if (chunk_done && !P.spectral) {
+      // outputs already written by the score pass: nothing to aggregate
+      for (int t = tid; t < M; t += SEG_T) mlen[P.out0 + t] = 0;
+      continue;
+    }
     int* va = reinterpret_cast<int*>(sb + L.va);
     int* vb = reinterpret_cast<int*>(sb + L.vb);
     int* f = reinterpret_cast<int*>(sb + L.f);
@@ -632,7 +637,7 @@ segment_grid_kernel(const ProbDesc* __restrict__ probs, const uint32_t* __restri
                     int pos_scheme, int pos_mode, char* sb, int64_t nmax, int64_t mmax,
                     int* __restrict__ perm, int* __restrict__ mstart, int* __restrict__ mlen,
                     int32_t* __restrict__ pos_out, int32_t* __restrict__ tok2macro,
-                    int* status) {
+                    int* status, int chunk_done) {
   __shared__ int sh_sort[512 + SEG_W * 256];
   __shared__ long long sh_ll[SEG_W + 1];
   __shared__ int sh_i[SEG_W + 1];
@@ -648,6 +653,10 @@ segment_grid_kernel(const ProbDesc* __restrict__ probs, const uint32_t* __restri
   const ProbDesc P = probs[0];
   const int n = P.n, M = P.m;
   if (n <= 0 || M <= 0) return;
+  if (chunk_done && !P.spectral) {  // the whole grid leaves before any grid barrier
+    for (int t = b * SEG_T + tid; t < M; t += G * SEG_T) mlen[P.out0 + t] = 0;
+    return;
+  }
   uint32_t* ka = reinterpret_cast<uint32_t*>(sb + L.ka);
   uint32_t* kb = reinterpret_cast<uint32_t*>(sb + L.kb);
   int* va = reinterpret_cast<int*>(sb + L.va);
@@ -873,7 +882,8 @@ __global__ void __launch_bounds__(SEGW_WARPS * 32)
 segment_warp_kernel(const ProbDesc* __restrict__ probs, int nprob,
                     const uint32_t* __restrict__ codes, int pos_scheme, int pos_mode,
                     int* __restrict__ perm, int* __restrict__ mstart, int* __restrict__ mlen,
-                    int32_t* __restrict__ pos_out, int32_t* __restrict__ tok2macro) {
+                    int32_t* __restrict__ pos_out, int32_t* __restrict__ tok2macro,
+                    int chunk_done) {
   const unsigned FULL = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int w0 = blockIdx.x * SEGW_WARPS + (threadIdx.x >> 5);
@@ -882,6 +892,10 @@ segment_warp_kernel(const ProbDesc* __restrict__ probs, int nprob,
     const ProbDesc P = probs[p];
     const int n = P.n, M = P.m;
     if (n <= 0 || M <= 0) continue;
+    if (chunk_done && !P.spectral) {
+      for (int t = lane; t < M; t += 32) mlen[P.out0 + t] = 0;
+      continue;
+    }
     const bool valid = lane < n;
     // ---- order: (code, token) for spectral windows, token order otherwise ----
     unsigned long long key = ~0ull;
@@ -1205,6 +1219,10 @@ agg_fill_kernel(const int* __restrict__ mlen, int64_t Mtot, int64_t Ntot, int G,
   const AggAux A = agg_aux(aux, Mtot, Ntot);
   const int nitems = A.counts[0];
   const int64_t rtot = A.counts[3];
+  // no items (every macro-token already written elsewhere): every CTA range
+  // is empty
+  if (nitems == 0 && blockIdx.x == 0)
+    for (int t = threadIdx.x; t <= G; t += blockDim.x) A.cta_first[t] = 0;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nitems; i += gridDim.x * blockDim.x) {
     // the macro of item i: the last m with it_start[m] <= i
     int lo = 0, hi = (int)Mtot - 1;
@@ -1796,14 +1814,230 @@ window_score_kernel(const T* __restrict__ X, int d, int64_t ldx,
   }
 }
 
+// ---------------------------------------------------------------------------
+// The score pass with the chunk path folded in (adaptive backend below rho =
+// 16, Sec. 3.6): the windows whose score falls below tau are averaged in
+// consecutive groups (numpy array_split of the window's n tokens into its m
+// macro-tokens), and those means need the same rows the score reads.  So the
+// score pass computes, for every window, the chunk macro-tokens as if it were
+// routed to the chunk path -- renormalised means (Eq. macro_embed), their
+// positions and the token map -- and the segment and aggregation steps then
+// handle the spectral windows only, whose outputs replace these.  Parts are
+// cut on group boundaries (about SCORE_PR rows each), so no group spans two
+// CTAs; a batch's shared-memory reduction carries, besides the row norms,
+// the squared norms of the group means that end in the batch.
+// ---------------------------------------------------------------------------
+
+// first token of chunk group g (g <= m; group m starts at n)
+__host__ __device__ inline int chunk_gstart(int n, int m, int g) {
+  const int q = n / m, rem = n % m;
+  return (g < rem) ? g * (q + 1) : rem * (q + 1) + (g - rem) * q;
+}
+// groups per part: about SCORE_PR rows, at least one group
+__host__ __device__ inline int chunk_gpp(int n, int m) {
+  const int gp = SCORE_PR / (n / m + 1);
+  return gp < 1 ? 1 : gp;
+}
+__host__ __device__ inline int chunk_nparts(int n, int m) {
+  const int gp = chunk_gpp(n, m);
+  return (m + gp - 1) / gp;
+}
+// a bound on chunk_nparts over windows of at most nmax tokens: every part but
+// the last holds at least SCORE_PR / 2 rows
+__host__ __device__ inline int chunk_parts_max(int64_t nmax) {
+  return (int)((nmax + SCORE_PR / 2 - 1) / (SCORE_PR / 2));
+}
+
+// Element e of a 16-byte word of X as loaded: four floats, or eight bf16
+// values widened exactly.  Keeping the loaded rows as raw words halves their
+// registers for bf16 inputs.
+template <typename T>
+SLS_DEV float raw_elem(const uint4& r, int e);
+template <>
+SLS_DEV float raw_elem<float>(const uint4& r, int e) {
+  const unsigned w = (e == 0) ? r.x : (e == 1) ? r.y : (e == 2) ? r.z : r.w;
+  return __uint_as_float(w);
+}
+template <>
+SLS_DEV float raw_elem<uint16_t>(const uint4& r, int e) {
+  const int k = e >> 1;
+  const unsigned w = (k == 0) ? r.x : (k == 1) ? r.y : (k == 2) ? r.z : r.w;
+  return (e & 1) ? __uint_as_float(w & 0xffff0000u) : __uint_as_float(w << 16);
+}
+
+template <typename T, int NV>
+__global__ void __launch_bounds__(AGG_T, 2)
+window_score_chunk_kernel(const T* __restrict__ X, int d, int64_t ldx,
+                          const ProbDesc* __restrict__ probs, int nprob, int KP,
+                          float* __restrict__ part, int pos_scheme, int pos_mode, int renorm,
+                          float* __restrict__ Xt, int32_t* __restrict__ pos_out,
+                          int32_t* __restrict__ tok2macro) {
+  constexpr int V = VecOf<T>::V;
+  constexpr int MB = agg_batch<NV>();
+  constexpr int NW = AGG_T / 32;
+  __shared__ float shq[2][MB][NW];  // row |x|^2 partials
+  __shared__ float shg[2][MB][NW];  // |group mean|^2 partials, slot = the group's last row
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int units = nprob * KP;
+  for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    const int p = u / KP, k = u % KP;
+    const ProbDesc P = probs[p];
+    const int n = P.n, m = P.m;
+    if (n <= 0 || m <= 0) continue;
+    const int gp = chunk_gpp(n, m);
+    if (k >= (m + gp - 1) / gp) continue;
+    const int g0 = k * gp, g1 = min(m, g0 + gp);
+    const int r0 = chunk_gstart(n, m, g0), r1 = chunk_gstart(n, m, g1);
+    const int q = n / m, rem = n % m;
+    // positions of the part's groups and the token map
+    for (int g = g0 + tid; g < g1; g += AGG_T) {
+      const int a = chunk_gstart(n, m, g), len = chunk_gstart(n, m, g + 1) - a;
+      int rp;
+      if (pos_scheme == SLS_POS_MAX) {
+        rp = a + len - 1;
+      } else if (pos_scheme == SLS_POS_MEDIAN) {
+        rp = a + (len - 1) / 2;
+      } else {
+        const unsigned long long sum =
+            (unsigned long long)len * a + (unsigned long long)len * (len - 1) / 2;
+        rp = (int)((2ull * sum + (unsigned long long)len) / (2ull * (unsigned long long)len));
+      }
+      pos_out[P.out0 + g] = (pos_mode == SLS_MODE_COMPACT) ? (P.out_local + g) : (P.pos0 + rp);
+    }
+    for (int i = r0 + tid; i < r1; i += AGG_T) {
+      const int g = (i < rem * (q + 1)) ? i / (q + 1) : rem + (i - rem * (q + 1)) / q;
+      tok2macro[P.tok_row + i] = P.out_local + g;
+    }
+    float cs[NV * V], ns[NV * V], gs[NV * V];
+#pragma unroll
+    for (int e = 0; e < NV * V; ++e) cs[e] = ns[e] = gs[e] = 0.f;
+    int gcur = g0, gend = chunk_gstart(n, m, g0 + 1), gcnt = 0;  // before the barrier
+    int pcur = g0, pend = gend, pcnt = 0;                          // after it
+    float geta = 0.f;
+    int buf = 0;
+    for (int s0 = r0; s0 < r1; s0 += MB, buf ^= 1) {
+      uint4 raw[MB][NV];
+#pragma unroll
+      for (int j = 0; j < MB; ++j) {
+        const bool live = s0 + j < r1;
+        const T* x = X + (P.tok_row + s0 + j) * ldx;
+#pragma unroll
+        for (int qv = 0; qv < NV; ++qv) {
+          const int c0 = (tid + qv * AGG_T) * V;
+          raw[j][qv] = (live && c0 < d) ? __ldg(reinterpret_cast<const uint4*>(x + c0))
+                                        : make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+      // before the barrier: row |x|^2 partials; the group sums, and for every
+      // group that ends in this batch its mean (stored unscaled; a singleton is
+      // its token) and the |mean|^2 partial
+#pragma unroll
+      for (int j = 0; j < MB; ++j) {
+        float sq = 0.f;
+#pragma unroll
+        for (int e = 0; e < NV * V; ++e) {
+          const float x = raw_elem<T>(raw[j][e / V], e % V);
+          sq = fmaf(x, x, sq);
+        }
+        sq = warp_sum_f(sq);
+        if (lane == 0) shq[buf][j][warp] = sq;
+        if (s0 + j < r1) {
+#pragma unroll
+          for (int e = 0; e < NV * V; ++e) gs[e] += raw_elem<T>(raw[j][e / V], e % V);
+          ++gcnt;
+          if (s0 + j + 1 == gend) {
+            const float ginv = (gcnt > 1) ? 1.0f / (float)gcnt : 1.0f;
+            float gq = 0.f;
+#pragma unroll
+            for (int e = 0; e < NV * V; ++e) {
+              if (gcnt > 1) gs[e] *= ginv;
+              gq = fmaf(gs[e], gs[e], gq);
+            }
+            gq = warp_sum_f(gq);
+            if (lane == 0) shg[buf][j][warp] = gq;
+            store_row<V, NV>(gs, 1.0f, d, Xt + (P.out0 + gcur) * (int64_t)d);
+#pragma unroll
+            for (int e = 0; e < NV * V; ++e) gs[e] = 0.f;
+            gcnt = 0;
+            ++gcur;
+            gend = chunk_gstart(n, m, gcur + 1);
+          }
+        }
+      }
+      __syncthreads();
+      // after it: the score sums, and each finished group's mean rescaled in
+      // place to the mean member norm (Eq. macro_embed)
+#pragma unroll
+      for (int j = 0; j < MB; ++j) {
+        if (s0 + j >= r1) break;
+        float tq = 0.f;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) tq += shq[buf][j][w];
+        const float nrm = sqrtf(tq);
+        const float inv = (tq > 0.f) ? 1.0f / nrm : 0.f;
+#pragma unroll
+        for (int e = 0; e < NV * V; ++e) {
+          const float x = raw_elem<T>(raw[j][e / V], e % V);
+          cs[e] += x;
+          ns[e] = fmaf(x, inv, ns[e]);
+        }
+        geta += nrm;
+        ++pcnt;
+        if (s0 + j + 1 == pend) {
+          if (pcnt > 1 && renorm) {
+            float gq = 0.f;
+#pragma unroll
+            for (int w = 0; w < NW; ++w) gq += shg[buf][j][w];
+            const float gn = sqrtf(gq);
+            if (gn >= 1e-30f) {
+              const float scale = (geta * (1.0f / (float)pcnt)) / gn;
+              float* out = Xt + (P.out0 + pcur) * (int64_t)d;
+#pragma unroll
+              for (int qv = 0; qv < NV; ++qv) {
+                const int c0 = (tid + qv * AGG_T) * V;
+                if (c0 < d)
+#pragma unroll
+                  for (int e = 0; e < V; e += 4) {
+                    const float4 mv = *reinterpret_cast<const float4*>(out + c0 + e);
+                    store_vec4(out + c0 + e, mv.x * scale, mv.y * scale, mv.z * scale,
+                               mv.w * scale);
+                  }
+              }
+            }
+          }
+          geta = 0.f;
+          pcnt = 0;
+          ++pcur;
+          pend = chunk_gstart(n, m, pcur + 1);
+        }
+      }
+    }
+    float* dst = part + (size_t)u * 2 * d;
+#pragma unroll
+    for (int qv = 0; qv < NV; ++qv) {
+      const int c0 = (tid + qv * AGG_T) * V;
+      if (c0 < d)
+#pragma unroll
+        for (int e = 0; e < V; e += 4) {
+          store_vec4(dst + c0 + e, cs[qv * V + e], cs[qv * V + e + 1], cs[qv * V + e + 2],
+                     cs[qv * V + e + 3]);
+          store_vec4(dst + d + c0 + e, ns[qv * V + e], ns[qv * V + e + 1], ns[qv * V + e + 2],
+                     ns[qv * V + e + 3]);
+        }
+    }
+    __syncthreads();
+  }
+}
+
 // score[p] = (sum of the parts' x / |x|) . (sum of the parts' x) / (n |sum x|)
 __global__ void __launch_bounds__(AGG_T)
 window_score_combine_kernel(int d, const ProbDesc* __restrict__ probs, int nprob, int KP,
-                            const float* __restrict__ part, float* __restrict__ score) {
+                            int chunked, const float* __restrict__ part,
+                            float* __restrict__ score) {
   __shared__ float sh[AGG_T / 32];
   for (int p = blockIdx.x; p < nprob; p += gridDim.x) {
     const int n = probs[p].n;
-    const int kp = score_parts(n);
+    const int kp = chunked ? chunk_nparts(n, probs[p].m) : score_parts(n);
     float dot = 0.f, cc = 0.f;
     for (int c = threadIdx.x; c < d; c += AGG_T) {
       float cs = 0.f, ns = 0.f;
@@ -1867,7 +2101,7 @@ int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const i
 int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int pos_scheme,
                    int pos_mode, void* scratch, int slots, int64_t nmax, int64_t mmax, int* perm,
                    int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro, int* status,
-                   cudaStream_t stream) {
+                   cudaStream_t stream, int chunk_done) {
   if (nprob <= 0) return SLS_OK;
   const SegLayout L = seg_layout(nmax, mmax);
   const size_t stride = L.total;
@@ -1876,7 +2110,8 @@ int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int 
     int64_t blocks = ((int64_t)nprob + SEGW_WARPS - 1) / SEGW_WARPS;
     if (blocks > 65535) blocks = 65535;
     segment_warp_kernel<<<(unsigned)blocks, SEGW_WARPS * 32, 0, stream>>>(
-        probs, nprob, codes, pos_scheme, pos_mode, perm, mstart, mlen, pos_out, tok2macro);
+        probs, nprob, codes, pos_scheme, pos_mode, perm, mstart, mlen, pos_out, tok2macro,
+        chunk_done);
     SLS_LAUNCH_CHECK();
     return SLS_OK;
   }
@@ -1894,7 +2129,8 @@ int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int 
     int64_t nm = nmax, mm = mmax;
     void* args[] = {(void*)&probs, (void*)&codes, (void*)&pos_scheme, (void*)&pos_mode,
                     (void*)&sb, (void*)&nm, (void*)&mm, (void*)&perm, (void*)&mstart,
-                    (void*)&mlen, (void*)&pos_out, (void*)&tok2macro, (void*)&status};
+                    (void*)&mlen, (void*)&pos_out, (void*)&tok2macro, (void*)&status,
+                    (void*)&chunk_done};
     SLS_CUDA_TRY(cudaLaunchCooperativeKernel((const void*)segment_grid_kernel, dim3(G), dim3(SEG_T),
                                              args, 0, stream));
     count_launch(1);
@@ -1903,7 +2139,7 @@ int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int 
   const int grid = nprob < slots ? nprob : slots;
   segment_kernel<<<grid, SEG_T, 0, stream>>>(probs, nprob, codes, pos_scheme, pos_mode,
                                              (char*)scratch, stride, nmax, mmax, perm, mstart,
-                                             mlen, pos_out, tok2macro);
+                                             mlen, pos_out, tok2macro, chunk_done);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
@@ -2052,14 +2288,64 @@ int launch_score_dtype(const void* X, int d, int64_t ldx, const ProbDesc* probs,
 #undef SLS_SCORE_NV
   SLS_LAUNCH_CHECK();
   const int cb = nprob < 4096 ? nprob : 4096;
-  window_score_combine_kernel<<<cb, AGG_T, 0, stream>>>(d, probs, nprob, KP, part, score);
+  window_score_combine_kernel<<<cb, AGG_T, 0, stream>>>(d, probs, nprob, KP, 0, part, score);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+}  // namespace
+
+namespace {
+template <typename T>
+int launch_score_chunk_dtype(const void* X, int d, int64_t ldx, const ProbDesc* probs, int nprob,
+                             int64_t nmax, float* part, float* score, int pos_scheme,
+                             int pos_mode, int renorm, float* Xt, int32_t* pos,
+                             int32_t* tok2macro, cudaStream_t stream) {
+  constexpr int V = VecOf<T>::V;
+  const int nv = (d / V + AGG_T - 1) / AGG_T;
+  const int KP = chunk_parts_max(nmax);
+  const int64_t units = (int64_t)nprob * KP;
+  const int blocks = (int)(units < 65535 ? units : 65535);
+#define SLS_SCORE_NV(N)                                                                  \
+  window_score_chunk_kernel<T, N><<<blocks, AGG_T, 0, stream>>>(                         \
+      (const T*)X, d, ldx, probs, nprob, KP, part, pos_scheme, pos_mode, renorm, Xt, pos, \
+      tok2macro)
+  if (nv <= 1)
+    SLS_SCORE_NV(1);
+  else if (nv <= 2)
+    SLS_SCORE_NV(2);
+  else if (nv <= 4)
+    SLS_SCORE_NV(4);
+  else if (nv <= 8)
+    SLS_SCORE_NV(8);
+  else
+    return SLS_ERR_UNSUPPORTED;
+#undef SLS_SCORE_NV
+  SLS_LAUNCH_CHECK();
+  const int cb = nprob < 4096 ? nprob : 4096;
+  window_score_combine_kernel<<<cb, AGG_T, 0, stream>>>(d, probs, nprob, KP, 1, part, score);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
 }  // namespace
 
 size_t score_part_floats(int64_t nprob, int64_t nmax, int d) {
-  return (size_t)nprob * score_parts(nmax) * 2 * (size_t)d;
+  const int64_t kp = chunk_parts_max(nmax) > score_parts(nmax) ? chunk_parts_max(nmax)
+                                                                 : score_parts(nmax);
+  return (size_t)nprob * (size_t)kp * 2 * (size_t)d;
+}
+
+int launch_window_score_chunk(const void* X, int x_dtype, int d, int64_t ldx,
+                              const ProbDesc* probs, int nprob, int64_t nmax, float* part,
+                              float* score, int pos_scheme, int pos_mode, int renorm, float* Xt,
+                              int32_t* pos, int32_t* tok2macro, cudaStream_t stream) {
+  if (nprob <= 0) return SLS_OK;
+  if (x_dtype == SLS_F32)
+    return launch_score_chunk_dtype<float>(X, d, ldx, probs, nprob, nmax, part, score,
+                                           pos_scheme, pos_mode, renorm, Xt, pos, tok2macro,
+                                           stream);
+  return launch_score_chunk_dtype<uint16_t>(X, d, ldx, probs, nprob, nmax, part, score,
+                                            pos_scheme, pos_mode, renorm, Xt, pos, tok2macro,
+                                            stream);
 }
 
 int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,

@@ -102,10 +102,13 @@ int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const i
                             int nspec_max, int64_t nmax, const int* r_eff, const float* U, int ldu,
                             const float* R, int ldr, int bits_max, uint32_t* codes,
                             cudaStream_t stream);
+// chunk_done: the chunk windows' outputs were written by the score pass
+// (launch_window_score_chunk); they are skipped here, their macro lengths set
+// to 0 so that the aggregation skips them too.
 int launch_segment(const ProbDesc* probs, int nprob, const uint32_t* codes, int pos_scheme,
                    int pos_mode, void* scratch, int slots, int64_t nmax, int64_t mmax, int* perm,
                    int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro, int* status,
-                   cudaStream_t stream);
+                   cudaStream_t stream, int chunk_done = 0);
 int launch_preserved(int64_t B, int64_t N, int64_t M, int pf, int pl, int pos_mode, int* perm,
                      int* mstart, int* mlen, int32_t* pos_out, int32_t* tok2macro,
                      cudaStream_t stream);
@@ -125,4 +128,12 @@ int launch_aggregate(const void* X, int x_dtype, int d, int64_t ldx, const int* 
 size_t score_part_floats(int64_t nprob, int64_t nmax, int d);
 int launch_window_score(const void* X, int x_dtype, int d, int64_t ldx, const ProbDesc* probs,
                         int nprob, int64_t nmax, float* part, float* score, cudaStream_t stream);
+// The same score pass, which also writes every window's chunk-path output
+// (array_split groups of its m macro-tokens: renormalised means into Xt,
+// positions, token map) -- final for the windows the router sends to the
+// chunk path, replaced by the spectral path for the others.
+int launch_window_score_chunk(const void* X, int x_dtype, int d, int64_t ldx,
+                              const ProbDesc* probs, int nprob, int64_t nmax, float* part,
+                              float* score, int pos_scheme, int pos_mode, int renorm, float* Xt,
+                              int32_t* pos, int32_t* tok2macro, cudaStream_t stream);
 }  // namespace sls

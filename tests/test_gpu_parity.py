@@ -505,6 +505,72 @@ def test_compress_adaptive_small_batch(sls, D):
                     assert np.array_equal(t[s:e], res.tok2macro[s:e])
 
 
+def _planted_adaptive_batch():
+    """Two low-redundancy prompts with a few windows made redundant (three
+    rows repeated over the window), so that the router sends those windows
+    to the spectral path and the rest to the chunk path."""
+    w = WL.scaled(WL.WORKLOADS["adaptive"], N=1000, d=64, batch=2)
+    X = np.stack([WL.make_prompt(w, index=i, dup_frac=0.0).X for i in range(2)]).copy()
+    for (i, k) in [(0, 1), (0, 4), (1, 2)]:
+        s0 = k * 96
+        X[i, s0:s0 + 96] = np.resize(X[i, s0:s0 + 3], (96, 64))
+    prm = WL.make_params(256, 64, 8, 32, 2 * 1000, "bf16")
+    return X, prm
+
+
+def _adaptive_case(sls, X, prm, rho, pl):
+    B = X.shape[0]
+    cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=256, r=8, window=96,
+                          preserve_last=pl)
+    Xt, pos, t2m, r_eff, route = sls.compress(to_torch_x(X, "bf16"), cfg,
+                                              to_torch_x(prm.W, "bf16"),
+                                              torch.from_numpy(prm.b).cuda(),
+                                              torch.from_numpy(prm.R).cuda(),
+                                              torch.from_numpy(prm.q1).cuda())
+    torch.cuda.synchronize()
+    M = sls.output_count(cfg, 1000)
+    bounds = O.window_bounds(1000 - pl, 96)
+    route = route.cpu().numpy()[:B * len(bounds)].reshape(B, len(bounds))
+    routes = []
+    for i in range(B):
+        x64 = WL.bf16_bits_to_f32(X[i]).astype(np.float64)
+        res = O.compress_adaptive(x64, prm.w_f64(), prm.b, prm.R, prm.q1[i * 1000:(i + 1) * 1000],
+                                  O.CompressConfig(rho=rho, D=256, r=8, window=96,
+                                                   preserve_last=pl))
+        tau = O.tau_schedule(rho)
+        for k, (sp, sc) in enumerate(zip(res.info["spectral"], res.info["scores"])):
+            if abs(sc - tau) > 1e-5:
+                assert route[i, k] == int(sp), (rho, i, k, sc)
+        _check_pass(sls, x64, Xt[i].cpu().numpy(), pos[i].cpu().numpy(), t2m[i].cpu().numpy(),
+                    M, 0, pl)
+        t = t2m[i].cpu().numpy()
+        for k, (s_, e_) in enumerate(bounds):
+            if not route[i, k]:  # chunk windows: the oracle's output exactly
+                assert np.array_equal(t[s_:e_], res.tok2macro[s_:e_])
+                ms = np.unique(res.tok2macro[s_:e_])
+                assert np.array_equal(pos[i].cpu().numpy()[ms], res.pos[ms])
+                assert np.max(np.abs(Xt[i].cpu().numpy()[ms] - res.Xt[ms])) <= EMB_TOL
+        routes.append(route[i])
+    return np.array(routes)
+
+
+def test_compress_adaptive_mixed_routes(sls):
+    """Below rho = 16 the score pass writes every window's chunk output and
+    the spectral windows replace theirs: a batch with both kinds of window."""
+    X, prm = _planted_adaptive_batch()
+    for rho in (2.0, 4.0, 8.0):
+        routes = _adaptive_case(sls, X, prm, rho, 12)
+        assert routes.sum() >= 1 and (routes == 0).sum() >= 1
+
+
+def test_compress_adaptive_all_chunk_no_preserved(sls):
+    """Every window on the chunk path and no preserved tokens: the
+    aggregation has no work item at all."""
+    X, prm = _planted_adaptive_batch()
+    routes = _adaptive_case(sls, X[:1], prm, 2.0, 0)
+    assert routes.sum() == 0
+
+
 BREAK_BAND = 30.0
 
 
