@@ -1865,6 +1865,24 @@ SLS_DEV float raw_elem<uint16_t>(const uint4& r, int e) {
   return (e & 1) ? __uint_as_float(w & 0xffff0000u) : __uint_as_float(w << 16);
 }
 
+// 16-byte asynchronous copy global -> shared (zero-filled when !live), and
+// the wait for all but the newest `pending` groups of a thread's copies.
+SLS_DEV void cp16_async(void* dst, const void* src, bool live) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
+               "r"(live ? 16 : 0)
+               : "memory");
+}
+SLS_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int PENDING>
+SLS_DEV void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(PENDING) : "memory");
+}
+
+// Rows of a batch staged per thread: slot [buffer][row][column group][thread];
+// two batches of MB * NV = 8 words, the next in flight while one is used (a
+// third stage measured slower: its registers spill).
+constexpr int CHK_RING_BYTES = 2 * 8 * AGG_T * 16;
+
 template <typename T, int NV>
 __global__ void __launch_bounds__(AGG_T, 2)
 window_score_chunk_kernel(const T* __restrict__ X, int d, int64_t ldx,
@@ -1875,8 +1893,10 @@ window_score_chunk_kernel(const T* __restrict__ X, int d, int64_t ldx,
   constexpr int V = VecOf<T>::V;
   constexpr int MB = agg_batch<NV>();
   constexpr int NW = AGG_T / 32;
+  static_assert(MB * NV == 8, "staging ring sized for eight 16-byte words per thread");
   __shared__ float shq[2][MB][NW];  // row |x|^2 partials
   __shared__ float shg[2][MB][NW];  // |group mean|^2 partials, slot = the group's last row
+  extern __shared__ uint4 chk_ring[];  // [2][MB][NV][AGG_T]: each thread reads only its own words
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int units = nprob * KP;
   for (int u = blockIdx.x; u < units; u += gridDim.x) {
@@ -1914,20 +1934,37 @@ window_score_chunk_kernel(const T* __restrict__ X, int d, int64_t ldx,
     int gcur = g0, gend = chunk_gstart(n, m, g0 + 1), gcnt = 0;  // before the barrier
     int pcur = g0, pend = gend, pcnt = 0;                          // after it
     float geta = 0.f;
-    int buf = 0;
-    for (int s0 = r0; s0 < r1; s0 += MB, buf ^= 1) {
-      uint4 raw[MB][NV];
+    // the copies of batch s0 go to ring slot b; the next batch is in flight
+    // while this one is processed
+    auto issue = [&](int s0, int b) {
 #pragma unroll
       for (int j = 0; j < MB; ++j) {
-        const bool live = s0 + j < r1;
-        const T* x = X + (P.tok_row + s0 + j) * ldx;
+        const bool rl = s0 + j < r1;
+        const T* x = X + (P.tok_row + (rl ? s0 + j : r0)) * ldx;
 #pragma unroll
         for (int qv = 0; qv < NV; ++qv) {
           const int c0 = (tid + qv * AGG_T) * V;
-          raw[j][qv] = (live && c0 < d) ? __ldg(reinterpret_cast<const uint4*>(x + c0))
-                                        : make_uint4(0u, 0u, 0u, 0u);
+          const bool live = rl && c0 < d;
+          cp16_async(&chk_ring[((b * MB + j) * NV + qv) * AGG_T + tid], live ? x + c0 : x, live);
         }
       }
+      cp_async_commit();
+    };
+    issue(r0, 0);
+    int buf = 0;
+    for (int s0 = r0; s0 < r1; s0 += MB, buf ^= 1) {
+      if (s0 + MB < r1) {
+        issue(s0 + MB, buf ^ 1);
+        cp_async_wait<1>();
+      } else {
+        cp_async_wait<0>();
+      }
+      uint4 raw[MB][NV];
+#pragma unroll
+      for (int j = 0; j < MB; ++j)
+#pragma unroll
+        for (int qv = 0; qv < NV; ++qv)
+          raw[j][qv] = chk_ring[((buf * MB + j) * NV + qv) * AGG_T + tid];
       // before the barrier: row |x|^2 partials; the group sums, and for every
       // group that ends in this batch its mean (stored unscaled; a singleton is
       // its token) and the |mean|^2 partial
@@ -2305,10 +2342,15 @@ int launch_score_chunk_dtype(const void* X, int d, int64_t ldx, const ProbDesc* 
   const int KP = chunk_parts_max(nmax);
   const int64_t units = (int64_t)nprob * KP;
   const int blocks = (int)(units < 65535 ? units : 65535);
-#define SLS_SCORE_NV(N)                                                                  \
-  window_score_chunk_kernel<T, N><<<blocks, AGG_T, 0, stream>>>(                         \
-      (const T*)X, d, ldx, probs, nprob, KP, part, pos_scheme, pos_mode, renorm, Xt, pos, \
-      tok2macro)
+#define SLS_SCORE_NV(N)                                                                   \
+  do {                                                                                     \
+    SLS_CUDA_TRY(cudaFuncSetAttribute(window_score_chunk_kernel<T, N>,                      \
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize,          \
+                                      CHK_RING_BYTES));                                     \
+    window_score_chunk_kernel<T, N><<<blocks, AGG_T, CHK_RING_BYTES, stream>>>(             \
+        (const T*)X, d, ldx, probs, nprob, KP, part, pos_scheme, pos_mode, renorm, Xt, pos, \
+        tok2macro);                                                                        \
+  } while (0)
   if (nv <= 1)
     SLS_SCORE_NV(1);
   else if (nv <= 2)
