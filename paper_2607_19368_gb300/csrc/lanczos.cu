@@ -25,6 +25,7 @@ namespace {
 // Ritz values of few problems: one CTA per eigenvalue, 256 shifts per round
 // (fewer, longer rounds: the faster form when the launch has few eigenvalues)
 constexpr int EIG_THREADS = 256;  // shifts per multisection round
+constexpr double kInvShifts = 1.0 / (double)(EIG_THREADS + 1);
 
 __global__ void __launch_bounds__(EIG_THREADS)
 tridiag_eigvals_cta_kernel(LanczosBatch bt) {
@@ -84,7 +85,7 @@ tridiag_eigvals_cta_kernel(LanczosBatch bt) {
   for (int round = 0; round < 40; ++round) {
     const double lo = s_lo, hi = s_hi;
     if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-120) break;
-    const double x = lo + (hi - lo) * ((double)(tid + 1) / (double)(EIG_THREADS + 1));
+    const double x = lo + (hi - lo) * ((double)(tid + 1) * kInvShifts);
     const int c = sturm_count(sa, sb2, n, df_from_double(x));
     const unsigned ball = __ballot_sync(0xffffffffu, c > k);
     if (lane == 0) s_first[warp] = ball ? warp * 32 + __ffs(ball) - 1 : EIG_THREADS;
@@ -93,10 +94,8 @@ tridiag_eigvals_cta_kernel(LanczosBatch bt) {
       int f = EIG_THREADS;
       for (int w = 0; w < EIG_THREADS / 32; ++w) f = min(f, s_first[w]);
       // count(x_t) is non-decreasing in t: the eigenvalue lies in (x_{f-1}, x_f]
-      const double step = (hi - lo) / (double)(EIG_THREADS + 1);
-      (void)step;
-      const double xf = lo + (hi - lo) * ((double)(f + 1) / (double)(EIG_THREADS + 1));
-      const double xp = lo + (hi - lo) * ((double)f / (double)(EIG_THREADS + 1));
+      const double xf = lo + (hi - lo) * ((double)(f + 1) * kInvShifts);
+      const double xp = lo + (hi - lo) * ((double)f * kInvShifts);
       if (f < EIG_THREADS) s_hi = xf;
       if (f > 0) s_lo = xp;
     }
@@ -169,7 +168,7 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
   const int k = n - 1 - m;  // ascending index of the wanted eigenvalue
   for (int round = 0; round < 40; ++round) {
     if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-120) break;
-    const double step = (hi - lo) / 33.0;
+    const double step = (hi - lo) * (1.0 / 33.0);
     const double x = lo + step * (double)(lane + 1);
     const int c = sturm_count(sa, sb2, n, df_from_double(x));
     // count(x_t) is non-decreasing in t: the eigenvalue lies in (x_{f-1}, x_f]
