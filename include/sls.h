@@ -386,6 +386,21 @@ int sls_set_phase_events(void* const* events, int count);
 int64_t sls_launch_count(void);
 
 /*
+ * Self-test of the device-side wait limits that end a stuck kernel: every
+ * wait of the library's kernels (on an mbarrier, a ring slot or a group
+ * barrier) gives up after about a second of clock cycles, records
+ * SLS_ERR_TIMEOUT in the workspace status word and returns, leaving the
+ * context usable.  This call launches a kernel whose wait can never be
+ * satisfied -- which = 0: an mbarrier that nothing arrives at; which = 1: a
+ * group barrier of two CTAs that one CTA never reaches -- so that the limit
+ * runs out (about one second).  workspace: at least 512 device bytes (status
+ * word, then barrier words); read the outcome with sls_workspace_status().
+ * Errors: INVALID_ARG (which), WORKSPACE, CUDA.
+ */
+int sls_selftest_wait_limit(int which, void* workspace, size_t workspace_bytes,
+                            void* stream);
+
+/*
  * Reads (synchronously, on `stream`) the device status word of a workspace
  * used by sls_lanczos_topr or sls_compress: SLS_OK, or SLS_ERR_TIMEOUT when
  * a device-side wait gave up.  Clears the word.

@@ -26,7 +26,7 @@ __all__ = [
     "lanczos_topr", "simhash", "aggregate", "compress", "output_count",
     "compress_workspace_size", "workspace_status", "EXPORTED", "PHASES",
     "set_phase_events", "launch_count", "Workspace", "embed_gather", "compress_tokens",
-    "compress_tokens_workspace_size", "TokensWorkspace",
+    "compress_tokens_workspace_size", "TokensWorkspace", "selftest_wait_limit",
 ]
 
 SLS_OK = 0
@@ -108,6 +108,7 @@ EXPORTED = {
     "sls_compress": (_i32, [ctypes.POINTER(Config), _vp, _i32, _i64, _i64, _i32, _i64,
                             ctypes.POINTER(_Params), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "sls_workspace_status": (_i32, [_vp, _vp]),
+    "sls_selftest_wait_limit": (_i32, [_i32, _vp, _sz, _vp]),
     "sls_embed_gather": (_i32, [_vp, _i32, _i64, _i32, _i64, _vp, _i64, _vp, _i64, _vp, _vp]),
     "sls_compress_tokens_workspace_size": (_sz, [ctypes.POINTER(Config), _i32, _i64, _i64,
                                                  _i32]),
@@ -461,6 +462,18 @@ def set_phase_events(events) -> None:
 def launch_count() -> int:
     """Kernels launched by libsls in this process so far."""
     return int(lib().sls_launch_count())
+
+
+def selftest_wait_limit(which: int, device="cuda") -> int:
+    """Run the self-test of the device-side wait limits (which = 0: an
+    mbarrier nothing completes; 1: a group barrier one CTA never reaches) and
+    return the status it leaves (SLS_ERR_TIMEOUT = 5 when the wait gave up as
+    designed).  Takes about one second."""
+    ws = _workspace(512, device)
+    st = lib().sls_selftest_wait_limit(int(which), _ptr(ws), ws.numel(),
+                                       _stream(ws))
+    _check("sls_selftest_wait_limit", st)
+    return int(lib().sls_workspace_status(_ptr(ws), _stream(ws)))
 
 
 def workspace_status(workspace: Workspace) -> int:

@@ -889,6 +889,13 @@ int sls_set_phase_events(void* const* events, int count) {
 
 int64_t sls_launch_count(void) { return (int64_t)g_launches.load(); }
 
+int sls_selftest_wait_limit(int which, void* workspace, size_t workspace_bytes, void* stream) {
+  if (which != 0 && which != 1) return SLS_ERR_INVALID_ARG;
+  if (!ptr_ok(workspace) || workspace_bytes < 512) return SLS_ERR_WORKSPACE;
+  return launch_selftest_wait_limit(which, (int*)workspace,
+                                    (unsigned*)((char*)workspace + 256), (cudaStream_t)stream);
+}
+
 int sls_workspace_status(void* workspace, void* stream) {
   if (!workspace) return SLS_ERR_INVALID_ARG;
   int h = 0;

@@ -26,6 +26,12 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
                                   void* Phi, const int* live, int nwin, int win,
                                   cudaStream_t stream, int* status, int phi_bf16 = 0);
 
+// ---- self-test of the device-side wait limits ---------------------------------
+// which = 0: an mbarrier wait nothing completes; 1: a two-CTA group barrier
+// one CTA never reaches.  The wait gives up and writes SLS_ERR_TIMEOUT to
+// *status; barw: 256 bytes of barrier words.
+int launch_selftest_wait_limit(int which, int* status, unsigned* barw, cudaStream_t stream);
+
 // ---- input embeddings: X = E[ids] (Sec. 3.1) ---------------------------------
 // Rows of a V x d table (row stride ld_table elements) gathered into X (row
 // stride ldx); an id outside [0, V) gives a zero row and is counted in *bad
