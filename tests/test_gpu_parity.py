@@ -406,6 +406,32 @@ def test_compress_global_tiny(sls):
     assert res.Xt.shape[0] == M
 
 
+def test_compress_global_batched(sls):
+    """The global backend on a batch of prompts of equal length: one Lanczos
+    problem per prompt in one launch of the batched plan.  Per prompt: r_eff
+    against the oracle, the output invariants and the oracle's macro
+    embeddings and positions of the GPU's own groups."""
+    w = WL.scaled(WL.WORKLOADS["mistral7b"], N=900, d=64, D=256, r=16, bits=10, rho=4.0)
+    prompts = [WL.make_prompt(w, index=i) for i in range(3)]
+    prm = WL.make_params(256, 64, 16, 32, 3 * 900, "bf16")
+    X = to_torch_x(np.stack([pp.X for pp in prompts]), "bf16")
+    cfg = sls.Config.make(rho=4.0, D=256, r=16, bits=10, preserve_first=2, preserve_last=12)
+    Xt, pos, t2m, r_eff, _ = sls.compress(X, cfg, to_torch_x(prm.W, "bf16"),
+                                          torch.from_numpy(prm.b).cuda(),
+                                          torch.from_numpy(prm.R).cuda(),
+                                          torch.from_numpy(prm.q1).cuda())
+    torch.cuda.synchronize()
+    M = sls.output_count(cfg, 900)
+    for i, pp in enumerate(prompts):
+        res = O.compress_global(pp.x_f64(), prm.w_f64(), prm.b, prm.R,
+                                prm.q1[i * 900:(i + 1) * 900],
+                                O.CompressConfig(rho=4.0, D=256, r=16, bits=10, preserve_first=2,
+                                                 preserve_last=12))
+        assert int(r_eff[i].item()) == res.info["r_eff"]
+        _check_pass(sls, pp.x_f64(), Xt[i].cpu().numpy(), pos[i].cpu().numpy(),
+                    t2m[i].cpu().numpy(), M, 2, 12)
+
+
 @pytest.mark.parametrize("scheme,mode,pf,pl", [(O.POS_MEDIAN, 0, 3, 5), (O.POS_MEAN, 0, 0, 0),
                                                (O.POS_MAX, 1, 2, 12)])
 def test_compress_options(sls, scheme, mode, pf, pl):
