@@ -189,7 +189,7 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
 
 // Eigenvectors of one cluster [first, last] of nearly equal Ritz values of
 // problem p (n = r_eff), written as columns of S: inverse iteration with
-// partial-pivoting LU of T - shift I in double-float, three iterations, each
+// partial-pivoting LU of T - shift I in double-float, two iterations, each
 // followed by modified Gram-Schmidt against the cluster members already
 // found.  One thread; the work arrays (n entries each) belong to the caller.
 SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int last,
@@ -257,7 +257,7 @@ SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int
         h ^= h >> 15;
         y[i] = make_float2(0.5f + (float)(h & 0xffffu) / 65536.f, 0.f);
       }
-      for (int it = 0; it < 3; ++it) {
+      for (int it = 0; it < 2; ++it) {
         for (int i = 0; i < n - 1; ++i) {
           if (!piv[i]) {
             y[i + 1] = f2(df_sub(dfv(y[i + 1]), df_mul(dfv(dl[i]), dfv(y[i]))));

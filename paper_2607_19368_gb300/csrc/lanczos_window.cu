@@ -193,7 +193,11 @@ lanczos_window_kernel(LanczosBatch bt) {
       }
       z -= corr;
     }
-    const double b = sqrt(warp_sum_d(z * z));
+    // beta = |z| and q = z / beta from one reciprocal square root (float64
+    // divides and square roots are long sequences on this GPU's FP64 pipe)
+    const double zz = warp_sum_d(z * z);
+    const double inv = (zz > 0.0) ? rsqrt(zz) : 0.0;
+    const double b = (zz > 0.0) ? zz * inv : 0.0;
     if (lane == 0) ad[j] = a;
     reff = j + 1;
     scale = fmax(scale, fabs(a) + b);
@@ -201,7 +205,7 @@ lanczos_window_kernel(LanczosBatch bt) {
     if (lane == 0) bd[j] = b;
     qprev = q;
     bprev = b;
-    q = z / b;
+    q = z * inv;
   }
   __syncwarp();
 
