@@ -84,7 +84,8 @@ tridiag_eigvals_cta_kernel(LanczosBatch bt) {
   const int k = n - 1 - m;  // ascending index of the wanted eigenvalue
   for (int round = 0; round < 40; ++round) {
     const double lo = s_lo, hi = s_hi;
-    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-120) break;
+    // 2^-46 relative, or one float64 unit of the scaled |T| <= 1
+    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-52) break;
     const double x = lo + (hi - lo) * ((double)(tid + 1) * kInvShifts);
     const int c = sturm_count(sa, sb2, n, df_from_double(x));
     const unsigned ball = __ballot_sync(0xffffffffu, c > k);
@@ -167,7 +168,7 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
   double lo = glo * sc - pad, hi = ghi * sc + pad;
   const int k = n - 1 - m;  // ascending index of the wanted eigenvalue
   for (int round = 0; round < 40; ++round) {
-    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-120) break;
+    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-52) break;
     const double step = (hi - lo) * (1.0 / 33.0);
     const double x = lo + step * (double)(lane + 1);
     const int c = sturm_count(sa, sb2, n, df_from_double(x));

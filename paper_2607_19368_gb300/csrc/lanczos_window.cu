@@ -256,7 +256,8 @@ lanczos_window_kernel(LanczosBatch bt) {
     double lo = glo * sc - pad, hi = ghi * sc + pad;
     const int kasc = k - 1 - lane;  // ascending index of the wanted eigenvalue
     for (int it = 0; it < 160; ++it) {
-      if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-120) break;
+      // 2^-46 relative, or one float64 unit of the scaled |T| <= 1
+      if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-52) break;
       const double x = 0.5 * (lo + hi);
       if (sturm_count(sa, sb2, k, df_from_double(x)) > kasc)
         hi = x;
