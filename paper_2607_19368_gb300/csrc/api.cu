@@ -856,7 +856,8 @@ int sls_compress_tokens(const sls_config_t* cfg, const void* table, int x_dtype,
                         const sls_params_t* params, float* Xt, int32_t* pos, int32_t* tok2macro,
                         int32_t* r_eff, int32_t* route, int32_t* bad_ids, void* workspace,
                         size_t workspace_bytes, void* stream) {
-  if (validate_config(cfg) != SLS_OK) return SLS_ERR_INVALID_ARG;
+  const int vst = validate_config(cfg);
+  if (vst != SLS_OK) return vst;
   if (B < 1 || N < 1 || V < 1 || d < 1 || ld_table < d) return SLS_ERR_INVALID_ARG;
   if (x_dtype != SLS_F32 && x_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
   if (!table || !ids) return SLS_ERR_INVALID_ARG;

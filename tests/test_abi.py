@@ -64,6 +64,13 @@ def test_host_side_errors_and_counts(lib):
     assert lib.sls_embed_gather(ctypes.c_void_p(16), 1, 10, 8, 8, None, 4, ctypes.c_void_p(16),
                                 8, None, None) == 1
     assert lib.sls_embed_gather(None, 1, 10, 8, 8, None, 0, None, 8, None, None) == 0  # N = 0
+    # bf16 storage of Phi with the normalised operator: unsupported, before any CUDA call
+    bad = sls.Config.make(rho=4.0, D=256, r=8, normalize=1, phi_dtype=sls.SLS_BF16)
+    assert sls.output_count(bad, 100) == -1
+    assert lib.sls_compress_tokens(ctypes.byref(bad), ctypes.c_void_p(256), 1, 10, 64, 64,
+                                   ctypes.c_void_p(256), 1, 100, None, None, None, None, None,
+                                   None, None, None, 0, None) == 2
+    assert lib.sls_selftest_wait_limit(2, None, 0, None) == 1          # which out of range
     cfg = sls.Config.make(rho=16.0, D=2048, r=64, bits=16)
     assert (sls.compress_tokens_workspace_size(cfg, torch.bfloat16, 1, 32768, 3584)
             >= sls.compress_workspace_size(cfg, 1, 32768, 3584) + 32768 * 3584 * 2)
