@@ -27,7 +27,30 @@ SLS_DEV uint32_t simhash_row(const float* __restrict__ u, int k, const float* __
   float acc[SLS_MAX_BITS];
 #pragma unroll
   for (int l = 0; l < SLS_MAX_BITS; ++l) acc[l] = 0.0f;
-  for (int m = 0; m < k; ++m) {
+  // the row in chunks of 16 (four 16-byte loads in flight) when it is 16-byte
+  // aligned; the chain over m keeps its order either way
+  const bool vec = ((reinterpret_cast<uintptr_t>(u) & 15) == 0);
+  int m0 = 0;
+  if (vec) {
+    for (; m0 + 16 <= k; m0 += 16) {
+      float x[16];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(u + m0) + q);
+        x[4 * q] = v.x;
+        x[4 * q + 1] = v.y;
+        x[4 * q + 2] = v.z;
+        x[4 * q + 3] = v.w;
+      }
+#pragma unroll
+      for (int t = 0; t < 16; ++t) {
+#pragma unroll
+        for (int l = 0; l < SLS_MAX_BITS; ++l)
+          if (l < bits) acc[l] = __fadd_rn(acc[l], __fmul_rn(x[t], Rs[l * k + m0 + t]));
+      }
+    }
+  }
+  for (int m = m0; m < k; ++m) {
     const float um = u[m];
 #pragma unroll
     for (int l = 0; l < SLS_MAX_BITS; ++l)
@@ -74,6 +97,41 @@ simhash_batched_kernel(const ProbDesc* __restrict__ probs, const int* __restrict
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < P.n;
        i += (int64_t)gridDim.x * blockDim.x)
     codes[P.phi_row + i] = simhash_row(U + (P.phi_row + i) * ldu, kk, Rs, bits);
+}
+
+// Small problems (windows of at most SH_FLAT_MAX tokens): one thread per
+// (problem, row) over all spectral problems, R read through the read-only
+// cache (row l of R at R + l * ldr), the same float32 chain as simhash_row.
+constexpr int SH_FLAT_MAX = 64;
+
+__global__ void __launch_bounds__(256)
+simhash_flat_kernel(const ProbDesc* __restrict__ probs, const int* __restrict__ spec_list,
+                    const int* __restrict__ nspec_dev, int nspec_max, int nmax,
+                    const int* __restrict__ r_eff, const float* __restrict__ U, int ldu,
+                    const float* __restrict__ R, int ldr, uint32_t* __restrict__ codes) {
+  int nspec = nspec_max;
+  if (nspec_dev) nspec = min(nspec, *nspec_dev);
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int s = (int)(t / nmax), i = (int)(t % nmax);
+  if (s >= nspec) return;
+  const ProbDesc P = probs[spec_list ? spec_list[s] : s];
+  if (i >= P.n) return;
+  const int k = min(ldu, max(0, r_eff[s]));
+  const float* __restrict__ u = U + (P.phi_row + i) * ldu;
+  float acc[SLS_MAX_BITS];
+#pragma unroll
+  for (int l = 0; l < SLS_MAX_BITS; ++l) acc[l] = 0.0f;
+  for (int m = 0; m < k; ++m) {
+    const float um = __ldg(u + m);
+#pragma unroll
+    for (int l = 0; l < SLS_MAX_BITS; ++l)
+      if (l < P.bits) acc[l] = __fadd_rn(acc[l], __fmul_rn(um, __ldg(R + (size_t)l * ldr + m)));
+  }
+  uint32_t code = 0;
+#pragma unroll
+  for (int l = 0; l < SLS_MAX_BITS; ++l)
+    if (l < P.bits && acc[l] > 0.0f) code |= (1u << l);
+  codes[P.phi_row + i] = code;
 }
 
 // ============================================================================
@@ -2122,6 +2180,15 @@ int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const i
                             const float* R, int ldr, int bits_max, uint32_t* codes,
                             cudaStream_t stream) {
   if (nspec_max <= 0) return SLS_OK;
+  if (nmax <= SH_FLAT_MAX) {
+    const int64_t threads = (int64_t)nspec_max * nmax;
+    const int64_t blocks = (threads + 255) / 256;
+    if (blocks > 0x7fffffffLL) return SLS_ERR_UNSUPPORTED;
+    simhash_flat_kernel<<<(unsigned)blocks, 256, 0, stream>>>(
+        probs, spec_list, nspec_dev, nspec_max, (int)nmax, r_eff, U, ldu, R, ldr, codes);
+    SLS_LAUNCH_CHECK();
+    return SLS_OK;
+  }
   const size_t smem = sizeof(float) * bits_max * ldu;
   int64_t bx = (nmax + 255) / 256;
   if (bx > 1024) bx = 1024;
