@@ -544,10 +544,10 @@ def _planted_adaptive_batch():
     return X, prm
 
 
-def _adaptive_case(sls, X, prm, rho, pl):
+def _adaptive_case(sls, X, prm, rho, pl, scheme=O.POS_MAX, mode=0, renorm=1):
     B = X.shape[0]
     cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=256, r=8, window=96,
-                          preserve_last=pl)
+                          preserve_last=pl, pos_scheme=scheme, pos_mode=mode, renorm=renorm)
     Xt, pos, t2m, r_eff, route = sls.compress(to_torch_x(X, "bf16"), cfg,
                                               to_torch_x(prm.W, "bf16"),
                                               torch.from_numpy(prm.b).cuda(),
@@ -562,13 +562,17 @@ def _adaptive_case(sls, X, prm, rho, pl):
         x64 = WL.bf16_bits_to_f32(X[i]).astype(np.float64)
         res = O.compress_adaptive(x64, prm.w_f64(), prm.b, prm.R, prm.q1[i * 1000:(i + 1) * 1000],
                                   O.CompressConfig(rho=rho, D=256, r=8, window=96,
-                                                   preserve_last=pl))
+                                                   preserve_last=pl, pos_scheme=scheme,
+                                                   pos_mode=mode, renorm=bool(renorm)))
         tau = O.tau_schedule(rho)
         for k, (sp, sc) in enumerate(zip(res.info["spectral"], res.info["scores"])):
             if abs(sc - tau) > 1e-5:
                 assert route[i, k] == int(sp), (rho, i, k, sc)
-        _check_pass(sls, x64, Xt[i].cpu().numpy(), pos[i].cpu().numpy(), t2m[i].cpu().numpy(),
-                    M, 0, pl)
+        if mode == O.MODE_COMPACT:
+            assert np.array_equal(pos[i].cpu().numpy(), np.arange(M))
+        else:
+            _check_pass(sls, x64, Xt[i].cpu().numpy(), pos[i].cpu().numpy(),
+                        t2m[i].cpu().numpy(), M, 0, pl, scheme, bool(renorm))
         t = t2m[i].cpu().numpy()
         for k, (s_, e_) in enumerate(bounds):
             if not route[i, k]:  # chunk windows: the oracle's output exactly
@@ -587,6 +591,16 @@ def test_compress_adaptive_mixed_routes(sls):
     for rho in (2.0, 4.0, 8.0):
         routes = _adaptive_case(sls, X, prm, rho, 12)
         assert routes.sum() >= 1 and (routes == 0).sum() >= 1
+
+
+@pytest.mark.parametrize("scheme,mode,renorm", [(O.POS_MEDIAN, 0, 1), (O.POS_MEAN, 0, 0),
+                                                (O.POS_MAX, 1, 1)])
+def test_compress_adaptive_options(sls, scheme, mode, renorm):
+    """The score pass's chunk outputs under the other position schemes, the
+    compact position mode and without the renormalisation."""
+    X, prm = _planted_adaptive_batch()
+    routes = _adaptive_case(sls, X, prm, 4.0, 12, scheme, mode, renorm)
+    assert (routes == 0).sum() >= 1
 
 
 def test_compress_adaptive_all_chunk_no_preserved(sls):
