@@ -350,7 +350,7 @@ tridiag_eigvecs_kernel(LanczosBatch bt) {
 // Small problems (r <= 32): one warp per problem, one lane per Ritz value;
 // the lane of a cluster's first member computes the whole cluster, with its
 // work arrays in local memory.
-constexpr int EIGW_WARPS = 4;
+constexpr int EIGW_WARPS = 1;  // one problem per CTA: the fewest idle SMs at the end
 constexpr int EIGW_MAXR = 32;
 
 __global__ void __launch_bounds__(EIGW_WARPS * 32)
