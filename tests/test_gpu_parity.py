@@ -76,6 +76,23 @@ def test_feature_map_ragged_and_empty(sls):
     assert out.shape == (0, 4)
 
 
+@pytest.mark.parametrize("N,d,D", [(300, 200, 512), (129, 8, 256), (1, 72, 256)])
+def test_feature_map_tc_partial_k_tile(sls, N, d, D):
+    """bf16 shapes on the tensor-core path whose d is not a multiple of the K
+    tile (the last K block is zero-filled by the copy engine) and whose row
+    count leaves a partial row tile."""
+    g = np.random.default_rng(N + d)
+    Xb = WL.f32_to_bf16_bits((g.standard_normal((N, d)) / math.sqrt(d)).astype(np.float32))
+    Wb = WL.f32_to_bf16_bits((g.standard_normal((D, d)) * d ** -0.25).astype(np.float32))
+    b = (g.random(D) * 2 * math.pi).astype(np.float32)
+    X64, W64 = widen(Xb, "bf16"), widen(Wb, "bf16")
+    phi = sls.feature_map(to_torch_x(Xb, "bf16"), to_torch_x(Wb, "bf16"),
+                          torch.from_numpy(b).cuda()).cpu().numpy().astype(np.float64)
+    want = O.rff_features(X64, W64, b)
+    tol = feature_tolerance(X64, W64, b.astype(np.float64))
+    assert np.all(np.abs(phi - want) <= tol)
+
+
 def test_feature_map_batched_live_windows(sls):
     """One launch over a batch of prompts (Sec. 3.2) that computes only the
     row tiles touching a live window (Sec. 3.6): computed rows match the
