@@ -235,40 +235,17 @@ SLS_DEV dfloat df_add_fast(dfloat a, dfloat b) {
   return df_make(h, l);
 }
 
-// Transposed butterfly over CR rows (CR a power of two <= 32), double-float:
-// every lane holds one partial per row; afterwards lane L holds the warp sum
-// of row L >> (5 - log2 CR).  CR - 1 + 5 - log2 CR shuffles instead of 5 per
-// row.
-template <int CR>
-SLS_DEV dfloat transpose_sum_df(dfloat (&v)[CR]) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int s = 0; s < 5; ++s) {
-    const int h = 16 >> s;
-    const int nv = (CR >> s) > 1 ? (CR >> s) : 1;
-    if (nv > 1) {
-      const bool up = (lane & h) != 0;
-#pragma unroll
-      for (int i = 0; i < nv / 2; ++i) {
-        const dfloat send = up ? v[i] : v[i + nv / 2];
-        const dfloat keep = up ? v[i + nv / 2] : v[i];
-        v[i] = df_add_fast(keep, shfl_xor_df(send, h));
-      }
-    } else {
-      v[0] = df_add_fast(v[0], shfl_xor_df(v[0], h));
-    }
-  }
-  return v[0];
-}
-
 // Sweep B over two ring chunks at once with all compute threads (D >= 4 *
 // LZ_CT): thread t owns the float4 column groups t + LZ_CT q of every row, w
-// for those columns sits in registers.  Each thread accumulates its part of
-// a row against its own offset Ct (a power of two above twice max|Phi| times
-// the l1 norm of its slice of w), so the FastTwoSum steps lose nothing to a
-// loose global bound; the 2 CR per-row double-float partials are then summed
-// over the warp by one transposed butterfly and the warp sums stored to
-// bp0 / bp1 [i * LZ_CW + warp].
+// for those columns sits in registers.  Every thread of a warp accumulates
+// its part of a row against the warp's offset Ct, a power of two above twice
+// max|Phi| times the l1 norm of the warp's slice of w: each partial s - Ct is
+// then exact, a multiple of ulp(Ct) / 2 below Ct / 2 in magnitude, and so is
+// every sum of them over the warp, which makes the high parts of the
+// transposed butterfly exact additions.  The rounding errors of the
+// accumulation (captured exactly by the offset FastTwoSum) travel in the low
+// parts; each warp sum is renormalised once by TwoSum and stored to bp0 / bp1
+// [i * LZ_CW + warp].
 template <int GPT, int CR, bool FULL, typename PT>
 SLS_DEV void sweepB_team_pair(const PT* __restrict__ c0, int nr0, const PT* __restrict__ c1,
                               int nr1, int C4, const f32x2_t (&wh)[GPT][2],
@@ -276,7 +253,7 @@ SLS_DEV void sweepB_team_pair(const PT* __restrict__ c0, int nr0, const PT* __re
                               float Ct, float2* __restrict__ bp0, float2* __restrict__ bp1) {
   constexpr int R2 = 2 * CR;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  dfloat v[R2];
+  float vh[R2], vl[R2];
 #pragma unroll
   for (int i = 0; i < R2; ++i) {
     const bool first = i < CR;
@@ -297,11 +274,15 @@ SLS_DEV void sweepB_team_pair(const PT* __restrict__ c0, int nr0, const PT* __re
     float sx, sy, lx, ly;
     upk2(s, sx, sy);
     upk2(lo, lx, ly);
-    const float x = sy - Ct;  // exact
-    const float s1 = sx + x;
-    v[i] = df_make(s1 - Ct, (lx + ly) + (x - (s1 - sx)));
+    vh[i] = (sx - Ct) + (sy - Ct);  // exact (one grid, below Ct / 2)
+    vl[i] = lx + ly;
   }
-  const dfloat r = transpose_sum_df<R2>(v);
+  // the high parts add exactly; the low parts are orders of magnitude smaller
+  const float th = transpose_sum_f<R2>(vh);
+  const float tl = transpose_sum_f<R2>(vl);
+  float rh, rl;
+  two_sum(th, tl, rh, rl);
+  const dfloat r = df_make(rh, rl);
   constexpr int SH = (R2 >= 32) ? 0 : (R2 >= 16) ? 1 : (R2 >= 8) ? 2 : (R2 >= 4) ? 3 : 4;
   if ((lane & ((1 << SH) - 1)) == 0) {
     const int i = lane >> SH;
@@ -1069,9 +1050,12 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           wl[q][1] = pk2(b.z, b.w);
           wt1 += (fabsf(a.x) + fabsf(a.y)) + (fabsf(a.z) + fabsf(a.w));
         }
-        // offset of this thread's row partials: each is bounded by
-        // max|Phi| * |w slice|_1
-        const float Ct = ofs_pow2(phimax * wt1);
+        // offset of the warp's row partials: every partial of a thread, and
+        // their sum over the warp, is bounded by max|Phi| * |warp's w slice|_1
+        float wtw = wt1;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) wtw += __shfl_xor_sync(0xffffffffu, wtw, o);
+        const float Ct = ofs_pow2(phimax * wtw);
         for (int t0p = 0; t0p < nch; t0p += 2) {
           const bool two = t0p + 1 < nch;
           const int kc0 = fwd ? t0p : nch - 1 - t0p;
