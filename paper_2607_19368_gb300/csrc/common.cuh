@@ -233,21 +233,19 @@ SLS_DEV void dot2_acc2(f32x2_t& sh, f32x2_t& sl, f32x2_t x, f32x2_t yh, f32x2_t 
   sl = add2(sl, add2(e, pe));
 }
 
-// Offset accumulation step on two lanes: (s, lo) += x * (yh + yl), nyh = -yh.
-// s carries a power-of-two offset C and every partial sum it accumulates is
-// at most C/2 in magnitude, so s stays in [C/2, 3C/2] and s + p (|p| <= C/2)
-// is an exact FastTwoSum (Dekker's condition: exponent of s >= exponent of
-// p).  8 operations per element instead of Dot2's 10; the value is
-// (s - C) + lo, and s - C is exact (Sterbenz).
-SLS_DEV void ofs_acc2n(f32x2_t& s, f32x2_t& lo, f32x2_t x, f32x2_t yh, f32x2_t nyh,
-                       f32x2_t yl) {
-  const f32x2_t np = mul2(x, nyh);            // -p, p = fl(x * yh)
-  f32x2_t e = fma2(x, yh, np);                // x * yh - p, exact
+// Offset accumulation step on two lanes: (s, lo) += x * (yh + yl), 5
+// operations.  s carries a power-of-two offset C and every partial sum it
+// accumulates is at most C/2 in magnitude, so s and s1 = fl(s + x * yh) both
+// lie in [C/2, 3C/2]: s1 - s is exact, and x * yh - (s1 - s) is the rounding
+// error of the fused step, formed by a second FMA (rounded once, at the scale
+// of the low part) before x * yl joins it in lo.  The value is (s - C) + lo,
+// and s - C is exact (Sterbenz).
+SLS_DEV void ofs_fma_acc2(f32x2_t& s, f32x2_t& lo, f32x2_t x, f32x2_t yh, f32x2_t yl) {
+  const f32x2_t s1 = fma2(x, yh, s);
+  f32x2_t e = fma2(x, yh, sub2(s, s1));  // x * yh - (s1 - s)
   e = fma2(x, yl, e);
-  const f32x2_t s1 = sub2(s, np);             // fl(s + p)
-  const f32x2_t fn = add2(np, sub2(s1, s));   // minus the rounding error of s + p
   s = s1;
-  lo = add2(lo, sub2(e, fn));
+  lo = add2(lo, e);
 }
 
 // The offset for a bound B on all partial sums: a power of two C > 2 B (with

@@ -243,14 +243,13 @@ SLS_DEV dfloat df_add_fast(dfloat a, dfloat b) {
 // then exact, a multiple of ulp(Ct) / 2 below Ct / 2 in magnitude, and so is
 // every sum of them over the warp, which makes the high parts of the
 // transposed butterfly exact additions.  The rounding errors of the
-// accumulation (captured exactly by the offset FastTwoSum) travel in the low
-// parts; each warp sum is renormalised once by TwoSum and stored to bp0 / bp1
+// accumulation (each formed by an FMA at the scale of the low part) travel in
+// the low parts; each warp sum is renormalised once by TwoSum and stored to bp0 / bp1
 // [i * LZ_CW + warp].
 template <int GPT, int CR, bool FULL, typename PT>
 SLS_DEV void sweepB_team_pair(const PT* __restrict__ c0, int nr0, const PT* __restrict__ c1,
                               int nr1, int C4, const f32x2_t (&wh)[GPT][2],
-                              const f32x2_t (&nwh)[GPT][2], const f32x2_t (&wl)[GPT][2],
-                              float Ct, float2* __restrict__ bp0, float2* __restrict__ bp1) {
+                              const f32x2_t (&wl)[GPT][2], float Ct, float2* __restrict__ bp0, float2* __restrict__ bp1) {
   constexpr int R2 = 2 * CR;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float vh[R2], vl[R2];
@@ -266,8 +265,8 @@ SLS_DEV void sweepB_team_pair(const PT* __restrict__ c0, int nr0, const PT* __re
         const int cg = tid + q * LZ_CT;
         if (FULL || cg < C4) {
           const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
-          ofs_acc2n(s, lo, pk2(f.x, f.y), wh[q][0], nwh[q][0], wl[q][0]);
-          ofs_acc2n(s, lo, pk2(f.z, f.w), wh[q][1], nwh[q][1], wl[q][1]);
+          ofs_fma_acc2(s, lo, pk2(f.x, f.y), wh[q][0], wl[q][0]);
+          ofs_fma_acc2(s, lo, pk2(f.z, f.w), wh[q][1], wl[q][1]);
         }
       }
     }
@@ -1012,7 +1011,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       dfloat nacc = df_make(0.f, 0.f);
       if (P == 1) {
         // this thread's columns of w_j, from the slices into registers
-        f32x2_t wh[GPT][2], nwh[GPT][2], wl[GPT][2];
+        f32x2_t wh[GPT][2], wl[GPT][2];
         float wt1 = 0.f;  // l1 norm of this thread's slice of w_j
         const float4* wr4 = reinterpret_cast<const float4*>(wred);
         float4 wv[GPT][2];
@@ -1044,8 +1043,6 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           }
           wh[q][0] = pk2(a.x, a.y);
           wh[q][1] = pk2(a.z, a.w);
-          nwh[q][0] = pk2(-a.x, -a.y);
-          nwh[q][1] = pk2(-a.z, -a.w);
           wl[q][0] = pk2(b.x, b.y);
           wl[q][1] = pk2(b.z, b.w);
           wt1 += (fabsf(a.x) + fabsf(a.y)) + (fabsf(a.z) + fabsf(a.w));
@@ -1103,10 +1100,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           }
           // row dots s = Phi w_j, warp sums into bpart[row * LZ_CW + warp]
           if (fullD && nr0 == TCR && nr1 == TCR)
-            sweepB_team_pair<GPT, TCR, true>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bpart,
+            sweepB_team_pair<GPT, TCR, true>(ch0, nr0, ch1, nr1, C4, wh, wl, Ct, bpart,
                                              bpart + TCR * LZ_CW);
           else
-            sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, wh, nwh, wl, Ct, bpart,
+            sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, wh, wl, Ct, bpart,
                                               bpart + TCR * LZ_CW);
           if constexpr (GPT != 1) {
 #pragma unroll
