@@ -193,15 +193,33 @@ SLS_DEV float transpose_sum_f(float (&v)[CR]) {
 }
 
 // Column pass over two ring chunks at once (D >= 4 * LZ_CT; CR rows each, the
-// second chunk may be absent: nr1 = 0): acc[c] += Phi[i, c] * z'_i, Dot2.
-// FULL: both chunks full and D = 4 LZ_CT GPT (the steady state), so the row
-// and column guards vanish.
+// second chunk may be absent: nr1 = 0): acc[c] += Phi[i, c] * z'_i.  The
+// pair's rows are summed against a power-of-two offset C above twice max|Phi|
+// times the l1 norm of their z' (offset accumulation, 5 operations per pair of
+// elements), then (s - C) + lo, exact in its high part, joins the column sums
+// (ah, al) by one TwoSum.  FULL: both chunks full and D = 4 LZ_CT GPT (the
+// steady state), so the row and column guards vanish.
 template <int GPT, int CR, bool FULL, typename PT>
 SLS_DEV void sweepA_team_pair(const PT* __restrict__ c0, int nr0, int lb0,
                               const PT* __restrict__ c1, int nr1, int lb1, int C4,
-                              const float2* __restrict__ us, f32x2_t (&ah)[GPT][2],
-                              f32x2_t (&al)[GPT][2]) {
+                              const float2* __restrict__ us, float phimax,
+                              f32x2_t (&ah)[GPT][2], f32x2_t (&al)[GPT][2]) {
   const int tid = threadIdx.x;
+  float ut1 = 0.f;
+#pragma unroll
+  for (int i = 0; i < 2 * CR; ++i) {
+    const bool first = i < CR;
+    const int ii = first ? i : i - CR;
+    if (FULL || ii < (first ? nr0 : nr1)) ut1 += fabsf(us[(first ? lb0 : lb1) + ii].x);
+  }
+  const float C = ofs_pow2(phimax * ut1);
+  const f32x2_t Cp = pk2(C, C);
+  f32x2_t s[GPT][2], lo[GPT][2];
+#pragma unroll
+  for (int q = 0; q < GPT; ++q) {
+    s[q][0] = s[q][1] = Cp;
+    lo[q][0] = lo[q][1] = 0ull;
+  }
 #pragma unroll
   for (int i = 0; i < 2 * CR; ++i) {
     const bool first = i < CR;
@@ -209,16 +227,28 @@ SLS_DEV void sweepA_team_pair(const PT* __restrict__ c0, int nr0, int lb0,
     if (FULL || ii < (first ? nr0 : nr1)) {
       const PT* ch = first ? c0 : c1;
       const float2 u = us[(first ? lb0 : lb1) + ii];
-      const f32x2_t uh = pk2(u.x, u.x), nuh = pk2(-u.x, -u.x), ul = pk2(u.y, u.y);
+      const f32x2_t uh = pk2(u.x, u.x), ul = pk2(u.y, u.y);
 #pragma unroll
       for (int q = 0; q < GPT; ++q) {
         const int cg = tid + q * LZ_CT;
         if (FULL || cg < C4) {
           const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
-          dot2_acc2n(ah[q][0], al[q][0], pk2(f.x, f.y), uh, nuh, ul);
-          dot2_acc2n(ah[q][1], al[q][1], pk2(f.z, f.w), uh, nuh, ul);
+          ofs_fma_acc2(s[q][0], lo[q][0], pk2(f.x, f.y), uh, ul);
+          ofs_fma_acc2(s[q][1], lo[q][1], pk2(f.z, f.w), uh, ul);
         }
       }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < GPT; ++q) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const f32x2_t x = sub2(s[q][h], Cp);  // exact (Sterbenz)
+      const f32x2_t t = add2(ah[q][h], x);
+      const f32x2_t bb = sub2(t, ah[q][h]);
+      const f32x2_t e = add2(sub2(ah[q][h], sub2(t, bb)), sub2(x, bb));  // TwoSum error
+      ah[q][h] = t;
+      al[q][h] = add2(al[q][h], add2(e, lo[q][h]));
     }
   }
 }
@@ -1159,10 +1189,11 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           named_sync(BAR_COMPUTE, LZ_CT);
           // columns: Phi^T z' for the next step
           if (fullD && nr0 == TCR && nr1 == TCR)
-            sweepA_team_pair<GPT, TCR, true>(ch0, nr0, kc0 * cr, ch1, nr1, kc1 * cr, C4, zps, ah, al);
+            sweepA_team_pair<GPT, TCR, true>(ch0, nr0, kc0 * cr, ch1, nr1, kc1 * cr, C4, zps, phimax,
+                                              ah, al);
           else
-            sweepA_team_pair<GPT, TCR, false>(ch0, nr0, kc0 * cr, ch1, nr1, kc1 * cr, C4, zps, ah,
-                                              al);
+            sweepA_team_pair<GPT, TCR, false>(ch0, nr0, kc0 * cr, ch1, nr1, kc1 * cr, C4, zps, phimax,
+                                               ah, al);
           __syncwarp();
           if (lane == 0) {
             mbar_arrive(&emptyb[s0]);

@@ -161,7 +161,12 @@ def test_lanczos_matches_oracle(sls, name, N, D, r):
     w, p, prm = _workload_inputs(name, N=N, D=D)
     phi32 = oracle_phi32(p.x_f64(), prm.w_f64(), prm.b)
     th, th_o, Ug, U_o, al, al_o = _lanczos_case(sls, phi32, prm.q1[:N], r)
-    assert np.allclose(al, al_o, rtol=1e-9, atol=1e-12 * abs(al_o).max())
+    # the diagonal of T entry by entry: each alpha_j carries rounding at the
+    # scale of the dominant eigenvalue (every step's matvec holds its
+    # component), so the absolute term is a small multiple of max|alpha|
+    # times the double-float unit (measured: 3e-9 relative at alpha_7 of
+    # the mistral7b shape, max|alpha| = 7952, with the Ritz values at 1e-13)
+    assert np.allclose(al, al_o, rtol=1e-9, atol=1e-11 * abs(al_o).max())
     # individual Ritz vectors agree (up to the sign convention, which both
     # sides fix) where the Ritz value is well separated
     gaps = np.minimum(np.abs(np.diff(np.r_[np.inf, th_o])), np.abs(np.diff(np.r_[th_o, -np.inf])))
