@@ -248,6 +248,15 @@ SLS_DEV void ofs_fma_acc2(f32x2_t& s, f32x2_t& lo, f32x2_t x, f32x2_t yh, f32x2_
   lo = add2(lo, e);
 }
 
+// The same step on one lane.
+SLS_DEV void ofs_fma_acc(float& s, float& lo, float x, float yh, float yl) {
+  const float s1 = __fmaf_rn(x, yh, s);
+  float e = __fmaf_rn(x, yh, __fsub_rn(s, s1));
+  e = __fmaf_rn(x, yl, e);
+  s = s1;
+  lo = __fadd_rn(lo, e);
+}
+
 // The offset for a bound B on all partial sums: a power of two C > 2 B (with
 // a little slack for the rounding of B itself), clamped to [2^-100, 2^126].
 SLS_DEV float ofs_pow2(float bound) {

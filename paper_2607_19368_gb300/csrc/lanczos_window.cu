@@ -7,8 +7,10 @@
 //   z -= alpha_j q_j + beta_{j-1} q_{j-1},  two passes of classical
 //   Gram-Schmidt against q_1..q_j,  beta_j = |z|,  and the scale-relative
 //   break test beta_j <= tol * max_i(|alpha_i| + beta_i).
-// The two products with Phi are double-float on the FP32 pipes (products of
-// Phi with a double-float vector are exact, sums are compensated); the
+// The two products with Phi are double-float on the FP32 pipes (offset
+// accumulation against a power of two above twice the bound of every partial
+// sum, from the window's max|Phi|; each step's rounding error is formed by an
+// FMA and kept in the low part); the
 // vector work of a step -- alpha, the recurrence, both Gram-Schmidt passes,
 // beta and q_{j+1} = z / beta -- is float64, as in the algorithm's own
 // statement: near a breakdown (a window whose Phi has lower rank than r) the
@@ -140,32 +142,45 @@ lanczos_window_kernel(LanczosBatch bt) {
   double q = mine ? v0 / nrm : 0.0;
   double qprev = 0.0, bprev = 0.0, scale = 0.0;
   int reff = 0;
+  // max |Phi| over the window: the bound behind the offsets of both products
+  float pm = 0.f;
+  for (int c = lane; c < D; c += 32)
+    for (int i = 0; i < n; ++i) pm = fmaxf(pm, fabsf(phi_ld(Phi, (size_t)i * D + c)));
+  for (int o = 16; o > 0; o >>= 1) pm = fmaxf(pm, __shfl_xor_sync(FULL, pm, o));
   for (int j = 0; j < rmax; ++j) {
     if (mine) Qs[lane * R1 + j] = q;
     qb[lane] = f2(df_from_double(q));
     __syncwarp();
-    // y = Phi^T q_j (all rows of a column are loaded before they are used)
+    // y = Phi^T q_j (all rows of a column are loaded before they are used),
+    // offset accumulation against Cy above twice max|Phi| |q_j|_1
+    float qa = mine ? fabsf((float)q) : 0.f;
+    for (int o = 16; o > 0; o >>= 1) qa += __shfl_xor_sync(FULL, qa, o);
+    const float Cy = ofs_pow2(pm * qa);
+    float ya = 0.f;  // l1 norm of this lane's columns of y: the bound of its row partials
 #pragma unroll CU
     for (int c = lane; c < D; c += 32) {
       float ph[NV];
 #pragma unroll
       for (int i = 0; i < NV; ++i) ph[i] = (i < n) ? phi_ld(Phi, (size_t)i * D + c) : 0.f;
-      float sh = 0.f, sl = 0.f;
+      float sh = Cy, sl = 0.f;
 #pragma unroll
       for (int i = 0; i < NV; ++i) {
         if (i < n) {
           const float2 qi = qb[i];
-          dot2_acc(sh, sl, ph[i], qi.x, qi.y);
+          ofs_fma_acc(sh, sl, ph[i], qi.x, qi.y);
         }
       }
-      ys[c] = f2(df_norm(sh, sl));
+      const dfloat yv = df_norm(sh - Cy, sl);  // sh - Cy exact
+      ya += fabsf(yv.hi);
+      ys[c] = f2(yv);
     }
     __syncwarp();
     // z = Phi y: per-lane partials over its columns for every row, then the
     // transposed butterfly hands row i's sum to lane i
+    const float Cz = ofs_pow2(pm * ya);
     dfloat part[NV];
 #pragma unroll
-    for (int i = 0; i < NV; ++i) part[i] = df_make(0.f, 0.f);
+    for (int i = 0; i < NV; ++i) part[i] = df_make(Cz, 0.f);
 #pragma unroll CU
     for (int c = lane; c < D; c += 32) {
       const float2 yc = ys[c];
@@ -174,10 +189,10 @@ lanczos_window_kernel(LanczosBatch bt) {
       for (int i = 0; i < NV; ++i) ph[i] = (i < n) ? phi_ld(Phi, (size_t)i * D + c) : 0.f;
 #pragma unroll
       for (int i = 0; i < NV; ++i)
-        if (i < n) dot2_acc(part[i].hi, part[i].lo, ph[i], yc.x, yc.y);
+        if (i < n) ofs_fma_acc(part[i].hi, part[i].lo, ph[i], yc.x, yc.y);
     }
 #pragma unroll
-    for (int i = 0; i < NV; ++i) part[i] = df_norm(part[i].hi, part[i].lo);
+    for (int i = 0; i < NV; ++i) part[i] = df_norm(part[i].hi - Cz, part[i].lo);
     const dfloat zdf = transpose_reduce<NV>(part, lane);
     double z = mine ? df_to_double(zdf) : 0.0;
     // alpha_j and the three-term recurrence
