@@ -61,6 +61,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the other workloads timed after the qwen7b headline")
+    ap.add_argument("--sweep-steps", type=int, default=20)
     ap.add_argument("--ref-sample", type=int, default=1024,
                     help="tokens the oracle compresses per step of --impl reference")
     return ap.parse_args()
@@ -164,6 +167,12 @@ def max_over_ranks(values, world, device):
         import torch.distributed as dist
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return [float(x) for x in t.tolist()]
+
+
+def lanczos_one_pass_bytes(n_tokens, D, r, esz=4):
+    """Per launch: what one fused pass per step has to move, one sweep over
+    Phi per step (r D esz bytes per token) plus the same basis traffic."""
+    return n_tokens * (esz * r * D + 16 * r * (r + 1))
 
 
 def lanczos_algorithmic_bytes(n_tokens, D, r, esz=4):
@@ -367,255 +376,360 @@ def vocab_table(X, ids, V, dev):
     return table
 
 
-def run_native(args, rank, world):
-    import numpy as np
-    import torch
-    import torch.distributed as dist
+def make_config(sls, w, rho, normalize=False, phi="f32"):
+    phi_code = sls.SLS_BF16 if phi == "bf16" else sls.SLS_F32
+    backend = {"adaptive": sls.BACKEND_ADAPTIVE, "local": sls.BACKEND_LOCAL}.get(
+        w.backend, sls.BACKEND_GLOBAL)
+    return sls.Config.make(backend=backend, rho=rho, D=w.D, r=w.r, bits=w.bits,
+                           window=w.window if windowed(w) else 2048,
+                           preserve_first=w.preserve_first, preserve_last=w.preserve_last,
+                           normalize=int(normalize), phi_dtype=phi_code)
 
+
+class Run:
+    """One workload resident on the device: inputs, parameters, outputs and
+    the compress workspace, ready for timed sls_compress calls."""
+
+    def __init__(self, sls, w, rho, rank, dev, normalize=False, phi="f32"):
+        import numpy as np
+        import torch
+        import workloads as WL
+        self.sls, self.w, self.rho, self.dev, self.phi = sls, w, rho, dev, phi
+        self.X, self.ids = device_inputs(w, rank, dev)
+        self.prm = WL.params_for(w)
+        self.Wt = torch.from_numpy(self.prm.W.view(np.int16)).view(torch.bfloat16).to(dev)
+        self.bt = torch.from_numpy(self.prm.b).to(dev)
+        self.Rt = torch.from_numpy(self.prm.R).to(dev)
+        self.qt = torch.from_numpy(self.prm.q1).to(dev)
+        self.cfg = make_config(sls, w, rho, normalize, phi)
+        B, N, d = w.batch, w.N, w.d
+        self.M = sls.output_count(self.cfg, N)
+        self.ws = sls.Workspace(self.cfg, B, N, d, dev)
+        self.out = (torch.empty((B, self.M, d), dtype=torch.float32, device=dev),
+                    torch.empty((B, self.M), dtype=torch.int32, device=dev),
+                    torch.empty((B, N), dtype=torch.int32, device=dev))
+        self.Xin = self.X if w.batch > 1 else self.X.view(1, N, d)
+
+    def step(self, X=None, out=None):
+        return self.sls.compress(self.Xin if X is None else X, self.cfg, self.Wt, self.bt,
+                                 self.Rt, self.qt, workspace=self.ws,
+                                 out=self.out if out is None else out)
+
+    def timed(self, steps, warmup, world):
+        """warmup untimed calls, then `steps` calls between CUDA events (max
+        over ranks), per-phase events, the launch count and the clocks
+        sampled meanwhile."""
+        import torch
+        import torch.distributed as dist
+        sls, w = self.sls, self.w
+        for _ in range(warmup):
+            res = self.step()
+        torch.cuda.synchronize()
+        if sls.workspace_status(self.ws) != 0:
+            raise RuntimeError("device wait timed out during warm-up")
+        B = w.batch
+        if windowed(w):
+            lens = window_lengths(w)
+            route = res[4].cpu().numpy()[:B * len(lens)].reshape(B, len(lens))
+            self.lz_tokens = int(sum(int(route[i, k]) * lens[k]
+                                     for i in range(B) for k in range(len(lens))))
+            self.n_spec = int(route.sum())
+        else:
+            self.lz_tokens = w.N - w.preserve_first - w.preserve_last
+            self.n_spec = 1
+        nph = len(sls.PHASES)
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * nph)]
+              for _ in range(steps)]
+        for evs in ev:  # events are created lazily: record each once before use
+            for e in evs:
+                e.record()
+        start = torch.cuda.Event(enable_timing=True)
+        end = torch.cuda.Event(enable_timing=True)
+        bus = str(self.dev.index)
+        try:
+            u = str(torch.cuda.get_device_properties(self.dev).uuid)
+            bus = u if u.startswith("GPU-") else "GPU-" + u
+        except Exception:
+            pass
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        clocks = Clocks(bus)
+        time.sleep(0.3)
+        launches0 = sls.launch_count()
+        start.record()
+        for k in range(steps):
+            sls.set_phase_events(ev[k])
+            self.step()
+        end.record()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        launches = sls.launch_count() - launches0
+        clk = clocks.stop()
+        sls.set_phase_events(None)
+        if sls.workspace_status(self.ws) != 0:
+            raise RuntimeError("device wait timed out during the timed region")
+        ms = start.elapsed_time(end) / steps
+        phases = {name: statistics.mean(ev[k][2 * i].elapsed_time(ev[k][2 * i + 1])
+                                        for k in range(steps))
+                  for i, name in enumerate(sls.PHASES)}
+        ms_max = max_over_ranks([ms], world, self.dev)[0]
+        return {"ms": ms_max, "phases": phases, "launches": launches, "clocks": clk,
+                "value": world * B * w.N / (ms_max / 1e3)}
+
+    def roofline(self, lanczos_ms):
+        """Roofline of the dominant kernel, the persistent Lanczos kernel, over
+        the Lanczos phase's CUDA-event time: the survey's algorithmic count
+        (two sweeps over Phi per step plus the basis traffic) and the count
+        of what one fused pass per step must move (one sweep over Phi per
+        step plus the basis traffic)."""
+        w = self.w
+        esz = 2 if self.phi == "bf16" else 4
+        alg = lanczos_algorithmic_bytes(self.lz_tokens, w.D, w.r, esz)
+        one = lanczos_one_pass_bytes(self.lz_tokens, w.D, w.r, esz)
+        lz_s = lanczos_ms / 1e3
+        peak, src = peaks()
+        achieved = alg / lz_s / 1e9 if lz_s > 0 else 0.0
+        ach1 = one / lz_s / 1e9 if lz_s > 0 else 0.0
+        roof = {"bound": "hbm", "kernel": "lanczos_kernel", "achieved": achieved, "peak": peak,
+                "unit": "GB/s", "frac": achieved / peak, "peak_source": src,
+                "algorithmic_bytes": alg, "one_pass_bytes": one,
+                "achieved_one_pass": ach1, "frac_one_pass": ach1 / peak, "traffic": None}
+        tr = os.path.join(ROOT, "profiles", "lanczos_traffic.json")
+        if os.path.exists(tr):
+            try:
+                with open(tr) as f:
+                    t = json.load(f)
+                if (t.get("workload") == w.name and t.get("kernel_rev") == LANCZOS_KERNEL_REV
+                        and self.phi == "f32" and abs(float(t.get("rho", w.rho)) - self.rho) < 1e-9):
+                    roof["traffic"] = t["dram_bytes_per_launch"]
+                    if lz_s > 0:
+                        roof["traffic_achieved"] = t["dram_bytes_per_launch"] / lz_s / 1e9
+                        roof["traffic_frac"] = roof["traffic_achieved"] / peak
+            except Exception:
+                pass
+        return roof
+
+
+def e2e_measure(run, args, world):
+    """The same metric end to end through the public API with host buffers:
+    every step copies its embeddings in from pinned host memory and its
+    outputs back out (serial and double-buffered patterns), and the path
+    from token ids with the embedding table resident on the device."""
+    import torch
+    sls, w, dev, cfg = run.sls, run.w, run.dev, run.cfg
+    Xin, out = run.Xin, run.out
+    Xt, pos, t2m = out
+    B, N, d = w.batch, w.N, w.d
+    Xh = Xin.cpu().pin_memory()
+
+    def host_outs():
+        return (torch.empty(Xt.shape, dtype=Xt.dtype).pin_memory(),
+                torch.empty(pos.shape, dtype=pos.dtype).pin_memory(),
+                torch.empty(t2m.shape, dtype=t2m.dtype).pin_memory())
+
+    def timed(fn, steps):
+        # warm-up: the first copies through freshly pinned buffers of a GB or
+        # more run several times slower than later ones
+        fn(3)
+        torch.cuda.synchronize()
+        s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s2.record()
+        fn(steps)
+        e2.record()
+        torch.cuda.synchronize()
+        return s2.elapsed_time(e2) / steps
+
+    # serial: copy in, compress, copy out, one after the other
+    Xd = torch.empty_like(Xin)
+    ho = host_outs()
+
+    def serial(n):
+        for _ in range(n):
+            Xd.copy_(Xh, non_blocking=True)
+            run.step(Xd, out)
+            for h, o in zip(ho, out):
+                h.copy_(o, non_blocking=True)
+
+    ms_serial = timed(serial, args.e2e_steps)
+    # pipelined (the serving pattern): two device buffers; a copy stream
+    # brings step k+1's inputs in and takes step k's outputs out while step k
+    # compresses on the compute stream
+    comp = torch.cuda.current_stream(dev)
+    cps = torch.cuda.Stream(device=dev)
+    outs = [out, (torch.empty_like(Xt), torch.empty_like(pos), torch.empty_like(t2m))]
+    hos = [ho, host_outs()]
+
+    def pipeline(Ih, call):
+        Ids = [torch.empty(Ih.shape, dtype=Ih.dtype, device=dev) for _ in range(2)]
+        h2d = [torch.cuda.Event() for _ in range(2)]
+        done = [torch.cuda.Event() for _ in range(2)]
+        d2h = [torch.cuda.Event() for _ in range(2)]
+
+        def go(n):
+            cps.wait_stream(comp)
+            with torch.cuda.stream(cps):
+                Ids[0].copy_(Ih, non_blocking=True)
+                h2d[0].record(cps)
+            for k in range(n):
+                b = k % 2
+                if k + 1 < n:
+                    nb = (k + 1) % 2
+                    with torch.cuda.stream(cps):
+                        if k >= 1:
+                            cps.wait_event(done[nb])
+                        Ids[nb].copy_(Ih, non_blocking=True)
+                        h2d[nb].record(cps)
+                comp.wait_event(h2d[b])
+                if k >= 2:
+                    comp.wait_event(d2h[b])
+                call(Ids[b], outs[b])
+                done[b].record(comp)
+                with torch.cuda.stream(cps):
+                    cps.wait_event(done[b])
+                    for h, o in zip(hos[b], outs[b]):
+                        h.copy_(o, non_blocking=True)
+                    d2h[b].record(cps)
+            comp.wait_stream(cps)
+        return go
+
+    ms_pipe = timed(pipeline(Xh, lambda x, o: run.step(x, o)), args.e2e_steps)
+    # from token ids: the model's embedding table stays in HBM and only the
+    # ids come in; the lookup X = E[ids] runs inside the call
+    adaptive = w.batch > 1
+    table = vocab_table(run.X, run.ids, w.V, dev)
+    Ih = torch.from_numpy(run.ids if adaptive else run.ids.reshape(N)).pin_memory()
+    tws = sls.TokensWorkspace(cfg, table.dtype, B, N, d, dev)
+    ms_ids = timed(pipeline(Ih, lambda i, o: sls.compress_tokens(i, table, cfg, run.Wt, run.bt,
+                                                                   run.Rt, run.qt, workspace=tws,
+                                                                   out=o)),
+                   args.e2e_steps)
+    del table, tws
+    m2 = max_over_ranks([ms_pipe, ms_serial, ms_ids], world, dev)
+    d2h_bytes = Xt.numel() * 4 + pos.numel() * 4 + t2m.numel() * 4
+    pipe_v = world * B * N / (m2[0] / 1e3)
+    serial_v = world * B * N / (m2[1] / 1e3)
+    # both patterns go through the public API; the faster one is reported
+    # (with copies of several GB per step the double-buffered pattern can lose
+    # to the serial one)
+    pipelined_wins = pipe_v >= serial_v
+    return {"value": max(pipe_v, serial_v), "unit": UNIT,
+            "h2d_bytes_per_step": Xin.numel() * 2,
+            "d2h_bytes_per_step": d2h_bytes,
+            "mode": ("pipelined: the copies of step k+1 in and step k out overlap the "
+                     "compression of step k on a second stream (double-buffered)")
+                    if pipelined_wins else
+                    ("serial: copy in, compress, copy out, one after the other (faster "
+                     "here than the double-buffered pattern)"),
+            "pipelined_value": pipe_v,
+            "serial_value": serial_v,
+            "from_token_ids": {
+                "value": world * B * N / (m2[2] / 1e3), "unit": UNIT,
+                "h2d_bytes_per_step": int(Ih.numel()) * 4,
+                "d2h_bytes_per_step": d2h_bytes,
+                "mode": "double-buffered as above; token ids in, the V x d bf16 embedding "
+                        "table resident on the device, lookup inside sls_compress_tokens"}}
+
+
+def full_config_oracle(run, rho):
+    """The oracle's whole pass on the full prompt of a single-prompt
+    workload, timed once with all cores and once on one core (a child
+    process with single-threaded BLAS), and the end-to-end agreement of the
+    GPU pass with it (fraction of identical SimHash codes, adjusted Rand index
+    of the token maps; reported, not pinned)."""
+    import numpy as np
     import workloads as WL
+    from tests.gpu_util import adjusted_rand_index
+    import oracle as O
+    w, sls = run.w, run.sls
+    p = WL.make_prompt(w)
+    X64 = p.x_f64()
+    cfg = oracle_config(w, rho)
+    t = time.perf_counter()
+    res = O.compress_global(X64, run.prm.w_f64(), run.prm.b, run.prm.R, run.prm.q1, cfg)
+    secs = time.perf_counter() - t
+    full = {"value": w.N / secs, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "seconds": round(secs, 2),
+            "sample": f"oracle compress_global (numpy float64, all cores) on the whole "
+                      f"{w.name} prompt, N={w.N} d={w.d} D={w.D} r={w.r} b={w.bits} "
+                      f"rho={rho:g}: the same config as the GPU line"}
+    one = single_core_baseline(w, rho, w.N, budget_s=0.0)
+    if one is not None:
+        full["single_core"] = one
+    # GPU codes from the kernels sls_compress runs, its token map from the
+    # last timed call
+    Nc = w.N - w.preserve_first - w.preserve_last
+    Xc = run.X[w.preserve_first:w.preserve_first + Nc]
+    phi = sls.feature_map(Xc, run.Wt, run.bt)
+    _, U, r_eff, _, _ = sls.lanczos_topr(phi, run.qt[:Nc], w.r)
+    codes_g = sls.simhash(U, run.Rt, res.info["bits"], k_dev=r_eff).cpu().numpy().view(np.uint32)
+    del phi, U
+    run.step()
+    t2m = run.out[2][0].cpu().numpy()
+    agree = {"workload": w.name,
+             "codes_identical": float(np.mean(codes_g == res.info["codes"])),
+             "ari_tok2macro": adjusted_rand_index(t2m, res.tok2macro),
+             "clusters_gpu": int(np.unique(codes_g).size),
+             "clusters_oracle": int(res.info["n_clusters"]),
+             "note": "reported, not pinned: float32 Phi and double-float Lanczos on the GPU "
+                     "against float64 in the oracle flip SimHash bits whose dot is near zero"}
+    return full, agree
+
+
+def sweep_entry(sls, name, rho, rank, dev, world, steps, warmup):
+    """One more workload timed in the same process (20 steps by default):
+    tokens/s, ms per step, the Lanczos roofline and the clocks."""
+    import torch
+    w = workload(name)
+    run = Run(sls, w, rho, rank, dev)
+    t = run.timed(steps, warmup, world)
+    roof = run.roofline(t["phases"]["lanczos"])
+    ent = {"workload": name, "N": w.N, "d": w.d, "D": w.D, "r": w.r, "rho": rho,
+           "batch": w.batch, "tokens_per_s": t["value"], "ms_per_step": t["ms"],
+           "lanczos_ms": t["phases"]["lanczos"], "lanczos_frac": roof["frac"],
+           "lanczos_frac_one_pass": roof["frac_one_pass"],
+           "lanczos_gbs_one_pass": roof["achieved_one_pass"],
+           "phases_ms": t["phases"], "clocks": t["clocks"], "steps": steps,
+           "spectral_tokens": run.lz_tokens}
+    if windowed(w):
+        ent["spectral_windows"] = run.n_spec
+    del run
+    torch.cuda.empty_cache()
+    return ent
+
+
+def run_native(args, rank, world):
+    import torch
+
     import paper_2607_19368_gb300 as sls
 
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
     w = workload(args.workload)
     rho = args.rho or w.rho
-    adaptive = w.backend == "adaptive"
-    local = w.backend == "local"
-    X, ids = device_inputs(w, rank, dev)
-    prm = WL.params_for(w)
-    Wt = torch.from_numpy(prm.W.view(np.int16)).view(torch.bfloat16).to(dev)
-    bt = torch.from_numpy(prm.b).to(dev)
-    Rt = torch.from_numpy(prm.R).to(dev)
-    qt = torch.from_numpy(prm.q1).to(dev)
-    phi_code = sls.SLS_BF16 if args.phi == "bf16" else sls.SLS_F32
-    if adaptive:
-        cfg = sls.Config.make(backend=sls.BACKEND_ADAPTIVE, rho=rho, D=w.D, r=w.r, bits=w.bits,
-                              window=w.window, preserve_first=w.preserve_first,
-                              preserve_last=w.preserve_last, normalize=int(args.normalize),
-                              phi_dtype=phi_code)
-    elif local:
-        cfg = sls.Config.make(backend=sls.BACKEND_LOCAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
-                              window=w.window, preserve_first=w.preserve_first,
-                              preserve_last=w.preserve_last, normalize=int(args.normalize),
-                              phi_dtype=phi_code)
-    else:
-        cfg = sls.Config.make(backend=sls.BACKEND_GLOBAL, rho=rho, D=w.D, r=w.r, bits=w.bits,
-                              preserve_first=w.preserve_first, preserve_last=w.preserve_last,
-                              normalize=int(args.normalize), phi_dtype=phi_code)
-    B, N, d = w.batch, w.N, w.d
-    M = sls.output_count(cfg, N)
-    ws = sls.Workspace(cfg, B, N, d, dev)
-    Xt = torch.empty((B, M, d), dtype=torch.float32, device=dev)
-    pos = torch.empty((B, M), dtype=torch.int32, device=dev)
-    t2m = torch.empty((B, N), dtype=torch.int32, device=dev)
-    out = (Xt, pos, t2m)
-    Xin = X if adaptive else X.view(1, N, d)
-
-    def step():
-        return sls.compress(Xin, cfg, Wt, bt, Rt, qt, workspace=ws, out=out)
-
-    for _ in range(args.warmup):
-        res = step()
-    torch.cuda.synchronize()
-    if sls.workspace_status(ws) != 0:
-        raise RuntimeError("device wait timed out during warm-up")
-    # tokens that run through the spectral chain (Lanczos)
-    if adaptive or local:
-        lens = window_lengths(w)
-        route = res[4].cpu().numpy()[:B * len(lens)].reshape(B, len(lens))
-        lz_tokens = int(sum(int(route[i, k]) * lens[k]
-                            for i in range(B) for k in range(len(lens))))
-        n_spec = int(route.sum())
-    else:
-        lz_tokens = N - w.preserve_first - w.preserve_last
-        n_spec = 1
-
-    nph = len(sls.PHASES)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * nph)]
-          for _ in range(args.steps)]
-    for evs in ev:  # events are created lazily: record each once before use
-        for e in evs:
-            e.record()
-    start = torch.cuda.Event(enable_timing=True)
-    end = torch.cuda.Event(enable_timing=True)
-    bus = str(dev.index)
-    try:
-        u = str(torch.cuda.get_device_properties(dev).uuid)
-        bus = u if u.startswith("GPU-") else "GPU-" + u
-    except Exception:
-        pass
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    clocks = Clocks(bus)
-    time.sleep(0.3)
-    launches0 = sls.launch_count()
-    start.record()
-    for k in range(args.steps):
-        sls.set_phase_events(ev[k])
-        step()
-    end.record()
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    launches = sls.launch_count() - launches0
-    clk = clocks.stop()
-    sls.set_phase_events(None)
-    if sls.workspace_status(ws) != 0:
-        raise RuntimeError("device wait timed out during the timed region")
-    ms = start.elapsed_time(end) / args.steps
-    phases = {name: statistics.mean(ev[k][2 * i].elapsed_time(ev[k][2 * i + 1])
-                                    for k in range(args.steps))
-              for i, name in enumerate(sls.PHASES)}
-    ms_max = max_over_ranks([ms], world, dev)[0]
-    value = world * B * N / (ms_max / 1e3)
-
-    # roofline of the dominant kernel (the persistent Lanczos kernel)
-    alg = lanczos_algorithmic_bytes(lz_tokens, w.D, w.r, 2 if args.phi == "bf16" else 4)
-    lz_s = phases["lanczos"] / 1e3
-    peak, src = peaks()
-    achieved = alg / lz_s / 1e9 if lz_s > 0 else 0.0
-    roof = {"bound": "hbm", "kernel": "lanczos_kernel", "achieved": achieved, "peak": peak,
-            "unit": "GB/s", "frac": achieved / peak, "peak_source": src,
-            "algorithmic_bytes": alg, "traffic": None}
-    tr = os.path.join(ROOT, "profiles", "lanczos_traffic.json")
-    if os.path.exists(tr):
-        try:
-            with open(tr) as f:
-                t = json.load(f)
-            if (t.get("workload") == w.name and t.get("kernel_rev") == LANCZOS_KERNEL_REV
-                    and not windowed(w) and args.phi == "f32"):
-                roof["traffic"] = t["dram_bytes_per_launch"]
-                # the same launch timed against the bytes DRAM actually moved:
-                # the fused pass reads Phi once per step, so the kernel is far
-                # from the HBM bound (its compensated arithmetic bounds it)
-                if lz_s > 0:
-                    roof["traffic_achieved"] = t["dram_bytes_per_launch"] / lz_s / 1e9
-                    roof["traffic_frac"] = roof["traffic_achieved"] / peak
-        except Exception:
-            pass
-
-    # end to end through the public API with host buffers: every step copies
-    # its embeddings in from pinned host memory and its outputs back out
-    e2e = None
-    if not args.no_e2e:
-        Xh = Xin.cpu().pin_memory()
-
-        def host_outs():
-            return (torch.empty(Xt.shape, dtype=Xt.dtype).pin_memory(),
-                    torch.empty(pos.shape, dtype=pos.dtype).pin_memory(),
-                    torch.empty(t2m.shape, dtype=t2m.dtype).pin_memory())
-
-        def timed(fn, steps):
-            # warm-up: the first copies through freshly pinned buffers of a
-            # GB or more run several times slower than later ones
-            fn(3)
-            torch.cuda.synchronize()
-            s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            s2.record()
-            fn(steps)
-            e2.record()
-            torch.cuda.synchronize()
-            return s2.elapsed_time(e2) / steps
-
-        # serial: copy in, compress, copy out, one after the other
-        Xd = torch.empty_like(Xin)
-        ho = host_outs()
-
-        def serial(n):
-            for _ in range(n):
-                Xd.copy_(Xh, non_blocking=True)
-                sls.compress(Xd, cfg, Wt, bt, Rt, qt, workspace=ws, out=out)
-                for h, o in zip(ho, out):
-                    h.copy_(o, non_blocking=True)
-
-        ms_serial = timed(serial, args.e2e_steps)
-        # pipelined (the serving pattern): two device buffers; a copy stream
-        # brings step k+1's inputs in and takes step k's outputs out while
-        # step k compresses on the compute stream
-        comp = torch.cuda.current_stream(dev)
-        cps = torch.cuda.Stream(device=dev)
-        outs = [out, (torch.empty_like(Xt), torch.empty_like(pos), torch.empty_like(t2m))]
-        hos = [ho, host_outs()]
-
-        def pipeline(Ih, run):
-            Ids = [torch.empty(Ih.shape, dtype=Ih.dtype, device=dev) for _ in range(2)]
-            h2d = [torch.cuda.Event() for _ in range(2)]
-            done = [torch.cuda.Event() for _ in range(2)]
-            d2h = [torch.cuda.Event() for _ in range(2)]
-
-            def go(n):
-                cps.wait_stream(comp)
-                with torch.cuda.stream(cps):
-                    Ids[0].copy_(Ih, non_blocking=True)
-                    h2d[0].record(cps)
-                for k in range(n):
-                    b = k % 2
-                    if k + 1 < n:
-                        nb = (k + 1) % 2
-                        with torch.cuda.stream(cps):
-                            if k >= 1:
-                                cps.wait_event(done[nb])
-                            Ids[nb].copy_(Ih, non_blocking=True)
-                            h2d[nb].record(cps)
-                    comp.wait_event(h2d[b])
-                    if k >= 2:
-                        comp.wait_event(d2h[b])
-                    run(Ids[b], outs[b])
-                    done[b].record(comp)
-                    with torch.cuda.stream(cps):
-                        cps.wait_event(done[b])
-                        for h, o in zip(hos[b], outs[b]):
-                            h.copy_(o, non_blocking=True)
-                        d2h[b].record(cps)
-                comp.wait_stream(cps)
-            return go
-
-        ms_pipe = timed(pipeline(Xh, lambda x, o: sls.compress(x, cfg, Wt, bt, Rt, qt,
-                                                                 workspace=ws, out=o)),
-                        args.e2e_steps)
-        # from token ids: the model's embedding table stays in HBM and only
-        # the ids come in; the lookup X = E[ids] runs inside the call
-        table = vocab_table(X, ids, w.V, dev)
-        Ih = torch.from_numpy(ids if adaptive else ids.reshape(N)).pin_memory()
-        tws = sls.TokensWorkspace(cfg, table.dtype, B, N, d, dev)
-        ms_ids = timed(pipeline(Ih, lambda i, o: sls.compress_tokens(i, table, cfg, Wt, bt, Rt,
-                                                                       qt, workspace=tws,
-                                                                       out=o)),
-                       args.e2e_steps)
-        del table, tws
-        m2 = max_over_ranks([ms_pipe, ms_serial, ms_ids], world, dev)
-        d2h_bytes = Xt.numel() * 4 + pos.numel() * 4 + t2m.numel() * 4
-        pipe_v = world * B * N / (m2[0] / 1e3)
-        serial_v = world * B * N / (m2[1] / 1e3)
-        # both patterns go through the public API; the faster one is reported
-        # (with copies of several GB per step the double-buffered pattern can
-        # lose to the serial one)
-        pipelined_wins = pipe_v >= serial_v
-        e2e = {"value": max(pipe_v, serial_v), "unit": UNIT,
-               "h2d_bytes_per_step": Xin.numel() * 2,
-               "d2h_bytes_per_step": d2h_bytes,
-               "mode": ("pipelined: the copies of step k+1 in and step k out overlap the "
-                        "compression of step k on a second stream (double-buffered)")
-                       if pipelined_wins else
-                       ("serial: copy in, compress, copy out, one after the other (faster "
-                        "here than the double-buffered pattern)"),
-               "pipelined_value": pipe_v,
-               "serial_value": serial_v,
-               "from_token_ids": {
-                   "value": world * B * N / (m2[2] / 1e3), "unit": UNIT,
-                   "h2d_bytes_per_step": int(Ih.numel()) * 4,
-                   "d2h_bytes_per_step": d2h_bytes,
-                   "mode": "double-buffered as above; token ids in, the V x d bf16 embedding "
-                           "table resident on the device, lookup inside "
-                           "sls_compress_tokens"}}
-
+    run = Run(sls, w, rho, rank, dev, args.normalize, args.phi)
+    t = run.timed(args.steps, args.warmup, world)
+    roof = run.roofline(t["phases"]["lanczos"])
+    e2e = None if args.no_e2e else e2e_measure(run, args, world)
+    cpu, agree, sweep = None, None, None
+    if rank == 0 and world == 1:
+        if not args.no_cpu_baseline:
+            p, pidx = sample_prompt(w)
+            cpu = cpu_baseline(w, rho, p.x_f64(), run.prm, args.cpu_sample, pidx)
+            if not windowed(w) and not args.normalize and args.phi == "f32":
+                cpu["full_config"], agree = full_config_oracle(run, rho)
+    B, N = w.batch, w.N
+    n_spec, lz_tokens = run.n_spec, run.lz_tokens
+    del run
+    torch.cuda.empty_cache()
+    if rank == 0 and world == 1 and not args.no_sweep and args.workload == "qwen7b" \
+            and not args.normalize and args.phi == "f32":
+        sweep = [sweep_entry(sls, nm, r_ or workload(nm).rho, rank, dev, world,
+                             args.sweep_steps, 3)
+                 for nm, r_ in (("mistral7b", None), ("qwen14b", None), ("adaptive", 16.0))]
     if rank != 0:
         return
-    cpu = None
-    if not args.no_cpu_baseline and world == 1:
-        p, pidx = sample_prompt(w)
-        cpu = cpu_baseline(w, rho, p.x_f64(), prm, args.cpu_sample, pidx)
     extra = {"parallelism": f"replicas x{world}",
              "inputs": "bf16 embeddings and Omega; float32 Phi; double-float Lanczos vectors"}
     if windowed(w):
@@ -625,14 +739,18 @@ def run_native(args, rank, world):
     if args.phi == "bf16":
         extra["inputs"] = ("bf16 embeddings and Omega; Phi stored as bf16 (opt-in); "
                            "double-float Lanczos vectors")
-    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
+    line = {"metric": METRIC, "value": t["value"], "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t["ms"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f32", "data": "synthetic",
             "config": config_dict(w, rho, extra),
-            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
-            "clocks": clk, "phases_ms": phases,
-            "lanczos_gbs_algorithmic": achieved}
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": t["launches"],
+            "clocks": t["clocks"], "phases_ms": t["phases"],
+            "lanczos_gbs_algorithmic": roof["achieved"]}
+    if agree is not None:
+        line["agreement"] = agree
+    if sweep is not None:
+        line["sweep"] = sweep
     print(json.dumps(line), flush=True)
 
 

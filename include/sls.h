@@ -197,7 +197,10 @@ size_t sls_lanczos_workspace_size(int64_t N, int D, int r);
  * Outputs: theta[r] doubles, Ritz values in descending order (entries past
  * r_eff are 0); U: N x r floats, column m the Ritz vector of theta[m], signed
  * so that the first component of the eigenvector of T is positive (columns
- * past r_eff are 0); r_eff: one int32 (device).  Optional (may be NULL):
+ * past r_eff are 0); r_eff: one int32 (device), set to -1 when the call is
+ * enqueued and left at -1 if a device-side wait of the Lanczos kernel gave up
+ * (sls_workspace_status then reports SLS_ERR_TIMEOUT; theta and U are then
+ * zero).  Optional (may be NULL):
  * alpha[r], beta[r] doubles receive the diagonal and off-diagonal of T.
  * Vectors are kept in double-float (two fp32) precision; Phi is read as
  * stored.  Errors: INVALID_ARG (sizes, NULL, r > SLS_MAX_R), WORKSPACE,
@@ -221,6 +224,38 @@ int sls_lanczos_topr_ex(const void* Phi, int phi_dtype, int64_t N, int D, int r,
                         const double* q1, double tol, double* theta, float* U,
                         int32_t* r_eff, double* alpha, double* beta,
                         void* workspace, size_t workspace_bytes, void* stream);
+
+/* Device workspace bytes needed by sls_lanczos_topr_batched. */
+size_t sls_lanczos_batched_workspace_size(int64_t rows, int64_t nmax, int D, int r,
+                                          int nprob);
+
+/*
+ * sls_lanczos_topr for nprob independent problems in one launch, with the
+ * launch plan sls_compress uses for the windows of its adaptive and local
+ * backends (Algorithm 2 per window, Sec. 3.5-3.6): the persistent kernel's
+ * CTAs form groups and each group runs one problem at a time, each CTA of a
+ * group a strip of the problem's rows; problems of at most 32 rows (r <= 32)
+ * run one warp per problem instead.
+ *   Phi: rows x D of phi_dtype (SLS_F32 or SLS_BF16, as sls_lanczos_topr_ex).
+ *   row0, n, q1off: device arrays of nprob entries; problem p owns the rows
+ *   [row0[p], row0[p] + n[p]) of Phi and of U, with 1 <= n[p] <= nmax and
+ *   row0[p] + n[p] <= rows, and its start vector is q1[q1off[p] ..
+ *   q1off[p] + n[p]) (q1off may be NULL: q1off = row0), normalised by the
+ *   callee.
+ *   Outputs: theta: nprob x r doubles (problem p at p * r, descending);
+ *   U: rows x r floats (problem p's Ritz vectors in its rows); r_eff: nprob
+ *   int32, -1 until the kernel finishes and left at -1 if a device-side wait
+ *   gave up; alpha, beta (may be NULL): nprob x r doubles.
+ * The problem table is read on the device only, so the host needs no copy of
+ * it; nmax is a host upper bound on n[p] that sizes the plan.  Errors:
+ * INVALID_ARG (sizes, NULL, misaligned Phi), UNSUPPORTED, WORKSPACE, CUDA.
+ */
+int sls_lanczos_topr_batched(const void* Phi, int phi_dtype, int D, int r, int nprob,
+                             const int64_t* row0, const int32_t* n, const int64_t* q1off,
+                             int64_t nmax, int64_t rows, const double* q1, double tol,
+                             double* theta, float* U, int32_t* r_eff, double* alpha,
+                             double* beta, void* workspace, size_t workspace_bytes,
+                             void* stream);
 
 /*
  * SimHash in the spectral subspace, Sec. 3.3 Eq. simhash:
@@ -283,7 +318,8 @@ size_t sls_compress_workspace_size(const sls_config_t* cfg, int64_t B,
  *   with M = sls_output_count(cfg, N).
  *   r_eff (may be NULL): device int32 per prompt (global backend) or per
  *   window (adaptive and local backends), the Lanczos steps kept (0 for chunk
- *   windows).
+ *   windows; -1 for a spectral problem whose Lanczos kernel gave up a
+ *   device-side wait, see sls_workspace_status).
  *   route (may be NULL): device int32 per window, 1 = spectral, 0 = chunk
  *   (adaptive backend; all 1 for the local backend).
  * The windowed backends (adaptive, local) cut the compressible region into
@@ -358,9 +394,14 @@ int sls_compress_tokens(const sls_config_t* cfg, const void* table, int x_dtype,
  * previous call's contents (what must start at zero is cleared by each
  * call), so calls that overlap on the GPU -- on different streams, or from
  * different host threads -- race and must be serialised by the caller.
- * *r_eff is set to -1 when the call is enqueued and stays -1 if a device-side
- * wait gave up.  Errors: those of sls_lanczos_topr, and SLS_ERR_WORKSPACE
- * when sls_lanczos_workspace_size(N, D, r) exceeds SLS_NOALLOC_MAX_BYTES.
+ * The looked-up address is cached for the life of the process: after a
+ * cudaDeviceReset() on a device (which destroys the array with the context)
+ * this entry point must not be called on that device again in the same
+ * process.  *r_eff is set to -1 when the call is enqueued and stays -1 if a
+ * device-side wait gave up.  Errors: those of sls_lanczos_topr (arguments are
+ * checked before anything is enqueued), and SLS_ERR_WORKSPACE, with nothing
+ * enqueued, when sls_lanczos_workspace_size(N, D, r) exceeds
+ * SLS_NOALLOC_MAX_BYTES.
  */
 #define SLS_NOALLOC_MAX_BYTES (32u << 20)
 int sls_lanczos_topr_noalloc(const float* Phi, int64_t N, int D, int r,
@@ -399,6 +440,22 @@ int64_t sls_launch_count(void);
  */
 int sls_selftest_wait_limit(int which, void* workspace, size_t workspace_bytes,
                             void* stream);
+
+/*
+ * Self-test of the Lanczos kernel's failure path (the paper has no
+ * counterpart): sls_lanczos_topr (float32 Phi, tol = 1e-10, same arguments
+ * and workspace) with its first CTA reporting, at its first barrier, a wait
+ * that gave up.  The kernel then takes the path of a real give-up: the other
+ * CTAs are released at once, the copy warps stop after their own bounded
+ * wait (about a second), the status word reads SLS_ERR_TIMEOUT, *r_eff stays
+ * -1, theta and U are zero, and the context stays usable.  No fault, trap or
+ * hang is involved.  Errors: those of sls_lanczos_topr; UNSUPPORTED when the
+ * problem runs on the one-warp small-window kernel (N <= 32), which has no
+ * barrier to fail.
+ */
+int sls_selftest_lanczos_giveup(const float* Phi, int64_t N, int D, int r, const double* q1,
+                                double* theta, float* U, int32_t* r_eff, void* workspace,
+                                size_t workspace_bytes, void* stream);
 
 /*
  * Reads (synchronously, on `stream`) the device status word of a workspace

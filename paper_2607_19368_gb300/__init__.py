@@ -27,6 +27,7 @@ __all__ = [
     "compress_workspace_size", "workspace_status", "EXPORTED", "PHASES",
     "set_phase_events", "launch_count", "Workspace", "embed_gather", "compress_tokens",
     "compress_tokens_workspace_size", "TokensWorkspace", "selftest_wait_limit",
+    "lanczos_topr_batched", "selftest_lanczos_giveup",
 ]
 
 SLS_OK = 0
@@ -117,6 +118,11 @@ EXPORTED = {
                                    _vp, _vp, _sz, _vp]),
     "sls_lanczos_topr_noalloc": (_i32, [_vp, _i64, _i32, _i32, _vp, _d, _vp, _vp, _vp, _vp,
                                         _vp, _vp]),
+    "sls_lanczos_batched_workspace_size": (_sz, [_i64, _i64, _i32, _i32, _i32]),
+    "sls_lanczos_topr_batched": (_i32, [_vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _i64, _i64,
+                                        _vp, _d, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "sls_selftest_lanczos_giveup": (_i32, [_vp, _i64, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _sz,
+                                           _vp]),
     "sls_set_phase_events": (_i32, [ctypes.POINTER(ctypes.c_void_p), _i32]),
     "sls_launch_count": (_i64, []),
 }
@@ -262,6 +268,66 @@ def lanczos_topr(Phi: torch.Tensor, q1: torch.Tensor, r: int, tol: float = 1e-10
                                _ptr(ws), ws.numel(), _stream(Phi))
     _check("sls_lanczos_topr_ex", st)
     return theta, U, r_eff, alpha, beta
+
+
+def lanczos_topr_batched(Phi: torch.Tensor, q1: torch.Tensor, r: int, row0, n, q1off=None,
+                         tol: float = 1e-10):
+    """Algorithm 2 and the Ritz pairs for several independent problems in one
+    launch, with the plan the windowed backends use (Sec. 3.5-3.6): problem p
+    owns rows row0[p] .. row0[p] + n[p] of Phi (float32 or bfloat16, rows x D)
+    and starts from q1[q1off[p]:] (q1off defaults to row0).  Returns (theta
+    [nprob, r] float64, U [rows, r] float32, r_eff [nprob] int32, alpha, beta)
+    as device tensors."""
+    _need_cuda(Phi, q1)
+    Phi = Phi.contiguous()
+    rows, D = Phi.shape
+    dev = Phi.device
+    row0_t = torch.as_tensor(row0, dtype=torch.int64).to(dev).contiguous()
+    n_t = torch.as_tensor(n, dtype=torch.int32).to(dev).contiguous()
+    nprob = int(n_t.numel())
+    q1off_t = (torch.as_tensor(q1off, dtype=torch.int64).to(dev).contiguous()
+               if q1off is not None else None)
+    nmax = int(torch.as_tensor(n).max().item())
+    q1 = q1.to(device=dev, dtype=torch.float64).contiguous()
+    theta = torch.empty((nprob, r), dtype=torch.float64, device=dev)
+    U = torch.zeros((rows, r), dtype=torch.float32, device=dev)
+    r_eff = torch.empty(nprob, dtype=torch.int32, device=dev)
+    alpha = torch.empty((nprob, r), dtype=torch.float64, device=dev)
+    beta = torch.empty((nprob, r), dtype=torch.float64, device=dev)
+    L = lib()
+    nbytes = L.sls_lanczos_batched_workspace_size(rows, nmax, D, r, nprob)
+    if nbytes == 0:
+        raise SLSError("sls_lanczos_batched_workspace_size", 2, "unsupported shape")
+    ws = _workspace(nbytes, dev)
+    st = L.sls_lanczos_topr_batched(_ptr(Phi), _dtype_code(Phi), D, r, nprob, _ptr(row0_t),
+                                    _ptr(n_t), _ptr(q1off_t), nmax, rows, _ptr(q1), float(tol),
+                                    _ptr(theta), _ptr(U), _ptr(r_eff), _ptr(alpha),
+                                    _ptr(beta), _ptr(ws), ws.numel(), _stream(Phi))
+    _check("sls_lanczos_topr_batched", st)
+    return theta, U, r_eff, alpha, beta
+
+
+def selftest_lanczos_giveup(Phi: torch.Tensor, q1: torch.Tensor, r: int):
+    """The Lanczos kernel's failure path on a real problem (see
+    sls_selftest_lanczos_giveup): returns (status word, theta, U, r_eff); the
+    status is SLS_ERR_TIMEOUT = 5 and r_eff -1 when the kernel gave up as
+    designed.  Takes about one second."""
+    _need_cuda(Phi, q1)
+    Phi = Phi.contiguous()
+    N, D = Phi.shape
+    dev = Phi.device
+    q1 = q1.to(device=dev, dtype=torch.float64).contiguous()
+    theta = torch.full((r,), 7.0, dtype=torch.float64, device=dev)
+    U = torch.full((N, r), 7.0, dtype=torch.float32, device=dev)
+    r_eff = torch.full((1,), 7, dtype=torch.int32, device=dev)
+    L = lib()
+    nbytes = L.sls_lanczos_workspace_size(N, D, r)
+    ws = _workspace(nbytes, dev)
+    st = L.sls_selftest_lanczos_giveup(_ptr(Phi), N, D, r, _ptr(q1), _ptr(theta), _ptr(U),
+                                       _ptr(r_eff), _ptr(ws), ws.numel(), _stream(Phi))
+    _check("sls_selftest_lanczos_giveup", st)
+    status = int(L.sls_workspace_status(_ptr(ws), _stream(ws)))
+    return status, theta, U, r_eff
 
 
 def simhash(U: torch.Tensor, R: torch.Tensor, bits: int, k: Optional[int] = None,

@@ -172,7 +172,8 @@ route_compact_kernel(ProbDesc* __restrict__ probs, int nprob, int mode,
                      const float* __restrict__ score, double rho, double tau,
                      int* __restrict__ spec_list, int64_t* __restrict__ lz_row0,
                      int* __restrict__ lz_n, int64_t* __restrict__ lz_q1off,
-                     int* __restrict__ nspec, int32_t* __restrict__ route_out) {
+                     int* __restrict__ nspec, int32_t* __restrict__ route_out,
+                     int* __restrict__ lz_reff) {
   __shared__ int sh[33];
   const int tid = threadIdx.x;
   const int chunk = (nprob + 1023) / 1024;
@@ -217,6 +218,9 @@ route_compact_kernel(ProbDesc* __restrict__ probs, int nprob, int mode,
       lz_row0[off] = probs[p].phi_row;
       lz_n[off] = probs[p].n;
       lz_q1off[off] = probs[p].q1off;
+      // -1 until the Lanczos kernel finishes; stays -1 if one of its waits
+      // gave up, and the eigen and Ritz kernels then treat the problem as empty
+      lz_reff[off] = -1;
       ++off;
     }
   }
@@ -430,6 +434,66 @@ size_t part_bytes(int64_t toks, int d) {
          sls_align256(agg_part_capacity(toks) * sizeof(float));
 }
 
+// One Lanczos problem (sls_lanczos_topr_ex); inject_fail = 1 runs the
+// failure self-test (the kernel's give-up path, see LanczosBatch).
+int lanczos_single(const void* Phi, int phi_dtype, int64_t N, int D, int r, const double* q1,
+                   double tol, double* theta, float* U, int32_t* r_eff, double* alpha,
+                   double* beta, void* workspace, size_t workspace_bytes, void* stream,
+                   int inject_fail) {
+  if (N < 1 || D < 4 || D > SLS_MAX_D || r < 1 || r > SLS_MAX_R || !(tol >= 0.0))
+    return SLS_ERR_INVALID_ARG;
+  if (phi_dtype != SLS_F32 && phi_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
+  if ((D & 3) != 0 || (phi_dtype == SLS_BF16 && (D & 7) != 0)) return SLS_ERR_UNSUPPORTED;
+  if (!ptr_ok(Phi) || !q1 || !theta || !U || !r_eff) return SLS_ERR_INVALID_ARG;
+  const size_t need = sls_lanczos_workspace_size(N, D, r);
+  if (need == 0) return SLS_ERR_UNSUPPORTED;
+  if (!workspace || workspace_bytes < need) return SLS_ERR_WORKSPACE;
+  int groups = 0, g = 0;
+  int st = lanczos_plan(N, D, r, 1, &groups, &g);
+  if (st != SLS_OK) return st;
+  cudaStream_t s = (cudaStream_t)stream;
+  Carver cv(workspace);
+  int* status = cv.take<int>(64);
+  float2* Q = cv.take<float2>((size_t)N * ((r + 1) & ~1));
+  double* al = cv.take<double>(r);
+  double* be = cv.take<double>(r);
+  double* S = cv.take<double>((size_t)r * r);
+  const size_t lzb = lanczos_scratch_bytes(N, D, r, groups, g);
+  void* lz = cv.take<char>(lzb);
+  SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
+  // -1 until the Lanczos kernel finishes; stays -1 if one of its waits gave
+  // up, and the eigen and Ritz kernels then treat the problem as empty
+  SLS_CUDA_TRY(cudaMemsetAsync(r_eff, 0xff, sizeof(int32_t), s));
+  LanczosBatch bt{};
+  bt.Phi = Phi;
+  bt.phi_bf16 = (phi_dtype == SLS_BF16) ? 1 : 0;
+  bt.D = D;
+  bt.r = r;
+  bt.tol = tol;
+  bt.q1 = q1;
+  bt.n_single = N;
+  bt.nprob_max = 1;
+  bt.Q = Q;
+  bt.alpha = al;
+  bt.beta = be;
+  bt.theta = theta;
+  bt.S = S;
+  bt.r_eff = r_eff;
+  bt.nmax = N;
+  bt.inject_fail = inject_fail;
+  const bool small = lanczos_window_fits(N, D, r);
+  if (small) {
+    if ((st = launch_lanczos_window(bt, s)) != SLS_OK) return st;
+  } else if ((st = launch_lanczos(bt, lz, lzb, status, groups, g, s)) != SLS_OK) {
+    return st;
+  }
+  if ((st = launch_tridiag_eigen(bt, s, small)) != SLS_OK) return st;
+  if ((st = launch_ritz_vectors(bt, U, s)) != SLS_OK) return st;
+  if (alpha) SLS_CUDA_TRY(cudaMemcpyAsync(alpha, al, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
+  if (beta) SLS_CUDA_TRY(cudaMemcpyAsync(beta, be, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
+  return SLS_OK;
+}
+
 }  // namespace
 
 // ===========================================================================
@@ -535,27 +599,61 @@ int sls_lanczos_topr(const float* Phi, int64_t N, int D, int r, const double* q1
 int sls_lanczos_topr_ex(const void* Phi, int phi_dtype, int64_t N, int D, int r, const double* q1,
                         double tol, double* theta, float* U, int32_t* r_eff, double* alpha,
                         double* beta, void* workspace, size_t workspace_bytes, void* stream) {
-  if (N < 1 || D < 4 || D > SLS_MAX_D || r < 1 || r > SLS_MAX_R || !(tol >= 0.0))
+  return lanczos_single(Phi, phi_dtype, N, D, r, q1, tol, theta, U, r_eff, alpha, beta, workspace,
+                        workspace_bytes, stream, 0);
+}
+
+int sls_selftest_lanczos_giveup(const float* Phi, int64_t N, int D, int r, const double* q1,
+                                double* theta, float* U, int32_t* r_eff, void* workspace,
+                                size_t workspace_bytes, void* stream) {
+  if (lanczos_window_fits(N, D, r)) return SLS_ERR_UNSUPPORTED;  // no group barrier there
+  return lanczos_single(Phi, SLS_F32, N, D, r, q1, 1e-10, theta, U, r_eff, nullptr, nullptr,
+                        workspace, workspace_bytes, stream, 1);
+}
+
+size_t sls_lanczos_batched_workspace_size(int64_t rows, int64_t nmax, int D, int r, int nprob) {
+  if (rows < 1 || nmax < 1 || D < 4 || r < 1 || r > SLS_MAX_R || nprob < 1) return 0;
+  int groups = 0, g = 0;
+  if (lanczos_plan(nmax, D, r, nprob, &groups, &g) != SLS_OK) return 0;
+  Carver cv(nullptr);
+  cv.take<int>(64);
+  cv.take<float2>((size_t)rows * ((r + 1) & ~1));
+  cv.take<double>((size_t)nprob * r);
+  cv.take<double>((size_t)nprob * r);
+  cv.take<double>((size_t)nprob * r * r);
+  cv.take<char>(lanczos_scratch_bytes(nmax, D, r, groups, g));
+  return cv.off;
+}
+
+int sls_lanczos_topr_batched(const void* Phi, int phi_dtype, int D, int r, int nprob,
+                             const int64_t* row0, const int32_t* n, const int64_t* q1off,
+                             int64_t nmax, int64_t rows, const double* q1, double tol,
+                             double* theta, float* U, int32_t* r_eff, double* alpha,
+                             double* beta, void* workspace, size_t workspace_bytes,
+                             void* stream) {
+  if (nprob < 1 || nmax < 1 || rows < 1 || D < 4 || D > SLS_MAX_D || r < 1 || r > SLS_MAX_R ||
+      !(tol >= 0.0))
     return SLS_ERR_INVALID_ARG;
   if (phi_dtype != SLS_F32 && phi_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
   if ((D & 3) != 0 || (phi_dtype == SLS_BF16 && (D & 7) != 0)) return SLS_ERR_UNSUPPORTED;
-  if (!ptr_ok(Phi) || !q1 || !theta || !U || !r_eff) return SLS_ERR_INVALID_ARG;
-  const size_t need = sls_lanczos_workspace_size(N, D, r);
+  if (!ptr_ok(Phi) || !row0 || !n || !q1 || !theta || !U || !r_eff) return SLS_ERR_INVALID_ARG;
+  const size_t need = sls_lanczos_batched_workspace_size(rows, nmax, D, r, nprob);
   if (need == 0) return SLS_ERR_UNSUPPORTED;
   if (!workspace || workspace_bytes < need) return SLS_ERR_WORKSPACE;
   int groups = 0, g = 0;
-  int st = lanczos_plan(N, D, r, 1, &groups, &g);
+  int st = lanczos_plan(nmax, D, r, nprob, &groups, &g);
   if (st != SLS_OK) return st;
   cudaStream_t s = (cudaStream_t)stream;
   Carver cv(workspace);
   int* status = cv.take<int>(64);
-  float2* Q = cv.take<float2>((size_t)N * ((r + 1) & ~1));
-  double* al = cv.take<double>(r);
-  double* be = cv.take<double>(r);
-  double* S = cv.take<double>((size_t)r * r);
-  const size_t lzb = lanczos_scratch_bytes(N, D, r, groups, g);
+  float2* Q = cv.take<float2>((size_t)rows * ((r + 1) & ~1));
+  double* al = cv.take<double>((size_t)nprob * r);
+  double* be = cv.take<double>((size_t)nprob * r);
+  double* S = cv.take<double>((size_t)nprob * r * r);
+  const size_t lzb = lanczos_scratch_bytes(nmax, D, r, groups, g);
   void* lz = cv.take<char>(lzb);
   SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
+  SLS_CUDA_TRY(cudaMemsetAsync(r_eff, 0xff, sizeof(int32_t) * (size_t)nprob, s));
   LanczosBatch bt{};
   bt.Phi = Phi;
   bt.phi_bf16 = (phi_dtype == SLS_BF16) ? 1 : 0;
@@ -563,16 +661,20 @@ int sls_lanczos_topr_ex(const void* Phi, int phi_dtype, int64_t N, int D, int r,
   bt.r = r;
   bt.tol = tol;
   bt.q1 = q1;
-  bt.n_single = N;
-  bt.nprob_max = 1;
+  bt.n_single = 0;
+  bt.nprob_max = nprob;
+  bt.nprob_dev = nullptr;
+  bt.row0 = row0;
+  bt.n = n;
+  bt.q1off = q1off;
   bt.Q = Q;
   bt.alpha = al;
   bt.beta = be;
   bt.theta = theta;
   bt.S = S;
   bt.r_eff = r_eff;
-  bt.nmax = N;
-  const bool small = lanczos_window_fits(N, D, r);
+  bt.nmax = nmax;
+  const bool small = lanczos_window_fits(nmax, D, r);
   if (small) {
     if ((st = launch_lanczos_window(bt, s)) != SLS_OK) return st;
   } else if ((st = launch_lanczos(bt, lz, lzb, status, groups, g, s)) != SLS_OK) {
@@ -580,8 +682,12 @@ int sls_lanczos_topr_ex(const void* Phi, int phi_dtype, int64_t N, int D, int r,
   }
   if ((st = launch_tridiag_eigen(bt, s, small)) != SLS_OK) return st;
   if ((st = launch_ritz_vectors(bt, U, s)) != SLS_OK) return st;
-  if (alpha) SLS_CUDA_TRY(cudaMemcpyAsync(alpha, al, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
-  if (beta) SLS_CUDA_TRY(cudaMemcpyAsync(beta, be, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
+  if (alpha)
+    SLS_CUDA_TRY(cudaMemcpyAsync(alpha, al, sizeof(double) * r * (size_t)nprob,
+                                 cudaMemcpyDeviceToDevice, s));
+  if (beta)
+    SLS_CUDA_TRY(cudaMemcpyAsync(beta, be, sizeof(double) * r * (size_t)nprob,
+                                 cudaMemcpyDeviceToDevice, s));
   return SLS_OK;
 }
 
@@ -732,7 +838,7 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   int32_t* rflags = route ? route : W.route;
   route_compact_kernel<<<1, 1024, 0, s>>>(W.probs, nprob, mode, W.score, cfg->rho, tau,
                                           W.spec_list, W.lz_row0, W.lz_n, W.lz_q1off, W.nspec,
-                                          rflags);
+                                          rflags, W.r_eff);
   SLS_LAUNCH_CHECK();
   phase_mark(0, 1, s);
   phase_mark(1, 0, s);

@@ -80,6 +80,10 @@ struct LanczosBatch {
   int* r_eff;
   int64_t nmax;             // max rows of any problem
   int phi_bf16;             // Phi stored as bfloat16 (D % 8 == 0)
+  // self-test of the failure path (0 in every ordinary call): the first CTA
+  // reports a failed wait at its first group barrier, as a wait that gave up
+  // would, so the kernel's give-up and clean-exit path runs without a fault
+  int inject_fail;
 };
 
 size_t lanczos_scratch_bytes(int64_t nmax, int D, int r, int groups, int ctas_per_group);

@@ -15,6 +15,13 @@ namespace sls {
 
 namespace {
 
+// Lanczos steps kept for problem p, clamped to [0, r]: r_eff is set to -1
+// before the Lanczos launch and keeps that value if a device-side wait of the
+// kernel gave up, so the later kernels then treat the problem as empty.
+SLS_DEV int reff_clamped(const LanczosBatch& bt, int p) {
+  return min(bt.r, max(0, bt.r_eff[p]));
+}
+
 // ----------------------------------------------------------------------------
 // Eigenvalues of T: multisection on Sturm counts.  The arithmetic of the
 // recurrences is double-float on the FP32 pipes: float64 on this part has a
@@ -37,7 +44,7 @@ tridiag_eigvals_cta_kernel(LanczosBatch bt) {
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
   if (p >= nprob) return;
   const int r = bt.r;
-  const int n = bt.r_eff[p];
+  const int n = reff_clamped(bt, p);
   double* theta = bt.theta + (size_t)p * r;
   if (m >= n) {
     if (tid == 0) theta[m] = 0.0;
@@ -120,7 +127,7 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
   if (p >= nprob) return;
   const int r = bt.r;
-  const int n = bt.r_eff[p];
+  const int n = reff_clamped(bt, p);
   const int m = blockIdx.x * EIG_WARPS + warp;  // descending index of this warp's value
   double* theta = bt.theta + (size_t)p * r;
   const double* a = bt.alpha + (size_t)p * r;
@@ -332,7 +339,7 @@ tridiag_eigvecs_kernel(LanczosBatch bt) {
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
   if (p >= nprob) return;
   const int r = bt.r;
-  const int n = bt.r_eff[p];
+  const int n = reff_clamped(bt, p);
   double* S = bt.S + (size_t)p * r * r;
   if (m >= n) {
     for (int k = lane; k < r; k += 32) S[(size_t)k * r + m] = 0.0;
@@ -361,7 +368,7 @@ tridiag_eigvecs_warp_kernel(LanczosBatch bt) {
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
   if (p >= nprob) return;
   const int r = bt.r;
-  const int n = bt.r_eff[p];
+  const int n = reff_clamped(bt, p);
   double* S = bt.S + (size_t)p * r * r;
   // S rows and columns beyond r_eff are zero
   for (int e = lane; e < r * r; e += 32) {
@@ -397,7 +404,7 @@ ritz_vectors_kernel(LanczosBatch bt, float* __restrict__ U) {
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
   if (p >= nprob) return;
   const int r = bt.r, ldq = q_ld(r);
-  const int kn = bt.r_eff[p];
+  const int kn = reff_clamped(bt, p);
   const int64_t row0 = bt.row0 ? bt.row0[p] : 0;
   const int64_t n = bt.n ? (int64_t)bt.n[p] : bt.n_single;
   const int cg = (r + 3) / 4, rg = RITZ_THREADS / cg, TR = rg * 4, qs = r + 1;

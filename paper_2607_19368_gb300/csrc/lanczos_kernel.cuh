@@ -905,6 +905,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       }
     }
 
+    if (bt.inject_fail && rank == 0 && tid == 0) lz_fail(status, &s_err);
     for (int j = 0; j < r; ++j) {
       if (!group_sync_named(bar, lgen, status, &sflag, &s_err, BAR_COMPUTE, LZ_CT)) return;
 

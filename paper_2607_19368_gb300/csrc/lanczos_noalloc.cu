@@ -17,6 +17,9 @@ void* g_scratch_addr[kMaxDevices] = {};
 
 // Device address of g_noalloc_scratch on the current device.  In host code
 // the array's name is only a stand-in for the symbol, never a device pointer.
+// The address is looked up once per device and cached for the process; a
+// cudaDeviceReset() destroys the context that holds the array, after which
+// the cached address is stale (the header says so).
 int scratch_address(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return SLS_ERR_CUDA;
@@ -40,15 +43,15 @@ extern "C" int sls_lanczos_topr_noalloc(const float* Phi, int64_t N, int D, int 
   if (N < 1 || D < 4 || D > SLS_MAX_D || r < 1 || r > SLS_MAX_R || !(tol >= 0.0))
     return SLS_ERR_INVALID_ARG;
   if ((D & 3) != 0) return SLS_ERR_UNSUPPORTED;
-  if (!Phi || !q1 || !theta || !U || !r_eff) return SLS_ERR_INVALID_ARG;
+  // the same pointer checks as sls_lanczos_topr, before anything is enqueued
+  if (Phi == nullptr || ((uintptr_t)Phi & 15u) != 0 || !q1 || !theta || !U || !r_eff)
+    return SLS_ERR_INVALID_ARG;
   const size_t need = sls_lanczos_workspace_size(N, D, r);
   if (need == 0) return SLS_ERR_UNSUPPORTED;
   if (need > (size_t)SLS_NOALLOC_MAX_BYTES) return SLS_ERR_WORKSPACE;
   void* ws = nullptr;
   const int st = scratch_address(&ws);
   if (st != SLS_OK) return st;
-  // -1 until the Lanczos kernel finishes; stays -1 if one of its waits gave up
-  SLS_CUDA_TRY(cudaMemsetAsync(r_eff, 0xff, sizeof(int32_t), (cudaStream_t)stream));
   return sls_lanczos_topr(Phi, N, D, r, q1, tol, theta, U, r_eff, alpha, beta, ws,
                           (size_t)SLS_NOALLOC_MAX_BYTES, stream);
 }

@@ -47,3 +47,54 @@ def oracle_phi32(X64, W64, b):
 
 def pinned(t):
     return t.pin_memory() if torch.cuda.is_available() else t
+
+
+def adjusted_rand_index(a, b):
+    """Adjusted Rand index of two labelings of the same items (Hubert and
+    Arabie, 1985): the pair-counting agreement of the two partitions,
+    corrected for chance; 1 for identical partitions."""
+    a = np.asarray(a, np.int64)
+    b = np.asarray(b, np.int64)
+    n = a.size
+    _, ia = np.unique(a, return_inverse=True)
+    _, ib = np.unique(b, return_inverse=True)
+    pair = ia * (int(ib.max()) + 1) + ib
+    _, nij = np.unique(pair, return_counts=True)
+    comb = lambda x: x.astype(np.float64) * (x - 1) / 2.0
+    s_ij = comb(nij).sum()
+    s_a = comb(np.bincount(ia)).sum()
+    s_b = comb(np.bincount(ib)).sum()
+    tot = n * (n - 1) / 2.0
+    expected = s_a * s_b / tot if tot > 0 else 0.0
+    top = 0.5 * (s_a + s_b)
+    if top == expected:
+        return 1.0
+    return float((s_ij - expected) / (top - expected))
+
+
+def code_agreement(sls, w, p, prm, X, Wt, bt, Rt, qt):
+    """End-to-end agreement of the GPU pass with the oracle's
+    compress_global on one prompt (reported, not pinned: float32 against
+    float64 Ritz vectors flip near-zero SimHash dots): the fraction of
+    identical codes (GPU codes from the same feature, Lanczos and SimHash
+    kernels sls_compress runs) and the adjusted Rand index of the two token
+    maps.  Returns a dict."""
+    Nc = w.N - w.preserve_first - w.preserve_last
+    cfg_o = O.CompressConfig(rho=w.rho, D=w.D, r=w.r, bits=w.bits,
+                             preserve_first=w.preserve_first, preserve_last=w.preserve_last)
+    res = O.compress_global(p.x_f64(), prm.w_f64(), prm.b, prm.R, prm.q1, cfg_o)
+    codes_o = res.info["codes"]
+    bits = res.info["bits"]
+    Xc = X[w.preserve_first:w.preserve_first + Nc]
+    phi = sls.feature_map(Xc, Wt, bt)
+    _, U, r_eff, _, _ = sls.lanczos_topr(phi, qt[:Nc], w.r)
+    codes_g = sls.simhash(U, Rt, bits, k_dev=r_eff).cpu().numpy().view(np.uint32)
+    cfg = sls.Config.make(backend=sls.BACKEND_GLOBAL, rho=w.rho, D=w.D, r=w.r, bits=w.bits,
+                          preserve_first=w.preserve_first, preserve_last=w.preserve_last)
+    _, _, t2m, _, _ = sls.compress(X.view(1, w.N, w.d), cfg, Wt, bt, Rt, qt)
+    t2m = t2m[0].cpu().numpy()
+    return {"workload": w.name, "tokens": Nc,
+            "codes_identical": float(np.mean(codes_g == codes_o)),
+            "ari_tok2macro": adjusted_rand_index(t2m, res.tok2macro),
+            "clusters_gpu": int(np.unique(codes_g).size),
+            "clusters_oracle": int(res.info["n_clusters"])}

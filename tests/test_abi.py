@@ -58,6 +58,19 @@ def test_host_side_errors_and_counts(lib):
     assert lib.sls_lanczos_topr(None, 4, 8, 0, None, 1e-10, None, None, None, None, None,
                                 None, 0, None) == 1                               # r = 0
     assert lib.sls_lanczos_workspace_size(1000, 256, 16) > 0
+    # batched Lanczos: no problems; a NULL problem table
+    assert lib.sls_lanczos_topr_batched(None, 0, 256, 16, 0, None, None, None, 100, 100, None,
+                                        1e-10, None, None, None, None, None, None, 0, None) == 1
+    assert lib.sls_lanczos_topr_batched(ctypes.c_void_p(256), 0, 256, 16, 2, None, None, None,
+                                        100, 200, ctypes.c_void_p(256), 1e-10,
+                                        ctypes.c_void_p(256), ctypes.c_void_p(256), None, None,
+                                        None, None, 0, None) == 1
+    assert lib.sls_lanczos_batched_workspace_size(200, 100, 256, 16, 2) > 0
+    # the give-up self-test has no barrier to fail in the one-warp window kernel
+    assert lib.sls_selftest_lanczos_giveup(ctypes.c_void_p(256), 20, 256, 16,
+                                           ctypes.c_void_p(256), ctypes.c_void_p(256),
+                                           ctypes.c_void_p(256), ctypes.c_void_p(256), None,
+                                           0, None) == 2
     # embedding lookup: table stride below d, unknown dtype, missing ids
     assert lib.sls_embed_gather(None, 1, 10, 8, 4, None, 4, None, 8, None, None) == 1
     assert lib.sls_embed_gather(None, 7, 10, 8, 8, None, 4, None, 8, None, None) == 1

@@ -40,3 +40,35 @@ def test_stuck_wait_ends_with_timeout_status(sls, which):
     want = O.rff_features(p.x_f64(), prm.w_f64(), prm.b)
     assert np.all(np.abs(got - want) <= feature_tolerance(p.x_f64(), prm.w_f64(),
                                                           prm.b.astype(np.float64)))
+
+
+def test_lanczos_giveup_leaves_empty_result_and_usable_context(sls):
+    """The persistent Lanczos kernel's own give-up path: one CTA reports a
+    failed wait at its first group barrier (as a wait that ran out would), so
+    the group is released, the copy warps stop after their bounded wait, the
+    status reads SLS_ERR_TIMEOUT, r_eff stays -1 and the later kernels treat
+    the problem as empty (theta and U zero) instead of reading stale values.
+    The same problem then runs normally and matches the oracle."""
+    g = np.random.default_rng(5)
+    N, D, r = 3000, 512, 24
+    X = g.standard_normal((N, 24)) / np.sqrt(24)
+    W = g.standard_normal((D, 24)) * 24 ** -0.25
+    b = g.random(D) * 2 * np.pi
+    phi32 = O.rff_features(X, W, b).astype(np.float32)
+    q1 = g.standard_normal(N)
+    Phi, Q1 = torch.from_numpy(phi32).cuda(), torch.from_numpy(q1).cuda()
+    t0 = time.time()
+    status, theta, U, r_eff = sls.selftest_lanczos_giveup(Phi, Q1, r)
+    torch.cuda.synchronize()
+    assert time.time() - t0 < 30.0
+    assert status == 5, status
+    assert int(r_eff.item()) == -1
+    assert float(theta.abs().max().item()) == 0.0
+    assert float(U.abs().max().item()) == 0.0
+    # the context still works, and a normal call gives the oracle's result
+    th, U2, k, _, _ = sls.lanczos_topr(Phi, Q1, r)
+    a, be, Q, ko = O.lanczos(phi32.astype(np.float64), q1, r)
+    th_o, _, U_o = O.ritz_pairs(a, be, Q)
+    assert int(k.item()) == ko
+    t = th.cpu().numpy()[:ko]
+    assert np.all(np.abs(t - th_o) <= 1e-4 * np.abs(th_o) + 1e-12 * abs(th_o[0]))

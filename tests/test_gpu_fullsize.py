@@ -181,14 +181,60 @@ def test_qwen7b_compress_full_size(sls):
 
 
 def test_qwen14b_compress_full_size(sls):
-    d = _compress_case(sls, "qwen14b", 128)
-    # the feature map at this shape, on sampled rows
-    rng = np.random.default_rng(73)
-    rows = np.sort(rng.choice(d["Nc"], size=128, replace=False))
-    Xr = d["X"][torch.from_numpy(rows).cuda()]
-    got = sls.feature_map(Xr, d["W"], d["b"]).cpu().numpy().astype(np.float64)
-    X64 = _rows64(d["p"], rows)
-    W64, b = d["prm"].w_f64(), d["prm"].b
+    _compress_case(sls, "qwen14b", 128)
+
+
+@pytest.fixture(scope="module")
+def q14(sls):
+    """The qwen14b-shaped prompt and the GPU feature matrix of its 131060
+    compressible rows from the launch sls_compress makes (one batched
+    tensor-core launch over all row tiles)."""
+    d = _inputs("qwen14b")
+    w, Nc = d["w"], d["Nc"]
+    d["phi"] = sls.feature_map_batched(d["X"].view(1, w.N, w.d), d["W"], d["b"], Nc)
+    return d
+
+
+def test_qwen14b_features_full_launch_sampled_rows(sls, q14):
+    rng = np.random.default_rng(74)
+    rows = np.sort(rng.choice(q14["Nc"], size=256, replace=False))
+    got = q14["phi"][torch.from_numpy(rows).cuda()].cpu().numpy().astype(np.float64)
+    X64 = _rows64(q14["p"], rows)
+    W64, b = q14["prm"].w_f64(), q14["prm"].b
     want = O.rff_features(X64, W64, b)
     tol = feature_tolerance(X64, W64, b.astype(np.float64))
-    assert np.all(np.abs(got - want) <= tol)
+    assert np.all(np.abs(got - want) <= tol), float(np.max(np.abs(got - want) / tol))
+
+
+def test_qwen14b_lanczos_full_size(sls, q14):
+    """Algorithm 2 at the qwen14b shape (N = 131060, D = 2048, r = 64) on the
+    GPU's own feature matrix against the oracle: Ritz values, the Ritz
+    subspace, orthonormality of the GPU's Ritz vectors and their residuals
+    |A u - theta u| against the oracle's (the persistent kernel applies one
+    classical Gram-Schmidt pass per step, the oracle two)."""
+    w, Nc = q14["w"], q14["Nc"]
+    theta, U, r_eff, _, _ = sls.lanczos_topr(q14["phi"], q14["q1"][:Nc], w.r)
+    torch.cuda.synchronize()
+    phi64 = q14["phi"].cpu().numpy().astype(np.float64)
+    q1 = q14["prm"].q1[:Nc]
+    a, be, Q, k = O.lanczos(phi64, q1, w.r)
+    th_o, _, U_o = O.ritz_pairs(a, be, Q)
+    assert int(r_eff.item()) == k == w.r
+    th = theta.cpu().numpy()[:k]
+    floor = ZERO_FLOOR * abs(th_o[0])
+    err = np.abs(th - th_o)
+    assert np.all(err <= RITZ_RTOL * np.abs(th_o) + floor), float(np.max(err / np.abs(th_o)))
+    Ug = U.cpu().numpy()[:, :k].astype(np.float64)
+    ang = max_subspace_angle(Ug, U_o)
+    assert ang <= ANGLE_TOL, ang
+    orth = float(np.max(np.abs(Ug.T @ Ug - np.eye(k))))
+    assert orth <= 1e-5, orth
+    # residuals of the Ritz pairs, A = Phi Phi^T applied in float64
+    def resid(Um, t):
+        AU = phi64 @ (phi64.T @ Um)
+        return np.linalg.norm(AU - Um * t[None, :], axis=0)
+    rg, ro = resid(Ug, th), resid(U_o, th_o)
+    assert np.all(rg <= ro + 1e-6 * abs(th_o[0])), float(np.max(rg - ro))
+    print(f"qwen14b Lanczos: max rel Ritz err {float(np.max(err / np.abs(th_o))):.2e}, "
+          f"angle {ang:.2e}, |U^T U - I| {orth:.2e}, max residual gpu {rg.max():.3e} "
+          f"oracle {ro.max():.3e}")

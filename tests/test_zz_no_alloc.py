@@ -54,12 +54,23 @@ def test_noalloc_matches_workspace_entry_point():
         ang = scipy.linalg.subspace_angles(U.cpu().numpy()[:, :kk].astype(np.float64),
                                            U_ref.cpu().numpy()[:, :kk].astype(np.float64))
         assert np.max(ang) <= 1e-3
-    # sizes past the fixed scratch are refused with a clear error
-    big = L.sls_lanczos_workspace_size(1 << 20, 2048, 128)
-    assert big > (32 << 20)
-    st = L.sls_lanczos_topr_noalloc(ctypes.c_void_p(Phi.data_ptr()), 1 << 20, 2048, 128,
+    # sizes past the fixed scratch are refused with a clear error, before
+    # anything is enqueued: real buffers of a problem whose workspace is just
+    # over the limit (the basis alone is 41 MB), r_eff left untouched
+    N, D, r = 40000, 256, 128
+    need = L.sls_lanczos_workspace_size(N, D, r)
+    assert (32 << 20) < need < (64 << 20)
+    phi, q1 = _problem(N, D, 3)
+    Phi = torch.from_numpy(phi).cuda()
+    Q1 = torch.from_numpy(q1).cuda()
+    theta = torch.zeros(r, dtype=torch.float64, device="cuda")
+    U = torch.zeros((N, r), dtype=torch.float32, device="cuda")
+    k = torch.full((1,), 12345, dtype=torch.int32, device="cuda")
+    st = L.sls_lanczos_topr_noalloc(ctypes.c_void_p(Phi.data_ptr()), N, D, r,
                                     ctypes.c_void_p(Q1.data_ptr()), 1e-10,
                                     ctypes.c_void_p(theta.data_ptr()),
                                     ctypes.c_void_p(U.data_ptr()),
                                     ctypes.c_void_p(k.data_ptr()), None, None, s)
     assert st == 3
+    torch.cuda.synchronize()
+    assert int(k.item()) == 12345
