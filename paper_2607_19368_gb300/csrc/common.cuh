@@ -354,6 +354,7 @@ SLS_DEV void named_sync(unsigned id, unsigned nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+
 // ---------------------------------------------------------------------------
 // memory-model helpers
 // ---------------------------------------------------------------------------

@@ -510,30 +510,40 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
                    int groups, int g, cudaStream_t stream) {
   const LzLayout L = lz_layout(bt.nmax, bt.D, bt.r, g);
   if ((size_t)groups * L.total > scratch_bytes) return SLS_ERR_WORKSPACE;
-  // barrier words of every group start at zero (one strided memset)
-  SLS_CUDA_TRY(cudaMemset2DAsync((char*)scratch + L.bar, L.total, 0, 256, groups, stream));
+  // barrier words and group sums of every group start at zero (one strided memset)
+  SLS_CUDA_TRY(cudaMemset2DAsync((char*)scratch + L.bar, L.total, 0, L.zero_end - L.bar, groups,
+                                 stream));
   const int C4 = bt.D / 4;
   const int P = (C4 >= LZ_CT) ? 1 : (LZ_CT / C4);
-  const int redn = (P > 1) ? P * bt.D : 0;
-  const int rows_cap = (int)((bt.nmax + g - 1) / g) + 1;
-  // shared memory besides the ring: w (hi, lo; only for D < 4 LZ_CT), phase
-  // partials, z' of the strip, row-dot warp sums, coefficient partials and c,
-  // barriers
-  const size_t other = sizeof(float) * 2 * (size_t)(P > 1 ? bt.D : 0) +
-                       sizeof(float2) * ((size_t)redn + (size_t)rows_cap + 16 * LZ_CW +
-                                         (size_t)(LZ_CW + 1) * (bt.r + 1)) +
-                       16 + 2 * RING_MAX_STAGES * 8;
+  const int gpt = gpt_of(bt.D);
+  if (gpt == 0) return SLS_ERR_UNSUPPORTED;
+  const int teams = lz_teams(gpt, P);
+  // z' of the strip, rounded up to an even count so the arrays after it stay
+  // 16-byte aligned
+  const int rows_cap = (int)(((bt.nmax + g - 1) / g + 2) & ~(int64_t)1);
   const size_t limit = 227 * 1024 - 1024;  // leave room for static shared memory
-  if (other >= limit) return SLS_ERR_UNSUPPORTED;
   if (bt.phi_bf16 && (bt.D % 8)) return SLS_ERR_UNSUPPORTED;  // 16-byte rows for the copies
-  const RingShape R = ring_shape(bt.D, q_ld(bt.r), limit - other, bt.phi_bf16 ? 2 : 4);
-  if (R.S < 2) return SLS_ERR_UNSUPPORTED;
-  const size_t smem = (size_t)R.S * R.stage + other;
-  const int stages = R.S;
+  const int esz = bt.phi_bf16 ? 2 : 4;
+  // the stage count and the mbarriers that go with it: take the largest S
+  // whose ring and other shared memory fit
+  RingShape R = ring_shape(bt.D, q_ld(bt.r), 0, esz, teams);
+  int stages = 0;
+  for (int s = RING_MAX_STAGES; s >= 1; --s) {
+    if ((size_t)s * R.stage + lz_smem_other(bt.D, bt.r, rows_cap, teams, s) <= limit) {
+      stages = s;
+      break;
+    }
+  }
+  // two chunks per team in flight at least, and room for the pass ends'
+  // scratch in the ring
+  if (stages < 2 * teams) return SLS_ERR_UNSUPPORTED;
+  if ((size_t)stages * R.stage < lz_pass_end_bytes(gpt, bt.r, teams)) return SLS_ERR_UNSUPPORTED;
+  const size_t smem = (size_t)stages * R.stage + lz_smem_other(bt.D, bt.r, rows_cap, teams, stages);
   const int kt = (bt.r <= 32) ? 1 : (bt.r <= 64) ? 2 : 4;  // 32-wide tiles of k < r
-#define SLS_LZ_CALL(fn) fn(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream, kt)
+#define SLS_LZ_CALL(fn) \
+  fn(bt, scratch, L.total, groups, g, rows_cap, stages, status, smem, stream, kt, teams)
   if (bt.phi_bf16) {
-    switch (gpt_of(bt.D)) {
+    switch (gpt) {
       case 1: return SLS_LZ_CALL(launch_lanczos_bf16_gpt1);
       case 2: return SLS_LZ_CALL(launch_lanczos_bf16_gpt2);
       case 4: return SLS_LZ_CALL(launch_lanczos_bf16_gpt4);
@@ -541,7 +551,7 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
       default: break;
     }
   } else {
-    switch (gpt_of(bt.D)) {
+    switch (gpt) {
       case 1: return SLS_LZ_CALL(launch_lanczos_gpt1);
       case 2: return SLS_LZ_CALL(launch_lanczos_gpt2);
       case 4: return SLS_LZ_CALL(launch_lanczos_gpt4);

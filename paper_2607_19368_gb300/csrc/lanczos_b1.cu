@@ -1,13 +1,15 @@
-// Lanczos kernel instantiations for 1 four-element column group(s) of Phi
-// per compute thread (D <= 1024), Phi stored as bfloat16, for every basis tile
-// count KT.
+// Lanczos kernel instantiations for 1 float4 column group(s) of Phi per
+// compute thread (D <= 1024), Phi stored as bfloat16, for every basis tile count KT, with
+// one team (D < 1024) or two (D = 1024) of compute warps.
 #include "lanczos_kernel.cuh"
 
 namespace sls {
 
 int launch_lanczos_bf16_gpt1(SLS_LZ_LAUNCH_ARGS) {
-  return launch_lanczos_kt<1, uint16_t>(bt, scratch, gstride, groups, g, rows_cap, stages,
-                                         status, smem, stream, kt);
+  return teams == 2 ? launch_lanczos_kt<1, uint16_t, 2>(bt, scratch, gstride, groups, g, rows_cap,
+                                                      stages, status, smem, stream, kt)
+                    : launch_lanczos_kt<1, uint16_t, 1>(bt, scratch, gstride, groups, g, rows_cap,
+                                                      stages, status, smem, stream, kt);
 }
 
 }  // namespace sls
