@@ -48,6 +48,9 @@ extern "C" {
 #define SLS_ERR_WORKSPACE 3    /* workspace missing or smaller than required     */
 #define SLS_ERR_CUDA 4         /* a CUDA launch or copy failed                   */
 #define SLS_ERR_TIMEOUT 5      /* a device-side wait reached its iteration limit */
+#define SLS_ERR_BOUNDS 6       /* debug build only: a device-side bounds check or a
+                                  workspace guard band caught an access outside its
+                                  range (the access was skipped)                  */
 
 /* Embedding dtypes. */
 #define SLS_F32 0
@@ -456,6 +459,22 @@ int sls_selftest_wait_limit(int which, void* workspace, size_t workspace_bytes,
 int sls_selftest_lanczos_giveup(const float* Phi, int64_t N, int D, int r, const double* q1,
                                 double* theta, float* U, int32_t* r_eff, void* workspace,
                                 size_t workspace_bytes, void* stream);
+
+/*
+ * Self-test of the debug build's checks (a library built with -DSLS_DEBUG,
+ * libsls_debug.so; the paper has no counterpart).  That build surrounds
+ * every region it carves from a workspace with a guard band, filled when a
+ * call starts and checked when it ends, and guards selected device-side
+ * accesses (row indices of the Lanczos kernel, member rows of the
+ * aggregation) so that an out-of-range access is skipped and reported as
+ * SLS_ERR_BOUNDS in the workspace status word instead of faulting.
+ * which = 0 writes into a guard band (inside the caller's workspace);
+ * which = 1 makes a guarded out-of-range write.  Either leaves
+ * SLS_ERR_BOUNDS in the status word (read it with sls_workspace_status).
+ * workspace: at least 1024 device bytes.  Errors: INVALID_ARG (which),
+ * WORKSPACE, UNSUPPORTED in the ordinary build (which has no checks).
+ */
+int sls_debug_selftest(int which, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * Reads (synchronously, on `stream`) the device status word of a workspace

@@ -40,7 +40,27 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 
 
 def lib_path() -> str:
-    return os.path.join(_HERE, "libsls.so")
+    """The library the binding loads: libsls.so next to this file, or the
+    path in the SLS_LIBRARY environment variable (e.g. the debug build
+    libsls_debug.so), read when the library is first loaded."""
+    return os.environ.get("SLS_LIBRARY") or os.path.join(_HERE, "libsls.so")
+
+
+def debug_lib_path() -> str:
+    return os.path.join(_HERE, "libsls_debug.so")
+
+
+# With SLS_CHECK_STATUS=1 every call that takes a workspace reads its status
+# word afterwards (synchronising) and raises on anything but SLS_OK: with the
+# debug build this turns each call into a bounds and guard-band check.
+_CHECK_STATUS = os.environ.get("SLS_CHECK_STATUS") == "1"
+
+
+def _check_ws(fn: str, ws: torch.Tensor):
+    if _CHECK_STATUS:
+        st = int(lib().sls_workspace_status(_ptr(ws), _stream(ws)))
+        if st != SLS_OK:
+            raise SLSError(fn + " (device status)", st, lib().sls_status_string(st).decode())
 
 
 class SLSError(RuntimeError):
@@ -123,6 +143,7 @@ EXPORTED = {
                                         _vp, _d, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "sls_selftest_lanczos_giveup": (_i32, [_vp, _i64, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _sz,
                                            _vp]),
+    "sls_debug_selftest": (_i32, [_i32, _vp, _sz, _vp]),
     "sls_set_phase_events": (_i32, [ctypes.POINTER(ctypes.c_void_p), _i32]),
     "sls_launch_count": (_i64, []),
 }
@@ -267,6 +288,7 @@ def lanczos_topr(Phi: torch.Tensor, q1: torch.Tensor, r: int, tol: float = 1e-10
                                _ptr(theta), _ptr(U), _ptr(r_eff), _ptr(alpha), _ptr(beta),
                                _ptr(ws), ws.numel(), _stream(Phi))
     _check("sls_lanczos_topr_ex", st)
+    _check_ws("sls_lanczos_topr_ex", ws)
     return theta, U, r_eff, alpha, beta
 
 
@@ -304,6 +326,7 @@ def lanczos_topr_batched(Phi: torch.Tensor, q1: torch.Tensor, r: int, row0, n, q
                                     _ptr(theta), _ptr(U), _ptr(r_eff), _ptr(alpha),
                                     _ptr(beta), _ptr(ws), ws.numel(), _stream(Phi))
     _check("sls_lanczos_topr_batched", st)
+    _check_ws("sls_lanczos_topr_batched", ws)
     return theta, U, r_eff, alpha, beta
 
 
@@ -365,6 +388,7 @@ def aggregate(X: torch.Tensor, codes: torch.Tensor, M_target: int, pos_scheme: i
                          M_target, pos_scheme, int(renorm), _ptr(Xt), _ptr(pos), _ptr(t2m),
                          _ptr(ws), ws.numel(), _stream(X))
     _check("sls_aggregate", st)
+    _check_ws("sls_aggregate", ws)
     return Xt, pos, t2m
 
 
@@ -441,6 +465,7 @@ def compress(X: torch.Tensor, cfg: Config, W: Optional[torch.Tensor] = None,
                             _ptr(Xt), _ptr(pos), _ptr(t2m), _ptr(r_eff), _ptr(route),
                             _ptr(workspace.buf), workspace.nbytes, _stream(X3))
     _check("sls_compress", st)
+    _check_ws("sls_compress", workspace.buf)
     del keep
     if not batched:
         return Xt[0], pos[0], t2m[0], r_eff, route

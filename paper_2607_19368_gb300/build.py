@@ -3,7 +3,10 @@
 Each translation unit under csrc/ is compiled by its own nvcc process (in
 parallel), then linked into ``paper_2607_19368_gb300/libsls.so`` with the
 CUDA runtime linked statically, so the library has no dependency beyond the
-driver.  Usage: ``python -m paper_2607_19368_gb300.build [--force]``.
+driver.  ``debug=True`` builds ``libsls_debug.so`` instead, with -DSLS_DEBUG:
+guard bands around every workspace region and device-side bounds guards that
+report SLS_ERR_BOUNDS (a stand-in for a memory checker).  Usage:
+``python -m paper_2607_19368_gb300.build [--force] [--debug]``.
 """
 from __future__ import annotations
 
@@ -17,6 +20,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libsls.so")
+BUILD_DEBUG = os.path.join(HERE, "_build_debug")
+LIB_DEBUG = os.path.join(HERE, "libsls_debug.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -48,8 +53,8 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def _compile(src: str, extra) -> str:
-    obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+def _compile(src: str, extra, outdir: str) -> str:
+    obj = os.path.join(outdir, os.path.basename(src)[:-3] + ".o")
     if _stale(obj, [src] + headers()):
         cmd = [nvcc()] + ARCH + NVCC_FLAGS + list(extra) + ["-c", src, "-o", obj]
         res = subprocess.run(cmd, capture_output=True, text=True)
@@ -58,27 +63,31 @@ def _compile(src: str, extra) -> str:
     return obj
 
 
-def build(force: bool = False, verbose: bool = False, extra=()) -> str:
-    """Compile every .cu file and link libsls.so; returns the library path."""
-    os.makedirs(BUILD, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, extra=(), debug: bool = False) -> str:
+    """Compile every .cu file and link libsls.so (libsls_debug.so with
+    debug=True); returns the library path."""
+    outdir, lib = (BUILD_DEBUG, LIB_DEBUG) if debug else (BUILD, LIB)
+    extra = list(extra) + (["-DSLS_DEBUG"] if debug else [])
+    os.makedirs(outdir, exist_ok=True)
     if force:
-        for f in os.listdir(BUILD):
+        for f in os.listdir(outdir):
             if f.endswith(".o"):
-                os.remove(os.path.join(BUILD, f))
+                os.remove(os.path.join(outdir, f))
     srcs = sources()
-    with cf.ThreadPoolExecutor(max_workers=min(8, len(srcs))) as ex:
-        objs = list(ex.map(lambda s: _compile(s, extra), srcs))
-    if force or _stale(LIB, objs):
-        tmp = LIB + ".tmp"
+    workers = max(1, min(16, os.cpu_count() or 1, len(srcs)))
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        objs = list(ex.map(lambda s: _compile(s, extra, outdir), srcs))
+    if force or _stale(lib, objs):
+        tmp = lib + ".tmp"
         cmd = [nvcc()] + ARCH + ["-shared", "-o", tmp] + objs
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
             raise RuntimeError(f"link failed:\n{res.stderr}")
-        os.replace(tmp, LIB)
+        os.replace(tmp, lib)
     if verbose:
-        print(f"built {LIB}")
-    return LIB
+        print(f"built {lib}")
+    return lib
 
 
 if __name__ == "__main__":
-    build(force="--force" in sys.argv, verbose=True)
+    build(force="--force" in sys.argv, verbose=True, debug="--debug" in sys.argv)

@@ -32,17 +32,86 @@ inline void phase_mark(int phase, int end, cudaStream_t s) {
 // workspace carving
 // ---------------------------------------------------------------------------
 
+// In the debug build (-DSLS_DEBUG) every carved region is followed by a
+// guard band of kGuardBytes filled with kGuardByte when a call starts and
+// checked when it ends (guard_check_kernel): a write past the end of a
+// region shows up as SLS_ERR_BOUNDS in the workspace status word.  The
+// ordinary build carves no guards.
+#ifdef SLS_DEBUG
+constexpr size_t kGuardBytes = 256;
+constexpr int kMaxGuards = 48;
+#else
+constexpr size_t kGuardBytes = 0;
+constexpr int kMaxGuards = 1;
+#endif
+constexpr unsigned char kGuardByte = 0xA5;
+
+struct GuardList {
+  int n;
+  size_t off[kMaxGuards];
+};
+
 struct Carver {
   char* base;
   size_t off = 0;
+  GuardList guards{};
   explicit Carver(void* b) : base((char*)b) {}
   template <typename T>
   T* take(size_t count) {
     T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
     off += sls_align256(count * sizeof(T));
+    if (kGuardBytes) {
+      if (guards.n < kMaxGuards) guards.off[guards.n++] = off;
+      off += kGuardBytes;
+    }
     return p;
   }
 };
+
+__global__ void guard_fill_kernel(unsigned char* base, GuardList g) {
+  if ((int)blockIdx.x >= g.n) return;
+  unsigned char* p = base + g.off[blockIdx.x];
+  for (int b = threadIdx.x; b < (int)kGuardBytes; b += blockDim.x) p[b] = kGuardByte;
+}
+
+__global__ void guard_check_kernel(const unsigned char* base, GuardList g, int* status) {
+  if ((int)blockIdx.x >= g.n) return;
+  const unsigned char* p = base + g.off[blockIdx.x];
+  for (int b = threadIdx.x; b < (int)kGuardBytes; b += blockDim.x)
+    if (p[b] != kGuardByte) atomicExch(status, SLS_ERR_BOUNDS);
+}
+
+// Debug-build self-test: which = 0 writes one element past the end of a
+// carved region of n ints (into its guard band: still inside the caller's
+// workspace); which = 1 makes a guarded write at index n, which the guard
+// skips.  Either must end in SLS_ERR_BOUNDS.
+__global__ void debug_selftest_kernel(int* region, int n, int which, int* status) {
+  if (threadIdx.x != 0) return;
+  if (which == 0) {
+    reinterpret_cast<unsigned char*>(region + n)[0] = (unsigned char)(kGuardByte ^ 0xFF);
+  } else {
+    const int idx = n;
+    SLS_DBG_GUARD(status, idx < n) region[idx] = 1;
+  }
+}
+
+// Debug build: fill the guard bands of a carved workspace (no-op otherwise).
+int guards_arm(const Carver& cv, cudaStream_t s) {
+  if (kGuardBytes == 0 || cv.base == nullptr || cv.guards.n == 0) return SLS_OK;
+  guard_fill_kernel<<<cv.guards.n, 256, 0, s>>>((unsigned char*)cv.base, cv.guards);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
+
+// Debug build: check the guard bands, SLS_ERR_BOUNDS into *status if one
+// was written (no-op otherwise).
+int guards_check(const Carver& cv, int* status, cudaStream_t s) {
+  if (kGuardBytes == 0 || cv.base == nullptr || cv.guards.n == 0) return SLS_OK;
+  guard_check_kernel<<<cv.guards.n, 256, 0, s>>>((const unsigned char*)cv.base, cv.guards,
+                                                 status);
+  SLS_LAUNCH_CHECK();
+  return SLS_OK;
+}
 
 // host-side configuration arithmetic (Sec. 3.3, 3.5, 3.6)
 struct Region {
@@ -298,6 +367,8 @@ struct CompressWs {
   int* counts;
   float *part, *part_eta;
   size_t total;
+  Carver cv{nullptr};    // the head of the workspace (guards in the debug build)
+  Carver tail{nullptr};  // the tail (aggregation partials, router partials)
 };
 
 int num_sms_host() {
@@ -396,9 +467,10 @@ void carve(const CompressPlan& P, void* ws, CompressWs* W) {
   W->pt_start = cv.take<int>(macs);
   W->items = cv.take<int2>(agg_item_capacity(macs, toks));
   W->counts = cv.take<int>(agg_aux_ints(macs, toks));
-  W->part = cv.take<float>(0);  // sized below (depends on d)
+  W->part = nullptr;  // carved from the tail (depends on d)
   W->part_eta = nullptr;
   W->total = cv.off;
+  W->cv = cv;
 }
 
 bool ptr_ok(const void* p) { return p != nullptr && ((uintptr_t)p & 15u) == 0; }
@@ -424,14 +496,14 @@ int validate_config(const sls_config_t* c) {
   return SLS_OK;
 }
 
-size_t score_bytes(const CompressPlan& P, int d, int backend) {
-  if (backend != SLS_BACKEND_ADAPTIVE) return 0;
-  return sls_align256(score_part_floats(P.nprob, P.nmax, d) * sizeof(float));
-}
-
-size_t part_bytes(int64_t toks, int d) {
-  return sls_align256(agg_part_capacity(toks) * (size_t)d * sizeof(float)) +
-         sls_align256(agg_part_capacity(toks) * sizeof(float));
+// Bytes of the workspace tail: the aggregation partials (and the router's
+// window partials for the adaptive backend), carved in this order.
+size_t tail_bytes(const CompressPlan& P, int64_t toks, int d, int backend) {
+  Carver cv(nullptr);
+  cv.take<float>(agg_part_capacity(toks) * (size_t)d);
+  cv.take<float>(agg_part_capacity(toks));
+  if (backend == SLS_BACKEND_ADAPTIVE) cv.take<float>(score_part_floats(P.nprob, P.nmax, d));
+  return cv.off;
 }
 
 // One Lanczos problem (sls_lanczos_topr_ex); inject_fail = 1 runs the
@@ -461,6 +533,7 @@ int lanczos_single(const void* Phi, int phi_dtype, int64_t N, int D, int r, cons
   const size_t lzb = lanczos_scratch_bytes(N, D, r, groups, g);
   void* lz = cv.take<char>(lzb);
   SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
+  if ((st = guards_arm(cv, s)) != SLS_OK) return st;
   // -1 until the Lanczos kernel finishes; stays -1 if one of its waits gave
   // up, and the eigen and Ritz kernels then treat the problem as empty
   SLS_CUDA_TRY(cudaMemsetAsync(r_eff, 0xff, sizeof(int32_t), s));
@@ -491,7 +564,7 @@ int lanczos_single(const void* Phi, int phi_dtype, int64_t N, int D, int r, cons
   if ((st = launch_ritz_vectors(bt, U, s)) != SLS_OK) return st;
   if (alpha) SLS_CUDA_TRY(cudaMemcpyAsync(alpha, al, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
   if (beta) SLS_CUDA_TRY(cudaMemcpyAsync(beta, be, sizeof(double) * r, cudaMemcpyDeviceToDevice, s));
-  return SLS_OK;
+  return guards_check(cv, status, s);
 }
 
 }  // namespace
@@ -510,6 +583,7 @@ const char* sls_status_string(int status) {
     case SLS_ERR_WORKSPACE: return "workspace missing or too small";
     case SLS_ERR_CUDA: return "CUDA launch or copy failed";
     case SLS_ERR_TIMEOUT: return "device wait reached its iteration limit";
+    case SLS_ERR_BOUNDS: return "debug build: an access outside its range was caught and skipped";
     default: return "unknown status";
   }
 }
@@ -653,6 +727,7 @@ int sls_lanczos_topr_batched(const void* Phi, int phi_dtype, int D, int r, int n
   const size_t lzb = lanczos_scratch_bytes(nmax, D, r, groups, g);
   void* lz = cv.take<char>(lzb);
   SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
+  if ((st = guards_arm(cv, s)) != SLS_OK) return st;
   SLS_CUDA_TRY(cudaMemsetAsync(r_eff, 0xff, sizeof(int32_t) * (size_t)nprob, s));
   LanczosBatch bt{};
   bt.Phi = Phi;
@@ -688,7 +763,7 @@ int sls_lanczos_topr_batched(const void* Phi, int phi_dtype, int D, int r, int n
   if (beta)
     SLS_CUDA_TRY(cudaMemcpyAsync(beta, be, sizeof(double) * r * (size_t)nprob,
                                  cudaMemcpyDeviceToDevice, s));
-  return SLS_OK;
+  return guards_check(cv, status, s);
 }
 
 int sls_simhash(const float* U, int64_t N, int k, int ldu, const int32_t* k_dev, const float* R,
@@ -712,7 +787,9 @@ size_t sls_aggregate_workspace_size(int64_t N, int d, int64_t M_target) {
   cv.take<int>(M_target);
   cv.take<int2>(agg_item_capacity(M_target, N));
   cv.take<int>(agg_aux_ints(M_target, N));
-  return cv.off + part_bytes(N, d);
+  cv.take<float>(agg_part_capacity(N) * (size_t)d);
+  cv.take<float>(agg_part_capacity(N));
+  return cv.off;
 }
 
 int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
@@ -742,14 +819,17 @@ int sls_aggregate(const void* X, int x_dtype, int64_t N, int d, int64_t ldx,
   float* part = cv.take<float>(agg_part_capacity(N) * (size_t)d);
   float* part_eta = cv.take<float>(agg_part_capacity(N));
   SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
+  int st;
+  if ((st = guards_arm(cv, s)) != SLS_OK) return st;
   single_prob_kernel<<<1, 1, 0, s>>>(prob, N, M_target, 32);
   SLS_LAUNCH_CHECK();
-  int st;
   if ((st = launch_segment(prob, 1, codes, pos_scheme, SLS_MODE_REPRESENTATIVE, seg, 1, N,
                            M_target, perm, mstart, mlen, pos, tok2macro, status, s)) != SLS_OK)
     return st;
-  return launch_aggregate(X, x_dtype, d, ldx, perm, mstart, mlen, M_target, N, renorm, Xt,
-                          pt_start, items, counts, part, part_eta, status, s);
+  if ((st = launch_aggregate(X, x_dtype, d, ldx, perm, mstart, mlen, M_target, N, renorm, Xt,
+                             pt_start, items, counts, part, part_eta, status, s)) != SLS_OK)
+    return st;
+  return guards_check(cv, status, s);
 }
 
 int64_t sls_output_count(const sls_config_t* cfg, int64_t N) {
@@ -767,7 +847,7 @@ size_t sls_compress_workspace_size(const sls_config_t* cfg, int64_t B, int64_t N
   if (make_plan(cfg, B, N, &P) != SLS_OK) return 0;
   CompressWs W;
   carve(P, nullptr, &W);
-  return W.total + part_bytes(B * N, d) + score_bytes(P, d, cfg->backend);
+  return W.total + tail_bytes(P, B * N, d, cfg->backend);
 }
 
 int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B, int64_t N, int d,
@@ -780,8 +860,11 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   if (x_dtype != SLS_F32 && x_dtype != SLS_BF16) return SLS_ERR_INVALID_ARG;
   if (!ptr_ok(X) || !Xt || !pos || !tok2macro) return SLS_ERR_INVALID_ARG;
   cudaStream_t s = (cudaStream_t)stream;
-  if (is_identity(cfg, N))
+  if (is_identity(cfg, N)) {
+    // the workspace (if any) holds only the status word
+    if (workspace && workspace_bytes >= 256) SLS_CUDA_TRY(cudaMemsetAsync(workspace, 0, 256, s));
     return launch_identity(X, x_dtype, B, N, d, ldx, Xt, pos, tok2macro, s);
+  }
   const int vec = (x_dtype == SLS_BF16) ? 8 : 4;
   if (d % vec || ldx % vec || d > SLS_MAX_D) return SLS_ERR_UNSUPPORTED;
   CompressPlan P;
@@ -795,7 +878,7 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
   }
   CompressWs W;
   carve(P, workspace, &W);
-  const size_t need = W.total + part_bytes(B * N, d) + score_bytes(P, d, cfg->backend);
+  const size_t need = W.total + tail_bytes(P, B * N, d, cfg->backend);
   if (!workspace || workspace_bytes < need) return SLS_ERR_WORKSPACE;
   {
     Carver tail((char*)workspace + W.total);
@@ -804,8 +887,11 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
     W.score_part = (cfg->backend == SLS_BACKEND_ADAPTIVE)
                        ? tail.take<float>(score_part_floats(P.nprob, P.nmax, d))
                        : nullptr;
+    W.tail = tail;
   }
   SLS_CUDA_TRY(cudaMemsetAsync(W.status, 0, 256, s));
+  if ((st = guards_arm(W.cv, s)) != SLS_OK) return st;
+  if ((st = guards_arm(W.tail, s)) != SLS_OK) return st;
   const int nprob = (int)P.nprob;
   phase_mark(0, 0, s);
   // problem table
@@ -935,7 +1021,9 @@ int sls_compress(const sls_config_t* cfg, const void* X, int x_dtype, int64_t B,
                         cfg->renorm, Xt, W.pt_start, W.items, W.counts, W.part, W.part_eta,
                         W.status, s);
   phase_mark(6, 1, s);
-  return st;
+  if (st != SLS_OK) return st;
+  if ((st = guards_check(W.cv, W.status, s)) != SLS_OK) return st;
+  return guards_check(W.tail, W.status, s);
 }
 
 int sls_embed_gather(const void* table, int x_dtype, int64_t V, int d, int64_t ld_table,
@@ -1001,6 +1089,23 @@ int sls_selftest_wait_limit(int which, void* workspace, size_t workspace_bytes, 
   if (!ptr_ok(workspace) || workspace_bytes < 512) return SLS_ERR_WORKSPACE;
   return launch_selftest_wait_limit(which, (int*)workspace,
                                     (unsigned*)((char*)workspace + 256), (cudaStream_t)stream);
+}
+
+int sls_debug_selftest(int which, void* workspace, size_t workspace_bytes, void* stream) {
+  if (which != 0 && which != 1) return SLS_ERR_INVALID_ARG;
+  if (kGuardBytes == 0) return SLS_ERR_UNSUPPORTED;  // the ordinary build has no checks
+  if (!ptr_ok(workspace)) return SLS_ERR_WORKSPACE;
+  cudaStream_t s = (cudaStream_t)stream;
+  Carver cv(workspace);
+  int* status = cv.take<int>(64);
+  int* region = cv.take<int>(64);
+  if (workspace_bytes < cv.off) return SLS_ERR_WORKSPACE;
+  SLS_CUDA_TRY(cudaMemsetAsync(status, 0, 256, s));
+  int st;
+  if ((st = guards_arm(cv, s)) != SLS_OK) return st;
+  debug_selftest_kernel<<<1, 32, 0, s>>>(region, 64, which, status);
+  SLS_LAUNCH_CHECK();
+  return guards_check(cv, status, s);
 }
 
 int sls_workspace_status(void* workspace, void* stream) {

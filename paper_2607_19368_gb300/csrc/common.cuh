@@ -442,6 +442,29 @@ SLS_DEV bool group_sync_named(const GroupBarrier& bar, unsigned& local_gen, int*
 }
 
 // ---------------------------------------------------------------------------
+// debug build (-DSLS_DEBUG): device-side bounds guards
+// ---------------------------------------------------------------------------
+// SLS_DBG_GUARD(status, cond) stmt;  runs stmt only when cond holds; in the
+// debug build a false cond records SLS_ERR_BOUNDS in *status (when status is
+// not NULL) and skips stmt instead of letting the access go out of bounds.
+// In the ordinary build the check and the guard vanish: stmt always runs.
+#ifdef SLS_DEBUG
+#define SLS_DBG_GUARD(status, cond)                                 \
+  if (!(cond)) {                                                    \
+    if ((status) != nullptr) atomicExch((status), SLS_ERR_BOUNDS);  \
+  } else
+#define SLS_DBG_CHECK(status, cond)                                     \
+  do {                                                                  \
+    if (!(cond) && (status) != nullptr) atomicExch((status), SLS_ERR_BOUNDS); \
+  } while (0)
+#else
+#define SLS_DBG_GUARD(status, cond)
+#define SLS_DBG_CHECK(status, cond) \
+  do {                              \
+  } while (0)
+#endif
+
+// ---------------------------------------------------------------------------
 // host-side helpers
 // ---------------------------------------------------------------------------
 

@@ -1580,9 +1580,10 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
                 const int2* __restrict__ items, const int* __restrict__ cta_first,
                 const int* __restrict__ pt_start, int renorm, float* __restrict__ Xt,
                 float* __restrict__ part, float* __restrict__ part_eta, int S, int stage_bytes,
-                int* status) {
+                int* status, int64_t ntot) {
   constexpr int V = VecOf<T>::V;
   extern __shared__ __align__(128) unsigned char agr_smem[];
+  (void)ntot;  // bounds of the member rows (debug-build checks)
   __shared__ uint64_t fullb[AGR_MAX_STAGES], emptyb[AGR_MAX_STAGES];
   __shared__ AggDesc dring[AGR_MAX_STAGES + 2];
   __shared__ float shq[2][AGR_CW][AGG_CH];
@@ -1649,7 +1650,16 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
               if (s == 0) dring[(kb + j) % DQ] = D;
               unsigned char* dst = agr_smem + (size_t)st * stage_bytes;
               mbar_expect_tx(&fullb[st], row_bytes);
-              bulk_g2s(dst, X + (int64_t)row * ldx, row_bytes, &fullb[st], pol);
+              int64_t src_row = row;
+#ifdef SLS_DEBUG
+              // a member row outside the token set is not fetched: the stage
+              // gets row 0 instead and the status records SLS_ERR_BOUNDS
+              if (!(row >= 0 && (int64_t)row < ntot)) {
+                atomicExch(status, SLS_ERR_BOUNDS);
+                src_row = 0;
+              }
+#endif
+              bulk_g2s(dst, X + src_row * ldx, row_bytes, &fullb[st], pol);
             }
           }
           ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
@@ -2325,7 +2335,7 @@ int launch_agg_t(const void* X, int d, int64_t ldx, const int* perm, const int* 
   const AggAux A = agg_aux(aux, Mtot, Ntot);
   agg_ring_kernel<T, NV><<<grid, AGR_THREADS, smem, stream>>>(
       (const T*)X, d, ldx, perm, mstart, mlen, items, A.cta_first, pt_start, renorm, Xt, part,
-      part_eta, S, stage, status);
+      part_eta, S, stage, status, Ntot);
   SLS_LAUNCH_CHECK();
   agg_final_kernel<V, NV><<<(unsigned)fblocks, AGG_T, 0, stream>>>(
       d, mlen, pt_start, Mtot, Ntot, renorm, aux, part, part_eta, Xt);

@@ -266,28 +266,71 @@ SLS_DEV void sweepA_team_pair(const PT* __restrict__ c0, int nr0, int lb0,
   const float C = ofs_pow2(phimax * ut1);
   const f32x2_t Cp = pk2(C, C);
   f32x2_t s[GPT][2], lo[GPT][2];
+  if constexpr (GPT == 1) {
+    // packed pairs
 #pragma unroll
-  for (int q = 0; q < GPT; ++q) {
-    s[q][0] = s[q][1] = Cp;
-    lo[q][0] = lo[q][1] = 0ull;
-  }
+    for (int q = 0; q < GPT; ++q) {
+      s[q][0] = s[q][1] = Cp;
+      lo[q][0] = lo[q][1] = 0ull;
+    }
 #pragma unroll
-  for (int i = 0; i < 2 * CR; ++i) {
-    const bool first = i < CR;
-    const int ii = first ? i : i - CR;
-    if (FULL || ii < (first ? nr0 : nr1)) {
-      const PT* ch = first ? c0 : c1;
-      const float2 u = us[(first ? lb0 : lb1) + ii];
-      const f32x2_t uh = pk2(u.x, u.x), ul = pk2(u.y, u.y);
+    for (int i = 0; i < 2 * CR; ++i) {
+      const bool first = i < CR;
+      const int ii = first ? i : i - CR;
+      if (FULL || ii < (first ? nr0 : nr1)) {
+        const PT* ch = first ? c0 : c1;
+        const float2 u = us[(first ? lb0 : lb1) + ii];
+        const f32x2_t uh = pk2(u.x, u.x), ul = pk2(u.y, u.y);
 #pragma unroll
-      for (int q = 0; q < GPT; ++q) {
-        const int cg = tt + q * LZ_CT;
-        if (FULL || cg < C4) {
-          const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
-          ofs_fma_acc2(s[q][0], lo[q][0], pk2(f.x, f.y), uh, ul);
-          ofs_fma_acc2(s[q][1], lo[q][1], pk2(f.z, f.w), uh, ul);
+        for (int q = 0; q < GPT; ++q) {
+          const int cg = tt + q * LZ_CT;
+          if (FULL || cg < C4) {
+            const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
+            ofs_fma_acc2(s[q][0], lo[q][0], pk2(f.x, f.y), uh, ul);
+            ofs_fma_acc2(s[q][1], lo[q][1], pk2(f.z, f.w), uh, ul);
+          }
         }
       }
+    }
+  } else {
+    // scalar steps for two or more column groups per thread: measured faster
+    // there (qwen7b shape, alternating builds), and the instruction counters
+    // show the packed form executing about 1.3 register moves per step, so
+    // it saves fewer issue slots than its halved arithmetic count suggests
+    float sc[GPT][4], lc[GPT][4];
+#pragma unroll
+    for (int q = 0; q < GPT; ++q)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        sc[q][e] = C;
+        lc[q][e] = 0.f;
+      }
+#pragma unroll
+    for (int i = 0; i < 2 * CR; ++i) {
+      const bool first = i < CR;
+      const int ii = first ? i : i - CR;
+      if (FULL || ii < (first ? nr0 : nr1)) {
+        const PT* ch = first ? c0 : c1;
+        const float2 u = us[(first ? lb0 : lb1) + ii];
+#pragma unroll
+        for (int q = 0; q < GPT; ++q) {
+          const int cg = tt + q * LZ_CT;
+          if (FULL || cg < C4) {
+            const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
+            ofs_fma_acc(sc[q][0], lc[q][0], f.x, u.x, u.y);
+            ofs_fma_acc(sc[q][1], lc[q][1], f.y, u.x, u.y);
+            ofs_fma_acc(sc[q][2], lc[q][2], f.z, u.x, u.y);
+            ofs_fma_acc(sc[q][3], lc[q][3], f.w, u.x, u.y);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < GPT; ++q) {
+      s[q][0] = pk2(sc[q][0], sc[q][1]);
+      s[q][1] = pk2(sc[q][2], sc[q][3]);
+      lo[q][0] = pk2(lc[q][0], lc[q][1]);
+      lo[q][1] = pk2(lc[q][2], lc[q][3]);
     }
   }
 #pragma unroll
@@ -339,22 +382,49 @@ SLS_DEV void sweepB_team_pair(const PT* __restrict__ c0, int nr0, const PT* __re
   for (int i = 0; i < R2; ++i) {
     const bool first = i < CR;
     const int ii = first ? i : i - CR;
-    f32x2_t s = pk2(Ct, Ct), lo = 0ull;
-    if (FULL || ii < (first ? nr0 : nr1)) {
-      const PT* ch = first ? c0 : c1;
+    float sx, sy, lx, ly;
+    if constexpr (GPT == 1) {
+      f32x2_t s = pk2(Ct, Ct), lo = 0ull;
+      if (FULL || ii < (first ? nr0 : nr1)) {
+        const PT* ch = first ? c0 : c1;
 #pragma unroll
-      for (int q = 0; q < GPT; ++q) {
-        const int cg = tt + q * LZ_CT;
-        if (FULL || cg < C4) {
-          const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
-          ofs_fma_acc2(s, lo, pk2(f.x, f.y), wh[q][0], wl[q][0]);
-          ofs_fma_acc2(s, lo, pk2(f.z, f.w), wh[q][1], wl[q][1]);
+        for (int q = 0; q < GPT; ++q) {
+          const int cg = tt + q * LZ_CT;
+          if (FULL || cg < C4) {
+            const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
+            ofs_fma_acc2(s, lo, pk2(f.x, f.y), wh[q][0], wl[q][0]);
+            ofs_fma_acc2(s, lo, pk2(f.z, f.w), wh[q][1], wl[q][1]);
+          }
+        }
+      }
+      upk2(s, sx, sy);
+      upk2(lo, lx, ly);
+    } else {
+      // scalar steps (see sweepA_team_pair)
+      sx = Ct;
+      sy = Ct;
+      lx = 0.f;
+      ly = 0.f;
+      if (FULL || ii < (first ? nr0 : nr1)) {
+        const PT* ch = first ? c0 : c1;
+#pragma unroll
+        for (int q = 0; q < GPT; ++q) {
+          const int cg = tt + q * LZ_CT;
+          if (FULL || cg < C4) {
+            const float4 f = phi_ld4(ch, (size_t)ii * C4 + cg);
+            float a0, a1, b0, b1, c0_, c1_, d0, d1;
+            upk2(wh[q][0], a0, a1);
+            upk2(wl[q][0], b0, b1);
+            upk2(wh[q][1], c0_, c1_);
+            upk2(wl[q][1], d0, d1);
+            ofs_fma_acc(sx, lx, f.x, a0, b0);
+            ofs_fma_acc(sy, ly, f.y, a1, b1);
+            ofs_fma_acc(sx, lx, f.z, c0_, d0);
+            ofs_fma_acc(sy, ly, f.w, c1_, d1);
+          }
         }
       }
     }
-    float sx, sy, lx, ly;
-    upk2(s, sx, sy);
-    upk2(lo, lx, ly);
     vh[i] = (sx - Ct) + (sy - Ct);  // exact (one grid, below Ct / 2)
     vl[i] = lx + ly;
   }
@@ -812,6 +882,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       for (int h = 0; h < 2; ++h) {
         const int t = t0 + h + S;
         if (t >= nch) break;
+        SLS_DBG_CHECK(status, t >= 0 && ring_adv(q0, h, S).slot < S);
         issue_chunk<PT>(base + (unsigned)t, ring_adv(q0, h, S).slot,
                         (pass & 1) ? nch - 1 - t : t, cr, nrows, D, ldq, stage, phib, ring, fullb,
                         slot_cnt, Phis, Qs, pol);
@@ -895,7 +966,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       dfloat nacc = df_make(0.f, 0.f);
       for (int il = tid; il < nrows; il += NCT) {
         const dfloat z = df_from_double(q1[rs + il]);
-        zps[il] = f2(z);
+        SLS_DBG_GUARD(status, il < rows_cap) zps[il] = f2(z);
         dot2_acc_df(nacc.hi, nacc.lo, z, z);
       }
       f32x2_t ah[GPT][2], al[GPT][2];
@@ -1147,6 +1218,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           const float2* qb1 = reinterpret_cast<const float2*>(ring + (size_t)s1 * stage + phib);
           const int nr0 = min(cr, nrows - kc0 * cr);
           const int nr1 = two ? min(cr, nrows - kc1 * cr) : 0;
+          SLS_DBG_CHECK(status, kc0 >= 0 && kc0 < nch && nr0 >= 1 && (!two || (kc1 >= 0 && kc1 < nch && nr1 >= 1)));
           // row work before the row dots: q_j of the warp's rows of the pair
           // (it feeds only the row work after them)
           dfloat qjv[RPW];
@@ -1166,7 +1238,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
               if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
               qjv[m] = df_mul(z1, invb_df);
               if (j > 0) qpv[m] = qrow[j - 1];
-              if (lane == 0) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
+              if (lane == 0) SLS_DBG_GUARD(status, il < nrows) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
             }
           }
           // row dots s = Phi w_j, warp sums into bp[row * LZ_CW + tw]
@@ -1207,7 +1279,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
               dfloat zp = df_sub(v[0], df_mul(alpha_df, qjv[m]));
               if (j > 0) zp = df_sub(zp, df_mul(beta_df, dfv(qpv[m])));
               if (lane == 0) {
-                zps[il] = f2(zp);
+                SLS_DBG_GUARD(status, il < nrows) zps[il] = f2(zp);
                 dot2_acc_df(nacc.hi, nacc.lo, zp, zp);
               }
 #pragma unroll
@@ -1250,12 +1322,12 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
             dfloat z1 = dfv(zps[il]);
             if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
             const dfloat qj = df_mul(z1, invb_df);
-            if (lane == 0) Qs[(size_t)il * ldq + j] = f2(qj);
+            if (lane == 0) SLS_DBG_GUARD(status, il < nrows) Qs[(size_t)il * ldq + j] = f2(qj);
             const dfloat s = row_dot_smem(chunk + (size_t)ii * D, D, wsh, wsl);
             dfloat zp = df_sub(s, df_mul(alpha_df, qj));
             if (j > 0) zp = df_sub(zp, df_mul(beta_df, dfv(qrow[j - 1])));
             if (lane == 0) {
-              zps[il] = f2(zp);
+              SLS_DBG_GUARD(status, il < nrows) zps[il] = f2(zp);
               dot2_acc_df(nacc.hi, nacc.lo, zp, zp);
             }
 #pragma unroll
