@@ -10,7 +10,9 @@ last 12 tokens preserved, global backend.  Prints one JSON line.
                   [--workload qwen7b|qwen14b|mistral7b|adaptive|local] [--rho R]
 
 --workload qwen14b (N = 131072, d = 5120) and mistral7b (N = 8192, d = 4096)
-time the other single-prompt shapes; --workload adaptive times the windowed
+time the other single-prompt shapes; --workload adaptive_mixed times the same
+batch shape with about half of the windows coherent, so that the router
+sends windows both ways at rho = 4 and 8; --workload adaptive times the windowed
 batch: 64 prompts of N = 16384, d = 4096 bf16 (duplication 0.6 p / 63 for
 prompt p), windows of 2048 routed to the chunk or the spectral chain, D = 1024,
 r = 32, bits from the window budget, rho from --rho (default 8); --workload
@@ -49,7 +51,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--workload", default="qwen7b",
-                    choices=["qwen7b", "qwen14b", "mistral7b", "adaptive", "local"])
+                    choices=["qwen7b", "qwen14b", "mistral7b", "adaptive", "adaptive_mixed",
+                             "local"])
     ap.add_argument("--rho", type=float, default=None,
                     help="compression ratio (default: the workload's)")
     ap.add_argument("--normalize", action="store_true",
@@ -83,8 +86,10 @@ def config_dict(w, rho, extra=None):
              "l2": (f"inputs larger than L2 (X {w.N * w.d * 2 / 1e6:.0f} MB per step), "
                     f"no flush")}
     elif w.batch > 1:
+        mix = (f", each window coherent (rows 0.8 t + 0.6 e_i) with probability "
+               f"{w.coherent_frac:g}" if w.coherent_frac > 0 else "")
         d = {"workload": f"{w.name}: {w.batch} prompts of N={w.N} d={w.d} bf16, windows of "
-                         f"{w.window}, D={w.D} r={w.r} b=auto rho={rho:g} "
+                         f"{w.window}{mix}, D={w.D} r={w.r} b=auto rho={rho:g} "
                          f"preserve_last={w.preserve_last}, adaptive backend",
              "B": w.batch, "window": w.window,
              "l2": (f"inputs larger than L2 (X {w.batch * w.N * w.d * 2 / 1e9:.1f} GB per "
@@ -104,7 +109,7 @@ def config_dict(w, rho, extra=None):
 # Revision of the persistent Lanczos kernel whose DRAM counters are recorded in
 # profiles/lanczos_traffic.json; bumped with every change of the kernel, so a
 # stale capture reads as "traffic": null.
-LANCZOS_KERNEL_REV = "fused-pass/8"
+LANCZOS_KERNEL_REV = "fused-pass/9"
 
 
 def peaks():
@@ -221,8 +226,15 @@ def sample_prompt(w):
     import workloads as WL
     if w.batch > 1:
         i = w.batch // 2
-        return WL.make_prompt(w, index=i, dup_frac=WL.adaptive_dup_frac(i, w.batch)), i
+        return WL.make_prompt(w, index=i, dup_frac=prompt_dup(w, i)), i
     return WL.make_prompt(w), 0
+
+
+def prompt_dup(w, i):
+    """Copied-span fraction of prompt i of a batch: varied over the prompts of
+    the adaptive workload, the workload's own otherwise."""
+    import workloads as WL
+    return WL.adaptive_dup_frac(i, w.batch) if w.name == "adaptive" else None
 
 
 def cpu_phases(w, rho, X64, prm, n):
@@ -351,10 +363,25 @@ def device_inputs(w, rank, dev):
         p = WL.make_prompt(w, index=rank)
         X = torch.from_numpy(p.X.view(np.int16)).view(torch.bfloat16).to(dev)
         return X, p.ids.astype(np.int32).reshape(1, w.N)
-    ids = [WL.prompt_ids(w, index=i, dup_frac=WL.adaptive_dup_frac(i, w.batch))
-           for i in range(w.batch)]
+    ids = [WL.prompt_ids(w, index=i, dup_frac=prompt_dup(w, i)) for i in range(w.batch)]
     uniq, inv = np.unique(np.concatenate(ids), return_inverse=True)
-    table = WL.f32_to_bf16_bits(WL.vocab_rows(WL.DATA_SEED, uniq, w.d).astype(np.float32))
+    rows = WL.vocab_rows(WL.DATA_SEED, uniq, w.d).astype(np.float32)
+    if w.coherent_frac > 0:
+        # coherent windows mix a topic direction into the float32 vocabulary
+        # rows on the device, then round to bf16 (the generator's recipe)
+        tab = torch.from_numpy(rows).to(dev)
+        idx = torch.from_numpy(inv.astype(np.int64)).to(dev)
+        X = torch.empty((w.batch, w.N, w.d), dtype=torch.bfloat16, device=dev)
+        a = w.coherent_mix
+        for i in range(w.batch):
+            Xi = tab.index_select(0, idx[i * w.N:(i + 1) * w.N])
+            for r0, r1, t in WL.coherent_windows(w, index=i):
+                tv = torch.from_numpy(t.astype(np.float32)).to(dev)
+                Xi[r0:r1] = a * tv[None, :] + math.sqrt(1.0 - a * a) * Xi[r0:r1]
+            X[i] = Xi.to(torch.bfloat16)
+        del tab
+        return X, np.stack(ids).astype(np.int32)
+    table = WL.f32_to_bf16_bits(rows)
     tab = torch.from_numpy(table.view(np.int16)).to(dev)
     idx = torch.from_numpy(inv.astype(np.int64)).to(dev)
     X = tab.index_select(0, idx).view(torch.bfloat16).view(w.batch, w.N, w.d)
@@ -596,17 +623,20 @@ def e2e_measure(run, args, world):
 
     ms_pipe = timed(pipeline(Xh, lambda x, o: run.step(x, o)), args.e2e_steps)
     # from token ids: the model's embedding table stays in HBM and only the
-    # ids come in; the lookup X = E[ids] runs inside the call
+    # ids come in; the lookup X = E[ids] runs inside the call (not for the
+    # coherent-window workload, whose embeddings are no table rows)
     adaptive = w.batch > 1
-    table = vocab_table(run.X, run.ids, w.V, dev)
-    Ih = torch.from_numpy(run.ids if adaptive else run.ids.reshape(N)).pin_memory()
-    tws = sls.TokensWorkspace(cfg, table.dtype, B, N, d, dev)
-    ms_ids = timed(pipeline(Ih, lambda i, o: sls.compress_tokens(i, table, cfg, run.Wt, run.bt,
-                                                                   run.Rt, run.qt, workspace=tws,
-                                                                   out=o)),
-                   args.e2e_steps)
-    del table, tws
-    m2 = max_over_ranks([ms_pipe, ms_serial, ms_ids], world, dev)
+    ms_ids = None
+    if w.coherent_frac <= 0:
+        table = vocab_table(run.X, run.ids, w.V, dev)
+        Ih = torch.from_numpy(run.ids if adaptive else run.ids.reshape(N)).pin_memory()
+        tws = sls.TokensWorkspace(cfg, table.dtype, B, N, d, dev)
+        ms_ids = timed(pipeline(Ih, lambda i, o: sls.compress_tokens(i, table, cfg, run.Wt,
+                                                                       run.bt, run.Rt, run.qt,
+                                                                       workspace=tws, out=o)),
+                       args.e2e_steps)
+        del table, tws
+    m2 = max_over_ranks([ms_pipe, ms_serial, ms_ids or 0.0], world, dev)
     d2h_bytes = Xt.numel() * 4 + pos.numel() * 4 + t2m.numel() * 4
     pipe_v = world * B * N / (m2[0] / 1e3)
     serial_v = world * B * N / (m2[1] / 1e3)
@@ -624,9 +654,9 @@ def e2e_measure(run, args, world):
                      "here than the double-buffered pattern)"),
             "pipelined_value": pipe_v,
             "serial_value": serial_v,
-            "from_token_ids": {
+            "from_token_ids": None if ms_ids is None else {
                 "value": world * B * N / (m2[2] / 1e3), "unit": UNIT,
-                "h2d_bytes_per_step": int(Ih.numel()) * 4,
+                "h2d_bytes_per_step": int(B * N) * 4,
                 "d2h_bytes_per_step": d2h_bytes,
                 "mode": "double-buffered as above; token ids in, the V x d bf16 embedding "
                         "table resident on the device, lookup inside sls_compress_tokens"}}
@@ -727,7 +757,8 @@ def run_native(args, rank, world):
             and not args.normalize and args.phi == "f32":
         sweep = [sweep_entry(sls, nm, r_ or workload(nm).rho, rank, dev, world,
                              args.sweep_steps, 3)
-                 for nm, r_ in (("mistral7b", None), ("qwen14b", None), ("adaptive", 16.0))]
+                 for nm, r_ in (("mistral7b", None), ("qwen14b", None), ("adaptive", 16.0),
+                                ("adaptive_mixed", 8.0))]
     if rank != 0:
         return
     extra = {"parallelism": f"replicas x{world}",

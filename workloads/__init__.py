@@ -24,6 +24,16 @@ available here):
 * ``local``     the ``qwen7b`` prompt at the paper's local-LSH defaults
                 (Sec. 5.1 hyperparameters: D=256, r=16, window 16, bits from
                 the window budget), rho=8.
+* ``adaptive_mixed`` 64 prompts of N=16384, d=4096, bf16 (the ``adaptive``
+                vocabulary, no copied spans) in which each 2048-token window
+                of the compressible region is, with probability 1/2 (seeded),
+                a coherent window: its rows are 0.8 t + 0.6 e_i with t a unit
+                topic direction drawn for the window and e_i the token's
+                vocabulary row.  A coherent window's tokens share a direction
+                (redundancy score about 0.8 on Eq. redundancy) while keeping
+                full rank; the others score near 0, so the adaptive router
+                sends about half of the windows to the spectral chain and half
+                to the chunk path at rho = 4 and 8.
 
 Vocabulary rows are N(0, 1/d) and are produced by a counter-based generator
 (numpy Philox keyed by the seed, counter = token id), so the V x d table is
@@ -78,6 +88,7 @@ def _rng(seed: int, stream: int) -> np.random.Generator:
 _STREAM_IDS = 11
 _STREAM_SPANS = 12
 _STREAM_NOISE = 13
+_STREAM_TOPIC = 14
 _STREAM_W = 21
 _STREAM_B = 22
 _STREAM_R = 23
@@ -184,6 +195,8 @@ class Workload:
     window: int = 0     # window length of the windowed backends (0 = global backend)
     rhos: tuple = ()    # swept compression ratios (adaptive workload)
     backend: str = "global"   # "global", "adaptive" or "local"
+    coherent_frac: float = 0.0  # share of coherent windows (adaptive_mixed)
+    coherent_mix: float = 0.8   # weight of the window's topic direction in them
 
 
 WORKLOADS = {
@@ -202,6 +215,11 @@ WORKLOADS = {
                          dtype="bf16", D=1024, r=32, bits=0, rho=8.0,
                          dup_frac=0.0, span_lo=64, span_hi=64, batch=64,
                          window=2048, rhos=(2.0, 4.0, 8.0, 16.0), backend="adaptive"),
+    "adaptive_mixed": Workload("adaptive_mixed", N=16384, d=4096, V=32768, zipf=1.1,
+                               dtype="bf16", D=1024, r=32, bits=0, rho=8.0,
+                               dup_frac=0.0, span_lo=64, span_hi=64, batch=64,
+                               window=2048, rhos=(4.0, 8.0), backend="adaptive",
+                               coherent_frac=0.5),
     "local": Workload("local", N=32768, d=3584, V=151936, zipf=1.05,
                       dtype="bf16", D=256, r=16, bits=0, rho=8.0,
                       dup_frac=0.3, span_lo=16, span_hi=256, window=16,
@@ -240,9 +258,34 @@ def prompt_ids(w: Workload, seed: int = DATA_SEED, index: int = 0,
     return ids
 
 
+def coherent_windows(w: Workload, seed: int = DATA_SEED, index: int = 0):
+    """The coherent windows of prompt ``index`` of a workload with
+    coherent_frac > 0: a list of (row start, row end, unit topic direction t)
+    over the windows of the compressible region [preserve_first, N -
+    preserve_last), each window coherent with probability coherent_frac."""
+    if w.coherent_frac <= 0 or w.window <= 0:
+        return []
+    rng = _rng(seed + 1000 * index, _STREAM_TOPIC)
+    pf, nc = w.preserve_first, w.N - w.preserve_first - w.preserve_last
+    out = []
+    for s0 in range(0, nc, w.window):
+        pick = rng.random() < w.coherent_frac
+        t = rng.standard_normal(w.d)
+        if pick:
+            out.append((pf + s0, pf + min(s0 + w.window, nc), t / np.linalg.norm(t)))
+    return out
+
+
 def make_prompt(w: Workload, seed: int = DATA_SEED, index: int = 0,
                 dup_frac: Optional[float] = None) -> Prompt:
     ids = prompt_ids(w, seed, index, dup_frac)
+    if w.coherent_frac > 0:
+        X = vocab_rows(seed, ids, w.d)
+        a = w.coherent_mix
+        for r0, r1, t in coherent_windows(w, seed, index):
+            X[r0:r1] = a * t[None, :] + math.sqrt(1.0 - a * a) * X[r0:r1]
+        X32 = X.astype(np.float32)
+        return Prompt(ids, f32_to_bf16_bits(X32) if w.dtype == "bf16" else X32, w.dtype)
     uniq, inv = np.unique(ids, return_inverse=True)
     table = vocab_rows(seed, uniq, w.d).astype(np.float32)
     if w.noise_var > 0:
