@@ -642,6 +642,16 @@ SLS_DEV void store_col_partials(const f32x2_t (&ah)[GPT][2], const f32x2_t (&al)
 // and every G-th basis index, then a butterfly within the segment.  The loads
 // of the first column batch are issued before the named barrier after which
 // c is ready (warp 0 fills it meanwhile); `synced` records that barrier.
+// True when the last warp of the CTA sums no column in the slice phase (the
+// column split of slice_columns below): it is free then for beta.
+template <int NCW>
+SLS_DEV bool slice_last_warp_idle(int ncol) {
+  constexpr int NCT = NCW * 32;
+  int G = 1;
+  while (G < 32 && G * 2 * ncol <= NCT) G *= 2;
+  return (NCW - 1) * (32 / G) >= ncol;
+}
+
 template <int NCW>
 SLS_DEV dfloat slice_columns(const float2* __restrict__ wpart, const float2* __restrict__ Wm,
                              float2* __restrict__ wred, const float2* __restrict__ cs, int g,
@@ -855,38 +865,46 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     const int cbeg = (int)((int64_t)rank * D / g), cend = (int)((int64_t)(rank + 1) * D / g);
 
     double scale = 0.0, alpha_prev = 0.0;
+    // beta_{j-1} = 1 / e_inv and the break test of the step, in lane 0 of
+    // warp bw: the last warp during the slice phase when that warp sums no
+    // column there (measured 2% faster at the qwen7b shape), else warp 0
+    // after group barrier 2
+    double e_inv = 0.0, e_bnew = 0.0;
+    int e_brk = 0;
+    const bool beta_early = slice_last_warp_idle<NCW>(cend - cbeg);
+    const int bw = beta_early ? NCW - 1 : 0;
     dfloat alpha_df = df_make(0.f, 0.f), beta_df = df_make(0.f, 0.f), invb_df;
     float phimax = 0.f;  // max |Phi| over this CTA's strip (prologue pass)
     int reff = 0;
     sbreak = 0;
 
     // The first min(S, nch) chunks of pass `pass` (0 = the prologue; passes
-    // alternate direction), issued by one thread once the ring is idle.
+    // alternate direction), issued once the ring is idle, chunk t by lane 0
+    // of warp t mod NCW: the thread that issues a bulk copy is held for a few
+    // hundred cycles, so the copies are spread over warps.
     auto issue_pass_head = [&](int pass) {
-      if (tid == 0) {
+      if (lane == 0) {
         const int m = min(S, nch);
-        RingPos q = ring_pos(base, S);
-        for (int t = 0; t < m; ++t) {
-          issue_chunk<PT>(base + (unsigned)t, q.slot, (pass & 1) ? nch - 1 - t : t, cr, nrows, D,
-                          ldq, stage, phib, ring, fullb, slot_cnt, Phis, Qs, pol);
-          q = ring_adv(q, 1, S);
-        }
+        for (int t = warp; t < m; t += NCW)
+          issue_chunk<PT>(base + (unsigned)t, ring_slot(base + (unsigned)t, S),
+                          (pass & 1) ? nch - 1 - t : t, cr, nrows, D, ldq, stage, phib, ring,
+                          fullb, slot_cnt, Phis, Qs, pol);
       }
     };
-    // Refill of a team's previous pair in pass `pass`: chunks t0 + S and
-    // t0 + 1 + S of the pass where they exist, into the slots of chunks t0
-    // and t0 + 1 at ring position q0 (called by the team's first thread after
-    // a team barrier, so no warp reads those slots any more).
-    auto refill_pair = [&](int pass, int t0, RingPos q0) {
-      if (t0 < 0) return;
-      for (int h = 0; h < 2; ++h) {
-        const int t = t0 + h + S;
-        if (t >= nch) break;
-        SLS_DBG_CHECK(status, t >= 0 && ring_adv(q0, h, S).slot < S);
-        issue_chunk<PT>(base + (unsigned)t, ring_adv(q0, h, S).slot,
-                        (pass & 1) ? nch - 1 - t : t, cr, nrows, D, ldq, stage, phib, ring, fullb,
-                        slot_cnt, Phis, Qs, pol);
-      }
+    // Refill of a team's previous pair in pass `pass`: chunk t0 + h + S of
+    // the pass where it exists, into the slot of chunk t0 + h at ring
+    // position q0 + h.  Called after a team barrier (no warp reads those
+    // slots any more) by lane 0 of the team's last two warps, one chunk each
+    // (measured 3.5% faster at the qwen7b shape than one thread issuing
+    // both).
+    auto refill_half = [&](int pass, int t0, RingPos q0) {
+      const int h = tw - (LZ_CW - 2);
+      if (t0 < 0 || lane != 0 || h < 0) return;
+      const int t = t0 + h + S;
+      if (t >= nch) return;
+      SLS_DBG_CHECK(status, t >= 0 && ring_adv(q0, h, S).slot < S);
+      issue_chunk<PT>(base + (unsigned)t, ring_adv(q0, h, S).slot, (pass & 1) ? nch - 1 - t : t,
+                      cr, nrows, D, ldq, stage, phib, ring, fullb, slot_cnt, Phis, Qs, pol);
     };
 
     // pass end: team 1's column sums join team 0's through the ring (idle
@@ -985,7 +1003,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         if (!chunk_wait(c0n, qc, fullb, slot_cnt)) lz_fail(status, &s_err);
         if (two && !chunk_wait(c0n + 1, q1p, fullb, slot_cnt)) lz_fail(status, &s_err);
         named_sync(bar_team, LZ_CT);
-        if (tt == 0) refill_pair(0, prev, qprev);
+        refill_half(0, prev, qprev);
         prev = t0p;
         qprev = qc;
         for (int h = 0; h < (two ? 2 : 1); ++h) {
@@ -1015,6 +1033,35 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         return;
       }
       const double* accj = acc + (size_t)(gstep & 1u) * accs;
+      // |z1|^2 = |z'|^2 - |c|^2 (Q orthonormal): beta_{j-1} and the break
+      // test (warp bw, once c is in shared memory)
+      auto beta_phase = [&]() {
+        const double zs = accj[r + 1];
+        dfloat cn = df_make(0.f, 0.f);
+#pragma unroll
+        for (int t2 = 0; t2 < KT; ++t2) {
+          const int k = lane + 32 * t2;
+          if (k < j) dot2_acc_df(cn.hi, cn.lo, dfv(cs[k]), dfv(cs[k]));
+        }
+        cn = df_norm(cn.hi, cn.lo);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) cn = df_add_fast(cn, shfl_xor_df(cn, o));
+        if (lane == 0) {
+          const double nrm2 = zs - df_to_double(cn);  // |z1|^2
+          // one reciprocal square root instead of a square root and two
+          // divides (float64 runs at a fraction of the float32 rate here)
+          e_inv = (nrm2 > 0.0) ? rsqrt(nrm2) : 0.0;  // 1 / beta
+          e_bnew = (nrm2 > 0.0) ? nrm2 * e_inv : 0.0;
+          e_brk = 0;
+          if (j > 0) {
+            scale = fmax(scale, fabs(alpha_prev) + e_bnew);
+            if (!(e_bnew > bt.tol * scale)) e_brk = 1;
+            else if (rank == 0) beta_out[j - 1] = e_bnew;
+          } else if (!(e_bnew > 0.0)) {
+            e_brk = 1;
+          }
+        }
+      };
 
       // ---------------- slice phase: c, Phi^T z1 for this CTA's columns ----------
       // c = Q^T z' (k < j) from the group sums; Phi^T z1 = Phi^T z' - sum_k
@@ -1032,6 +1079,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         bool synced = false;
         dfloat sq = slice_columns<NCW>(wpart, Wm, wred, cs, g, D, j, cbeg, cend, synced);
         if (!synced) named_sync(BAR_ALL, NCT);
+        if (beta_early && warp == NCW - 1) beta_phase();
         sq = df_norm(sq.hi, sq.lo);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) sq = df_add_fast(sq, shfl_xor_df(sq, o));
@@ -1064,40 +1112,15 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           }
         }
       }
-      if (warp == 0) {
-        // |z1|^2 = |z'|^2 - |c|^2 (Q orthonormal), |Phi^T z1|^2
-        const double s = accj[r + 1];
-        const double q = accj[r + 2];
-        dfloat cn = df_make(0.f, 0.f);
-#pragma unroll
-        for (int t2 = 0; t2 < KT; ++t2) {
-          const int k = lane + 32 * t2;
-          if (k < j) dot2_acc_df(cn.hi, cn.lo, dfv(cs[k]), dfv(cs[k]));
-        }
-        cn = df_norm(cn.hi, cn.lo);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) cn = df_add_fast(cn, shfl_xor_df(cn, o));
-        if (lane == 0) {
-          const double nrm2 = s - df_to_double(cn);  // |z1|^2
-          // one reciprocal square root instead of a square root and two
-          // divides (float64 runs at a fraction of the float32 rate here)
-          const double inv = (nrm2 > 0.0) ? rsqrt(nrm2) : 0.0;    // 1 / beta
-          const double bnew = (nrm2 > 0.0) ? nrm2 * inv : 0.0;
-          int brk = 0;
-          if (j > 0) {
-            scale = fmax(scale, fabs(alpha_prev) + bnew);
-            if (!(bnew > bt.tol * scale)) brk = 1;
-            else if (rank == 0) beta_out[j - 1] = bnew;
-          } else if (!(bnew > 0.0)) {
-            brk = 1;
-          }
-          const double a = brk ? 0.0 : (q * inv) * inv;
-          if (!brk && rank == 0) alpha_out[j] = a;
-          shd[1] = brk ? 0.0 : inv;
-          shd[2] = a;
-          shd[3] = (j > 0) ? bnew : 0.0;
-          sbreak = brk;
-        }
+      if (!beta_early && warp == 0) beta_phase();
+      if (warp == bw && lane == 0) {
+        const double q = accj[r + 2];  // |Phi^T z1|^2
+        const double a = e_brk ? 0.0 : (q * e_inv) * e_inv;
+        if (!e_brk && rank == 0) alpha_out[j] = a;
+        shd[1] = e_brk ? 0.0 : e_inv;
+        shd[2] = a;
+        shd[3] = (j > 0) ? e_bnew : 0.0;
+        sbreak = e_brk;
       }
       named_sync(BAR_ALL, NCT);
       if (sbreak) {
@@ -1223,34 +1246,51 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           // (it feeds only the row work after them)
           dfloat qjv[RPW];
           float2 qpv[RPW];
-#pragma unroll
-          for (int m = 0; m < RPW; ++m) {
-            const int ri = tw + m * LZ_CW;
-            const bool first = ri < TCR;
-            const int ii = first ? ri : ri - TCR;
-            qjv[m] = df_make(0.f, 0.f);
-            qpv[m] = make_float2(0.f, 0.f);
-            if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
-              const int il = (first ? kc0 : kc1) * cr + ii;
-              const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
-              const float corr = row_corr<KT>(qrow, cs, j);
-              dfloat z1 = dfv(zps[il]);
-              if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
-              qjv[m] = df_mul(z1, invb_df);
-              if (j > 0) qpv[m] = qrow[j - 1];
-              if (lane == 0) SLS_DBG_GUARD(status, il < nrows) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
-            }
-          }
-          // row dots s = Phi w_j, warp sums into bp[row * LZ_CW + tw]
-          if (fullD && nr0 == TCR && nr1 == TCR)
+          if (fullD && nr0 == TCR && nr1 == TCR && 2 * TCR >= LZ_CW) {
+            // steady state, every warp owns one row of the pair: q_j of that
+            // row and the row dots in one block, so that the warp reduction
+            // of q_j interleaves with the sweep's arithmetic (measured 2.9%
+            // faster at the qwen7b shape than q_j ahead of the sweep)
+            const bool first = tw < TCR;
+            const int ii = first ? tw : tw - TCR;
+            const int il = (first ? kc0 : kc1) * cr + ii;
+            const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
+            const float corr = row_corr<KT>(qrow, cs, j);  // 0 at j = 0
+            qjv[0] = df_mul(df_add(dfv(zps[il]), df_make(-corr, 0.f)), invb_df);
+            qpv[0] = (j > 0) ? qrow[j > 0 ? j - 1 : 0] : make_float2(0.f, 0.f);
             sweepB_team_pair<GPT, TCR, true>(ch0, nr0, ch1, nr1, C4, tt, wh, wl, Ct, bp,
                                              bp + TCR * LZ_CW);
-          else
-            sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, tt, wh, wl, Ct, bp,
-                                              bp + TCR * LZ_CW);
+            if (lane == 0) SLS_DBG_GUARD(status, il < nrows) Qs[(size_t)il * ldq + j] = f2(qjv[0]);
+          } else {
+#pragma unroll
+            for (int m = 0; m < RPW; ++m) {
+              const int ri = tw + m * LZ_CW;
+              const bool first = ri < TCR;
+              const int ii = first ? ri : ri - TCR;
+              qjv[m] = df_make(0.f, 0.f);
+              qpv[m] = make_float2(0.f, 0.f);
+              if (ri < 2 * TCR && ii < (first ? nr0 : nr1)) {
+                const int il = (first ? kc0 : kc1) * cr + ii;
+                const float2* qrow = (first ? qb0 : qb1) + (size_t)ii * ldq;
+                const float corr = row_corr<KT>(qrow, cs, j);
+                dfloat z1 = dfv(zps[il]);
+                if (j > 0) z1 = df_add(z1, df_make(-corr, 0.f));
+                qjv[m] = df_mul(z1, invb_df);
+                if (j > 0) qpv[m] = qrow[j - 1];
+                if (lane == 0) SLS_DBG_GUARD(status, il < nrows) Qs[(size_t)il * ldq + j] = f2(qjv[m]);
+              }
+            }
+            // row dots s = Phi w_j, warp sums into bp[row * LZ_CW + tw]
+            if (fullD && nr0 == TCR && nr1 == TCR)
+              sweepB_team_pair<GPT, TCR, true>(ch0, nr0, ch1, nr1, C4, tt, wh, wl, Ct, bp,
+                                               bp + TCR * LZ_CW);
+            else
+              sweepB_team_pair<GPT, TCR, false>(ch0, nr0, ch1, nr1, C4, tt, wh, wl, Ct, bp,
+                                                bp + TCR * LZ_CW);
+          }
           named_sync(bar_team, LZ_CT);
           // every warp of the team is past its previous pair: refill those slots
-          if (tt == 0) refill_pair(pass, prev, qprev);
+          refill_half(pass, prev, qprev);
           prev = t0p;
           qprev = qc;
           qc = ring_adv(qc, 2 * TEAMS, S);
