@@ -18,12 +18,17 @@
 //           256-column fp32 accumulators in tensor memory; tcgen05.commit
 //           releases ring stages and hands finished accumulators over;
 //   warps 2-5 epilogue: tcgen05.ld 32x32b (one TMEM lane = one output row
-//           per thread), cos epilogue, global stores; then release the
-//           accumulator, so the next tile's MMAs overlap this epilogue.
+//           per thread), cos epilogue; float32 features go through a
+//           128B-swizzled 32 x 32 staging block per warp (two per warp, in
+//           turn) and leave by TMA tensor stores, bfloat16 ones by direct
+//           stores; then release the accumulator, so the next tile's MMAs
+//           overlap this epilogue.
 // Every wait is bounded; a wait that gives up records SLS_ERR_TIMEOUT, the
 // other roles stop at their next wait, in-flight copies and MMAs are drained
 // and the tensor memory is freed before the CTA exits.
 #include <cuda.h>
+
+#include <cstring>
 
 #include "common.cuh"
 #include "kernels.cuh"
@@ -41,7 +46,10 @@ constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;
 constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
 constexpr int TC_THREADS = 192;
 constexpr int TC_TMEM_COLS = 2 * TC_BN;
-constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES + 1024 + 256;
+constexpr int TC_EPI_WARPS = 4;
+constexpr int TC_OUT_BYTES = 32 * 32 * 4;  // one 32 x 32 float32 staging block
+constexpr size_t TC_SMEM =
+    (size_t)TC_STAGES * TC_STAGE_BYTES + (size_t)TC_EPI_WARPS * 2 * TC_OUT_BYTES + 1024 + 256;
 
 __device__ int g_fm_status;  // timeouts when the caller passes no status word
 
@@ -113,6 +121,57 @@ SLS_DEV bool tc_wait(uint64_t* bar, unsigned parity, volatile int* abort_flag) {
   return false;
 }
 
+// cos(x) for the epilogue, branch-free for |x| <= 8192: Cody and Waite's
+// reduction (W. J. Cody and W. Waite, "Software Manual for the Elementary
+// Functions", 1980) by k = rint(x 2/pi) against pi/2 split into three
+// float32 parts (P1 + P2 + P3, each the float32 rounding of what the
+// previous parts leave of pi/2; with fused multiply-adds the first step is
+// exact for |k| < 2^13), then the Taylor series of cos and sin on the
+// reduced |r| <= pi/4 (truncation below 2e-9) in Horner form, and the
+// quadrant k mod 4 picks cos r, -sin r, -cos r or sin r.  Larger or
+// non-finite arguments take the library cosine (rff_cos_wide).
+constexpr float RFF_COS_FAST_MAX = 8192.f;
+
+__device__ __noinline__ float rff_cos_wide(float x) { return cosf(x); }
+
+SLS_DEV float rff_cos_fast(float x) {
+  const float k = rintf(x * 0x1.45f306p-1f);  // x * (2/pi)
+  float r = __fmaf_rn(-k, 0x1.921fb6p+0f, x);
+  r = __fmaf_rn(-k, -0x1.777a5cp-25f, r);
+  r = __fmaf_rn(-k, -0x1.ee59dap-50f, r);
+  const float z = r * r;
+  // cos r = 1 - z/2! + z^2/4! - z^3/6! + z^4/8! - z^5/10!
+  float c = __fmaf_rn(z, -1.f / 3628800.f, 1.f / 40320.f);
+  c = __fmaf_rn(z, c, -1.f / 720.f);
+  c = __fmaf_rn(z, c, 1.f / 24.f);
+  c = __fmaf_rn(z, c, -0.5f);
+  c = __fmaf_rn(z, c, 1.f);
+  // sin r = r (1 - z/3! + z^2/5! - z^3/7! + z^4/9!)
+  float s = __fmaf_rn(z, 1.f / 362880.f, -1.f / 5040.f);
+  s = __fmaf_rn(z, s, 1.f / 120.f);
+  s = __fmaf_rn(z, s, -1.f / 6.f);
+  s = __fmaf_rn(r * z, s, r);
+  const int q = (int)k;
+  const float v = (q & 1) ? s : c;
+  // quadrants 1 and 2 are negative
+  return __uint_as_float(__float_as_uint(v) ^ ((unsigned)((q + 1) & 2) << 30));
+}
+
+// TMA tensor store of a 32 x 32 float32 block (3-d map: feature, row, prompt)
+// from shared memory, tracked as a bulk async group of the issuing thread.
+SLS_DEV void tma_store_3d(const CUtensorMap* map, uint32_t src, int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(src), "r"(x), "r"(y), "r"(z)
+      : "memory");
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// at most one bulk group of this thread still reading shared memory
+SLS_DEV void bulk_wait_read_le1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+SLS_DEV void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+SLS_DEV void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
 // Rows of one launch: nb prompts of `rows` rows each, prompt b starting at
 // X row b * x_stride (of the tensor map) and Phi row b * rows.  live, when
 // set, holds one flag per window of `win` rows (nwin per prompt,
@@ -135,9 +194,8 @@ SLS_DEV bool fm_tile_live(const FmJob& J, int b, int mb) {
   return false;
 }
 
-// Four consecutive features: one 16-byte store (float32), or one 8-byte
-// store of four bfloat16 values rounded to nearest even.
-SLS_DEV void store4(float* p, float4 o) { *reinterpret_cast<float4*>(p) = o; }
+// Four consecutive bfloat16 features, rounded to nearest even: one 8-byte
+// store.
 SLS_DEV void store4(uint16_t* p, float4 o) {
   const __nv_bfloat162 a = __floats2bfloat162_rn(o.x, o.y), b = __floats2bfloat162_rn(o.z, o.w);
   uint2 u;
@@ -150,7 +208,8 @@ SLS_DEV void store4(uint16_t* p, float4 o) {
 template <typename OT>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
-                      const __grid_constant__ CUtensorMap tmW, const float* __restrict__ bvec,
+                      const __grid_constant__ CUtensorMap tmW,
+                      const __grid_constant__ CUtensorMap tmPhi, const float* __restrict__ bvec,
                       OT* __restrict__ Phi, FmJob J, int D, int K, float scale, int* status) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES], tfull[2], tempty[2], done_bar;
@@ -277,7 +336,12 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
   } else {
     // ------------------------------ epilogue ----------------------------------
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    unsigned acc_it = 0;
+    // two 32 x 32 float32 staging blocks of this warp, 1024-byte aligned (the
+    // 128-byte swizzle repeats every eight rows of 128 bytes)
+    const uint32_t stg0 = smem_base + (uint32_t)(TC_STAGES * TC_STAGE_BYTES) +
+                          (uint32_t)((warp - 2) * 2 * TC_OUT_BYTES);
+    unsigned char* stg0p = smem + TC_STAGES * TC_STAGE_BYTES + (warp - 2) * 2 * TC_OUT_BYTES;
+    unsigned acc_it = 0, blk = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
       const int pb = tile / per_prompt, rem = tile % per_prompt;
       const int mb = rem / n_tiles, nb = rem % n_tiles;
@@ -290,21 +354,50 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       }
       tc_fence_after();
       const int row = mb * TC_BM + q * 32 + lane;
-      OT* out = Phi + ((int64_t)pb * J.rows + row) * D + (int64_t)nb * TC_BN;
       const float* bb = bvec + (size_t)nb * TC_BN;
-      for (int c0 = 0; c0 < TC_BN; c0 += 32) {
+      for (int c0 = 0; c0 < TC_BN; c0 += 32, ++blk) {
         uint32_t v[32];
         tc_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN + c0), v);
-        if (row < J.rows) {
+        float th[32];
+        float amax = 0.f;
 #pragma unroll
-          for (int e = 0; e < 32; e += 4) {
-            const float4 bq = __ldg(reinterpret_cast<const float4*>(bb + c0 + e));
-            float4 o;
-            o.x = scale * cosf(__uint_as_float(v[e + 0]) + bq.x);
-            o.y = scale * cosf(__uint_as_float(v[e + 1]) + bq.y);
-            o.z = scale * cosf(__uint_as_float(v[e + 2]) + bq.z);
-            o.w = scale * cosf(__uint_as_float(v[e + 3]) + bq.w);
-            store4(out + c0 + e, o);
+        for (int e = 0; e < 32; e += 4) {
+          const float4 bq = __ldg(reinterpret_cast<const float4*>(bb + c0 + e));
+          th[e + 0] = __uint_as_float(v[e + 0]) + bq.x;
+          th[e + 1] = __uint_as_float(v[e + 1]) + bq.y;
+          th[e + 2] = __uint_as_float(v[e + 2]) + bq.z;
+          th[e + 3] = __uint_as_float(v[e + 3]) + bq.w;
+          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(th[e]), fabsf(th[e + 1])),
+                                   fmaxf(fabsf(th[e + 2]), fabsf(th[e + 3]))));
+        }
+        if (__all_sync(0xffffffffu, amax <= RFF_COS_FAST_MAX)) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) th[e] = scale * rff_cos_fast(th[e]);
+        } else {
+          for (int e = 0; e < 32; ++e) th[e] = scale * rff_cos_wide(th[e]);
+        }
+        if constexpr (sizeof(OT) == 4) {
+          // row `lane` of the block: its eight 16-byte pieces at the swizzled
+          // positions (piece c of row l goes to c ^ (l mod 8))
+          const uint32_t sb = (blk & 1u) ? TC_OUT_BYTES : 0u;
+          if (lane == 0) bulk_wait_read_le1();  // the block's previous store has read it
+          __syncwarp();
+          unsigned char* rowp = stg0p + sb + lane * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            *reinterpret_cast<float4*>(rowp + ((c ^ (lane & 7)) << 4)) =
+                make_float4(th[4 * c], th[4 * c + 1], th[4 * c + 2], th[4 * c + 3]);
+          fence_async_smem();
+          __syncwarp();
+          // a block wholly past the prompt's last row is not stored at all
+          if (lane == 0 && mb * TC_BM + q * 32 < J.rows)
+            tma_store_3d(&tmPhi, stg0 + sb, nb * TC_BN + c0, mb * TC_BM + q * 32, pb);
+        } else {
+          if (row < J.rows) {
+            OT* out = Phi + ((int64_t)pb * J.rows + row) * D + (int64_t)nb * TC_BN + c0;
+#pragma unroll
+            for (int e = 0; e < 32; e += 4)
+              store4(out + e, make_float4(th[e], th[e + 1], th[e + 2], th[e + 3]));
           }
         }
       }
@@ -313,6 +406,9 @@ feature_map_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       if (lane == 0) mbar_arrive(&tempty[acc]);
       ++acc_it;
     }
+    // every tensor store of this warp has completed before the CTA exits
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
   }
   __syncthreads();
   if (warp == 1) {
@@ -356,6 +452,20 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// float32 output map: dims (D, rows, nb), 32 x 32 x 1 boxes, 128-byte
+// swizzle (one box row is 128 bytes)
+bool make_out_map(CUtensorMap* map, void* base, uint64_t D, uint64_t rows, uint64_t nb) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {D, rows, nb};
+  const cuuint64_t strides[2] = {D * 4, rows * D * 4};
+  const cuuint32_t box[3] = {32, 32, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int sm_count() {
   static int sms = 0;
   if (sms == 0) {
@@ -385,10 +495,17 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
   if (live && (nwin < 1 || win < 1)) return SLS_ERR_INVALID_ARG;
   if (((uintptr_t)X & 15) || ((uintptr_t)W & 15) || ((uintptr_t)b & 15) || ((uintptr_t)Phi & 15))
     return SLS_ERR_UNSUPPORTED;
-  CUtensorMap mx, mw;
+  CUtensorMap mx, mw, mp;
   if (!make_map(&mx, X, (uint64_t)map_rows, (uint64_t)d, (uint64_t)ldx, TC_BM))
     return SLS_ERR_UNSUPPORTED;
   if (!make_map(&mw, W, (uint64_t)D, (uint64_t)d, (uint64_t)d, TC_BN)) return SLS_ERR_UNSUPPORTED;
+  // float32 Phi as (feature, row, prompt): a block's rows past the prompt's
+  // last row fall outside the map and are not written
+  if (phi_bf16) {
+    memset(&mp, 0, sizeof(mp));
+  } else if (!make_out_map(&mp, Phi, (uint64_t)D, (uint64_t)rows, (uint64_t)nb)) {
+    return SLS_ERR_UNSUPPORTED;
+  }
   int* st = status;
   if (!st) SLS_CUDA_TRY(cudaGetSymbolAddress((void**)&st, g_fm_status));
   SLS_CUDA_TRY(cudaFuncSetAttribute(feature_map_tc_kernel<float>,
@@ -401,10 +518,10 @@ int launch_feature_map_tc_batched(const void* X, int64_t nb, int64_t rows, int64
   FmJob J{(int)nb, (int)rows, (int)x_stride, live, nwin, win};
   if (phi_bf16)
     feature_map_tc_kernel<uint16_t><<<grid, TC_THREADS, TC_SMEM, stream>>>(
-        mx, mw, b, (uint16_t*)Phi, J, D, d, scale, st);
+        mx, mw, mp, b, (uint16_t*)Phi, J, D, d, scale, st);
   else
-    feature_map_tc_kernel<float><<<grid, TC_THREADS, TC_SMEM, stream>>>(mx, mw, b, (float*)Phi, J,
-                                                                      D, d, scale, st);
+    feature_map_tc_kernel<float><<<grid, TC_THREADS, TC_SMEM, stream>>>(mx, mw, mp, b, (float*)Phi,
+                                                                      J, D, d, scale, st);
   SLS_LAUNCH_CHECK();
   return SLS_OK;
 }
