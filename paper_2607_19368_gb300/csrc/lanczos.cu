@@ -534,9 +534,13 @@ int launch_lanczos(const LanczosBatch& bt, void* scratch, size_t scratch_bytes, 
       break;
     }
   }
-  // two chunks per team in flight at least, and room for the pass ends'
-  // scratch in the ring
-  if (stages < 2 * teams) return SLS_ERR_UNSUPPORTED;
+  // Room for the pass ends' scratch in the ring, and at least 2 teams + 2
+  // stages: a team refills the slots of its previous pair after the first
+  // barrier of its current pair, so chunk c is issued after the first barrier
+  // of the pair `teams` pairs after the one holding chunk c - S; with fewer
+  // stages (or 2 teams + 1) a team would wait for a chunk that only its own
+  // later refill issues.
+  if (stages < 2 * teams + 2) return SLS_ERR_UNSUPPORTED;
   if ((size_t)stages * R.stage < lz_pass_end_bytes(gpt, bt.r, teams)) return SLS_ERR_UNSUPPORTED;
   const size_t smem = (size_t)stages * R.stage + lz_smem_other(bt.D, bt.r, rows_cap, teams, stages);
   const int kt = (bt.r <= 32) ? 1 : (bt.r <= 64) ? 2 : 4;  // 32-wide tiles of k < r

@@ -882,8 +882,14 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     // alternate direction), issued once the ring is idle, chunk t by lane 0
     // of warp t mod NCW: the thread that issues a bulk copy is held for a few
     // hundred cycles, so the copies are spread over warps.
+    //
+    // No chunk is issued once a wait of this CTA has given up (s_err, set
+    // before the team or CTA barrier that precedes every issue): a slot then
+    // never receives a chunk whose predecessor in the slot was not seen to
+    // land, so the phase parity of each slot's mbarrier stays that of its
+    // last chunk number and drain() waits for every copy still in flight.
     auto issue_pass_head = [&](int pass) {
-      if (lane == 0) {
+      if (lane == 0 && !s_err) {
         const int m = min(S, nch);
         for (int t = warp; t < m; t += NCW)
           issue_chunk<PT>(base + (unsigned)t, ring_slot(base + (unsigned)t, S),
@@ -899,7 +905,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
     // both).
     auto refill_half = [&](int pass, int t0, RingPos q0) {
       const int h = tw - (LZ_CW - 2);
-      if (t0 < 0 || lane != 0 || h < 0) return;
+      if (t0 < 0 || lane != 0 || h < 0 || s_err) return;
       const int t = t0 + h + S;
       if (t >= nch) return;
       SLS_DBG_CHECK(status, t >= 0 && ring_adv(q0, h, S).slot < S);
@@ -1383,7 +1389,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           sweepA_chunk<GPT, false>(chunk, nr, D, kc * cr, tt, zps, ah, al, &mx);
           // every warp is done with this chunk: refill its slot
           named_sync(BAR_ALL, NCT);
-          if (tid == 0 && t + S < nch)
+          if (tid == 0 && t + S < nch && !s_err)
             issue_chunk<PT>(base + (unsigned)(t + S), slot, fwd ? t + S : nch - 1 - (t + S), cr,
                             nrows, D, ldq, stage, phib, ring, fullb, slot_cnt, Phis, Qs, pol);
         }
