@@ -617,10 +617,11 @@ SLS_DEV void store_col_partials(const f32x2_t (&ah)[GPT][2], const f32x2_t (&al)
         upk2(al[q][0], l0, l1);
         upk2(ah[q][1], h2, h3);
         upk2(al[q][1], l2, l3);
-        d[4 * cg + 0] = f2(df_norm(h0, l0));
-        d[4 * cg + 1] = f2(df_norm(h1, l1));
-        d[4 * cg + 2] = f2(df_norm(h2, l2));
-        d[4 * cg + 3] = f2(df_norm(h3, l3));
+        const dfloat n0 = df_norm(h0, l0), n1 = df_norm(h1, l1);
+        const dfloat n2 = df_norm(h2, l2), n3 = df_norm(h3, l3);
+        float4* d4 = reinterpret_cast<float4*>(d + 4 * cg);
+        d4[0] = make_float4(n0.hi, n0.lo, n1.hi, n1.lo);
+        d4[1] = make_float4(n2.hi, n2.lo, n3.hi, n3.lo);
       }
     }
   }
@@ -652,10 +653,20 @@ SLS_DEV bool slice_last_warp_idle(int ncol) {
   return (NCW - 1) * (32 / G) >= ncol;
 }
 
+// c itself (cs[k] = the group sum accj[k], k < j) is loaded by warp cwarp:
+// after it has issued its first batch when it sums columns, so that both
+// round trips to L2 overlap, else before it reaches the named barrier.
+template <int NCW>
+SLS_DEV void load_c(float2* __restrict__ cs, const double* __restrict__ accj, int j) {
+  const int lane = threadIdx.x & 31;
+  for (int k = lane; k < j; k += 32) cs[k] = f2(df_from_double(accj[k]));
+}
+
 template <int NCW>
 SLS_DEV dfloat slice_columns(const float2* __restrict__ wpart, const float2* __restrict__ Wm,
-                             float2* __restrict__ wred, const float2* __restrict__ cs, int g,
-                             int D, int j, int cbeg, int cend, bool& synced) {
+                             float2* __restrict__ wred, float2* __restrict__ cs,
+                             const double* __restrict__ accj, int cwarp, int g, int D, int j,
+                             int cbeg, int cend, bool& synced) {
   constexpr int NCT = NCW * 32;
   constexpr int BATCH = 8;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -677,6 +688,7 @@ SLS_DEV dfloat slice_columns(const float2* __restrict__ wpart, const float2* __r
       pv[u] = (valid && b < g) ? wpart[(size_t)b * D + c] : make_float2(0.f, 0.f);
       wv[u] = (valid && b < j) ? Wm[(size_t)b * D + c] : make_float2(0.f, 0.f);
     }
+    if (!synced && warp == cwarp) load_c<NCW>(cs, accj, j);
     dfloat s = df_make(0.f, 0.f);
 #pragma unroll
     for (int u = 0; u < BATCH; ++u) s = df_add_fast(s, dfv(pv[u]));
@@ -719,6 +731,7 @@ SLS_DEV dfloat slice_columns(const float2* __restrict__ wpart, const float2* __r
       dot2_acc_df(sq.hi, sq.lo, s, s);
     }
   }
+  if (!synced && warp == cwarp) load_c<NCW>(cs, accj, j);  // a warp without columns
   return sq;
 }
 
@@ -967,15 +980,23 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         store_col_partials<GPT>(ah, al, P, C4, D, tt, wpart + (size_t)rank * D, red, bar_team,
                                 LZ_CT);
       }
-      for (int k = tid; k < K; k += NCT) {
+      // coefficient k: the NCW warp partials summed by four lanes (each over
+      // every fourth warp) and a butterfly over the four
+      constexpr int LPK = 4;
+      for (int k0 = 0; k0 < K; k0 += NCT / LPK) {
+        const int k = k0 + tid / LPK, part = tid % LPK;
         dfloat s = df_make(0.f, 0.f);
-        for (int w = 0; w < NCW; ++w) s = df_add(s, dfv(cw[(size_t)w * (r + 1) + k]));
-        red_add_f64(accn + k, df_to_double(s));
+        if (k < K)
+          for (int w = part; w < NCW; w += LPK) s = df_add(s, dfv(cw[(size_t)w * (r + 1) + k]));
+        s = df_add_fast(s, shfl_xor_df(s, 1));
+        s = df_add_fast(s, shfl_xor_df(s, 2));
+        if (part == 0 && k < K) red_add_f64(accn + k, df_to_double(s));
       }
-      if (tid == 0) {
-        dfloat t = df_make(0.f, 0.f);
-        for (int w = 0; w < NCW; ++w) t = df_add(t, dfv(tmpw[w]));
-        red_add_f64(accn + r + 1, df_to_double(t));
+      if (warp == NCW - 1) {
+        dfloat t = (lane < NCW) ? dfv(tmpw[lane]) : df_make(0.f, 0.f);
+#pragma unroll
+        for (int o = 1; o < NCW; o <<= 1) t = df_add_fast(t, shfl_xor_df(t, o));
+        if (lane == 0) red_add_f64(accn + r + 1, df_to_double(t));
       }
       // the column of Q written in this pass reaches the bulk reads of the
       // next pass (async proxy)
@@ -1074,16 +1095,16 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
       // c_k w_k with w_k = Phi^T q_k kept in Wm.  The group sums of the other
       // parity were read in the previous step by every CTA (all of them have
       // passed barrier 1 since): the first CTA clears them for the next step.
-      if (warp == 0) {
-        for (int k = lane; k < j; k += 32) cs[k] = f2(df_from_double(accj[k]));
-      }
       if (rank == 0) {
         double* accz = acc + (size_t)((gstep + 1u) & 1u) * accs;
         for (int k = tid; k < accs; k += NCT) accz[k] = 0.0;
       }
       {
+        // c is loaded by the last warp when it sums no column (it waits for
+        // beta there anyway), else by warp 0
         bool synced = false;
-        dfloat sq = slice_columns<NCW>(wpart, Wm, wred, cs, g, D, j, cbeg, cend, synced);
+        dfloat sq = slice_columns<NCW>(wpart, Wm, wred, cs, accj, beta_early ? NCW - 1 : 0, g, D,
+                                       j, cbeg, cend, synced);
         if (!synced) named_sync(BAR_ALL, NCT);
         if (beta_early && warp == NCW - 1) beta_phase();
         sq = df_norm(sq.hi, sq.lo);
@@ -1091,10 +1112,12 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         for (int o = 16; o > 0; o >>= 1) sq = df_add_fast(sq, shfl_xor_df(sq, o));
         if (lane == 0) tmpw[warp] = f2(sq);
         named_sync(BAR_ALL, NCT);
-        if (tid == 0) {
-          dfloat s = df_make(0.f, 0.f);
-          for (int w = 0; w < NCW; ++w) s = df_add(s, dfv(tmpw[w]));
-          red_add_f64(const_cast<double*>(accj) + r + 2, df_to_double(s));
+        if (warp == 0) {
+          // the NCW warp sums by a butterfly over the first NCW lanes
+          dfloat t = (lane < NCW) ? dfv(tmpw[lane]) : df_make(0.f, 0.f);
+#pragma unroll
+          for (int o = 1; o < NCW; o <<= 1) t = df_add_fast(t, shfl_xor_df(t, o));
+          if (lane == 0) red_add_f64(const_cast<double*>(accj) + r + 2, df_to_double(t));
         }
       }
       if (!group_sync_named(bar, lgen, status, &sflag, &s_err, BAR_ALL, NCT)) {
