@@ -1275,7 +1275,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
           // (it feeds only the row work after them)
           dfloat qjv[RPW];
           float2 qpv[RPW];
-          if (fullD && nr0 == TCR && nr1 == TCR && 2 * TCR >= LZ_CW) {
+          if (fullD && nr0 == TCR && nr1 == TCR && 2 * TCR == LZ_CW) {
             // steady state, every warp owns one row of the pair: q_j of that
             // row and the row dots in one block, so that the warp reduction
             // of q_j interleaves with the sweep's arithmetic (measured 2.9%
