@@ -93,6 +93,31 @@ def test_feature_map_tc_partial_k_tile(sls, N, d, D):
     assert np.all(np.abs(phi - want) <= tol)
 
 
+def test_feature_map_tc_cosine_ranges(sls):
+    """The tensor-core epilogue's cosine over a wide range of arguments: rows
+    scaled so that theta = x.w + b runs from about 1e-3 to beyond 8192 (where
+    a 32-column block falls back to the library cosine), and rows of zeros
+    (theta = b exactly).  Every feature within the float32 bound of the
+    oracle's Eq. rff_map."""
+    g = np.random.default_rng(7)
+    N, d, D = 384, 64, 512
+    X = g.standard_normal((N, d)) / math.sqrt(d)
+    scale = np.repeat([1e-3, 1.0, 30.0, 400.0, 20000.0, 0.0], N // 6)
+    X = X * scale[:, None]
+    Xb = WL.f32_to_bf16_bits(X.astype(np.float32))
+    Wb = WL.f32_to_bf16_bits((g.standard_normal((D, d)) * d ** -0.25).astype(np.float32))
+    b = (g.random(D) * 2 * math.pi).astype(np.float32)
+    X64, W64 = widen(Xb, "bf16"), widen(Wb, "bf16")
+    theta = X64 @ W64.T + b.astype(np.float64)
+    assert np.max(np.abs(theta)) > 8192.0 and np.min(np.abs(theta)) < 1.0
+    phi = sls.feature_map(to_torch_x(Xb, "bf16"), to_torch_x(Wb, "bf16"),
+                          torch.from_numpy(b).cuda()).cpu().numpy().astype(np.float64)
+    want = O.rff_features(X64, W64, b)
+    tol = feature_tolerance(X64, W64, b.astype(np.float64))
+    err = np.abs(phi - want)
+    assert np.all(err <= tol), float(np.max(err / tol))
+
+
 def test_feature_map_batched_live_windows(sls):
     """One launch over a batch of prompts (Sec. 3.2) that computes only the
     row tiles touching a live window (Sec. 3.6): computed rows match the
