@@ -200,6 +200,15 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
 // partial-pivoting LU of T - shift I in double-float, two iterations, each
 // followed by modified Gram-Schmidt against the cluster members already
 // found.  One thread; the work arrays (n entries each) belong to the caller.
+// The recurrences carry their running values in registers (the factorisation
+// the current pivot row, the solves the last one or two entries), so a step's
+// dependent chain holds no memory access, and the back substitution
+// multiplies by the pivots' reciprocals, formed during the factorisation off
+// that chain; sums over n run as four interleaved partial sums.
+SLS_DEV dfloat sum4_df(dfloat (&acc)[4]) {
+  return df_add(df_add(acc[0], acc[1]), df_add(acc[2], acc[3]));
+}
+
 SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int last,
                             float2* __restrict__ d, float2* __restrict__ du,
                             float2* __restrict__ du2, float2* __restrict__ dl,
@@ -216,47 +225,49 @@ SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int
   const double sc = ldexp(1.0, -ex);
   const double pert = 0x1p-44 * tnorm * sc;
   const dfloat pert_df = df_from_double(pert);
+  const dfloat one = df_make(1.f, 0.f);
   for (int mm = first; mm <= last; ++mm) {
     // distinct shifts inside a cluster
     const dfloat shift = df_from_double((th[mm] - (double)(mm - first) * 4.0 * (pert / sc)) * sc);
+    // the diagonal of T - shift I (d) and the off-diagonal (dl), unfactored
     for (int i = 0; i < n; ++i) {
       d[i] = f2(df_sub(df_from_double(a[i] * sc), shift));
-      if (i < n - 1) {
-        du[i] = f2(df_from_double(b[i] * sc));
-        dl[i] = du[i];
-      }
-      du2[i] = make_float2(0.f, 0.f);
+      if (i < n - 1) dl[i] = f2(df_from_double(b[i] * sc));
     }
     if (n == 1) {
       y[0] = make_float2(1.f, 0.f);
     } else {
-      // LU with partial pivoting of T - shift I
+      // LU with partial pivoting of T - shift I; cd, cu: the current pivot
+      // row's diagonal and superdiagonal entries as the elimination has left
+      // them.  d[i] then holds the reciprocal of pivot i.
+      dfloat cd = dfv(d[0]), cu = dfv(dl[0]);
       for (int i = 0; i < n - 1; ++i) {
-        dfloat di = dfv(d[i]);
         const dfloat li = dfv(dl[i]);
-        if (fabsf(di.hi) >= fabsf(li.hi)) {
-          if (di.hi == 0.f) di = pert_df;
-          const dfloat f = df_div(li, di);
-          d[i] = f2(di);
+        const dfloat dn0 = dfv(d[i + 1]);
+        const dfloat un0 = (i < n - 2) ? dfv(dl[i + 1]) : df_make(0.f, 0.f);
+        if (fabsf(cd.hi) >= fabsf(li.hi)) {
+          if (cd.hi == 0.f) cd = pert_df;
+          const dfloat f = df_div(li, cd);
+          d[i] = f2(df_div(one, cd));
           dl[i] = f2(f);
-          d[i + 1] = f2(df_sub(dfv(d[i + 1]), df_mul(f, dfv(du[i]))));
+          du[i] = f2(cu);
+          du2[i] = make_float2(0.f, 0.f);
+          cd = df_sub(dn0, df_mul(f, cu));
+          cu = un0;
           piv[i] = 0;
         } else {
-          const dfloat f = df_div(di, li);
-          const dfloat dn = dfv(d[i + 1]);
-          d[i] = f2(li);
+          const dfloat f = df_div(cd, li);
+          d[i] = f2(df_div(one, li));
           dl[i] = f2(f);
-          const dfloat tmp = dfv(du[i]);
-          du[i] = f2(dn);
-          d[i + 1] = f2(df_sub(tmp, df_mul(f, dn)));
-          if (i < n - 2) {
-            du2[i] = du[i + 1];
-            du[i + 1] = f2(df_neg(df_mul(f, dfv(du[i + 1]))));
-          }
+          du[i] = f2(dn0);
+          du2[i] = f2(un0);
+          cd = df_sub(cu, df_mul(f, dn0));
+          cu = df_neg(df_mul(f, un0));
           piv[i] = 1;
         }
       }
-      if (d[n - 1].x == 0.f) d[n - 1] = f2(pert_df);
+      if (cd.hi == 0.f) cd = pert_df;
+      d[n - 1] = f2(df_div(one, cd));
       // deterministic start vector
       for (int i = 0; i < n; ++i) {
         unsigned h = (unsigned)(i + 1) * 2654435761u ^ (unsigned)(mm + 7) * 40503u;
@@ -266,22 +277,31 @@ SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int
         y[i] = make_float2(0.5f + (float)(h & 0xffffu) / 65536.f, 0.f);
       }
       for (int it = 0; it < 2; ++it) {
+        // forward substitution with the row interchanges; cy: the running y[i]
+        dfloat cy = dfv(y[0]);
         for (int i = 0; i < n - 1; ++i) {
+          const dfloat yn = dfv(y[i + 1]);
+          const dfloat li = dfv(dl[i]);
           if (!piv[i]) {
-            y[i + 1] = f2(df_sub(dfv(y[i + 1]), df_mul(dfv(dl[i]), dfv(y[i]))));
+            y[i] = f2(cy);
+            cy = df_sub(yn, df_mul(li, cy));
           } else {
-            const dfloat t = dfv(y[i]);
-            y[i] = y[i + 1];
-            y[i + 1] = f2(df_sub(t, df_mul(dfv(dl[i]), dfv(y[i]))));
+            y[i] = f2(yn);
+            cy = df_sub(cy, df_mul(li, yn));
           }
         }
-        y[n - 1] = f2(df_div(dfv(y[n - 1]), dfv(d[n - 1])));
-        y[n - 2] = f2(df_div(df_sub(dfv(y[n - 2]), df_mul(dfv(du[n - 2]), dfv(y[n - 1]))),
-                             dfv(d[n - 2])));
+        // back substitution; c1, c2: y[i + 1], y[i + 2]
+        dfloat c1 = df_mul(cy, dfv(d[n - 1]));
+        y[n - 1] = f2(c1);
+        dfloat c2 = c1;
+        c1 = df_mul(df_sub(dfv(y[n - 2]), df_mul(dfv(du[n - 2]), c1)), dfv(d[n - 2]));
+        y[n - 2] = f2(c1);
         for (int i = n - 3; i >= 0; --i) {
-          const dfloat t = df_sub(df_sub(dfv(y[i]), df_mul(dfv(du[i]), dfv(y[i + 1]))),
-                                  df_mul(dfv(du2[i]), dfv(y[i + 2])));
-          y[i] = f2(df_div(t, dfv(d[i])));
+          const dfloat t = df_sub(df_sub(dfv(y[i]), df_mul(dfv(du[i]), c1)),
+                                  df_mul(dfv(du2[i]), c2));
+          c2 = c1;
+          c1 = df_mul(t, dfv(d[i]));
+          y[i] = f2(c1);
         }
         // keep the iterate in range: divide by its largest entry (a power of two)
         float ymax = 0.f;
@@ -294,15 +314,19 @@ SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int
         }
         // orthogonalise against the cluster members found so far
         for (int pm = first; pm < mm; ++pm) {
-          dfloat dot = df_make(0.f, 0.f);
+          dfloat acc[4] = {df_make(0.f, 0.f), df_make(0.f, 0.f), df_make(0.f, 0.f),
+                           df_make(0.f, 0.f)};
           for (int i = 0; i < n; ++i)
-            dot = df_add(dot, df_mul(df_from_double(S[(size_t)i * r + pm]), dfv(y[i])));
+            acc[i & 3] = df_add(acc[i & 3],
+                                df_mul(df_from_double(S[(size_t)i * r + pm]), dfv(y[i])));
+          const dfloat dot = sum4_df(acc);
           for (int i = 0; i < n; ++i)
             y[i] = f2(df_sub(dfv(y[i]), df_mul(dot, df_from_double(S[(size_t)i * r + pm]))));
         }
-        dfloat nr2 = df_make(0.f, 0.f);
-        for (int i = 0; i < n; ++i) nr2 = df_add(nr2, df_mul(dfv(y[i]), dfv(y[i])));
-        const double nr = sqrt(df_to_double(nr2));
+        dfloat acc[4] = {df_make(0.f, 0.f), df_make(0.f, 0.f), df_make(0.f, 0.f),
+                         df_make(0.f, 0.f)};
+        for (int i = 0; i < n; ++i) acc[i & 3] = df_add(acc[i & 3], df_mul(dfv(y[i]), dfv(y[i])));
+        const double nr = sqrt(df_to_double(sum4_df(acc)));
         if (!(nr > 0.0) || !isfinite(nr)) {
           for (int i = 0; i < n; ++i) y[i] = make_float2((i == mm) ? 1.f : 0.f, 0.f);
         } else {
