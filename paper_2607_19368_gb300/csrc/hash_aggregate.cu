@@ -1608,6 +1608,7 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
     // Lane j holds the descriptor of local item kb + j; the member ids of the
     // batch are fetched 32 rows at a time, one chunk ahead of the copies.
     const uint64_t pol = l2_policy_evict_first();
+    const int GP = S / 2 < 8 ? (S / 2 < 1 ? 1 : S / 2) : 8;  // rows issued together
     unsigned issued = 0;
     bool ok = true;
     int kb = 0;
@@ -1628,10 +1629,16 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
         int nrid = 0, nrj = 0, nrs = 0;
         if (f0 + 32 < nrows) agr_fetch_row(perm, pre, nrows, cd.off, f0 + 32, lane, nrid, nrj, nrs);
         const int cnt = min(32, nrows - f0);
-        for (int l = 0; l < cnt; ++l) {
-          const int row = __shfl_sync(0xffffffffu, rid, l);
-          const int j = __shfl_sync(0xffffffffu, rj, l);
-          const int s = __shfl_sync(0xffffffffu, rs, l);
+        // rows g0 .. g0 + GP - 1 of the batch go out together, one per lane:
+        // each lane waits for its own ring stage, then issues its copy (a
+        // thread issuing a bulk copy is held for a few hundred cycles, so
+        // one lane issuing every row made the producer the bottleneck)
+        for (int g0 = 0; g0 < cnt; g0 += GP) {
+          const int gn = min(GP, cnt - g0);
+          const bool act = lane < gn;
+          const int row = __shfl_sync(0xffffffffu, rid, (g0 + lane) & 31);
+          const int j = __shfl_sync(0xffffffffu, rj, (g0 + lane) & 31);
+          const int s = __shfl_sync(0xffffffffu, rs, (g0 + lane) & 31);
           AggDesc D;
           D.m = __shfl_sync(0xffffffffu, cd.m, j);
           D.c = __shfl_sync(0xffffffffu, cd.c, j);
@@ -1639,32 +1646,35 @@ agg_ring_kernel(const T* __restrict__ X, int d, int64_t ldx, const int* __restri
           D.len = __shfl_sync(0xffffffffu, cd.len, j);
           D.ps = __shfl_sync(0xffffffffu, cd.ps, j);
           D.pad0 = D.pad1 = D.pad2 = 0;
-          if (lane == 0) {
-            const int st = (int)(issued % (unsigned)S);
-            const unsigned par = (issued / (unsigned)S) & 1u;
-            if (!agr_wait<false>(&emptyb[st], par ^ 1u, &s_abort)) {
-              ok = false;
+          const unsigned mine = issued + (unsigned)lane;
+          const int st = (int)(mine % (unsigned)S);
+          const unsigned par = (mine / (unsigned)S) & 1u;
+          bool w_ok = true;
+          if (act) w_ok = agr_wait<false>(&emptyb[st], par ^ 1u, &s_abort);
+          if (!__all_sync(0xffffffffu, w_ok)) {
+            ok = false;
+            if (lane == 0) {
               s_abort = 1;
               atomicExch(status, SLS_ERR_TIMEOUT);
-            } else {
-              if (s == 0) dring[(kb + j) % DQ] = D;
-              unsigned char* dst = agr_smem + (size_t)st * stage_bytes;
-              mbar_expect_tx(&fullb[st], row_bytes);
-              int64_t src_row = row;
-#ifdef SLS_DEBUG
-              // a member row outside the token set is not fetched: the stage
-              // gets row 0 instead and the status records SLS_ERR_BOUNDS
-              if (!(row >= 0 && (int64_t)row < ntot)) {
-                atomicExch(status, SLS_ERR_BOUNDS);
-                src_row = 0;
-              }
-#endif
-              bulk_g2s(dst, X + src_row * ldx, row_bytes, &fullb[st], pol);
             }
+            break;
           }
-          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-          if (!ok) break;
-          ++issued;
+          if (act) {
+            if (s == 0) dring[(kb + j) % DQ] = D;
+            unsigned char* dst = agr_smem + (size_t)st * stage_bytes;
+            mbar_expect_tx(&fullb[st], row_bytes);
+            int64_t src_row = row;
+#ifdef SLS_DEBUG
+            // a member row outside the token set is not fetched: the stage
+            // gets row 0 instead and the status records SLS_ERR_BOUNDS
+            if (!(row >= 0 && (int64_t)row < ntot)) {
+              atomicExch(status, SLS_ERR_BOUNDS);
+              src_row = 0;
+            }
+#endif
+            bulk_g2s(dst, X + src_row * ldx, row_bytes, &fullb[st], pol);
+          }
+          issued += (unsigned)gn;
         }
         rid = nrid;
         rj = nrj;
