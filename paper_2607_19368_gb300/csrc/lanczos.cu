@@ -209,20 +209,40 @@ SLS_DEV dfloat sum4_df(dfloat (&acc)[4]) {
   return df_add(df_add(acc[0], acc[1]), df_add(acc[2], acc[3]));
 }
 
+// A power-of-two scale of T for problem p (the eigenvectors do not change):
+// 1 / 2^ceil(log2 |T|), |T| from the extreme Ritz values.
+SLS_DEV double eig_scale(const double* th, int n, double* tnorm_out) {
+  const double tnorm = fmax(fabs(th[0]), fabs(th[n - 1])) + DBL_MIN;
+  int ex = 0;
+  frexp(tnorm, &ex);
+  *tnorm_out = tnorm;
+  return ldexp(1.0, -ex);
+}
+
+// The scaled diagonal sa[i] = alpha_i sc and off-diagonal sb[i] = beta_i sc of
+// problem p as double-float, entries i = t, t + nt, ... for the nt calling
+// threads (t = their index): every eigenvector of the problem starts from
+// them, and the float64 products and splits, whose dependent latency is long
+// on this part, run once per problem and in parallel.
+SLS_DEV void eig_scaled_T(const LanczosBatch& bt, int p, int n, double sc, int t, int nt,
+                          float2* __restrict__ sa, float2* __restrict__ sb) {
+  const double* a = bt.alpha + (size_t)p * bt.r;
+  const double* b = bt.beta + (size_t)p * bt.r;
+  for (int i = t; i < n; i += nt) {
+    sa[i] = f2(df_from_double(a[i] * sc));
+    if (i < n - 1) sb[i] = f2(df_from_double(b[i] * sc));
+  }
+}
+
 SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int last,
-                            float2* __restrict__ d, float2* __restrict__ du,
-                            float2* __restrict__ du2, float2* __restrict__ dl,
-                            float2* __restrict__ y, unsigned char* __restrict__ piv) {
+                            double sc, double tnorm, const float2* __restrict__ sa,
+                            const float2* __restrict__ sb, float2* __restrict__ d,
+                            float2* __restrict__ du, float2* __restrict__ du2,
+                            float2* __restrict__ dl, float2* __restrict__ y,
+                            unsigned char* __restrict__ piv) {
   const int r = bt.r;
   double* S = bt.S + (size_t)p * r * r;
   const double* th = bt.theta + (size_t)p * r;
-  const double* a = bt.alpha + (size_t)p * r;
-  const double* b = bt.beta + (size_t)p * r;
-  const double tnorm = fmax(fabs(th[0]), fabs(th[n - 1])) + DBL_MIN;
-  // a power-of-two scale of T (the eigenvectors do not change)
-  int ex = 0;
-  frexp(tnorm, &ex);
-  const double sc = ldexp(1.0, -ex);
   const double pert = 0x1p-44 * tnorm * sc;
   const dfloat pert_df = df_from_double(pert);
   const dfloat one = df_make(1.f, 0.f);
@@ -231,8 +251,8 @@ SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int
     const dfloat shift = df_from_double((th[mm] - (double)(mm - first) * 4.0 * (pert / sc)) * sc);
     // the diagonal of T - shift I (d) and the off-diagonal (dl), unfactored
     for (int i = 0; i < n; ++i) {
-      d[i] = f2(df_sub(df_from_double(a[i] * sc), shift));
-      if (i < n - 1) dl[i] = f2(df_from_double(b[i] * sc));
+      d[i] = f2(df_sub(dfv(sa[i]), shift));
+      if (i < n - 1) dl[i] = sb[i];
     }
     if (n == 1) {
       y[0] = make_float2(1.f, 0.f);
@@ -336,6 +356,7 @@ SLS_DEV void eigvec_cluster(const LanczosBatch& bt, int p, int n, int first, int
       }
     }
     const double sg = (y[0].x < 0.f) ? -1.0 : 1.0;
+#pragma unroll 4
     for (int i = 0; i < n; ++i) S[(size_t)i * r + mm] = sg * df_to_double(dfv(y[i]));
   }
 }
@@ -356,7 +377,7 @@ SLS_DEV void eig_cluster(const double* th, int n, int m, int& first, int& last) 
 __global__ void __launch_bounds__(32)
 tridiag_eigvecs_kernel(LanczosBatch bt) {
   __shared__ float2 d[SLS_MAX_R], du[SLS_MAX_R], du2[SLS_MAX_R], dl[SLS_MAX_R];
-  __shared__ float2 y[SLS_MAX_R];
+  __shared__ float2 y[SLS_MAX_R], sa[SLS_MAX_R], sb[SLS_MAX_R];
   __shared__ unsigned char piv[SLS_MAX_R];
   const int m = blockIdx.x, p = blockIdx.y, lane = threadIdx.x;
   int nprob = bt.nprob_max;
@@ -374,8 +395,12 @@ tridiag_eigvecs_kernel(LanczosBatch bt) {
   if (first != m) return;  // another CTA (the first member of this cluster) writes this column
   for (int k = lane + n; k < r; k += 32)
     for (int mm = first; mm <= last; ++mm) S[(size_t)k * r + mm] = 0.0;
+  double tnorm;
+  const double sc = eig_scale(bt.theta + (size_t)p * r, n, &tnorm);
+  eig_scaled_T(bt, p, n, sc, lane, 32, sa, sb);
+  __syncwarp();
   if (lane != 0) return;
-  eigvec_cluster(bt, p, n, first, last, d, du, du2, dl, y, piv);
+  eigvec_cluster(bt, p, n, first, last, sc, tnorm, sa, sb, d, du, du2, dl, y, piv);
 }
 
 // Small problems (r <= 32): one warp per problem, one lane per Ritz value;
@@ -399,13 +424,20 @@ tridiag_eigvecs_warp_kernel(LanczosBatch bt) {
     const int i = e / r, m = e % r;
     if (i >= n || m >= n) S[e] = 0.0;
   }
+  __shared__ float2 sa[EIGW_WARPS][EIGW_MAXR], sb[EIGW_WARPS][EIGW_MAXR];
+  double tnorm = 1.0, sc = 1.0;
+  if (n > 0) {
+    sc = eig_scale(bt.theta + (size_t)p * r, n, &tnorm);
+    eig_scaled_T(bt, p, n, sc, lane, 32, sa[warp], sb[warp]);
+  }
+  __syncwarp();
   if (lane >= n) return;
   int first, last;
   eig_cluster(bt.theta + (size_t)p * r, n, lane, first, last);
   if (first != lane) return;
   float2 d[EIGW_MAXR], du[EIGW_MAXR], du2[EIGW_MAXR], dl[EIGW_MAXR], y[EIGW_MAXR];
   unsigned char piv[EIGW_MAXR];
-  eigvec_cluster(bt, p, n, first, last, d, du, du2, dl, y, piv);
+  eigvec_cluster(bt, p, n, first, last, sc, tnorm, sa[warp], sb[warp], d, du, du2, dl, y, piv);
 }
 
 // ----------------------------------------------------------------------------
