@@ -785,6 +785,7 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
   __shared__ float2 tmpw[NCW];
   __shared__ float s_red1[NCW];  // per-warp max |Phi| (offset bounds)
   __shared__ double shd[4];
+  __shared__ float2 sdf[3];  // 1 / beta, alpha, beta of the step as double-float
   __shared__ int sflag, sbreak;
   __shared__ volatile unsigned slot_cnt[RING_MAX_STAGES];  // last chunk issued per slot
   __shared__ volatile int s_err;      // a wait of this CTA gave up
@@ -1149,6 +1150,11 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         shd[1] = e_brk ? 0.0 : e_inv;
         shd[2] = a;
         shd[3] = (j > 0) ? e_bnew : 0.0;
+        // converted once here: float64 runs at a small fraction of the
+        // float32 rate on this part, and every thread needs these
+        sdf[0] = f2(df_from_double(shd[1]));
+        sdf[1] = f2(df_from_double(a));
+        sdf[2] = f2(df_from_double(shd[3]));
         sbreak = e_brk;
       }
       named_sync(BAR_ALL, NCT);
@@ -1156,10 +1162,10 @@ lanczos_kernel(LanczosBatch bt, char* scratch, size_t gstride, int g, int ngroup
         reff = j;
         break;
       }
-      invb_df = df_from_double(shd[1]);
+      invb_df = dfv(sdf[0]);
       alpha_prev = shd[2];
-      alpha_df = df_from_double(shd[2]);
-      beta_df = df_from_double(shd[3]);
+      alpha_df = dfv(sdf[1]);
+      beta_df = dfv(sdf[2]);
       if (j == 0) {
 #pragma unroll
         for (int w = 0; w < NCW; ++w) phimax = fmaxf(phimax, s_red1[w]);
