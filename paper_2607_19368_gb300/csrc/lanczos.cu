@@ -32,13 +32,14 @@ SLS_DEV int reff_clamped(const LanczosBatch& bt, int p) {
 // Ritz values of few problems: one CTA per eigenvalue, 256 shifts per round
 // (fewer, longer rounds: the faster form when the launch has few eigenvalues)
 constexpr int EIG_THREADS = 256;  // shifts per multisection round
-constexpr double kInvShifts = 1.0 / (double)(EIG_THREADS + 1);
+constexpr float kInvShiftsF = 1.0f / (float)(EIG_THREADS + 1);
 
 __global__ void __launch_bounds__(EIG_THREADS)
 tridiag_eigvals_cta_kernel(LanczosBatch bt) {
   __shared__ float2 sa[SLS_MAX_R], sb2[SLS_MAX_R];
   __shared__ int s_first[EIG_THREADS / 32];
-  __shared__ double s_lo, s_hi, s_sc;
+  __shared__ double s_sc;
+  __shared__ float2 s_lo, s_hi;  // the interval, double-float
   const int m = blockIdx.x, p = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int nprob = bt.nprob_max;
   if (bt.nprob_dev) nprob = min(nprob, *bt.nprob_dev);
@@ -73,8 +74,8 @@ tridiag_eigvals_cta_kernel(LanczosBatch bt) {
       const double sc = ldexp(1.0, -ex);  // exact scaling
       double lo = glo * sc, hi = ghi * sc;
       const double pad = 0x1p-40 * fmax(fabs(lo), fabs(hi)) + 0x1p-100;
-      s_lo = lo - pad;
-      s_hi = hi + pad;
+      s_lo = f2(df_from_double(lo - pad));
+      s_hi = f2(df_from_double(hi + pad));
       s_sc = sc;
     }
   }
@@ -90,26 +91,27 @@ tridiag_eigvals_cta_kernel(LanczosBatch bt) {
   __syncthreads();
   const int k = n - 1 - m;  // ascending index of the wanted eigenvalue
   for (int round = 0; round < 40; ++round) {
-    const double lo = s_lo, hi = s_hi;
+    const dfloat lo = dfv(s_lo), hi = dfv(s_hi);
+    const dfloat w = df_sub(hi, lo);
     // 2^-46 relative, or one float64 unit of the scaled |T| <= 1
-    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-52) break;
-    const double x = lo + (hi - lo) * ((double)(tid + 1) * kInvShifts);
-    const int c = sturm_count(sa, sb2, n, df_from_double(x));
+    if (w.hi <= 0x1p-46f * fmaxf(fabsf(lo.hi), fabsf(hi.hi)) || w.hi <= 0x1p-52f) break;
+    // shift t: lo + (t + 1) (hi - lo) / (EIG_THREADS + 1), in double-float on
+    // the float32 pipes (every thread computes one per round)
+    const dfloat step = df_mul_f(w, kInvShiftsF);
+    const int c = sturm_count(sa, sb2, n, df_add(lo, df_mul_f(step, (float)(tid + 1))));
     const unsigned ball = __ballot_sync(0xffffffffu, c > k);
     if (lane == 0) s_first[warp] = ball ? warp * 32 + __ffs(ball) - 1 : EIG_THREADS;
     __syncthreads();
     if (tid == 0) {
       int f = EIG_THREADS;
-      for (int w = 0; w < EIG_THREADS / 32; ++w) f = min(f, s_first[w]);
+      for (int w2 = 0; w2 < EIG_THREADS / 32; ++w2) f = min(f, s_first[w2]);
       // count(x_t) is non-decreasing in t: the eigenvalue lies in (x_{f-1}, x_f]
-      const double xf = lo + (hi - lo) * ((double)(f + 1) * kInvShifts);
-      const double xp = lo + (hi - lo) * ((double)f * kInvShifts);
-      if (f < EIG_THREADS) s_hi = xf;
-      if (f > 0) s_lo = xp;
+      if (f < EIG_THREADS) s_hi = f2(df_add(lo, df_mul_f(step, (float)(f + 1))));
+      if (f > 0) s_lo = f2(df_add(lo, df_mul_f(step, (float)f)));
     }
     __syncthreads();
   }
-  if (tid == 0) theta[m] = (0.5 * (s_lo + s_hi)) / sc;
+  if (tid == 0) theta[m] = (0.5 * df_to_double(df_add(dfv(s_lo), dfv(s_hi)))) / sc;
 }
 
 constexpr int EIG_WARPS = 8;  // eigenvalues per CTA (one warp each)
@@ -172,22 +174,25 @@ tridiag_eigvals_kernel(LanczosBatch bt) {
     return;
   }
   const double pad = 0x1p-40 * fmax(fabs(glo * sc), fabs(ghi * sc)) + 0x1p-100;
-  double lo = glo * sc - pad, hi = ghi * sc + pad;
+  // the interval in double-float: the shifts and updates of every round run
+  // on the float32 pipes (float64 throughput is a small fraction here, and
+  // every lane of every warp computes a shift per round)
+  dfloat lo = df_from_double(glo * sc - pad), hi = df_from_double(ghi * sc + pad);
   const int k = n - 1 - m;  // ascending index of the wanted eigenvalue
   for (int round = 0; round < 40; ++round) {
-    if (hi - lo <= 0x1p-46 * fmax(fabs(lo), fabs(hi)) || hi - lo <= 0x1p-52) break;
-    const double step = (hi - lo) * (1.0 / 33.0);
-    const double x = lo + step * (double)(lane + 1);
-    const int c = sturm_count(sa, sb2, n, df_from_double(x));
+    const dfloat w = df_sub(hi, lo);
+    if (w.hi <= 0x1p-46f * fmaxf(fabsf(lo.hi), fabsf(hi.hi)) || w.hi <= 0x1p-52f) break;
+    const dfloat step = df_mul_f(w, 1.0f / 33.0f);
+    const int c = sturm_count(sa, sb2, n, df_add(lo, df_mul_f(step, (float)(lane + 1))));
     // count(x_t) is non-decreasing in t: the eigenvalue lies in (x_{f-1}, x_f]
     const unsigned ball = __ballot_sync(0xffffffffu, c > k);
     const int f = ball ? __ffs(ball) - 1 : 32;
-    const double nhi = (f < 32) ? lo + step * (double)(f + 1) : hi;
-    const double nlo = (f > 0) ? lo + step * (double)f : lo;
+    const dfloat nhi = (f < 32) ? df_add(lo, df_mul_f(step, (float)(f + 1))) : hi;
+    const dfloat nlo = (f > 0) ? df_add(lo, df_mul_f(step, (float)f)) : lo;
     lo = nlo;
     hi = nhi;
   }
-  if (lane == 0) theta[m] = (0.5 * (lo + hi)) / sc;
+  if (lane == 0) theta[m] = (0.5 * df_to_double(df_add(lo, hi))) / sc;
 }
 
 // ----------------------------------------------------------------------------
