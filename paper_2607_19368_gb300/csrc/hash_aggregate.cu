@@ -78,7 +78,13 @@ simhash_kernel(const float* __restrict__ U, int64_t N, int k, int ldu,
 }
 
 // Batched over spectral problems: rows of problem p start at phi_row, k is
-// the problem's r_eff, bits its own bit count.
+// the problem's r_eff, bits its own bit count.  One lane per hyperplane: a
+// warp takes 32 / BP rows at a time (BP = bits rounded up to a power of two),
+// lane slot * BP + l forms row slot's dot with hyperplane l by the same
+// float32 chain as simhash_row (m = 0 .. k-1, multiply and add rounded
+// separately), the row's elements read by every lane of its slot (the same
+// addresses: one transaction), R from shared memory with a padded row stride
+// (no bank conflicts between hyperplanes), and a ballot assembles the codes.
 __global__ void __launch_bounds__(256)
 simhash_batched_kernel(const ProbDesc* __restrict__ probs, const int* __restrict__ spec_list,
                        const int* __restrict__ nspec_dev, int nspec_max,
@@ -92,11 +98,29 @@ simhash_batched_kernel(const ProbDesc* __restrict__ probs, const int* __restrict
   const ProbDesc P = probs[spec_list ? spec_list[s] : s];
   const int kk = min(ldu, max(0, r_eff[s]));
   const int bits = P.bits;
-  for (int e = threadIdx.x; e < bits * kk; e += blockDim.x) Rs[e] = R[(e / kk) * ldr + e % kk];
+  const int rs = kk + 1;  // padded row stride of R in shared memory
+  for (int e = threadIdx.x; e < bits * kk; e += blockDim.x) Rs[(e / kk) * rs + e % kk] = R[(e / kk) * ldr + e % kk];
   __syncthreads();
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < P.n;
-       i += (int64_t)gridDim.x * blockDim.x)
-    codes[P.phi_row + i] = simhash_row(U + (P.phi_row + i) * ldu, kk, Rs, bits);
+  int BP = 1;
+  while (BP < bits) BP <<= 1;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int slot = lane / BP, l = lane % BP, rpw = 32 / BP;
+  const float* rl = Rs + (size_t)min(l, max(bits, 1) - 1) * rs;
+  const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t w0 = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; w0 * rpw < P.n; w0 += nw) {
+    const int64_t i = w0 * rpw + slot;
+    const bool live = i < P.n;
+    float acc = 0.0f;
+    if (live) {
+      const float* u = U + (P.phi_row + i) * ldu;
+      for (int m = 0; m < kk; ++m) acc = __fadd_rn(acc, __fmul_rn(__ldg(u + m), rl[m]));
+    }
+    const unsigned ball = __ballot_sync(0xffffffffu, live && l < bits && acc > 0.0f);
+    if (live && l == 0) {
+      const unsigned mask = (BP == 32) ? 0xffffffffu : ((1u << BP) - 1u);
+      codes[P.phi_row + i] = (ball >> (slot * BP)) & mask;
+    }
+  }
 }
 
 // Small problems (windows of at most SH_FLAT_MAX tokens): one thread per
@@ -2241,8 +2265,12 @@ int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const i
     SLS_LAUNCH_CHECK();
     return SLS_OK;
   }
-  const size_t smem = sizeof(float) * bits_max * ldu;
-  int64_t bx = (nmax + 255) / 256;
+  const size_t smem = sizeof(float) * bits_max * (ldu + 1);
+  // warps of 32 / BP rows (BP: bits rounded up to a power of two): enough
+  // CTAs of 8 warps for the rows of the largest problem
+  int bpmax = 1;
+  while (bpmax < bits_max) bpmax <<= 1;
+  int64_t bx = (nmax * bpmax + 255) / 256;
   if (bx > 1024) bx = 1024;
   if (bx < 1) bx = 1;
   if (smem > 48 * 1024)
