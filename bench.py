@@ -109,7 +109,7 @@ def config_dict(w, rho, extra=None):
 # Revision of the persistent Lanczos kernel whose DRAM counters are recorded in
 # profiles/lanczos_traffic.json; bumped with every change of the kernel, so a
 # stale capture reads as "traffic": null.
-LANCZOS_KERNEL_REV = "fused-pass/12"
+LANCZOS_KERNEL_REV = "fused-pass/13"
 
 
 def peaks():
