@@ -2272,6 +2272,11 @@ int launch_simhash_problems(const ProbDesc* probs, const int* spec_list, const i
   while (bpmax < bits_max) bpmax <<= 1;
   int64_t bx = (nmax * bpmax + 255) / 256;
   if (bx > 1024) bx = 1024;
+  // at most about 8192 CTAs in all (the CTAs loop over their problem's
+  // rows): the launch is sized by the bound on the spectral problems, most
+  // of which may be empty at run time
+  const int64_t cap = 8192 / (nspec_max > 0 ? nspec_max : 1);
+  if (bx > cap) bx = cap;
   if (bx < 1) bx = 1;
   if (smem > 48 * 1024)
     SLS_CUDA_TRY(cudaFuncSetAttribute(simhash_batched_kernel,
