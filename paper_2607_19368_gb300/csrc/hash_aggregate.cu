@@ -22,45 +22,43 @@ namespace sls {
 
 namespace {
 
-SLS_DEV uint32_t simhash_row(const float* __restrict__ u, int k, const float* __restrict__ Rs,
-                             int bits) {
-  float acc[SLS_MAX_BITS];
-#pragma unroll
-  for (int l = 0; l < SLS_MAX_BITS; ++l) acc[l] = 0.0f;
-  // the row in chunks of 16 (four 16-byte loads in flight) when it is 16-byte
-  // aligned; the chain over m keeps its order either way
-  const bool vec = ((reinterpret_cast<uintptr_t>(u) & 15) == 0);
-  int m0 = 0;
-  if (vec) {
-    for (; m0 + 16 <= k; m0 += 16) {
-      float x[16];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float4 v = __ldg(reinterpret_cast<const float4*>(u + m0) + q);
-        x[4 * q] = v.x;
-        x[4 * q + 1] = v.y;
-        x[4 * q + 2] = v.z;
-        x[4 * q + 3] = v.w;
-      }
-#pragma unroll
-      for (int t = 0; t < 16; ++t) {
-#pragma unroll
-        for (int l = 0; l < SLS_MAX_BITS; ++l)
-          if (l < bits) acc[l] = __fadd_rn(acc[l], __fmul_rn(x[t], Rs[l * k + m0 + t]));
-      }
+// SimHash of rows 0 .. n-1 with one lane per hyperplane: a warp takes
+// 32 / BP rows at a time (BP = bits rounded up to a power of two), lane
+// slot * BP + l forms row slot's dot with hyperplane l by the fixed float32
+// chain of the specification (acc = 0; for m = 0 .. k-1:
+// acc = fl(acc + fl(U[i,m] * R[l,m])), multiply and add rounded separately),
+// the row's elements read by every lane of its slot (the same addresses: one
+// transaction), R from shared memory with the padded row stride rs (no bank
+// conflicts between hyperplanes), and a ballot assembles the codes.  Warps
+// w0, w0 + wstride, ... of the launch.
+SLS_DEV void simhash_lanes(const float* __restrict__ U, int64_t n, int ldu, int kk,
+                           const float* __restrict__ Rs, int rs, int bits,
+                           uint32_t* __restrict__ codes, int64_t w0, int64_t wstride) {
+  int BP = 1;
+  while (BP < bits) BP <<= 1;
+  const int lane = threadIdx.x & 31;
+  const int slot = lane / BP, l = lane % BP, rpw = 32 / BP;
+  const float* rl = Rs + (size_t)min(l, max(bits, 1) - 1) * rs;
+  for (int64_t w = w0; w * rpw < n; w += wstride) {
+    const int64_t i = w * rpw + slot;
+    const bool live = i < n;
+    float acc = 0.0f;
+    if (live) {
+      const float* u = U + i * ldu;
+      for (int m = 0; m < kk; ++m) acc = __fadd_rn(acc, __fmul_rn(__ldg(u + m), rl[m]));
+    }
+    const unsigned ball = __ballot_sync(0xffffffffu, live && l < bits && acc > 0.0f);
+    if (live && l == 0) {
+      const unsigned mask = (BP == 32) ? 0xffffffffu : ((1u << BP) - 1u);
+      codes[i] = (ball >> (slot * BP)) & mask;
     }
   }
-  for (int m = m0; m < k; ++m) {
-    const float um = u[m];
-#pragma unroll
-    for (int l = 0; l < SLS_MAX_BITS; ++l)
-      if (l < bits) acc[l] = __fadd_rn(acc[l], __fmul_rn(um, Rs[l * k + m]));
-  }
-  uint32_t code = 0;
-#pragma unroll
-  for (int l = 0; l < SLS_MAX_BITS; ++l)
-    if (l < bits && acc[l] > 0.0f) code |= (1u << l);
-  return code;
+}
+
+// R (bits x kk) into shared memory with row stride kk + 1
+SLS_DEV void simhash_stage_R(const float* __restrict__ R, int ldr, int bits, int kk, float* Rs) {
+  for (int e = threadIdx.x; e < bits * kk; e += blockDim.x)
+    Rs[(e / kk) * (kk + 1) + e % kk] = R[(e / kk) * ldr + e % kk];
 }
 
 __global__ void __launch_bounds__(256)
@@ -70,21 +68,15 @@ simhash_kernel(const float* __restrict__ U, int64_t N, int k, int ldu,
   extern __shared__ float Rs[];
   int kk = k;
   if (k_dev) kk = min(kk, max(0, (int)*k_dev));
-  for (int e = threadIdx.x; e < bits * kk; e += blockDim.x) Rs[e] = R[(e / kk) * ldr + e % kk];
+  simhash_stage_R(R, ldr, bits, kk, Rs);
   __syncthreads();
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < N;
-       i += (int64_t)gridDim.x * blockDim.x)
-    codes[i] = simhash_row(U + i * ldu, kk, Rs, bits);
+  const int64_t wpb = blockDim.x >> 5;
+  simhash_lanes(U, N, ldu, kk, Rs, kk + 1, bits, codes,
+                (int64_t)blockIdx.x * wpb + (threadIdx.x >> 5), (int64_t)gridDim.x * wpb);
 }
 
 // Batched over spectral problems: rows of problem p start at phi_row, k is
-// the problem's r_eff, bits its own bit count.  One lane per hyperplane: a
-// warp takes 32 / BP rows at a time (BP = bits rounded up to a power of two),
-// lane slot * BP + l forms row slot's dot with hyperplane l by the same
-// float32 chain as simhash_row (m = 0 .. k-1, multiply and add rounded
-// separately), the row's elements read by every lane of its slot (the same
-// addresses: one transaction), R from shared memory with a padded row stride
-// (no bank conflicts between hyperplanes), and a ballot assembles the codes.
+// the problem's r_eff, bits its own bit count; simhash_lanes per problem.
 __global__ void __launch_bounds__(256)
 simhash_batched_kernel(const ProbDesc* __restrict__ probs, const int* __restrict__ spec_list,
                        const int* __restrict__ nspec_dev, int nspec_max,
@@ -97,35 +89,17 @@ simhash_batched_kernel(const ProbDesc* __restrict__ probs, const int* __restrict
   if (s >= nspec) return;
   const ProbDesc P = probs[spec_list ? spec_list[s] : s];
   const int kk = min(ldu, max(0, r_eff[s]));
-  const int bits = P.bits;
-  const int rs = kk + 1;  // padded row stride of R in shared memory
-  for (int e = threadIdx.x; e < bits * kk; e += blockDim.x) Rs[(e / kk) * rs + e % kk] = R[(e / kk) * ldr + e % kk];
+  simhash_stage_R(R, ldr, P.bits, kk, Rs);
   __syncthreads();
-  int BP = 1;
-  while (BP < bits) BP <<= 1;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int slot = lane / BP, l = lane % BP, rpw = 32 / BP;
-  const float* rl = Rs + (size_t)min(l, max(bits, 1) - 1) * rs;
-  const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t w0 = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; w0 * rpw < P.n; w0 += nw) {
-    const int64_t i = w0 * rpw + slot;
-    const bool live = i < P.n;
-    float acc = 0.0f;
-    if (live) {
-      const float* u = U + (P.phi_row + i) * ldu;
-      for (int m = 0; m < kk; ++m) acc = __fadd_rn(acc, __fmul_rn(__ldg(u + m), rl[m]));
-    }
-    const unsigned ball = __ballot_sync(0xffffffffu, live && l < bits && acc > 0.0f);
-    if (live && l == 0) {
-      const unsigned mask = (BP == 32) ? 0xffffffffu : ((1u << BP) - 1u);
-      codes[P.phi_row + i] = (ball >> (slot * BP)) & mask;
-    }
-  }
+  const int64_t wpb = blockDim.x >> 5;
+  simhash_lanes(U + (int64_t)P.phi_row * ldu, P.n, ldu, kk, Rs, kk + 1, P.bits,
+                codes + P.phi_row, (int64_t)blockIdx.x * wpb + (threadIdx.x >> 5),
+                (int64_t)gridDim.x * wpb);
 }
 
 // Small problems (windows of at most SH_FLAT_MAX tokens): one thread per
 // (problem, row) over all spectral problems, R read through the read-only
-// cache (row l of R at R + l * ldr), the same float32 chain as simhash_row.
+// cache (row l of R at R + l * ldr), the same float32 chain as simhash_lanes.
 constexpr int SH_FLAT_MAX = 64;
 
 __global__ void __launch_bounds__(256)
@@ -2236,8 +2210,10 @@ window_score_combine_kernel(int d, const ProbDesc* __restrict__ probs, int nprob
 int launch_simhash(const float* U, int64_t N, int k, int ldu, const int32_t* k_dev,
                    const float* R, int bits, int ldr, uint32_t* codes, cudaStream_t stream) {
   if (N == 0) return SLS_OK;
-  const size_t smem = sizeof(float) * bits * k;
-  int64_t blocks = (N + 255) / 256;
+  const size_t smem = sizeof(float) * bits * (k + 1);
+  int bp = 1;
+  while (bp < bits) bp <<= 1;
+  int64_t blocks = (N * bp + 255) / 256;  // 8 warps of 32 / bp rows
   if (blocks > 4096) blocks = 4096;
   if (smem > 48 * 1024)
     SLS_CUDA_TRY(cudaFuncSetAttribute(simhash_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
