@@ -507,7 +507,7 @@ class Run:
 
     def roofline(self, lanczos_ms):
         """Roofline of the dominant kernel, the persistent Lanczos kernel, over
-        the Lanczos phase's CUDA-event time: the survey's algorithmic count
+        the Lanczos phase's CUDA-event time: the two-sweep algorithmic count
         (two sweeps over Phi per step plus the basis traffic) and the count
         of what one fused pass per step must move (one sweep over Phi per
         step plus the basis traffic)."""
