@@ -1196,7 +1196,6 @@ __global__ void identity_kernel(const T* __restrict__ X, int64_t B, int64_t N, i
 
 constexpr int AGG_T = 256;
 constexpr int AGG_CH = 64;      // members per work item
-constexpr int AGG_MAXV = 32;    // accumulators per thread (d <= 8192)
 
 // Work items: macro-token m is split into ceil(len / AGG_CH) items, listed in
 // macro order.  Three grid-wide passes: per-block totals over the macro

@@ -50,13 +50,6 @@ __host__ __device__ inline int lw_warp_f2(int nmax, int D, int r) {
   return D + 32 + nmax * (r + 1) + 64 + 64;
 }
 
-SLS_DEV dfloat shfl_df(dfloat v, int src) {
-  dfloat r;
-  r.hi = __shfl_sync(FULL, v.hi, src);
-  r.lo = __shfl_sync(FULL, v.lo, src);
-  return r;
-}
-
 SLS_DEV dfloat shfl_xor_df(dfloat v, int o) {
   dfloat r;
   r.hi = __shfl_xor_sync(FULL, v.hi, o);
